@@ -1,0 +1,191 @@
+"""fp64 CPU oracle for PaDoc ancestor-masked attention (ctypes wrapper of padoc_oracle.c).
+
+TEST INFRASTRUCTURE ONLY: tests/, ``__graft_entry__.smoke()`` and bench.py's cpu_baseline and
+reference legs may use it; the product path never does. It imports nothing from the CUDA
+package. Pages are given as objects with ``prefix_len``, ``layout_len``, ``fork_offset`` and
+``branch_len`` (or as ``(P, L, forks, lens)`` tuples).
+
+Every function follows the paper's definition of the visibility (Sec. 3.2 ancestor sets;
+App. C.1 packed statement; App. E.1 additive-bias softmax and Algorithm 1); the C source states
+the readings taken where the paper is silent. Parity of all functions is pinned by
+tests/test_oracle_pins.py against closed forms, torch's SDPA, a simulator of Algorithm 1's mask
+recurrence and hand-derived fixtures.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+import threading
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "padoc_oracle.c")
+_LIB_PATH = os.path.join(_HERE, "_build", "libpadoc_oracle.so")
+_lib = None
+_lock = threading.Lock()
+
+_i32p = ctypes.POINTER(ctypes.c_int32)
+_i64p = ctypes.POINTER(ctypes.c_int64)
+_f32p = ctypes.POINTER(ctypes.c_float)
+_f64p = ctypes.POINTER(ctypes.c_double)
+_u8p = ctypes.POINTER(ctypes.c_uint8)
+_i8p = ctypes.POINTER(ctypes.c_int8)
+
+
+def build(force: bool = False) -> str:
+    """Compile padoc_oracle.c with gcc (fp64, OpenMP) into oracle/_build/."""
+    if force or not os.path.exists(_LIB_PATH) or os.path.getmtime(_LIB_PATH) < os.path.getmtime(_SRC):
+        os.makedirs(os.path.dirname(_LIB_PATH), exist_ok=True)
+        tmp = _LIB_PATH + f".tmp{os.getpid()}"
+        subprocess.check_call(["gcc", "-O2", "-fopenmp", "-fPIC", "-shared", "-std=c11", "-o", tmp, _SRC, "-lm"])
+        os.replace(tmp, _LIB_PATH)
+    return _LIB_PATH
+
+
+def _load():
+    global _lib
+    with _lock:
+        if _lib is None:
+            lib = ctypes.CDLL(build())
+            lib.oracle_total_tokens.restype = ctypes.c_int64
+            lib.oracle_total_tokens.argtypes = [_i32p, ctypes.c_int32, _i32p]
+            lib.oracle_dense_mask.argtypes = [_i32p, ctypes.c_int32, _i32p, _i32p, ctypes.c_int32, _u8p]
+            lib.oracle_spans.argtypes = [_i32p, ctypes.c_int32, _i32p, _i32p, _i32p]
+            pre = [_i32p, ctypes.c_int32, _i32p, _i32p, _f32p, _f32p, _f32p, ctypes.c_int32,
+                   ctypes.c_int32, ctypes.c_int32, ctypes.c_double, _f64p, _f64p]
+            lib.oracle_prefill_dense.argtypes = pre
+            lib.oracle_prefill_gather.argtypes = pre
+            lib.oracle_decode.argtypes = [ctypes.c_int32, _i32p, _i32p, _i32p, _i64p, _i64p, _f32p, _f32p,
+                                          _f32p, _f32p, _f32p, ctypes.c_int32, ctypes.c_int32,
+                                          ctypes.c_int32, ctypes.c_double, _f64p, _f64p]
+            lib.oracle_merge.argtypes = [_f64p, _f64p, ctypes.c_int32, ctypes.c_int64, ctypes.c_int32,
+                                         _f64p, _f64p]
+            lib.oracle_tile_kinds.argtypes = [_i32p, ctypes.c_int32, _i32p, _i32p, ctypes.c_int32,
+                                              ctypes.c_int32, _i8p]
+            _lib = lib
+    return _lib
+
+
+def _ptr(a, t):
+    return a.ctypes.data_as(t)
+
+
+def _flat(pages):
+    pln, forks, lens = [], [], []
+    for pg in pages:
+        if isinstance(pg, tuple):
+            P, L, f, n = pg
+        else:
+            P, L, f, n = pg.prefix_len, pg.layout_len, pg.fork_offset, pg.branch_len
+        assert len(f) == len(n)
+        pln += [int(P), int(L), len(n)]
+        forks += [int(x) for x in f]
+        lens += [int(x) for x in n]
+    z = lambda x: np.ascontiguousarray(np.asarray(x if x else [0], np.int32))
+    return z(pln), len(pages), z(forks), z(lens)
+
+
+def _f32(x):
+    """Exact fp32 copy of a torch tensor or array (bf16 and fp32 convert exactly)."""
+    try:
+        import torch
+        if isinstance(x, torch.Tensor):
+            return np.ascontiguousarray(x.detach().to("cpu", torch.float32).numpy())
+    except ImportError:  # pragma: no cover
+        pass
+    return np.ascontiguousarray(np.asarray(x, np.float32))
+
+
+def total_tokens(pages) -> int:
+    pln, n, f, b = _flat(pages)
+    return int(_load().oracle_total_tokens(_ptr(pln, _i32p), n, _ptr(b, _i32p)))
+
+
+def dense_mask(pages, page: int) -> np.ndarray:
+    """[S_p][S_p] visibility (uint8) of one page, from node membership and ancestor sets."""
+    pln, n, f, b = _flat(pages)
+    pg = pages[page]
+    S = pg[0] + pg[1] + sum(pg[3]) if isinstance(pg, tuple) else pg.prefix_len + pg.layout_len + sum(pg.branch_len)
+    m = np.zeros((S, S), np.uint8)
+    _load().oracle_dense_mask(_ptr(pln, _i32p), n, _ptr(f, _i32p), _ptr(b, _i32p), page, _ptr(m, _u8p))
+    return m
+
+
+def spans(pages) -> np.ndarray:
+    """[T][4] int32 visible spans {kv0_begin, kv0_end, kv1_begin, kv1_end} (absolute packed)."""
+    pln, n, f, b = _flat(pages)
+    T = total_tokens(pages)
+    out = np.zeros((max(T, 1), 4), np.int32)
+    _load().oracle_spans(_ptr(pln, _i32p), n, _ptr(f, _i32p), _ptr(b, _i32p), _ptr(out, _i32p))
+    return out[:T]
+
+
+def _prefill(fn_name, pages, q, k, v, scale):
+    pln, n, f, b = _flat(pages)
+    q, k, v = _f32(q), _f32(k), _f32(v)
+    T, Hq, d = q.shape
+    Hkv = k.shape[1]
+    assert k.shape == (T, Hkv, d) and v.shape == (T, Hkv, d) and Hq % Hkv == 0
+    o = np.zeros((T, Hq, d), np.float64)
+    lse = np.zeros((T, Hq), np.float64)
+    getattr(_load(), fn_name)(_ptr(pln, _i32p), n, _ptr(f, _i32p), _ptr(b, _i32p), _ptr(q, _f32p),
+                              _ptr(k, _f32p), _ptr(v, _f32p), Hq, Hkv, d, float(scale),
+                              _ptr(o, _f64p), _ptr(lse, _f64p))
+    return o, lse
+
+
+def prefill_dense(pages, q, k, v, scale):
+    """Packed prefill via the dense ancestor visibility. Returns fp64 (O [T][Hq][d], LSE [T][Hq])."""
+    return _prefill("oracle_prefill_dense", pages, q, k, v, scale)
+
+
+def prefill_gather(pages, q, k, v, scale):
+    """Packed prefill via per-branch gather and bottom-right causal attention."""
+    return _prefill("oracle_prefill_gather", pages, q, k, v, scale)
+
+
+def decode(stream_page, shared_len, priv_len, page_off, priv_off, stream_k, stream_v, priv_k, priv_v,
+           q, scale):
+    """One decode step over logical (unpaged) K/V; see padoc_oracle.c:oracle_decode."""
+    sp = np.ascontiguousarray(np.asarray(stream_page, np.int32))
+    sh = np.ascontiguousarray(np.asarray(shared_len, np.int32))
+    pl = np.ascontiguousarray(np.asarray(priv_len, np.int32))
+    po = np.ascontiguousarray(np.asarray(page_off, np.int64))
+    vo = np.ascontiguousarray(np.asarray(priv_off, np.int64))
+    sk, sv, pk, pv, qq = (_f32(x) for x in (stream_k, stream_v, priv_k, priv_v, q))
+    S, Hq, d = qq.shape
+    Hkv = sk.shape[1] if sk.size else pk.shape[1]
+    guard = lambda a: a if a.size else np.zeros((1, Hkv, d), np.float32)
+    sk, sv, pk, pv = guard(sk), guard(sv), guard(pk), guard(pv)
+    o = np.zeros((S, Hq, d), np.float64)
+    lse = np.zeros((S, Hq), np.float64)
+    if S:
+        _load().oracle_decode(S, _ptr(sp, _i32p), _ptr(sh, _i32p), _ptr(pl, _i32p), _ptr(po, _i64p),
+                              _ptr(vo, _i64p), _ptr(sk, _f32p), _ptr(sv, _f32p), _ptr(pk, _f32p),
+                              _ptr(pv, _f32p), _ptr(qq, _f32p), Hq, Hkv, d, float(scale),
+                              _ptr(o, _f64p), _ptr(lse, _f64p))
+    return o, lse
+
+
+def merge(part_o, part_lse):
+    """Merge partial softmax results over disjoint key sets: part_o [S][rows][d], part_lse [S][rows]."""
+    po = np.ascontiguousarray(np.asarray(part_o, np.float64))
+    pl = np.ascontiguousarray(np.asarray(part_lse, np.float64))
+    S, R, d = po.shape
+    o = np.zeros((R, d), np.float64)
+    lse = np.zeros((R,), np.float64)
+    _load().oracle_merge(_ptr(po, _f64p), _ptr(pl, _f64p), S, R, d, _ptr(o, _f64p), _ptr(lse, _f64p))
+    return o, lse
+
+
+def tile_kinds(pages, q_tile: int, k_tile: int) -> np.ndarray:
+    """[q_tiles][k_tiles] int8: 0 no visible pair, 1 PARTIAL, 2 FULL (brute force; small inputs)."""
+    pln, n, f, b = _flat(pages)
+    T = total_tokens(pages)
+    nq, nk = -(-T // q_tile), -(-T // k_tile)
+    out = np.zeros((max(nq, 1), max(nk, 1)), np.int8)
+    _load().oracle_tile_kinds(_ptr(pln, _i32p), n, _ptr(f, _i32p), _ptr(b, _i32p), q_tile, k_tile,
+                              _ptr(out, _i8p))
+    return out[:nq, :nk]
