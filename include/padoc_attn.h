@@ -1,0 +1,268 @@
+/*
+ * padoc_attn.h -- C ABI of padoc_attn, ancestor-masked attention over one shared page
+ * representation for PaDoc's layout-grounded parallel decoding, on one NVIDIA GB300 (sm_103a).
+ *
+ * The visibility rule (Sec. 3.2, ancestor sets Anc(B_k) = {X, B_<k}, Anc(Y_k) = {X, B_<=k};
+ * App. C.1, Q_M -> K_M causal and Q_{Y_k} -> [K_{M<=f_k}; K_{Y_k}] with bottom-right causality;
+ * App. E.1, the additive-bias softmax and Algorithm 1). A page is packed as
+ *
+ *     [ prefix X (P tokens) | layout stream (L tokens) | Y_1 (n_1) | ... | Y_N (n_N) ]
+ *
+ * and a token at page-local position q may see page-local key j exactly when
+ *     q < P + L          :  j <= q                                   (one causal stream)
+ *     q = ybase_k + i    :  j < P + f_k   or   ybase_k <= j <= q     (two spans)
+ * Tokens of different pages never see each other. f_k (0 <= f_k <= L) is the number of
+ * layout-stream tokens visible to branch k: Algorithm 1 forks a branch with a copy of the layout
+ * stream's row taken before the region's boundary output is appended. Any order of f_k and ties
+ * are legal (one branch-start token per extra branch at a higher-arity fork, Sec. 3.2).
+ *
+ * For each query and query head h, with KV head g = h / (Hq / Hkv):
+ *     s_j = scale * q . k_j (visible j),  lse = ln sum_j exp(s_j),  o = sum_j exp(s_j - lse) v_j.
+ *
+ * Conventions for every call
+ *   - Ownership: the caller owns every buffer. The library never allocates device memory, never
+ *     keeps a pointer after a call returns and never synchronizes, except
+ *     padoc_check_device_errors.
+ *   - Host pointers are marked (host); device pointers (device). Device calls are asynchronous on
+ *     the given stream (a cudaStream_t; NULL is the legacy default stream).
+ *   - Every argument is validated on the host before any launch; a failed check returns
+ *     PADOC_ERR_INVALID_ARGUMENT (or _UNSUPPORTED / _WORKSPACE_TOO_SMALL / _CAPACITY) and launches
+ *     nothing. There is no fallback path: an unsupported combination is an error.
+ *   - Block ids read on the device are range-checked; a bad id sets a device error word (read with
+ *     padoc_check_device_errors), the block is not read, and the call's outputs are undefined.
+ *   - Every wait inside a kernel is bounded; a wait that runs out sets the device error word and
+ *     the kernel returns.
+ *   - Query heads map to KV heads in consecutive groups: h -> h / (Hq / Hkv).
+ *   - LSE is the natural-log log-sum-exp, fp32, laid out [query][head].
+ */
+#ifndef PADOC_ATTN_H
+#define PADOC_ATTN_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define PADOC_ATTN_VERSION 1
+
+/* A CUDA stream handle; identical to cudaStream_t. */
+typedef struct CUstream_st *padoc_stream_t;
+
+typedef enum {
+    PADOC_OK = 0,
+    PADOC_ERR_INVALID_ARGUMENT = 1,    /* a size, range, pointer or layout check failed */
+    PADOC_ERR_UNSUPPORTED = 2,         /* valid, but not a combination this build implements */
+    PADOC_ERR_WORKSPACE_TOO_SMALL = 3, /* workspace_bytes below padoc_decode_workspace_size */
+    PADOC_ERR_CUDA = 4,                /* a CUDA runtime call or launch failed */
+    PADOC_ERR_DEVICE_CHECK = 5,        /* a kernel reported a failed device-side check */
+    PADOC_ERR_CAPACITY = 6             /* a caller-sized output array is too small */
+} padoc_status;
+
+typedef enum { PADOC_DTYPE_F32 = 0, PADOC_DTYPE_BF16 = 1 } padoc_dtype;
+
+/* Tile classes of the prefill tile map. */
+enum { PADOC_TILE_PARTIAL = 1, PADOC_TILE_FULL = 2 };
+
+/* One page (host). Sec. 3.2 / App. C.1.
+ *   prefix_len   P >= 0: image and prompt tokens (the node X), causal inside.
+ *   layout_len   L >= 0: layout-stream tokens (B_1..B_N serialized), causal, sees all of X.
+ *   num_branches N >= 0.
+ *   fork_offset  [N], 0 <= f_k <= L: layout tokens visible to branch k.
+ *   branch_len   [N], >= 1: prefill: tokens of Y_k (its branch-start token included);
+ *                decode: private KV length of branch k, including the token being decoded
+ *                (Algorithm 1 appends every live stream's input before it decodes).
+ * A page must hold at least one token. */
+typedef struct {
+    int32_t prefix_len;
+    int32_t layout_len;
+    int32_t num_branches;
+    const int32_t *fork_offset;
+    const int32_t *branch_len;
+} padoc_page;
+
+/* ============================================================================================
+ * C1: ancestor descriptors (host, integer only, bit-exact; caller-allocated outputs)
+ * ========================================================================================== */
+
+/* Total packed tokens T = sum over pages of P + L + sum_k n_k (must be < 2^31).
+ * Errors: INVALID_ARGUMENT for a null pointer or a malformed page. */
+padoc_status padoc_packed_size(const padoc_page *pages, int32_t num_pages, int64_t *total_tokens);
+
+/* Per-query visible spans (App. C.1 packed relation), absolute packed indices (pages packed
+ * back to back in the given order):
+ *   spans[4t+0], spans[4t+1] : first span  [kv0_begin, kv0_end)
+ *   spans[4t+2], spans[4t+3] : second span [kv1_begin, kv1_end)
+ * Prefix/layout token q of a page starting at pb: first = [pb, q+1), second empty.
+ * Branch token q of Y_k: first = [pb, pb+P+f_k), second = [ybase_k, q+1).
+ * An empty second span is written {kv0_end, kv0_end}. spans: (host) int32 [capacity_tokens][4].
+ * Errors: INVALID_ARGUMENT; CAPACITY when capacity_tokens < T. */
+padoc_status padoc_build_query_spans(const padoc_page *pages, int32_t num_pages, int32_t *spans,
+                                     int64_t capacity_tokens);
+
+/* Tile shape (q_tile, k_tile) the prefill kernel for (dtype, head_dim) consumes. */
+padoc_status padoc_prefill_tile_shape(padoc_dtype dtype, int32_t head_dim, int32_t *q_tile, int32_t *k_tile);
+
+/* Size of the prefill tile map for tiles of q_tile query rows by k_tile key columns:
+ * num_q_tiles = ceil(T / q_tile); nnz = number of (q-tile, k-tile) pairs with a visible entry. */
+padoc_status padoc_tile_map_size(const padoc_page *pages, int32_t num_pages, int32_t q_tile, int32_t k_tile,
+                                 int64_t *num_q_tiles, int64_t *nnz);
+
+/* Prefill work list in CSR form (Flex-Attention-style block skipping, App. C.1): for q-tile r,
+ * entries [row_ptr[r], row_ptr[r+1]) list the k-tiles holding at least one visible
+ * (query, key) pair, in ascending k-tile order, with kinds[e] = PADOC_TILE_FULL when every query
+ * row of the tile that exists (< T) sees all k_tile columns (a k-tile reaching past T is never
+ * FULL) and PADOC_TILE_PARTIAL otherwise. Fully masked tiles are absent.
+ * row_ptr: (host) int32 [num_q_tiles + 1]; k_tiles: (host) int32 [capacity_nnz];
+ * kinds: (host) int8 [capacity_nnz]. Errors: INVALID_ARGUMENT; CAPACITY when capacity_nnz < nnz. */
+padoc_status padoc_build_tile_map(const padoc_page *pages, int32_t num_pages, int32_t q_tile, int32_t k_tile,
+                                  int32_t *row_ptr, int32_t *k_tiles, int8_t *kinds, int64_t capacity_nnz);
+
+/* ============================================================================================
+ * C5 + C2 + C4: paged KV cache and one decode step for every live stream (App. E.1, Alg. 1)
+ * ========================================================================================== */
+
+/* The paged KV pool (device), C5. Blocks of block_size tokens; per block, per KV head, the
+ * block_size x head_dim rows are contiguous: k_pool/v_pool are [num_blocks][num_kv_heads]
+ * [block_size][head_dim] in dtype, 16-byte aligned. A page's shared stream (prefix + layout, the
+ * tokens every branch of the page shares) is stored once, addressed by the page's block table;
+ * each stream's private tokens live in its own blocks starting at block offset 0, addressed by
+ * the stream's block table. Visibility is a per-stream column cutoff, so nothing is duplicated
+ * (the paper's serving reuses only complete shared blocks and re-prefills the tail, App. E.2). */
+typedef struct {
+    const void *k_pool;
+    const void *v_pool;
+    int32_t num_blocks;
+    int32_t block_size;   /* 16 */
+    int32_t num_kv_heads;
+    int32_t head_dim;     /* 128 (bf16) or 64/128 (f32) */
+    padoc_dtype dtype;
+} padoc_kv_pool;
+
+typedef struct {
+    int32_t num_q_heads;
+    int32_t num_kv_heads;
+    int32_t head_dim;
+    int32_t block_size;      /* must equal the pool's block_size */
+    int32_t layout_streams;  /* 1: also decode each page's layout stream (Alg. 1 decodes every live
+                                stream): cutoff P + L over the shared stream, no private rows */
+    int32_t split_tokens;    /* shared-stream tokens per split-K partial; 0 = library default;
+                                a positive value must be a multiple of block_size */
+} padoc_decode_config;
+
+/* Host summary of a decode plan, filled by padoc_build_decode_plan. The int32 plan blob it
+ * describes must be copied to the device unchanged and passed as plan_dev.
+ * Streams are ordered page by page: the page's branches in the given order, then (with
+ * layout_streams) its layout stream. Q, out and lse rows follow this order. */
+typedef struct {
+    padoc_decode_config cfg;
+    int32_t num_pages;
+    int32_t num_streams;
+    int32_t num_items;         /* work items of the split-K decode kernels */
+    int32_t num_tc_items;      /* of which use the tensor-core shared-stream kernel */
+    int32_t num_slots;         /* split-K partial results per query head */
+    int32_t max_page_blocks;   /* page block-table width the plan needs */
+    int32_t max_stream_blocks; /* stream block-table width the plan needs */
+    int64_t plan_ints;         /* int32 words in the plan blob */
+    int64_t off_stream_page;   /* offsets (int32 words) of the blob's arrays */
+    int64_t off_shared_len;
+    int64_t off_private_len;
+    int64_t off_slot_ptr;
+    int64_t off_items;
+    int64_t off_page_len;
+    int64_t kv_tokens;         /* algorithmic KV tokens read: each page's stream once + all private */
+} padoc_decode_plan;
+
+/* Size in int32 words of the plan blob for these pages and config. */
+padoc_status padoc_decode_plan_size(const padoc_page *pages, int32_t num_pages, const padoc_decode_config *cfg,
+                                    int64_t *plan_ints);
+
+/* Builds the decode plan (C1's per-branch plan {page, shared_len = P + f_k, private_len} plus the
+ * split-K work list and partial-result slots). pages: branch_len = private KV lengths.
+ * plan: (host) int32 [capacity_ints]; info: (host) summary.
+ * Errors: INVALID_ARGUMENT; UNSUPPORTED for head layouts the kernels do not implement;
+ * CAPACITY when capacity_ints is too small. */
+padoc_status padoc_build_decode_plan(const padoc_page *pages, int32_t num_pages, const padoc_decode_config *cfg,
+                                     int32_t *plan, int64_t capacity_ints, padoc_decode_plan *info);
+
+/* Workspace (device) bytes padoc_branch_decode_attn needs for this plan (split-K partials). */
+padoc_status padoc_decode_workspace_size(const padoc_decode_plan *info, size_t *bytes);
+
+/* One decode step for every live stream of every page (Alg. 1 "Decode o for all streams using the
+ * additive bias A_M", App. E.1): stream s of page p attends to the page's shared stream rows
+ * [0, shared_len_s) and to its private rows [0, private_len_s), where the newest private row is
+ * the token being decoded.
+ *   pool:          the paged KV pool (device pointers inside).
+ *   info, plan_dev: host summary and device copy of the plan blob.
+ *   page_block_table   (device) int32 [num_pages][page_table_stride], block ids of each page's
+ *                      shared stream; stride >= info->max_page_blocks.
+ *   stream_block_table (device) int32 [num_streams][stream_table_stride], block ids of each
+ *                      stream's private rows; stride >= max(info->max_stream_blocks, 1).
+ *   q:   (device) [num_streams][Hq][head_dim] in pool dtype.
+ *   out: (device) [num_streams][Hq][head_dim] in pool dtype.  lse: (device) fp32 [num_streams][Hq].
+ *   workspace: (device) >= padoc_decode_workspace_size bytes, 256-byte aligned.
+ * bf16 path: head_dim 128, Hq / Hkv = 8, block_size 16. f32 path (bring-up): head_dim 64 or 128,
+ * any Hq multiple of Hkv, block_size 16; it needs no workspace.
+ * Errors: INVALID_ARGUMENT, UNSUPPORTED, WORKSPACE_TOO_SMALL, CUDA. */
+padoc_status padoc_branch_decode_attn(const padoc_kv_pool *pool, const padoc_decode_plan *info,
+                                      const int32_t *plan_dev, const int32_t *page_block_table,
+                                      int32_t page_table_stride, const int32_t *stream_block_table,
+                                      int32_t stream_table_stride, const void *q, float scale, void *out,
+                                      float *lse, void *workspace, size_t workspace_bytes,
+                                      padoc_stream_t stream);
+
+/* C4: merge of split-K partial softmax results (softmax over a union of disjoint key sets):
+ *   lse_r = ln sum_s exp(part_lse[s][r]),  out_r = sum_s exp(part_lse[s][r] - lse_r) part_o[s][r].
+ * A part with lse = -inf weighs 0; a row whose parts are all -inf gets lse = -inf and out = 0.
+ * part_o: (device) fp32 [num_splits][rows][head_dim]; part_lse: (device) fp32 [num_splits][rows];
+ * out: (device) [rows][head_dim] in out_dtype; lse: (device) fp32 [rows] (may be NULL).
+ * head_dim a multiple of 4, <= 256. Errors: INVALID_ARGUMENT, CUDA. */
+padoc_status padoc_splitk_combine(const float *part_o, const float *part_lse, int32_t num_splits, int64_t rows,
+                                  int32_t head_dim, padoc_dtype out_dtype, void *out, float *lse,
+                                  padoc_stream_t stream);
+
+/* ============================================================================================
+ * C3: packed variable-length ancestor prefill (training forward / branch prefill)
+ * ========================================================================================== */
+
+/* Every packed token is a query under the ancestor rule (App. C.1: the causal problem over M and
+ * one bottom-right-aligned causal problem per branch over [K_{M<=f_k}; K_{Y_k}], computed in
+ * packed order without any gather). Fully masked tiles are skipped via the tile map.
+ *   q: (device) [T][Hq][head_dim]; k, v: (device) [T][Hkv][head_dim]; all in dtype, 16-byte aligned.
+ *   spans_dev: (device) int32 [T][4] from padoc_build_query_spans.
+ *   tile_row_ptr_dev / tile_k_dev / tile_kind_dev: (device) the tile map from
+ *   padoc_build_tile_map built with (q_tile, k_tile) = padoc_prefill_tile_shape(dtype, head_dim)
+ *   (the f32 path reads only the spans and accepts NULL tile pointers).
+ *   out: (device) [T][Hq][head_dim] in dtype; lse: (device) fp32 [T][Hq].
+ * bf16 path: head_dim 128, Hq a multiple of Hkv. f32 path: head_dim 64 or 128.
+ * Errors: INVALID_ARGUMENT, UNSUPPORTED, CUDA. */
+padoc_status padoc_ancestor_prefill_attn(const void *q, const void *k, const void *v, padoc_dtype dtype,
+                                         int64_t total_tokens, int32_t num_q_heads, int32_t num_kv_heads,
+                                         int32_t head_dim, const int32_t *spans_dev,
+                                         const int32_t *tile_row_ptr_dev, const int32_t *tile_k_dev,
+                                         const int8_t *tile_kind_dev, int32_t q_tile, int32_t k_tile,
+                                         float scale, void *out, float *lse, padoc_stream_t stream);
+
+/* ============================================================================================
+ * Status
+ * ========================================================================================== */
+
+/* Synchronizes `stream`, then reads and clears the current device's error word. Returns
+ * PADOC_ERR_DEVICE_CHECK if a kernel recorded a failed check since the last call (code and detail
+ * via padoc_last_device_error), PADOC_ERR_CUDA if the stream reports an error, else PADOC_OK. */
+padoc_status padoc_check_device_errors(padoc_stream_t stream);
+
+/* The code and detail of the device error found by the last padoc_check_device_errors on this
+ * thread: code 1 = block id out of range (detail = the id), 2 = bounded wait ran out
+ * (detail = the kernel's wait site). */
+void padoc_last_device_error(int32_t *code, int32_t *detail);
+
+const char *padoc_status_string(padoc_status status);
+int32_t padoc_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* PADOC_ATTN_H */

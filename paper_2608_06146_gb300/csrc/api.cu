@@ -1,0 +1,111 @@
+// api.cu -- status reporting, the per-device error word and tensor-map encoding for padoc_attn.
+#include <cudaTypedefs.h>
+#include <mutex>
+
+#include "common.cuh"
+
+namespace {
+
+__device__ int g_padoc_error[4];
+
+constexpr int kMaxDevices = 64;
+int *g_err_ptr[kMaxDevices] = {nullptr};
+std::mutex g_mu;
+thread_local int32_t t_last_code = 0, t_last_detail = 0;
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn()
+{
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void *p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+    });
+    return fn;
+}
+
+}  // namespace
+
+int *padoc_device_error_word()
+{
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return nullptr;
+    std::lock_guard<std::mutex> lk(g_mu);
+    if (!g_err_ptr[dev]) {
+        void *p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_padoc_error) != cudaSuccess) return nullptr;
+        g_err_ptr[dev] = (int *)p;
+    }
+    return g_err_ptr[dev];
+}
+
+bool padoc_make_tmap_bf16(CUtensorMap *map, const void *base, uint64_t cols, uint64_t rows, uint64_t row_stride_bytes,
+                          uint32_t box_cols, uint32_t box_rows)
+{
+    PFN_cuTensorMapEncodeTiled_v12000 fn = encode_fn();
+    if (!fn) return false;
+    if ((((uintptr_t)base) & 15) || (row_stride_bytes & 15) || rows == 0 || cols == 0) return false;
+    cuuint64_t dims[2] = {cols, rows};
+    cuuint64_t strides[1] = {row_stride_bytes};
+    cuuint32_t box[2] = {box_cols, box_rows};
+    cuuint32_t estr[2] = {1, 1};
+    CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(base), dims, strides, box, estr,
+                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                    CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS;
+}
+
+padoc_status padoc_launch_status()
+{
+    return cudaPeekAtLastError() == cudaSuccess ? PADOC_OK : (cudaGetLastError(), PADOC_ERR_CUDA);
+}
+
+int padoc_num_sms()
+{
+    int dev = 0, n = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+    return n > 0 ? n : 1;
+}
+
+extern "C" padoc_status padoc_check_device_errors(padoc_stream_t stream)
+{
+    t_last_code = 0;
+    t_last_detail = 0;
+    if (cudaStreamSynchronize((cudaStream_t)stream) != cudaSuccess) return PADOC_ERR_CUDA;
+    int *p = padoc_device_error_word();
+    if (!p) return PADOC_ERR_CUDA;
+    int host[4] = {0, 0, 0, 0};
+    if (cudaMemcpy(host, p, sizeof(host), cudaMemcpyDeviceToHost) != cudaSuccess) return PADOC_ERR_CUDA;
+    if (host[0] == 0) return PADOC_OK;
+    t_last_code = host[0];
+    t_last_detail = host[1];
+    const int zero[4] = {0, 0, 0, 0};
+    if (cudaMemcpy(p, zero, sizeof(zero), cudaMemcpyHostToDevice) != cudaSuccess) return PADOC_ERR_CUDA;
+    return PADOC_ERR_DEVICE_CHECK;
+}
+
+extern "C" void padoc_last_device_error(int32_t *code, int32_t *detail)
+{
+    if (code) *code = t_last_code;
+    if (detail) *detail = t_last_detail;
+}
+
+extern "C" const char *padoc_status_string(padoc_status status)
+{
+    switch (status) {
+    case PADOC_OK: return "ok";
+    case PADOC_ERR_INVALID_ARGUMENT: return "invalid argument";
+    case PADOC_ERR_UNSUPPORTED: return "unsupported combination";
+    case PADOC_ERR_WORKSPACE_TOO_SMALL: return "workspace too small";
+    case PADOC_ERR_CUDA: return "CUDA error";
+    case PADOC_ERR_DEVICE_CHECK: return "device-side check failed";
+    case PADOC_ERR_CAPACITY: return "output capacity too small";
+    }
+    return "unknown status";
+}
+
+extern "C" int32_t padoc_version(void) { return PADOC_ATTN_VERSION; }

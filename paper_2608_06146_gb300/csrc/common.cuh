@@ -1,0 +1,183 @@
+// common.cuh -- device helpers of padoc_attn (sm_103a): error word, bounded mbarrier waits,
+// TMA tile loads, warp-level bf16 MMA, and host helpers for tensor maps and launches.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "padoc_attn.h"
+#include "plan_internal.h"
+
+// ------------------------------------------------------------------------------------------------
+// Device error word: [0] = code (first error wins), [1] = detail.
+// ------------------------------------------------------------------------------------------------
+#define PADOC_DEVERR_BLOCK_ID 1
+#define PADOC_DEVERR_TIMEOUT 2
+
+__device__ __forceinline__ void padoc_record_error(int *err, int code, int detail)
+{
+    if (atomicCAS(err, 0, code) == 0) atomicExch(err + 1, detail);
+}
+
+// Upper bound of any single wait inside a kernel (ns of %globaltimer).
+#define PADOC_WAIT_LIMIT_NS 2000000000ull
+
+__device__ __forceinline__ uint64_t padoc_globaltimer()
+{
+    uint64_t t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+
+// ------------------------------------------------------------------------------------------------
+// mbarrier
+// ------------------------------------------------------------------------------------------------
+__device__ __forceinline__ uint32_t smem_u32(const void *p)
+{
+    return (uint32_t)__cvta_generic_to_shared(p);
+}
+
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count)
+{
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ void fence_barrier_init()
+{
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+
+__device__ __forceinline__ void fence_proxy_async_smem()
+{
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, uint32_t bytes)
+{
+    asm volatile("mbarrier.arrive.expect_tx.release.cta.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
+                 : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(uint32_t bar)
+{
+    asm volatile("mbarrier.arrive.release.cta.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity)
+{
+    uint32_t ok;
+    asm volatile(
+        "{\n .reg .pred p;\n"
+        " mbarrier.try_wait.parity.acquire.cta.shared::cta.b64 p, [%1], %2;\n"
+        " selp.u32 %0, 1, 0, p;\n}"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
+// Waits for the phase with the given parity to complete; false (and the error word set) if it
+// does not complete within PADOC_WAIT_LIMIT_NS.
+__device__ __forceinline__ bool mbar_wait_bounded(uint32_t bar, uint32_t parity, int *err, int site)
+{
+    if (mbar_try_wait(bar, parity)) return true;
+    const uint64_t t0 = padoc_globaltimer();
+    for (uint32_t i = 1;; ++i) {
+        if (mbar_try_wait(bar, parity)) return true;
+        if ((i & 255u) == 0 && padoc_globaltimer() - t0 > PADOC_WAIT_LIMIT_NS) {
+            padoc_record_error(err, PADOC_DEVERR_TIMEOUT, site);
+            return false;
+        }
+    }
+}
+
+// ------------------------------------------------------------------------------------------------
+// TMA (cp.async.bulk.tensor), 2-D tiles into shared memory, completion on an mbarrier.
+// x is the innermost coordinate (elements); callers keep x * sizeof(elem) a multiple of 16.
+// ------------------------------------------------------------------------------------------------
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap *map, int32_t x, int32_t y, uint32_t bar)
+{
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar)
+        : "memory");
+}
+
+__device__ __forceinline__ void tma_prefetch_desc(const CUtensorMap *map)
+{
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
+}
+
+// Byte offset of element (row, col) of a [rows][64] bf16 panel written by TMA with 128-byte
+// swizzle (16-byte chunk index XOR row % 8); panels start on 1024-byte boundaries.
+__device__ __forceinline__ uint32_t sw128_offset(uint32_t row, uint32_t col)
+{
+    return row * 128u + ((((col >> 3) ^ row) & 7u) << 4) + ((col & 7u) << 1);
+}
+
+// ------------------------------------------------------------------------------------------------
+// Warp-level MMA (mma.sync m16n8k16 bf16 -> fp32), ldmatrix, movmatrix
+// ------------------------------------------------------------------------------------------------
+__device__ __forceinline__ void mma_bf16_16816(float (&c)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1)
+{
+    asm volatile(
+        "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%0,%1,%2,%3};"
+        : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+        : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+
+__device__ __forceinline__ void ldmatrix_x4(uint32_t (&r)[4], uint32_t addr)
+{
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
+                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+                 : "r"(addr));
+}
+
+__device__ __forceinline__ void ldmatrix_x4_trans(uint32_t (&r)[4], uint32_t addr)
+{
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
+                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+                 : "r"(addr));
+}
+
+__device__ __forceinline__ uint32_t movmatrix_trans(uint32_t x)
+{
+    uint32_t y;
+    asm volatile("movmatrix.sync.aligned.m8n8.trans.b16 %0, %1;" : "=r"(y) : "r"(x));
+    return y;
+}
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi)
+{
+    __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+    return *reinterpret_cast<uint32_t *>(&v);
+}
+
+__device__ __forceinline__ float fast_exp2(float x)
+{
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
+#define PADOC_LOG2E 1.4426950408889634f
+#define PADOC_LN2 0.6931471805599453f
+
+// ------------------------------------------------------------------------------------------------
+// Host helpers (defined in api.cu)
+// ------------------------------------------------------------------------------------------------
+// Device address of the current device's error word (set up once per device).
+int *padoc_device_error_word();
+// 2-D bf16 tensor map: rows x cols elements with a row pitch of `row_stride_bytes`, box of
+// box_rows x 64 columns, 128-byte swizzle. Returns false if the driver rejects it.
+bool padoc_make_tmap_bf16(CUtensorMap *map, const void *base, uint64_t cols, uint64_t rows,
+                          uint64_t row_stride_bytes, uint32_t box_cols, uint32_t box_rows);
+padoc_status padoc_launch_status();
+int padoc_num_sms();
+
+#define PADOC_CUDA_TRY(expr)                                   \
+    do {                                                       \
+        if ((expr) != cudaSuccess) return PADOC_ERR_CUDA;      \
+    } while (0)

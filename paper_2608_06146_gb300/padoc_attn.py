@@ -1,0 +1,301 @@
+"""Python binding of the padoc_attn C ABI (include/padoc_attn.h): argument marshalling only.
+
+Every function has the name of the C entry point it calls. Device buffers are torch CUDA tensors
+(PyTorch supplies memory and streams); every step of the computation runs in the library's CUDA
+kernels. There is no fallback: if the shared library is missing or a call fails, an exception is
+raised.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from typing import Optional, Sequence
+
+import numpy as np
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_PKG, "_build", "libpadoc_attn.so")
+
+PADOC_OK = 0
+PADOC_DTYPE_F32 = 0
+PADOC_DTYPE_BF16 = 1
+PADOC_TILE_PARTIAL = 1
+PADOC_TILE_FULL = 2
+
+_STATUS = {0: "ok", 1: "invalid argument", 2: "unsupported combination", 3: "workspace too small",
+           4: "CUDA error", 5: "device-side check failed", 6: "output capacity too small"}
+
+
+class PadocError(RuntimeError):
+    def __init__(self, fn: str, status: int):
+        self.status = status
+        super().__init__(f"{fn} failed: {_STATUS.get(status, status)} (status {status})")
+
+
+class padoc_page(ctypes.Structure):
+    _fields_ = [("prefix_len", ctypes.c_int32), ("layout_len", ctypes.c_int32), ("num_branches", ctypes.c_int32),
+                ("fork_offset", ctypes.POINTER(ctypes.c_int32)), ("branch_len", ctypes.POINTER(ctypes.c_int32))]
+
+
+class padoc_kv_pool(ctypes.Structure):
+    _fields_ = [("k_pool", ctypes.c_void_p), ("v_pool", ctypes.c_void_p), ("num_blocks", ctypes.c_int32),
+                ("block_size", ctypes.c_int32), ("num_kv_heads", ctypes.c_int32), ("head_dim", ctypes.c_int32),
+                ("dtype", ctypes.c_int)]
+
+
+class padoc_decode_config(ctypes.Structure):
+    _fields_ = [("num_q_heads", ctypes.c_int32), ("num_kv_heads", ctypes.c_int32), ("head_dim", ctypes.c_int32),
+                ("block_size", ctypes.c_int32), ("layout_streams", ctypes.c_int32), ("split_tokens", ctypes.c_int32)]
+
+
+class padoc_decode_plan(ctypes.Structure):
+    _fields_ = [("cfg", padoc_decode_config), ("num_pages", ctypes.c_int32), ("num_streams", ctypes.c_int32),
+                ("num_items", ctypes.c_int32), ("num_tc_items", ctypes.c_int32), ("num_slots", ctypes.c_int32),
+                ("max_page_blocks", ctypes.c_int32), ("max_stream_blocks", ctypes.c_int32),
+                ("plan_ints", ctypes.c_int64), ("off_stream_page", ctypes.c_int64), ("off_shared_len", ctypes.c_int64),
+                ("off_private_len", ctypes.c_int64), ("off_slot_ptr", ctypes.c_int64), ("off_items", ctypes.c_int64),
+                ("off_page_len", ctypes.c_int64), ("kv_tokens", ctypes.c_int64)]
+
+
+_lib = None
+_i32p = ctypes.POINTER(ctypes.c_int32)
+_i64p = ctypes.POINTER(ctypes.c_int64)
+_i8p = ctypes.POINTER(ctypes.c_int8)
+_vp = ctypes.c_void_p
+
+
+def load_library(path: Optional[str] = None):
+    """Load libpadoc_attn.so (built in-tree by paper_2608_06146_gb300.build). Raises if absent."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    path = path or LIB_PATH
+    if not os.path.exists(path):
+        raise RuntimeError(f"padoc_attn CUDA library not built: {path} is missing (run __graft_entry__.build())")
+    lib = ctypes.CDLL(path)
+    P = ctypes.POINTER(padoc_page)
+    sig = {
+        "padoc_packed_size": [P, ctypes.c_int32, _i64p],
+        "padoc_build_query_spans": [P, ctypes.c_int32, _i32p, ctypes.c_int64],
+        "padoc_prefill_tile_shape": [ctypes.c_int, ctypes.c_int32, _i32p, _i32p],
+        "padoc_tile_map_size": [P, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32, _i64p, _i64p],
+        "padoc_build_tile_map": [P, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32, _i32p, _i32p, _i8p, ctypes.c_int64],
+        "padoc_decode_plan_size": [P, ctypes.c_int32, ctypes.POINTER(padoc_decode_config), _i64p],
+        "padoc_build_decode_plan": [P, ctypes.c_int32, ctypes.POINTER(padoc_decode_config), _i32p, ctypes.c_int64,
+                                    ctypes.POINTER(padoc_decode_plan)],
+        "padoc_decode_workspace_size": [ctypes.POINTER(padoc_decode_plan), ctypes.POINTER(ctypes.c_size_t)],
+        "padoc_branch_decode_attn": [ctypes.POINTER(padoc_kv_pool), ctypes.POINTER(padoc_decode_plan), _vp, _vp,
+                                     ctypes.c_int32, _vp, ctypes.c_int32, _vp, ctypes.c_float, _vp, _vp, _vp,
+                                     ctypes.c_size_t, _vp],
+        "padoc_splitk_combine": [_vp, _vp, ctypes.c_int32, ctypes.c_int64, ctypes.c_int32, ctypes.c_int, _vp, _vp, _vp],
+        "padoc_ancestor_prefill_attn": [_vp, _vp, _vp, ctypes.c_int, ctypes.c_int64, ctypes.c_int32, ctypes.c_int32,
+                                        ctypes.c_int32, _vp, _vp, _vp, _vp, ctypes.c_int32, ctypes.c_int32,
+                                        ctypes.c_float, _vp, _vp, _vp],
+        "padoc_check_device_errors": [_vp],
+        "padoc_last_device_error": [_i32p, _i32p],
+        "padoc_status_string": [ctypes.c_int],
+        "padoc_version": [],
+    }
+    for name, args in sig.items():
+        f = getattr(lib, name)
+        f.argtypes = args
+        f.restype = ctypes.c_int
+    lib.padoc_status_string.restype = ctypes.c_char_p
+    lib.padoc_last_device_error.restype = None
+    _lib = lib
+    return lib
+
+
+def exported_symbols() -> Sequence[str]:
+    return [n for n in ("padoc_packed_size", "padoc_build_query_spans", "padoc_prefill_tile_shape",
+                        "padoc_tile_map_size", "padoc_build_tile_map", "padoc_decode_plan_size",
+                        "padoc_build_decode_plan", "padoc_decode_workspace_size", "padoc_branch_decode_attn",
+                        "padoc_splitk_combine", "padoc_ancestor_prefill_attn", "padoc_check_device_errors",
+                        "padoc_last_device_error", "padoc_status_string", "padoc_version")]
+
+
+def _check(fn: str, st: int):
+    if st != PADOC_OK:
+        raise PadocError(fn, st)
+
+
+class _Pages:
+    """C array of padoc_page; keeps the per-page int32 arrays alive."""
+
+    def __init__(self, pages):
+        self.keep = []
+        self.arr = (padoc_page * max(len(pages), 1))()
+        for i, pg in enumerate(pages):
+            f = np.ascontiguousarray(np.asarray(pg.fork_offset, np.int32))
+            n = np.ascontiguousarray(np.asarray(pg.branch_len, np.int32))
+            self.keep += [f, n]
+            self.arr[i].prefix_len = int(pg.prefix_len)
+            self.arr[i].layout_len = int(pg.layout_len)
+            self.arr[i].num_branches = len(n)
+            self.arr[i].fork_offset = f.ctypes.data_as(_i32p)
+            self.arr[i].branch_len = n.ctypes.data_as(_i32p)
+        self.n = len(pages)
+
+
+def _stream_ptr(stream):
+    if stream is None:
+        import torch
+        return torch.cuda.current_stream().cuda_stream
+    return getattr(stream, "cuda_stream", stream)
+
+
+def _dtype_code(t):
+    import torch
+    if t.dtype == torch.bfloat16:
+        return PADOC_DTYPE_BF16
+    if t.dtype == torch.float32:
+        return PADOC_DTYPE_F32
+    raise TypeError(f"unsupported dtype {t.dtype}")
+
+
+def _dev(t, name):
+    if t is None:
+        return None
+    if not t.is_cuda or not t.is_contiguous():
+        raise ValueError(f"{name} must be a contiguous CUDA tensor")
+    return t.data_ptr()
+
+
+# ------------------------------------------------------------------------------------------------
+# C1: descriptors
+# ------------------------------------------------------------------------------------------------
+
+def padoc_packed_size(pages) -> int:
+    lib, P = load_library(), _Pages(pages)
+    t = ctypes.c_int64()
+    _check("padoc_packed_size", lib.padoc_packed_size(P.arr, P.n, ctypes.byref(t)))
+    return t.value
+
+
+def padoc_build_query_spans(pages) -> np.ndarray:
+    lib, P = load_library(), _Pages(pages)
+    T = padoc_packed_size(pages)
+    out = np.zeros((max(T, 1), 4), np.int32)
+    _check("padoc_build_query_spans", lib.padoc_build_query_spans(P.arr, P.n, out.ctypes.data_as(_i32p), T))
+    return out[:T]
+
+
+def padoc_prefill_tile_shape(dtype: int, head_dim: int):
+    lib = load_library()
+    a, b = ctypes.c_int32(), ctypes.c_int32()
+    _check("padoc_prefill_tile_shape", lib.padoc_prefill_tile_shape(dtype, head_dim, ctypes.byref(a), ctypes.byref(b)))
+    return a.value, b.value
+
+
+def padoc_tile_map_size(pages, q_tile: int, k_tile: int):
+    lib, P = load_library(), _Pages(pages)
+    a, b = ctypes.c_int64(), ctypes.c_int64()
+    _check("padoc_tile_map_size", lib.padoc_tile_map_size(P.arr, P.n, q_tile, k_tile, ctypes.byref(a), ctypes.byref(b)))
+    return a.value, b.value
+
+
+def padoc_build_tile_map(pages, q_tile: int, k_tile: int):
+    """Returns (row_ptr int32 [q_tiles+1], k_tiles int32 [nnz], kinds int8 [nnz])."""
+    lib, P = load_library(), _Pages(pages)
+    nqt, nnz = padoc_tile_map_size(pages, q_tile, k_tile)
+    row_ptr = np.zeros(nqt + 1, np.int32)
+    kt = np.zeros(max(nnz, 1), np.int32)
+    kind = np.zeros(max(nnz, 1), np.int8)
+    _check("padoc_build_tile_map", lib.padoc_build_tile_map(P.arr, P.n, q_tile, k_tile, row_ptr.ctypes.data_as(_i32p),
+                                                            kt.ctypes.data_as(_i32p), kind.ctypes.data_as(_i8p), nnz))
+    return row_ptr, kt[:nnz], kind[:nnz]
+
+
+# ------------------------------------------------------------------------------------------------
+# Decode
+# ------------------------------------------------------------------------------------------------
+
+def make_decode_config(num_q_heads, num_kv_heads, head_dim, block_size=16, layout_streams=False, split_tokens=0):
+    return padoc_decode_config(num_q_heads, num_kv_heads, head_dim, block_size, int(bool(layout_streams)), split_tokens)
+
+
+def padoc_decode_plan_size(pages, cfg: padoc_decode_config) -> int:
+    lib, P = load_library(), _Pages(pages)
+    n = ctypes.c_int64()
+    _check("padoc_decode_plan_size", lib.padoc_decode_plan_size(P.arr, P.n, ctypes.byref(cfg), ctypes.byref(n)))
+    return n.value
+
+
+def padoc_build_decode_plan(pages, cfg: padoc_decode_config):
+    """Returns (plan blob int32 numpy array, padoc_decode_plan host summary)."""
+    lib, P = load_library(), _Pages(pages)
+    n = padoc_decode_plan_size(pages, cfg)
+    plan = np.zeros(max(n, 1), np.int32)
+    info = padoc_decode_plan()
+    _check("padoc_build_decode_plan", lib.padoc_build_decode_plan(P.arr, P.n, ctypes.byref(cfg),
+                                                                  plan.ctypes.data_as(_i32p), n, ctypes.byref(info)))
+    return plan[:n], info
+
+
+def padoc_decode_workspace_size(info: padoc_decode_plan) -> int:
+    lib = load_library()
+    b = ctypes.c_size_t()
+    _check("padoc_decode_workspace_size", lib.padoc_decode_workspace_size(ctypes.byref(info), ctypes.byref(b)))
+    return b.value
+
+
+def padoc_branch_decode_attn(k_pool, v_pool, info: padoc_decode_plan, plan_dev, page_table, stream_table, q, scale,
+                             out, lse, workspace=None, stream=None):
+    """k_pool/v_pool: [num_blocks][Hkv][16][d]; page_table [pages][stride]; stream_table [streams][stride]
+    (int32 CUDA tensors); q/out: [streams][Hq][d]; lse: fp32 [streams][Hq]; workspace: uint8 CUDA tensor."""
+    lib = load_library()
+    pool = padoc_kv_pool(_dev(k_pool, "k_pool"), _dev(v_pool, "v_pool"), k_pool.shape[0], k_pool.shape[2],
+                         k_pool.shape[1], k_pool.shape[3], _dtype_code(k_pool))
+    ws = _dev(workspace, "workspace") if workspace is not None else None
+    wsb = workspace.numel() * workspace.element_size() if workspace is not None else 0
+    st = lib.padoc_branch_decode_attn(ctypes.byref(pool), ctypes.byref(info), _dev(plan_dev, "plan_dev"),
+                                      _dev(page_table, "page_table"), page_table.shape[1],
+                                      _dev(stream_table, "stream_table"), stream_table.shape[1], _dev(q, "q"),
+                                      float(scale), _dev(out, "out"), _dev(lse, "lse"), ws, wsb, _stream_ptr(stream))
+    _check("padoc_branch_decode_attn", st)
+
+
+def padoc_splitk_combine(part_o, part_lse, out, lse=None, stream=None):
+    """part_o fp32 [S][rows][d], part_lse fp32 [S][rows] -> out [rows][d] (bf16 or fp32), lse fp32 [rows]."""
+    lib = load_library()
+    S, R, d = part_o.shape
+    st = lib.padoc_splitk_combine(_dev(part_o, "part_o"), _dev(part_lse, "part_lse"), S, R, d, _dtype_code(out),
+                                  _dev(out, "out"), _dev(lse, "lse"), _stream_ptr(stream))
+    _check("padoc_splitk_combine", st)
+
+
+# ------------------------------------------------------------------------------------------------
+# Prefill
+# ------------------------------------------------------------------------------------------------
+
+def padoc_ancestor_prefill_attn(q, k, v, spans_dev, row_ptr_dev, k_tiles_dev, kinds_dev, scale, out, lse,
+                                q_tile=128, k_tile=128, stream=None):
+    """q/out [T][Hq][d]; k/v [T][Hkv][d]; spans_dev int32 [T][4]; tile map on the device (or None for fp32)."""
+    lib = load_library()
+    T, Hq, d = q.shape
+    Hkv = k.shape[1]
+    st = lib.padoc_ancestor_prefill_attn(_dev(q, "q"), _dev(k, "k"), _dev(v, "v"), _dtype_code(q), T, Hq, Hkv, d,
+                                         _dev(spans_dev, "spans"), _dev(row_ptr_dev, "row_ptr"),
+                                         _dev(k_tiles_dev, "k_tiles"), _dev(kinds_dev, "kinds"), q_tile, k_tile,
+                                         float(scale), _dev(out, "out"), _dev(lse, "lse"), _stream_ptr(stream))
+    _check("padoc_ancestor_prefill_attn", st)
+
+
+def padoc_check_device_errors(stream=None):
+    """Synchronizes the stream and raises PadocError if a kernel recorded a failed device check."""
+    lib = load_library()
+    st = lib.padoc_check_device_errors(_stream_ptr(stream))
+    if st != PADOC_OK:
+        code, detail = ctypes.c_int32(), ctypes.c_int32()
+        lib.padoc_last_device_error(ctypes.byref(code), ctypes.byref(detail))
+        err = PadocError("padoc_check_device_errors", st)
+        err.device_code, err.device_detail = code.value, detail.value
+        raise err
+
+
+def padoc_status_string(status: int) -> str:
+    return load_library().padoc_status_string(status).decode()
+
+
+def padoc_version() -> int:
+    return load_library().padoc_version()

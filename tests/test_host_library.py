@@ -1,0 +1,174 @@
+"""CPU tests of the C-ABI library: it loads, exports every declared entry point, and its host-side
+C1 planners (spans, tile map, decode plan) are bit-exact against the oracle and valid."""
+import os
+import re
+
+import numpy as np
+import pytest
+
+import oracle
+from paper_2608_06146_gb300 import build as pbuild
+from paper_2608_06146_gb300 import inputs
+from paper_2608_06146_gb300 import padoc_attn as pa
+from paper_2608_06146_gb300.inputs import PageSpec
+
+HEADER = os.path.join(os.path.dirname(os.path.dirname(__file__)), "include", "padoc_attn.h")
+
+
+@pytest.fixture(scope="module", autouse=True)
+def lib():
+    pbuild.build()
+    return pa.load_library()
+
+
+def _rand_pages(rng, n_pages, P_max=300, L_max=64, N_max=8, n_max=90):
+    pages = []
+    for _ in range(n_pages):
+        P = int(rng.integers(0, P_max + 1)); L = int(rng.integers(0, L_max + 1)); N = int(rng.integers(0, N_max + 1))
+        forks = [int(rng.integers(0, L + 1)) for _ in range(N)]
+        lens = [int(rng.integers(1, n_max + 1)) for _ in range(N)]
+        if P + L + sum(lens) == 0:
+            P = 1
+        pages.append(PageSpec(P, L, forks, lens))
+    return pages
+
+
+def test_exports_every_declared_symbol(lib):
+    declared = set(re.findall(r"^\w[\w\s\*]*?\b(padoc_\w+)\s*\(", open(HEADER).read(), re.M))
+    assert declared, "no declarations parsed"
+    for name in declared:
+        assert hasattr(lib, name), f"{name} not exported"
+    assert set(pa.exported_symbols()) == declared
+    assert pa.padoc_version() == 1
+    assert pa.padoc_status_string(0) == "ok"
+
+
+@pytest.mark.parametrize("seed", range(8))
+def test_spans_bit_exact_vs_oracle(seed):
+    rng = np.random.default_rng(seed)
+    pages = _rand_pages(rng, int(rng.integers(1, 6)))
+    np.testing.assert_array_equal(pa.padoc_build_query_spans(pages), oracle.spans(pages))
+
+
+@pytest.mark.parametrize("wl_name", ["tiny", "packed_prefill"])
+def test_spans_bit_exact_on_workloads(wl_name):
+    wl = inputs.WORKLOADS[wl_name]()
+    np.testing.assert_array_equal(pa.padoc_build_query_spans(wl.pages), oracle.spans(wl.pages))
+    shuffled = inputs.packed_prefill(shuffle_branches=True)
+    np.testing.assert_array_equal(pa.padoc_build_query_spans(shuffled.pages), oracle.spans(shuffled.pages))
+
+
+def _dense_kinds_from_map(row_ptr, kt, kind, nqt, nkt):
+    out = np.zeros((nqt, nkt), np.int8)
+    for r in range(nqt):
+        for e in range(row_ptr[r], row_ptr[r + 1]):
+            out[r, kt[e]] = kind[e]
+    return out
+
+
+@pytest.mark.parametrize("seed", range(6))
+@pytest.mark.parametrize("qb,kb", [(128, 128), (16, 32), (64, 16)])
+def test_tile_map_bit_exact_vs_oracle_brute_force(seed, qb, kb):
+    rng = np.random.default_rng(100 + seed)
+    pages = _rand_pages(rng, int(rng.integers(1, 5)))
+    row_ptr, kt, kind = pa.padoc_build_tile_map(pages, qb, kb)
+    T = oracle.total_tokens(pages)
+    want = oracle.tile_kinds(pages, qb, kb)
+    nqt, nkt = want.shape
+    assert len(row_ptr) == nqt + 1 and row_ptr[0] == 0 and row_ptr[-1] == len(kt)
+    for r in range(nqt):   # ascending k-tiles within each q-tile
+        assert np.all(np.diff(kt[row_ptr[r]:row_ptr[r + 1]]) > 0)
+    np.testing.assert_array_equal(_dense_kinds_from_map(row_ptr, kt, kind, nqt, nkt), want)
+    assert pa.padoc_tile_map_size(pages, qb, kb) == (nqt, len(kt))
+    assert T > 0
+
+
+def test_tile_map_full_size_packed_prefill_matches_interval_count():
+    # 32768 tokens is too large for the quadratic brute force; count visible pairs per tile from the
+    # oracle's spans with interval arithmetic instead.
+    wl = inputs.packed_prefill()
+    sp = oracle.spans(wl.pages)
+    T = sp.shape[0]
+    row_ptr, kt, kind = pa.padoc_build_tile_map(wl.pages, 128, 128)
+    nqt, nkt = -(-T // 128), -(-T // 128)
+    cnt = np.zeros((nqt, nkt), np.int64)
+    cols = np.arange(nkt) * 128
+    for s in (0, 2):
+        a = sp[:, s][:, None]; b = sp[:, s + 1][:, None]
+        ov = np.clip(np.minimum(b, cols + 128) - np.maximum(a, cols), 0, None)   # [T][nkt]
+        np.add.at(cnt, np.arange(T) // 128, ov)
+    rows = np.minimum(128, T - np.arange(nqt) * 128)[:, None]
+    want = np.where(cnt == 0, 0, np.where(cnt == rows * 128, 2, 1)).astype(np.int8)
+    np.testing.assert_array_equal(_dense_kinds_from_map(row_ptr, kt, kind, nqt, nkt), want)
+
+
+@pytest.mark.parametrize("bad", [
+    [PageSpec(10, 4, [5], [3])],          # fork offset beyond the layout stream
+    [PageSpec(10, 4, [-1], [3])],         # negative fork offset
+    [PageSpec(10, 4, [2], [0])],          # a branch without its branch-start token
+    [PageSpec(0, 0, [], [])],             # an empty page
+    [PageSpec(-1, 4, [], [])],
+])
+def test_malformed_pages_rejected(bad):
+    with pytest.raises(pa.PadocError) as e:
+        pa.padoc_build_query_spans(bad)
+    assert e.value.status == 1
+    with pytest.raises(pa.PadocError):
+        pa.padoc_build_tile_map(bad, 128, 128)
+
+
+def _plan_items(plan, info):
+    items = plan[info.off_items: info.off_items + 8 * info.num_items].reshape(-1, 8)
+    return items
+
+
+@pytest.mark.parametrize("wl_name,layout", [("decode_page", False), ("dense_page", False), ("serving_batch", True),
+                                            ("tiny", False)])
+def test_decode_plan_covers_every_visible_token_once(wl_name, layout):
+    wl = inputs.WORKLOADS[wl_name]()
+    cfg = pa.make_decode_config(wl.num_q_heads, wl.num_kv_heads, wl.head_dim, 16, layout, 0)
+    plan, info = pa.padoc_build_decode_plan(wl.pages, cfg)
+    sp, sh, pl = inputs.decode_streams(wl, layout)
+    S = len(sp)
+    assert info.num_streams == S
+    np.testing.assert_array_equal(plan[info.off_stream_page: info.off_stream_page + S], sp)
+    np.testing.assert_array_equal(plan[info.off_shared_len: info.off_shared_len + S], sh)
+    np.testing.assert_array_equal(plan[info.off_private_len: info.off_private_len + S], pl)
+    slot_ptr = plan[info.off_slot_ptr: info.off_slot_ptr + S + 1]
+    assert slot_ptr[0] == 0 and slot_ptr[-1] == info.num_slots and np.all(np.diff(slot_ptr) >= 1)
+    items = _plan_items(plan, info)
+    # coverage[(stream, kv_head)] counts how often each visible token is read
+    cov_sh = {(s, g): np.zeros(sh[s], np.int32) for s in range(S) for g in range(wl.num_kv_heads)}
+    cov_pv = {(s, g): np.zeros(pl[s], np.int32) for s in range(S) for g in range(wl.num_kv_heads)}
+    slots_used = {(s, g): [] for s in range(S) for g in range(wl.num_kv_heads)}
+    page_first = {}
+    for s in range(S):
+        page_first.setdefault(int(sp[s]), s)
+    for kind, idx, g, tb, te, fs, ns, slot in items:
+        assert tb % 16 == 0 and te > tb and 1 <= ns <= 4
+        for s in range(fs, fs + ns):
+            if kind == 0:
+                assert sp[s] == idx
+                hi = min(te, sh[s])
+                if hi > tb:
+                    cov_sh[(s, g)][tb:hi] += 1
+            else:
+                assert s == idx and ns == 1
+                cov_pv[(s, g)][tb:te] += 1
+            slots_used[(s, g)].append(slot)
+    for key in cov_sh:
+        assert np.all(cov_sh[key] == 1) and np.all(cov_pv[key] == 1)
+        s = key[0]
+        assert sorted(slots_used[key]) == list(range(slot_ptr[s + 1] - slot_ptr[s]))
+    need = pa.padoc_decode_workspace_size(info)
+    assert need >= info.num_slots * wl.num_q_heads * (wl.head_dim + 1) * 4
+
+
+def test_decode_plan_rejects_bad_config():
+    wl = inputs.decode_page()
+    for cfg in [pa.make_decode_config(16, 3, 128), pa.make_decode_config(16, 2, 128, split_tokens=100)]:
+        with pytest.raises(pa.PadocError):
+            pa.padoc_build_decode_plan(wl.pages, cfg)
+    with pytest.raises(pa.PadocError) as e:
+        pa.padoc_build_decode_plan(wl.pages, pa.make_decode_config(16, 2, 128, block_size=32))
+    assert e.value.status == 2
