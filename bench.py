@@ -1,0 +1,448 @@
+"""Benchmark of padoc_attn on one GB300 (or N independent GPUs, weak scaling).
+
+A step is one pass of the hot path over one batch:
+  decode  -- one decode step for every branch of the 32-page concurrent serving batch (prefix
+             uniform in [1024,4096], Poisson(20) branches per page, log-normal private lengths):
+             the decode plan's split-K kernel over the paged bf16 cache plus the split-K merge;
+  prefill -- the packed ancestor prefill of 8 pages x 4096 tokens (reported in "prefill").
+Headline metric: decode queries/s (one query = one branch's newest token, all 16 query heads).
+
+Timing: W untimed warm-up steps, then K steps between CUDA events on the launching stream, with
+a barrier and a synchronize on both sides; the max over ranks is reported. Decode rotates over
+input replicas in distinct memory whose total exceeds 4x L2, so no step reads a previous step's
+data from L2. Prefill flushes L2 between steps (a write of a buffer larger than L2) and times
+each step with its own events. nvidia-smi samples clocks during the timed region.
+
+--impl reference times the fp64 CPU oracle on the host cores on a bounded sample of the same
+decode workload (the paper has no code; the oracle is the reference program here).
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "ancestor-attn decode queries/s, % of HBM roofline; packed prefill TFLOP/s"
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+# dram__bytes_read.sum + dram__bytes_write.sum per launch from the ncu captures summarised under
+# profiles/ (None until a capture of the current kernel exists).
+TRAFFIC_BYTES = {"decode": None, "prefill": None}
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return d, "measured"
+    return dict(FALLBACK_PEAKS), "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi clock/throttle sampling in the background during the timed region."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def __enter__(self):
+        fd, self.path = tempfile.mkstemp(prefix="clocks", suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+        time.sleep(0.3)
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            time.sleep(0.25)
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self):
+        if not self.path or not os.path.exists(self.path):
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        rows = []
+        for line in open(self.path):
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                rows.append((float(parts[1]), float(parts[2]), float(parts[3]) if parts[3] not in ("[N/A]", "N/A") else 0.0,
+                             parts[5], parts[6], parts[7], parts[8]))
+            except ValueError:
+                continue
+        os.unlink(self.path)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+        loaded = [r for r in rows if r[2] > 0.3 * max(x[2] for x in rows)] or rows
+        reasons = set()
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        for r in rows:
+            for n, v in zip(names, r[3:]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        return {"sm_mhz": statistics.median(r[0] for r in loaded), "sm_max_mhz": max(r[1] for r in rows),
+                "samples": len(rows), "reasons": sorted(reasons)}
+
+
+# ------------------------------------------------------------------------------------------------
+# Workloads
+# ------------------------------------------------------------------------------------------------
+
+def decode_bytes(wl, streams_sp, streams_sh, streams_pl):
+    """Minimum HBM bytes of one decode step: each page's visible shared stream once per KV head,
+    every private row once, Q in, O and LSE out."""
+    Hq, Hkv, d = wl.num_q_heads, wl.num_kv_heads, wl.head_dim
+    esz = 2
+    shared = 0
+    for p in range(len(wl.pages)):
+        mask = streams_sp == p
+        if mask.any():
+            shared += int(streams_sh[mask].max())
+    priv = int(streams_pl.sum())
+    S = len(streams_sp)
+    return (shared + priv) * Hkv * d * 2 * esz + S * Hq * d * esz * 2 + S * Hq * 4
+
+
+def prefill_flops(wl):
+    from paper_2608_06146_gb300.engine import visible_pairs
+    return 4.0 * wl.head_dim * wl.num_q_heads * visible_pairs(wl.pages)
+
+
+def l2_bytes(torch):
+    try:
+        return int(torch.cuda.get_device_properties(torch.cuda.current_device()).L2_cache_size)
+    except Exception:
+        return 129 * 1024 * 1024
+
+
+def bench_decode(args, torch, dev, rank, world):
+    from paper_2608_06146_gb300 import inputs
+    from paper_2608_06146_gb300 import padoc_attn as pa
+    from paper_2608_06146_gb300.engine import DecodePlan
+
+    wl = inputs.serving_batch(seed=3 + 1000 * rank)
+    scale = 1.0 / math.sqrt(wl.head_dim)
+    di = inputs.decode_inputs(wl, 3 + 1000 * rank, pool_slack=1.0)
+    plan = DecodePlan(wl.pages, wl.num_q_heads, wl.num_kv_heads, wl.head_dim, dev)
+    S = plan.num_streams
+    per_replica = (di.k_pool.numel() + di.v_pool.numel()) * 2
+    R = args.replicas if args.replicas > 0 else max(2, math.ceil(4 * l2_bytes(torch) / per_replica) + 1)
+    k_pools = [di.k_pool.to(dev) for _ in range(R)]
+    v_pools = [di.v_pool.to(dev) for _ in range(R)]
+    qs = [di.q.to(dev) for _ in range(R)]
+    page_table = torch.from_numpy(di.page_table).to(dev)
+    stream_table = torch.from_numpy(di.stream_table).to(dev)
+    outs = [torch.empty((S, wl.num_q_heads, wl.head_dim), dtype=torch.bfloat16, device=dev) for _ in range(R)]
+    lses = [torch.empty((S, wl.num_q_heads), dtype=torch.float32, device=dev) for _ in range(R)]
+    stream = torch.cuda.current_stream()
+
+    def step(i):
+        r = i % R
+        plan.run(k_pools[r], v_pools[r], page_table, stream_table, qs[r], scale, outs[r], lses[r], stream)
+
+    for i in range(args.warmup):
+        step(i)
+    pa.padoc_check_device_errors(stream)
+    barrier(torch, world)
+    torch.cuda.synchronize()
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(physical_gpu_index(torch.cuda.current_device())) as clk:
+        ev0.record(stream)
+        for i in range(args.steps):
+            step(args.warmup + i)
+        ev1.record(stream)
+        torch.cuda.synchronize()
+    barrier(torch, world)
+    pa.padoc_check_device_errors(stream)
+    ms = ev0.elapsed_time(ev1) / args.steps
+
+    sp, sh, pl = inputs.decode_streams(wl)
+    nbytes = decode_bytes(wl, sp, sh, pl)
+    launches = (1 if plan.info.num_items > 0 else 0) + 1
+    res = dict(ms=ms, streams=S, bytes=nbytes, launches=launches, clocks=clk.summary(), replicas=R,
+               pages=len(wl.pages), e2e_ms=None, h2d=0, d2h=0)
+    if args.no_e2e:
+        return res
+
+    # end to end through the public API: host C1 plan, host->device copies of the step's inputs
+    # (plan blob, block tables, queries, from pinned memory), the decode, and the read-back of O/LSE
+    q_host = di.q.pin_memory()
+    pt_host = torch.from_numpy(di.page_table).pin_memory()
+    st_host = torch.from_numpy(di.stream_table).pin_memory()
+    o_host = torch.empty((S, wl.num_q_heads, wl.head_dim), dtype=torch.bfloat16).pin_memory()
+    l_host = torch.empty((S, wl.num_q_heads), dtype=torch.float32).pin_memory()
+    q_dev = torch.empty_like(qs[0])
+    pt_dev, st_dev = torch.empty_like(page_table), torch.empty_like(stream_table)
+    cfg = plan.cfg
+    plan_dev = torch.empty(int(plan.info.plan_ints), dtype=torch.int32, device=dev)
+
+    def e2e_step(i):
+        r = i % R
+        blob, info = pa.padoc_build_decode_plan(wl.pages, cfg)
+        blob_t = torch.from_numpy(blob).pin_memory()
+        plan_dev.copy_(blob_t, non_blocking=True)
+        q_dev.copy_(q_host, non_blocking=True)
+        pt_dev.copy_(pt_host, non_blocking=True)
+        st_dev.copy_(st_host, non_blocking=True)
+        pa.padoc_branch_decode_attn(k_pools[r], v_pools[r], info, plan_dev, pt_dev, st_dev, q_dev, scale, outs[r],
+                                    lses[r], plan.workspace, stream)
+        o_host.copy_(outs[r], non_blocking=True)
+        l_host.copy_(lses[r], non_blocking=True)
+        return blob_t.numel() * 4
+
+    for i in range(max(args.warmup, 1)):
+        e2e_step(i)
+    torch.cuda.synchronize()
+    barrier(torch, world)
+    t0 = time.perf_counter()
+    blob_bytes = 0
+    e2e_steps = min(args.steps, 500)
+    for i in range(e2e_steps):
+        blob_bytes = e2e_step(i)
+    torch.cuda.synchronize()
+    e2e_ms = (time.perf_counter() - t0) * 1e3 / e2e_steps
+    barrier(torch, world)
+    h2d = blob_bytes + q_host.numel() * 2 + pt_host.numel() * 4 + st_host.numel() * 4
+    d2h = o_host.numel() * 2 + l_host.numel() * 4
+    res.update(e2e_ms=e2e_ms, h2d=h2d, d2h=d2h)
+    return res
+
+
+def bench_prefill(args, torch, dev, rank, world):
+    from paper_2608_06146_gb300 import inputs
+    from paper_2608_06146_gb300 import padoc_attn as pa
+    from paper_2608_06146_gb300.engine import PrefillPlan
+
+    wl = inputs.packed_prefill(seed=4 + 1000 * rank)
+    q, k, v = inputs.packed_qkv(wl, 4 + 1000 * rank)
+    plan = PrefillPlan(wl.pages, wl.dtype, wl.head_dim, dev)
+    q, k, v = q.to(dev), k.to(dev), v.to(dev)
+    out = torch.empty(q.shape, dtype=q.dtype, device=dev)
+    lse = torch.empty(q.shape[:2], dtype=torch.float32, device=dev)
+    scale = 1.0 / math.sqrt(wl.head_dim)
+    flush = torch.empty(2 * l2_bytes(torch), dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream()
+    steps = max(3, min(args.steps, 20))
+    for _ in range(max(args.warmup, 3)):
+        plan.run(q, k, v, scale, out, lse, stream)
+    pa.padoc_check_device_errors(stream)
+    barrier(torch, world)
+    times = []
+    for _ in range(steps):
+        flush.fill_(1)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        plan.run(q, k, v, scale, out, lse, stream)
+        e1.record(stream)
+        e1.synchronize()
+        times.append(e0.elapsed_time(e1))
+    pa.padoc_check_device_errors(stream)
+    barrier(torch, world)
+    ms = sum(times) / len(times)
+    return dict(ms=ms, flops=prefill_flops(wl), tokens=plan.T, steps=steps)
+
+
+# ------------------------------------------------------------------------------------------------
+# Distributed plumbing (one process per GPU; no data-path collective: pages are independent)
+# ------------------------------------------------------------------------------------------------
+
+def physical_gpu_index(local: int) -> int:
+    vis = os.environ.get("CUDA_VISIBLE_DEVICES")
+    if vis:
+        ids = [x.strip() for x in vis.split(",") if x.strip()]
+        if local < len(ids) and ids[local].isdigit():
+            return int(ids[local])
+    return local
+
+
+def barrier(torch, world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def max_over_ranks(torch, world, x: float) -> float:
+    if world == 1:
+        return x
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def cpu_baseline_decode(max_seconds=20.0):
+    """The fp64 oracle as it stands on this host's cores, on a bounded sample of the serving batch:
+    the first pages of the batch, as many as fit the time budget (at least one)."""
+    import oracle
+    from paper_2608_06146_gb300 import inputs
+    wl_full = inputs.serving_batch(seed=3)
+    scale = 1.0 / math.sqrt(wl_full.head_dim)
+    cores = int(os.environ.get("OMP_NUM_THREADS", os.cpu_count() or 1))
+    done_streams, elapsed, pages_used = 0, 0.0, 0
+    for p in range(len(wl_full.pages)):
+        wl = inputs.Workload("sample", [wl_full.pages[p]], 16, 2, 128, wl_full.dtype, "decode")
+        di = inputs.decode_inputs(wl, 3)
+        t0 = time.perf_counter()
+        oracle.decode(di.stream_page, di.shared_len, di.priv_len, di.page_off, di.priv_off, di.stream_k, di.stream_v,
+                      di.priv_k, di.priv_v, di.q, scale)
+        elapsed += time.perf_counter() - t0
+        done_streams += len(di.stream_page)
+        pages_used += 1
+        if elapsed > max_seconds / 2:
+            break
+    return {"value": done_streams / elapsed, "unit": "queries/s", "cores": cores, "kind": "oracle",
+            "sample": f"decode step of the first {pages_used} of 32 serving-batch pages ({done_streams} branch "
+                      f"queries x 16 heads), fp64, OpenMP, {elapsed:.2f} s"}
+
+
+def run_reference(args):
+    """The oracle as the reference arm: each step is the decode of a bounded sample of the serving
+    batch (the first 2 pages) on the host cores."""
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return 0
+    import oracle
+    from paper_2608_06146_gb300 import inputs
+    oracle.build()
+    wl_full = inputs.serving_batch(seed=3)
+    wl = inputs.Workload("sample", wl_full.pages[:2], 16, 2, 128, wl_full.dtype, "decode")
+    di = inputs.decode_inputs(wl, 3)
+    scale = 1.0 / math.sqrt(wl.head_dim)
+    S = len(di.stream_page)
+
+    def step():
+        oracle.decode(di.stream_page, di.shared_len, di.priv_len, di.page_off, di.priv_off, di.stream_k, di.stream_v,
+                      di.priv_k, di.priv_v, di.q, scale)
+
+    for _ in range(args.warmup):
+        step()
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        step()
+    dt = (time.perf_counter() - t0) / args.steps
+    value = S / dt
+    cores = int(os.environ.get("OMP_NUM_THREADS", os.cpu_count() or 1))
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "queries/s", "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": dt * 1e3, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": "concurrent serving batch decode step (sample: first 2 of 32 pages)",
+                       "streams": S, "num_q_heads": 16, "num_kv_heads": 2, "head_dim": 128, "block_size": 16},
+            "cpu_baseline": {"value": value, "unit": "queries/s", "cores": cores, "kind": "oracle",
+                             "sample": f"first 2 of 32 serving-batch pages, {S} branch queries per step"},
+            "e2e": {"value": value, "unit": "queries/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line))
+    return 0
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=4000)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="padoc", choices=["padoc", "reference"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--only", default="all", choices=["all", "decode", "prefill"])
+    ap.add_argument("--replicas", type=int, default=0, help="decode input replicas (0: enough to exceed 4x L2)")
+    ap.add_argument("--no-e2e", action="store_true")
+    args = ap.parse_args()
+    if args.impl == "reference":
+        return run_reference(args)
+
+    import torch
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("gloo")
+    torch.cuda.set_device(local)
+    dev = f"cuda:{local}"
+
+    # CPU baseline first: the oracle runs on the host cores before any GPU work of this process
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        import oracle
+        oracle.build()
+        cpu = cpu_baseline_decode()
+
+    from paper_2608_06146_gb300 import build as pbuild
+    pbuild.build()
+    if args.only == "prefill":
+        p = bench_prefill(args, torch, dev, rank, world)
+        pms = max_over_ranks(torch, world, p["ms"])
+        if rank == 0:
+            print(json.dumps({"prefill_ms": pms, "tflops": p["flops"] * world / (pms * 1e-3) / 1e12}))
+        return 0
+    d = bench_decode(args, torch, dev, rank, world)
+    p = None if args.only == "decode" else bench_prefill(args, torch, dev, rank, world)
+
+    peaks, peak_src = load_peaks()
+    ms = max_over_ranks(torch, world, d["ms"])
+    e2e_ms = max_over_ranks(torch, world, d["e2e_ms"] if d["e2e_ms"] is not None else float("nan"))
+    total_streams = d["streams"] * world   # each rank decodes its own batch of the same shape
+    value = total_streams / (ms * 1e-3)
+    achieved = d["bytes"] / (d["ms"] * 1e-3) / 1e9
+    roof = {"bound": "hbm", "achieved": achieved, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+            "frac": achieved / peaks["hbm_gbs"], "traffic": TRAFFIC_BYTES["decode"],
+            "peak_source": f"{peak_src} hbm_gbs", "kernel": "decode step (split-K kernel + merge)",
+            "algorithmic_bytes": d["bytes"], "frac_of_nominal_8tbs": achieved / 8000.0}
+    line = {"metric": METRIC, "value": value, "unit": "queries/s", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+            "config": {"workload": "concurrent serving batch decode step: 32 pages, prefix U[1024,4096], "
+                                   "Poisson(20) branches/page, log-normal private KV (median 96, cap 2048)",
+                       "pages": d["pages"], "streams_per_gpu": d["streams"], "num_q_heads": 16, "num_kv_heads": 2,
+                       "head_dim": 128, "block_size": 16, "parallelism": f"replicas x{world} (pages per GPU)",
+                       "l2": f"{d['replicas']} rotating input replicas > 4x L2"},
+            "roofline": roof, "gpu_launches": d["launches"] * args.steps, "clocks": d["clocks"],
+            "e2e": {"value": total_streams / (e2e_ms * 1e-3), "unit": "queries/s", "h2d_bytes_per_step": d["h2d"],
+                    "d2h_bytes_per_step": d["d2h"]}}
+    if cpu is not None:
+        line["cpu_baseline"] = cpu
+    if p is not None:
+        pms = max_over_ranks(torch, world, p["ms"])
+        tflops = p["flops"] * world / (pms * 1e-3) / 1e12
+        line["prefill"] = {"value": tflops, "unit": "TFLOP/s", "ms_per_step": pms, "steps": p["steps"],
+                           "workload": "packed ancestor prefill, 8 pages x 4096 tokens (32768), unmasked-entry FLOPs",
+                           "l2": "flushed between steps",
+                           "roofline": {"bound": "tensor", "achieved": p["flops"] / (p["ms"] * 1e-3) / 1e12,
+                                        "peak": peaks["bf16_tflops"], "unit": "TFLOP/s",
+                                        "frac": p["flops"] / (p["ms"] * 1e-3) / 1e12 / peaks["bf16_tflops"],
+                                        "traffic": TRAFFIC_BYTES["prefill"],
+                                        "peak_source": f"{peak_src} bf16_tflops (burst)",
+                                        "algorithmic_flops": p["flops"]}}
+    if rank == 0:
+        print(json.dumps(line))
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())
