@@ -212,6 +212,31 @@ padoc_status padoc_branch_decode_attn(const padoc_kv_pool *pool, const padoc_dec
                                       float *lse, void *workspace, size_t workspace_bytes,
                                       padoc_stream_t stream);
 
+/* Size of the device array that padoc_branch_decode_attn_noalloc uses as its workspace. */
+#define PADOC_STATIC_WORKSPACE_BYTES (16u << 20)
+
+/* padoc_branch_decode_attn for callers that cannot allocate device memory (a plugin inside a
+ * framework that owns all device memory and offers it no allocator, or a latency-critical decode
+ * loop that must not call cudaMalloc, which may synchronize the device). The paper has no
+ * counterpart: it is a deployment convenience of this library.
+ * Arguments, layouts and results are those of padoc_branch_decode_attn without the workspace
+ * arguments. The split-K partials go to a fixed 256-byte-aligned device array of
+ * PADOC_STATIC_WORKSPACE_BYTES (16 MiB) that every GPU which loads this library holds until the
+ * process exits; the call allocates nothing (no cudaMalloc, cudaFree or allocating library call).
+ *   - The first call on a device looks up that device's address of the array (once per device,
+ *     with that device current); make that first call before any stream capture.
+ *   - Every call shares the one array, and it keeps the last call's contents. The decode writes
+ *     every partial it later reads, so nothing needs clearing, but calls that overlap on the GPU
+ *     (other streams, other host threads, concurrent graph launches) race on it: serialize them.
+ *   - A plan whose padoc_decode_workspace_size exceeds PADOC_STATIC_WORKSPACE_BYTES is rejected
+ *     with PADOC_ERR_WORKSPACE_TOO_SMALL before any launch.
+ * Errors: as padoc_branch_decode_attn. */
+padoc_status padoc_branch_decode_attn_noalloc(const padoc_kv_pool *pool, const padoc_decode_plan *info,
+                                              const int32_t *plan_dev, const int32_t *page_block_table,
+                                              int32_t page_table_stride, const int32_t *stream_block_table,
+                                              int32_t stream_table_stride, const void *q, float scale, void *out,
+                                              float *lse, padoc_stream_t stream);
+
 /* C4: merge of split-K partial softmax results (softmax over a union of disjoint key sets):
  *   lse_r = ln sum_s exp(part_lse[s][r]),  out_r = sum_s exp(part_lse[s][r] - lse_r) part_o[s][r].
  * A part with lse = -inf weighs 0; a row whose parts are all -inf gets lse = -inf and out = 0.

@@ -16,6 +16,8 @@
 // movmatrix; the online softmax runs per head over the token axis with shuffles.
 #include <math.h>
 
+#include <mutex>
+
 #include "common.cuh"
 
 namespace {
@@ -472,4 +474,55 @@ extern "C" padoc_status padoc_splitk_combine(const float *part_o, const float *p
     else
         return PADOC_ERR_INVALID_ARGUMENT;
     return padoc_launch_status();
+}
+
+// ------------------------------------------------------------------------------------------------
+// Decode without caller-provided workspace.
+//
+// Some callers cannot allocate device memory: a plugin inside a host framework that owns all device
+// memory and hands its plugins no allocator, or a latency-critical decode loop where a cudaMalloc
+// (which may synchronize the device) is not acceptable. For them the split-K partials live in a
+// fixed array that every device loading this library holds until the process exits.
+// ------------------------------------------------------------------------------------------------
+namespace {
+
+__device__ __align__(256) uint8_t g_static_workspace[PADOC_STATIC_WORKSPACE_BYTES];
+
+constexpr int kMaxStaticDevices = 64;
+void *g_static_ws_ptr[kMaxStaticDevices] = {nullptr};
+std::mutex g_static_ws_mu;
+
+// Device address of this device's copy of the array. Host code must not pass the symbol itself to a
+// kernel: on the host it names a host-side stand-in, not device memory.
+void *static_workspace_address()
+{
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxStaticDevices) return nullptr;
+    std::lock_guard<std::mutex> lk(g_static_ws_mu);
+    if (!g_static_ws_ptr[dev]) {
+        void *p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_static_workspace) != cudaSuccess) return nullptr;
+        g_static_ws_ptr[dev] = p;
+    }
+    return g_static_ws_ptr[dev];
+}
+
+}  // namespace
+
+extern "C" padoc_status padoc_branch_decode_attn_noalloc(const padoc_kv_pool *pool, const padoc_decode_plan *info,
+                                                         const int32_t *plan_dev, const int32_t *page_block_table,
+                                                         int32_t page_table_stride, const int32_t *stream_block_table,
+                                                         int32_t stream_table_stride, const void *q, float scale,
+                                                         void *out, float *lse, padoc_stream_t stream)
+{
+    if (!info) return PADOC_ERR_INVALID_ARGUMENT;
+    size_t need = 0;
+    padoc_status st = padoc_decode_workspace_size(info, &need);
+    if (st != PADOC_OK) return st;
+    if (need > (size_t)PADOC_STATIC_WORKSPACE_BYTES) return PADOC_ERR_WORKSPACE_TOO_SMALL;
+    void *ws = static_workspace_address();
+    if (!ws) return PADOC_ERR_CUDA;
+    return padoc_branch_decode_attn(pool, info, plan_dev, page_block_table, page_table_stride, stream_block_table,
+                                    stream_table_stride, q, scale, out, lse, ws, (size_t)PADOC_STATIC_WORKSPACE_BYTES,
+                                    stream);
 }

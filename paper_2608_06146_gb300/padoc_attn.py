@@ -87,6 +87,9 @@ def load_library(path: Optional[str] = None):
         "padoc_branch_decode_attn": [ctypes.POINTER(padoc_kv_pool), ctypes.POINTER(padoc_decode_plan), _vp, _vp,
                                      ctypes.c_int32, _vp, ctypes.c_int32, _vp, ctypes.c_float, _vp, _vp, _vp,
                                      ctypes.c_size_t, _vp],
+        "padoc_branch_decode_attn_noalloc": [ctypes.POINTER(padoc_kv_pool), ctypes.POINTER(padoc_decode_plan), _vp,
+                                             _vp, ctypes.c_int32, _vp, ctypes.c_int32, _vp, ctypes.c_float, _vp, _vp,
+                                             _vp],
         "padoc_splitk_combine": [_vp, _vp, ctypes.c_int32, ctypes.c_int64, ctypes.c_int32, ctypes.c_int, _vp, _vp, _vp],
         "padoc_ancestor_prefill_attn": [_vp, _vp, _vp, ctypes.c_int, ctypes.c_int64, ctypes.c_int32, ctypes.c_int32,
                                         ctypes.c_int32, _vp, _vp, _vp, _vp, ctypes.c_int32, ctypes.c_int32,
@@ -110,6 +113,7 @@ def exported_symbols() -> Sequence[str]:
     return [n for n in ("padoc_packed_size", "padoc_build_query_spans", "padoc_prefill_tile_shape",
                         "padoc_tile_map_size", "padoc_build_tile_map", "padoc_decode_plan_size",
                         "padoc_build_decode_plan", "padoc_decode_workspace_size", "padoc_branch_decode_attn",
+                        "padoc_branch_decode_attn_noalloc",
                         "padoc_splitk_combine", "padoc_ancestor_prefill_attn", "padoc_check_device_errors",
                         "padoc_last_device_error", "padoc_status_string", "padoc_version")]
 
@@ -253,6 +257,23 @@ def padoc_branch_decode_attn(k_pool, v_pool, info: padoc_decode_plan, plan_dev, 
                                       _dev(stream_table, "stream_table"), stream_table.shape[1], _dev(q, "q"),
                                       float(scale), _dev(out, "out"), _dev(lse, "lse"), ws, wsb, _stream_ptr(stream))
     _check("padoc_branch_decode_attn", st)
+
+
+PADOC_STATIC_WORKSPACE_BYTES = 16 << 20
+
+
+def padoc_branch_decode_attn_noalloc(k_pool, v_pool, info: padoc_decode_plan, plan_dev, page_table, stream_table, q,
+                                     scale, out, lse, stream=None):
+    """padoc_branch_decode_attn for callers that cannot allocate device memory: the split-K partials
+    go to the library's fixed 16 MiB device array (shared by every call; serialize calls)."""
+    lib = load_library()
+    pool = padoc_kv_pool(_dev(k_pool, "k_pool"), _dev(v_pool, "v_pool"), k_pool.shape[0], k_pool.shape[2],
+                         k_pool.shape[1], k_pool.shape[3], _dtype_code(k_pool))
+    st = lib.padoc_branch_decode_attn_noalloc(ctypes.byref(pool), ctypes.byref(info), _dev(plan_dev, "plan_dev"),
+                                              _dev(page_table, "page_table"), page_table.shape[1],
+                                              _dev(stream_table, "stream_table"), stream_table.shape[1], _dev(q, "q"),
+                                              float(scale), _dev(out, "out"), _dev(lse, "lse"), _stream_ptr(stream))
+    _check("padoc_branch_decode_attn_noalloc", st)
 
 
 def padoc_splitk_combine(part_o, part_lse, out, lse=None, stream=None):
