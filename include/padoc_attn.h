@@ -273,6 +273,15 @@ padoc_status padoc_ancestor_prefill_attn(const void *q, const void *k, const voi
  * Status
  * ========================================================================================== */
 
+/* Self-check of the tensor-core encodings the bf16 kernels rely on (no counterpart in the paper:
+ * a hardware check a caller may run once per device). With a, bk, v (device) bf16 [128][128]
+ * row-major, computes on one CTA with tcgen05 MMAs whose operands sit in 128-byte-swizzled shared
+ * memory: c1 = a . bk^T (both operands K-major) and c2 = a . v (v as an MN-major operand), fp32
+ * [128][128] row-major (device). The caller compares them with its own product.
+ * Errors: INVALID_ARGUMENT, CUDA. */
+padoc_status padoc_selftest_tcgen05(const void *a, const void *bk, const void *v, float *c1, float *c2,
+                                    padoc_stream_t stream);
+
 /* Synchronizes `stream`, then reads and clears the current device's error word. Returns
  * PADOC_ERR_DEVICE_CHECK if a kernel recorded a failed check since the last call (code and detail
  * via padoc_last_device_error), PADOC_ERR_CUDA if the stream reports an error, else PADOC_OK. */

@@ -175,6 +175,12 @@ int *padoc_device_error_word();
 bool padoc_make_tmap_bf16(CUtensorMap *map, const void *base, uint64_t cols, uint64_t rows,
                           uint64_t row_stride_bytes, uint32_t box_cols, uint32_t box_rows);
 padoc_status padoc_launch_status();
+// tcgen05 packed prefill (prefill_tc.cu); arguments validated by the caller.
+padoc_status padoc_launch_prefill_tc(const void *q, const void *k, const void *v, int64_t total_tokens,
+                                     int32_t num_q_heads, int32_t num_kv_heads, const int32_t *spans_dev,
+                                     const int32_t *tile_row_ptr_dev, const int32_t *tile_k_dev,
+                                     const int8_t *tile_kind_dev, float scale_log2, void *out, float *lse,
+                                     cudaStream_t stream);
 int padoc_num_sms();
 
 #define PADOC_CUDA_TRY(expr)                                   \

@@ -294,31 +294,6 @@ extern "C" padoc_status padoc_ancestor_prefill_attn(const void *q, const void *k
     if (head_dim != kD) return PADOC_ERR_UNSUPPORTED;
     if (q_tile != kQT || k_tile != kKT) return PADOC_ERR_INVALID_ARGUMENT;
     if (!tile_row_ptr_dev || !tile_k_dev || !tile_kind_dev) return PADOC_ERR_INVALID_ARGUMENT;
-    int *err = padoc_device_error_word();
-    if (!err) return PADOC_ERR_CUDA;
-    const int64_t nqt = (total_tokens + kQT - 1) / kQT;
-    if (nqt > 65535) return PADOC_ERR_UNSUPPORTED;
-
-    CUtensorMap qmap, kmap, vmap;
-    if (!padoc_make_tmap_bf16(&qmap, q, (uint64_t)num_q_heads * kD, total_tokens, (uint64_t)num_q_heads * kD * 2, 64, kQT) ||
-        !padoc_make_tmap_bf16(&kmap, k, (uint64_t)num_kv_heads * kD, total_tokens, (uint64_t)num_kv_heads * kD * 2, 64, kKT) ||
-        !padoc_make_tmap_bf16(&vmap, v, (uint64_t)num_kv_heads * kD, total_tokens, (uint64_t)num_kv_heads * kD * 2, 64, kKT))
-        return PADOC_ERR_CUDA;
-    PrefillParams prm;
-    prm.spans = spans_dev;
-    prm.row_ptr = tile_row_ptr_dev;
-    prm.tile_k = tile_k_dev;
-    prm.tile_kind = tile_kind_dev;
-    prm.T = total_tokens;
-    prm.num_q_heads = num_q_heads;
-    prm.num_kv_heads = num_kv_heads;
-    prm.num_q_tiles = (int32_t)nqt;
-    prm.scale_log2 = sl2;
-    prm.out = (__nv_bfloat16 *)out;
-    prm.lse = lse;
-    prm.err = err;
-    PADOC_CUDA_TRY(cudaFuncSetAttribute(prefill_mma_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kPrefillSmem));
-    dim3 grid((unsigned)num_q_heads, (unsigned)nqt);
-    prefill_mma_kernel<<<grid, 256, kPrefillSmem, cs>>>(qmap, kmap, vmap, prm);
-    return padoc_launch_status();
+    return padoc_launch_prefill_tc(q, k, v, total_tokens, num_q_heads, num_kv_heads, spans_dev, tile_row_ptr_dev,
+                                   tile_k_dev, tile_kind_dev, sl2, out, lse, cs);
 }

@@ -94,6 +94,7 @@ def load_library(path: Optional[str] = None):
         "padoc_ancestor_prefill_attn": [_vp, _vp, _vp, ctypes.c_int, ctypes.c_int64, ctypes.c_int32, ctypes.c_int32,
                                         ctypes.c_int32, _vp, _vp, _vp, _vp, ctypes.c_int32, ctypes.c_int32,
                                         ctypes.c_float, _vp, _vp, _vp],
+        "padoc_selftest_tcgen05": [_vp, _vp, _vp, _vp, _vp, _vp],
         "padoc_check_device_errors": [_vp],
         "padoc_last_device_error": [_i32p, _i32p],
         "padoc_status_string": [ctypes.c_int],
@@ -114,7 +115,8 @@ def exported_symbols() -> Sequence[str]:
                         "padoc_tile_map_size", "padoc_build_tile_map", "padoc_decode_plan_size",
                         "padoc_build_decode_plan", "padoc_decode_workspace_size", "padoc_branch_decode_attn",
                         "padoc_branch_decode_attn_noalloc",
-                        "padoc_splitk_combine", "padoc_ancestor_prefill_attn", "padoc_check_device_errors",
+                        "padoc_splitk_combine", "padoc_ancestor_prefill_attn", "padoc_selftest_tcgen05",
+                        "padoc_check_device_errors",
                         "padoc_last_device_error", "padoc_status_string", "padoc_version")]
 
 
@@ -300,6 +302,13 @@ def padoc_ancestor_prefill_attn(q, k, v, spans_dev, row_ptr_dev, k_tiles_dev, ki
                                          _dev(k_tiles_dev, "k_tiles"), _dev(kinds_dev, "kinds"), q_tile, k_tile,
                                          float(scale), _dev(out, "out"), _dev(lse, "lse"), _stream_ptr(stream))
     _check("padoc_ancestor_prefill_attn", st)
+
+
+def padoc_selftest_tcgen05(a, bk, v, c1, c2, stream=None):
+    """c1 = a . bk^T and c2 = a . v on the tensor cores (bf16 [128][128] inputs, fp32 outputs)."""
+    lib = load_library()
+    _check("padoc_selftest_tcgen05", lib.padoc_selftest_tcgen05(_dev(a, "a"), _dev(bk, "bk"), _dev(v, "v"),
+                                                                _dev(c1, "c1"), _dev(c2, "c2"), _stream_ptr(stream)))
 
 
 def padoc_check_device_errors(stream=None):
