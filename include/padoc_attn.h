@@ -276,10 +276,10 @@ padoc_status padoc_ancestor_prefill_attn(const void *q, const void *k, const voi
 /* Self-check of the tensor-core encodings the bf16 kernels rely on (no counterpart in the paper:
  * a hardware check a caller may run once per device). With a, bk, v (device) bf16 [128][128]
  * row-major, computes on one CTA with tcgen05 MMAs whose operands sit in 128-byte-swizzled shared
- * memory: c1 = a . bk^T (both operands K-major) and c2 = a . v (v as an MN-major operand), fp32
- * [128][128] row-major (device). The caller compares them with its own product.
- * Errors: INVALID_ARGUMENT, CUDA. */
-padoc_status padoc_selftest_tcgen05(const void *a, const void *bk, const void *v, float *c1, float *c2,
+ * memory: c1 = a . bk^T (both operands K-major), c2 = a . v (v as an MN-major operand) and
+ * c3 = a . v with a read from tensor memory, fp32 [128][128] row-major (device). The caller
+ * compares them with its own product. Errors: INVALID_ARGUMENT, CUDA. */
+padoc_status padoc_selftest_tcgen05(const void *a, const void *bk, const void *v, float *c1, float *c2, float *c3,
                                     padoc_stream_t stream);
 
 /* Synchronizes `stream`, then reads and clears the current device's error word. Returns

@@ -2,17 +2,22 @@
 // (App. C.1: the causal problem over M and one bottom-right-aligned causal problem per branch over
 // [K_{M<=f_k}; K_{Y_k}], computed in packed order without a gather).
 //
-// One CTA per (128-row q-tile, query head), walking the q-tile's entries of the tile map (fully
-// masked k-tiles are never visited; FULL tiles skip masking; PARTIAL tiles mask each row with its
-// two spans). Warp roles:
-//   warps 0-3  softmax + epilogue; thread t owns query row t (TMEM lane t), so row max and row sum
-//              need no shuffles;
-//   warp 4     TMA producer: Q once, then K and V tiles (128 keys x 128 dims, two 64-column
-//              panels each, 128-byte swizzle) into a 2-stage ring;
-//   warp 5     TMEM allocation and the MMA issuer (one thread).
-// TMEM (512 columns): S double-buffered at columns 0 and 128 (so S_{j+1} = Q K_{j+1}^T runs on the
-// tensor cores while the softmax of tile j runs), O at column 256. P is written as bf16 into a
-// 128-byte-swizzled K-major shared-memory tile and consumed by O += P V (V as an MN-major operand).
+// One CTA per (128-row q-tile, pair of query heads sharing a KV head); with an odd GQA group the
+// CTA takes one head. It walks the q-tile's entries of the tile map: fully masked k-tiles are never
+// visited, FULL tiles skip masking, PARTIAL tiles mask each row with its two spans. The two heads
+// share every K/V tile the producer stages, and their softmax warpgroups alternate with the tensor
+// core (while one warpgroup exponentiates, the MMAs of the other head run).
+//
+// Warp roles (320 threads):
+//   warps 0-3 / 4-7  softmax + epilogue of head 0 / head 1; thread t owns query row t (TMEM lane
+//                    t), so row max and row sum need no shuffles;
+//   warp 8           TMA producer: both heads' Q once, then K and V tiles (128 keys x 128 dims,
+//                    two 64-column panels each, 128-byte swizzle) into a 2-stage ring;
+//   warp 9           TMEM allocation and the MMA issuer (one thread).
+// TMEM (512 columns): head i keeps S_i at columns 128i..128i+127 and O_i at 256+128i. The softmax
+// writes P_i as packed bf16 over the first 64 columns of S_i, and O_i += P_i V reads P_i straight
+// from TMEM (V as an MN-major shared-memory operand). For head i the MMAs run S_i(j) -> P_i(j) ->
+// PV_i(j) -> S_i(j+1) in issue order, so S_i(j+1) never overwrites a P_i still being read.
 // O is rescaled lazily: the reference maximum only moves when a row's maximum grows by more than
 // 2^8, which keeps every P entry <= 256 and the arithmetic exact up to rounding.
 // Every wait is bounded; a wait that runs out records an error, all roles leave their loops, the
@@ -31,28 +36,27 @@ constexpr int kPanel = 128 * 128;    // [128 rows][64 bf16]
 constexpr int kTile = 2 * kPanel;    // 32 KB
 constexpr int kStages = 2;
 constexpr uint32_t kTmemCols = 512;
-constexpr uint32_t kColO = 256;
+constexpr int kThreads = 320;
 
 enum {
     B_Q = 0,
-    B_KFULL = 1,     // [2]
-    B_VFULL = 3,     // [2]
-    B_KVEMPTY = 5,   // [2]
-    B_SFULL = 7,     // [2]
-    B_SFREE = 9,     // [2]
-    B_PFULL = 11,
-    B_PVDONE = 12,
+    B_KFULL = 1,     // [stage]
+    B_VFULL = 3,     // [stage]
+    B_KVEMPTY = 5,   // [stage]
+    B_SFULL = 7,     // [head]
+    B_PFULL = 9,     // [head], 128 arrivals
+    B_PVDONE = 11,   // [head]
     B_FINAL = 13,
     B_COUNT = 14
 };
 
-constexpr size_t kSmemBytes = 1024 + (size_t)kTile * (1 + 2 * kStages + 1) + B_COUNT * 8 + 64;
+constexpr size_t kSmemBytes = 1024 + (size_t)kTile * (2 + 2 * kStages) + B_COUNT * 8 + 64;
 
 struct TcPrefillParams {
     const int32_t *spans, *row_ptr, *tile_k;
     const int8_t *tile_kind;
     int64_t T;
-    int32_t num_q_heads, num_kv_heads, num_q_tiles;
+    int32_t num_q_heads, num_kv_heads, num_q_tiles, heads_per_cta;
     float scale_log2;
     __nv_bfloat16 *out;
     float *lse;
@@ -67,36 +71,35 @@ __device__ __forceinline__ bool wait_or_abort(uint32_t bar, uint32_t parity, int
     return false;
 }
 
-__global__ void __launch_bounds__(192, 1)
+__device__ __forceinline__ int clamp_tile(int x) { return min(max(x, 0), kKT); }
+
+__global__ void __launch_bounds__(kThreads, 1)
 prefill_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__ CUtensorMap kmap,
                   const __grid_constant__ CUtensorMap vmap, const TcPrefillParams prm)
 {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
-    uint8_t *sq = smem;
-    uint8_t *sk = sq + kTile;                 // [kStages] tiles
+    uint8_t *sq = smem;                       // [2 heads] tiles
+    uint8_t *sk = sq + 2 * kTile;             // [kStages] tiles
     uint8_t *sv = sk + kStages * kTile;       // [kStages] tiles
-    uint8_t *sp = sv + kStages * kTile;       // P
-    uint64_t *bars = (uint64_t *)(sp + kTile);
+    uint64_t *bars = (uint64_t *)(sv + kStages * kTile);
     uint32_t *tmem_slot = (uint32_t *)(bars + B_COUNT);
     volatile int *abort_flag = (volatile int *)(tmem_slot + 1);
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int h = blockIdx.x;
-    const int qt = prm.num_q_tiles - 1 - (int)blockIdx.y;
-    const int g = h / (prm.num_q_heads / prm.num_kv_heads);
+    const int nh = prm.heads_per_cta;
+    const int h0 = blockIdx.x * nh;
+    const int qt = prm.num_q_tiles - 1 - (int)blockIdx.y;   // heavier tiles (later in a page) first
+    const int g = h0 / (prm.num_q_heads / prm.num_kv_heads);
     const int e0 = prm.row_ptr[qt], ne = prm.row_ptr[qt + 1] - e0;
     auto bar = [&](int i) { return smem_u32(&bars[i]); };
 
     if (tid == 0) {
-        for (int i = 0; i < B_COUNT; ++i) {
-            const int cnt = (i == B_SFREE || i == B_SFREE + 1 || i == B_PFULL) ? 128 : 1;
-            mbar_init(bar(i), cnt);
-        }
+        for (int i = 0; i < B_COUNT; ++i) mbar_init(bar(i), (i == B_PFULL || i == B_PFULL + 1) ? 128 : 1);
         *abort_flag = 0;
         fence_barrier_init();
     }
-    if (warp == 5) {
+    if (warp == 9) {
         tmem_alloc(smem_u32(tmem_slot), kTmemCols);
         tmem_relinquish();
     }
@@ -105,15 +108,17 @@ prefill_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constan
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
 
-    if (warp == 4) {
+    if (warp == 8) {
         // ---------------------------------------------------------------- TMA producer
         if (lane == 0 && ne > 0) {
             tma_prefetch_desc(&qmap);
             tma_prefetch_desc(&kmap);
             tma_prefetch_desc(&vmap);
-            mbar_arrive_expect_tx(bar(B_Q), kTile);
-            tma_load_2d(smem_u32(sq), &qmap, h * kD, qt * kQT, bar(B_Q));
-            tma_load_2d(smem_u32(sq) + kPanel, &qmap, h * kD + 64, qt * kQT, bar(B_Q));
+            mbar_arrive_expect_tx(bar(B_Q), nh * kTile);
+            for (int i = 0; i < nh; ++i) {
+                tma_load_2d(smem_u32(sq + i * kTile), &qmap, (h0 + i) * kD, qt * kQT, bar(B_Q));
+                tma_load_2d(smem_u32(sq + i * kTile) + kPanel, &qmap, (h0 + i) * kD + 64, qt * kQT, bar(B_Q));
+            }
             int issued = 0;
             for (int j = 0; j < ne; ++j) {
                 const int s = j & 1;
@@ -135,148 +140,174 @@ prefill_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constan
                 mbar_wait_bounded(bar(B_VFULL + (j & 1)), (j >> 1) & 1, prm.err, 23);
             }
         }
-    } else if (warp == 5) {
+    } else if (warp == 9) {
         // ---------------------------------------------------------------- MMA issuer
         if (lane == 0 && ne > 0) {
             const uint32_t idS = umma_idesc_bf16(128, kKT, false);
             const uint32_t idPV = umma_idesc_bf16(128, kD, true);
-            const uint32_t uq = smem_u32(sq), up = smem_u32(sp);
-            bool ok = wait_or_abort(bar(B_Q), 0, prm.err, 30, abort_flag);
-            for (int j = 0; ok && j <= ne; ++j) {
-                if (j < ne) {
-                    const int s = j & 1;
-                    if (!wait_or_abort(bar(B_KFULL + s), (j >> 1) & 1, prm.err, 31, abort_flag)) break;
-                    if (j >= 2 && !wait_or_abort(bar(B_SFREE + s), ((j - 2) >> 1) & 1, prm.err, 32, abort_flag)) break;
-                    tc_fence_after();
-                    const uint32_t ub = smem_u32(sk + s * kTile);
+            auto issue_s = [&](int i, int stage) {
+                const uint32_t uq = smem_u32(sq + i * kTile), ub = smem_u32(sk + stage * kTile);
 #pragma unroll
-                    for (int ks = 0; ks < 8; ++ks) {
-                        const uint32_t off = (ks >> 2) * kPanel + (ks & 3) * 32;
-                        umma_bf16_ss(tmem + s * 128, umma_desc_sw128(uq + off, 16, 1024),
-                                     umma_desc_sw128(ub + off, 16, 1024), idS, ks > 0);
-                    }
-                    umma_commit(bar(B_SFULL + s));
+                for (int ks = 0; ks < 8; ++ks) {
+                    const uint32_t off = (ks >> 2) * kPanel + (ks & 3) * 32;
+                    umma_bf16_ss(tmem + 128 * i, umma_desc_sw128(uq + off, 16, 1024),
+                                 umma_desc_sw128(ub + off, 16, 1024), idS, ks > 0);
                 }
-                if (j >= 1) {
-                    const int jp = j - 1, s = jp & 1;
-                    if (!wait_or_abort(bar(B_PFULL), jp & 1, prm.err, 33, abort_flag)) break;
-                    if (!wait_or_abort(bar(B_VFULL + s), (jp >> 1) & 1, prm.err, 34, abort_flag)) break;
+                umma_commit(bar(B_SFULL + i));
+            };
+            bool ok = wait_or_abort(bar(B_Q), 0, prm.err, 30, abort_flag) &&
+                      wait_or_abort(bar(B_KFULL), 0, prm.err, 31, abort_flag);
+            if (ok) {
+                tc_fence_after();
+                for (int i = 0; i < nh; ++i) issue_s(i, 0);
+            }
+            for (int j = 0; ok && j < ne; ++j) {
+                const int s = j & 1, sn = (j + 1) & 1;
+                for (int i = 0; ok && i < nh; ++i) {
+                    if (!wait_or_abort(bar(B_PFULL + i), j & 1, prm.err, 32, abort_flag)) { ok = false; break; }
+                    if (i == 0 && !wait_or_abort(bar(B_VFULL + s), (j >> 1) & 1, prm.err, 33, abort_flag)) { ok = false; break; }
                     tc_fence_after();
                     const uint32_t uv = smem_u32(sv + s * kTile);
 #pragma unroll
-                    for (int kk = 0; kk < 8; ++kk) {
-                        const uint32_t aoff = (kk >> 2) * kPanel + (kk & 3) * 32;
-                        umma_bf16_ss(tmem + kColO, umma_desc_sw128(up + aoff, 16, 1024),
-                                     umma_desc_sw128(uv + kk * 2048, kPanel, 1024), idPV, (jp > 0 || kk > 0));
+                    for (int kk = 0; kk < 8; ++kk)
+                        umma_bf16_ts(tmem + 256 + 128 * i, tmem + 128 * i + kk * 8,
+                                     umma_desc_sw128(uv + kk * 2048, kPanel, 1024), idPV, (j > 0 || kk > 0));
+                    umma_commit(bar(B_PVDONE + i));
+                    if (i == nh - 1) umma_commit(bar(B_KVEMPTY + s));
+                    if (j + 1 < ne) {
+                        if (i == 0 && !wait_or_abort(bar(B_KFULL + sn), ((j + 1) >> 1) & 1, prm.err, 34, abort_flag)) { ok = false; break; }
+                        tc_fence_after();
+                        issue_s(i, sn);
                     }
-                    umma_commit(bar(B_PVDONE));
-                    umma_commit(bar(B_KVEMPTY + s));
                 }
             }
             // every MMA issued above must complete before TMEM is released
             umma_commit(bar(B_FINAL));
             mbar_wait_bounded(bar(B_FINAL), 0, prm.err, 35);
         }
-    } else {
+    } else if (warp / 4 < nh) {
         // ---------------------------------------------------------------- softmax + epilogue
-        const int row = tid;
+        const int hi = warp / 4;                    // head index inside the CTA
+        const int h = h0 + hi;
+        const int row = tid & 127;
         const int64_t t = (int64_t)qt * kQT + row;
         int a0 = 0, a1 = 0, b0 = 0, b1 = 0;
         if (t < prm.T) {
             const int4 v = *reinterpret_cast<const int4 *>(prm.spans + 4 * t);
             a0 = v.x; a1 = v.y; b0 = v.z; b1 = v.w;
         }
-        const uint32_t lane_base = tmem + ((uint32_t)(warp * 32) << 16);
+        const uint32_t lanes = (uint32_t)((warp & 3) * 32) << 16;
+        const uint32_t tS = tmem + lanes + 128 * hi, tO = tmem + lanes + 256 + 128 * hi;
+        const float c = prm.scale_log2;
         // every decision below is warp-uniform: the TMEM loads and stores are warp-collective
         auto wait_all = [&](int b, uint32_t parity, int site) {
             const bool r = wait_or_abort(bar(b), parity, prm.err, site, abort_flag);
             return __all_sync(0xffffffffu, r);
         };
-        float m_ref = -INFINITY, l = 0.f;
+        float m_ref = -INFINITY, l = 0.f;   // m_ref in raw score units
         bool ok = ne > 0;
+        int kt_next = ne > 0 ? prm.tile_k[e0] : 0, kind_next = ne > 0 ? prm.tile_kind[e0] : 0;
         for (int j = 0; ok && j < ne; ++j) {
-            const int s = j & 1;
-            if (!wait_all(B_SFULL + s, (j >> 1) & 1, 40)) { ok = false; break; }
+            const int kt = kt_next;
+            const bool full = kind_next == PADOC_TILE_FULL;   // the same for every row of the CTA
+            if (j + 1 < ne) { kt_next = prm.tile_k[e0 + j + 1]; kind_next = prm.tile_kind[e0 + j + 1]; }
+            if (!wait_all(B_SFULL + hi, j & 1, 40)) { ok = false; break; }
             tc_fence_after();
-            uint32_t sr[4][32];
+            // pass 1: row maximum, 32 columns at a time; a PARTIAL tile also writes its masked
+            // scores back so that pass 2 reads them unmasked
+            float mx4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+            if (full) {
 #pragma unroll
-            for (int c = 0; c < 4; ++c) tmem_ld32(lane_base + s * 128 + c * 32, sr[c]);
-            tmem_ld_wait();
-            tc_fence_before();
-            mbar_arrive(bar(B_SFREE + s));
-
-            const int kt = prm.tile_k[e0 + j];
-            const bool full = prm.tile_kind[e0 + j] == PADOC_TILE_FULL;
-            const int cbase = kt * kKT;
-            float mx = -INFINITY;
+                for (int q = 0; q < 4; ++q) {
+                    uint32_t sr[32];
+                    tmem_ld32(tS + q * 32, sr);
+                    tmem_ld_wait();
 #pragma unroll
-            for (int c = 0; c < 4; ++c) {
-#pragma unroll
-                for (int i = 0; i < 32; ++i) {
-                    float x = __uint_as_float(sr[c][i]) * prm.scale_log2;
-                    if (!full) {
-                        const int jj = cbase + c * 32 + i;
-                        const bool vis = (jj >= a0 && jj < a1) || (jj >= b0 && jj < b1);
-                        x = vis ? x : -INFINITY;
+                    for (int i = 0; i < 32; i += 8) {
+                        mx4[0] = fmax3f(mx4[0], __uint_as_float(sr[i]), __uint_as_float(sr[i + 1]));
+                        mx4[1] = fmax3f(mx4[1], __uint_as_float(sr[i + 2]), __uint_as_float(sr[i + 3]));
+                        mx4[2] = fmax3f(mx4[2], __uint_as_float(sr[i + 4]), __uint_as_float(sr[i + 5]));
+                        mx4[3] = fmax3f(mx4[3], __uint_as_float(sr[i + 6]), __uint_as_float(sr[i + 7]));
                     }
-                    sr[c][i] = __float_as_uint(x);
-                    mx = fmaxf(mx, x);
                 }
+            } else {
+                const int cb = kt * kKT;
+                const int lo0 = clamp_tile(a0 - cb), w0 = max(clamp_tile(a1 - cb) - lo0, 0);
+                const int lo1 = clamp_tile(b0 - cb), w1 = max(clamp_tile(b1 - cb) - lo1, 0);
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    const uint32_t vis = interval_bits(lo0, w0, q * 32) | interval_bits(lo1, w1, q * 32);
+                    uint32_t sr[32];
+                    tmem_ld32(tS + q * 32, sr);
+                    tmem_ld_wait();
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) sr[i] = (vis >> i) & 1u ? sr[i] : 0xff800000u;   // -inf
+#pragma unroll
+                    for (int i = 0; i < 32; i += 8) {
+                        mx4[0] = fmax3f(mx4[0], __uint_as_float(sr[i]), __uint_as_float(sr[i + 1]));
+                        mx4[1] = fmax3f(mx4[1], __uint_as_float(sr[i + 2]), __uint_as_float(sr[i + 3]));
+                        mx4[2] = fmax3f(mx4[2], __uint_as_float(sr[i + 4]), __uint_as_float(sr[i + 5]));
+                        mx4[3] = fmax3f(mx4[3], __uint_as_float(sr[i + 6]), __uint_as_float(sr[i + 7]));
+                    }
+                    tmem_st32(tS + q * 32, sr);
+                }
+                tmem_st_wait();
             }
+            const float mx = fmaxf(fmax3f(mx4[0], mx4[1], mx4[2]), mx4[3]);
             const float m_new = fmaxf(m_ref, mx);
             // a row with nothing accumulated yet (O holds zeros) adopts the new maximum directly;
             // otherwise the reference only moves when the maximum grew by more than 2^8
-            const bool rescale = m_ref != -INFINITY && m_new > m_ref + 8.f;
+            const bool rescale = m_ref != -INFINITY && (m_new - m_ref) * c > 8.f;
             if (m_ref == -INFINITY) m_ref = m_new;
             if (__any_sync(0xffffffffu, rescale)) {
-                if (!wait_all(B_PVDONE, (j - 1) & 1, 41)) { ok = false; break; }
-                tc_fence_after();
-                const float alpha = rescale ? fast_exp2(m_ref - m_new) : 1.f;
+                // PV_i(j-1) completed before S_i(j) (issue order), so O_i is quiescent here
+                const float alpha = rescale ? fast_exp2((m_ref - m_new) * c) : 1.f;
 #pragma unroll
-                for (int c = 0; c < 4; ++c) {
+                for (int q = 0; q < 4; ++q) {
                     uint32_t o[32];
-                    tmem_ld32(lane_base + kColO + c * 32, o);
+                    tmem_ld32(tO + q * 32, o);
                     tmem_ld_wait();
 #pragma unroll
                     for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * alpha);
-                    tmem_st32(lane_base + kColO + c * 32, o);
+                    tmem_st32(tO + q * 32, o);
                 }
-                tmem_st_wait();
                 if (rescale) { l *= alpha; m_ref = m_new; }
             }
-            const float mref = m_ref == -INFINITY ? 0.f : m_ref;
-            uint32_t pk[64];
-            float rs = 0.f;
+            const float moff = m_ref == -INFINITY ? 0.f : m_ref * c;
+            // pass 2: P = exp2(S * c - m * c) as packed bf16 over the first 64 columns of S
+            float rs[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-            for (int c = 0; c < 4; ++c) {
+            for (int half = 0; half < 2; ++half) {
+                uint32_t pk[32];
 #pragma unroll
-                for (int i = 0; i < 32; i += 2) {
-                    const float p0 = fast_exp2(__uint_as_float(sr[c][i]) - mref);
-                    const float p1 = fast_exp2(__uint_as_float(sr[c][i + 1]) - mref);
-                    rs += p0 + p1;
-                    pk[c * 16 + i / 2] = pack_bf16x2(p0, p1);
+                for (int qq = 0; qq < 2; ++qq) {
+                    const int q = half * 2 + qq;
+                    uint32_t sr[32];
+                    tmem_ld32(tS + q * 32, sr);
+                    tmem_ld_wait();
+#pragma unroll
+                    for (int i = 0; i < 32; i += 2) {
+                        const float p0 = fast_exp2(fmaf(__uint_as_float(sr[i]), c, -moff));
+                        const float p1 = fast_exp2(fmaf(__uint_as_float(sr[i + 1]), c, -moff));
+                        rs[(i >> 1) & 3] += p0 + p1;
+                        pk[qq * 16 + (i >> 1)] = pack_bf16x2(p0, p1);
+                    }
                 }
+                tmem_st32(tS + half * 32, pk);
             }
-            l += rs;
-            // the P tile is free once PV_{j-1} has read it
-            if (j >= 1 && !wait_all(B_PVDONE, (j - 1) & 1, 42)) { ok = false; break; }
-#pragma unroll
-            for (int c = 0; c < 16; ++c) {
-                const uint32_t off = (uint32_t)(c >> 3) * kPanel + sw128_offset(row, (c & 7) * 8);
-                *reinterpret_cast<uint4 *>(sp + off) = make_uint4(pk[4 * c], pk[4 * c + 1], pk[4 * c + 2], pk[4 * c + 3]);
-            }
-            fence_proxy_async_smem();
+            l += (rs[0] + rs[1]) + (rs[2] + rs[3]);
+            tmem_st_wait();
             tc_fence_before();
-            mbar_arrive(bar(B_PFULL));
+            mbar_arrive(bar(B_PFULL + hi));
         }
-        if (ok && wait_all(B_PVDONE, (ne - 1) & 1, 43)) {
+        if (ok && wait_all(B_PVDONE + hi, (ne - 1) & 1, 43)) {
             tc_fence_after();
             const float inv = l > 0.f ? 1.f / l : 0.f;
             __nv_bfloat16 *orow = prm.out + ((size_t)(t < prm.T ? t : 0) * prm.num_q_heads + h) * kD;
 #pragma unroll
-            for (int c = 0; c < 4; ++c) {
+            for (int q = 0; q < 4; ++q) {
                 uint32_t o[32];
-                tmem_ld32(lane_base + kColO + c * 32, o);
+                tmem_ld32(tO + q * 32, o);
                 tmem_ld_wait();
                 if (t < prm.T) {
 #pragma unroll
@@ -286,16 +317,17 @@ prefill_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constan
                         w.y = pack_bf16x2(__uint_as_float(o[i + 2]) * inv, __uint_as_float(o[i + 3]) * inv);
                         w.z = pack_bf16x2(__uint_as_float(o[i + 4]) * inv, __uint_as_float(o[i + 5]) * inv);
                         w.w = pack_bf16x2(__uint_as_float(o[i + 6]) * inv, __uint_as_float(o[i + 7]) * inv);
-                        *reinterpret_cast<uint4 *>(orow + c * 32 + i) = w;
+                        *reinterpret_cast<uint4 *>(orow + q * 32 + i) = w;
                     }
                 }
             }
-            if (t < prm.T) prm.lse[(size_t)t * prm.num_q_heads + h] = l > 0.f ? (m_ref + log2f(l)) * PADOC_LN2 : -INFINITY;
+            if (t < prm.T)
+                prm.lse[(size_t)t * prm.num_q_heads + h] = l > 0.f ? (m_ref * c + log2f(l)) * PADOC_LN2 : -INFINITY;
         }
     }
     tc_fence_before();
     __syncthreads();
-    if (warp == 5) {
+    if (warp == 9) {
         tc_fence_after();
         tmem_dealloc(tmem, kTmemCols);
     }
@@ -327,12 +359,13 @@ padoc_status padoc_launch_prefill_tc(const void *q, const void *k, const void *v
     prm.num_q_heads = num_q_heads;
     prm.num_kv_heads = num_kv_heads;
     prm.num_q_tiles = (int32_t)nqt;
+    prm.heads_per_cta = ((num_q_heads / num_kv_heads) % 2 == 0) ? 2 : 1;   // a pair must share its KV head
     prm.scale_log2 = scale_log2;
     prm.out = (__nv_bfloat16 *)out;
     prm.lse = lse;
     prm.err = err;
     PADOC_CUDA_TRY(cudaFuncSetAttribute(prefill_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes));
-    dim3 grid((unsigned)num_q_heads, (unsigned)nqt);
-    prefill_tc_kernel<<<grid, 192, kSmemBytes, stream>>>(qmap, kmap, vmap, prm);
+    dim3 grid((unsigned)(num_q_heads / prm.heads_per_cta), (unsigned)nqt);
+    prefill_tc_kernel<<<grid, kThreads, kSmemBytes, stream>>>(qmap, kmap, vmap, prm);
     return padoc_launch_status();
 }

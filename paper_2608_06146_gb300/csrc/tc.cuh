@@ -70,6 +70,18 @@ __device__ __forceinline__ void umma_bf16_ss(uint32_t d_tmem, uint64_t adesc, ui
         : "memory");
 }
 
+// D[tmem] (+)= A[tmem] . B[smem]^T, issued by one thread. A occupies M lanes x (K/2) columns: column c
+// of lane m holds A[m][2c] in its low and A[m][2c+1] in its high 16 bits.
+__device__ __forceinline__ void umma_bf16_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t bdesc, uint32_t idesc,
+                                             uint32_t accumulate)
+{
+    asm volatile(
+        "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+        " tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n}" ::"r"(d_tmem),
+        "r"(a_tmem), "l"(bdesc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+
 // Arrives once on the mbarrier when every tcgen05 operation issued so far by this thread completes.
 __device__ __forceinline__ void umma_commit(uint32_t mbar)
 {
@@ -104,6 +116,24 @@ __device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&r)[32
 
 __device__ __forceinline__ void tmem_ld_wait() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
 __device__ __forceinline__ void tmem_st_wait() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
+
+// Three-input maximum (one instruction on sm_100-family GPUs).
+__device__ __forceinline__ float fmax3f(float a, float b, float c)
+{
+    float r;
+    asm("max.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(a), "f"(b), "f"(c));
+    return r;
+}
+
+// Bits [s, e) of a 32-bit word, for the part of the column interval [lo, lo + w) that falls in the
+// 32 columns starting at base.
+__device__ __forceinline__ uint32_t interval_bits(int lo, int w, int base)
+{
+    const int s = max(lo - base, 0), e = min(lo + w - base, 32);
+    if (e <= s) return 0u;
+    const uint32_t ones = (e - s) >= 32 ? 0xffffffffu : ((1u << (e - s)) - 1u);
+    return ones << s;
+}
 
 __device__ __forceinline__ uint32_t elect_one()
 {

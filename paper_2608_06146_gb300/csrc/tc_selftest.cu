@@ -1,7 +1,7 @@
 // tc_selftest.cu -- a self-check of the tcgen05 encodings every tensor-core kernel of padoc_attn
 // relies on: 128-byte-swizzled K-major and MN-major shared-memory operands, the kind::f16
 // instruction descriptor, MMA completion through tcgen05.commit, and the 32x32b TMEM load layout
-// (TMEM lane = accumulator row).
+// (TMEM lane = accumulator row), and an A operand held in TMEM (written with tcgen05.st).
 #include "common.cuh"
 #include "tc.cuh"
 
@@ -13,7 +13,8 @@ constexpr size_t kSelftestSmem = 1024 + 3 * (size_t)kMat + 64;
 
 __global__ void __launch_bounds__(128, 1)
 tc_selftest_kernel(const __nv_bfloat16 *__restrict__ a, const __nv_bfloat16 *__restrict__ bk,
-                   const __nv_bfloat16 *__restrict__ v, float *__restrict__ c1, float *__restrict__ c2, int *err)
+                   const __nv_bfloat16 *__restrict__ v, float *__restrict__ c1, float *__restrict__ c2,
+                   float *__restrict__ c3, int *err)
 {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
@@ -36,13 +37,25 @@ tc_selftest_kernel(const __nv_bfloat16 *__restrict__ a, const __nv_bfloat16 *__r
         fence_barrier_init();
     }
     if (warp == 0) {
-        tmem_alloc(smem_u32(tmem_slot), 256);
+        tmem_alloc(smem_u32(tmem_slot), 512);
         tmem_relinquish();
     }
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
+    {   // A copied into TMEM columns 256..319: thread row r writes its 64 packed bf16 pairs
+        const int row = warp * 32 + lane;
+        for (int h = 0; h < 2; ++h) {
+            uint32_t r[32];
+            for (int j = 0; j < 32; ++j) r[j] = *reinterpret_cast<const uint32_t *>(a + row * 128 + h * 64 + 2 * j);
+            tmem_st32(tmem + ((uint32_t)(warp * 32) << 16) + 256 + h * 32, r);
+        }
+        tmem_st_wait();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
 
     if (tid == 0) {
         const uint32_t ua = smem_u32(sa), ub = smem_u32(sb), uv = smem_u32(sv);
@@ -56,6 +69,9 @@ tc_selftest_kernel(const __nv_bfloat16 *__restrict__ a, const __nv_bfloat16 *__r
             umma_bf16_ss(tmem + 128, umma_desc_sw128(ua + off, 16, 1024),
                          umma_desc_sw128(uv + ks * 2048, kPanel, 1024), umma_idesc_bf16(128, 128, true), ks > 0);
         }
+        for (int ks = 0; ks < 8; ++ks)     // C3 = A . V with A read from TMEM
+            umma_bf16_ts(tmem + 384, tmem + 256 + ks * 8, umma_desc_sw128(uv + ks * 2048, kPanel, 1024),
+                         umma_idesc_bf16(128, 128, true), ks > 0);
         umma_commit(smem_u32(bar));
     }
     __syncwarp();
@@ -63,11 +79,12 @@ tc_selftest_kernel(const __nv_bfloat16 *__restrict__ a, const __nv_bfloat16 *__r
     tc_fence_after();
     if (ok) {
         const int row = warp * 32 + lane;
-        for (int m = 0; m < 2; ++m) {
-            float *c = m == 0 ? c1 : c2;
+        for (int m = 0; m < 3; ++m) {
+            float *c = m == 0 ? c1 : (m == 1 ? c2 : c3);
+            const int col0 = m == 2 ? 384 : m * 128;
             for (int cc = 0; cc < 4; ++cc) {
                 uint32_t r[32];
-                tmem_ld32(tmem + ((uint32_t)(warp * 32) << 16) + m * 128 + cc * 32, r);
+                tmem_ld32(tmem + ((uint32_t)(warp * 32) << 16) + col0 + cc * 32, r);
                 tmem_ld_wait();
                 for (int j = 0; j < 32; ++j) c[row * 128 + cc * 32 + j] = __uint_as_float(r[j]);
             }
@@ -75,20 +92,20 @@ tc_selftest_kernel(const __nv_bfloat16 *__restrict__ a, const __nv_bfloat16 *__r
     }
     tc_fence_before();
     __syncthreads();
-    if (warp == 0) tmem_dealloc(tmem, 256);
+    if (warp == 0) tmem_dealloc(tmem, 512);
 }
 
 }  // namespace
 
 extern "C" padoc_status padoc_selftest_tcgen05(const void *a, const void *bk, const void *v, float *c1, float *c2,
-                                               padoc_stream_t stream)
+                                               float *c3, padoc_stream_t stream)
 {
-    if (!a || !bk || !v || !c1 || !c2) return PADOC_ERR_INVALID_ARGUMENT;
+    if (!a || !bk || !v || !c1 || !c2 || !c3) return PADOC_ERR_INVALID_ARGUMENT;
     if ((((uintptr_t)a) | ((uintptr_t)bk) | ((uintptr_t)v)) & 15) return PADOC_ERR_INVALID_ARGUMENT;
     int *err = padoc_device_error_word();
     if (!err) return PADOC_ERR_CUDA;
     PADOC_CUDA_TRY(cudaFuncSetAttribute(tc_selftest_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSelftestSmem));
     tc_selftest_kernel<<<1, 128, kSelftestSmem, (cudaStream_t)stream>>>(
-        (const __nv_bfloat16 *)a, (const __nv_bfloat16 *)bk, (const __nv_bfloat16 *)v, c1, c2, err);
+        (const __nv_bfloat16 *)a, (const __nv_bfloat16 *)bk, (const __nv_bfloat16 *)v, c1, c2, c3, err);
     return padoc_launch_status();
 }

@@ -94,7 +94,7 @@ def load_library(path: Optional[str] = None):
         "padoc_ancestor_prefill_attn": [_vp, _vp, _vp, ctypes.c_int, ctypes.c_int64, ctypes.c_int32, ctypes.c_int32,
                                         ctypes.c_int32, _vp, _vp, _vp, _vp, ctypes.c_int32, ctypes.c_int32,
                                         ctypes.c_float, _vp, _vp, _vp],
-        "padoc_selftest_tcgen05": [_vp, _vp, _vp, _vp, _vp, _vp],
+        "padoc_selftest_tcgen05": [_vp, _vp, _vp, _vp, _vp, _vp, _vp],
         "padoc_check_device_errors": [_vp],
         "padoc_last_device_error": [_i32p, _i32p],
         "padoc_status_string": [ctypes.c_int],
@@ -304,11 +304,13 @@ def padoc_ancestor_prefill_attn(q, k, v, spans_dev, row_ptr_dev, k_tiles_dev, ki
     _check("padoc_ancestor_prefill_attn", st)
 
 
-def padoc_selftest_tcgen05(a, bk, v, c1, c2, stream=None):
-    """c1 = a . bk^T and c2 = a . v on the tensor cores (bf16 [128][128] inputs, fp32 outputs)."""
+def padoc_selftest_tcgen05(a, bk, v, c1, c2, c3, stream=None):
+    """c1 = a . bk^T, c2 = a . v and c3 = a . v (a from tensor memory) on the tensor cores
+    (bf16 [128][128] inputs, fp32 outputs)."""
     lib = load_library()
     _check("padoc_selftest_tcgen05", lib.padoc_selftest_tcgen05(_dev(a, "a"), _dev(bk, "bk"), _dev(v, "v"),
-                                                                _dev(c1, "c1"), _dev(c2, "c2"), _stream_ptr(stream)))
+                                                                _dev(c1, "c1"), _dev(c2, "c2"), _dev(c3, "c3"),
+                                                                _stream_ptr(stream)))
 
 
 def padoc_check_device_errors(stream=None):
