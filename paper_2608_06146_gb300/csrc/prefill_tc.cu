@@ -73,6 +73,7 @@ __device__ __forceinline__ bool wait_or_abort(uint32_t bar, uint32_t parity, int
 
 __device__ __forceinline__ int clamp_tile(int x) { return min(max(x, 0), kKT); }
 
+template <int NH>
 __global__ void __launch_bounds__(kThreads, 1)
 prefill_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__ CUtensorMap kmap,
                   const __grid_constant__ CUtensorMap vmap, const TcPrefillParams prm)
@@ -87,7 +88,7 @@ prefill_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constan
     volatile int *abort_flag = (volatile int *)(tmem_slot + 1);
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int nh = prm.heads_per_cta;
+    constexpr int nh = NH;
     const int h0 = blockIdx.x * nh;
     const int qt = prm.num_q_tiles - 1 - (int)blockIdx.y;   // heavier tiles (later in a page) first
     const int g = h0 / (prm.num_q_heads / prm.num_kv_heads);
@@ -141,48 +142,60 @@ prefill_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constan
             }
         }
     } else if (warp == 9) {
-        // ---------------------------------------------------------------- MMA issuer
-        if (lane == 0 && ne > 0) {
-            const uint32_t idS = umma_idesc_bf16(128, kKT, false);
-            const uint32_t idPV = umma_idesc_bf16(128, kD, true);
+        // ---------------------------------------------------------------- MMA issuer (whole warp)
+        if (ne > 0) {
+            constexpr uint32_t idS = umma_idesc_bf16(128, kKT, false);
+            constexpr uint32_t idPV = umma_idesc_bf16(128, kD, true);
+            // descriptor bases; a K-step adds a constant to the 14-bit start-address field
+            // (addresses stay below 256 KB, so the field never carries)
+            const uint64_t dq0 = umma_desc_sw128(smem_u32(sq), 16, 1024);
+            const uint64_t dq1 = umma_desc_sw128(smem_u32(sq + kTile), 16, 1024);
+            const uint64_t dk0 = umma_desc_sw128(smem_u32(sk), 16, 1024);
+            const uint64_t dk1 = umma_desc_sw128(smem_u32(sk + kTile), 16, 1024);
+            const uint64_t dv0 = umma_desc_sw128(smem_u32(sv), kPanel, 1024);
+            const uint64_t dv1 = umma_desc_sw128(smem_u32(sv + kTile), kPanel, 1024);
+            auto wait_w = [&](int b, uint32_t parity, int site) {
+                const bool r = wait_or_abort(bar(b), parity, prm.err, site, abort_flag);
+                return __all_sync(0xffffffffu, r);
+            };
             auto issue_s = [&](int i, int stage) {
-                const uint32_t uq = smem_u32(sq + i * kTile), ub = smem_u32(sk + stage * kTile);
+                const uint64_t da = i ? dq1 : dq0, db = stage ? dk1 : dk0;
 #pragma unroll
                 for (int ks = 0; ks < 8; ++ks) {
-                    const uint32_t off = (ks >> 2) * kPanel + (ks & 3) * 32;
-                    umma_bf16_ss(tmem + 128 * i, umma_desc_sw128(uq + off, 16, 1024),
-                                 umma_desc_sw128(ub + off, 16, 1024), idS, ks > 0);
+                    const uint32_t off = ((ks >> 2) * kPanel + (ks & 3) * 32) >> 4;
+                    umma_bf16_ss_warp(tmem + 128 * i, da + off, db + off, idS, ks > 0);
                 }
-                umma_commit(bar(B_SFULL + i));
+                umma_commit_warp(bar(B_SFULL + i));
             };
-            bool ok = wait_or_abort(bar(B_Q), 0, prm.err, 30, abort_flag) &&
-                      wait_or_abort(bar(B_KFULL), 0, prm.err, 31, abort_flag);
+            bool ok = wait_w(B_Q, 0, 30) && wait_w(B_KFULL, 0, 31);
             if (ok) {
                 tc_fence_after();
-                for (int i = 0; i < nh; ++i) issue_s(i, 0);
+#pragma unroll
+                for (int i = 0; i < NH; ++i) issue_s(i, 0);
             }
             for (int j = 0; ok && j < ne; ++j) {
                 const int s = j & 1, sn = (j + 1) & 1;
-                for (int i = 0; ok && i < nh; ++i) {
-                    if (!wait_or_abort(bar(B_PFULL + i), j & 1, prm.err, 32, abort_flag)) { ok = false; break; }
-                    if (i == 0 && !wait_or_abort(bar(B_VFULL + s), (j >> 1) & 1, prm.err, 33, abort_flag)) { ok = false; break; }
+#pragma unroll
+                for (int i = 0; i < NH; ++i) {
+                    if (!wait_w(B_PFULL + i, j & 1, 32)) { ok = false; break; }
+                    if (i == 0 && !wait_w(B_VFULL + s, (j >> 1) & 1, 33)) { ok = false; break; }
                     tc_fence_after();
-                    const uint32_t uv = smem_u32(sv + s * kTile);
+                    const uint64_t db = s ? dv1 : dv0;
 #pragma unroll
                     for (int kk = 0; kk < 8; ++kk)
-                        umma_bf16_ts(tmem + 256 + 128 * i, tmem + 128 * i + kk * 8,
-                                     umma_desc_sw128(uv + kk * 2048, kPanel, 1024), idPV, (j > 0 || kk > 0));
-                    umma_commit(bar(B_PVDONE + i));
-                    if (i == nh - 1) umma_commit(bar(B_KVEMPTY + s));
+                        umma_bf16_ts_warp(tmem + 256 + 128 * i, tmem + 128 * i + kk * 8, db + kk * (2048 >> 4), idPV,
+                                          (j > 0 || kk > 0));
+                    umma_commit_warp(bar(B_PVDONE + i));
+                    if (i == NH - 1) umma_commit_warp(bar(B_KVEMPTY + s));
                     if (j + 1 < ne) {
-                        if (i == 0 && !wait_or_abort(bar(B_KFULL + sn), ((j + 1) >> 1) & 1, prm.err, 34, abort_flag)) { ok = false; break; }
+                        if (i == 0 && !wait_w(B_KFULL + sn, ((j + 1) >> 1) & 1, 34)) { ok = false; break; }
                         tc_fence_after();
                         issue_s(i, sn);
                     }
                 }
             }
             // every MMA issued above must complete before TMEM is released
-            umma_commit(bar(B_FINAL));
+            umma_commit_warp(bar(B_FINAL));
             mbar_wait_bounded(bar(B_FINAL), 0, prm.err, 35);
         }
     } else if (warp / 4 < nh) {
@@ -218,17 +231,20 @@ prefill_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constan
             float mx4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
             if (full) {
 #pragma unroll
-                for (int q = 0; q < 4; ++q) {
-                    uint32_t sr[32];
-                    tmem_ld32(tS + q * 32, sr);
+                for (int q = 0; q < 4; q += 2) {
+                    uint32_t sr[2][32];
+                    tmem_ld32(tS + q * 32, sr[0]);
+                    tmem_ld32(tS + q * 32 + 32, sr[1]);
                     tmem_ld_wait();
 #pragma unroll
-                    for (int i = 0; i < 32; i += 8) {
-                        mx4[0] = fmax3f(mx4[0], __uint_as_float(sr[i]), __uint_as_float(sr[i + 1]));
-                        mx4[1] = fmax3f(mx4[1], __uint_as_float(sr[i + 2]), __uint_as_float(sr[i + 3]));
-                        mx4[2] = fmax3f(mx4[2], __uint_as_float(sr[i + 4]), __uint_as_float(sr[i + 5]));
-                        mx4[3] = fmax3f(mx4[3], __uint_as_float(sr[i + 6]), __uint_as_float(sr[i + 7]));
-                    }
+                    for (int u = 0; u < 2; ++u)
+#pragma unroll
+                        for (int i = 0; i < 32; i += 8) {
+                            mx4[0] = fmax3f(mx4[0], __uint_as_float(sr[u][i]), __uint_as_float(sr[u][i + 1]));
+                            mx4[1] = fmax3f(mx4[1], __uint_as_float(sr[u][i + 2]), __uint_as_float(sr[u][i + 3]));
+                            mx4[2] = fmax3f(mx4[2], __uint_as_float(sr[u][i + 4]), __uint_as_float(sr[u][i + 5]));
+                            mx4[3] = fmax3f(mx4[3], __uint_as_float(sr[u][i + 6]), __uint_as_float(sr[u][i + 7]));
+                        }
                 }
             } else {
                 const int cb = kt * kKT;
@@ -279,16 +295,16 @@ prefill_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constan
 #pragma unroll
             for (int half = 0; half < 2; ++half) {
                 uint32_t pk[32];
+                uint32_t sr[2][32];
+                tmem_ld32(tS + half * 64, sr[0]);
+                tmem_ld32(tS + half * 64 + 32, sr[1]);
+                tmem_ld_wait();
 #pragma unroll
                 for (int qq = 0; qq < 2; ++qq) {
-                    const int q = half * 2 + qq;
-                    uint32_t sr[32];
-                    tmem_ld32(tS + q * 32, sr);
-                    tmem_ld_wait();
 #pragma unroll
                     for (int i = 0; i < 32; i += 2) {
-                        const float p0 = fast_exp2(fmaf(__uint_as_float(sr[i]), c, -moff));
-                        const float p1 = fast_exp2(fmaf(__uint_as_float(sr[i + 1]), c, -moff));
+                        const float p0 = fast_exp2(fmaf(__uint_as_float(sr[qq][i]), c, -moff));
+                        const float p1 = fast_exp2(fmaf(__uint_as_float(sr[qq][i + 1]), c, -moff));
                         rs[(i >> 1) & 3] += p0 + p1;
                         pk[qq * 16 + (i >> 1)] = pack_bf16x2(p0, p1);
                     }
@@ -364,8 +380,13 @@ padoc_status padoc_launch_prefill_tc(const void *q, const void *k, const void *v
     prm.out = (__nv_bfloat16 *)out;
     prm.lse = lse;
     prm.err = err;
-    PADOC_CUDA_TRY(cudaFuncSetAttribute(prefill_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes));
     dim3 grid((unsigned)(num_q_heads / prm.heads_per_cta), (unsigned)nqt);
-    prefill_tc_kernel<<<grid, kThreads, kSmemBytes, stream>>>(qmap, kmap, vmap, prm);
+    if (prm.heads_per_cta == 2) {
+        PADOC_CUDA_TRY(cudaFuncSetAttribute(prefill_tc_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes));
+        prefill_tc_kernel<2><<<grid, kThreads, kSmemBytes, stream>>>(qmap, kmap, vmap, prm);
+    } else {
+        PADOC_CUDA_TRY(cudaFuncSetAttribute(prefill_tc_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes));
+        prefill_tc_kernel<1><<<grid, kThreads, kSmemBytes, stream>>>(qmap, kmap, vmap, prm);
+    }
     return padoc_launch_status();
 }
