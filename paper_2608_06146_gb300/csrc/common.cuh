@@ -181,6 +181,11 @@ padoc_status padoc_launch_prefill_tc(const void *q, const void *k, const void *v
                                      const int32_t *tile_row_ptr_dev, const int32_t *tile_k_dev,
                                      const int8_t *tile_kind_dev, float scale_log2, void *out, float *lse,
                                      cudaStream_t stream);
+// tcgen05 shared-stream decode (decode_tc.cu): the plan's tensor-core items.
+padoc_status padoc_launch_decode_tc(const CUtensorMap *kmap, const CUtensorMap *vmap, const int32_t *plan,
+                                    const padoc_decode_plan *info, const int32_t *page_table, int32_t page_stride,
+                                    int32_t num_blocks, const void *q, float *part_o, float *part_lse, float scale_log2,
+                                    int *err, cudaStream_t stream);
 int padoc_num_sms();
 
 #define PADOC_CUDA_TRY(expr)                                   \

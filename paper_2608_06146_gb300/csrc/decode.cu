@@ -3,13 +3,16 @@
 // merge of partial softmax results, and the fp32 bring-up path.
 //
 // bf16 path. The planner cuts each page's shared stream into split-K pieces and each stream's
-// private rows into pieces; a work item is one piece for one KV head. A shared item covers up to
-// four streams of the page, so the piece's K/V is fetched from HBM once for all of them; every
-// stream keeps its own column cutoff P + f_k. Each 16-token paged block is one TMA box per
-// 64-column half (128-byte swizzle), staged through a 4-deep ring of 64-token stages.
+// private rows into pieces; a work item is one piece for one KV head. Pages whose branches x
+// query heads fill dense M = 128 tiles read their shared stream on the tensor cores
+// (decode_tc.cu): each K/V tile is fetched once for all of the page's streams. Every private
+// history, and the shared stream of pages with few branches, is read by the warp kernel below.
+// A split-K merge then joins each (stream, head)'s partials.
 //
-// Warp-level math ("heads as the N dimension"): for one stream the 8 query heads of a KV head
-// are the N = 8 columns of mma.m16n8k16, and the 16 tokens of a paged block are its M = 16 rows:
+// Warp kernel: every warp owns one work item and runs on its own: a 3-deep ring of 16-token
+// paged blocks fetched by TMA (one box per 64-column half of K and V, 128-byte swizzle) with its
+// own mbarriers, so no warp ever waits for another. The math puts the 8 query heads of a KV head
+// in the N = 8 columns of mma.m16n8k16 and the 16 tokens of a block in its M = 16 rows:
 //     S^T[16 tok x 8 heads] = K[16 x 128] . Q^T[128 x 8]             (8 MMAs)
 //     O^T[128 x 8 heads]   += V^T[128 x 16 tok] . P^T[16 tok x 8]    (8 MMAs)
 // so no MMA lane is padding. The P^T operand is the score fragment transposed in registers with
@@ -25,97 +28,73 @@ namespace {
 constexpr int kD = 128;          // head_dim of the bf16 path
 constexpr int kGroup = 8;        // query heads per KV head of the bf16 path
 constexpr int kBlk = 16;         // tokens per paged block
-constexpr int kStageBlocks = 4;  // paged blocks per pipeline stage
-constexpr int kStages = 4;       // pipeline depth
-constexpr int kWarps = 4;
-constexpr int kPanelBytes = kStageBlocks * kBlk * 128;   // [64 rows][64 cols] bf16
-constexpr int kStageBytes = 4 * kPanelBytes;             // K lo, K hi, V lo, V hi
-constexpr int kMergeStride = 132;                        // floats per head row of the merge area
-constexpr int kMergeWarpFloats = kGroup * kMergeStride + 2 * kGroup;
-constexpr size_t kDecodeSmem = 1024 + (size_t)kStages * kStageBytes + (size_t)kWarps * kMergeWarpFloats * 4 + 64;
+constexpr int kWarps = 8;              // warps (independent work items) per CTA
+constexpr int kWStages = 3;            // paged blocks in flight per warp
+constexpr int kBoxBytes = kBlk * 128;  // one 16-row x 64-column box
+constexpr int kWStageBytes = 4 * kBoxBytes;   // K lo, K hi, V lo, V hi
+constexpr int kWarpSmem = kWStages * kWStageBytes;
+constexpr size_t kDecodeSmem = 1024 + (size_t)kWarps * kWarpSmem + (size_t)kWarps * kWStages * 8 + 64;
+constexpr int kMergeStride = 132;      // floats per head row when a warp stages its O^T
 
 struct DecodeParams {
     const int32_t *stream_page, *shared_len, *private_len, *slot_ptr;
     const padoc_item *items;
+    int32_t first_item, num_items;
     const int32_t *page_table;
     const int32_t *stream_table;
     int32_t page_stride, stream_stride;
-    int32_t num_blocks, num_kv_heads, num_q_heads;
+    int32_t num_blocks, num_kv_heads, num_q_heads, pool_rows;
     const __nv_bfloat16 *q;
     float *part_o, *part_lse;
     float scale_log2;
     int *err;
 };
 
-__global__ void __launch_bounds__(128, 1)
-decode_mma_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap,
-                  const DecodeParams prm)
+__global__ void __launch_bounds__(kWarps * 32, 1)
+decode_warp_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap,
+                   const DecodeParams prm)
 {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
-    float *merge = (float *)(smem + (size_t)kStages * kStageBytes);
-    uint64_t *full_bar = (uint64_t *)(merge + kWarps * kMergeWarpFloats);
-
-    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const padoc_item it = prm.items[blockIdx.x];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int wi = blockIdx.x * kWarps + warp;
+    if (wi >= prm.num_items) return;   // warps are independent: no CTA-wide barrier follows
+    uint8_t *wbuf = smem + (size_t)warp * kWarpSmem;
+    uint64_t *full_bar = (uint64_t *)(smem + (size_t)kWarps * kWarpSmem) + warp * kWStages;
+    const padoc_item it = prm.items[prm.first_item + wi];
     const bool is_shared = it.kind == PADOC_ITEM_SHARED;
-    const int nb = it.num_streams;
-    const int wpb = nb == 1 ? 4 : (nb == 2 ? 2 : 1);   // warps per stream
-    const int my_b = warp / wpb, phase = warp % wpb;
-    const bool active = my_b < nb;
     const int g = it.kv_head;
+    const int s = it.first_stream;
     const int32_t *table = is_shared ? prm.page_table + (size_t)it.index * prm.page_stride
-                                     : prm.stream_table + (size_t)it.index * prm.stream_stride;
+                                     : prm.stream_table + (size_t)s * prm.stream_stride;
+    const int cutoff = min(is_shared ? prm.shared_len[s] : prm.private_len[s], it.tok_end);
     const int blk0 = it.tok_begin / kBlk;
-    const int nblk = (it.tok_end - it.tok_begin + kBlk - 1) / kBlk;
-    const int nstages = (nblk + kStageBlocks - 1) / kStageBlocks;
+    const int nblk = cutoff > it.tok_begin ? (cutoff - it.tok_begin + kBlk - 1) / kBlk : 0;
 
-    if (tid == 0) {
-        for (int i = 0; i < kStages; ++i) mbar_init(smem_u32(&full_bar[i]), 1);
+    if (lane == 0) {
+        for (int i = 0; i < kWStages; ++i) mbar_init(smem_u32(&full_bar[i]), 1);
         fence_barrier_init();
-        tma_prefetch_desc(&kmap);
-        tma_prefetch_desc(&vmap);
     }
-    __syncthreads();
-
-    auto issue = [&](int st) {
-        const uint32_t base = smem_u32(smem + (size_t)(st % kStages) * kStageBytes);
-        const uint32_t bar = smem_u32(&full_bar[st % kStages]);
-        uint32_t bytes = 0;
-        int32_t ids[kStageBlocks];
-        for (int b = 0; b < kStageBlocks; ++b) {
-            const int bi = st * kStageBlocks + b;
-            ids[b] = -1;
-            if (bi >= nblk) continue;
-            const int32_t id = table[blk0 + bi];
-            if (id < 0 || id >= prm.num_blocks) {
-                padoc_record_error(prm.err, PADOC_DEVERR_BLOCK_ID, id);
-                continue;
-            }
-            ids[b] = id;
-            bytes += 4 * kBlk * 128;
-        }
-        mbar_arrive_expect_tx(bar, bytes);
-        for (int b = 0; b < kStageBlocks; ++b) {
-            if (ids[b] < 0) continue;
-            const int32_t row = (ids[b] * prm.num_kv_heads + g) * kBlk;
-            const uint32_t off = (uint32_t)b * (kBlk * 128);
-            tma_load_2d(base + 0 * kPanelBytes + off, &kmap, 0, row, bar);
-            tma_load_2d(base + 1 * kPanelBytes + off, &kmap, 64, row, bar);
-            tma_load_2d(base + 2 * kPanelBytes + off, &vmap, 0, row, bar);
-            tma_load_2d(base + 3 * kPanelBytes + off, &vmap, 64, row, bar);
-        }
+    __syncwarp();
+    auto issue = [&](int bi) {   // lane 0 only
+        const uint32_t base = smem_u32(wbuf + (bi % kWStages) * kWStageBytes);
+        const uint32_t bar = smem_u32(&full_bar[bi % kWStages]);
+        const int32_t id = table[blk0 + bi];
+        int32_t row = prm.pool_rows;   // out of range: zero fill
+        if (id >= 0 && id < prm.num_blocks) row = (id * prm.num_kv_heads + g) * kBlk;
+        else padoc_record_error(prm.err, PADOC_DEVERR_BLOCK_ID, id);
+        mbar_arrive_expect_tx(bar, kWStageBytes);
+        tma_load_2d(base + 0 * kBoxBytes, &kmap, 0, row, bar);
+        tma_load_2d(base + 1 * kBoxBytes, &kmap, 64, row, bar);
+        tma_load_2d(base + 2 * kBoxBytes, &vmap, 0, row, bar);
+        tma_load_2d(base + 3 * kBoxBytes, &vmap, 64, row, bar);
     };
-    if (tid == 0)
-        for (int st = 0; st < kStages && st < nstages; ++st) issue(st);
+    if (lane == 0)
+        for (int bi = 0; bi < kWStages && bi < nblk; ++bi) issue(bi);
 
-    // per-thread state: heads h0 = 2*(lane%4), h0+1 of this warp's stream
-    const int s = it.first_stream + (active ? my_b : 0);
-    int cutoff = 0;
+    // query fragments: B operand Q^T[128 dims x 8 heads]
     uint32_t qb[8][2];
-    if (active) {
-        cutoff = is_shared ? prm.shared_len[s] : prm.private_len[s];
-        cutoff = min(cutoff, it.tok_end);
+    {
         const __nv_bfloat16 *qrow = prm.q + ((size_t)s * prm.num_q_heads + g * kGroup + (lane >> 2)) * kD;
 #pragma unroll
         for (int ks = 0; ks < 8; ++ks) {
@@ -123,128 +102,103 @@ decode_mma_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constan
             qb[ks][1] = *reinterpret_cast<const uint32_t *>(qrow + ks * 16 + 8 + (lane & 3) * 2);
         }
     }
-    float m[2] = {-INFINITY, -INFINITY}, l[2] = {0.f, 0.f};
+    float m[2] = {-INFINITY, -INFINITY}, l[2] = {0.f, 0.f};   // heads h0 = 2*(lane%4), h0+1
     float o[8][4];
 #pragma unroll
     for (int mt = 0; mt < 8; ++mt) o[mt][0] = o[mt][1] = o[mt][2] = o[mt][3] = 0.f;
 
-    int st = 0;
-    bool aborted = false;
-    for (; st < nstages; ++st) {
-        const bool ok = mbar_wait_bounded(smem_u32(&full_bar[st % kStages]), (st / kStages) & 1, prm.err, 1);
-        if (__syncthreads_or(!ok)) { aborted = true; break; }
-        const uint32_t base = smem_u32(smem + (size_t)(st % kStages) * kStageBytes);
-        if (active) {
-            for (int j = 0; j < kStageBlocks; ++j) {
-                const int bi = st * kStageBlocks + j;
-                if (bi >= nblk || (bi % wpb) != phase) continue;
-                const int tokbase = (blk0 + bi) * kBlk;
-                if (tokbase >= cutoff) continue;
-                // S^T = K . Q^T
-                float acc[4] = {0.f, 0.f, 0.f, 0.f};
+    int bi = 0;
+    for (; bi < nblk; ++bi) {
+        const bool ok = mbar_wait_bounded(smem_u32(&full_bar[bi % kWStages]), (bi / kWStages) & 1, prm.err, 1);
+        if (!__all_sync(0xffffffffu, ok)) break;
+        const uint32_t base = smem_u32(wbuf + (bi % kWStages) * kWStageBytes);
+        const int tokbase = (blk0 + bi) * kBlk;
+        // S^T = K . Q^T
+        float acc[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-                for (int ks = 0; ks < 8; ++ks) {
-                    const uint32_t row = j * kBlk + (lane & 15);
-                    const uint32_t col = (ks & 3) * 16 + (lane >> 4) * 8;
-                    uint32_t a[4];
-                    ldmatrix_x4(a, base + (ks >> 2) * kPanelBytes + sw128_offset(row, col));
-                    mma_bf16_16816(acc, a, qb[ks][0], qb[ks][1]);
-                }
-                const int t0 = tokbase + (lane >> 2), t1 = t0 + 8;
-                float sc[4];
-                sc[0] = t0 < cutoff ? acc[0] * prm.scale_log2 : -INFINITY;
-                sc[1] = t0 < cutoff ? acc[1] * prm.scale_log2 : -INFINITY;
-                sc[2] = t1 < cutoff ? acc[2] * prm.scale_log2 : -INFINITY;
-                sc[3] = t1 < cutoff ? acc[3] * prm.scale_log2 : -INFINITY;
-                float mx0 = fmaxf(sc[0], sc[2]), mx1 = fmaxf(sc[1], sc[3]);
-#pragma unroll
-                for (int sh = 4; sh < 32; sh <<= 1) {
-                    mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, sh));
-                    mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, sh));
-                }
-                const float mn0 = fmaxf(m[0], mx0), mn1 = fmaxf(m[1], mx1);
-                // a head whose columns are all masked so far keeps m = -inf and contributes 0
-                const float al0 = mn0 == -INFINITY ? 1.f : fast_exp2(m[0] - mn0);
-                const float al1 = mn1 == -INFINITY ? 1.f : fast_exp2(m[1] - mn1);
-                const float p0 = mn0 == -INFINITY ? 0.f : fast_exp2(sc[0] - mn0);
-                const float p1 = mn1 == -INFINITY ? 0.f : fast_exp2(sc[1] - mn1);
-                const float p2 = mn0 == -INFINITY ? 0.f : fast_exp2(sc[2] - mn0);
-                const float p3 = mn1 == -INFINITY ? 0.f : fast_exp2(sc[3] - mn1);
-                m[0] = mn0; m[1] = mn1;
-                l[0] = l[0] * al0 + p0 + p2;
-                l[1] = l[1] * al1 + p1 + p3;
-                const uint32_t b0 = movmatrix_trans(pack_bf16x2(p0, p1));
-                const uint32_t b1 = movmatrix_trans(pack_bf16x2(p2, p3));
-#pragma unroll
-                for (int mt = 0; mt < 8; ++mt) {
-                    o[mt][0] *= al0; o[mt][1] *= al1; o[mt][2] *= al0; o[mt][3] *= al1;
-                    const int i = lane >> 3;
-                    const uint32_t row = j * kBlk + (lane & 7) + (i >= 2 ? 8 : 0);
-                    const uint32_t col = (mt & 3) * 16 + (i & 1) * 8;
-                    uint32_t a[4];
-                    ldmatrix_x4_trans(a, base + (2 + (mt >> 2)) * kPanelBytes + sw128_offset(row, col));
-                    mma_bf16_16816(o[mt], a, b0, b1);
-                }
-            }
+        for (int ks = 0; ks < 8; ++ks) {
+            const uint32_t row = lane & 15;
+            const uint32_t col = (ks & 3) * 16 + (lane >> 4) * 8;
+            uint32_t a[4];
+            ldmatrix_x4(a, base + (ks >> 2) * kBoxBytes + sw128_offset(row, col));
+            mma_bf16_16816(acc, a, qb[ks][0], qb[ks][1]);
         }
-        __syncthreads();
-        if (tid == 0 && st + kStages < nstages) issue(st + kStages);
+        const int t0 = tokbase + (lane >> 2), t1 = t0 + 8;
+        float sc[4];
+        sc[0] = t0 < cutoff ? acc[0] * prm.scale_log2 : -INFINITY;
+        sc[1] = t0 < cutoff ? acc[1] * prm.scale_log2 : -INFINITY;
+        sc[2] = t1 < cutoff ? acc[2] * prm.scale_log2 : -INFINITY;
+        sc[3] = t1 < cutoff ? acc[3] * prm.scale_log2 : -INFINITY;
+        float mx0 = fmaxf(sc[0], sc[2]), mx1 = fmaxf(sc[1], sc[3]);
+#pragma unroll
+        for (int sh = 4; sh < 32; sh <<= 1) {
+            mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, sh));
+            mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, sh));
+        }
+        const float mn0 = fmaxf(m[0], mx0), mn1 = fmaxf(m[1], mx1);
+        // a head whose columns are all masked so far keeps m = -inf and contributes 0
+        const float al0 = mn0 == -INFINITY ? 1.f : fast_exp2(m[0] - mn0);
+        const float al1 = mn1 == -INFINITY ? 1.f : fast_exp2(m[1] - mn1);
+        const float r0 = mn0 == -INFINITY ? 0.f : mn0, r1 = mn1 == -INFINITY ? 0.f : mn1;
+        const float p0 = fast_exp2(sc[0] - r0), p1 = fast_exp2(sc[1] - r1);
+        const float p2 = fast_exp2(sc[2] - r0), p3 = fast_exp2(sc[3] - r1);
+        m[0] = mn0; m[1] = mn1;
+        l[0] = l[0] * al0 + p0 + p2;
+        l[1] = l[1] * al1 + p1 + p3;
+        const uint32_t b0 = movmatrix_trans(pack_bf16x2(p0, p1));
+        const uint32_t b1 = movmatrix_trans(pack_bf16x2(p2, p3));
+#pragma unroll
+        for (int mt = 0; mt < 8; ++mt) {
+            o[mt][0] *= al0; o[mt][1] *= al1; o[mt][2] *= al0; o[mt][3] *= al1;
+            const int i = lane >> 3;
+            const uint32_t row = (lane & 7) + (i >= 2 ? 8 : 0);
+            const uint32_t col = (mt & 3) * 16 + (i & 1) * 8;
+            uint32_t a[4];
+            ldmatrix_x4_trans(a, base + (2 + (mt >> 2)) * kBoxBytes + sw128_offset(row, col));
+            mma_bf16_16816(o[mt], a, b0, b1);
+        }
+        __syncwarp();
+        if (lane == 0 && bi + kWStages < nblk) issue(bi + kWStages);
     }
-    if (aborted) {
-        // let the copies still in flight land before the CTA's shared memory is released
-        if (tid == 0)
-            for (int r = st + 1; r < nstages && r < st + kStages; ++r)
-                mbar_wait_bounded(smem_u32(&full_bar[r % kStages]), (r / kStages) & 1, prm.err, 2);
+    if (bi < nblk) {   // a wait ran out: let the copies in flight land, then leave
+        if (lane == 0)
+            for (int r = bi + 1; r < nblk && r < bi + kWStages; ++r)
+                mbar_wait_bounded(smem_u32(&full_bar[r % kWStages]), (r / kWStages) & 1, prm.err, 2);
         return;
     }
-
     // complete the row sums over the 8 token lanes of each head
 #pragma unroll
     for (int sh = 4; sh < 32; sh <<= 1) {
         l[0] += __shfl_xor_sync(0xffffffffu, l[0], sh);
         l[1] += __shfl_xor_sync(0xffffffffu, l[1], sh);
     }
-    float *mw = merge + warp * kMergeWarpFloats;   // [8 heads][kMergeStride] O^T, then m[8], l[8]
-    if (active) {
+    // stage O^T through this warp's (now idle) ring and write the partial with 16-byte stores
+    float *st = reinterpret_cast<float *>(wbuf);   // [8 heads][132]
+    {
         const int h0 = (lane & 3) * 2;
+        const float i0 = l[0] > 0.f ? 1.f / l[0] : 0.f, i1 = l[1] > 0.f ? 1.f / l[1] : 0.f;
 #pragma unroll
         for (int mt = 0; mt < 8; ++mt) {
             const int d0 = mt * 16 + (lane >> 2);
-            mw[h0 * kMergeStride + d0] = o[mt][0];
-            mw[(h0 + 1) * kMergeStride + d0] = o[mt][1];
-            mw[h0 * kMergeStride + d0 + 8] = o[mt][2];
-            mw[(h0 + 1) * kMergeStride + d0 + 8] = o[mt][3];
-        }
-        if (lane < 4) {
-            mw[kGroup * kMergeStride + h0] = m[0];
-            mw[kGroup * kMergeStride + h0 + 1] = m[1];
-            mw[kGroup * kMergeStride + kGroup + h0] = l[0];
-            mw[kGroup * kMergeStride + kGroup + h0 + 1] = l[1];
+            st[h0 * kMergeStride + d0] = o[mt][0] * i0;
+            st[(h0 + 1) * kMergeStride + d0] = o[mt][1] * i1;
+            st[h0 * kMergeStride + d0 + 8] = o[mt][2] * i0;
+            st[(h0 + 1) * kMergeStride + d0 + 8] = o[mt][3] * i1;
         }
     }
-    __syncthreads();
-    // merge the wpb warps of each stream and write this item's partial results
-    for (int idx = tid; idx < nb * kGroup * kD; idx += blockDim.x) {
-        const int b = idx / (kGroup * kD), hl = (idx / kD) % kGroup, dd = idx % kD;
-        float mstar = -INFINITY;
-        for (int w = 0; w < wpb; ++w)
-            mstar = fmaxf(mstar, merge[(b * wpb + w) * kMergeWarpFloats + kGroup * kMergeStride + hl]);
-        float lsum = 0.f, osum = 0.f;
-        if (mstar != -INFINITY) {
-            for (int w = 0; w < wpb; ++w) {
-                const float *mwp = merge + (b * wpb + w) * kMergeWarpFloats;
-                const float f = exp2f(mwp[kGroup * kMergeStride + hl] - mstar);
-                lsum += f * mwp[kGroup * kMergeStride + kGroup + hl];
-                osum += f * mwp[hl * kMergeStride + dd];
-            }
-        }
-        const int sidx = it.first_stream + b;
-        const int slot = prm.slot_ptr[sidx] + it.slot;
-        const int h = g * kGroup + hl;
-        const size_t row = (size_t)slot * prm.num_q_heads + h;
-        const bool empty = !(lsum > 0.f);
-        prm.part_o[row * kD + dd] = empty ? 0.f : osum / lsum;
-        if (dd == 0) prm.part_lse[row] = empty ? -INFINITY : (mstar + log2f(lsum)) * PADOC_LN2;
+    __syncwarp();
+    const size_t row0 = (size_t)(prm.slot_ptr[s] + it.slot) * prm.num_q_heads + g * kGroup;
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+        const int idx = k * 32 + lane;          // float4 index over [8 heads][32 float4]
+        const int hl = idx >> 5, d4 = idx & 31;
+        const float *src = st + hl * kMergeStride + d4 * 4;
+        *reinterpret_cast<float4 *>(prm.part_o + (row0 + hl) * kD + d4 * 4) = make_float4(src[0], src[1], src[2], src[3]);
+    }
+    if (lane < 4) {
+        const int h0 = lane * 2;
+        prm.part_lse[row0 + h0] = l[0] > 0.f ? (m[0] + log2f(l[0])) * PADOC_LN2 : -INFINITY;
+        prm.part_lse[row0 + h0 + 1] = l[1] > 0.f ? (m[1] + log2f(l[1])) * PADOC_LN2 : -INFINITY;
     }
 }
 
@@ -419,12 +373,25 @@ extern "C" padoc_status padoc_branch_decode_attn(const padoc_kv_pool *pool, cons
         !padoc_make_tmap_bf16(&vmap, pool->v_pool, kD, rows, kD * 2, 64, kBlk))
         return PADOC_ERR_CUDA;
 
+    if ((int64_t)pool->num_blocks * cfg.num_kv_heads * kBlk >= INT32_MAX) return PADOC_ERR_UNSUPPORTED;
+    float *part_o = (float *)workspace;
+    float *part_lse = (float *)((uint8_t *)workspace + padoc_align256((size_t)info->num_slots * cfg.num_q_heads * kD * 4));
+    const float sl2 = scale * PADOC_LOG2E;
+
+    // shared streams of dense pages on the tensor cores
+    padoc_status st = padoc_launch_decode_tc(&kmap, &vmap, plan, info, page_block_table, page_table_stride,
+                                             pool->num_blocks, q, part_o, part_lse, sl2, err, cs);
+    if (st != PADOC_OK) return st;
+
+    // private histories and the shared streams of sparse pages, one warp per item
     DecodeParams prm;
     prm.stream_page = plan + info->off_stream_page;
     prm.shared_len = plan + info->off_shared_len;
     prm.private_len = plan + info->off_private_len;
     prm.slot_ptr = plan + info->off_slot_ptr;
     prm.items = reinterpret_cast<const padoc_item *>(plan + info->off_items);
+    prm.first_item = info->num_tc_items;
+    prm.num_items = info->num_items - info->num_tc_items;
     prm.page_table = page_block_table;
     prm.stream_table = stream_block_table;
     prm.page_stride = page_table_stride;
@@ -432,20 +399,16 @@ extern "C" padoc_status padoc_branch_decode_attn(const padoc_kv_pool *pool, cons
     prm.num_blocks = pool->num_blocks;
     prm.num_kv_heads = cfg.num_kv_heads;
     prm.num_q_heads = cfg.num_q_heads;
+    prm.pool_rows = pool->num_blocks * cfg.num_kv_heads * kBlk;
     prm.q = (const __nv_bfloat16 *)q;
-    prm.part_o = (float *)workspace;
-    prm.part_lse = (float *)((uint8_t *)workspace + padoc_align256((size_t)info->num_slots * cfg.num_q_heads * kD * 4));
-    prm.scale_log2 = scale * PADOC_LOG2E;
+    prm.part_o = part_o;
+    prm.part_lse = part_lse;
+    prm.scale_log2 = sl2;
     prm.err = err;
-
-    static bool attr_set = false;   // per process; the attribute is per function
-    if (!attr_set) {
-        PADOC_CUDA_TRY(cudaFuncSetAttribute(decode_mma_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kDecodeSmem));
-        attr_set = true;
-    }
-    if (info->num_items > 0) {
-        decode_mma_kernel<<<info->num_items, 128, kDecodeSmem, cs>>>(kmap, vmap, prm);
-        padoc_status st = padoc_launch_status();
+    if (prm.num_items > 0) {
+        PADOC_CUDA_TRY(cudaFuncSetAttribute(decode_warp_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kDecodeSmem));
+        decode_warp_kernel<<<(prm.num_items + kWarps - 1) / kWarps, kWarps * 32, kDecodeSmem, cs>>>(kmap, vmap, prm);
+        st = padoc_launch_status();
         if (st != PADOC_OK) return st;
     }
     const int64_t out_rows = (int64_t)info->num_streams * cfg.num_q_heads;

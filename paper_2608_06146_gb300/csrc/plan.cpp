@@ -202,7 +202,6 @@ padoc_status build_parts(const padoc_page *pages, int32_t num_pages, const padoc
     const int32_t split = cfg->split_tokens > 0 ? cfg->split_tokens : PADOC_DEFAULT_SPLIT_TOKENS;
     const int32_t psplit = PADOC_PRIVATE_SPLIT_TOKENS;
     const int32_t group = cfg->num_q_heads / cfg->num_kv_heads;
-    (void)group;
 
     for (int32_t p = 0; p < num_pages; ++p) {
         const padoc_page &pg = pages[p];
@@ -248,49 +247,49 @@ padoc_status build_parts(const padoc_page *pages, int32_t num_pages, const padoc
         pp.slot_ptr[s + 1] = pp.slot_ptr[s] + np + nv;
     }
 
-    // work items, one set per KV head
+    // work items, one set per KV head: tensor-core items first, then warp items
+    std::vector<padoc_item> tc_items, warp_items;
     for (int32_t g = 0; g < cfg->num_kv_heads; ++g) {
         for (int32_t p = 0; p < num_pages; ++p) {
             const int32_t f0 = pp.page_first_stream[p], ns = pp.page_num_streams[p];
             int32_t vis = 0;
             for (int32_t s = f0; s < f0 + ns; ++s) vis = std::max(vis, pp.streams[s].shared_len);
+            const bool use_tc = (int64_t)ns * group >= PADOC_TC_MIN_ROWS;
             for (int32_t j = 0; j < page_splits[p]; ++j) {
                 const int32_t tb = j * split, te = std::min(vis, tb + split);
-                for (int32_t r = 0; r < ns; r += PADOC_MMA_ROW_STREAMS) {
-                    padoc_item it;
-                    it.kind = PADOC_ITEM_SHARED;
-                    it.index = p;
-                    it.kv_head = g;
-                    it.tok_begin = tb;
-                    it.tok_end = te;
-                    it.first_stream = f0 + r;
-                    it.num_streams = std::min(PADOC_MMA_ROW_STREAMS, ns - r);
-                    it.slot = j;
-                    pp.items.push_back(it);
+                if (use_tc) {
+                    for (int32_t r = 0; r < ns; r += PADOC_TC_ITEM_STREAMS)
+                        tc_items.push_back({PADOC_ITEM_SHARED_TC, p, g, tb, te, f0 + r,
+                                            std::min(PADOC_TC_ITEM_STREAMS, ns - r), j});
+                } else {
+                    for (int32_t s = f0; s < f0 + ns; ++s) {
+                        const int32_t tes = std::min(te, pp.streams[s].shared_len);
+                        if (tes <= tb) {
+                            // nothing of this split is visible to the stream: an empty partial
+                            warp_items.push_back({PADOC_ITEM_SHARED, p, g, tb, tb, s, 1, j});
+                        } else {
+                            warp_items.push_back({PADOC_ITEM_SHARED, p, g, tb, tes, s, 1, j});
+                        }
+                    }
                 }
             }
         }
         for (int32_t s = 0; s < S; ++s) {
             const int32_t np = page_splits[pp.streams[s].page];
             const int32_t L = pp.streams[s].private_len;
-            for (int32_t tb = 0, i = 0; tb < L; tb += psplit, ++i) {
-                padoc_item it;
-                it.kind = PADOC_ITEM_PRIVATE;
-                it.index = s;
-                it.kv_head = g;
-                it.tok_begin = tb;
-                it.tok_end = std::min(L, tb + psplit);
-                it.first_stream = s;
-                it.num_streams = 1;
-                it.slot = np + i;
-                pp.items.push_back(it);
-            }
+            for (int32_t tb = 0, i = 0; tb < L; tb += psplit, ++i)
+                warp_items.push_back({PADOC_ITEM_PRIVATE, s, g, tb, std::min(L, tb + psplit), s, 1, np + i});
         }
     }
-    // longest items first (LPT order), ties by position for determinism
-    std::stable_sort(pp.items.begin(), pp.items.end(), [](const padoc_item &a, const padoc_item &b) {
-        return (a.tok_end - a.tok_begin) * (int64_t)(a.num_streams + 3) > (b.tok_end - b.tok_begin) * (int64_t)(b.num_streams + 3);
-    });
+    // longest items first (LPT order) within each kernel's list, ties by position for determinism
+    auto longer = [](const padoc_item &a, const padoc_item &b) {
+        return (int64_t)(a.tok_end - a.tok_begin) * (a.num_streams + 15) > (int64_t)(b.tok_end - b.tok_begin) * (b.num_streams + 15);
+    };
+    std::stable_sort(tc_items.begin(), tc_items.end(), longer);
+    std::stable_sort(warp_items.begin(), warp_items.end(), longer);
+    pp.num_tc_items = (int32_t)tc_items.size();
+    pp.items = tc_items;
+    pp.items.insert(pp.items.end(), warp_items.begin(), warp_items.end());
     return PADOC_OK;
 }
 

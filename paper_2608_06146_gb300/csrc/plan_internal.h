@@ -9,20 +9,26 @@
 #define PADOC_PREFILL_Q_TILE 128
 #define PADOC_PREFILL_K_TILE 128
 
-// Decode split-K: shared-stream tokens per partial result, private tokens per partial result, and
-// streams (8 query heads each) per warp-MMA work item.
+// Decode split-K: shared-stream tokens per partial result and private tokens per partial result.
 #define PADOC_DEFAULT_SPLIT_TOKENS 512
 #define PADOC_PRIVATE_SPLIT_TOKENS 512
-#define PADOC_MMA_ROW_STREAMS 4
+// Shared-stream rows (streams x query heads of one KV head) from which the tensor-core kernel
+// takes a page: below this the rows are too few for a dense M = 128 contraction and each stream
+// reads the shared stream with warp-level MMAs instead.
+#define PADOC_TC_MIN_ROWS 64
+// Streams per tensor-core work item: two M = 128 tiles of 16 streams x 8 query heads.
+#define PADOC_TC_ITEM_STREAMS 32
 
 #define PADOC_ITEM_INTS 8
-enum { PADOC_ITEM_SHARED = 0, PADOC_ITEM_PRIVATE = 1 };
+enum { PADOC_ITEM_SHARED = 0, PADOC_ITEM_PRIVATE = 1, PADOC_ITEM_SHARED_TC = 2 };
 
-// One split-K work item of the decode kernels (8 int32 words in the plan blob).
-//   kind        PADOC_ITEM_SHARED: tokens [tok_begin, tok_end) of page `index`'s shared stream for
-//               streams [first_stream, first_stream + num_streams) of that page, each with its own
-//               column cutoff shared_len;
-//               PADOC_ITEM_PRIVATE: private tokens [tok_begin, tok_end) of stream `index`.
+// One split-K work item of the decode kernels (8 int32 words in the plan blob). The blob holds
+// the tensor-core items first ([0, num_tc_items)), then the warp items.
+//   kind        PADOC_ITEM_SHARED_TC: tokens [tok_begin, tok_end) of page `index`'s shared stream for
+//               streams [first_stream, first_stream + num_streams) (<= 32) of that page, each with
+//               its own column cutoff shared_len (tensor-core kernel);
+//               PADOC_ITEM_SHARED: the same for the one stream first_stream (warp kernel);
+//               PADOC_ITEM_PRIVATE: private tokens [tok_begin, tok_end) of stream `index` (warp kernel).
 //   kv_head     the KV head; the item covers that head's Hq/Hkv query heads of every stream.
 //   slot        partial-result slot of each covered stream s: slot_ptr[s] + slot.
 typedef struct {

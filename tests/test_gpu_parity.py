@@ -100,6 +100,23 @@ def test_decode_bf16_edge_pages():
     assert_close(*run_decode(wl, 3, layout_streams=True), torch.bfloat16)
 
 
+def test_decode_bf16_tensor_core_edge_pages():
+    # pages whose branches x heads fill M = 128 tiles: 10 branches (one M-tile), 17 (two M-tiles, the
+    # second nearly empty), 33 (two items of 32 + 1 streams); unaligned shared lengths, f_k = 0 and
+    # f_k = L ties, one-token private histories and a split boundary inside the layout stream
+    rng = np.random.default_rng(8)
+    def page(P, L, n):
+        forks = [int(x) for x in rng.integers(0, L + 1, size=n)]
+        forks[0], forks[-1] = 0, L
+        lens = [int(x) for x in rng.integers(1, 300, size=n)]
+        lens[1] = 1
+        return PageSpec(P, L, forks, lens)
+    pages = [page(37, 21, 10), page(700, 40, 17), page(1200, 264, 33), page(5, 3, 8)]
+    wl = Workload("tc edge", pages, 16, 2, 128, torch.bfloat16, "decode")
+    assert_close(*run_decode(wl, 9, layout_streams=True), torch.bfloat16)
+    assert_close(*run_decode(wl, 10, split_tokens=128), torch.bfloat16)
+
+
 def test_decode_bad_block_id_reports_device_error():
     wl = inputs.decode_page()
     di = inputs.decode_inputs(wl, 4)

@@ -123,7 +123,7 @@ def _plan_items(plan, info):
 
 
 @pytest.mark.parametrize("wl_name,layout", [("decode_page", False), ("dense_page", False), ("serving_batch", True),
-                                            ("tiny", False)])
+                                            ("serving_batch", False), ("tiny", False)])
 def test_decode_plan_covers_every_visible_token_once(wl_name, layout):
     wl = inputs.WORKLOADS[wl_name]()
     cfg = pa.make_decode_config(wl.num_q_heads, wl.num_kv_heads, wl.head_dim, 16, layout, 0)
@@ -144,16 +144,25 @@ def test_decode_plan_covers_every_visible_token_once(wl_name, layout):
     page_first = {}
     for s in range(S):
         page_first.setdefault(int(sp[s]), s)
+    ntc = info.num_tc_items
+    assert all(items[:ntc, 0] == 2) and not any(items[ntc:, 0] == 2)
+    page_streams = np.bincount(sp, minlength=len(wl.pages))
     for kind, idx, g, tb, te, fs, ns, slot in items:
-        assert tb % 16 == 0 and te > tb and 1 <= ns <= 4
+        assert tb % 16 == 0
+        if kind == 2:      # tensor-core item: up to 32 streams of a page with >= 64 rows
+            assert 1 <= ns <= 32 and te > tb and page_streams[idx] * 8 >= 64
+        elif kind == 0:    # warp item over one stream's view of the shared stream
+            assert ns == 1 and te >= tb and page_streams[idx] * 8 < 64
+        else:
+            assert kind == 1 and ns == 1 and te > tb
         for s in range(fs, fs + ns):
-            if kind == 0:
+            if kind in (0, 2):
                 assert sp[s] == idx
                 hi = min(te, sh[s])
                 if hi > tb:
                     cov_sh[(s, g)][tb:hi] += 1
             else:
-                assert s == idx and ns == 1
+                assert s == idx
                 cov_pv[(s, g)][tb:te] += 1
             slots_used[(s, g)].append(slot)
     for key in cov_sh:
