@@ -162,6 +162,11 @@ __device__ __forceinline__ float fast_exp2(float x)
     return y;
 }
 
+// Programmatic dependent launch: a grid lets the next grid in its stream start launching, and a
+// dependent grid waits until its prerequisite grid has completed and its writes are visible.
+__device__ __forceinline__ void pdl_launch_dependents() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+__device__ __forceinline__ void pdl_wait_prerequisite() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
 #define PADOC_LOG2E 1.4426950408889634f
 #define PADOC_LN2 0.6931471805599453f
 

@@ -44,11 +44,19 @@ struct DecodeParams {
     const int32_t *stream_table;
     int32_t page_stride, stream_stride;
     int32_t num_blocks, num_kv_heads, num_q_heads, pool_rows;
+    int32_t after_tc;    // launched as a programmatic dependent of the tensor-core grid
     const __nv_bfloat16 *q;
     float *part_o, *part_lse;
     float scale_log2;
     int *err;
 };
+
+// When this grid runs as a programmatic dependent of the tensor-core grid, each warp waits for
+// that grid before it exits, so the merge kernel that follows in the stream sees both grids' writes.
+__device__ __forceinline__ void finish_warp(const DecodeParams &prm)
+{
+    if (prm.after_tc) pdl_wait_prerequisite();
+}
 
 __global__ void __launch_bounds__(kWarps * 32, 1)
 decode_warp_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap,
@@ -58,7 +66,7 @@ decode_warp_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_consta
     uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int wi = blockIdx.x * kWarps + warp;
-    if (wi >= prm.num_items) return;   // warps are independent: no CTA-wide barrier follows
+    if (wi >= prm.num_items) { finish_warp(prm); return; }   // warps are independent: no CTA barrier follows
     uint8_t *wbuf = smem + (size_t)warp * kWarpSmem;
     uint64_t *full_bar = (uint64_t *)(smem + (size_t)kWarps * kWarpSmem) + warp * kWStages;
     const padoc_item it = prm.items[prm.first_item + wi];
@@ -164,6 +172,7 @@ decode_warp_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_consta
         if (lane == 0)
             for (int r = bi + 1; r < nblk && r < bi + kWStages; ++r)
                 mbar_wait_bounded(smem_u32(&full_bar[r % kWStages]), (r / kWStages) & 1, prm.err, 2);
+        finish_warp(prm);
         return;
     }
     // complete the row sums over the 8 token lanes of each head
@@ -200,6 +209,7 @@ decode_warp_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_consta
         prm.part_lse[row0 + h0] = l[0] > 0.f ? (m[0] + log2f(l[0])) * PADOC_LN2 : -INFINITY;
         prm.part_lse[row0 + h0 + 1] = l[1] > 0.f ? (m[1] + log2f(l[1])) * PADOC_LN2 : -INFINITY;
     }
+    finish_warp(prm);
 }
 
 // ------------------------------------------------------------------------------------------------
@@ -240,7 +250,21 @@ __global__ void __launch_bounds__(128) combine_kernel(Slots sl, const float *__r
     for (int c0 = lane * 4; c0 < d; c0 += 128) {
         float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
         if (tot != -INFINITY) {
-            for (int i = 0; i < n; ++i) {
+            int i = 0;
+            for (; i + 4 <= n; i += 4) {   // four partials in flight at a time
+                float w[4];
+                float4 v[4];
+#pragma unroll
+                for (int u = 0; u < 4; ++u) {
+                    const int64_t pr = sl.part_row(row, i + u);
+                    w[u] = expf(part_lse[pr] - tot);
+                    v[u] = *reinterpret_cast<const float4 *>(part_o + pr * d + c0);
+                }
+#pragma unroll
+                for (int u = 0; u < 4; ++u)
+                    if (w[u] != 0.f) { acc.x += w[u] * v[u].x; acc.y += w[u] * v[u].y; acc.z += w[u] * v[u].z; acc.w += w[u] * v[u].w; }
+            }
+            for (; i < n; ++i) {
                 const int64_t pr = sl.part_row(row, i);
                 const float w = expf(part_lse[pr] - tot);
                 if (w == 0.f) continue;
@@ -405,9 +429,20 @@ extern "C" padoc_status padoc_branch_decode_attn(const padoc_kv_pool *pool, cons
     prm.part_lse = part_lse;
     prm.scale_log2 = sl2;
     prm.err = err;
+    prm.after_tc = info->num_tc_items > 0 ? 1 : 0;
     if (prm.num_items > 0) {
         PADOC_CUDA_TRY(cudaFuncSetAttribute(decode_warp_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kDecodeSmem));
-        decode_warp_kernel<<<(prm.num_items + kWarps - 1) / kWarps, kWarps * 32, kDecodeSmem, cs>>>(kmap, vmap, prm);
+        cudaLaunchConfig_t lc = {};
+        lc.gridDim = dim3((unsigned)((prm.num_items + kWarps - 1) / kWarps));
+        lc.blockDim = dim3(kWarps * 32);
+        lc.dynamicSmemBytes = kDecodeSmem;
+        lc.stream = cs;
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        attr[0].val.programmaticStreamSerializationAllowed = 1;
+        lc.attrs = attr;
+        lc.numAttrs = prm.after_tc ? 1 : 0;
+        PADOC_CUDA_TRY(cudaLaunchKernelEx(&lc, decode_warp_kernel, kmap, vmap, prm));
         st = padoc_launch_status();
         if (st != PADOC_OK) return st;
     }

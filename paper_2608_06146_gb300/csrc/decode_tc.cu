@@ -278,7 +278,7 @@ __device__ __forceinline__ void decode_tc_body(const CUtensorMap *kmap, const CU
             mbar_arrive(bar(B_PFULL + mi));
         }
         // partial result of this piece: O / l (fp32) and its natural-log LSE
-        const bool have = ok && (ne == 0 || wait_all(B_PVDONE + mi, (ne - 1) & 1, 71));
+        const bool have = ne == 0 || (ok && wait_all(B_PVDONE + mi, (ne - 1) & 1, 71));
         if (have) {
             tc_fence_after();
             const bool empty = !(l > 0.f);
@@ -316,6 +316,9 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
     uint32_t *tmem_slot = (uint32_t *)(bars + B_COUNT);
     volatile int *abort_flag = (volatile int *)(tmem_slot + 1);
     const int tid = threadIdx.x, warp = tid >> 5;
+    // the warp kernel that follows reads nothing this grid writes before its final wait, so it may
+    // start filling SMs as soon as every CTA of this grid is resident
+    pdl_launch_dependents();
     const padoc_item it = prm.items[blockIdx.x];
     const int mt = it.num_streams > 16 ? 2 : 1;
 

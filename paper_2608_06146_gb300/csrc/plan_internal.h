@@ -10,8 +10,8 @@
 #define PADOC_PREFILL_K_TILE 128
 
 // Decode split-K: shared-stream tokens per partial result and private tokens per partial result.
-#define PADOC_DEFAULT_SPLIT_TOKENS 512
-#define PADOC_PRIVATE_SPLIT_TOKENS 512
+#define PADOC_DEFAULT_SPLIT_TOKENS 1024
+#define PADOC_PRIVATE_SPLIT_TOKENS 256
 // Shared-stream rows (streams x query heads of one KV head) from which the tensor-core kernel
 // takes a page: below this the rows are too few for a dense M = 128 contraction and each stream
 // reads the shared stream with warp-level MMAs instead.
