@@ -37,7 +37,7 @@ METRIC = "ancestor-attn decode queries/s, % of HBM roofline; packed prefill TFLO
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 # dram__bytes_read.sum + dram__bytes_write.sum per launch from the ncu captures summarised under
 # profiles/ (None until a capture of the current kernel exists).
-TRAFFIC_BYTES = {"decode": None, "prefill": None}
+TRAFFIC_BYTES = {"decode": None, "prefill": 260_600_000}   # prefill: profiles/prefill_tc_packed_32k.md
 
 
 def load_peaks():

@@ -4,8 +4,7 @@
 #include <stddef.h>
 #include <stdint.h>
 
-// Prefill tiles: 128 query rows x 128 key columns (one tcgen05 M=128 tile by N=128 keys; the
-// warp-MMA kernel walks the same tile map).
+// Prefill tiles: 128 query rows x 128 key columns (one tcgen05 M = 128 tile by N = 128 keys).
 #define PADOC_PREFILL_Q_TILE 128
 #define PADOC_PREFILL_K_TILE 128
 

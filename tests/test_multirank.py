@@ -1,0 +1,61 @@
+"""The multi-GPU path is page sharding with no data-path collective: each rank decodes its own
+pages (pages never see each other), and the benchmark reduces only its timing. These checks run
+the host side of that path as two gloo ranks on the CPU."""
+import os
+import socket
+
+import pytest
+import torch
+import torch.distributed as dist
+import torch.multiprocessing as mp
+
+from paper_2608_06146_gb300.engine import shard_pages
+
+
+def _free_port():
+    s = socket.socket()
+    s.bind(("127.0.0.1", 0))
+    port = s.getsockname()[1]
+    s.close()
+    return port
+
+
+def _rank_main(rank, world, port, num_pages, q):
+    os.environ["MASTER_ADDR"] = "127.0.0.1"
+    os.environ["MASTER_PORT"] = str(port)
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    try:
+        mine = shard_pages(num_pages, rank, world)
+        gathered = [None] * world
+        dist.all_gather_object(gathered, mine)
+        import bench
+        t = bench.max_over_ranks(torch, world, float(rank + 1) * 1.5)
+        dist.barrier()
+        q.put((rank, gathered, t))
+    finally:
+        dist.destroy_process_group()
+
+
+@pytest.mark.parametrize("num_pages", [32, 7, 1])
+def test_two_gloo_ranks_partition_pages_and_reduce_timing(num_pages):
+    world = 2
+    ctx = mp.get_context("spawn")
+    q = ctx.Queue()
+    port = _free_port()
+    procs = [ctx.Process(target=_rank_main, args=(r, world, port, num_pages, q)) for r in range(world)]
+    for p in procs:
+        p.start()
+    results = [q.get(timeout=120) for _ in range(world)]
+    for p in procs:
+        p.join(timeout=60)
+        assert p.exitcode == 0
+    for rank, gathered, t in results:
+        flat = sorted(x for shard in gathered for x in shard)
+        assert flat == list(range(num_pages)), "shards must partition the pages"
+        assert max(len(s) for s in gathered) - min(len(s) for s in gathered) <= 1
+        assert t == 3.0, "max over ranks of (rank+1)*1.5"
+
+
+def test_shard_pages_rejects_bad_rank():
+    with pytest.raises(ValueError):
+        shard_pages(4, 2, 2)
