@@ -164,6 +164,7 @@ typedef struct {
     int32_t num_slots;         /* split-K partial results per query head */
     int32_t max_page_blocks;   /* page block-table width the plan needs */
     int32_t max_stream_blocks; /* stream block-table width the plan needs */
+    int32_t max_stream_slots;  /* most split-K partials of one stream */
     int64_t plan_ints;         /* int32 words in the plan blob */
     int64_t off_stream_page;   /* offsets (int32 words) of the blob's arrays */
     int64_t off_shared_len;

@@ -58,6 +58,24 @@ bool padoc_make_tmap_bf16(CUtensorMap *map, const void *base, uint64_t cols, uin
     return r == CUDA_SUCCESS;
 }
 
+bool padoc_make_tmap_bf16_4d(CUtensorMap *map, const void *base, const uint64_t dims[4], const uint64_t strides_bytes[3],
+                             const uint32_t box[4])
+{
+    PFN_cuTensorMapEncodeTiled_v12000 fn = encode_fn();
+    if (!fn) return false;
+    if (((uintptr_t)base) & 15) return false;
+    for (int i = 0; i < 3; ++i)
+        if (strides_bytes[i] & 15) return false;
+    cuuint64_t d[4] = {dims[0], dims[1], dims[2], dims[3]};
+    cuuint64_t st[3] = {strides_bytes[0], strides_bytes[1], strides_bytes[2]};
+    cuuint32_t bx[4] = {box[0], box[1], box[2], box[3]};
+    cuuint32_t estr[4] = {1, 1, 1, 1};
+    CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void *>(base), d, st, bx, estr,
+                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                    CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS;
+}
+
 padoc_status padoc_launch_status()
 {
     return cudaPeekAtLastError() == cudaSuccess ? PADOC_OK : (cudaGetLastError(), PADOC_ERR_CUDA);

@@ -105,6 +105,15 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap *map
         : "memory");
 }
 
+__device__ __forceinline__ void tma_load_4d(uint32_t dst, const CUtensorMap *map, int32_t c0, int32_t c1, int32_t c2,
+                                            int32_t c3, uint32_t bar)
+{
+    asm volatile(
+        "cp.async.bulk.tensor.4d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4, %5}], [%6];" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(c2), "r"(c3), "r"(bar)
+        : "memory");
+}
+
 __device__ __forceinline__ void tma_prefetch_desc(const CUtensorMap *map)
 {
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
@@ -179,6 +188,9 @@ int *padoc_device_error_word();
 // box_rows x 64 columns, 128-byte swizzle. Returns false if the driver rejects it.
 bool padoc_make_tmap_bf16(CUtensorMap *map, const void *base, uint64_t cols, uint64_t rows,
                           uint64_t row_stride_bytes, uint32_t box_cols, uint32_t box_rows);
+// 4-D bf16 tensor map (dims[0] innermost, strides of dims 1..3 in bytes), 128-byte swizzle.
+bool padoc_make_tmap_bf16_4d(CUtensorMap *map, const void *base, const uint64_t dims[4], const uint64_t strides_bytes[3],
+                             const uint32_t box[4]);
 padoc_status padoc_launch_status();
 // tcgen05 packed prefill (prefill_tc.cu); arguments validated by the caller.
 padoc_status padoc_launch_prefill_tc(const void *q, const void *k, const void *v, int64_t total_tokens,
@@ -187,7 +199,7 @@ padoc_status padoc_launch_prefill_tc(const void *q, const void *k, const void *v
                                      const int8_t *tile_kind_dev, float scale_log2, void *out, float *lse,
                                      cudaStream_t stream);
 // tcgen05 shared-stream decode (decode_tc.cu): the plan's tensor-core items.
-padoc_status padoc_launch_decode_tc(const CUtensorMap *kmap, const CUtensorMap *vmap, const int32_t *plan,
+padoc_status padoc_launch_decode_tc(const CUtensorMap *kmap, const CUtensorMap *vmap, const CUtensorMap *qmap, const int32_t *plan,
                                     const padoc_decode_plan *info, const int32_t *page_table, int32_t page_stride,
                                     int32_t num_blocks, const void *q, float *part_o, float *part_lse, float scale_log2,
                                     int *err, cudaStream_t stream);

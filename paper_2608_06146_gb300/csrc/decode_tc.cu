@@ -10,11 +10,12 @@
 // the shared-stream and private-history partials.
 //
 // The CTA layout follows the packed-prefill kernel: warps 0-3 / 4-7 run the softmax of M-tile 0 / 1
-// (thread t owns row t; the warps also gather the queries into swizzled shared memory), warp 8 is
-// the TMA producer (lanes 0-7 each fetch one 16-token paged block of K and of V per tile, two
-// 64-column boxes each; blocks past the piece or with an out-of-range id are fetched from an
-// out-of-range coordinate, which fills zeros), warp 9 allocates TMEM and issues the MMAs as a
-// converged warp. TMEM: S_i / P_i at columns 128i, O_i at 256 + 128i.
+// (thread t owns row t), warp 8 is the TMA producer (the item's queries as one 4-D box per panel;
+// the item's block rows looked up once; then lanes 0-7 each fetch one 16-token paged block of K and
+// of V per tile, two 64-column boxes each; blocks past the piece or with an out-of-range id are
+// fetched from an out-of-range coordinate, which fills zeros), warp 9 allocates TMEM and issues the
+// MMAs as a converged warp. A stage's K is released when the tile's last QK^T completes and its V
+// when the last PV completes. TMEM: S_i / P_i at columns 128i, O_i at 256 + 128i.
 #include <math.h>
 
 #include "common.cuh"
@@ -36,15 +37,17 @@ enum {
     B_Q = 0,
     B_KFULL = 1,     // [stage]
     B_VFULL = 3,     // [stage]
-    B_KVEMPTY = 5,   // [stage]
-    B_SFULL = 7,     // [m-tile]
-    B_PFULL = 9,     // [m-tile], 128 arrivals
-    B_PVDONE = 11,   // [m-tile]
-    B_FINAL = 13,
-    B_COUNT = 14
+    B_KEMPTY = 5,    // [stage]: the last QK^T of the tile has completed
+    B_VEMPTY = 7,    // [stage]: the last PV of the tile has completed
+    B_SFULL = 9,     // [m-tile]
+    B_PFULL = 11,    // [m-tile], 128 arrivals
+    B_PVDONE = 13,   // [m-tile]
+    B_FINAL = 15,
+    B_COUNT = 16
 };
 
-constexpr size_t kSmemBytes = 1024 + (size_t)kTile * (2 + 2 * kStages) + B_COUNT * 8 + 64;
+constexpr int kMaxItemBlocks = PADOC_TC_MAX_ITEM_TOKENS / kBlk;   // block rows an item looks up once
+constexpr size_t kSmemBytes = 1024 + (size_t)kTile * (2 + 2 * kStages) + B_COUNT * 8 + 64 + kMaxItemBlocks * 4;
 
 struct TcDecodeParams {
     const int32_t *shared_len, *slot_ptr;
@@ -68,8 +71,9 @@ __device__ __forceinline__ bool wait_or_abort(uint32_t bar, uint32_t parity, int
 }
 
 template <int MT>
-__device__ __forceinline__ void decode_tc_body(const CUtensorMap *kmap, const CUtensorMap *vmap, const TcDecodeParams &prm,
-                                               const padoc_item &it, uint8_t *smem, uint64_t *bars, uint32_t tmem,
+__device__ __forceinline__ void decode_tc_body(const CUtensorMap *kmap, const CUtensorMap *vmap, const CUtensorMap *qmap,
+                                               const TcDecodeParams &prm, const padoc_item &it, uint8_t *smem,
+                                               uint64_t *bars, int32_t *block_rows, uint32_t tmem,
                                                volatile int *abort_flag)
 {
     uint8_t *sq = smem;
@@ -83,41 +87,70 @@ __device__ __forceinline__ void decode_tc_body(const CUtensorMap *kmap, const CU
 
     if (warp == 8) {
         // ---------------------------------------------------------------- TMA producer (whole warp)
+        // queries first: one 4-D box per 64-column panel gathers 16 streams x 8 heads of KV head g
+        if (lane == 0 && ne > 0) {
+            mbar_arrive_expect_tx(bar(B_Q), MT * kTile);
+#pragma unroll
+            for (int i = 0; i < MT; ++i) {
+                tma_load_4d(smem_u32(sq + i * kTile), qmap, 0, 0, g, it.first_stream + 16 * i, bar(B_Q));
+                tma_load_4d(smem_u32(sq + i * kTile) + kPanel, qmap, 64, 0, g, it.first_stream + 16 * i, bar(B_Q));
+            }
+        }
+        // the item's block rows, looked up once (out-of-range ids and blocks past the piece read
+        // from an out-of-range row, which fills zeros)
         const int32_t *table = prm.page_table + (size_t)it.index * prm.page_stride;
+        const int nblk = ne * (kKT / kBlk);
+        auto lookup = [&](int bi) {
+            const int tok0 = tb + bi * kBlk;
+            int32_t row = prm.pool_rows;
+            if (tok0 < te) {
+                const int32_t id = table[tok0 / kBlk];
+                if (id >= 0 && id < prm.num_blocks) row = (id * prm.num_kv_heads + g) * kBlk;
+                else padoc_record_error(prm.err, PADOC_DEVERR_BLOCK_ID, id);
+            }
+            block_rows[bi] = row;
+        };
+        // the first tile's rows first, so its loads start before the remaining lookups
+        if (lane < kKT / kBlk && lane < nblk) lookup(lane);
+        __syncwarp();
         int issued = 0;
         for (int j = 0; j < ne; ++j) {
-            const int s = j & 1;
-            bool ok = true;
-            if (j >= 2) ok = wait_or_abort(bar(B_KVEMPTY + s), ((j - 2) >> 1) & 1, prm.err, 50, abort_flag);
-            if (!__all_sync(0xffffffffu, ok)) break;
-            if (lane == 0) {
-                mbar_arrive_expect_tx(bar(B_KFULL + s), kTile);
-                mbar_arrive_expect_tx(bar(B_VFULL + s), kTile);
+            if (j == 1) {
+                for (int bi = kKT / kBlk + lane; bi < nblk; bi += 32) lookup(bi);
+                __syncwarp();
             }
+            const int s = j & 1;
+            const uint32_t off = (uint32_t)lane * (kBlk * 128);
+            const int32_t row = lane < kKT / kBlk ? block_rows[j * (kKT / kBlk) + lane] : 0;
+            bool ok = true;
+            if (j >= 2) ok = wait_or_abort(bar(B_KEMPTY + s), ((j - 2) >> 1) & 1, prm.err, 50, abort_flag);
+            if (!__all_sync(0xffffffffu, ok)) break;
+            if (lane == 0) mbar_arrive_expect_tx(bar(B_KFULL + s), kTile);
             __syncwarp();
             if (lane < kKT / kBlk) {
-                const int tok0 = tb + j * kKT + lane * kBlk;
-                int32_t row = prm.pool_rows;   // out of range: zero fill
-                if (tok0 < te) {
-                    const int32_t id = table[tok0 / kBlk];
-                    if (id >= 0 && id < prm.num_blocks) row = (id * prm.num_kv_heads + g) * kBlk;
-                    else padoc_record_error(prm.err, PADOC_DEVERR_BLOCK_ID, id);
-                }
-                const uint32_t off = (uint32_t)lane * (kBlk * 128);
-                const uint32_t kb = smem_u32(sk + s * kTile) + off, vb = smem_u32(sv + s * kTile) + off;
+                const uint32_t kb = smem_u32(sk + s * kTile) + off;
                 tma_load_2d(kb, kmap, 0, row, bar(B_KFULL + s));
                 tma_load_2d(kb + kPanel, kmap, 64, row, bar(B_KFULL + s));
+            }
+            if (j >= 2) ok = wait_or_abort(bar(B_VEMPTY + s), ((j - 2) >> 1) & 1, prm.err, 53, abort_flag);
+            if (!__all_sync(0xffffffffu, ok)) break;
+            if (lane == 0) mbar_arrive_expect_tx(bar(B_VFULL + s), kTile);
+            __syncwarp();
+            if (lane < kKT / kBlk) {
+                const uint32_t vb = smem_u32(sv + s * kTile) + off;
                 tma_load_2d(vb, vmap, 0, row, bar(B_VFULL + s));
                 tma_load_2d(vb + kPanel, vmap, 64, row, bar(B_VFULL + s));
             }
             issued = j + 1;
         }
         // copies still in flight must land before the CTA's shared memory is released
-        if (lane == 0)
+        if (lane == 0) {
+            if (ne > 0) mbar_wait_bounded(bar(B_Q), 0, prm.err, 54);
             for (int j = (issued > 2 ? issued - 2 : 0); j < issued; ++j) {
                 mbar_wait_bounded(bar(B_KFULL + (j & 1)), (j >> 1) & 1, prm.err, 51);
                 mbar_wait_bounded(bar(B_VFULL + (j & 1)), (j >> 1) & 1, prm.err, 52);
             }
+        }
     } else if (warp == 9) {
         // ---------------------------------------------------------------- MMA issuer (whole warp)
         constexpr uint32_t idS = umma_idesc_bf16(128, kKT, false);
@@ -146,6 +179,7 @@ __device__ __forceinline__ void decode_tc_body(const CUtensorMap *kmap, const CU
             tc_fence_after();
 #pragma unroll
             for (int i = 0; i < MT; ++i) issue_s(i, 0);
+            umma_commit_warp(bar(B_KEMPTY));
         }
         for (int j = 0; ok && j < ne; ++j) {
             const int s = j & 1, sn = (j + 1) & 1;
@@ -160,11 +194,12 @@ __device__ __forceinline__ void decode_tc_body(const CUtensorMap *kmap, const CU
                     umma_bf16_ts_warp(tmem + 256 + 128 * i, tmem + 128 * i + kk * 8, db + kk * (2048 >> 4), idPV,
                                       (j > 0 || kk > 0));
                 umma_commit_warp(bar(B_PVDONE + i));
-                if (i == MT - 1) umma_commit_warp(bar(B_KVEMPTY + s));
+                if (i == MT - 1) umma_commit_warp(bar(B_VEMPTY + s));
                 if (j + 1 < ne) {
                     if (i == 0 && !wait_w(B_KFULL + sn, ((j + 1) >> 1) & 1, 64)) { ok = false; break; }
                     tc_fence_after();
                     issue_s(i, sn);
+                    if (i == MT - 1) umma_commit_warp(bar(B_KEMPTY + sn));
                 }
             }
         }
@@ -179,18 +214,6 @@ __device__ __forceinline__ void decode_tc_body(const CUtensorMap *kmap, const CU
         const bool valid = b < it.num_streams;
         const int s = it.first_stream + (valid ? b : 0);
         const int h = g * kGroup + hl;
-        // gather this row's query into the swizzled K-major tile (zeros for padding rows)
-        {
-            const uint4 *src = reinterpret_cast<const uint4 *>(prm.q + ((size_t)s * prm.num_q_heads + h) * kD);
-            uint8_t *dst = sq + mi * kTile;
-#pragma unroll
-            for (int c = 0; c < 16; ++c) {
-                const uint4 v = valid ? src[c] : make_uint4(0, 0, 0, 0);
-                *reinterpret_cast<uint4 *>(dst + (c >> 3) * kPanel + sw128_offset(row, (c & 7) * 8)) = v;
-            }
-            fence_proxy_async_smem();
-            mbar_arrive(bar(B_Q));
-        }
         const int cutoff = valid ? min(prm.shared_len[s], te) : tb;   // visible tokens end here
         const uint32_t lanes = (uint32_t)((warp & 3) * 32) << 16;
         const uint32_t tS = tmem + lanes + 128 * mi, tO = tmem + lanes + 256 + 128 * mi;
@@ -308,13 +331,14 @@ __device__ __forceinline__ void decode_tc_body(const CUtensorMap *kmap, const CU
 
 __global__ void __launch_bounds__(kThreads, 1)
 decode_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap,
-                 const TcDecodeParams prm)
+                 const __grid_constant__ CUtensorMap qmap, const TcDecodeParams prm)
 {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     uint64_t *bars = (uint64_t *)(smem + (size_t)kTile * (2 + 2 * kStages));
     uint32_t *tmem_slot = (uint32_t *)(bars + B_COUNT);
     volatile int *abort_flag = (volatile int *)(tmem_slot + 1);
+    int32_t *block_rows = (int32_t *)(tmem_slot + 16);
     const int tid = threadIdx.x, warp = tid >> 5;
     // the warp kernel that follows reads nothing this grid writes before its final wait, so it may
     // start filling SMs as soon as every CTA of this grid is resident
@@ -326,13 +350,13 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
         for (int i = 0; i < B_COUNT; ++i) {
             uint32_t cnt = 1;
             if (i == B_PFULL || i == B_PFULL + 1) cnt = 128;
-            if (i == B_Q) cnt = 128 * mt;
             mbar_init(smem_u32(&bars[i]), cnt);
         }
         *abort_flag = 0;
         fence_barrier_init();
         tma_prefetch_desc(&kmap);
         tma_prefetch_desc(&vmap);
+        tma_prefetch_desc(&qmap);
     }
     if (warp == 9) {
         tmem_alloc(smem_u32(tmem_slot), kTmemCols);
@@ -342,8 +366,8 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
-    if (mt == 2) decode_tc_body<2>(&kmap, &vmap, prm, it, smem, bars, tmem, abort_flag);
-    else decode_tc_body<1>(&kmap, &vmap, prm, it, smem, bars, tmem, abort_flag);
+    if (mt == 2) decode_tc_body<2>(&kmap, &vmap, &qmap, prm, it, smem, bars, block_rows, tmem, abort_flag);
+    else decode_tc_body<1>(&kmap, &vmap, &qmap, prm, it, smem, bars, block_rows, tmem, abort_flag);
     tc_fence_before();
     __syncthreads();
     if (warp == 9) {
@@ -354,7 +378,7 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
 
 }  // namespace
 
-padoc_status padoc_launch_decode_tc(const CUtensorMap *kmap, const CUtensorMap *vmap, const int32_t *plan,
+padoc_status padoc_launch_decode_tc(const CUtensorMap *kmap, const CUtensorMap *vmap, const CUtensorMap *qmap, const int32_t *plan,
                                     const padoc_decode_plan *info, const int32_t *page_table, int32_t page_stride,
                                     int32_t num_blocks, const void *q, float *part_o, float *part_lse, float scale_log2,
                                     int *err, cudaStream_t stream)
@@ -376,6 +400,6 @@ padoc_status padoc_launch_decode_tc(const CUtensorMap *kmap, const CUtensorMap *
     prm.scale_log2 = scale_log2;
     prm.err = err;
     PADOC_CUDA_TRY(cudaFuncSetAttribute(decode_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes));
-    decode_tc_kernel<<<info->num_tc_items, kThreads, kSmemBytes, stream>>>(*kmap, *vmap, prm);
+    decode_tc_kernel<<<info->num_tc_items, kThreads, kSmemBytes, stream>>>(*kmap, *vmap, *qmap, prm);
     return padoc_launch_status();
 }

@@ -199,7 +199,8 @@ padoc_status build_parts(const padoc_page *pages, int32_t num_pages, const padoc
     if (cfg->split_tokens < 0 || (cfg->split_tokens > 0 && cfg->split_tokens % cfg->block_size != 0))
         return PADOC_ERR_INVALID_ARGUMENT;
     const int32_t bs = cfg->block_size;
-    const int32_t split = cfg->split_tokens > 0 ? cfg->split_tokens : PADOC_DEFAULT_SPLIT_TOKENS;
+    const int32_t split = std::min(cfg->split_tokens > 0 ? cfg->split_tokens : PADOC_DEFAULT_SPLIT_TOKENS,
+                                   PADOC_TC_MAX_ITEM_TOKENS);
     const int32_t psplit = PADOC_PRIVATE_SPLIT_TOKENS;
     const int32_t group = cfg->num_q_heads / cfg->num_kv_heads;
 
@@ -328,6 +329,8 @@ extern "C" padoc_status padoc_build_decode_plan(const padoc_page *pages, int32_t
     info->num_slots = pp.slot_ptr.back();
     info->max_page_blocks = pp.max_page_blocks;
     info->max_stream_blocks = pp.max_stream_blocks;
+    for (int64_t st = 0; st < S; ++st)
+        info->max_stream_slots = std::max<int32_t>(info->max_stream_slots, pp.slot_ptr[st + 1] - pp.slot_ptr[st]);
     info->plan_ints = need;
     info->kv_tokens = pp.kv_tokens;
     int64_t o = 0;

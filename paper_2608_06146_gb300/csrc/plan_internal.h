@@ -17,6 +17,8 @@
 #define PADOC_TC_MIN_ROWS 64
 // Streams per tensor-core work item: two M = 128 tiles of 16 streams x 8 query heads.
 #define PADOC_TC_ITEM_STREAMS 32
+// Longest shared-stream piece of one tensor-core work item.
+#define PADOC_TC_MAX_ITEM_TOKENS 4096
 
 #define PADOC_ITEM_INTS 8
 enum { PADOC_ITEM_SHARED = 0, PADOC_ITEM_PRIVATE = 1, PADOC_ITEM_SHARED_TC = 2 };

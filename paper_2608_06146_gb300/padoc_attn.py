@@ -52,6 +52,7 @@ class padoc_decode_plan(ctypes.Structure):
     _fields_ = [("cfg", padoc_decode_config), ("num_pages", ctypes.c_int32), ("num_streams", ctypes.c_int32),
                 ("num_items", ctypes.c_int32), ("num_tc_items", ctypes.c_int32), ("num_slots", ctypes.c_int32),
                 ("max_page_blocks", ctypes.c_int32), ("max_stream_blocks", ctypes.c_int32),
+                ("max_stream_slots", ctypes.c_int32),
                 ("plan_ints", ctypes.c_int64), ("off_stream_page", ctypes.c_int64), ("off_shared_len", ctypes.c_int64),
                 ("off_private_len", ctypes.c_int64), ("off_slot_ptr", ctypes.c_int64), ("off_items", ctypes.c_int64),
                 ("off_page_len", ctypes.c_int64), ("kv_tokens", ctypes.c_int64)]
