@@ -119,6 +119,23 @@ __device__ __forceinline__ void tma_prefetch_desc(const CUtensorMap *map)
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
 }
 
+// ------------------------------------------------------------------------------------------------
+// cp.async (16 bytes per thread, L2 only). A source size of 0 fills the 16 bytes with zeros.
+// ------------------------------------------------------------------------------------------------
+__device__ __forceinline__ void cp_async_16(uint32_t dst, const void *src, uint32_t src_bytes)
+{
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(src_bytes) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
+// Arrives on the mbarrier once every cp.async this thread issued so far has completed; the arrival is
+// one of the barrier's expected arrivals (no pending-count increment).
+__device__ __forceinline__ void cp_async_mbar_arrive(uint32_t bar)
+{
+    asm volatile("cp.async.mbarrier.arrive.noinc.shared::cta.b64 [%0];" ::"r"(bar) : "memory");
+}
+
 // Byte offset of element (row, col) of a [rows][64] bf16 panel written by TMA with 128-byte
 // swizzle (16-byte chunk index XOR row % 8); panels start on 1024-byte boundaries.
 __device__ __forceinline__ uint32_t sw128_offset(uint32_t row, uint32_t col)

@@ -10,8 +10,10 @@
 // A split-K merge then joins each (stream, head)'s partials.
 //
 // Warp kernel: every warp owns one work item and runs on its own: a 3-deep ring of 16-token
-// paged blocks fetched by TMA (one box per 64-column half of K and V, 128-byte swizzle) with its
-// own mbarriers, so no warp ever waits for another. The math puts the 8 query heads of a KV head
+// paged blocks fetched with cp.async (each lane copies 16 of the block's 512 16-byte chunks into
+// a 128-byte-swizzled [16][64] panel per half of K and V), one cp.async group per block, so no
+// warp ever waits for another. cp.async rather than TMA: a 16-token block is only four 2 KB
+// boxes, and an SM issues a TMA box only every ~70 cycles. The math puts the 8 query heads of a KV head
 // in the N = 8 columns of mma.m16n8k16 and the 16 tokens of a block in its M = 16 rows:
 //     S^T[16 tok x 8 heads] = K[16 x 128] . Q^T[128 x 8]             (8 MMAs)
 //     O^T[128 x 8 heads]   += V^T[128 x 16 tok] . P^T[16 tok x 8]    (8 MMAs)
@@ -33,7 +35,7 @@ constexpr int kWStages = 3;            // paged blocks in flight per warp
 constexpr int kBoxBytes = kBlk * 128;  // one 16-row x 64-column box
 constexpr int kWStageBytes = 4 * kBoxBytes;   // K lo, K hi, V lo, V hi
 constexpr int kWarpSmem = kWStages * kWStageBytes;
-constexpr size_t kDecodeSmem = 1024 + (size_t)kWarps * kWarpSmem + (size_t)kWarps * kWStages * 8 + 64;
+constexpr size_t kDecodeSmem = 1024 + (size_t)kWarps * kWarpSmem;
 constexpr int kMergeStride = 132;      // floats per head row when a warp stages its O^T
 
 struct DecodeParams {
@@ -45,6 +47,7 @@ struct DecodeParams {
     int32_t page_stride, stream_stride;
     int32_t num_blocks, num_kv_heads, num_q_heads, pool_rows;
     int32_t after_tc;    // launched as a programmatic dependent of the tensor-core grid
+    const __nv_bfloat16 *k_pool, *v_pool;
     const __nv_bfloat16 *q;
     float *part_o, *part_lse;
     float scale_log2;
@@ -59,8 +62,7 @@ __device__ __forceinline__ void finish_warp(const DecodeParams &prm)
 }
 
 __global__ void __launch_bounds__(kWarps * 32, 1)
-decode_warp_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap,
-                   const DecodeParams prm)
+decode_warp_kernel(const DecodeParams prm)
 {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
@@ -68,7 +70,6 @@ decode_warp_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_consta
     const int wi = blockIdx.x * kWarps + warp;
     if (wi >= prm.num_items) { finish_warp(prm); return; }   // warps are independent: no CTA barrier follows
     uint8_t *wbuf = smem + (size_t)warp * kWarpSmem;
-    uint64_t *full_bar = (uint64_t *)(smem + (size_t)kWarps * kWarpSmem) + warp * kWStages;
     const padoc_item it = prm.items[prm.first_item + wi];
     const bool is_shared = it.kind == PADOC_ITEM_SHARED;
     const int g = it.kv_head;
@@ -79,26 +80,27 @@ decode_warp_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_consta
     const int blk0 = it.tok_begin / kBlk;
     const int nblk = cutoff > it.tok_begin ? (cutoff - it.tok_begin + kBlk - 1) / kBlk : 0;
 
-    if (lane == 0) {
-        for (int i = 0; i < kWStages; ++i) mbar_init(smem_u32(&full_bar[i]), 1);
-        fence_barrier_init();
-    }
-    __syncwarp();
-    auto issue = [&](int bi) {   // lane 0 only
-        const uint32_t base = smem_u32(wbuf + (bi % kWStages) * kWStageBytes);
-        const uint32_t bar = smem_u32(&full_bar[bi % kWStages]);
-        const int32_t id = table[blk0 + bi];
-        int32_t row = prm.pool_rows;   // out of range: zero fill
-        if (id >= 0 && id < prm.num_blocks) row = (id * prm.num_kv_heads + g) * kBlk;
-        else padoc_record_error(prm.err, PADOC_DEVERR_BLOCK_ID, id);
-        mbar_arrive_expect_tx(bar, kWStageBytes);
-        tma_load_2d(base + 0 * kBoxBytes, &kmap, 0, row, bar);
-        tma_load_2d(base + 1 * kBoxBytes, &kmap, 64, row, bar);
-        tma_load_2d(base + 2 * kBoxBytes, &vmap, 0, row, bar);
-        tma_load_2d(base + 3 * kBoxBytes, &vmap, 64, row, bar);
+    // block bi into stage bi % kWStages: chunk q = lane + 32k of the block's 512 16-byte chunks is
+    // panel q / 128 (K lo, K hi, V lo, V hi), row (q / 8) % 16, 16-byte column q % 8 (swizzled)
+    auto issue = [&](int bi) {   // whole warp; always commits a group, possibly empty
+        if (bi < nblk) {
+            const int32_t id = table[blk0 + bi];
+            const bool okid = id >= 0 && id < prm.num_blocks;
+            if (!okid && lane == 0) padoc_record_error(prm.err, PADOC_DEVERR_BLOCK_ID, id);
+            const size_t rowbase = okid ? ((size_t)id * prm.num_kv_heads + g) * kBlk : 0;
+            const uint32_t base = smem_u32(wbuf + (bi % kWStages) * kWStageBytes);
+#pragma unroll
+            for (int k = 0; k < 16; ++k) {
+                const int q = lane + 32 * k;
+                const int panel = q >> 7, r = (q >> 3) & 15, cc = q & 7;
+                const __nv_bfloat16 *src = (panel < 2 ? prm.k_pool : prm.v_pool) +
+                                           (rowbase + r) * kD + (panel & 1) * 64 + cc * 8;
+                cp_async_16(base + panel * kBoxBytes + r * 128 + ((cc ^ (r & 7)) << 4), src, okid ? 16u : 0u);
+            }
+        }
+        cp_async_commit();
     };
-    if (lane == 0)
-        for (int bi = 0; bi < kWStages && bi < nblk; ++bi) issue(bi);
+    for (int bi = 0; bi < kWStages; ++bi) issue(bi);
 
     // query fragments: B operand Q^T[128 dims x 8 heads]
     uint32_t qb[8][2];
@@ -115,10 +117,9 @@ decode_warp_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_consta
 #pragma unroll
     for (int mt = 0; mt < 8; ++mt) o[mt][0] = o[mt][1] = o[mt][2] = o[mt][3] = 0.f;
 
-    int bi = 0;
-    for (; bi < nblk; ++bi) {
-        const bool ok = mbar_wait_bounded(smem_u32(&full_bar[bi % kWStages]), (bi / kWStages) & 1, prm.err, 1);
-        if (!__all_sync(0xffffffffu, ok)) break;
+    for (int bi = 0; bi < nblk; ++bi) {
+        cp_async_wait<kWStages - 1>();   // block bi has landed (one group per block)
+        __syncwarp();
         const uint32_t base = smem_u32(wbuf + (bi % kWStages) * kWStageBytes);
         const int tokbase = (blk0 + bi) * kBlk;
         // S^T = K . Q^T
@@ -165,16 +166,10 @@ decode_warp_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_consta
             ldmatrix_x4_trans(a, base + (2 + (mt >> 2)) * kBoxBytes + sw128_offset(row, col));
             mma_bf16_16816(o[mt], a, b0, b1);
         }
-        __syncwarp();
-        if (lane == 0 && bi + kWStages < nblk) issue(bi + kWStages);
+        __syncwarp();   // every lane is done with the stage before it is refilled
+        issue(bi + kWStages);
     }
-    if (bi < nblk) {   // a wait ran out: let the copies in flight land, then leave
-        if (lane == 0)
-            for (int r = bi + 1; r < nblk && r < bi + kWStages; ++r)
-                mbar_wait_bounded(smem_u32(&full_bar[r % kWStages]), (r / kWStages) & 1, prm.err, 2);
-        finish_warp(prm);
-        return;
-    }
+    cp_async_wait<0>();
     // complete the row sums over the 8 token lanes of each head
 #pragma unroll
     for (int sh = 4; sh < 32; sh <<= 1) {
@@ -503,6 +498,8 @@ extern "C" padoc_status padoc_branch_decode_attn(const padoc_kv_pool *pool, cons
     prm.num_kv_heads = cfg.num_kv_heads;
     prm.num_q_heads = cfg.num_q_heads;
     prm.pool_rows = pool->num_blocks * cfg.num_kv_heads * kBlk;
+    prm.k_pool = (const __nv_bfloat16 *)pool->k_pool;
+    prm.v_pool = (const __nv_bfloat16 *)pool->v_pool;
     prm.q = (const __nv_bfloat16 *)q;
     prm.part_o = part_o;
     prm.part_lse = part_lse;
@@ -521,7 +518,7 @@ extern "C" padoc_status padoc_branch_decode_attn(const padoc_kv_pool *pool, cons
         attr[0].val.programmaticStreamSerializationAllowed = 1;
         lc.attrs = attr;
         lc.numAttrs = prm.after_tc ? 1 : 0;
-        PADOC_CUDA_TRY(cudaLaunchKernelEx(&lc, decode_warp_kernel, kmap, vmap, prm));
+        PADOC_CUDA_TRY(cudaLaunchKernelEx(&lc, decode_warp_kernel, prm));
         st = padoc_launch_status();
         if (st != PADOC_OK) return st;
     }
