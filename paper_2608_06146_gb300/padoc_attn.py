@@ -126,22 +126,37 @@ def _check(fn: str, st: int):
         raise PadocError(fn, st)
 
 
+_PAGE_DTYPE = np.dtype({"names": ["prefix_len", "layout_len", "num_branches", "fork_offset", "branch_len"],
+                        "formats": [np.int32, np.int32, np.int32, np.uint64, np.uint64],
+                        "offsets": [0, 4, 8, 16, 24], "itemsize": ctypes.sizeof(padoc_page)})
+
+
 class _Pages:
-    """C array of padoc_page; keeps the per-page int32 arrays alive."""
+    """C array of padoc_page built with vectorized numpy (one pass over the pages); keeps the
+    concatenated fork-offset and branch-length arrays alive."""
 
     def __init__(self, pages):
-        self.keep = []
-        self.arr = (padoc_page * max(len(pages), 1))()
-        for i, pg in enumerate(pages):
-            f = np.ascontiguousarray(np.asarray(pg.fork_offset, np.int32))
-            n = np.ascontiguousarray(np.asarray(pg.branch_len, np.int32))
-            self.keep += [f, n]
-            self.arr[i].prefix_len = int(pg.prefix_len)
-            self.arr[i].layout_len = int(pg.layout_len)
-            self.arr[i].num_branches = len(n)
-            self.arr[i].fork_offset = f.ctypes.data_as(_i32p)
-            self.arr[i].branch_len = n.ctypes.data_as(_i32p)
-        self.n = len(pages)
+        import itertools
+        n = len(pages)
+        counts = np.fromiter((len(pg.branch_len) for pg in pages), np.int64, count=n)
+        total = int(counts.sum())
+        self.forks = np.fromiter(itertools.chain.from_iterable(pg.fork_offset for pg in pages), np.int32, count=total)
+        self.lens = np.fromiter(itertools.chain.from_iterable(pg.branch_len for pg in pages), np.int32, count=total)
+        if total == 0:
+            self.forks = np.zeros(1, np.int32)
+            self.lens = np.zeros(1, np.int32)
+        offs = np.zeros(max(n, 1), np.int64)
+        if n > 1:
+            offs[1:] = np.cumsum(counts)[:-1]
+        rec = np.zeros(max(n, 1), _PAGE_DTYPE)
+        rec["prefix_len"][:n] = np.fromiter((pg.prefix_len for pg in pages), np.int32, count=n)
+        rec["layout_len"][:n] = np.fromiter((pg.layout_len for pg in pages), np.int32, count=n)
+        rec["num_branches"][:n] = counts
+        rec["fork_offset"][:n] = self.forks.ctypes.data + 4 * offs[:n]
+        rec["branch_len"][:n] = self.lens.ctypes.data + 4 * offs[:n]
+        self.rec = rec
+        self.arr = ctypes.cast(rec.ctypes.data, ctypes.POINTER(padoc_page))
+        self.n = n
 
 
 def _stream_ptr(stream):
@@ -228,15 +243,25 @@ def padoc_decode_plan_size(pages, cfg: padoc_decode_config) -> int:
     return n.value
 
 
-def padoc_build_decode_plan(pages, cfg: padoc_decode_config):
-    """Returns (plan blob int32 numpy array, padoc_decode_plan host summary)."""
+def padoc_build_decode_plan(pages, cfg: padoc_decode_config, out=None):
+    """Returns (plan blob int32 numpy array, padoc_decode_plan host summary). ``out`` may be an int32
+    numpy array (e.g. a view of pinned host memory) that receives the blob; a view of it is returned."""
     lib, P = load_library(), _Pages(pages)
-    n = padoc_decode_plan_size(pages, cfg)
-    plan = np.zeros(max(n, 1), np.int32)
     info = padoc_decode_plan()
+    if out is not None:   # one planner pass when the caller's buffer is large enough
+        st = lib.padoc_build_decode_plan(P.arr, P.n, ctypes.byref(cfg), out.ctypes.data_as(_i32p), out.size,
+                                         ctypes.byref(info))
+        if st == PADOC_OK:
+            return out[:info.plan_ints], info
+        if st != 6:   # PADOC_ERR_CAPACITY
+            _check("padoc_build_decode_plan", st)
+    n = ctypes.c_int64()
+    _check("padoc_decode_plan_size", lib.padoc_decode_plan_size(P.arr, P.n, ctypes.byref(cfg), ctypes.byref(n)))
+    n = n.value
+    out = np.zeros(max(n, 1), np.int32)
     _check("padoc_build_decode_plan", lib.padoc_build_decode_plan(P.arr, P.n, ctypes.byref(cfg),
-                                                                  plan.ctypes.data_as(_i32p), n, ctypes.byref(info)))
-    return plan[:n], info
+                                                                  out.ctypes.data_as(_i32p), n, ctypes.byref(info)))
+    return out[:n], info
 
 
 def padoc_decode_workspace_size(info: padoc_decode_plan) -> int:
