@@ -148,7 +148,7 @@ def bench_decode(args, torch, dev, rank, world):
     wl = inputs.serving_batch(seed=3 + 1000 * rank)
     scale = 1.0 / math.sqrt(wl.head_dim)
     di = inputs.decode_inputs(wl, 3 + 1000 * rank, pool_slack=1.0)
-    plan = DecodePlan(wl.pages, wl.num_q_heads, wl.num_kv_heads, wl.head_dim, dev)
+    plan = DecodePlan(wl.pages, wl.num_q_heads, wl.num_kv_heads, wl.head_dim, dev, tc_ctas=args.tc_ctas)
     S = plan.num_streams
     per_replica = (di.k_pool.numel() + di.v_pool.numel()) * 2
     R = args.replicas if args.replicas > 0 else max(2, math.ceil(4 * l2_bytes(torch) / per_replica) + 1)
@@ -373,6 +373,7 @@ def main():
     ap.add_argument("--only", default="all", choices=["all", "decode", "prefill"])
     ap.add_argument("--replicas", type=int, default=0, help="decode input replicas (0: enough to exceed 4x L2)")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--tc-ctas", type=int, default=0, help="tensor-core decode CTAs (0: one per SM)")
     args = ap.parse_args()
     if args.impl == "reference":
         return run_reference(args)

@@ -147,8 +147,11 @@ typedef struct {
     int32_t block_size;      /* must equal the pool's block_size */
     int32_t layout_streams;  /* 1: also decode each page's layout stream (Alg. 1 decodes every live
                                 stream): cutoff P + L over the shared stream, no private rows */
-    int32_t split_tokens;    /* shared-stream tokens per split-K partial; 0 = library default;
+    int32_t split_tokens;    /* shared-stream tokens per split-K partial of the warp kernel (pages with
+                                too few streams for the tensor cores); 0 = library default;
                                 a positive value must be a multiple of block_size */
+    int32_t tc_ctas;         /* CTAs the tensor-core shared-stream work is balanced over (one range of
+                                equal work each); 0 = the current device's multiprocessor count */
 } padoc_decode_config;
 
 /* Host summary of a decode plan, filled by padoc_build_decode_plan. The int32 plan blob it
@@ -161,10 +164,11 @@ typedef struct {
     int32_t num_streams;
     int32_t num_items;         /* work items of the split-K decode kernels */
     int32_t num_tc_items;      /* of which use the tensor-core shared-stream kernel */
-    int32_t num_slots;         /* split-K partial results per query head */
+    int32_t tc_ctas;           /* CTAs of the tensor-core kernel (0 when num_tc_items is 0) */
+    int32_t num_slots;         /* split-K partial results, each for one (stream, KV head) */
     int32_t max_page_blocks;   /* page block-table width the plan needs */
     int32_t max_stream_blocks; /* stream block-table width the plan needs */
-    int32_t max_stream_slots;  /* most split-K partials of one stream */
+    int32_t max_stream_slots;  /* most split-K partials of one (stream, KV head) */
     int64_t plan_ints;         /* int32 words in the plan blob */
     int64_t off_stream_page;   /* offsets (int32 words) of the blob's arrays */
     int64_t off_shared_len;
@@ -172,6 +176,7 @@ typedef struct {
     int64_t off_slot_ptr;
     int64_t off_items;
     int64_t off_page_len;
+    int64_t off_cta_ptr;
     int64_t kv_tokens;         /* algorithmic KV tokens read: each page's stream once + all private */
 } padoc_decode_plan;
 
@@ -214,7 +219,7 @@ padoc_status padoc_branch_decode_attn(const padoc_kv_pool *pool, const padoc_dec
                                       padoc_stream_t stream);
 
 /* Size of the device array that padoc_branch_decode_attn_noalloc uses as its workspace. */
-#define PADOC_STATIC_WORKSPACE_BYTES (16u << 20)
+#define PADOC_STATIC_WORKSPACE_BYTES (32u << 20)
 
 /* padoc_branch_decode_attn for callers that cannot allocate device memory (a plugin inside a
  * framework that owns all device memory and offers it no allocator, or a latency-critical decode
@@ -222,7 +227,7 @@ padoc_status padoc_branch_decode_attn(const padoc_kv_pool *pool, const padoc_dec
  * counterpart: it is a deployment convenience of this library.
  * Arguments, layouts and results are those of padoc_branch_decode_attn without the workspace
  * arguments. The split-K partials go to a fixed 256-byte-aligned device array of
- * PADOC_STATIC_WORKSPACE_BYTES (16 MiB) that every GPU which loads this library holds until the
+ * PADOC_STATIC_WORKSPACE_BYTES (32 MiB) that every GPU which loads this library holds until the
  * process exits; the call allocates nothing (no cudaMalloc, cudaFree or allocating library call).
  *   - The first call on a device looks up that device's address of the array (once per device,
  *     with that device current); make that first call before any stream capture.
@@ -290,7 +295,9 @@ padoc_status padoc_check_device_errors(padoc_stream_t stream);
 
 /* The code and detail of the device error found by the last padoc_check_device_errors on this
  * thread: code 1 = block id out of range (detail = the id), 2 = bounded wait ran out
- * (detail = the kernel's wait site). */
+ * (detail = the kernel's wait site), 3 = a kernel's dynamic shared memory did not start on the
+ * 1024-byte boundary its swizzled tiles need (detail = the start address mod 1024; the kernel did
+ * no work). */
 void padoc_last_device_error(int32_t *code, int32_t *detail);
 
 const char *padoc_status_string(padoc_status status);

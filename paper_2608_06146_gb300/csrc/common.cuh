@@ -15,6 +15,7 @@
 // ------------------------------------------------------------------------------------------------
 #define PADOC_DEVERR_BLOCK_ID 1
 #define PADOC_DEVERR_TIMEOUT 2
+#define PADOC_DEVERR_SMEM_ALIGN 3
 
 __device__ __forceinline__ void padoc_record_error(int *err, int code, int detail)
 {
@@ -114,6 +115,15 @@ __device__ __forceinline__ void tma_load_4d(uint32_t dst, const CUtensorMap *map
         : "memory");
 }
 
+// Pulls a 4-D box into L2 without a destination or completion signal.
+__device__ __forceinline__ void tma_prefetch_l2_4d(const CUtensorMap *map, int32_t c0, int32_t c1, int32_t c2, int32_t c3)
+{
+    asm volatile("cp.async.bulk.prefetch.tensor.4d.L2.global.tile [%0, {%1, %2, %3, %4}];" ::"l"(
+                     reinterpret_cast<uint64_t>(map)),
+                 "r"(c0), "r"(c1), "r"(c2), "r"(c3)
+                 : "memory");
+}
+
 __device__ __forceinline__ void tma_prefetch_desc(const CUtensorMap *map)
 {
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
@@ -190,6 +200,21 @@ __device__ __forceinline__ float fast_exp2(float x)
 
 // Programmatic dependent launch: a grid lets the next grid in its stream start launching, and a
 // dependent grid waits until its prerequisite grid has completed and its writes are visible.
+// One 32-byte store of eight floats (p 32-byte aligned): a whole sector per lane.
+__device__ __forceinline__ void st_global_v8(float *p, float a0, float a1, float a2, float a3, float a4, float a5,
+                                             float a6, float a7)
+{
+    asm volatile("st.global.v8.f32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};" ::"l"(p), "f"(a0), "f"(a1), "f"(a2),
+                 "f"(a3), "f"(a4), "f"(a5), "f"(a6), "f"(a7)
+                 : "memory");
+}
+
+// Named barrier `id` (1..15) over `count` threads (a multiple of 32) of the CTA.
+__device__ __forceinline__ void named_bar_sync(int id, int count)
+{
+    asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(count) : "memory");
+}
+
 __device__ __forceinline__ void pdl_launch_dependents() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
 __device__ __forceinline__ void pdl_wait_prerequisite() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 
@@ -218,8 +243,8 @@ padoc_status padoc_launch_prefill_tc(const void *q, const void *k, const void *v
 // tcgen05 shared-stream decode (decode_tc.cu): the plan's tensor-core items.
 padoc_status padoc_launch_decode_tc(const CUtensorMap *kmap, const CUtensorMap *vmap, const CUtensorMap *qmap, const int32_t *plan,
                                     const padoc_decode_plan *info, const int32_t *page_table, int32_t page_stride,
-                                    int32_t num_blocks, const void *q, float *part_o, float *part_lse, float scale_log2,
-                                    int *err, cudaStream_t stream);
+                                    int32_t num_blocks, float *part_o, float *part_lse, float scale_log2, int *err,
+                                    cudaStream_t stream);
 int padoc_num_sms();
 
 #define PADOC_CUDA_TRY(expr)                                   \

@@ -191,7 +191,7 @@ decode_warp_kernel(const DecodeParams prm)
         }
     }
     __syncwarp();
-    const size_t row0 = (size_t)(prm.slot_ptr[s] + it.slot) * prm.num_q_heads + g * kGroup;
+    const size_t row0 = (size_t)(prm.slot_ptr[(size_t)s * prm.num_kv_heads + g] + it.slot) * kGroup;
 #pragma unroll
     for (int k = 0; k < 8; ++k) {
         const int idx = k * 32 + lane;          // float4 index over [8 heads][32 float4]
@@ -210,11 +210,14 @@ decode_warp_kernel(const DecodeParams prm)
 // ------------------------------------------------------------------------------------------------
 // Split-K merge (C4): one warp per output row, 4 consecutive dims per lane.
 // ------------------------------------------------------------------------------------------------
-struct RaggedSlots {   // decode: row = s * Hq + h, slots [slot_ptr[s], slot_ptr[s+1])
+struct RaggedSlots {   // decode: row = s * Hq + h = (s * Hkv + g) * group + hl; slots of (s, g)
     const int32_t *slot_ptr;
-    int32_t hq;
-    __device__ int count(int64_t row) const { return slot_ptr[row / hq + 1] - slot_ptr[row / hq]; }
-    __device__ int64_t part_row(int64_t row, int i) const { return (int64_t)(slot_ptr[row / hq] + i) * hq + row % hq; }
+    int32_t group;
+    __device__ int count(int64_t row) const { return slot_ptr[row / group + 1] - slot_ptr[row / group]; }
+    __device__ int64_t part_row(int64_t row, int i) const
+    {
+        return (int64_t)(slot_ptr[row / group] + i) * group + row % group;
+    }
 };
 struct UniformSlots {  // public combine: part_row = split * rows + row
     int32_t splits;
@@ -223,55 +226,55 @@ struct UniformSlots {  // public combine: part_row = split * rows + row
     __device__ int64_t part_row(int64_t row, int i) const { return (int64_t)i * rows + row; }
 };
 
-// Decode merge: one CTA per stream, 16 heads x 8 threads, each thread 16 of the 128 dims. The
-// weights exp(lse_s - lse) of every (slot, head) are computed once into shared memory, then every
-// thread streams its dims of all partials with the loads of four partials in flight.
+// Decode merge: one CTA per (stream, KV head), its 8 query heads x 16 threads, each thread 8 of
+// the 128 dims. The weights exp(lse_s - lse) of every (slot, head) are computed once into shared
+// memory, then every thread streams its dims of all partials with two partials' loads in flight.
 constexpr int kCombineMaxSlots = 64;
 
 __global__ void __launch_bounds__(128) decode_combine_kernel(const int32_t *__restrict__ slot_ptr,
                                                              const float *__restrict__ part_o,
-                                                             const float *__restrict__ part_lse, int32_t hq,
+                                                             const float *__restrict__ part_lse,
                                                              __nv_bfloat16 *__restrict__ out, float *__restrict__ lse_out)
 {
-    __shared__ float w_sh[kCombineMaxSlots][16];
-    __shared__ float tot_sh[16];
-    const int s = blockIdx.x;
+    __shared__ float w_sh[kCombineMaxSlots][kGroup];
+    __shared__ float tot_sh[kGroup];
+    const int key = blockIdx.x;                      // s * Hkv + g; output rows key * 8 + h
     const int tid = threadIdx.x;
-    const int p0 = slot_ptr[s], n = slot_ptr[s + 1] - p0;
-    const int h = tid >> 3, part = tid & 7;          // head, 16-dim slice
-    if (n > kCombineMaxSlots || hq != 16) return;    // the host routes such plans elsewhere
-    // per head: max and log-sum-exp over slots (8 threads of the head cooperate)
+    const int p0 = slot_ptr[key], n = slot_ptr[key + 1] - p0;
+    const int h = tid >> 4, part = tid & 15;         // head, 8-dim slice
+    if (n > kCombineMaxSlots) return;                // the host routes such plans elsewhere
+    // per head: max and log-sum-exp over slots (16 threads of the head cooperate)
     float mx = -INFINITY;
-    for (int i = part; i < n; i += 8) mx = fmaxf(mx, part_lse[(size_t)(p0 + i) * hq + h]);
+    for (int i = part; i < n; i += 16) mx = fmaxf(mx, part_lse[(size_t)(p0 + i) * kGroup + h]);
 #pragma unroll
-    for (int sh = 1; sh < 8; sh <<= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, sh));
+    for (int sh = 1; sh < 16; sh <<= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, sh));
     float sum = 0.f;
     if (mx != -INFINITY)
-        for (int i = part; i < n; i += 8) sum += expf(part_lse[(size_t)(p0 + i) * hq + h] - mx);
+        for (int i = part; i < n; i += 16) sum += expf(part_lse[(size_t)(p0 + i) * kGroup + h] - mx);
 #pragma unroll
-    for (int sh = 1; sh < 8; sh <<= 1) sum += __shfl_xor_sync(0xffffffffu, sum, sh);
+    for (int sh = 1; sh < 16; sh <<= 1) sum += __shfl_xor_sync(0xffffffffu, sum, sh);
     const float tot = mx == -INFINITY ? -INFINITY : mx + logf(sum);
-    for (int i = part; i < n; i += 8)
-        w_sh[i][h] = tot == -INFINITY ? 0.f : expf(part_lse[(size_t)(p0 + i) * hq + h] - tot);
+    for (int i = part; i < n; i += 16)
+        w_sh[i][h] = tot == -INFINITY ? 0.f : expf(part_lse[(size_t)(p0 + i) * kGroup + h] - tot);
     if (part == 0) tot_sh[h] = tot;
     __syncthreads();
-    float4 acc[4];
+    float4 acc[2];
 #pragma unroll
-    for (int c = 0; c < 4; ++c) acc[c] = make_float4(0.f, 0.f, 0.f, 0.f);
-    const float *base = part_o + ((size_t)p0 * hq + h) * 128 + part * 16;
-    const size_t slot_stride = (size_t)hq * 128;
+    for (int c = 0; c < 2; ++c) acc[c] = make_float4(0.f, 0.f, 0.f, 0.f);
+    const float *base = part_o + ((size_t)p0 * kGroup + h) * kD + part * 8;
+    constexpr size_t slot_stride = (size_t)kGroup * kD;
     int i = 0;
     for (; i + 2 <= n; i += 2) {
-        float4 v[2][4];
+        float4 v[2][2];
 #pragma unroll
         for (int u = 0; u < 2; ++u)
 #pragma unroll
-            for (int c = 0; c < 4; ++c) v[u][c] = *reinterpret_cast<const float4 *>(base + (i + u) * slot_stride + c * 4);
+            for (int c = 0; c < 2; ++c) v[u][c] = *reinterpret_cast<const float4 *>(base + (i + u) * slot_stride + c * 4);
 #pragma unroll
         for (int u = 0; u < 2; ++u) {
             const float w = w_sh[i + u][h];
 #pragma unroll
-            for (int c = 0; c < 4; ++c) {
+            for (int c = 0; c < 2; ++c) {
                 acc[c].x += w * v[u][c].x; acc[c].y += w * v[u][c].y; acc[c].z += w * v[u][c].z; acc[c].w += w * v[u][c].w;
             }
         }
@@ -279,20 +282,17 @@ __global__ void __launch_bounds__(128) decode_combine_kernel(const int32_t *__re
     for (; i < n; ++i) {
         const float w = w_sh[i][h];
 #pragma unroll
-        for (int c = 0; c < 4; ++c) {
+        for (int c = 0; c < 2; ++c) {
             const float4 v = *reinterpret_cast<const float4 *>(base + i * slot_stride + c * 4);
             acc[c].x += w * v.x; acc[c].y += w * v.y; acc[c].z += w * v.z; acc[c].w += w * v.w;
         }
     }
-    __nv_bfloat16 *o = out + ((size_t)s * hq + h) * 128 + part * 16;
-    uint4 pk0, pk1;
-    pk0.x = pack_bf16x2(acc[0].x, acc[0].y); pk0.y = pack_bf16x2(acc[0].z, acc[0].w);
-    pk0.z = pack_bf16x2(acc[1].x, acc[1].y); pk0.w = pack_bf16x2(acc[1].z, acc[1].w);
-    pk1.x = pack_bf16x2(acc[2].x, acc[2].y); pk1.y = pack_bf16x2(acc[2].z, acc[2].w);
-    pk1.z = pack_bf16x2(acc[3].x, acc[3].y); pk1.w = pack_bf16x2(acc[3].z, acc[3].w);
-    *reinterpret_cast<uint4 *>(o) = pk0;
-    *reinterpret_cast<uint4 *>(o + 8) = pk1;
-    if (part == 0) lse_out[(size_t)s * hq + h] = tot_sh[h];
+    __nv_bfloat16 *o = out + ((size_t)key * kGroup + h) * kD + part * 8;
+    uint4 pk;
+    pk.x = pack_bf16x2(acc[0].x, acc[0].y); pk.y = pack_bf16x2(acc[0].z, acc[0].w);
+    pk.z = pack_bf16x2(acc[1].x, acc[1].y); pk.w = pack_bf16x2(acc[1].z, acc[1].w);
+    *reinterpret_cast<uint4 *>(o) = pk;
+    if (part == 0) lse_out[(size_t)key * kGroup + h] = tot_sh[h];
 }
 
 template <class Slots, class OutT>
@@ -466,7 +466,7 @@ extern "C" padoc_status padoc_branch_decode_attn(const padoc_kv_pool *pool, cons
 
     if ((int64_t)pool->num_blocks * cfg.num_kv_heads * kBlk >= INT32_MAX) return PADOC_ERR_UNSUPPORTED;
     float *part_o = (float *)workspace;
-    float *part_lse = (float *)((uint8_t *)workspace + padoc_align256((size_t)info->num_slots * cfg.num_q_heads * kD * 4));
+    float *part_lse = (float *)((uint8_t *)workspace + padoc_align256((size_t)info->num_slots * kGroup * kD * 4));
     const float sl2 = scale * PADOC_LOG2E;
 
     // shared streams of dense pages on the tensor cores
@@ -478,7 +478,7 @@ extern "C" padoc_status padoc_branch_decode_attn(const padoc_kv_pool *pool, cons
         if (info->num_tc_items > 0 && !padoc_make_tmap_bf16_4d(&qmap, q, dims, strides, box)) return PADOC_ERR_CUDA;
     }
     padoc_status st = padoc_launch_decode_tc(&kmap, &vmap, &qmap, plan, info, page_block_table, page_table_stride,
-                                             pool->num_blocks, q, part_o, part_lse, sl2, err, cs);
+                                             pool->num_blocks, part_o, part_lse, sl2, err, cs);
     if (st != PADOC_OK) return st;
 
     // private histories and the shared streams of sparse pages, one warp per item
@@ -523,11 +523,11 @@ extern "C" padoc_status padoc_branch_decode_attn(const padoc_kv_pool *pool, cons
         if (st != PADOC_OK) return st;
     }
     const int64_t out_rows = (int64_t)info->num_streams * cfg.num_q_heads;
-    if (cfg.num_q_heads == 16 && info->max_stream_slots <= kCombineMaxSlots) {
-        decode_combine_kernel<<<(unsigned)info->num_streams, 128, 0, cs>>>(prm.slot_ptr, part_o, part_lse,
-                                                                           cfg.num_q_heads, (__nv_bfloat16 *)out, lse);
+    if (info->max_stream_slots <= kCombineMaxSlots) {
+        decode_combine_kernel<<<(unsigned)((int64_t)info->num_streams * cfg.num_kv_heads), 128, 0, cs>>>(
+            prm.slot_ptr, part_o, part_lse, (__nv_bfloat16 *)out, lse);
     } else {
-        RaggedSlots sl{prm.slot_ptr, cfg.num_q_heads};
+        RaggedSlots sl{prm.slot_ptr, kGroup};
         combine_kernel<RaggedSlots, __nv_bfloat16><<<(unsigned)((out_rows + 3) / 4), 128, 0, cs>>>(
             sl, part_o, part_lse, out_rows, kD, (__nv_bfloat16 *)out, lse);
     }

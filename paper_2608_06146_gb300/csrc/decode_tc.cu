@@ -1,21 +1,32 @@
 // decode_tc.cu -- C2 on the 5th-generation tensor cores: the shared-stream part of one decode step.
 //
-// For a page whose branches x query heads (of one KV head) fill dense M = 128 tiles, a work item
-// covers a split-K piece [tok_begin, tok_end) of the page's shared stream (prefix + layout, stored
-// once in the paged KV cache) for up to 32 of its streams: two M-tiles of 16 streams x 8 query
-// heads. Each K/V tile of 128 tokens is fetched from HBM once and multiplied against every
-// stream's queries; row (stream b, head h) sees the columns before its own cutoff P + f_k
-// (Algorithm 1's mask row restricted to the shared stream). The item writes one partial
-// (normalized O, natural-log LSE) per (stream, head) into its split-K slot; the merge kernel joins
-// the shared-stream and private-history partials.
+// For a page whose branches x query heads (of one KV head) fill dense M = 128 tiles, the page's
+// shared stream (prefix + layout, stored once in the paged KV cache) is read once per K/V tile of
+// 128 tokens and multiplied against the queries of up to 32 of its streams: two M-tiles of 16
+// streams x 8 query heads. Row (stream b, head h) sees the columns before its own cutoff P + f_k
+// (Algorithm 1's mask row restricted to the shared stream).
 //
-// The CTA layout follows the packed-prefill kernel: warps 0-3 / 4-7 run the softmax of M-tile 0 / 1
-// (thread t owns row t), warp 8 is the TMA producer (the item's queries as one 4-D box per panel;
-// the item's block rows looked up once; then lanes 0-7 each fetch one 16-token paged block of K and
-// of V per tile, two 64-column boxes each; blocks past the piece or with an out-of-range id are
-// fetched from an out-of-range coordinate, which fills zeros), warp 9 allocates TMEM and issues the
-// MMAs as a converged warp. A stage's K is released when the tile's last QK^T completes and its V
-// when the last PV completes. TMEM: S_i / P_i at columns 128i, O_i at 256 + 128i.
+// The kernel is persistent and stream-K balanced: the planner lays every (KV head, page, stream
+// group) tile sequence end to end and gives each CTA one contiguous range of equal work, which
+// becomes a list of pieces (a piece = the tiles of one sequence inside the range). A CTA walks its
+// pieces back to back; its K/V ring, barrier phases and TMEM carry over from one piece to the next,
+// so the next piece's tiles are in flight while the current one finishes. Each piece writes one
+// partial (normalized O, natural-log LSE) per (stream, head) into its split-K slot; the merge
+// kernel joins the partials of a (stream, KV head).
+//
+// CTA layout: warps 0-7 run the softmax and epilogue of one M-tile at a time (M-tile 0, then 1,
+// tile by tile): warp w reads TMEM lanes 32 (w % 4) ... (one row per thread) and column half w / 4,
+// and the two threads of a row swap their partial row max (and, at the end, row sum) through
+// shared memory. While they work on one M-tile, the tensor cores run the other M-tile's PV and
+// next QK^T. Warps 8 and 10 are the TMA producers of the K ring (3 tiles: a K tile is free once
+// its QK^T completes, so K runs two tiles ahead) and the V ring (2 tiles: V is held until the
+// tile's PV completes): lanes 0-7 each fetch one 16-token paged block per tile, two 64-column boxes,
+// with the block ids looked up one tile ahead; blocks past the piece or with an out-of-range id are
+// fetched from an out-of-range coordinate, which fills zeros. Warp 8 also fetches each piece's
+// queries (one 4-D box per panel) once the previous piece's last QK^T has completed. Warp 9
+// allocates TMEM and issues the MMAs as a converged warp.
+// TMEM: S_i / P_i at columns 128i, O_i at 256 + 128i. The next piece's first PV overwrites O_i; it
+// waits for P_i of that piece, which the softmax warps publish only after reading O_i out.
 #include <math.h>
 
 #include "common.cuh"
@@ -29,34 +40,41 @@ constexpr int kBlk = 16;         // tokens per paged block
 constexpr int kKT = 128;         // tokens per K/V tile
 constexpr int kPanel = 128 * 128;
 constexpr int kTile = 2 * kPanel;
-constexpr int kStages = 2;
+constexpr int kKStages = 3;       // K tiles in the ring: K is released early (after QK^T)
+constexpr int kVStages = 2;       // V tiles in the ring: V is held until the tile's PV completes
 constexpr uint32_t kTmemCols = 512;
-constexpr int kThreads = 320;
+constexpr int kThreads = 352;
 
 enum {
-    B_Q = 0,
-    B_KFULL = 1,     // [stage]
-    B_VFULL = 3,     // [stage]
-    B_KEMPTY = 5,    // [stage]: the last QK^T of the tile has completed
-    B_VEMPTY = 7,    // [stage]: the last PV of the tile has completed
-    B_SFULL = 9,     // [m-tile]
-    B_PFULL = 11,    // [m-tile], 128 arrivals
-    B_PVDONE = 13,   // [m-tile]
-    B_FINAL = 15,
-    B_COUNT = 16
+    B_Q = 0,         // the piece's queries have landed
+    B_QFREE = 1,     // the piece's last QK^T has completed: the query buffer may be refilled
+    B_KFULL = 2,     // [K stage]
+    B_KEMPTY = 5,    // [K stage]: the last QK^T of the tile has completed
+    B_VFULL = 8,     // [V stage]
+    B_VEMPTY = 10,   // [V stage]: the last PV of the tile has completed
+    B_SFULL = 12,    // [m-tile]
+    B_PFULL = 14,    // [m-tile], one arrival per softmax warp
+    B_PVDONE = 16,   // [m-tile]
+    B_FINAL = 18,
+    B_COUNT = 19
 };
 
-constexpr int kMaxItemBlocks = PADOC_TC_MAX_ITEM_TOKENS / kBlk;   // block rows an item looks up once
-constexpr size_t kSmemBytes = 1024 + (size_t)kTile * (2 + 2 * kStages) + B_COUNT * 8 + 64 + kMaxItemBlocks * 4;
+constexpr int kSoftmaxWarps = 8;
+constexpr int kXchBytes = 2 * 2 * 128 * 4;   // row max / sum swap: [buffer][column half][row] floats
+// Q (two M-tiles), the K and V rings, then barriers and the swap buffer: 231,680 bytes, so there is
+// no room to align the start by hand; the kernel checks that the driver placed it on a 1024-byte
+// boundary (the base of a CTA's dynamic shared memory is) and refuses to run otherwise.
+constexpr size_t kTilesBytes = (size_t)kTile * (2 + kKStages + kVStages);
+constexpr size_t kSmemBytes = kTilesBytes + 256 + kXchBytes;
+static_assert(kSmemBytes <= 232448, "shared memory per CTA");
 
 struct TcDecodeParams {
-    const int32_t *shared_len, *slot_ptr;
+    const int32_t *shared_len, *slot_ptr, *cta_ptr;
     const padoc_item *items;
     const int32_t *page_table;
     int32_t page_stride;
-    int32_t num_blocks, num_kv_heads, num_q_heads;
+    int32_t num_blocks, num_kv_heads;
     int32_t pool_rows;           // num_blocks * num_kv_heads * 16: first out-of-range row
-    const __nv_bfloat16 *q;
     float *part_o, *part_lse;
     float scale_log2;
     int *err;
@@ -70,288 +88,40 @@ __device__ __forceinline__ bool wait_or_abort(uint32_t bar, uint32_t parity, int
     return false;
 }
 
-template <int MT>
-__device__ __forceinline__ void decode_tc_body(const CUtensorMap *kmap, const CUtensorMap *vmap, const CUtensorMap *qmap,
-                                               const TcDecodeParams &prm, const padoc_item &it, uint8_t *smem,
-                                               uint64_t *bars, int32_t *block_rows, uint32_t tmem,
-                                               volatile int *abort_flag)
+__device__ __forceinline__ int piece_tiles(const padoc_item &it)
 {
-    uint8_t *sq = smem;
-    uint8_t *sk = sq + 2 * kTile;
-    uint8_t *sv = sk + kStages * kTile;
-    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int g = it.kv_head;
-    const int tb = it.tok_begin, te = it.tok_end;
-    const int ne = (te - tb + kKT - 1) / kKT;   // K/V tiles of this piece
-    auto bar = [&](int i) { return smem_u32(&bars[i]); };
-
-    if (warp == 8) {
-        // ---------------------------------------------------------------- TMA producer (whole warp)
-        // queries first: one 4-D box per 64-column panel gathers 16 streams x 8 heads of KV head g
-        if (lane == 0 && ne > 0) {
-            mbar_arrive_expect_tx(bar(B_Q), MT * kTile);
-#pragma unroll
-            for (int i = 0; i < MT; ++i) {
-                tma_load_4d(smem_u32(sq + i * kTile), qmap, 0, 0, g, it.first_stream + 16 * i, bar(B_Q));
-                tma_load_4d(smem_u32(sq + i * kTile) + kPanel, qmap, 64, 0, g, it.first_stream + 16 * i, bar(B_Q));
-            }
-        }
-        // the item's block rows, looked up once (out-of-range ids and blocks past the piece read
-        // from an out-of-range row, which fills zeros)
-        const int32_t *table = prm.page_table + (size_t)it.index * prm.page_stride;
-        const int nblk = ne * (kKT / kBlk);
-        auto lookup = [&](int bi) {
-            const int tok0 = tb + bi * kBlk;
-            int32_t row = prm.pool_rows;
-            if (tok0 < te) {
-                const int32_t id = table[tok0 / kBlk];
-                if (id >= 0 && id < prm.num_blocks) row = (id * prm.num_kv_heads + g) * kBlk;
-                else padoc_record_error(prm.err, PADOC_DEVERR_BLOCK_ID, id);
-            }
-            block_rows[bi] = row;
-        };
-        // the first tile's rows first, so its loads start before the remaining lookups
-        if (lane < kKT / kBlk && lane < nblk) lookup(lane);
-        __syncwarp();
-        int issued = 0;
-        for (int j = 0; j < ne; ++j) {
-            if (j == 1) {
-                for (int bi = kKT / kBlk + lane; bi < nblk; bi += 32) lookup(bi);
-                __syncwarp();
-            }
-            const int s = j & 1;
-            const uint32_t off = (uint32_t)lane * (kBlk * 128);
-            const int32_t row = lane < kKT / kBlk ? block_rows[j * (kKT / kBlk) + lane] : 0;
-            bool ok = true;
-            if (j >= 2) ok = wait_or_abort(bar(B_KEMPTY + s), ((j - 2) >> 1) & 1, prm.err, 50, abort_flag);
-            if (!__all_sync(0xffffffffu, ok)) break;
-            if (lane == 0) mbar_arrive_expect_tx(bar(B_KFULL + s), kTile);
-            __syncwarp();
-            if (lane < kKT / kBlk) {
-                const uint32_t kb = smem_u32(sk + s * kTile) + off;
-                tma_load_2d(kb, kmap, 0, row, bar(B_KFULL + s));
-                tma_load_2d(kb + kPanel, kmap, 64, row, bar(B_KFULL + s));
-            }
-            if (j >= 2) ok = wait_or_abort(bar(B_VEMPTY + s), ((j - 2) >> 1) & 1, prm.err, 53, abort_flag);
-            if (!__all_sync(0xffffffffu, ok)) break;
-            if (lane == 0) mbar_arrive_expect_tx(bar(B_VFULL + s), kTile);
-            __syncwarp();
-            if (lane < kKT / kBlk) {
-                const uint32_t vb = smem_u32(sv + s * kTile) + off;
-                tma_load_2d(vb, vmap, 0, row, bar(B_VFULL + s));
-                tma_load_2d(vb + kPanel, vmap, 64, row, bar(B_VFULL + s));
-            }
-            issued = j + 1;
-        }
-        // copies still in flight must land before the CTA's shared memory is released
-        if (lane == 0) {
-            if (ne > 0) mbar_wait_bounded(bar(B_Q), 0, prm.err, 54);
-            for (int j = (issued > 2 ? issued - 2 : 0); j < issued; ++j) {
-                mbar_wait_bounded(bar(B_KFULL + (j & 1)), (j >> 1) & 1, prm.err, 51);
-                mbar_wait_bounded(bar(B_VFULL + (j & 1)), (j >> 1) & 1, prm.err, 52);
-            }
-        }
-    } else if (warp == 9) {
-        // ---------------------------------------------------------------- MMA issuer (whole warp)
-        constexpr uint32_t idS = umma_idesc_bf16(128, kKT, false);
-        constexpr uint32_t idPV = umma_idesc_bf16(128, kD, true);
-        const uint64_t dq0 = umma_desc_sw128(smem_u32(sq), 16, 1024);
-        const uint64_t dq1 = umma_desc_sw128(smem_u32(sq + kTile), 16, 1024);
-        const uint64_t dk0 = umma_desc_sw128(smem_u32(sk), 16, 1024);
-        const uint64_t dk1 = umma_desc_sw128(smem_u32(sk + kTile), 16, 1024);
-        const uint64_t dv0 = umma_desc_sw128(smem_u32(sv), kPanel, 1024);
-        const uint64_t dv1 = umma_desc_sw128(smem_u32(sv + kTile), kPanel, 1024);
-        auto wait_w = [&](int b, uint32_t parity, int site) {
-            const bool r = wait_or_abort(bar(b), parity, prm.err, site, abort_flag);
-            return __all_sync(0xffffffffu, r);
-        };
-        auto issue_s = [&](int i, int stage) {
-            const uint64_t da = i ? dq1 : dq0, db = stage ? dk1 : dk0;
-#pragma unroll
-            for (int ks = 0; ks < 8; ++ks) {
-                const uint32_t off = ((ks >> 2) * kPanel + (ks & 3) * 32) >> 4;
-                umma_bf16_ss_warp(tmem + 128 * i, da + off, db + off, idS, ks > 0);
-            }
-            umma_commit_warp(bar(B_SFULL + i));
-        };
-        bool ok = ne > 0 && wait_w(B_Q, 0, 60) && wait_w(B_KFULL, 0, 61);
-        if (ok) {
-            tc_fence_after();
-#pragma unroll
-            for (int i = 0; i < MT; ++i) issue_s(i, 0);
-            umma_commit_warp(bar(B_KEMPTY));
-        }
-        for (int j = 0; ok && j < ne; ++j) {
-            const int s = j & 1, sn = (j + 1) & 1;
-#pragma unroll
-            for (int i = 0; i < MT; ++i) {
-                if (!wait_w(B_PFULL + i, j & 1, 62)) { ok = false; break; }
-                if (i == 0 && !wait_w(B_VFULL + s, (j >> 1) & 1, 63)) { ok = false; break; }
-                tc_fence_after();
-                const uint64_t db = s ? dv1 : dv0;
-#pragma unroll
-                for (int kk = 0; kk < 8; ++kk)
-                    umma_bf16_ts_warp(tmem + 256 + 128 * i, tmem + 128 * i + kk * 8, db + kk * (2048 >> 4), idPV,
-                                      (j > 0 || kk > 0));
-                umma_commit_warp(bar(B_PVDONE + i));
-                if (i == MT - 1) umma_commit_warp(bar(B_VEMPTY + s));
-                if (j + 1 < ne) {
-                    if (i == 0 && !wait_w(B_KFULL + sn, ((j + 1) >> 1) & 1, 64)) { ok = false; break; }
-                    tc_fence_after();
-                    issue_s(i, sn);
-                    if (i == MT - 1) umma_commit_warp(bar(B_KEMPTY + sn));
-                }
-            }
-        }
-        // every MMA issued above must complete before TMEM is released
-        umma_commit_warp(bar(B_FINAL));
-        mbar_wait_bounded(bar(B_FINAL), 0, prm.err, 65);
-    } else if (warp / 4 < MT) {
-        // ---------------------------------------------------------------- queries, softmax, epilogue
-        const int mi = warp / 4;                    // M-tile
-        const int row = tid & 127;
-        const int b = mi * 16 + row / kGroup, hl = row % kGroup;
-        const bool valid = b < it.num_streams;
-        const int s = it.first_stream + (valid ? b : 0);
-        const int h = g * kGroup + hl;
-        const int cutoff = valid ? min(prm.shared_len[s], te) : tb;   // visible tokens end here
-        const uint32_t lanes = (uint32_t)((warp & 3) * 32) << 16;
-        const uint32_t tS = tmem + lanes + 128 * mi, tO = tmem + lanes + 256 + 128 * mi;
-        const float c = prm.scale_log2;
-        auto wait_all = [&](int bb, uint32_t parity, int site) {
-            const bool r = wait_or_abort(bar(bb), parity, prm.err, site, abort_flag);
-            return __all_sync(0xffffffffu, r);
-        };
-        float m_ref = -INFINITY, l = 0.f;
-        bool ok = ne > 0;
-        for (int j = 0; ok && j < ne; ++j) {
-            const int w = min(max(cutoff - (tb + j * kKT), 0), kKT);   // visible columns [0, w)
-            const bool full = __all_sync(0xffffffffu, w == kKT);
-            if (!wait_all(B_SFULL + mi, j & 1, 70)) { ok = false; break; }
-            tc_fence_after();
-            float mx4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
-#pragma unroll
-            for (int q = 0; q < 4; q += 2) {
-                uint32_t sr[2][32];
-                tmem_ld32(tS + q * 32, sr[0]);
-                tmem_ld32(tS + q * 32 + 32, sr[1]);
-                tmem_ld_wait();
-                if (!full) {
-#pragma unroll
-                    for (int u = 0; u < 2; ++u) {
-                        const uint32_t vis = interval_bits(0, w, (q + u) * 32);
-#pragma unroll
-                        for (int i = 0; i < 32; ++i) sr[u][i] = (vis >> i) & 1u ? sr[u][i] : 0xff800000u;
-                        tmem_st32(tS + (q + u) * 32, sr[u]);
-                    }
-                }
-#pragma unroll
-                for (int u = 0; u < 2; ++u)
-#pragma unroll
-                    for (int i = 0; i < 32; i += 8) {
-                        mx4[0] = fmax3f(mx4[0], __uint_as_float(sr[u][i]), __uint_as_float(sr[u][i + 1]));
-                        mx4[1] = fmax3f(mx4[1], __uint_as_float(sr[u][i + 2]), __uint_as_float(sr[u][i + 3]));
-                        mx4[2] = fmax3f(mx4[2], __uint_as_float(sr[u][i + 4]), __uint_as_float(sr[u][i + 5]));
-                        mx4[3] = fmax3f(mx4[3], __uint_as_float(sr[u][i + 6]), __uint_as_float(sr[u][i + 7]));
-                    }
-            }
-            if (!full) tmem_st_wait();
-            const float mx = fmaxf(fmax3f(mx4[0], mx4[1], mx4[2]), mx4[3]);
-            const float m_new = fmaxf(m_ref, mx);
-            const bool rescale = m_ref != -INFINITY && (m_new - m_ref) * c > 8.f;
-            if (m_ref == -INFINITY) m_ref = m_new;
-            if (__any_sync(0xffffffffu, rescale)) {
-                // PV_i(j-1) completed before S_i(j) (issue order), so O_i is quiescent here
-                const float alpha = rescale ? fast_exp2((m_ref - m_new) * c) : 1.f;
-#pragma unroll
-                for (int q = 0; q < 4; ++q) {
-                    uint32_t o[32];
-                    tmem_ld32(tO + q * 32, o);
-                    tmem_ld_wait();
-#pragma unroll
-                    for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * alpha);
-                    tmem_st32(tO + q * 32, o);
-                }
-                if (rescale) { l *= alpha; m_ref = m_new; }
-            }
-            const float moff = m_ref == -INFINITY ? 0.f : m_ref * c;
-            float rs[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll
-            for (int half = 0; half < 2; ++half) {
-                uint32_t pk[32];
-                uint32_t sr[2][32];
-                tmem_ld32(tS + half * 64, sr[0]);
-                tmem_ld32(tS + half * 64 + 32, sr[1]);
-                tmem_ld_wait();
-#pragma unroll
-                for (int qq = 0; qq < 2; ++qq) {
-#pragma unroll
-                    for (int i = 0; i < 32; i += 2) {
-                        const float p0 = fast_exp2(fmaf(__uint_as_float(sr[qq][i]), c, -moff));
-                        const float p1 = fast_exp2(fmaf(__uint_as_float(sr[qq][i + 1]), c, -moff));
-                        rs[(i >> 1) & 3] += p0 + p1;
-                        pk[qq * 16 + (i >> 1)] = pack_bf16x2(p0, p1);
-                    }
-                }
-                tmem_st32(tS + half * 32, pk);
-            }
-            l += (rs[0] + rs[1]) + (rs[2] + rs[3]);
-            tmem_st_wait();
-            tc_fence_before();
-            mbar_arrive(bar(B_PFULL + mi));
-        }
-        // partial result of this piece: O / l (fp32) and its natural-log LSE
-        const bool have = ne == 0 || (ok && wait_all(B_PVDONE + mi, (ne - 1) & 1, 71));
-        if (have) {
-            tc_fence_after();
-            const bool empty = !(l > 0.f);
-            const float inv = empty ? 0.f : 1.f / l;
-            const size_t prow = (size_t)(prm.slot_ptr[s] + it.slot) * prm.num_q_heads + h;
-            float *dst = prm.part_o + prow * kD;
-#pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                uint32_t o[32];
-                if (ne > 0) {
-                    tmem_ld32(tO + q * 32, o);
-                    tmem_ld_wait();
-                }
-                if (valid) {
-#pragma unroll
-                    for (int i = 0; i < 32; i += 4)
-                        *reinterpret_cast<float4 *>(dst + q * 32 + i) =
-                            empty ? make_float4(0.f, 0.f, 0.f, 0.f)
-                                  : make_float4(__uint_as_float(o[i]) * inv, __uint_as_float(o[i + 1]) * inv,
-                                                __uint_as_float(o[i + 2]) * inv, __uint_as_float(o[i + 3]) * inv);
-                }
-            }
-            if (valid) prm.part_lse[prow] = empty ? -INFINITY : (m_ref * c + log2f(l)) * PADOC_LN2;
-        }
-    }
+    return it.tok_end > it.tok_begin ? (it.tok_end - it.tok_begin + kKT - 1) / kKT : 0;
 }
+
+__device__ __forceinline__ int piece_mtiles(const padoc_item &it) { return it.num_streams > 16 ? 2 : 1; }
 
 __global__ void __launch_bounds__(kThreads, 1)
 decode_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap,
                  const __grid_constant__ CUtensorMap qmap, const TcDecodeParams prm)
 {
-    extern __shared__ uint8_t smem_raw[];
-    uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
-    uint64_t *bars = (uint64_t *)(smem + (size_t)kTile * (2 + 2 * kStages));
-    uint32_t *tmem_slot = (uint32_t *)(bars + B_COUNT);
-    volatile int *abort_flag = (volatile int *)(tmem_slot + 1);
-    int32_t *block_rows = (int32_t *)(tmem_slot + 16);
-    const int tid = threadIdx.x, warp = tid >> 5;
+    extern __shared__ __align__(1024) uint8_t smem[];
+    if (smem_u32(smem) & 1023u) {
+        if (threadIdx.x == 0) padoc_record_error(prm.err, PADOC_DEVERR_SMEM_ALIGN, (int)(smem_u32(smem) & 1023u));
+        return;
+    }
+    uint8_t *sq = smem;
+    uint8_t *sk = sq + 2 * kTile;
+    uint8_t *sv = sk + kKStages * kTile;
+    uint8_t *misc = smem + kTilesBytes;
+    uint64_t *bars = (uint64_t *)misc;
+    uint32_t *tmem_slot = (uint32_t *)(misc + 192);
+    volatile int *abort_flag = (volatile int *)(misc + 196);
+    float *xch = (float *)(misc + 256);
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    auto bar = [&](int i) { return smem_u32(&bars[i]); };
     // the warp kernel that follows reads nothing this grid writes before its final wait, so it may
     // start filling SMs as soon as every CTA of this grid is resident
     pdl_launch_dependents();
-    const padoc_item it = prm.items[blockIdx.x];
-    const int mt = it.num_streams > 16 ? 2 : 1;
+    const int u0 = prm.cta_ptr[blockIdx.x], u1 = prm.cta_ptr[blockIdx.x + 1];
 
     if (tid == 0) {
-        for (int i = 0; i < B_COUNT; ++i) {
-            uint32_t cnt = 1;
-            if (i == B_PFULL || i == B_PFULL + 1) cnt = 128;
-            mbar_init(smem_u32(&bars[i]), cnt);
-        }
+        for (int i = 0; i < B_COUNT; ++i)
+            mbar_init(smem_u32(&bars[i]), (i == B_PFULL || i == B_PFULL + 1) ? kSoftmaxWarps : 1);
         *abort_flag = 0;
         fence_barrier_init();
         tma_prefetch_desc(&kmap);
@@ -366,8 +136,352 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
-    if (mt == 2) decode_tc_body<2>(&kmap, &vmap, &qmap, prm, it, smem, bars, block_rows, tmem, abort_flag);
-    else decode_tc_body<1>(&kmap, &vmap, &qmap, prm, it, smem, bars, block_rows, tmem, abort_flag);
+
+    if (warp == 8 || warp == 10) {
+        // ---------------------------------------------------------------- TMA producers (whole warps)
+        // warp 8 fills the K ring (and loads each piece's queries), warp 10 the V ring, each as far
+        // ahead as its ring allows. Lane l < 8 owns paged block l of every tile; its block id is read
+        // one tile ahead.
+        const bool is_k = warp == 8;
+        const int nst = is_k ? kKStages : kVStages;
+        const CUtensorMap *map = is_k ? &kmap : &vmap;
+        uint8_t *ring = is_k ? sk : sv;
+        const int b_full = is_k ? B_KFULL : B_VFULL, b_empty = is_k ? B_KEMPTY : B_VEMPTY;
+        int32_t id_next = 0;
+        bool in_next = false;
+        auto fetch_id = [&](int uu, int jj) {
+            const padoc_item &p = prm.items[uu];
+            const int tok0 = p.tok_begin + jj * kKT + lane * kBlk;
+            in_next = lane < kKT / kBlk && tok0 < p.tok_end;
+            id_next = in_next ? prm.page_table[(size_t)p.index * prm.page_stride + tok0 / kBlk] : 0;
+        };
+        // a piece's queries: one 4-D box per 64-column panel gathers 16 streams x the 8 heads of the
+        // KV head; the next piece's boxes are pulled into L2 meanwhile, so that its reload (which
+        // must wait for this piece's last QK^T) is short
+        auto load_q = [&](const padoc_item &p, int uu) {
+            const int mt = piece_mtiles(p);
+            mbar_arrive_expect_tx(bar(B_Q), mt * kTile);
+            for (int i = 0; i < mt; ++i) {
+                tma_load_4d(smem_u32(sq + i * kTile), &qmap, 0, 0, p.kv_head, p.first_stream + 16 * i, bar(B_Q));
+                tma_load_4d(smem_u32(sq + i * kTile) + kPanel, &qmap, 64, 0, p.kv_head, p.first_stream + 16 * i, bar(B_Q));
+            }
+            if (uu + 1 < u1) {
+                const padoc_item &n = prm.items[uu + 1];
+                for (int i = 0; i < piece_mtiles(n); ++i) {
+                    tma_prefetch_l2_4d(&qmap, 0, 0, n.kv_head, n.first_stream + 16 * i);
+                    tma_prefetch_l2_4d(&qmap, 64, 0, n.kv_head, n.first_stream + 16 * i);
+                }
+            }
+        };
+        if (u0 < u1) fetch_id(u0, 0);
+        int n = 0, nq = 0;   // tiles and query sets issued
+        // the first piece's queries go out before anything else (they wait for nothing)
+        const bool q_first = is_k && u0 < u1 && piece_tiles(prm.items[u0]) > 0;
+        if (q_first) {
+            if (lane == 0) load_q(prm.items[u0], u0);
+            nq = 1;
+        }
+        bool ok = true;
+        for (int u = u0; ok && u < u1; ++u) {
+            const padoc_item it = prm.items[u];
+            const int ne = piece_tiles(it);
+            if (ne == 0) {
+                if (u + 1 < u1) fetch_id(u + 1, 0);
+                continue;
+            }
+            for (int j = 0; j < ne; ++j) {
+                const int32_t id = id_next;
+                const bool in = in_next;
+                if (j + 1 < ne) fetch_id(u, j + 1);
+                else if (u + 1 < u1) fetch_id(u + 1, 0);
+                int32_t row = prm.pool_rows;
+                if (in) {
+                    if (id >= 0 && id < prm.num_blocks) row = (id * prm.num_kv_heads + it.kv_head) * kBlk;
+                    else if (is_k) padoc_record_error(prm.err, PADOC_DEVERR_BLOCK_ID, id);
+                }
+                const int s = n % nst, use = n / nst;
+                if (use > 0) ok = wait_or_abort(bar(b_empty + s), (use - 1) & 1, prm.err, is_k ? 50 : 53, abort_flag);
+                if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
+                if (lane == 0) mbar_arrive_expect_tx(bar(b_full + s), kTile);
+                __syncwarp();
+                if (lane < kKT / kBlk) {
+                    const uint32_t dst = smem_u32(ring + s * kTile) + (uint32_t)lane * (kBlk * 128);
+                    tma_load_2d(dst, map, 0, row, bar(b_full + s));
+                    tma_load_2d(dst + kPanel, map, 64, row, bar(b_full + s));
+                }
+                ++n;
+                if (is_k && j == 0 && !(q_first && u == u0)) {
+                    // this piece's queries, once the previous piece's last QK^T has read the buffer
+                    if (nq > 0) ok = wait_or_abort(bar(B_QFREE), (nq - 1) & 1, prm.err, 55, abort_flag);
+                    if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
+                    if (lane == 0) load_q(it, u);
+                    ++nq;
+                }
+            }
+        }
+        // copies still in flight must land before the CTA's shared memory is released
+        if (lane == 0) {
+            if (nq > 0) mbar_wait_bounded(bar(B_Q), (nq - 1) & 1, prm.err, 54);
+            for (int J = (n > nst ? n - nst : 0); J < n; ++J)
+                mbar_wait_bounded(bar(b_full + J % nst), (J / nst) & 1, prm.err, is_k ? 51 : 52);
+        }
+    } else if (warp == 9) {
+        // ---------------------------------------------------------------- MMA issuer (whole warp)
+        constexpr uint32_t idS = umma_idesc_bf16(128, kKT, false);
+        constexpr uint32_t idPV = umma_idesc_bf16(128, kD, true);
+        const uint64_t dq0 = umma_desc_sw128(smem_u32(sq), 16, 1024);
+        const uint64_t dq1 = umma_desc_sw128(smem_u32(sq + kTile), 16, 1024);
+        // stage descriptors differ only in the start-address field (address >> 4)
+        const uint64_t dk0 = umma_desc_sw128(smem_u32(sk), 16, 1024);
+        const uint64_t dv0 = umma_desc_sw128(smem_u32(sv), kPanel, 1024);
+        auto wait_w = [&](int b, uint32_t parity, int site) {
+            const bool r = wait_or_abort(bar(b), parity, prm.err, site, abort_flag);
+            return __all_sync(0xffffffffu, r);
+        };
+        auto issue_s = [&](int i, int stage) {
+            const uint64_t da = i ? dq1 : dq0, db = dk0 + (uint64_t)(stage * (kTile >> 4));
+#pragma unroll
+            for (int ks = 0; ks < 8; ++ks) {
+                const uint32_t off = ((ks >> 2) * kPanel + (ks & 3) * 32) >> 4;
+                umma_bf16_ss_warp(tmem + 128 * i, da + off, db + off, idS, ks > 0);
+            }
+            umma_commit_warp(bar(B_SFULL + i));
+        };
+        int J = 0, nq = 0, c0 = 0, c1 = 0;   // tiles done, query sets used, tiles per M-tile
+        bool ok = true;
+        for (int u = u0; ok && u < u1; ++u) {
+            const padoc_item it = prm.items[u];
+            const int ne = piece_tiles(it), mt = piece_mtiles(it);
+            if (ne == 0) continue;
+            if (!wait_w(B_Q, nq & 1, 60) || !wait_w(B_KFULL + J % kKStages, (J / kKStages) & 1, 61)) { ok = false; break; }
+            ++nq;
+            tc_fence_after();
+            issue_s(0, J % kKStages);
+            if (mt == 2) issue_s(1, J % kKStages);
+            umma_commit_warp(bar(B_KEMPTY + J % kKStages));
+            if (ne == 1) umma_commit_warp(bar(B_QFREE));
+            for (int j = 0; ok && j < ne; ++j) {
+                const int Jj = J + j, s = Jj % kVStages, kn = (Jj + 1) % kKStages;
+#pragma unroll
+                for (int i = 0; i < 2; ++i) {
+                    if (i >= mt) break;
+                    const int ci = i ? c1 : c0;
+                    if (!wait_w(B_PFULL + i, ci & 1, 62)) { ok = false; break; }
+                    if (i == 0 && !wait_w(B_VFULL + s, (Jj / kVStages) & 1, 63)) { ok = false; break; }
+                    tc_fence_after();
+                    const uint64_t db = dv0 + (uint64_t)(s * (kTile >> 4));
+#pragma unroll
+                    for (int kk = 0; kk < 8; ++kk)
+                        umma_bf16_ts_warp(tmem + 256 + 128 * i, tmem + 128 * i + kk * 8, db + kk * (2048 >> 4), idPV,
+                                          (j > 0 || kk > 0));
+                    umma_commit_warp(bar(B_PVDONE + i));
+                    if (i == mt - 1) umma_commit_warp(bar(B_VEMPTY + s));
+                    if (i) ++c1; else ++c0;
+                    if (j + 1 < ne) {
+                        if (i == 0 && !wait_w(B_KFULL + kn, ((Jj + 1) / kKStages) & 1, 64)) { ok = false; break; }
+                        tc_fence_after();
+                        issue_s(i, kn);
+                        if (i == mt - 1) {
+                            umma_commit_warp(bar(B_KEMPTY + kn));
+                            if (j + 2 == ne) umma_commit_warp(bar(B_QFREE));
+                        }
+                    }
+                }
+            }
+            J += ne;
+        }
+        // every MMA issued above must complete before TMEM is released
+        umma_commit_warp(bar(B_FINAL));
+        mbar_wait_bounded(bar(B_FINAL), 0, prm.err, 65);
+    } else {
+        // ---------------------------------------------------------------- softmax and epilogue
+        const int quad = warp & 3, hc = warp >> 2;   // TMEM lane quarter, column half
+        const int row = quad * 32 + lane;            // row of the M-tile = TMEM lane
+        const int hl = row % kGroup;
+        const uint32_t lanes = (uint32_t)(quad * 32) << 16;
+        const float c = prm.scale_log2;
+        auto wait_all = [&](int bb, uint32_t parity, int site) {
+            const bool r = wait_or_abort(bar(bb), parity, prm.err, site, abort_flag);
+            return __all_sync(0xffffffffu, r);
+        };
+        // The 8 warps meet at a named barrier for every swap, so none may leave the loops early: after
+        // a failed wait (ok = false) a warp skips the work but still takes every swap.
+        int nx = 0;   // row-value swaps so far (double-buffered)
+        auto swap_row = [&](float v) {   // returns the value the other column half passed for this row
+            float *buf = xch + (nx & 1) * 256;
+            buf[hc * 128 + row] = v;
+            named_bar_sync(1, kSoftmaxWarps * 32);
+            const float o = buf[(hc ^ 1) * 128 + row];
+            ++nx;
+            return o;
+        };
+        int cnt0 = 0, cnt1 = 0;   // tiles of M-tile 0 / 1 so far
+        bool ok = true;
+        // The next piece's fields are read while the current piece runs (its item at the piece's
+        // start, the rows' cutoffs after its first tile), so no global load latency sits between
+        // two pieces. Rows (stream b = 16 mi + row / 8, head row % 8) of M-tile mi see the shared
+        // columns before their cutoff.
+        const int b0 = row / kGroup, b1 = 16 + row / kGroup;
+        int n_tb = 0, n_te = 0, n_nstr = 0, n_first = 0, n_kvh = 0, n_slot = 0, n_cut0 = 0, n_cut1 = 0;
+        auto fetch_item = [&](int uu) {
+            const padoc_item *p = prm.items + uu;
+            n_tb = p->tok_begin;
+            n_te = p->tok_end;
+            n_nstr = p->num_streams;
+            n_first = p->first_stream;
+            n_kvh = p->kv_head;
+            n_slot = p->slot;
+        };
+        auto fetch_cut = [&]() {
+            n_cut0 = b0 < n_nstr ? min(prm.shared_len[n_first + b0], n_te) : n_tb;
+            n_cut1 = b1 < n_nstr ? min(prm.shared_len[n_first + b1], n_te) : n_tb;
+        };
+        if (u0 < u1) {
+            fetch_item(u0);
+            fetch_cut();
+        }
+        for (int u = u0; u < u1; ++u) {
+            const int tb = n_tb, te = n_te, nstr = n_nstr, first = n_first, kvh = n_kvh, slot = n_slot;
+            const int cut0 = n_cut0, cut1 = n_cut1;
+            const int ne = te > tb ? (te - tb + kKT - 1) / kKT : 0, mt = nstr > 16 ? 2 : 1;
+            if (u + 1 < u1) fetch_item(u + 1);
+            // first partial slot of each row's (stream, KV head), read during the piece's last tile
+            int pb0 = 0, pb1 = 0;
+            auto fetch_slots = [&]() {
+                pb0 = prm.slot_ptr[(size_t)(first + (b0 < nstr ? b0 : 0)) * prm.num_kv_heads + kvh] + slot;
+                if (mt == 2) pb1 = prm.slot_ptr[(size_t)(first + (b1 < nstr ? b1 : 0)) * prm.num_kv_heads + kvh] + slot;
+            };
+            float m0 = -INFINITY, l0 = 0.f, m1 = -INFINITY, l1 = 0.f;
+            for (int j = 0; j < ne; ++j) {
+                if (j == 1 && u + 1 < u1) fetch_cut();
+                if (j == ne - 1) fetch_slots();
+#pragma unroll
+                for (int mi = 0; mi < 2; ++mi) {
+                    if (mi >= mt) break;
+                    const uint32_t tS = tmem + lanes + 128 * mi, tO = tS + 256;
+                    const int cnt = mi ? cnt1 : cnt0;
+                    float &m_ref = mi ? m1 : m0;
+                    float &l = mi ? l1 : l0;
+                    // visible columns of this half: [0, w)
+                    const int w = min(max((mi ? cut1 : cut0) - (tb + j * kKT) - 64 * hc, 0), 64);
+                    const bool full = __all_sync(0xffffffffu, w == 64);
+                    ok = ok && wait_all(B_SFULL + mi, cnt & 1, 70);
+                    if (mi) ++cnt1; else ++cnt0;
+                    if (!ok) {
+                        swap_row(0.f);
+                        continue;
+                    }
+                    tc_fence_after();
+                    uint32_t sr[2][32];
+                    tmem_ld32(tS + 64 * hc, sr[0]);
+                    tmem_ld32(tS + 64 * hc + 32, sr[1]);
+                    tmem_ld_wait();
+                    if (!full) {
+#pragma unroll
+                        for (int uu = 0; uu < 2; ++uu) {
+                            const uint32_t vis = interval_bits(0, w, uu * 32);
+#pragma unroll
+                            for (int i = 0; i < 32; ++i) sr[uu][i] = (vis >> i) & 1u ? sr[uu][i] : 0xff800000u;
+                        }
+                    }
+                    float mx4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+#pragma unroll
+                    for (int uu = 0; uu < 2; ++uu)
+#pragma unroll
+                        for (int i = 0; i < 32; i += 8) {
+                            mx4[0] = fmax3f(mx4[0], __uint_as_float(sr[uu][i]), __uint_as_float(sr[uu][i + 1]));
+                            mx4[1] = fmax3f(mx4[1], __uint_as_float(sr[uu][i + 2]), __uint_as_float(sr[uu][i + 3]));
+                            mx4[2] = fmax3f(mx4[2], __uint_as_float(sr[uu][i + 4]), __uint_as_float(sr[uu][i + 5]));
+                            mx4[3] = fmax3f(mx4[3], __uint_as_float(sr[uu][i + 6]), __uint_as_float(sr[uu][i + 7]));
+                        }
+                    float mx = fmaxf(fmax3f(mx4[0], mx4[1], mx4[2]), mx4[3]);
+                    // every P store below lands after both halves have read their S columns
+                    mx = fmaxf(mx, swap_row(mx));
+                    const float m_new = fmaxf(m_ref, mx);
+                    // lazy rescaling: the reference max moves only when the row max grew by more
+                    // than 2^8 in probability
+                    const bool rescale = m_ref != -INFINITY && (m_new - m_ref) * c > 8.f;
+                    if (m_ref == -INFINITY) m_ref = m_new;
+                    float alpha = 1.f;
+                    if (rescale) {
+                        alpha = fast_exp2((m_ref - m_new) * c);
+                        l *= alpha;
+                        m_ref = m_new;
+                    }
+                    const float moff = m_ref == -INFINITY ? 0.f : m_ref * c;
+                    float rs[4] = {0.f, 0.f, 0.f, 0.f};
+                    uint32_t pk[32];
+#pragma unroll
+                    for (int qq = 0; qq < 2; ++qq) {
+#pragma unroll
+                        for (int i = 0; i < 32; i += 2) {
+                            const float p0 = fast_exp2(fmaf(__uint_as_float(sr[qq][i]), c, -moff));
+                            const float p1 = fast_exp2(fmaf(__uint_as_float(sr[qq][i + 1]), c, -moff));
+                            rs[(i >> 1) & 3] += p0 + p1;
+                            pk[qq * 16 + (i >> 1)] = pack_bf16x2(p0, p1);
+                        }
+                    }
+                    tmem_st32(tS + 32 * hc, pk);   // P (bf16 pairs) of columns [64 hc, 64 hc + 64)
+                    l += (rs[0] + rs[1]) + (rs[2] + rs[3]);
+                    if (__any_sync(0xffffffffu, rescale)) {
+                        // PV_i(j-1) completed before S_i(j) (issue order) and PV_i(j) waits for this
+                        // warp's P, so O_i is quiescent here
+#pragma unroll
+                        for (int q = 0; q < 2; ++q) {
+                            uint32_t o[32];
+                            tmem_ld32(tO + 64 * hc + q * 32, o);
+                            tmem_ld_wait();
+#pragma unroll
+                            for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * alpha);
+                            tmem_st32(tO + 64 * hc + q * 32, o);
+                        }
+                    }
+                    tmem_st_wait();
+                    tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(bar(B_PFULL + mi));
+                }
+            }
+            if (ne < 2 && u + 1 < u1) fetch_cut();
+            if (ne == 0) fetch_slots();
+            // partials of this piece: O / l (fp32) and the natural-log LSE of every row
+#pragma unroll
+            for (int mi = 0; mi < 2; ++mi) {
+                if (mi >= mt) break;
+                const int cnt = mi ? cnt1 : cnt0;
+                const float m_ref = mi ? m1 : m0;
+                float l = mi ? l1 : l0;
+                if (ne > 0) ok = ok && wait_all(B_PVDONE + mi, (cnt - 1) & 1, 71);
+                l += swap_row(l);   // plus the other column half's sum
+                if (!ok) continue;
+                tc_fence_after();
+                const int b = mi * 16 + row / kGroup;
+                const bool valid = b < nstr;
+                const bool empty = !(l > 0.f);
+                const float inv = empty ? 0.f : 1.f / l;
+                const size_t prow = (size_t)(mi ? pb1 : pb0) * kGroup + hl;
+                float *dst = prm.part_o + prow * kD + 64 * hc;
+                const uint32_t tO = tmem + lanes + 256 + 128 * mi + 64 * hc;
+#pragma unroll
+                for (int q = 0; q < 2; ++q) {
+                    uint32_t o[32];
+                    if (ne > 0) {
+                        tmem_ld32(tO + q * 32, o);
+                        tmem_ld_wait();
+                    }
+                    if (valid) {
+                        // a row's half is 256 contiguous bytes: whole 32-byte sectors per store
+#pragma unroll
+                        for (int i = 0; i < 32; i += 8) {
+                            auto v = [&](int k) { return empty ? 0.f : __uint_as_float(o[i + k]) * inv; };
+                            st_global_v8(dst + q * 32 + i, v(0), v(1), v(2), v(3), v(4), v(5), v(6), v(7));
+                        }
+                    }
+                }
+                if (valid && hc == 0) prm.part_lse[prow] = empty ? -INFINITY : (m_ref * c + log2f(l)) * PADOC_LN2;
+            }
+        }
+    }
     tc_fence_before();
     __syncthreads();
     if (warp == 9) {
@@ -380,26 +494,25 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
 
 padoc_status padoc_launch_decode_tc(const CUtensorMap *kmap, const CUtensorMap *vmap, const CUtensorMap *qmap, const int32_t *plan,
                                     const padoc_decode_plan *info, const int32_t *page_table, int32_t page_stride,
-                                    int32_t num_blocks, const void *q, float *part_o, float *part_lse, float scale_log2,
-                                    int *err, cudaStream_t stream)
+                                    int32_t num_blocks, float *part_o, float *part_lse, float scale_log2, int *err,
+                                    cudaStream_t stream)
 {
-    if (info->num_tc_items == 0) return PADOC_OK;
+    if (info->num_tc_items == 0 || info->tc_ctas == 0) return PADOC_OK;
     TcDecodeParams prm;
     prm.shared_len = plan + info->off_shared_len;
     prm.slot_ptr = plan + info->off_slot_ptr;
+    prm.cta_ptr = plan + info->off_cta_ptr;
     prm.items = reinterpret_cast<const padoc_item *>(plan + info->off_items);
     prm.page_table = page_table;
     prm.page_stride = page_stride;
     prm.num_blocks = num_blocks;
     prm.num_kv_heads = info->cfg.num_kv_heads;
-    prm.num_q_heads = info->cfg.num_q_heads;
     prm.pool_rows = num_blocks * info->cfg.num_kv_heads * kBlk;
-    prm.q = (const __nv_bfloat16 *)q;
     prm.part_o = part_o;
     prm.part_lse = part_lse;
     prm.scale_log2 = scale_log2;
     prm.err = err;
     PADOC_CUDA_TRY(cudaFuncSetAttribute(decode_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes));
-    decode_tc_kernel<<<info->num_tc_items, kThreads, kSmemBytes, stream>>>(*kmap, *vmap, *qmap, prm);
+    decode_tc_kernel<<<info->tc_ctas, kThreads, kSmemBytes, stream>>>(*kmap, *vmap, *qmap, prm);
     return padoc_launch_status();
 }

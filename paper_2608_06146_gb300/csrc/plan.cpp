@@ -10,6 +10,8 @@
 #include <numeric>
 #include <vector>
 
+#include <cuda_runtime.h>
+
 #include "padoc_attn.h"
 #include "plan_internal.h"
 
@@ -178,12 +180,24 @@ namespace {
 
 struct Stream { int32_t page, shared_len, private_len; };
 
+// Multiprocessor count of the current CUDA device, or 152 (one GB300) when none is visible.
+int32_t padoc_default_ctas()
+{
+    int dev = 0, n = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n < 1) {
+        cudaGetLastError();
+        return 152;
+    }
+    return n;
+}
+
 struct PlanParts {
     std::vector<Stream> streams;
     std::vector<int32_t> page_len, page_first_stream, page_num_streams;
-    std::vector<int32_t> slot_ptr;
+    std::vector<int32_t> slot_ptr;      // [S * Hkv + 1]: partial slots of each (stream, KV head)
+    std::vector<int32_t> cta_ptr;       // [tc_ctas + 1]: tensor-core items of each CTA
     std::vector<padoc_item> items;
-    int32_t num_tc_items = 0;
+    int32_t num_tc_items = 0, tc_ctas = 0;
     int32_t max_page_blocks = 0, max_stream_blocks = 0;
     int64_t kv_tokens = 0;
 };
@@ -199,8 +213,8 @@ padoc_status build_parts(const padoc_page *pages, int32_t num_pages, const padoc
     if (cfg->split_tokens < 0 || (cfg->split_tokens > 0 && cfg->split_tokens % cfg->block_size != 0))
         return PADOC_ERR_INVALID_ARGUMENT;
     const int32_t bs = cfg->block_size;
-    const int32_t split = std::min(cfg->split_tokens > 0 ? cfg->split_tokens : PADOC_DEFAULT_SPLIT_TOKENS,
-                                   PADOC_TC_MAX_ITEM_TOKENS);
+    if (cfg->tc_ctas < 0) return PADOC_ERR_INVALID_ARGUMENT;
+    const int32_t split = cfg->split_tokens > 0 ? cfg->split_tokens : PADOC_DEFAULT_SPLIT_TOKENS;
     const int32_t psplit = PADOC_PRIVATE_SPLIT_TOKENS;
     const int32_t group = cfg->num_q_heads / cfg->num_kv_heads;
 
@@ -232,66 +246,109 @@ padoc_status build_parts(const padoc_page *pages, int32_t num_pages, const padoc
         pp.kv_tokens += s.private_len;
     }
 
-    // split-K slots: shared splits of the stream's page, then its private splits
-    std::vector<int32_t> page_splits(num_pages);
-    for (int32_t p = 0; p < num_pages; ++p) {
-        // only the part of the stream some stream of the page can see needs reading
-        int32_t vis = 0;
-        for (int32_t s = pp.page_first_stream[p]; s < pp.page_first_stream[p] + pp.page_num_streams[p]; ++s)
-            vis = std::max(vis, pp.streams[s].shared_len);
-        page_splits[p] = (vis + split - 1) / split;
-    }
-    pp.slot_ptr.assign((size_t)S + 1, 0);
-    for (int32_t s = 0; s < S; ++s) {
-        const int32_t np = page_splits[pp.streams[s].page];
-        const int32_t nv = (pp.streams[s].private_len + psplit - 1) / psplit;
-        pp.slot_ptr[s + 1] = pp.slot_ptr[s] + np + nv;
-    }
-
-    // work items, one set per KV head: tensor-core items first, then warp items
-    std::vector<padoc_item> tc_items, warp_items;
-    for (int32_t g = 0; g < cfg->num_kv_heads; ++g) {
+    // ---- tensor-core work: stream-K over the concatenated shared-stream tiles ----------------
+    // A segment is one (KV head, page, group of <= 32 streams) with the tiles of the shared stream
+    // the group can see. The segments are laid end to end and cut into one range of equal weight
+    // per CTA (a tile weighs PADOC_TC_WEIGHT_2M for a group of two M-tiles and PADOC_TC_WEIGHT_1M
+    // for one: the one-M-tile chain cannot overlap its softmax with another M-tile's MMAs); a range
+    // becomes the pieces where it overlaps segments.
+    struct Segment { int32_t g, p, first, ns, vis, ntiles, weight; };
+    std::vector<Segment> segs;
+    for (int32_t g = 0; g < cfg->num_kv_heads; ++g)
         for (int32_t p = 0; p < num_pages; ++p) {
             const int32_t f0 = pp.page_first_stream[p], ns = pp.page_num_streams[p];
-            int32_t vis = 0;
-            for (int32_t s = f0; s < f0 + ns; ++s) vis = std::max(vis, pp.streams[s].shared_len);
-            const bool use_tc = (int64_t)ns * group >= PADOC_TC_MIN_ROWS;
-            for (int32_t j = 0; j < page_splits[p]; ++j) {
-                const int32_t tb = j * split, te = std::min(vis, tb + split);
-                if (use_tc) {
-                    for (int32_t r = 0; r < ns; r += PADOC_TC_ITEM_STREAMS)
-                        tc_items.push_back({PADOC_ITEM_SHARED_TC, p, g, tb, te, f0 + r,
-                                            std::min(PADOC_TC_ITEM_STREAMS, ns - r), j});
-                } else {
-                    for (int32_t s = f0; s < f0 + ns; ++s) {
-                        const int32_t tes = std::min(te, pp.streams[s].shared_len);
-                        if (tes <= tb) {
-                            // nothing of this split is visible to the stream: an empty partial
-                            warp_items.push_back({PADOC_ITEM_SHARED, p, g, tb, tb, s, 1, j});
-                        } else {
-                            warp_items.push_back({PADOC_ITEM_SHARED, p, g, tb, tes, s, 1, j});
-                        }
-                    }
-                }
+            if ((int64_t)ns * group < PADOC_TC_MIN_ROWS) continue;
+            for (int32_t r = 0; r < ns; r += PADOC_TC_ITEM_STREAMS) {
+                const int32_t nb = std::min(PADOC_TC_ITEM_STREAMS, ns - r);
+                int32_t vis = 0;
+                for (int32_t st = f0 + r; st < f0 + r + nb; ++st) vis = std::max(vis, pp.streams[st].shared_len);
+                if (vis <= 0) continue;
+                segs.push_back({g, p, f0 + r, nb, vis, (vis + PADOC_TC_TILE_TOKENS - 1) / PADOC_TC_TILE_TOKENS,
+                                nb > PADOC_TC_ITEM_STREAMS / 2 ? PADOC_TC_WEIGHT_2M : PADOC_TC_WEIGHT_1M});
             }
         }
-        for (int32_t s = 0; s < S; ++s) {
-            const int32_t np = page_splits[pp.streams[s].page];
-            const int32_t L = pp.streams[s].private_len;
-            for (int32_t tb = 0, i = 0; tb < L; tb += psplit, ++i)
-                warp_items.push_back({PADOC_ITEM_PRIVATE, s, g, tb, std::min(L, tb + psplit), s, 1, np + i});
+    const int32_t Hkv = cfg->num_kv_heads;
+    std::vector<int32_t> cnt((size_t)S * Hkv, 0);   // partial slots handed out per (stream, KV head)
+    std::vector<padoc_item> tc_items;
+    int64_t total_w = 0;
+    for (const Segment &sg : segs) total_w += (int64_t)sg.ntiles * sg.weight;
+    int32_t ctas = 0;
+    if (total_w > 0) {
+        int32_t want = cfg->tc_ctas > 0 ? cfg->tc_ctas : padoc_default_ctas();
+        int64_t total_tiles = 0;
+        for (const Segment &sg : segs) total_tiles += sg.ntiles;
+        ctas = (int32_t)std::min<int64_t>(want, total_tiles);
+        pp.cta_ptr.assign((size_t)ctas + 1, 0);
+        // tile t of segment k starts at weight position W_k + t * w_k; it goes to the CTA whose
+        // range [c W / ctas, (c+1) W / ctas) holds that position
+        int64_t wpos = 0;
+        int32_t cur_cta = 0;
+        for (const Segment &sg : segs) {
+            int32_t t = 0;
+            while (t < sg.ntiles) {
+                while (cur_cta + 1 < ctas && wpos >= (int64_t)(cur_cta + 1) * total_w / ctas) {
+                    ++cur_cta;
+                    pp.cta_ptr[cur_cta] = (int32_t)tc_items.size();
+                }
+                const int64_t end_w = (int64_t)(cur_cta + 1) * total_w / ctas;
+                int32_t t1 = t;
+                while (t1 < sg.ntiles && (cur_cta + 1 == ctas || wpos + (int64_t)(t1 - t) * sg.weight < end_w)) ++t1;
+                if (t1 == t) t1 = t + 1;
+                const int32_t tb = t * PADOC_TC_TILE_TOKENS, te = std::min(sg.vis, t1 * PADOC_TC_TILE_TOKENS);
+                const int32_t slot = cnt[(size_t)sg.first * Hkv + sg.g];
+                for (int32_t st = sg.first; st < sg.first + sg.ns; ++st) ++cnt[(size_t)st * Hkv + sg.g];
+                tc_items.push_back({PADOC_ITEM_SHARED_TC, sg.p, sg.g, tb, te, sg.first, sg.ns, slot});
+                wpos += (int64_t)(t1 - t) * sg.weight;
+                t = t1;
+            }
+        }
+        for (int32_t c = cur_cta + 1; c <= ctas; ++c) pp.cta_ptr[c] = (int32_t)tc_items.size();
+    }
+    pp.tc_ctas = ctas;
+
+    // ---- warp work: shared streams of sparse pages (per stream) and every private history ------
+    std::vector<padoc_item> warp_items;
+    for (int32_t g = 0; g < Hkv; ++g) {
+        for (int32_t p = 0; p < num_pages; ++p) {
+            const int32_t f0 = pp.page_first_stream[p], ns = pp.page_num_streams[p];
+            if ((int64_t)ns * group >= PADOC_TC_MIN_ROWS) continue;
+            for (int32_t st = f0; st < f0 + ns; ++st)
+                for (int32_t tb = 0; tb < pp.streams[st].shared_len; tb += split)
+                    warp_items.push_back({PADOC_ITEM_SHARED, p, g, tb, std::min(pp.streams[st].shared_len, tb + split),
+                                          st, 1, cnt[(size_t)st * Hkv + g]++});
+        }
+        for (int32_t st = 0; st < S; ++st) {
+            const int32_t L = pp.streams[st].private_len;
+            for (int32_t tb = 0; tb < L; tb += psplit)
+                warp_items.push_back({PADOC_ITEM_PRIVATE, st, g, tb, std::min(L, tb + psplit), st, 1,
+                                      cnt[(size_t)st * Hkv + g]++});
         }
     }
-    // longest items first (LPT order) within each kernel's list, ties by position for determinism
-    auto longer = [](const padoc_item &a, const padoc_item &b) {
-        return (int64_t)(a.tok_end - a.tok_begin) * (a.num_streams + 15) > (int64_t)(b.tok_end - b.tok_begin) * (b.num_streams + 15);
-    };
-    std::stable_sort(tc_items.begin(), tc_items.end(), longer);
-    std::stable_sort(warp_items.begin(), warp_items.end(), longer);
+    // longest warp items first (LPT order), ties by position for determinism
+    std::stable_sort(warp_items.begin(), warp_items.end(), [](const padoc_item &a, const padoc_item &b) {
+        return a.tok_end - a.tok_begin > b.tok_end - b.tok_begin;
+    });
+    // a (stream, KV head) with nothing visible at all still gets one (empty) partial
+    for (int32_t st = 0; st < S; ++st)
+        for (int32_t g = 0; g < Hkv; ++g)
+            if (cnt[(size_t)st * Hkv + g] == 0) {
+                warp_items.push_back({PADOC_ITEM_SHARED, pp.streams[st].page, g, 0, 0, st, 1, 0});
+                cnt[(size_t)st * Hkv + g] = 1;
+            }
+    pp.slot_ptr.assign((size_t)S * Hkv + 1, 0);
+    for (size_t i = 0; i < (size_t)S * Hkv; ++i) pp.slot_ptr[i + 1] = pp.slot_ptr[i] + cnt[i];
     pp.num_tc_items = (int32_t)tc_items.size();
     pp.items = tc_items;
     pp.items.insert(pp.items.end(), warp_items.begin(), warp_items.end());
     return PADOC_OK;
+}
+
+// int32 words of the plan blob: stream_page, shared_len, private_len [S], slot_ptr [S Hkv + 1],
+// items [num_items][8], page_len [num_pages], cta_ptr [tc_ctas + 1]
+int64_t blob_ints(const PlanParts &pp, int32_t num_pages, int32_t hkv)
+{
+    const int64_t S = (int64_t)pp.streams.size();
+    return 3 * S + (S * hkv + 1) + (int64_t)pp.items.size() * PADOC_ITEM_INTS + num_pages + (int64_t)pp.cta_ptr.size();
 }
 
 }  // namespace
@@ -303,8 +360,7 @@ extern "C" padoc_status padoc_decode_plan_size(const padoc_page *pages, int32_t 
     PlanParts pp;
     padoc_status st = build_parts(pages, num_pages, cfg, pp);
     if (st != PADOC_OK) return st;
-    const int64_t S = (int64_t)pp.streams.size();
-    *plan_ints = 3 * S + (S + 1) + (int64_t)pp.items.size() * PADOC_ITEM_INTS + num_pages;
+    *plan_ints = blob_ints(pp, num_pages, cfg->num_kv_heads);
     return PADOC_OK;
 }
 
@@ -317,7 +373,7 @@ extern "C" padoc_status padoc_build_decode_plan(const padoc_page *pages, int32_t
     padoc_status st = build_parts(pages, num_pages, cfg, pp);
     if (st != PADOC_OK) return st;
     const int64_t S = (int64_t)pp.streams.size();
-    const int64_t need = 3 * S + (S + 1) + (int64_t)pp.items.size() * PADOC_ITEM_INTS + num_pages;
+    const int64_t need = blob_ints(pp, num_pages, cfg->num_kv_heads);
     if (capacity_ints < need) return PADOC_ERR_CAPACITY;
     if (need > 0 && !plan) return PADOC_ERR_INVALID_ARGUMENT;
     std::memset(info, 0, sizeof(*info));
@@ -326,34 +382,38 @@ extern "C" padoc_status padoc_build_decode_plan(const padoc_page *pages, int32_t
     info->num_streams = (int32_t)S;
     info->num_items = (int32_t)pp.items.size();
     info->num_tc_items = pp.num_tc_items;
+    info->tc_ctas = pp.tc_ctas;
     info->num_slots = pp.slot_ptr.back();
     info->max_page_blocks = pp.max_page_blocks;
     info->max_stream_blocks = pp.max_stream_blocks;
-    for (int64_t st = 0; st < S; ++st)
-        info->max_stream_slots = std::max<int32_t>(info->max_stream_slots, pp.slot_ptr[st + 1] - pp.slot_ptr[st]);
+    for (size_t i = 0; i + 1 < pp.slot_ptr.size(); ++i)
+        info->max_stream_slots = std::max<int32_t>(info->max_stream_slots, pp.slot_ptr[i + 1] - pp.slot_ptr[i]);
     info->plan_ints = need;
     info->kv_tokens = pp.kv_tokens;
     int64_t o = 0;
     info->off_stream_page = o; o += S;
     info->off_shared_len = o; o += S;
     info->off_private_len = o; o += S;
-    info->off_slot_ptr = o; o += S + 1;
+    info->off_slot_ptr = o; o += (int64_t)pp.slot_ptr.size();
     info->off_items = o; o += (int64_t)pp.items.size() * PADOC_ITEM_INTS;
     info->off_page_len = o; o += num_pages;
+    info->off_cta_ptr = o; o += (int64_t)pp.cta_ptr.size();
     for (int64_t s = 0; s < S; ++s) {
         plan[info->off_stream_page + s] = pp.streams[s].page;
         plan[info->off_shared_len + s] = pp.streams[s].shared_len;
         plan[info->off_private_len + s] = pp.streams[s].private_len;
     }
-    for (int64_t s = 0; s <= S; ++s) plan[info->off_slot_ptr + s] = pp.slot_ptr[s];
+    std::memcpy(plan + info->off_slot_ptr, pp.slot_ptr.data(), pp.slot_ptr.size() * sizeof(int32_t));
     std::memcpy(plan + info->off_items, pp.items.data(), pp.items.size() * sizeof(padoc_item));
     for (int32_t p = 0; p < num_pages; ++p) plan[info->off_page_len + p] = pp.page_len[p];
+    if (!pp.cta_ptr.empty()) std::memcpy(plan + info->off_cta_ptr, pp.cta_ptr.data(), pp.cta_ptr.size() * sizeof(int32_t));
     return PADOC_OK;
 }
 
 extern "C" padoc_status padoc_decode_workspace_size(const padoc_decode_plan *info, size_t *bytes)
 {
     if (!info || !bytes) return PADOC_ERR_INVALID_ARGUMENT;
-    *bytes = padoc_decode_workspace_bytes(info->num_slots, info->cfg.num_q_heads, info->cfg.head_dim);
+    *bytes = padoc_decode_workspace_bytes(info->num_slots, info->cfg.num_q_heads / info->cfg.num_kv_heads,
+                                          info->cfg.head_dim);
     return PADOC_OK;
 }

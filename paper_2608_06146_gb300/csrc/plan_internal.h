@@ -17,29 +17,34 @@
 #define PADOC_TC_MIN_ROWS 64
 // Streams per tensor-core work item: two M = 128 tiles of 16 streams x 8 query heads.
 #define PADOC_TC_ITEM_STREAMS 32
-// Longest shared-stream piece of one tensor-core work item.
-#define PADOC_TC_MAX_ITEM_TOKENS 4096
+// Tokens per K/V tile of the tensor-core kernel, and the relative cost of one tile for a group of
+// more than 16 streams (two M-tiles) and of at most 16 (one M-tile), used to balance CTAs.
+#define PADOC_TC_TILE_TOKENS 128
+#define PADOC_TC_WEIGHT_2M 8
+#define PADOC_TC_WEIGHT_1M 7
 
 #define PADOC_ITEM_INTS 8
 enum { PADOC_ITEM_SHARED = 0, PADOC_ITEM_PRIVATE = 1, PADOC_ITEM_SHARED_TC = 2 };
 
 // One split-K work item of the decode kernels (8 int32 words in the plan blob). The blob holds
-// the tensor-core items first ([0, num_tc_items)), then the warp items.
+// the tensor-core items first ([0, num_tc_items)), CTA c of the tensor-core grid owning items
+// [cta_ptr[c], cta_ptr[c+1]) in order, then the warp items.
 //   kind        PADOC_ITEM_SHARED_TC: tokens [tok_begin, tok_end) of page `index`'s shared stream for
 //               streams [first_stream, first_stream + num_streams) (<= 32) of that page, each with
 //               its own column cutoff shared_len (tensor-core kernel);
 //               PADOC_ITEM_SHARED: the same for the one stream first_stream (warp kernel);
 //               PADOC_ITEM_PRIVATE: private tokens [tok_begin, tok_end) of stream `index` (warp kernel).
 //   kv_head     the KV head; the item covers that head's Hq/Hkv query heads of every stream.
-//   slot        partial-result slot of each covered stream s: slot_ptr[s] + slot.
+//   slot        partial-result slot of each covered stream s: slot_ptr[s * Hkv + kv_head] + slot.
 typedef struct {
     int32_t kind, index, kv_head, tok_begin, tok_end, first_stream, num_streams, slot;
 } padoc_item;
 
 static inline size_t padoc_align256(size_t x) { return (x + 255) & ~(size_t)255; }
 
-// Workspace: part_o fp32 [slots][Hq][d], then part_lse fp32 [slots][Hq] at a 256-byte boundary.
-static inline size_t padoc_decode_workspace_bytes(int64_t slots, int32_t hq, int32_t d)
+// Workspace: part_o fp32 [slots][group][d], then part_lse fp32 [slots][group] at a 256-byte
+// boundary; a slot holds one partial of the group = Hq / Hkv query heads of one (stream, KV head).
+static inline size_t padoc_decode_workspace_bytes(int64_t slots, int32_t group, int32_t d)
 {
-    return padoc_align256((size_t)slots * hq * d * 4) + padoc_align256((size_t)slots * hq * 4);
+    return padoc_align256((size_t)slots * group * d * 4) + padoc_align256((size_t)slots * group * 4);
 }

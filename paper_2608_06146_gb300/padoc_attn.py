@@ -45,17 +45,19 @@ class padoc_kv_pool(ctypes.Structure):
 
 class padoc_decode_config(ctypes.Structure):
     _fields_ = [("num_q_heads", ctypes.c_int32), ("num_kv_heads", ctypes.c_int32), ("head_dim", ctypes.c_int32),
-                ("block_size", ctypes.c_int32), ("layout_streams", ctypes.c_int32), ("split_tokens", ctypes.c_int32)]
+                ("block_size", ctypes.c_int32), ("layout_streams", ctypes.c_int32), ("split_tokens", ctypes.c_int32),
+                ("tc_ctas", ctypes.c_int32)]
 
 
 class padoc_decode_plan(ctypes.Structure):
     _fields_ = [("cfg", padoc_decode_config), ("num_pages", ctypes.c_int32), ("num_streams", ctypes.c_int32),
-                ("num_items", ctypes.c_int32), ("num_tc_items", ctypes.c_int32), ("num_slots", ctypes.c_int32),
+                ("num_items", ctypes.c_int32), ("num_tc_items", ctypes.c_int32), ("tc_ctas", ctypes.c_int32),
+                ("num_slots", ctypes.c_int32),
                 ("max_page_blocks", ctypes.c_int32), ("max_stream_blocks", ctypes.c_int32),
                 ("max_stream_slots", ctypes.c_int32),
                 ("plan_ints", ctypes.c_int64), ("off_stream_page", ctypes.c_int64), ("off_shared_len", ctypes.c_int64),
                 ("off_private_len", ctypes.c_int64), ("off_slot_ptr", ctypes.c_int64), ("off_items", ctypes.c_int64),
-                ("off_page_len", ctypes.c_int64), ("kv_tokens", ctypes.c_int64)]
+                ("off_page_len", ctypes.c_int64), ("off_cta_ptr", ctypes.c_int64), ("kv_tokens", ctypes.c_int64)]
 
 
 _lib = None
@@ -232,8 +234,10 @@ def padoc_build_tile_map(pages, q_tile: int, k_tile: int):
 # Decode
 # ------------------------------------------------------------------------------------------------
 
-def make_decode_config(num_q_heads, num_kv_heads, head_dim, block_size=16, layout_streams=False, split_tokens=0):
-    return padoc_decode_config(num_q_heads, num_kv_heads, head_dim, block_size, int(bool(layout_streams)), split_tokens)
+def make_decode_config(num_q_heads, num_kv_heads, head_dim, block_size=16, layout_streams=False, split_tokens=0,
+                       tc_ctas=0):
+    return padoc_decode_config(num_q_heads, num_kv_heads, head_dim, block_size, int(bool(layout_streams)), split_tokens,
+                               tc_ctas)
 
 
 def padoc_decode_plan_size(pages, cfg: padoc_decode_config) -> int:
@@ -287,13 +291,13 @@ def padoc_branch_decode_attn(k_pool, v_pool, info: padoc_decode_plan, plan_dev, 
     _check("padoc_branch_decode_attn", st)
 
 
-PADOC_STATIC_WORKSPACE_BYTES = 16 << 20
+PADOC_STATIC_WORKSPACE_BYTES = 32 << 20
 
 
 def padoc_branch_decode_attn_noalloc(k_pool, v_pool, info: padoc_decode_plan, plan_dev, page_table, stream_table, q,
                                      scale, out, lse, stream=None):
     """padoc_branch_decode_attn for callers that cannot allocate device memory: the split-K partials
-    go to the library's fixed 16 MiB device array (shared by every call; serialize calls)."""
+    go to the library's fixed 32 MiB device array (shared by every call; serialize calls)."""
     lib = load_library()
     pool = padoc_kv_pool(_dev(k_pool, "k_pool"), _dev(v_pool, "v_pool"), k_pool.shape[0], k_pool.shape[2],
                          k_pool.shape[1], k_pool.shape[3], _dtype_code(k_pool))

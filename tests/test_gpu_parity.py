@@ -34,10 +34,10 @@ def _tols(dtype):
     return (BF16_O_TOL, BF16_LSE_TOL) if dtype == torch.bfloat16 else (F32_TOL, F32_TOL)
 
 
-def run_decode(wl: Workload, seed: int, layout_streams=False, split_tokens=0, scale_in=1.0):
+def run_decode(wl: Workload, seed: int, layout_streams=False, split_tokens=0, scale_in=1.0, tc_ctas=0):
     di = inputs.decode_inputs(wl, seed, layout_streams=layout_streams, scale=scale_in)
     plan = DecodePlan(wl.pages, wl.num_q_heads, wl.num_kv_heads, wl.head_dim, DEV, wl.block_size, layout_streams,
-                      split_tokens)
+                      split_tokens, tc_ctas)
     S = plan.num_streams
     q = di.q.to(DEV)
     out = torch.full((S, wl.num_q_heads, wl.head_dim), float("nan"), dtype=wl.dtype, device=DEV)
@@ -115,6 +115,21 @@ def test_decode_bf16_tensor_core_edge_pages():
     wl = Workload("tc edge", pages, 16, 2, 128, torch.bfloat16, "decode")
     assert_close(*run_decode(wl, 9, layout_streams=True), torch.bfloat16)
     assert_close(*run_decode(wl, 10, split_tokens=128), torch.bfloat16)
+
+
+@pytest.mark.parametrize("tc_ctas", [1, 3, 7, 40, 1000])
+def test_decode_bf16_tensor_core_ctas_walk_many_pieces(tc_ctas):
+    # few CTAs: each walks many pieces of different pages, KV heads and M-tile counts back to back
+    # (the K/V ring, barrier phases and query reloads carry across pieces); many CTAs: one-tile
+    # pieces and CTAs with empty ranges
+    rng = np.random.default_rng(11)
+    pages = []
+    for n in [40, 9, 17, 33, 12, 64, 8]:
+        P, L = int(rng.integers(1, 1500)), 8 * n
+        pages.append(PageSpec(P, L, [int(x) for x in rng.integers(0, L + 1, size=n)],
+                              [int(x) for x in rng.integers(1, 200, size=n)]))
+    wl = Workload("tc walk", pages, 16, 2, 128, torch.bfloat16, "decode")
+    assert_close(*run_decode(wl, 12, layout_streams=bool(tc_ctas & 1), tc_ctas=tc_ctas), torch.bfloat16)
 
 
 def test_decode_bad_block_id_reports_device_error():

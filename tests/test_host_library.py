@@ -122,11 +122,13 @@ def _plan_items(plan, info):
     return items
 
 
+@pytest.mark.parametrize("tc_ctas", [0, 1, 7, 5000])
 @pytest.mark.parametrize("wl_name,layout", [("decode_page", False), ("dense_page", False), ("serving_batch", True),
                                             ("serving_batch", False), ("tiny", False)])
-def test_decode_plan_covers_every_visible_token_once(wl_name, layout):
+def test_decode_plan_covers_every_visible_token_once(wl_name, layout, tc_ctas):
     wl = inputs.WORKLOADS[wl_name]()
-    cfg = pa.make_decode_config(wl.num_q_heads, wl.num_kv_heads, wl.head_dim, 16, layout, 0)
+    Hkv = wl.num_kv_heads
+    cfg = pa.make_decode_config(wl.num_q_heads, Hkv, wl.head_dim, 16, layout, 0, tc_ctas)
     plan, info = pa.padoc_build_decode_plan(wl.pages, cfg)
     sp, sh, pl = inputs.decode_streams(wl, layout)
     S = len(sp)
@@ -134,23 +136,21 @@ def test_decode_plan_covers_every_visible_token_once(wl_name, layout):
     np.testing.assert_array_equal(plan[info.off_stream_page: info.off_stream_page + S], sp)
     np.testing.assert_array_equal(plan[info.off_shared_len: info.off_shared_len + S], sh)
     np.testing.assert_array_equal(plan[info.off_private_len: info.off_private_len + S], pl)
-    slot_ptr = plan[info.off_slot_ptr: info.off_slot_ptr + S + 1]
+    slot_ptr = plan[info.off_slot_ptr: info.off_slot_ptr + S * Hkv + 1]
     assert slot_ptr[0] == 0 and slot_ptr[-1] == info.num_slots and np.all(np.diff(slot_ptr) >= 1)
+    assert info.max_stream_slots == np.diff(slot_ptr).max()
     items = _plan_items(plan, info)
     # coverage[(stream, kv_head)] counts how often each visible token is read
-    cov_sh = {(s, g): np.zeros(sh[s], np.int32) for s in range(S) for g in range(wl.num_kv_heads)}
-    cov_pv = {(s, g): np.zeros(pl[s], np.int32) for s in range(S) for g in range(wl.num_kv_heads)}
-    slots_used = {(s, g): [] for s in range(S) for g in range(wl.num_kv_heads)}
-    page_first = {}
-    for s in range(S):
-        page_first.setdefault(int(sp[s]), s)
+    cov_sh = {(s, g): np.zeros(sh[s], np.int32) for s in range(S) for g in range(Hkv)}
+    cov_pv = {(s, g): np.zeros(pl[s], np.int32) for s in range(S) for g in range(Hkv)}
+    slots_used = {(s, g): [] for s in range(S) for g in range(Hkv)}
     ntc = info.num_tc_items
     assert all(items[:ntc, 0] == 2) and not any(items[ntc:, 0] == 2)
     page_streams = np.bincount(sp, minlength=len(wl.pages))
     for kind, idx, g, tb, te, fs, ns, slot in items:
         assert tb % 16 == 0
-        if kind == 2:      # tensor-core item: up to 32 streams of a page with >= 64 rows
-            assert 1 <= ns <= 32 and te > tb and page_streams[idx] * 8 >= 64
+        if kind == 2:      # tensor-core piece: whole 128-token tiles of up to 32 streams of a page
+            assert 1 <= ns <= 32 and te > tb and page_streams[idx] * 8 >= 64 and tb % 128 == 0
         elif kind == 0:    # warp item over one stream's view of the shared stream
             assert ns == 1 and te >= tb and page_streams[idx] * 8 < 64
         else:
@@ -167,15 +167,28 @@ def test_decode_plan_covers_every_visible_token_once(wl_name, layout):
             slots_used[(s, g)].append(slot)
     for key in cov_sh:
         assert np.all(cov_sh[key] == 1) and np.all(cov_pv[key] == 1)
-        s = key[0]
-        assert sorted(slots_used[key]) == list(range(slot_ptr[s + 1] - slot_ptr[s]))
+        s, g = key
+        assert sorted(slots_used[key]) == list(range(slot_ptr[s * Hkv + g + 1] - slot_ptr[s * Hkv + g]))
+    # the tensor-core CTAs own consecutive item ranges covering every tensor-core item once
+    if ntc:
+        cta = plan[info.off_cta_ptr: info.off_cta_ptr + info.tc_ctas + 1]
+        assert cta[0] == 0 and cta[-1] == ntc and np.all(np.diff(cta) >= 0)
+        assert info.tc_ctas == min(tc_ctas or 152, sum(-(-(te - tb) // 128) for k, _, _, tb, te, *_ in items[:ntc]))
+        # balance: each CTA's work is within one tile of the mean
+        wts = [8 if ns > 16 else 7 for *_, ns, _ in items[:ntc]]
+        work = [sum(-(-(items[u, 4] - items[u, 3]) // 128) * wts[u] for u in range(cta[c], cta[c + 1]))
+                for c in range(info.tc_ctas)]
+        assert max(work) - min(work) <= 2 * 8
+    else:
+        assert info.tc_ctas == 0
     need = pa.padoc_decode_workspace_size(info)
-    assert need >= info.num_slots * wl.num_q_heads * (wl.head_dim + 1) * 4
+    assert need >= info.num_slots * (wl.num_q_heads // Hkv) * (wl.head_dim + 1) * 4
 
 
 def test_decode_plan_rejects_bad_config():
     wl = inputs.decode_page()
-    for cfg in [pa.make_decode_config(16, 3, 128), pa.make_decode_config(16, 2, 128, split_tokens=100)]:
+    for cfg in [pa.make_decode_config(16, 3, 128), pa.make_decode_config(16, 2, 128, split_tokens=100),
+                pa.make_decode_config(16, 2, 128, tc_ctas=-1)]:
         with pytest.raises(pa.PadocError):
             pa.padoc_build_decode_plan(wl.pages, cfg)
     with pytest.raises(pa.PadocError) as e:
