@@ -148,7 +148,8 @@ def bench_decode(args, torch, dev, rank, world):
     wl = inputs.serving_batch(seed=3 + 1000 * rank)
     scale = 1.0 / math.sqrt(wl.head_dim)
     di = inputs.decode_inputs(wl, 3 + 1000 * rank, pool_slack=1.0)
-    plan = DecodePlan(wl.pages, wl.num_q_heads, wl.num_kv_heads, wl.head_dim, dev, tc_ctas=args.tc_ctas)
+    plan = DecodePlan(wl.pages, wl.num_q_heads, wl.num_kv_heads, wl.head_dim, dev, tc_ctas=args.tc_ctas,
+                      warp_ctas=args.warp_ctas)
     S = plan.num_streams
     per_replica = (di.k_pool.numel() + di.v_pool.numel()) * 2
     R = args.replicas if args.replicas > 0 else max(2, math.ceil(4 * l2_bytes(torch) / per_replica) + 1)
@@ -184,7 +185,7 @@ def bench_decode(args, torch, dev, rank, world):
     sp, sh, pl = inputs.decode_streams(wl)
     nbytes = decode_bytes(wl, sp, sh, pl)
     info = plan.info
-    launches = (1 if info.num_tc_items > 0 else 0) + (1 if info.num_items > info.num_tc_items else 0) + 1
+    launches = (1 if info.num_tc_items > 0 else 0) + (1 if info.num_warps > 0 else 0) + 1   # + the merge
     res = dict(ms=ms, streams=S, bytes=nbytes, launches=launches, clocks=clk.summary(), replicas=R,
                pages=len(wl.pages), e2e_ms=None, h2d=0, d2h=0)
     if args.no_e2e:
@@ -374,6 +375,7 @@ def main():
     ap.add_argument("--replicas", type=int, default=0, help="decode input replicas (0: enough to exceed 4x L2)")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--tc-ctas", type=int, default=0, help="tensor-core decode CTAs (0: one per SM)")
+    ap.add_argument("--warp-ctas", type=int, default=0, help="warp-kernel decode CTAs (0: one per SM)")
     args = ap.parse_args()
     if args.impl == "reference":
         return run_reference(args)

@@ -148,10 +148,13 @@ typedef struct {
     int32_t layout_streams;  /* 1: also decode each page's layout stream (Alg. 1 decodes every live
                                 stream): cutoff P + L over the shared stream, no private rows */
     int32_t split_tokens;    /* shared-stream tokens per split-K partial of the warp kernel (pages with
-                                too few streams for the tensor cores); 0 = library default;
-                                a positive value must be a multiple of block_size */
+                                too few streams for the tensor cores); 0 = library default (512);
+                                a positive value must be a multiple of block_size; values above
+                                512 act as 512 */
     int32_t tc_ctas;         /* CTAs the tensor-core shared-stream work is balanced over (one range of
                                 equal work each); 0 = the current device's multiprocessor count */
+    int32_t warp_ctas;       /* CTAs (of 8 warps) the warp-kernel work is balanced over, one wave;
+                                0 = the current device's multiprocessor count */
 } padoc_decode_config;
 
 /* Host summary of a decode plan, filled by padoc_build_decode_plan. The int32 plan blob it
@@ -165,6 +168,7 @@ typedef struct {
     int32_t num_items;         /* work items of the split-K decode kernels */
     int32_t num_tc_items;      /* of which use the tensor-core shared-stream kernel */
     int32_t tc_ctas;           /* CTAs of the tensor-core kernel (0 when num_tc_items is 0) */
+    int32_t num_warps;         /* warps of the warp kernel (at most one per warp item) */
     int32_t num_slots;         /* split-K partial results, each for one (stream, KV head) */
     int32_t max_page_blocks;   /* page block-table width the plan needs */
     int32_t max_stream_blocks; /* stream block-table width the plan needs */
@@ -177,6 +181,7 @@ typedef struct {
     int64_t off_items;
     int64_t off_page_len;
     int64_t off_cta_ptr;
+    int64_t off_warp_ptr;
     int64_t kv_tokens;         /* algorithmic KV tokens read: each page's stream once + all private */
 } padoc_decode_plan;
 

@@ -30,18 +30,21 @@ namespace {
 constexpr int kD = 128;          // head_dim of the bf16 path
 constexpr int kGroup = 8;        // query heads per KV head of the bf16 path
 constexpr int kBlk = 16;         // tokens per paged block
-constexpr int kWarps = 8;              // warps (independent work items) per CTA
+constexpr int kWarps = PADOC_WARP_KERNEL_WARPS;   // independent warps per CTA
 constexpr int kWStages = 3;            // paged blocks in flight per warp
 constexpr int kBoxBytes = kBlk * 128;  // one 16-row x 64-column box
 constexpr int kWStageBytes = 4 * kBoxBytes;   // K lo, K hi, V lo, V hi
-constexpr int kWarpSmem = kWStages * kWStageBytes;
-constexpr size_t kDecodeSmem = 1024 + (size_t)kWarps * kWarpSmem;
+constexpr int kWarpRing = kWStages * kWStageBytes;
 constexpr int kMergeStride = 132;      // floats per head row when a warp stages its O^T
+constexpr int kWarpStage = kGroup * kMergeStride * 4;   // a warp's O^T staging buffer
+constexpr size_t kDecodeSmem = 1024 + (size_t)kWarps * (kWarpRing + kWarpStage);
 
 struct DecodeParams {
     const int32_t *stream_page, *shared_len, *private_len, *slot_ptr;
     const padoc_item *items;
-    int32_t first_item, num_items;
+    int32_t first_item;          // warp items start here
+    const int32_t *warp_ptr;     // warp w owns warp items [warp_ptr[w], warp_ptr[w+1])
+    int32_t num_warps;
     const int32_t *page_table;
     const int32_t *stream_table;
     int32_t page_stride, stream_stride;
@@ -68,27 +71,59 @@ decode_warp_kernel(const DecodeParams prm)
     uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int wi = blockIdx.x * kWarps + warp;
-    if (wi >= prm.num_items) { finish_warp(prm); return; }   // warps are independent: no CTA barrier follows
-    uint8_t *wbuf = smem + (size_t)warp * kWarpSmem;
-    const padoc_item it = prm.items[prm.first_item + wi];
-    const bool is_shared = it.kind == PADOC_ITEM_SHARED;
-    const int g = it.kv_head;
-    const int s = it.first_stream;
-    const int32_t *table = is_shared ? prm.page_table + (size_t)it.index * prm.page_stride
-                                     : prm.stream_table + (size_t)s * prm.stream_stride;
-    const int cutoff = min(is_shared ? prm.shared_len[s] : prm.private_len[s], it.tok_end);
-    const int blk0 = it.tok_begin / kBlk;
-    const int nblk = cutoff > it.tok_begin ? (cutoff - it.tok_begin + kBlk - 1) / kBlk : 0;
+    if (wi >= prm.num_warps) { finish_warp(prm); return; }   // warps are independent: no CTA barrier follows
+    uint8_t *wbuf = smem + (size_t)warp * kWarpRing;
+    float *st = reinterpret_cast<float *>(smem + (size_t)kWarps * kWarpRing + (size_t)warp * kWarpStage);   // [8][132]
+    const padoc_item *items = prm.items + prm.first_item;
+    const int i0 = prm.warp_ptr[wi], i1 = prm.warp_ptr[wi + 1];
+    // Every global read the loop depends on is issued at least one item ahead: item headers two
+    // items ahead, block ids (one per lane) and query fragments one item ahead, so a warp never
+    // waits on a load between two paged blocks.
+    auto load_item = [&](int u) { return items[u]; };   // 4-byte loads: the blob has no 16-byte alignment
+    struct Walk {   // what the producer needs of an item
+        const int32_t *table;
+        int blk0, nblk, g;
+    };
+    auto walk_of = [&](const padoc_item &it) {
+        Walk w;
+        w.table = it.kind == PADOC_ITEM_SHARED ? prm.page_table + (size_t)it.index * prm.page_stride
+                                               : prm.stream_table + (size_t)it.first_stream * prm.stream_stride;
+        w.blk0 = it.tok_begin / kBlk;
+        w.nblk = it.tok_end > it.tok_begin ? (it.tok_end - it.tok_begin + kBlk - 1) / kBlk : 0;
+        w.g = it.kv_head;
+        return w;
+    };
+    auto ids_of = [&](const Walk &w) { return lane < w.nblk ? w.table[w.blk0 + lane] : 0; };
 
-    // block bi into stage bi % kWStages: chunk q = lane + 32k of the block's 512 16-byte chunks is
-    // panel q / 128 (K lo, K hi, V lo, V hi), row (q / 8) % 16, 16-byte column q % 8 (swizzled)
-    auto issue = [&](int bi) {   // whole warp; always commits a group, possibly empty
-        if (bi < nblk) {
-            const int32_t id = table[blk0 + bi];
+    // The warp walks its items with one ring of kWStages paged blocks that runs on from one item
+    // into the next. Producer: the next block to fetch is block pb of item pu (walk pc, ids ids_c);
+    // item pu + 1 (walk pn, ids ids_n) and the header of item pu + 2 (hn2) are already on the way.
+    int pu = i0, pb = 0;
+    Walk pc{prm.page_table, 0, 0, 0}, pn{prm.page_table, 0, 0, 0};
+    int32_t ids_c = 0, ids_n = 0;
+    padoc_item hn2 = {};
+    if (i0 < i1) { pc = walk_of(load_item(i0)); ids_c = ids_of(pc); }
+    if (i0 + 1 < i1) { pn = walk_of(load_item(i0 + 1)); ids_n = ids_of(pn); }
+    if (i0 + 2 < i1) hn2 = load_item(i0 + 2);
+    int ring = 0;   // blocks issued so far: block n goes to stage n % kWStages
+    // chunk q = lane + 32k of a block's 512 16-byte chunks is panel q / 128 (K lo, K hi, V lo, V hi),
+    // row (q / 8) % 16, 16-byte column q % 8 (swizzled)
+    auto issue_next = [&]() {   // whole warp; always commits a group, possibly empty
+        while (pu < i1 && pb >= pc.nblk) {
+            ++pu;
+            pb = 0;
+            pc = pn;
+            ids_c = ids_n;
+            if (pu + 1 < i1) { pn = walk_of(hn2); ids_n = ids_of(pn); }
+            if (pu + 2 < i1) hn2 = load_item(pu + 2);
+        }
+        if (pu < i1) {
+            // block ids past the 32 a warp holds are read directly (the planner keeps items shorter)
+            const int32_t id = pb < 32 ? __shfl_sync(0xffffffffu, ids_c, pb) : pc.table[pc.blk0 + pb];
             const bool okid = id >= 0 && id < prm.num_blocks;
             if (!okid && lane == 0) padoc_record_error(prm.err, PADOC_DEVERR_BLOCK_ID, id);
-            const size_t rowbase = okid ? ((size_t)id * prm.num_kv_heads + g) * kBlk : 0;
-            const uint32_t base = smem_u32(wbuf + (bi % kWStages) * kWStageBytes);
+            const size_t rowbase = okid ? ((size_t)id * prm.num_kv_heads + pc.g) * kBlk : 0;
+            const uint32_t base = smem_u32(wbuf + (ring % kWStages) * kWStageBytes);
 #pragma unroll
             for (int k = 0; k < 16; ++k) {
                 const int q = lane + 32 * k;
@@ -97,113 +132,138 @@ decode_warp_kernel(const DecodeParams prm)
                                            (rowbase + r) * kD + (panel & 1) * 64 + cc * 8;
                 cp_async_16(base + panel * kBoxBytes + r * 128 + ((cc ^ (r & 7)) << 4), src, okid ? 16u : 0u);
             }
+            ++pb;
+            ++ring;
         }
         cp_async_commit();
     };
-    for (int bi = 0; bi < kWStages; ++bi) issue(bi);
+    for (int k = 0; k < kWStages; ++k) issue_next();
 
-    // query fragments: B operand Q^T[128 dims x 8 heads]
-    uint32_t qb[8][2];
-    {
-        const __nv_bfloat16 *qrow = prm.q + ((size_t)s * prm.num_q_heads + g * kGroup + (lane >> 2)) * kD;
+    // Consumer: header of the next item (ch_n) and of the one after (ch_n2), and the next item's
+    // query fragments (B operand Q^T[128 dims x 8 heads]) and first partial row.
+    padoc_item ch_n = {}, ch_n2 = {};
+    uint32_t qn[8][2];
+    size_t row_n = 0;
+    auto load_q = [&](const padoc_item &it) {
+        const __nv_bfloat16 *qrow =
+            prm.q + ((size_t)it.first_stream * prm.num_q_heads + it.kv_head * kGroup + (lane >> 2)) * kD;
 #pragma unroll
         for (int ks = 0; ks < 8; ++ks) {
-            qb[ks][0] = *reinterpret_cast<const uint32_t *>(qrow + ks * 16 + (lane & 3) * 2);
-            qb[ks][1] = *reinterpret_cast<const uint32_t *>(qrow + ks * 16 + 8 + (lane & 3) * 2);
+            qn[ks][0] = *reinterpret_cast<const uint32_t *>(qrow + ks * 16 + (lane & 3) * 2);
+            qn[ks][1] = *reinterpret_cast<const uint32_t *>(qrow + ks * 16 + 8 + (lane & 3) * 2);
         }
-    }
-    float m[2] = {-INFINITY, -INFINITY}, l[2] = {0.f, 0.f};   // heads h0 = 2*(lane%4), h0+1
-    float o[8][4];
+        row_n = (size_t)(prm.slot_ptr[(size_t)it.first_stream * prm.num_kv_heads + it.kv_head] + it.slot) * kGroup;
+    };
+    if (i0 < i1) { ch_n = load_item(i0); load_q(ch_n); }
+    if (i0 + 1 < i1) ch_n2 = load_item(i0 + 1);
+    int gc = 0;   // blocks consumed so far
+    for (int cu = i0; cu < i1; ++cu) {
+        const padoc_item it = ch_n;
+        uint32_t qb[8][2];
 #pragma unroll
-    for (int mt = 0; mt < 8; ++mt) o[mt][0] = o[mt][1] = o[mt][2] = o[mt][3] = 0.f;
+        for (int ks = 0; ks < 8; ++ks) { qb[ks][0] = qn[ks][0]; qb[ks][1] = qn[ks][1]; }
+        const size_t row0 = row_n;
+        if (cu + 1 < i1) {
+            ch_n = ch_n2;
+            load_q(ch_n);
+            if (cu + 2 < i1) ch_n2 = load_item(cu + 2);
+        }
+        const int cutoff = it.tok_end;   // the planner keeps warp items inside their stream's cutoff
+        const int blk0 = it.tok_begin / kBlk;
+        const int nblk = cutoff > it.tok_begin ? (cutoff - it.tok_begin + kBlk - 1) / kBlk : 0;
+        float m[2] = {-INFINITY, -INFINITY}, l[2] = {0.f, 0.f};   // heads h0 = 2*(lane%4), h0+1
+        float o[8][4];
+#pragma unroll
+        for (int mt = 0; mt < 8; ++mt) o[mt][0] = o[mt][1] = o[mt][2] = o[mt][3] = 0.f;
 
-    for (int bi = 0; bi < nblk; ++bi) {
-        cp_async_wait<kWStages - 1>();   // block bi has landed (one group per block)
-        __syncwarp();
-        const uint32_t base = smem_u32(wbuf + (bi % kWStages) * kWStageBytes);
-        const int tokbase = (blk0 + bi) * kBlk;
-        // S^T = K . Q^T
-        float acc[4] = {0.f, 0.f, 0.f, 0.f};
+        for (int bi = 0; bi < nblk; ++bi, ++gc) {
+            cp_async_wait<kWStages - 1>();   // block gc has landed (one group per block)
+            __syncwarp();
+            const uint32_t base = smem_u32(wbuf + (gc % kWStages) * kWStageBytes);
+            const int tokbase = (blk0 + bi) * kBlk;
+            // S^T = K . Q^T
+            float acc[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-        for (int ks = 0; ks < 8; ++ks) {
-            const uint32_t row = lane & 15;
-            const uint32_t col = (ks & 3) * 16 + (lane >> 4) * 8;
-            uint32_t a[4];
-            ldmatrix_x4(a, base + (ks >> 2) * kBoxBytes + sw128_offset(row, col));
-            mma_bf16_16816(acc, a, qb[ks][0], qb[ks][1]);
+            for (int ks = 0; ks < 8; ++ks) {
+                const uint32_t row = lane & 15;
+                const uint32_t col = (ks & 3) * 16 + (lane >> 4) * 8;
+                uint32_t a[4];
+                ldmatrix_x4(a, base + (ks >> 2) * kBoxBytes + sw128_offset(row, col));
+                mma_bf16_16816(acc, a, qb[ks][0], qb[ks][1]);
+            }
+            const int t0 = tokbase + (lane >> 2), t1 = t0 + 8;
+            float sc[4];
+            sc[0] = t0 < cutoff ? acc[0] * prm.scale_log2 : -INFINITY;
+            sc[1] = t0 < cutoff ? acc[1] * prm.scale_log2 : -INFINITY;
+            sc[2] = t1 < cutoff ? acc[2] * prm.scale_log2 : -INFINITY;
+            sc[3] = t1 < cutoff ? acc[3] * prm.scale_log2 : -INFINITY;
+            float mx0 = fmaxf(sc[0], sc[2]), mx1 = fmaxf(sc[1], sc[3]);
+#pragma unroll
+            for (int sh = 4; sh < 32; sh <<= 1) {
+                mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, sh));
+                mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, sh));
+            }
+            const float mn0 = fmaxf(m[0], mx0), mn1 = fmaxf(m[1], mx1);
+            // a head whose columns are all masked so far keeps m = -inf and contributes 0
+            const float al0 = mn0 == -INFINITY ? 1.f : fast_exp2(m[0] - mn0);
+            const float al1 = mn1 == -INFINITY ? 1.f : fast_exp2(m[1] - mn1);
+            const float r0 = mn0 == -INFINITY ? 0.f : mn0, r1 = mn1 == -INFINITY ? 0.f : mn1;
+            const float p0 = fast_exp2(sc[0] - r0), p1 = fast_exp2(sc[1] - r1);
+            const float p2 = fast_exp2(sc[2] - r0), p3 = fast_exp2(sc[3] - r1);
+            m[0] = mn0; m[1] = mn1;
+            l[0] = l[0] * al0 + p0 + p2;
+            l[1] = l[1] * al1 + p1 + p3;
+            const uint32_t b0 = movmatrix_trans(pack_bf16x2(p0, p1));
+            const uint32_t b1 = movmatrix_trans(pack_bf16x2(p2, p3));
+#pragma unroll
+            for (int mt = 0; mt < 8; ++mt) {
+                o[mt][0] *= al0; o[mt][1] *= al1; o[mt][2] *= al0; o[mt][3] *= al1;
+                const int i = lane >> 3;
+                const uint32_t row = (lane & 7) + (i >= 2 ? 8 : 0);
+                const uint32_t col = (mt & 3) * 16 + (i & 1) * 8;
+                uint32_t a[4];
+                ldmatrix_x4_trans(a, base + (2 + (mt >> 2)) * kBoxBytes + sw128_offset(row, col));
+                mma_bf16_16816(o[mt], a, b0, b1);
+            }
+            __syncwarp();   // every lane is done with the stage before it is refilled
+            issue_next();
         }
-        const int t0 = tokbase + (lane >> 2), t1 = t0 + 8;
-        float sc[4];
-        sc[0] = t0 < cutoff ? acc[0] * prm.scale_log2 : -INFINITY;
-        sc[1] = t0 < cutoff ? acc[1] * prm.scale_log2 : -INFINITY;
-        sc[2] = t1 < cutoff ? acc[2] * prm.scale_log2 : -INFINITY;
-        sc[3] = t1 < cutoff ? acc[3] * prm.scale_log2 : -INFINITY;
-        float mx0 = fmaxf(sc[0], sc[2]), mx1 = fmaxf(sc[1], sc[3]);
+        // complete the row sums over the 8 token lanes of each head
 #pragma unroll
         for (int sh = 4; sh < 32; sh <<= 1) {
-            mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, sh));
-            mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, sh));
+            l[0] += __shfl_xor_sync(0xffffffffu, l[0], sh);
+            l[1] += __shfl_xor_sync(0xffffffffu, l[1], sh);
         }
-        const float mn0 = fmaxf(m[0], mx0), mn1 = fmaxf(m[1], mx1);
-        // a head whose columns are all masked so far keeps m = -inf and contributes 0
-        const float al0 = mn0 == -INFINITY ? 1.f : fast_exp2(m[0] - mn0);
-        const float al1 = mn1 == -INFINITY ? 1.f : fast_exp2(m[1] - mn1);
-        const float r0 = mn0 == -INFINITY ? 0.f : mn0, r1 = mn1 == -INFINITY ? 0.f : mn1;
-        const float p0 = fast_exp2(sc[0] - r0), p1 = fast_exp2(sc[1] - r1);
-        const float p2 = fast_exp2(sc[2] - r0), p3 = fast_exp2(sc[3] - r1);
-        m[0] = mn0; m[1] = mn1;
-        l[0] = l[0] * al0 + p0 + p2;
-        l[1] = l[1] * al1 + p1 + p3;
-        const uint32_t b0 = movmatrix_trans(pack_bf16x2(p0, p1));
-        const uint32_t b1 = movmatrix_trans(pack_bf16x2(p2, p3));
+        // stage O^T and write the partial with 16-byte stores
+        {
+            const int h0 = (lane & 3) * 2;
+            const float i0f = l[0] > 0.f ? 1.f / l[0] : 0.f, i1f = l[1] > 0.f ? 1.f / l[1] : 0.f;
 #pragma unroll
-        for (int mt = 0; mt < 8; ++mt) {
-            o[mt][0] *= al0; o[mt][1] *= al1; o[mt][2] *= al0; o[mt][3] *= al1;
-            const int i = lane >> 3;
-            const uint32_t row = (lane & 7) + (i >= 2 ? 8 : 0);
-            const uint32_t col = (mt & 3) * 16 + (i & 1) * 8;
-            uint32_t a[4];
-            ldmatrix_x4_trans(a, base + (2 + (mt >> 2)) * kBoxBytes + sw128_offset(row, col));
-            mma_bf16_16816(o[mt], a, b0, b1);
+            for (int mt = 0; mt < 8; ++mt) {
+                const int d0 = mt * 16 + (lane >> 2);
+                st[h0 * kMergeStride + d0] = o[mt][0] * i0f;
+                st[(h0 + 1) * kMergeStride + d0] = o[mt][1] * i1f;
+                st[h0 * kMergeStride + d0 + 8] = o[mt][2] * i0f;
+                st[(h0 + 1) * kMergeStride + d0 + 8] = o[mt][3] * i1f;
+            }
         }
-        __syncwarp();   // every lane is done with the stage before it is refilled
-        issue(bi + kWStages);
+        __syncwarp();
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+            const int idx = k * 32 + lane;          // float4 index over [8 heads][32 float4]
+            const int hl = idx >> 5, d4 = idx & 31;
+            const float *src = st + hl * kMergeStride + d4 * 4;
+            *reinterpret_cast<float4 *>(prm.part_o + (row0 + hl) * kD + d4 * 4) =
+                make_float4(src[0], src[1], src[2], src[3]);
+        }
+        if (lane < 4) {
+            const int h0 = lane * 2;
+            prm.part_lse[row0 + h0] = l[0] > 0.f ? (m[0] + log2f(l[0])) * PADOC_LN2 : -INFINITY;
+            prm.part_lse[row0 + h0 + 1] = l[1] > 0.f ? (m[1] + log2f(l[1])) * PADOC_LN2 : -INFINITY;
+        }
+        __syncwarp();   // the staging buffer is read before the next item overwrites it
     }
     cp_async_wait<0>();
-    // complete the row sums over the 8 token lanes of each head
-#pragma unroll
-    for (int sh = 4; sh < 32; sh <<= 1) {
-        l[0] += __shfl_xor_sync(0xffffffffu, l[0], sh);
-        l[1] += __shfl_xor_sync(0xffffffffu, l[1], sh);
-    }
-    // stage O^T through this warp's (now idle) ring and write the partial with 16-byte stores
-    float *st = reinterpret_cast<float *>(wbuf);   // [8 heads][132]
-    {
-        const int h0 = (lane & 3) * 2;
-        const float i0 = l[0] > 0.f ? 1.f / l[0] : 0.f, i1 = l[1] > 0.f ? 1.f / l[1] : 0.f;
-#pragma unroll
-        for (int mt = 0; mt < 8; ++mt) {
-            const int d0 = mt * 16 + (lane >> 2);
-            st[h0 * kMergeStride + d0] = o[mt][0] * i0;
-            st[(h0 + 1) * kMergeStride + d0] = o[mt][1] * i1;
-            st[h0 * kMergeStride + d0 + 8] = o[mt][2] * i0;
-            st[(h0 + 1) * kMergeStride + d0 + 8] = o[mt][3] * i1;
-        }
-    }
-    __syncwarp();
-    const size_t row0 = (size_t)(prm.slot_ptr[(size_t)s * prm.num_kv_heads + g] + it.slot) * kGroup;
-#pragma unroll
-    for (int k = 0; k < 8; ++k) {
-        const int idx = k * 32 + lane;          // float4 index over [8 heads][32 float4]
-        const int hl = idx >> 5, d4 = idx & 31;
-        const float *src = st + hl * kMergeStride + d4 * 4;
-        *reinterpret_cast<float4 *>(prm.part_o + (row0 + hl) * kD + d4 * 4) = make_float4(src[0], src[1], src[2], src[3]);
-    }
-    if (lane < 4) {
-        const int h0 = lane * 2;
-        prm.part_lse[row0 + h0] = l[0] > 0.f ? (m[0] + log2f(l[0])) * PADOC_LN2 : -INFINITY;
-        prm.part_lse[row0 + h0 + 1] = l[1] > 0.f ? (m[1] + log2f(l[1])) * PADOC_LN2 : -INFINITY;
-    }
     finish_warp(prm);
 }
 
@@ -489,7 +549,8 @@ extern "C" padoc_status padoc_branch_decode_attn(const padoc_kv_pool *pool, cons
     prm.slot_ptr = plan + info->off_slot_ptr;
     prm.items = reinterpret_cast<const padoc_item *>(plan + info->off_items);
     prm.first_item = info->num_tc_items;
-    prm.num_items = info->num_items - info->num_tc_items;
+    prm.warp_ptr = plan + info->off_warp_ptr;
+    prm.num_warps = info->num_warps;
     prm.page_table = page_block_table;
     prm.stream_table = stream_block_table;
     prm.page_stride = page_table_stride;
@@ -506,10 +567,10 @@ extern "C" padoc_status padoc_branch_decode_attn(const padoc_kv_pool *pool, cons
     prm.scale_log2 = sl2;
     prm.err = err;
     prm.after_tc = info->num_tc_items > 0 ? 1 : 0;
-    if (prm.num_items > 0) {
+    if (prm.num_warps > 0) {
         PADOC_CUDA_TRY(cudaFuncSetAttribute(decode_warp_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kDecodeSmem));
         cudaLaunchConfig_t lc = {};
-        lc.gridDim = dim3((unsigned)((prm.num_items + kWarps - 1) / kWarps));
+        lc.gridDim = dim3((unsigned)((prm.num_warps + kWarps - 1) / kWarps));
         lc.blockDim = dim3(kWarps * 32);
         lc.dynamicSmemBytes = kDecodeSmem;
         lc.stream = cs;

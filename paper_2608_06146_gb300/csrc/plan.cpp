@@ -8,6 +8,7 @@
 #include <cstdint>
 #include <cstring>
 #include <numeric>
+#include <queue>
 #include <vector>
 
 #include <cuda_runtime.h>
@@ -196,8 +197,9 @@ struct PlanParts {
     std::vector<int32_t> page_len, page_first_stream, page_num_streams;
     std::vector<int32_t> slot_ptr;      // [S * Hkv + 1]: partial slots of each (stream, KV head)
     std::vector<int32_t> cta_ptr;       // [tc_ctas + 1]: tensor-core items of each CTA
+    std::vector<int32_t> warp_ptr;      // [num_warps + 1]: warp items of each warp (from the first)
     std::vector<padoc_item> items;
-    int32_t num_tc_items = 0, tc_ctas = 0;
+    int32_t num_tc_items = 0, tc_ctas = 0, num_warps = 0;
     int32_t max_page_blocks = 0, max_stream_blocks = 0;
     int64_t kv_tokens = 0;
 };
@@ -213,8 +215,9 @@ padoc_status build_parts(const padoc_page *pages, int32_t num_pages, const padoc
     if (cfg->split_tokens < 0 || (cfg->split_tokens > 0 && cfg->split_tokens % cfg->block_size != 0))
         return PADOC_ERR_INVALID_ARGUMENT;
     const int32_t bs = cfg->block_size;
-    if (cfg->tc_ctas < 0) return PADOC_ERR_INVALID_ARGUMENT;
-    const int32_t split = cfg->split_tokens > 0 ? cfg->split_tokens : PADOC_DEFAULT_SPLIT_TOKENS;
+    if (cfg->tc_ctas < 0 || cfg->warp_ctas < 0) return PADOC_ERR_INVALID_ARGUMENT;
+    const int32_t split = std::min(cfg->split_tokens > 0 ? cfg->split_tokens : PADOC_DEFAULT_SPLIT_TOKENS,
+                                   PADOC_WARP_MAX_ITEM_TOKENS);
     const int32_t psplit = PADOC_PRIVATE_SPLIT_TOKENS;
     const int32_t group = cfg->num_q_heads / cfg->num_kv_heads;
 
@@ -337,18 +340,62 @@ padoc_status build_parts(const padoc_page *pages, int32_t num_pages, const padoc
             }
     pp.slot_ptr.assign((size_t)S * Hkv + 1, 0);
     for (size_t i = 0; i < (size_t)S * Hkv; ++i) pp.slot_ptr[i + 1] = pp.slot_ptr[i] + cnt[i];
+
+    // the warp grid runs as one wave: items go to CTAs, longest item to the least loaded CTA (an
+    // SM's warps share its memory bandwidth, so CTA totals are what must match), then within each
+    // CTA to its warps the same way (cost: 16-token blocks plus a fixed start-up cost per item)
+    using Load = std::pair<int64_t, int32_t>;   // (cost so far, bin)
+    using MinHeap = std::priority_queue<Load, std::vector<Load>, std::greater<Load>>;
+    auto item_cost = [](const padoc_item &it) {
+        return (int64_t)(it.tok_end - it.tok_begin + 15) / 16 + PADOC_WARP_ITEM_COST;
+    };
+    const int64_t nitems = (int64_t)warp_items.size();
+    const int32_t wctas = (int32_t)std::min<int64_t>(cfg->warp_ctas > 0 ? cfg->warp_ctas : padoc_default_ctas(),
+                                                     (nitems + PADOC_WARP_KERNEL_WARPS - 1) / PADOC_WARP_KERNEL_WARPS);
+    const int32_t nwarps = (int32_t)std::min<int64_t>((int64_t)wctas * PADOC_WARP_KERNEL_WARPS, nitems);
+    std::vector<std::vector<int32_t>> lists((size_t)nwarps);
+    if (nwarps > 0) {
+        std::vector<std::vector<int32_t>> per_cta((size_t)wctas);
+        MinHeap heap;
+        for (int32_t c = 0; c < wctas; ++c) heap.push({0, c});
+        for (int32_t i = 0; i < (int32_t)nitems; ++i) {   // warp_items are in LPT order
+            Load top = heap.top();
+            heap.pop();
+            per_cta[(size_t)top.second].push_back(i);
+            heap.push({top.first + item_cost(warp_items[(size_t)i]), top.second});
+        }
+        for (int32_t c = 0; c < wctas; ++c) {
+            const int32_t w0 = c * PADOC_WARP_KERNEL_WARPS;
+            const int32_t nw = std::min<int32_t>(PADOC_WARP_KERNEL_WARPS, nwarps - w0);
+            if (nw <= 0) break;
+            MinHeap wheap;
+            for (int32_t w = 0; w < nw; ++w) wheap.push({0, w0 + w});
+            for (int32_t i : per_cta[(size_t)c]) {
+                Load top = wheap.top();
+                wheap.pop();
+                lists[(size_t)top.second].push_back(i);
+                wheap.push({top.first + item_cost(warp_items[(size_t)i]), top.second});
+            }
+        }
+    }
+    pp.warp_ptr.assign((size_t)nwarps + 1, 0);
     pp.num_tc_items = (int32_t)tc_items.size();
     pp.items = tc_items;
-    pp.items.insert(pp.items.end(), warp_items.begin(), warp_items.end());
+    for (int32_t w = 0; w < nwarps; ++w) {
+        for (int32_t i : lists[(size_t)w]) pp.items.push_back(warp_items[(size_t)i]);
+        pp.warp_ptr[(size_t)w + 1] = (int32_t)(pp.items.size() - tc_items.size());
+    }
+    pp.num_warps = nwarps;
     return PADOC_OK;
 }
 
 // int32 words of the plan blob: stream_page, shared_len, private_len [S], slot_ptr [S Hkv + 1],
-// items [num_items][8], page_len [num_pages], cta_ptr [tc_ctas + 1]
+// items [num_items][8], page_len [num_pages], cta_ptr [tc_ctas + 1], warp_ptr [num_warps + 1]
 int64_t blob_ints(const PlanParts &pp, int32_t num_pages, int32_t hkv)
 {
     const int64_t S = (int64_t)pp.streams.size();
-    return 3 * S + (S * hkv + 1) + (int64_t)pp.items.size() * PADOC_ITEM_INTS + num_pages + (int64_t)pp.cta_ptr.size();
+    return 3 * S + (S * hkv + 1) + (int64_t)pp.items.size() * PADOC_ITEM_INTS + num_pages + (int64_t)pp.cta_ptr.size() +
+           (int64_t)pp.warp_ptr.size();
 }
 
 }  // namespace
@@ -383,6 +430,7 @@ extern "C" padoc_status padoc_build_decode_plan(const padoc_page *pages, int32_t
     info->num_items = (int32_t)pp.items.size();
     info->num_tc_items = pp.num_tc_items;
     info->tc_ctas = pp.tc_ctas;
+    info->num_warps = pp.num_warps;
     info->num_slots = pp.slot_ptr.back();
     info->max_page_blocks = pp.max_page_blocks;
     info->max_stream_blocks = pp.max_stream_blocks;
@@ -398,6 +446,7 @@ extern "C" padoc_status padoc_build_decode_plan(const padoc_page *pages, int32_t
     info->off_items = o; o += (int64_t)pp.items.size() * PADOC_ITEM_INTS;
     info->off_page_len = o; o += num_pages;
     info->off_cta_ptr = o; o += (int64_t)pp.cta_ptr.size();
+    info->off_warp_ptr = o; o += (int64_t)pp.warp_ptr.size();
     for (int64_t s = 0; s < S; ++s) {
         plan[info->off_stream_page + s] = pp.streams[s].page;
         plan[info->off_shared_len + s] = pp.streams[s].shared_len;
@@ -407,6 +456,7 @@ extern "C" padoc_status padoc_build_decode_plan(const padoc_page *pages, int32_t
     std::memcpy(plan + info->off_items, pp.items.data(), pp.items.size() * sizeof(padoc_item));
     for (int32_t p = 0; p < num_pages; ++p) plan[info->off_page_len + p] = pp.page_len[p];
     if (!pp.cta_ptr.empty()) std::memcpy(plan + info->off_cta_ptr, pp.cta_ptr.data(), pp.cta_ptr.size() * sizeof(int32_t));
+    std::memcpy(plan + info->off_warp_ptr, pp.warp_ptr.data(), pp.warp_ptr.size() * sizeof(int32_t));
     return PADOC_OK;
 }
 

@@ -9,7 +9,9 @@
 #define PADOC_PREFILL_K_TILE 128
 
 // Decode split-K: shared-stream tokens per partial result and private tokens per partial result.
-#define PADOC_DEFAULT_SPLIT_TOKENS 1024
+#define PADOC_DEFAULT_SPLIT_TOKENS 512
+// Longest warp item: a warp keeps one block id per lane, so an item spans at most 32 blocks.
+#define PADOC_WARP_MAX_ITEM_TOKENS 512
 #define PADOC_PRIVATE_SPLIT_TOKENS 256
 // Shared-stream rows (streams x query heads of one KV head) from which the tensor-core kernel
 // takes a page: below this the rows are too few for a dense M = 128 contraction and each stream
@@ -23,12 +25,19 @@
 #define PADOC_TC_WEIGHT_2M 8
 #define PADOC_TC_WEIGHT_1M 7
 
+// Warps per CTA of the warp kernel, and the start-up cost of one warp item in 16-token blocks
+// (query fragments, the first blocks' latency, the partial's write), used to balance warps.
+#define PADOC_WARP_KERNEL_WARPS 8
+#define PADOC_WARP_ITEM_COST 2
+
 #define PADOC_ITEM_INTS 8
 enum { PADOC_ITEM_SHARED = 0, PADOC_ITEM_PRIVATE = 1, PADOC_ITEM_SHARED_TC = 2 };
 
 // One split-K work item of the decode kernels (8 int32 words in the plan blob). The blob holds
 // the tensor-core items first ([0, num_tc_items)), CTA c of the tensor-core grid owning items
-// [cta_ptr[c], cta_ptr[c+1]) in order, then the warp items.
+// [cta_ptr[c], cta_ptr[c+1]) in order, then the warp items, warp w of the warp grid owning
+// items num_tc_items + [warp_ptr[w], warp_ptr[w+1]) in order. A warp item's tok_end never passes
+// its stream's cutoff (shared_len or private_len), so the warp kernel reads no cutoff.
 //   kind        PADOC_ITEM_SHARED_TC: tokens [tok_begin, tok_end) of page `index`'s shared stream for
 //               streams [first_stream, first_stream + num_streams) (<= 32) of that page, each with
 //               its own column cutoff shared_len (tensor-core kernel);

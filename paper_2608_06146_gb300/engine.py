@@ -16,9 +16,9 @@ class DecodePlan:
     """Decode plan (C1) uploaded to the device, with its split-K workspace (C4)."""
 
     def __init__(self, pages, num_q_heads: int, num_kv_heads: int, head_dim: int, device, block_size: int = 16,
-                 layout_streams: bool = False, split_tokens: int = 0, tc_ctas: int = 0):
+                 layout_streams: bool = False, split_tokens: int = 0, tc_ctas: int = 0, warp_ctas: int = 0):
         self.cfg = pa.make_decode_config(num_q_heads, num_kv_heads, head_dim, block_size, layout_streams, split_tokens,
-                                         tc_ctas)
+                                         tc_ctas, warp_ctas)
         plan, self.info = pa.padoc_build_decode_plan(pages, self.cfg)
         self.plan_host = plan
         self.plan_dev = torch.from_numpy(plan.copy()).to(device)

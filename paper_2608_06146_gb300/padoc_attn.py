@@ -46,18 +46,20 @@ class padoc_kv_pool(ctypes.Structure):
 class padoc_decode_config(ctypes.Structure):
     _fields_ = [("num_q_heads", ctypes.c_int32), ("num_kv_heads", ctypes.c_int32), ("head_dim", ctypes.c_int32),
                 ("block_size", ctypes.c_int32), ("layout_streams", ctypes.c_int32), ("split_tokens", ctypes.c_int32),
-                ("tc_ctas", ctypes.c_int32)]
+                ("tc_ctas", ctypes.c_int32), ("warp_ctas", ctypes.c_int32)]
 
 
 class padoc_decode_plan(ctypes.Structure):
     _fields_ = [("cfg", padoc_decode_config), ("num_pages", ctypes.c_int32), ("num_streams", ctypes.c_int32),
                 ("num_items", ctypes.c_int32), ("num_tc_items", ctypes.c_int32), ("tc_ctas", ctypes.c_int32),
+                ("num_warps", ctypes.c_int32),
                 ("num_slots", ctypes.c_int32),
                 ("max_page_blocks", ctypes.c_int32), ("max_stream_blocks", ctypes.c_int32),
                 ("max_stream_slots", ctypes.c_int32),
                 ("plan_ints", ctypes.c_int64), ("off_stream_page", ctypes.c_int64), ("off_shared_len", ctypes.c_int64),
                 ("off_private_len", ctypes.c_int64), ("off_slot_ptr", ctypes.c_int64), ("off_items", ctypes.c_int64),
-                ("off_page_len", ctypes.c_int64), ("off_cta_ptr", ctypes.c_int64), ("kv_tokens", ctypes.c_int64)]
+                ("off_page_len", ctypes.c_int64), ("off_cta_ptr", ctypes.c_int64), ("off_warp_ptr", ctypes.c_int64),
+                ("kv_tokens", ctypes.c_int64)]
 
 
 _lib = None
@@ -235,9 +237,9 @@ def padoc_build_tile_map(pages, q_tile: int, k_tile: int):
 # ------------------------------------------------------------------------------------------------
 
 def make_decode_config(num_q_heads, num_kv_heads, head_dim, block_size=16, layout_streams=False, split_tokens=0,
-                       tc_ctas=0):
+                       tc_ctas=0, warp_ctas=0):
     return padoc_decode_config(num_q_heads, num_kv_heads, head_dim, block_size, int(bool(layout_streams)), split_tokens,
-                               tc_ctas)
+                               tc_ctas, warp_ctas)
 
 
 def padoc_decode_plan_size(pages, cfg: padoc_decode_config) -> int:

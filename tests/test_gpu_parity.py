@@ -34,10 +34,11 @@ def _tols(dtype):
     return (BF16_O_TOL, BF16_LSE_TOL) if dtype == torch.bfloat16 else (F32_TOL, F32_TOL)
 
 
-def run_decode(wl: Workload, seed: int, layout_streams=False, split_tokens=0, scale_in=1.0, tc_ctas=0):
+def run_decode(wl: Workload, seed: int, layout_streams=False, split_tokens=0, scale_in=1.0, tc_ctas=0,
+               warp_ctas=0):
     di = inputs.decode_inputs(wl, seed, layout_streams=layout_streams, scale=scale_in)
     plan = DecodePlan(wl.pages, wl.num_q_heads, wl.num_kv_heads, wl.head_dim, DEV, wl.block_size, layout_streams,
-                      split_tokens, tc_ctas)
+                      split_tokens, tc_ctas, warp_ctas)
     S = plan.num_streams
     q = di.q.to(DEV)
     out = torch.full((S, wl.num_q_heads, wl.head_dim), float("nan"), dtype=wl.dtype, device=DEV)
@@ -117,11 +118,12 @@ def test_decode_bf16_tensor_core_edge_pages():
     assert_close(*run_decode(wl, 10, split_tokens=128), torch.bfloat16)
 
 
-@pytest.mark.parametrize("tc_ctas", [1, 3, 7, 40, 1000])
-def test_decode_bf16_tensor_core_ctas_walk_many_pieces(tc_ctas):
+@pytest.mark.parametrize("tc_ctas,warp_ctas", [(1, 1), (3, 2), (7, 5), (40, 0), (1000, 1000)])
+def test_decode_bf16_tensor_core_ctas_walk_many_pieces(tc_ctas, warp_ctas):
     # few CTAs: each walks many pieces of different pages, KV heads and M-tile counts back to back
-    # (the K/V ring, barrier phases and query reloads carry across pieces); many CTAs: one-tile
-    # pieces and CTAs with empty ranges
+    # (the K/V ring, barrier phases and query reloads carry across pieces), and each warp of the
+    # warp kernel walks a long list of items with one cp.async ring; many CTAs: one-tile pieces,
+    # CTAs with empty ranges and one item per warp
     rng = np.random.default_rng(11)
     pages = []
     for n in [40, 9, 17, 33, 12, 64, 8]:
@@ -129,7 +131,26 @@ def test_decode_bf16_tensor_core_ctas_walk_many_pieces(tc_ctas):
         pages.append(PageSpec(P, L, [int(x) for x in rng.integers(0, L + 1, size=n)],
                               [int(x) for x in rng.integers(1, 200, size=n)]))
     wl = Workload("tc walk", pages, 16, 2, 128, torch.bfloat16, "decode")
-    assert_close(*run_decode(wl, 12, layout_streams=bool(tc_ctas & 1), tc_ctas=tc_ctas), torch.bfloat16)
+    assert_close(*run_decode(wl, 12, layout_streams=bool(tc_ctas & 1), tc_ctas=tc_ctas, warp_ctas=warp_ctas),
+                 torch.bfloat16)
+
+
+def test_decode_repeated_calls_on_one_workspace():
+    # one plan and workspace serve several calls with new inputs; each call is exact
+    wl = inputs.serving_batch(num_pages=6)
+    plan = DecodePlan(wl.pages, wl.num_q_heads, wl.num_kv_heads, wl.head_dim, DEV)
+    for seed in (31, 32, 33):
+        di = inputs.decode_inputs(wl, seed)
+        S = plan.num_streams
+        out = torch.full((S, 16, 128), float("nan"), dtype=torch.bfloat16, device=DEV)
+        lse = torch.full((S, 16), float("nan"), dtype=torch.float32, device=DEV)
+        scale = 1.0 / math.sqrt(wl.head_dim)
+        plan.run(di.k_pool.to(DEV), di.v_pool.to(DEV), torch.from_numpy(di.page_table).to(DEV),
+                 torch.from_numpy(di.stream_table).to(DEV), di.q.to(DEV), scale, out, lse)
+        pa.padoc_check_device_errors()
+        ref_o, ref_lse = oracle.decode(di.stream_page, di.shared_len, di.priv_len, di.page_off, di.priv_off,
+                                       di.stream_k, di.stream_v, di.priv_k, di.priv_v, di.q, scale)
+        assert_close(out.float().cpu().numpy(), lse.cpu().numpy(), ref_o, ref_lse, torch.bfloat16)
 
 
 def test_decode_bad_block_id_reports_device_error():

@@ -122,13 +122,13 @@ def _plan_items(plan, info):
     return items
 
 
-@pytest.mark.parametrize("tc_ctas", [0, 1, 7, 5000])
+@pytest.mark.parametrize("tc_ctas,warp_ctas", [(0, 0), (1, 1), (7, 3), (5000, 5000)])
 @pytest.mark.parametrize("wl_name,layout", [("decode_page", False), ("dense_page", False), ("serving_batch", True),
                                             ("serving_batch", False), ("tiny", False)])
-def test_decode_plan_covers_every_visible_token_once(wl_name, layout, tc_ctas):
+def test_decode_plan_covers_every_visible_token_once(wl_name, layout, tc_ctas, warp_ctas):
     wl = inputs.WORKLOADS[wl_name]()
     Hkv = wl.num_kv_heads
-    cfg = pa.make_decode_config(wl.num_q_heads, Hkv, wl.head_dim, 16, layout, 0, tc_ctas)
+    cfg = pa.make_decode_config(wl.num_q_heads, Hkv, wl.head_dim, 16, layout, 0, tc_ctas, warp_ctas)
     plan, info = pa.padoc_build_decode_plan(wl.pages, cfg)
     sp, sh, pl = inputs.decode_streams(wl, layout)
     S = len(sp)
@@ -181,6 +181,24 @@ def test_decode_plan_covers_every_visible_token_once(wl_name, layout, tc_ctas):
         assert max(work) - min(work) <= 2 * 8
     else:
         assert info.tc_ctas == 0
+    # the warp grid: warp lists cover the warp items in order, one wave, balanced by cost
+    nw_items = info.num_items - ntc
+    wp = plan[info.off_warp_ptr: info.off_warp_ptr + info.num_warps + 1]
+    wctas = min(warp_ctas or 152, -(-nw_items // 8))
+    assert info.num_warps == min(wctas * 8, nw_items)
+    assert wp[0] == 0 and wp[-1] == nw_items and np.all(np.diff(wp) >= 0)
+    cost = [-(-(te - tb) // 16) + 2 for _, _, _, tb, te, *_ in items[ntc:]]
+    loads = np.array([sum(cost[wp[w]:wp[w + 1]]) for w in range(info.num_warps)])
+    # CTA totals (LPT over CTAs) and the warps inside each CTA (LPT again) are balanced
+    cta_loads = [loads[c * 8:(c + 1) * 8].sum() for c in range(-(-info.num_warps // 8))]
+    assert max(cta_loads) - min(cta_loads) <= max(cost) or len(cta_loads) == 1
+    for c in range(len(cta_loads)):
+        wl_ = loads[c * 8:(c + 1) * 8]
+        if len(wl_) == 8 and wl_.min() > 0:
+            assert wl_.max() - wl_.min() <= max(cost)
+    # a warp item never reaches past its stream's cutoff (the warp kernel reads none)
+    for kind, idx, g, tb, te, fs, ns, slot in items[ntc:]:
+        assert te <= (sh[fs] if kind == 0 else pl[fs])
     need = pa.padoc_decode_workspace_size(info)
     assert need >= info.num_slots * (wl.num_q_heads // Hkv) * (wl.head_dim + 1) * 4
 
@@ -188,7 +206,7 @@ def test_decode_plan_covers_every_visible_token_once(wl_name, layout, tc_ctas):
 def test_decode_plan_rejects_bad_config():
     wl = inputs.decode_page()
     for cfg in [pa.make_decode_config(16, 3, 128), pa.make_decode_config(16, 2, 128, split_tokens=100),
-                pa.make_decode_config(16, 2, 128, tc_ctas=-1)]:
+                pa.make_decode_config(16, 2, 128, tc_ctas=-1), pa.make_decode_config(16, 2, 128, warp_ctas=-1)]:
         with pytest.raises(pa.PadocError):
             pa.padoc_build_decode_plan(wl.pages, cfg)
     with pytest.raises(pa.PadocError) as e:
