@@ -203,14 +203,20 @@ def bench_decode(args, torch, dev, rank, world):
     cfg = plan.cfg
     plan_dev = torch.empty(int(plan.info.plan_ints), dtype=torch.int32, device=dev)
 
-    blob_pinned = torch.empty(int(plan.info.plan_ints) + 4096, dtype=torch.int32).pin_memory()
-    blob_np = blob_pinned.numpy()
+    # two pinned plan buffers: the host builds step i+1's plan into one while step i's copy from the
+    # other may still be in flight (an event per buffer says when it may be overwritten)
+    blob_pinned = [torch.empty(int(plan.info.plan_ints) + 4096, dtype=torch.int32).pin_memory() for _ in range(2)]
+    blob_np = [b.numpy() for b in blob_pinned]
+    blob_free = [torch.cuda.Event(), torch.cuda.Event()]
 
     def e2e_step(i):
         r = i % R
-        blob, info = pa.padoc_build_decode_plan(wl.pages, cfg, out=blob_np)
-        blob_t = blob_pinned[: blob.size]
+        b = i & 1
+        blob_free[b].synchronize()
+        blob, info = pa.padoc_build_decode_plan(wl.pages, cfg, out=blob_np[b])
+        blob_t = blob_pinned[b][: blob.size]
         plan_dev[: blob.size].copy_(blob_t, non_blocking=True)
+        blob_free[b].record(stream)
         q_dev.copy_(q_host, non_blocking=True)
         pt_dev.copy_(pt_host, non_blocking=True)
         st_dev.copy_(st_host, non_blocking=True)

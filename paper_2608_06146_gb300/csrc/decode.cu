@@ -270,15 +270,6 @@ decode_warp_kernel(const DecodeParams prm)
 // ------------------------------------------------------------------------------------------------
 // Split-K merge (C4): one warp per output row, 4 consecutive dims per lane.
 // ------------------------------------------------------------------------------------------------
-struct RaggedSlots {   // decode: row = s * Hq + h = (s * Hkv + g) * group + hl; slots of (s, g)
-    const int32_t *slot_ptr;
-    int32_t group;
-    __device__ int count(int64_t row) const { return slot_ptr[row / group + 1] - slot_ptr[row / group]; }
-    __device__ int64_t part_row(int64_t row, int i) const
-    {
-        return (int64_t)(slot_ptr[row / group] + i) * group + row % group;
-    }
-};
 struct UniformSlots {  // public combine: part_row = split * rows + row
     int32_t splits;
     int64_t rows;
@@ -286,73 +277,55 @@ struct UniformSlots {  // public combine: part_row = split * rows + row
     __device__ int64_t part_row(int64_t row, int i) const { return (int64_t)i * rows + row; }
 };
 
-// Decode merge: one CTA per (stream, KV head), its 8 query heads x 16 threads, each thread 8 of
-// the 128 dims. The weights exp(lse_s - lse) of every (slot, head) are computed once into shared
-// memory, then every thread streams its dims of all partials with two partials' loads in flight.
-constexpr int kCombineMaxSlots = 64;
-
+// Decode merge: one CTA per (stream, KV head), its 8 query heads x 16 threads, each thread 8 of the
+// 128 dims. One pass over the slots with an online reference (the running max of lse_s): four
+// partials' LSE and O loads are in flight per thread at a time.
 __global__ void __launch_bounds__(128) decode_combine_kernel(const int32_t *__restrict__ slot_ptr,
                                                              const float *__restrict__ part_o,
                                                              const float *__restrict__ part_lse,
                                                              __nv_bfloat16 *__restrict__ out, float *__restrict__ lse_out)
 {
-    __shared__ float w_sh[kCombineMaxSlots][kGroup];
-    __shared__ float tot_sh[kGroup];
     const int key = blockIdx.x;                      // s * Hkv + g; output rows key * 8 + h
     const int tid = threadIdx.x;
-    const int p0 = slot_ptr[key], n = slot_ptr[key + 1] - p0;
     const int h = tid >> 4, part = tid & 15;         // head, 8-dim slice
-    if (n > kCombineMaxSlots) return;                // the host routes such plans elsewhere
-    // per head: max and log-sum-exp over slots (16 threads of the head cooperate)
-    float mx = -INFINITY;
-    for (int i = part; i < n; i += 16) mx = fmaxf(mx, part_lse[(size_t)(p0 + i) * kGroup + h]);
+    const int p0 = slot_ptr[key], n = slot_ptr[key + 1] - p0;
+    const float *bo = part_o + ((size_t)p0 * kGroup + h) * kD + part * 8;
+    const float *bl = part_lse + (size_t)p0 * kGroup + h;
+    constexpr size_t kSlotO = (size_t)kGroup * kD;
+    float mref = -INFINITY, ssum = 0.f;
+    float4 acc0 = make_float4(0.f, 0.f, 0.f, 0.f), acc1 = acc0;
+    for (int i = 0; i < n; i += 4) {
+        float li[4];
+        float4 v0[4], v1[4];
 #pragma unroll
-    for (int sh = 1; sh < 16; sh <<= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, sh));
-    float sum = 0.f;
-    if (mx != -INFINITY)
-        for (int i = part; i < n; i += 16) sum += expf(part_lse[(size_t)(p0 + i) * kGroup + h] - mx);
+        for (int u = 0; u < 4; ++u) {
+            const bool in = i + u < n;
+            li[u] = in ? bl[(size_t)(i + u) * kGroup] : -INFINITY;
+            v0[u] = in ? *reinterpret_cast<const float4 *>(bo + (i + u) * kSlotO) : make_float4(0.f, 0.f, 0.f, 0.f);
+            v1[u] = in ? *reinterpret_cast<const float4 *>(bo + (i + u) * kSlotO + 4) : make_float4(0.f, 0.f, 0.f, 0.f);
+        }
 #pragma unroll
-    for (int sh = 1; sh < 16; sh <<= 1) sum += __shfl_xor_sync(0xffffffffu, sum, sh);
-    const float tot = mx == -INFINITY ? -INFINITY : mx + logf(sum);
-    for (int i = part; i < n; i += 16)
-        w_sh[i][h] = tot == -INFINITY ? 0.f : expf(part_lse[(size_t)(p0 + i) * kGroup + h] - tot);
-    if (part == 0) tot_sh[h] = tot;
-    __syncthreads();
-    float4 acc[2];
-#pragma unroll
-    for (int c = 0; c < 2; ++c) acc[c] = make_float4(0.f, 0.f, 0.f, 0.f);
-    const float *base = part_o + ((size_t)p0 * kGroup + h) * kD + part * 8;
-    constexpr size_t slot_stride = (size_t)kGroup * kD;
-    int i = 0;
-    for (; i + 2 <= n; i += 2) {
-        float4 v[2][2];
-#pragma unroll
-        for (int u = 0; u < 2; ++u)
-#pragma unroll
-            for (int c = 0; c < 2; ++c) v[u][c] = *reinterpret_cast<const float4 *>(base + (i + u) * slot_stride + c * 4);
-#pragma unroll
-        for (int u = 0; u < 2; ++u) {
-            const float w = w_sh[i + u][h];
-#pragma unroll
-            for (int c = 0; c < 2; ++c) {
-                acc[c].x += w * v[u][c].x; acc[c].y += w * v[u][c].y; acc[c].z += w * v[u][c].z; acc[c].w += w * v[u][c].w;
+        for (int u = 0; u < 4; ++u) {
+            if (li[u] == -INFINITY) continue;   // an empty partial weighs nothing
+            if (li[u] > mref) {
+                const float a = mref == -INFINITY ? 0.f : expf(mref - li[u]);
+                ssum *= a;
+                acc0.x *= a; acc0.y *= a; acc0.z *= a; acc0.w *= a;
+                acc1.x *= a; acc1.y *= a; acc1.z *= a; acc1.w *= a;
+                mref = li[u];
             }
+            const float w = expf(li[u] - mref);
+            ssum += w;
+            acc0.x += w * v0[u].x; acc0.y += w * v0[u].y; acc0.z += w * v0[u].z; acc0.w += w * v0[u].w;
+            acc1.x += w * v1[u].x; acc1.y += w * v1[u].y; acc1.z += w * v1[u].z; acc1.w += w * v1[u].w;
         }
     }
-    for (; i < n; ++i) {
-        const float w = w_sh[i][h];
-#pragma unroll
-        for (int c = 0; c < 2; ++c) {
-            const float4 v = *reinterpret_cast<const float4 *>(base + i * slot_stride + c * 4);
-            acc[c].x += w * v.x; acc[c].y += w * v.y; acc[c].z += w * v.z; acc[c].w += w * v.w;
-        }
-    }
-    __nv_bfloat16 *o = out + ((size_t)key * kGroup + h) * kD + part * 8;
+    const float inv = ssum > 0.f ? 1.f / ssum : 0.f;
     uint4 pk;
-    pk.x = pack_bf16x2(acc[0].x, acc[0].y); pk.y = pack_bf16x2(acc[0].z, acc[0].w);
-    pk.z = pack_bf16x2(acc[1].x, acc[1].y); pk.w = pack_bf16x2(acc[1].z, acc[1].w);
-    *reinterpret_cast<uint4 *>(o) = pk;
-    if (part == 0) lse_out[(size_t)key * kGroup + h] = tot_sh[h];
+    pk.x = pack_bf16x2(acc0.x * inv, acc0.y * inv); pk.y = pack_bf16x2(acc0.z * inv, acc0.w * inv);
+    pk.z = pack_bf16x2(acc1.x * inv, acc1.y * inv); pk.w = pack_bf16x2(acc1.z * inv, acc1.w * inv);
+    *reinterpret_cast<uint4 *>(out + ((size_t)key * kGroup + h) * kD + part * 8) = pk;
+    if (part == 0) lse_out[(size_t)key * kGroup + h] = ssum > 0.f ? mref + logf(ssum) : -INFINITY;
 }
 
 template <class Slots, class OutT>
@@ -583,15 +556,8 @@ extern "C" padoc_status padoc_branch_decode_attn(const padoc_kv_pool *pool, cons
         st = padoc_launch_status();
         if (st != PADOC_OK) return st;
     }
-    const int64_t out_rows = (int64_t)info->num_streams * cfg.num_q_heads;
-    if (info->max_stream_slots <= kCombineMaxSlots) {
-        decode_combine_kernel<<<(unsigned)((int64_t)info->num_streams * cfg.num_kv_heads), 128, 0, cs>>>(
-            prm.slot_ptr, part_o, part_lse, (__nv_bfloat16 *)out, lse);
-    } else {
-        RaggedSlots sl{prm.slot_ptr, kGroup};
-        combine_kernel<RaggedSlots, __nv_bfloat16><<<(unsigned)((out_rows + 3) / 4), 128, 0, cs>>>(
-            sl, part_o, part_lse, out_rows, kD, (__nv_bfloat16 *)out, lse);
-    }
+    decode_combine_kernel<<<(unsigned)((int64_t)info->num_streams * cfg.num_kv_heads), 128, 0, cs>>>(
+        prm.slot_ptr, part_o, part_lse, (__nv_bfloat16 *)out, lse);
     return padoc_launch_status();
 }
 

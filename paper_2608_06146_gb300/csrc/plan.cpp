@@ -8,7 +8,6 @@
 #include <cstdint>
 #include <cstring>
 #include <numeric>
-#include <queue>
 #include <vector>
 
 #include <cuda_runtime.h>
@@ -327,10 +326,6 @@ padoc_status build_parts(const padoc_page *pages, int32_t num_pages, const padoc
                                       cnt[(size_t)st * Hkv + g]++});
         }
     }
-    // longest warp items first (LPT order), ties by position for determinism
-    std::stable_sort(warp_items.begin(), warp_items.end(), [](const padoc_item &a, const padoc_item &b) {
-        return a.tok_end - a.tok_begin > b.tok_end - b.tok_begin;
-    });
     // a (stream, KV head) with nothing visible at all still gets one (empty) partial
     for (int32_t st = 0; st < S; ++st)
         for (int32_t g = 0; g < Hkv; ++g)
@@ -341,49 +336,78 @@ padoc_status build_parts(const padoc_page *pages, int32_t num_pages, const padoc
     pp.slot_ptr.assign((size_t)S * Hkv + 1, 0);
     for (size_t i = 0; i < (size_t)S * Hkv; ++i) pp.slot_ptr[i + 1] = pp.slot_ptr[i] + cnt[i];
 
-    // the warp grid runs as one wave: items go to CTAs, longest item to the least loaded CTA (an
-    // SM's warps share its memory bandwidth, so CTA totals are what must match), then within each
-    // CTA to its warps the same way (cost: 16-token blocks plus a fixed start-up cost per item)
-    using Load = std::pair<int64_t, int32_t>;   // (cost so far, bin)
-    using MinHeap = std::priority_queue<Load, std::vector<Load>, std::greater<Load>>;
-    auto item_cost = [](const padoc_item &it) {
-        return (int64_t)(it.tok_end - it.tok_begin + 15) / 16 + PADOC_WARP_ITEM_COST;
-    };
-    const int64_t nitems = (int64_t)warp_items.size();
+    // The warp grid runs as one wave. Items are taken longest first (LPT; a counting sort on the
+    // block count keeps ties in plan order) and each goes to the least loaded CTA (an SM's warps
+    // share its memory bandwidth, so CTA totals are what must match), then within each CTA to its
+    // least loaded warp. Cost: 16-token blocks plus a fixed start-up cost per item.
+    const int32_t nitems = (int32_t)warp_items.size();
+    std::vector<int32_t> cost((size_t)nitems), order((size_t)nitems);
+    int32_t maxb = 0;
+    for (int32_t i = 0; i < nitems; ++i) {
+        const int32_t nb = (warp_items[(size_t)i].tok_end - warp_items[(size_t)i].tok_begin + 15) / 16;
+        cost[(size_t)i] = nb;
+        maxb = std::max(maxb, nb);
+    }
+    {
+        std::vector<int32_t> start((size_t)maxb + 2, 0);
+        for (int32_t i = 0; i < nitems; ++i) ++start[(size_t)(maxb - cost[(size_t)i]) + 1];
+        for (int32_t b = 0; b <= maxb; ++b) start[(size_t)b + 1] += start[(size_t)b];
+        for (int32_t i = 0; i < nitems; ++i) order[(size_t)start[(size_t)(maxb - cost[(size_t)i])]++] = i;
+    }
+    for (int32_t i = 0; i < nitems; ++i) cost[(size_t)i] += PADOC_WARP_ITEM_COST;
     const int32_t wctas = (int32_t)std::min<int64_t>(cfg->warp_ctas > 0 ? cfg->warp_ctas : padoc_default_ctas(),
-                                                     (nitems + PADOC_WARP_KERNEL_WARPS - 1) / PADOC_WARP_KERNEL_WARPS);
+                                                     ((int64_t)nitems + PADOC_WARP_KERNEL_WARPS - 1) / PADOC_WARP_KERNEL_WARPS);
     const int32_t nwarps = (int32_t)std::min<int64_t>((int64_t)wctas * PADOC_WARP_KERNEL_WARPS, nitems);
-    std::vector<std::vector<int32_t>> lists((size_t)nwarps);
+    pp.warp_ptr.assign((size_t)nwarps + 1, 0);
+    pp.num_tc_items = (int32_t)tc_items.size();
+    pp.items.resize(tc_items.size() + (size_t)nitems);
+    std::copy(tc_items.begin(), tc_items.end(), pp.items.begin());
     if (nwarps > 0) {
-        std::vector<std::vector<int32_t>> per_cta((size_t)wctas);
-        MinHeap heap;
-        for (int32_t c = 0; c < wctas; ++c) heap.push({0, c});
-        for (int32_t i = 0; i < (int32_t)nitems; ++i) {   // warp_items are in LPT order
-            Load top = heap.top();
-            heap.pop();
-            per_cta[(size_t)top.second].push_back(i);
-            heap.push({top.first + item_cost(warp_items[(size_t)i]), top.second});
+        // least loaded CTA: loads only grow and the minimum never falls, so CTAs sit in FIFO buckets
+        // by load and a cursor walks up to the lowest non-empty bucket (O(1) per item)
+        int64_t total = 0;
+        for (int32_t i = 0; i < nitems; ++i) total += cost[(size_t)i];
+        const int64_t nbuckets = total / wctas + maxb + PADOC_WARP_ITEM_COST + 2;
+        std::vector<int32_t> head((size_t)nbuckets, -1), tail((size_t)nbuckets, -1), next((size_t)wctas, -1);
+        auto push = [&](int64_t load, int32_t c) {
+            next[(size_t)c] = -1;
+            if (tail[(size_t)load] < 0) head[(size_t)load] = c; else next[(size_t)tail[(size_t)load]] = c;
+            tail[(size_t)load] = c;
+        };
+        for (int32_t c = 0; c < wctas; ++c) push(0, c);
+        std::vector<int32_t> cta_of((size_t)nitems), cstart((size_t)wctas + 1, 0);
+        int64_t cur = 0;
+        for (int32_t k : order) {
+            while (head[(size_t)cur] < 0) ++cur;
+            const int32_t c = head[(size_t)cur];
+            head[(size_t)cur] = next[(size_t)c];
+            if (head[(size_t)cur] < 0) tail[(size_t)cur] = -1;
+            cta_of[(size_t)k] = c;
+            ++cstart[(size_t)c + 1];
+            push(cur + cost[(size_t)k], c);
         }
+        for (int32_t c = 0; c < wctas; ++c) cstart[(size_t)c + 1] += cstart[(size_t)c];
+        std::vector<int32_t> by_cta((size_t)nitems), cpos(cstart.begin(), cstart.end() - 1);
+        for (int32_t k : order) by_cta[(size_t)cpos[(size_t)cta_of[(size_t)k]]++] = k;   // LPT order per CTA
+        std::vector<int32_t> warp_of((size_t)nitems);
         for (int32_t c = 0; c < wctas; ++c) {
             const int32_t w0 = c * PADOC_WARP_KERNEL_WARPS;
             const int32_t nw = std::min<int32_t>(PADOC_WARP_KERNEL_WARPS, nwarps - w0);
-            if (nw <= 0) break;
-            MinHeap wheap;
-            for (int32_t w = 0; w < nw; ++w) wheap.push({0, w0 + w});
-            for (int32_t i : per_cta[(size_t)c]) {
-                Load top = wheap.top();
-                wheap.pop();
-                lists[(size_t)top.second].push_back(i);
-                wheap.push({top.first + item_cost(warp_items[(size_t)i]), top.second});
+            int64_t load[PADOC_WARP_KERNEL_WARPS] = {0};
+            for (int32_t j = cstart[(size_t)c]; j < cstart[(size_t)c + 1]; ++j) {
+                const int32_t k = by_cta[(size_t)j];
+                int32_t best = 0;
+                for (int32_t w = 1; w < nw; ++w)
+                    if (load[w] < load[best]) best = w;
+                warp_of[(size_t)k] = w0 + best;
+                load[best] += cost[(size_t)k];
+                ++pp.warp_ptr[(size_t)(w0 + best) + 1];
             }
         }
-    }
-    pp.warp_ptr.assign((size_t)nwarps + 1, 0);
-    pp.num_tc_items = (int32_t)tc_items.size();
-    pp.items = tc_items;
-    for (int32_t w = 0; w < nwarps; ++w) {
-        for (int32_t i : lists[(size_t)w]) pp.items.push_back(warp_items[(size_t)i]);
-        pp.warp_ptr[(size_t)w + 1] = (int32_t)(pp.items.size() - tc_items.size());
+        for (int32_t w = 0; w < nwarps; ++w) pp.warp_ptr[(size_t)w + 1] += pp.warp_ptr[(size_t)w];
+        std::vector<int32_t> wpos(pp.warp_ptr.begin(), pp.warp_ptr.end() - 1);
+        padoc_item *dst = pp.items.data() + tc_items.size();
+        for (int32_t k : by_cta) dst[wpos[(size_t)warp_of[(size_t)k]]++] = warp_items[(size_t)k];
     }
     pp.num_warps = nwarps;
     return PADOC_OK;
