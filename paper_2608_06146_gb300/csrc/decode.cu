@@ -181,16 +181,18 @@ decode_warp_kernel(const DecodeParams prm)
             __syncwarp();
             const uint32_t base = smem_u32(wbuf + (gc % kWStages) * kWStageBytes);
             const int tokbase = (blk0 + bi) * kBlk;
-            // S^T = K . Q^T
-            float acc[4] = {0.f, 0.f, 0.f, 0.f};
+            // S^T = K . Q^T, as two independent MMA chains (even / odd k-steps) added at the end
+            float acc[4] = {0.f, 0.f, 0.f, 0.f}, acc2[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
             for (int ks = 0; ks < 8; ++ks) {
                 const uint32_t row = lane & 15;
                 const uint32_t col = (ks & 3) * 16 + (lane >> 4) * 8;
                 uint32_t a[4];
                 ldmatrix_x4(a, base + (ks >> 2) * kBoxBytes + sw128_offset(row, col));
-                mma_bf16_16816(acc, a, qb[ks][0], qb[ks][1]);
+                mma_bf16_16816((ks & 1) ? acc2 : acc, a, qb[ks][0], qb[ks][1]);
             }
+#pragma unroll
+            for (int i = 0; i < 4; ++i) acc[i] += acc2[i];
             const int t0 = tokbase + (lane >> 2), t1 = t0 + 8;
             float sc[4];
             sc[0] = t0 < cutoff ? acc[0] * prm.scale_log2 : -INFINITY;
@@ -215,9 +217,14 @@ decode_warp_kernel(const DecodeParams prm)
             l[1] = l[1] * al1 + p1 + p3;
             const uint32_t b0 = movmatrix_trans(pack_bf16x2(p0, p1));
             const uint32_t b1 = movmatrix_trans(pack_bf16x2(p2, p3));
+            if (__any_sync(0xffffffffu, al0 != 1.f || al1 != 1.f)) {   // a head's running max moved
+#pragma unroll
+                for (int mt = 0; mt < 8; ++mt) {
+                    o[mt][0] *= al0; o[mt][1] *= al1; o[mt][2] *= al0; o[mt][3] *= al1;
+                }
+            }
 #pragma unroll
             for (int mt = 0; mt < 8; ++mt) {
-                o[mt][0] *= al0; o[mt][1] *= al1; o[mt][2] *= al0; o[mt][3] *= al1;
                 const int i = lane >> 3;
                 const uint32_t row = (lane & 7) + (i >= 2 ? 8 : 0);
                 const uint32_t col = (mt & 3) * 16 + (i & 1) * 8;

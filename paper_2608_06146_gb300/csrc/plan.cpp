@@ -250,10 +250,9 @@ padoc_status build_parts(const padoc_page *pages, int32_t num_pages, const padoc
 
     // ---- tensor-core work: stream-K over the concatenated shared-stream tiles ----------------
     // A segment is one (KV head, page, group of <= 32 streams) with the tiles of the shared stream
-    // the group can see. The segments are laid end to end and cut into one range of equal weight
-    // per CTA (a tile weighs PADOC_TC_WEIGHT_2M for a group of two M-tiles and PADOC_TC_WEIGHT_1M
-    // for one: the one-M-tile chain cannot overlap its softmax with another M-tile's MMAs); a range
-    // becomes the pieces where it overlaps segments.
+    // the group can see. The segments are laid end to end and cut into one contiguous range per CTA
+    // (a tile weighs PADOC_TC_WEIGHT_2M for a group of two M-tiles and PADOC_TC_WEIGHT_1M for one);
+    // a range becomes the pieces where it overlaps segments.
     struct Segment { int32_t g, p, first, ns, vis, ntiles, weight; };
     std::vector<Segment> segs;
     for (int32_t g = 0; g < cfg->num_kv_heads; ++g)
@@ -272,39 +271,50 @@ padoc_status build_parts(const padoc_page *pages, int32_t num_pages, const padoc
     const int32_t Hkv = cfg->num_kv_heads;
     std::vector<int32_t> cnt((size_t)S * Hkv, 0);   // partial slots handed out per (stream, KV head)
     std::vector<padoc_item> tc_items;
-    int64_t total_w = 0;
-    for (const Segment &sg : segs) total_w += (int64_t)sg.ntiles * sg.weight;
-    int32_t ctas = 0;
-    if (total_w > 0) {
-        int32_t want = cfg->tc_ctas > 0 ? cfg->tc_ctas : padoc_default_ctas();
-        int64_t total_tiles = 0;
-        for (const Segment &sg : segs) total_tiles += sg.ntiles;
-        ctas = (int32_t)std::min<int64_t>(want, total_tiles);
-        pp.cta_ptr.assign((size_t)ctas + 1, 0);
-        // tile t of segment k starts at weight position W_k + t * w_k; it goes to the CTA whose
-        // range [c W / ctas, (c+1) W / ctas) holds that position
-        int64_t wpos = 0;
-        int32_t cur_cta = 0;
+    // CTA loads count every piece's own cost too (its epilogue, and the query reload before it):
+    // the smallest bound T for which a greedy walk along the sequences needs at most `want` CTAs
+    // is found by bisection, then the walk is made once more to emit the pieces.
+    const int64_t piece_w = PADOC_TC_PIECE_COST;
+    int64_t total_w = 0, max_w = 0;
+    for (const Segment &sg : segs) {
+        total_w += (int64_t)sg.ntiles * sg.weight + piece_w;
+        max_w = std::max<int64_t>(max_w, sg.weight);
+    }
+    auto walk = [&](int64_t T, bool emit) {
+        int64_t used = 0, load = 0;
         for (const Segment &sg : segs) {
             int32_t t = 0;
             while (t < sg.ntiles) {
-                while (cur_cta + 1 < ctas && wpos >= (int64_t)(cur_cta + 1) * total_w / ctas) {
-                    ++cur_cta;
-                    pp.cta_ptr[cur_cta] = (int32_t)tc_items.size();
+                int64_t room = used > 0 ? (T - load - piece_w) / sg.weight : 0;
+                if (room < 1) {   // close the current CTA, open the next
+                    if (emit) pp.cta_ptr.push_back((int32_t)tc_items.size());
+                    ++used;
+                    load = 0;
+                    room = std::max<int64_t>(1, (T - piece_w) / sg.weight);
                 }
-                const int64_t end_w = (int64_t)(cur_cta + 1) * total_w / ctas;
-                int32_t t1 = t;
-                while (t1 < sg.ntiles && (cur_cta + 1 == ctas || wpos + (int64_t)(t1 - t) * sg.weight < end_w)) ++t1;
-                if (t1 == t) t1 = t + 1;
-                const int32_t tb = t * PADOC_TC_TILE_TOKENS, te = std::min(sg.vis, t1 * PADOC_TC_TILE_TOKENS);
-                const int32_t slot = cnt[(size_t)sg.first * Hkv + sg.g];
-                for (int32_t st = sg.first; st < sg.first + sg.ns; ++st) ++cnt[(size_t)st * Hkv + sg.g];
-                tc_items.push_back({PADOC_ITEM_SHARED_TC, sg.p, sg.g, tb, te, sg.first, sg.ns, slot});
-                wpos += (int64_t)(t1 - t) * sg.weight;
+                const int32_t t1 = (int32_t)std::min<int64_t>(sg.ntiles, t + room);
+                load += piece_w + (int64_t)(t1 - t) * sg.weight;
+                if (emit) {
+                    const int32_t tb = t * PADOC_TC_TILE_TOKENS, te = std::min(sg.vis, t1 * PADOC_TC_TILE_TOKENS);
+                    const int32_t slot = cnt[(size_t)sg.first * Hkv + sg.g];
+                    for (int32_t st = sg.first; st < sg.first + sg.ns; ++st) ++cnt[(size_t)st * Hkv + sg.g];
+                    tc_items.push_back({PADOC_ITEM_SHARED_TC, sg.p, sg.g, tb, te, sg.first, sg.ns, slot});
+                }
                 t = t1;
             }
         }
-        for (int32_t c = cur_cta + 1; c <= ctas; ++c) pp.cta_ptr[c] = (int32_t)tc_items.size();
+        return used;
+    };
+    int32_t ctas = 0;
+    if (!segs.empty()) {
+        const int64_t want = cfg->tc_ctas > 0 ? cfg->tc_ctas : padoc_default_ctas();
+        int64_t lo = max_w + piece_w, hi = total_w + max_w;   // walk(hi) needs one CTA
+        while (lo < hi) {
+            const int64_t mid = lo + (hi - lo) / 2;
+            if (walk(mid, false) <= want) hi = mid; else lo = mid + 1;
+        }
+        ctas = (int32_t)walk(lo, true);
+        pp.cta_ptr.push_back((int32_t)tc_items.size());
     }
     pp.tc_ctas = ctas;
 

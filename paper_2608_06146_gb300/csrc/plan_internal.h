@@ -24,6 +24,9 @@
 #define PADOC_TC_TILE_TOKENS 128
 #define PADOC_TC_WEIGHT_2M 8
 #define PADOC_TC_WEIGHT_1M 7
+// Fixed cost of one tensor-core piece in the same units (its partials' epilogue and the reload of
+// the queries before it: about a tile and a half)
+#define PADOC_TC_PIECE_COST 12
 
 // Warps per CTA of the warp kernel, and the start-up cost of one warp item in 16-token blocks
 // (query fragments, the first blocks' latency, the partial's write), used to balance warps.
