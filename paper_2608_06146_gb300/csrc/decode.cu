@@ -35,9 +35,7 @@ constexpr int kWStages = 3;            // paged blocks in flight per warp
 constexpr int kBoxBytes = kBlk * 128;  // one 16-row x 64-column box
 constexpr int kWStageBytes = 4 * kBoxBytes;   // K lo, K hi, V lo, V hi
 constexpr int kWarpRing = kWStages * kWStageBytes;
-constexpr int kMergeStride = 132;      // floats per head row when a warp stages its O^T
-constexpr int kWarpStage = kGroup * kMergeStride * 4;   // a warp's O^T staging buffer
-constexpr size_t kDecodeSmem = 1024 + (size_t)kWarps * (kWarpRing + kWarpStage);
+constexpr size_t kDecodeSmem = 1024 + (size_t)kWarps * kWarpRing;
 
 struct DecodeParams {
     const int32_t *stream_page, *shared_len, *private_len, *slot_ptr;
@@ -67,13 +65,14 @@ __device__ __forceinline__ void finish_warp(const DecodeParams &prm)
 __global__ void __launch_bounds__(kWarps * 32, 1)
 decode_warp_kernel(const DecodeParams prm)
 {
+    // the merge that follows waits for this whole grid before it reads anything, so it may launch now
+    pdl_launch_dependents();
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int wi = blockIdx.x * kWarps + warp;
     if (wi >= prm.num_warps) { finish_warp(prm); return; }   // warps are independent: no CTA barrier follows
     uint8_t *wbuf = smem + (size_t)warp * kWarpRing;
-    float *st = reinterpret_cast<float *>(smem + (size_t)kWarps * kWarpRing + (size_t)warp * kWarpStage);   // [8][132]
     const padoc_item *items = prm.items + prm.first_item;
     const int i0 = prm.warp_ptr[wi], i1 = prm.warp_ptr[wi + 1];
     // Every global read the loop depends on is issued at least one item ahead: item headers two
@@ -241,34 +240,26 @@ decode_warp_kernel(const DecodeParams prm)
             l[0] += __shfl_xor_sync(0xffffffffu, l[0], sh);
             l[1] += __shfl_xor_sync(0xffffffffu, l[1], sh);
         }
-        // stage O^T and write the partial with 16-byte stores
+        // the partial, straight from the accumulators: for each (mt, register) the 8 lanes of a head
+        // write 8 consecutive dims, so every store fills whole 32-byte sectors
         {
             const int h0 = (lane & 3) * 2;
             const float i0f = l[0] > 0.f ? 1.f / l[0] : 0.f, i1f = l[1] > 0.f ? 1.f / l[1] : 0.f;
+            float *o0 = prm.part_o + (row0 + h0) * kD + (lane >> 2);
+            float *o1 = o0 + kD;
 #pragma unroll
             for (int mt = 0; mt < 8; ++mt) {
-                const int d0 = mt * 16 + (lane >> 2);
-                st[h0 * kMergeStride + d0] = o[mt][0] * i0f;
-                st[(h0 + 1) * kMergeStride + d0] = o[mt][1] * i1f;
-                st[h0 * kMergeStride + d0 + 8] = o[mt][2] * i0f;
-                st[(h0 + 1) * kMergeStride + d0 + 8] = o[mt][3] * i1f;
+                o0[mt * 16] = o[mt][0] * i0f;
+                o1[mt * 16] = o[mt][1] * i1f;
+                o0[mt * 16 + 8] = o[mt][2] * i0f;
+                o1[mt * 16 + 8] = o[mt][3] * i1f;
             }
-        }
-        __syncwarp();
-#pragma unroll
-        for (int k = 0; k < 8; ++k) {
-            const int idx = k * 32 + lane;          // float4 index over [8 heads][32 float4]
-            const int hl = idx >> 5, d4 = idx & 31;
-            const float *src = st + hl * kMergeStride + d4 * 4;
-            *reinterpret_cast<float4 *>(prm.part_o + (row0 + hl) * kD + d4 * 4) =
-                make_float4(src[0], src[1], src[2], src[3]);
         }
         if (lane < 4) {
             const int h0 = lane * 2;
             prm.part_lse[row0 + h0] = l[0] > 0.f ? (m[0] + log2f(l[0])) * PADOC_LN2 : -INFINITY;
             prm.part_lse[row0 + h0 + 1] = l[1] > 0.f ? (m[1] + log2f(l[1])) * PADOC_LN2 : -INFINITY;
         }
-        __syncwarp();   // the staging buffer is read before the next item overwrites it
     }
     cp_async_wait<0>();
     finish_warp(prm);
@@ -292,6 +283,10 @@ __global__ void __launch_bounds__(128) decode_combine_kernel(const int32_t *__re
                                                              const float *__restrict__ part_lse,
                                                              __nv_bfloat16 *__restrict__ out, float *__restrict__ lse_out)
 {
+    // launched programmatically after the decode kernels: wait for them (and their partials), then
+    // let the next step's first kernel launch (it waits for this grid before touching memory)
+    pdl_wait_prerequisite();
+    pdl_launch_dependents();
     const int key = blockIdx.x;                      // s * Hkv + g; output rows key * 8 + h
     const int tid = threadIdx.x;
     const int h = tid >> 4, part = tid & 15;         // head, 8-dim slice
@@ -563,8 +558,19 @@ extern "C" padoc_status padoc_branch_decode_attn(const padoc_kv_pool *pool, cons
         st = padoc_launch_status();
         if (st != PADOC_OK) return st;
     }
-    decode_combine_kernel<<<(unsigned)((int64_t)info->num_streams * cfg.num_kv_heads), 128, 0, cs>>>(
-        prm.slot_ptr, part_o, part_lse, (__nv_bfloat16 *)out, lse);
+    {
+        cudaLaunchConfig_t lc = {};
+        lc.gridDim = dim3((unsigned)((int64_t)info->num_streams * cfg.num_kv_heads));
+        lc.blockDim = dim3(128);
+        lc.stream = cs;
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;   // see the kernel's wait
+        attr[0].val.programmaticStreamSerializationAllowed = 1;
+        lc.attrs = attr;
+        lc.numAttrs = 1;
+        PADOC_CUDA_TRY(cudaLaunchKernelEx(&lc, decode_combine_kernel, prm.slot_ptr, (const float *)part_o,
+                                          (const float *)part_lse, (__nv_bfloat16 *)out, lse));
+    }
     return padoc_launch_status();
 }
 

@@ -114,11 +114,6 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
     float *xch = (float *)(misc + 256);
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     auto bar = [&](int i) { return smem_u32(&bars[i]); };
-    // the warp kernel that follows reads nothing this grid writes before its final wait, so it may
-    // start filling SMs as soon as every CTA of this grid is resident
-    pdl_launch_dependents();
-    const int u0 = prm.cta_ptr[blockIdx.x], u1 = prm.cta_ptr[blockIdx.x + 1];
-
     if (tid == 0) {
         for (int i = 0; i < B_COUNT; ++i)
             mbar_init(smem_u32(&bars[i]), (i == B_PFULL || i == B_PFULL + 1) ? kSoftmaxWarps : 1);
@@ -136,6 +131,13 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
+    // Nothing above touches global memory, so under a programmatic launch it overlaps the end of
+    // the previous kernel in the stream. From here on the grid reads its inputs and writes partials
+    // (which the previous step's merge may still be reading), so it first waits for that kernel, and
+    // only then lets the warp kernel (which writes partials too) launch.
+    pdl_wait_prerequisite();
+    pdl_launch_dependents();
+    const int u0 = prm.cta_ptr[blockIdx.x], u1 = prm.cta_ptr[blockIdx.x + 1];
 
     if (warp == 8 || warp == 10) {
         // ---------------------------------------------------------------- TMA producers (whole warps)
@@ -513,6 +515,16 @@ padoc_status padoc_launch_decode_tc(const CUtensorMap *kmap, const CUtensorMap *
     prm.scale_log2 = scale_log2;
     prm.err = err;
     PADOC_CUDA_TRY(cudaFuncSetAttribute(decode_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes));
-    decode_tc_kernel<<<info->tc_ctas, kThreads, kSmemBytes, stream>>>(*kmap, *vmap, *qmap, prm);
+    cudaLaunchConfig_t lc = {};
+    lc.gridDim = dim3((unsigned)info->tc_ctas);
+    lc.blockDim = dim3(kThreads);
+    lc.dynamicSmemBytes = kSmemBytes;
+    lc.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;   // see the kernel's wait
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    lc.attrs = attr;
+    lc.numAttrs = 1;
+    PADOC_CUDA_TRY(cudaLaunchKernelEx(&lc, decode_tc_kernel, *kmap, *vmap, *qmap, prm));
     return padoc_launch_status();
 }

@@ -187,17 +187,18 @@ def test_decode_plan_covers_every_visible_token_once(wl_name, layout, tc_ctas, w
     # the warp grid: warp lists cover the warp items in order, one wave, balanced by cost
     nw_items = info.num_items - ntc
     wp = plan[info.off_warp_ptr: info.off_warp_ptr + info.num_warps + 1]
-    wctas = min(warp_ctas or 152, -(-nw_items // 8))
-    assert info.num_warps == min(wctas * 8, nw_items)
+    W = 8   # warps per CTA of the warp kernel
+    wctas = min(warp_ctas or 152, -(-nw_items // W))
+    assert info.num_warps == min(wctas * W, nw_items)
     assert wp[0] == 0 and wp[-1] == nw_items and np.all(np.diff(wp) >= 0)
     cost = [-(-(te - tb) // 16) + 2 for _, _, _, tb, te, *_ in items[ntc:]]
     loads = np.array([sum(cost[wp[w]:wp[w + 1]]) for w in range(info.num_warps)])
     # CTA totals (LPT over CTAs) and the warps inside each CTA (LPT again) are balanced
-    cta_loads = [loads[c * 8:(c + 1) * 8].sum() for c in range(-(-info.num_warps // 8))]
+    cta_loads = [loads[c * W:(c + 1) * W].sum() for c in range(-(-info.num_warps // W))]
     assert max(cta_loads) - min(cta_loads) <= max(cost) or len(cta_loads) == 1
     for c in range(len(cta_loads)):
-        wl_ = loads[c * 8:(c + 1) * 8]
-        if len(wl_) == 8 and wl_.min() > 0:
+        wl_ = loads[c * W:(c + 1) * W]
+        if len(wl_) == W and wl_.min() > 0:
             assert wl_.max() - wl_.min() <= max(cost)
     # a warp item never reaches past its stream's cutoff (the warp kernel reads none)
     for kind, idx, g, tb, te, fs, ns, slot in items[ntc:]:
