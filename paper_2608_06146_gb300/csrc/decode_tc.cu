@@ -71,6 +71,7 @@ static_assert(kSmemBytes <= 232448, "shared memory per CTA");
 struct TcDecodeParams {
     const int32_t *shared_len, *slot_ptr, *cta_ptr;
     const padoc_item *items;
+    int32_t num_tc_items, num_pages;
     const int32_t *page_table;
     int32_t page_stride;
     int32_t num_blocks, num_kv_heads;
@@ -114,6 +115,33 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
     float *xch = (float *)(misc + 256);
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     auto bar = [&](int i) { return smem_u32(&bars[i]); };
+    if (warp == 8 || warp == 10) {
+        // Before this grid waits for the previous kernel, the producers pull the CTA's first queries
+        // and first two K/V tiles into L2. L2 is where every write lands, so a prefetch can only
+        // warm it, never serve stale data later; every index is range-checked first, and a tensor
+        // prefetch past the pool fetches nothing.
+        const int a0 = prm.cta_ptr[blockIdx.x], a1 = prm.cta_ptr[blockIdx.x + 1];
+        if (a0 >= 0 && a0 < a1 && a0 < prm.num_tc_items) {
+            const padoc_item it = prm.items[a0];
+            const CUtensorMap *map = warp == 8 ? &kmap : &vmap;
+            const int j = lane >> 3, b = lane & 7;   // lanes 0-15: tiles 0-1, blocks 0-7
+            const int tok0 = it.tok_begin + j * kKT + b * kBlk;
+            if (lane < 16 && it.index >= 0 && it.index < prm.num_pages && tok0 >= 0 && tok0 < it.tok_end &&
+                tok0 / kBlk < prm.page_stride) {
+                const int32_t id = prm.page_table[(size_t)it.index * prm.page_stride + tok0 / kBlk];
+                if (id >= 0 && id < prm.num_blocks) {
+                    const int32_t row = (id * prm.num_kv_heads + it.kv_head) * kBlk;
+                    tma_prefetch_l2_2d(map, 0, row);
+                    tma_prefetch_l2_2d(map, 64, row);
+                }
+            }
+            if (warp == 8 && lane == 16)
+                for (int i = 0; i < piece_mtiles(it); ++i) {
+                    tma_prefetch_l2_4d(&qmap, 0, 0, it.kv_head, it.first_stream + 16 * i);
+                    tma_prefetch_l2_4d(&qmap, 64, 0, it.kv_head, it.first_stream + 16 * i);
+                }
+        }
+    }
     if (tid == 0) {
         for (int i = 0; i < B_COUNT; ++i)
             mbar_init(smem_u32(&bars[i]), (i == B_PFULL || i == B_PFULL + 1) ? kSoftmaxWarps : 1);
@@ -505,6 +533,8 @@ padoc_status padoc_launch_decode_tc(const CUtensorMap *kmap, const CUtensorMap *
     prm.slot_ptr = plan + info->off_slot_ptr;
     prm.cta_ptr = plan + info->off_cta_ptr;
     prm.items = reinterpret_cast<const padoc_item *>(plan + info->off_items);
+    prm.num_tc_items = info->num_tc_items;
+    prm.num_pages = info->num_pages;
     prm.page_table = page_table;
     prm.page_stride = page_stride;
     prm.num_blocks = num_blocks;
