@@ -334,13 +334,14 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
             const bool r = wait_or_abort(bar(bb), parity, prm.err, site, abort_flag);
             return __all_sync(0xffffffffu, r);
         };
-        // The 8 warps meet at a named barrier for every swap, so none may leave the loops early: after
-        // a failed wait (ok = false) a warp skips the work but still takes every swap.
+        // Warps w and w + 4 (the same TMEM lanes, the two column halves) meet at a named barrier of
+        // their own (1 + w % 4) for every swap, so neither may leave the loops early: after a failed
+        // wait (ok = false) a warp skips the work but still takes every swap.
         int nx = 0;   // row-value swaps so far (double-buffered)
         auto swap_row = [&](float v) {   // returns the value the other column half passed for this row
             float *buf = xch + (nx & 1) * 256;
             buf[hc * 128 + row] = v;
-            named_bar_sync(1, kSoftmaxWarps * 32);
+            named_bar_sync(1 + quad, 64);
             const float o = buf[(hc ^ 1) * 128 + row];
             ++nx;
             return o;
