@@ -104,6 +104,7 @@ decode_warp_kernel(const DecodeParams prm)
     if (i0 < i1) { pc = walk_of(load_item(i0)); ids_c = ids_of(pc); }
     if (i0 + 1 < i1) { pn = walk_of(load_item(i0 + 1)); ids_n = ids_of(pn); }
     if (i0 + 2 < i1) hn2 = load_item(i0 + 2);
+    const uint64_t kv_policy = l2_evict_first_policy();   // paged blocks are read once per call
     int ring = 0;   // blocks issued so far: block n goes to stage n % kWStages
     // chunk q = lane + 32k of a block's 512 16-byte chunks is panel q / 128 (K lo, K hi, V lo, V hi),
     // row (q / 8) % 16, 16-byte column q % 8 (swizzled)
@@ -129,7 +130,8 @@ decode_warp_kernel(const DecodeParams prm)
                 const int panel = q >> 7, r = (q >> 3) & 15, cc = q & 7;
                 const __nv_bfloat16 *src = (panel < 2 ? prm.k_pool : prm.v_pool) +
                                            (rowbase + r) * kD + (panel & 1) * 64 + cc * 8;
-                cp_async_16(base + panel * kBoxBytes + r * 128 + ((cc ^ (r & 7)) << 4), src, okid ? 16u : 0u);
+                cp_async_16_hint(base + panel * kBoxBytes + r * 128 + ((cc ^ (r & 7)) << 4), src, okid ? 16u : 0u,
+                                 kv_policy);
             }
             ++pb;
             ++ring;

@@ -177,6 +177,7 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
         const CUtensorMap *map = is_k ? &kmap : &vmap;
         uint8_t *ring = is_k ? sk : sv;
         const int b_full = is_k ? B_KFULL : B_VFULL, b_empty = is_k ? B_KEMPTY : B_VEMPTY;
+        const uint64_t kv_policy = l2_evict_first_policy();   // K/V tiles are read once per call
         int32_t id_next = 0;
         bool in_next = false;
         auto fetch_id = [&](int uu, int jj) {
@@ -236,8 +237,8 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
                 __syncwarp();
                 if (lane < kKT / kBlk) {
                     const uint32_t dst = smem_u32(ring + s * kTile) + (uint32_t)lane * (kBlk * 128);
-                    tma_load_2d(dst, map, 0, row, bar(b_full + s));
-                    tma_load_2d(dst + kPanel, map, 64, row, bar(b_full + s));
+                    tma_load_2d_hint(dst, map, 0, row, bar(b_full + s), kv_policy);
+                    tma_load_2d_hint(dst + kPanel, map, 64, row, bar(b_full + s), kv_policy);
                 }
                 ++n;
                 if (is_k && j == 0 && !(q_first && u == u0)) {
