@@ -242,19 +242,19 @@ decode_warp_kernel(const DecodeParams prm)
             l[0] += __shfl_xor_sync(0xffffffffu, l[0], sh);
             l[1] += __shfl_xor_sync(0xffffffffu, l[1], sh);
         }
-        // the partial, straight from the accumulators: for each (mt, register) the 8 lanes of a head
-        // write 8 consecutive dims, so every store fills whole 32-byte sectors
+        // the partial, straight from the accumulators, in the slot layout [16 chunks of 8 dims]
+        // [8 heads][8]: for each (mt, register) the 8 lanes of a head write one chunk's 8 dims, so
+        // every store fills whole 32-byte sectors
         {
             const int h0 = (lane & 3) * 2;
             const float i0f = l[0] > 0.f ? 1.f / l[0] : 0.f, i1f = l[1] > 0.f ? 1.f / l[1] : 0.f;
-            float *o0 = prm.part_o + (row0 + h0) * kD + (lane >> 2);
-            float *o1 = o0 + kD;
+            float *p = prm.part_o + row0 * kD + h0 * 8 + (lane >> 2);   // row0 = slot * 8
 #pragma unroll
             for (int mt = 0; mt < 8; ++mt) {
-                o0[mt * 16] = o[mt][0] * i0f;
-                o1[mt * 16] = o[mt][1] * i1f;
-                o0[mt * 16 + 8] = o[mt][2] * i0f;
-                o1[mt * 16 + 8] = o[mt][3] * i1f;
+                p[mt * 128] = o[mt][0] * i0f;           // chunk 2 mt, head h0
+                p[mt * 128 + 8] = o[mt][1] * i1f;       // chunk 2 mt, head h0 + 1
+                p[mt * 128 + 64] = o[mt][2] * i0f;      // chunk 2 mt + 1, head h0
+                p[mt * 128 + 72] = o[mt][3] * i1f;      // chunk 2 mt + 1, head h0 + 1
             }
         }
         if (lane < 4) {
@@ -277,8 +277,8 @@ struct UniformSlots {  // public combine: part_row = split * rows + row
     __device__ int64_t part_row(int64_t row, int i) const { return (int64_t)i * rows + row; }
 };
 
-// Decode merge: one CTA per (stream, KV head), its 8 query heads x 16 threads, each thread 8 of the
-// 128 dims. One pass over the slots with an online reference (the running max of lse_s): four
+// Decode merge: one CTA per (stream, KV head), 16 dim chunks x its 8 query heads, each thread 8 of
+// the 128 dims of one head. One pass over the slots with an online reference (the running max of lse_s): four
 // partials' LSE and O loads are in flight per thread at a time.
 __global__ void __launch_bounds__(128) decode_combine_kernel(const int32_t *__restrict__ slot_ptr,
                                                              const float *__restrict__ part_o,
@@ -291,9 +291,9 @@ __global__ void __launch_bounds__(128) decode_combine_kernel(const int32_t *__re
     pdl_launch_dependents();
     const int key = blockIdx.x;                      // s * Hkv + g; output rows key * 8 + h
     const int tid = threadIdx.x;
-    const int h = tid >> 4, part = tid & 15;         // head, 8-dim slice
+    const int h = tid & 7, part = tid >> 3;          // head, 8-dim chunk: a warp reads 4 chunks x 8 heads, contiguous
     const int p0 = slot_ptr[key], n = slot_ptr[key + 1] - p0;
-    const float *bo = part_o + ((size_t)p0 * kGroup + h) * kD + part * 8;
+    const float *bo = part_o + (size_t)p0 * kGroup * kD + (part * kGroup + h) * 8;   // chunk `part` of head h
     const float *bl = part_lse + (size_t)p0 * kGroup + h;
     constexpr size_t kSlotO = (size_t)kGroup * kD;
     float mref = -INFINITY, ssum = 0.f;

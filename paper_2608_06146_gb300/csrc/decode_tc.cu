@@ -492,7 +492,9 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
                 const bool empty = !(l > 0.f);
                 const float inv = empty ? 0.f : 1.f / l;
                 const size_t prow = (size_t)(mi ? pb1 : pb0) * kGroup + hl;
-                float *dst = prm.part_o + prow * kD + 64 * hc;
+                // slot layout [16 chunks of 8 dims][8 heads][8]: the 8 rows (heads) of a stream write
+                // one contiguous 256-byte run per chunk
+                float *sb = prm.part_o + (size_t)(mi ? pb1 : pb0) * (kGroup * kD) + hl * 8;
                 const uint32_t tO = tmem + lanes + 256 + 128 * mi + 64 * hc;
 #pragma unroll
                 for (int q = 0; q < 2; ++q) {
@@ -502,11 +504,11 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
                         tmem_ld_wait();
                     }
                     if (valid) {
-                        // a row's half is 256 contiguous bytes: whole 32-byte sectors per store
 #pragma unroll
                         for (int i = 0; i < 32; i += 8) {
                             auto v = [&](int k) { return empty ? 0.f : __uint_as_float(o[i + k]) * inv; };
-                            st_global_v8(dst + q * 32 + i, v(0), v(1), v(2), v(3), v(4), v(5), v(6), v(7));
+                            const int chunk = 8 * hc + 4 * q + i / 8;
+                            st_global_v8(sb + chunk * (kGroup * 8), v(0), v(1), v(2), v(3), v(4), v(5), v(6), v(7));
                         }
                     }
                 }

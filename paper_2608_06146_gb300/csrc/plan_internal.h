@@ -54,8 +54,10 @@ typedef struct {
 
 static inline size_t padoc_align256(size_t x) { return (x + 255) & ~(size_t)255; }
 
-// Workspace: part_o fp32 [slots][group][d], then part_lse fp32 [slots][group] at a 256-byte
-// boundary; a slot holds one partial of the group = Hq / Hkv query heads of one (stream, KV head).
+// Workspace: part_o fp32 [slots][d / 8][group][8] (a slot's dims in chunks of 8, the group's heads
+// inside a chunk, so that the heads of one stream are written as one contiguous run per chunk), then
+// part_lse fp32 [slots][group] at a 256-byte boundary; a slot holds one partial of the
+// group = Hq / Hkv query heads of one (stream, KV head).
 static inline size_t padoc_decode_workspace_bytes(int64_t slots, int32_t group, int32_t d)
 {
     return padoc_align256((size_t)slots * group * d * 4) + padoc_align256((size_t)slots * group * 4);
