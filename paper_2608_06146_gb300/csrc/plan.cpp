@@ -274,10 +274,14 @@ padoc_status build_parts(const padoc_page *pages, int32_t num_pages, const padoc
     // CTA loads count every piece's own cost too (its epilogue, and the query reload before it):
     // the smallest bound T for which a greedy walk along the sequences needs at most `want` CTAs
     // is found by bisection, then the walk is made once more to emit the pieces.
-    const int64_t piece_w = PADOC_TC_PIECE_COST;
+    auto piece_cost = [](const Segment &sg) -> int64_t {
+        return sg.weight == PADOC_TC_WEIGHT_2M ? PADOC_TC_PIECE_COST_2M : PADOC_TC_PIECE_COST_1M;
+    };
+    int64_t max_piece = 0;
     int64_t total_w = 0, max_w = 0;
     for (const Segment &sg : segs) {
-        total_w += (int64_t)sg.ntiles * sg.weight + piece_w;
+        total_w += (int64_t)sg.ntiles * sg.weight + piece_cost(sg);
+        max_piece = std::max(max_piece, piece_cost(sg));
         max_w = std::max<int64_t>(max_w, sg.weight);
     }
     auto walk = [&](int64_t T, bool emit) {
@@ -285,6 +289,7 @@ padoc_status build_parts(const padoc_page *pages, int32_t num_pages, const padoc
         for (const Segment &sg : segs) {
             int32_t t = 0;
             while (t < sg.ntiles) {
+                const int64_t piece_w = piece_cost(sg);
                 int64_t room = used > 0 ? (T - load - piece_w) / sg.weight : 0;
                 if (room < 1) {   // close the current CTA, open the next
                     if (emit) pp.cta_ptr.push_back((int32_t)tc_items.size());
@@ -308,7 +313,7 @@ padoc_status build_parts(const padoc_page *pages, int32_t num_pages, const padoc
     int32_t ctas = 0;
     if (!segs.empty()) {
         const int64_t want = cfg->tc_ctas > 0 ? cfg->tc_ctas : padoc_default_ctas();
-        int64_t lo = max_w + piece_w, hi = total_w + max_w;   // walk(hi) needs one CTA
+        int64_t lo = max_w + max_piece, hi = total_w + max_w;   // walk(hi) needs one CTA
         while (lo < hi) {
             const int64_t mid = lo + (hi - lo) / 2;
             if (walk(mid, false) <= want) hi = mid; else lo = mid + 1;

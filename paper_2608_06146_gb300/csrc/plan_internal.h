@@ -25,8 +25,10 @@
 #define PADOC_TC_WEIGHT_2M 8
 #define PADOC_TC_WEIGHT_1M 7
 // Fixed cost of one tensor-core piece in the same units (its partials' epilogue and the reload of
-// the queries before it: about a tile and a half)
-#define PADOC_TC_PIECE_COST 12
+// the queries before it), fitted on GB300 to per-CTA timelines of the serving batch: about one tile
+// for a one-M-tile piece, a tile and a half for a two-M-tile piece
+#define PADOC_TC_PIECE_COST_1M 7
+#define PADOC_TC_PIECE_COST_2M 11
 
 // Warps per CTA of the warp kernel, and the start-up cost of one warp item in 16-token blocks
 // (query fragments, the first blocks' latency, the partial's write), used to balance warps.

@@ -178,10 +178,10 @@ def test_decode_plan_covers_every_visible_token_once(wl_name, layout, tc_ctas, w
         # balance: CTA loads (tiles by weight plus a fixed cost per piece) stay within one tile and
         # one piece of the average over the CTAs asked for, and none is empty
         wts = [8 if ns > 16 else 7 for *_, ns, _ in items[:ntc]]
-        work = [sum(-(-(items[u, 4] - items[u, 3]) // 128) * wts[u] + 12 for u in range(cta[c], cta[c + 1]))
-                for c in range(info.tc_ctas)]
+        work = [sum(-(-(items[u, 4] - items[u, 3]) // 128) * wts[u] + (11 if wts[u] == 8 else 7)
+                    for u in range(cta[c], cta[c + 1])) for c in range(info.tc_ctas)]
         if info.tc_ctas == want:
-            assert max(work) <= sum(work) / want + 2 * (8 + 12)
+            assert max(work) <= sum(work) / want + 2 * (8 + 11)
     else:
         assert info.tc_ctas == 0
     # the warp grid: warp lists cover the warp items in order, one wave, balanced by cost
