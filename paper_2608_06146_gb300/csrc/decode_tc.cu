@@ -24,7 +24,7 @@
 // with the block ids looked up one tile ahead; blocks past the piece or with an out-of-range id are
 // fetched from an out-of-range coordinate, which fills zeros. Warp 8 also fetches each piece's
 // queries (one 4-D box per panel) once the previous piece's last QK^T has completed. Warp 9
-// allocates TMEM and issues the MMAs as a converged warp.
+// allocates TMEM; warps 9 and 11 issue the MMAs of M-tile 0 and M-tile 1, each as a converged warp.
 // TMEM: S_i / P_i at columns 128i, O_i at 256 + 128i. The next piece's first PV overwrites O_i; it
 // waits for P_i of that piece, which the softmax warps publish only after reading O_i out.
 #include <math.h>
@@ -43,7 +43,7 @@ constexpr int kTile = 2 * kPanel;
 constexpr int kKStages = 3;       // K tiles in the ring: K is released early (after QK^T)
 constexpr int kVStages = 2;       // V tiles in the ring: V is held until the tile's PV completes
 constexpr uint32_t kTmemCols = 512;
-constexpr int kThreads = 352;
+constexpr int kThreads = 384;
 
 enum {
     B_Q = 0,         // the piece's queries have landed
@@ -144,7 +144,11 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
     }
     if (tid == 0) {
         for (int i = 0; i < B_COUNT; ++i)
-            mbar_init(smem_u32(&bars[i]), (i == B_PFULL || i == B_PFULL + 1) ? kSoftmaxWarps : 1);
+            mbar_init(smem_u32(&bars[i]), (i == B_PFULL || i == B_PFULL + 1) ? kSoftmaxWarps
+                                          : (i == B_QFREE || (i >= B_KEMPTY && i < B_KEMPTY + kKStages) ||
+                                             (i >= B_VEMPTY && i < B_VEMPTY + kVStages) || i == B_FINAL)
+                                                ? 2     // one commit from each MMA warp
+                                                : 1);
         *abort_flag = 0;
         fence_barrier_init();
         tma_prefetch_desc(&kmap);
@@ -256,67 +260,73 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
             for (int J = (n > nst ? n - nst : 0); J < n; ++J)
                 mbar_wait_bounded(bar(b_full + J % nst), (J / nst) & 1, prm.err, is_k ? 51 : 52);
         }
-    } else if (warp == 9) {
-        // ---------------------------------------------------------------- MMA issuer (whole warp)
+    } else if (warp == 9 || warp == 11) {
+        // ---------------------------------------------------------------- MMA issuers (whole warps)
+        // warp 9 issues M-tile 0's MMAs and warp 11 M-tile 1's, so that the waits, fences and
+        // commits of one chain (each costs the issuing warp ~200 cycles) overlap the other chain's
+        // MMAs on the tensor pipe. Both commit to the K/V-release, query-release and final
+        // barriers (two arrivals each); on a one-M-tile piece warp 11 only commits.
+        const int mi = warp == 9 ? 0 : 1;
         constexpr uint32_t idS = umma_idesc_bf16(128, kKT, false);
         constexpr uint32_t idPV = umma_idesc_bf16(128, kD, true);
-        const uint64_t dq0 = umma_desc_sw128(smem_u32(sq), 16, 1024);
-        const uint64_t dq1 = umma_desc_sw128(smem_u32(sq + kTile), 16, 1024);
+        const uint64_t dq = umma_desc_sw128(smem_u32(sq + mi * kTile), 16, 1024);
         // stage descriptors differ only in the start-address field (address >> 4)
         const uint64_t dk0 = umma_desc_sw128(smem_u32(sk), 16, 1024);
         const uint64_t dv0 = umma_desc_sw128(smem_u32(sv), kPanel, 1024);
+        const uint32_t tS = tmem + 128 * mi, tO = tmem + 256 + 128 * mi;
         auto wait_w = [&](int b, uint32_t parity, int site) {
             const bool r = wait_or_abort(bar(b), parity, prm.err, site, abort_flag);
             return __all_sync(0xffffffffu, r);
         };
-        auto issue_s = [&](int i, int stage) {
-            const uint64_t da = i ? dq1 : dq0, db = dk0 + (uint64_t)(stage * (kTile >> 4));
+        auto issue_s = [&](int stage) {
+            const uint64_t db = dk0 + (uint64_t)(stage * (kTile >> 4));
 #pragma unroll
             for (int ks = 0; ks < 8; ++ks) {
                 const uint32_t off = ((ks >> 2) * kPanel + (ks & 3) * 32) >> 4;
-                umma_bf16_ss_warp(tmem + 128 * i, da + off, db + off, idS, ks > 0);
+                umma_bf16_ss_warp(tS, dq + off, db + off, idS, ks > 0);
             }
-            umma_commit_warp(bar(B_SFULL + i));
+            umma_commit_warp(bar(B_SFULL + mi));
         };
-        int J = 0, nq = 0, c0 = 0, c1 = 0;   // tiles done, query sets used, tiles per M-tile
+        int J = 0, nq = 0, ci = 0;   // tiles done, query sets used, tiles of this M-tile
         bool ok = true;
         for (int u = u0; ok && u < u1; ++u) {
             const padoc_item it = prm.items[u];
-            const int ne = piece_tiles(it), mt = piece_mtiles(it);
+            const int ne = piece_tiles(it);
+            const bool act = mi < piece_mtiles(it);   // this warp's M-tile is part of the piece
             if (ne == 0) continue;
             if (!wait_w(B_Q, nq & 1, 60) || !wait_w(B_KFULL + J % kKStages, (J / kKStages) & 1, 61)) { ok = false; break; }
             ++nq;
             tc_fence_after();
-            issue_s(0, J % kKStages);
-            if (mt == 2) issue_s(1, J % kKStages);
+            if (act) issue_s(J % kKStages);
             umma_commit_warp(bar(B_KEMPTY + J % kKStages));
             if (ne == 1) umma_commit_warp(bar(B_QFREE));
             for (int j = 0; ok && j < ne; ++j) {
                 const int Jj = J + j, s = Jj % kVStages, kn = (Jj + 1) % kKStages;
-#pragma unroll
-                for (int i = 0; i < 2; ++i) {
-                    if (i >= mt) break;
-                    const int ci = i ? c1 : c0;
-                    if (!wait_w(B_PFULL + i, ci & 1, 62)) { ok = false; break; }
-                    if (i == 0 && !wait_w(B_VFULL + s, (Jj / kVStages) & 1, 63)) { ok = false; break; }
+                if (act) {
+                    if (!wait_w(B_PFULL + mi, ci & 1, 62) || !wait_w(B_VFULL + s, (Jj / kVStages) & 1, 63)) { ok = false; break; }
                     tc_fence_after();
                     const uint64_t db = dv0 + (uint64_t)(s * (kTile >> 4));
 #pragma unroll
                     for (int kk = 0; kk < 8; ++kk)
-                        umma_bf16_ts_warp(tmem + 256 + 128 * i, tmem + 128 * i + kk * 8, db + kk * (2048 >> 4), idPV,
-                                          (j > 0 || kk > 0));
-                    umma_commit_warp(bar(B_PVDONE + i));
-                    if (i == mt - 1) umma_commit_warp(bar(B_VEMPTY + s));
-                    if (i) ++c1; else ++c0;
-                    if (j + 1 < ne) {
-                        if (i == 0 && !wait_w(B_KFULL + kn, ((Jj + 1) / kKStages) & 1, 64)) { ok = false; break; }
+                        umma_bf16_ts_warp(tO, tS + kk * 8, db + kk * (2048 >> 4), idPV, (j > 0 || kk > 0));
+                    umma_commit_warp(bar(B_PVDONE + mi));
+                    ++ci;
+                } else if (!wait_w(B_VFULL + s, (Jj / kVStages) & 1, 63)) {
+                    // an idle warp releases a V tile only once it has landed, so that it never
+                    // arrives twice on one phase of the release barrier (K and query releases are
+                    // gated the same way by the waits on the next K tile and the queries)
+                    ok = false;
+                    break;
+                }
+                umma_commit_warp(bar(B_VEMPTY + s));
+                if (j + 1 < ne) {
+                    if (!wait_w(B_KFULL + kn, ((Jj + 1) / kKStages) & 1, 64)) { ok = false; break; }
+                    if (act) {
                         tc_fence_after();
-                        issue_s(i, kn);
-                        if (i == mt - 1) {
-                            umma_commit_warp(bar(B_KEMPTY + kn));
-                            if (j + 2 == ne) umma_commit_warp(bar(B_QFREE));
-                        }
+                        issue_s(kn);
                     }
+                    umma_commit_warp(bar(B_KEMPTY + kn));
+                    if (j + 2 == ne) umma_commit_warp(bar(B_QFREE));
                 }
             }
             J += ne;
