@@ -54,7 +54,7 @@ enum {
     B_VEMPTY = 10,   // [V stage]: the last PV of the tile has completed
     B_SFULL = 12,    // [m-tile]
     B_PFULL = 14,    // [m-tile], one arrival per softmax warp
-    B_PVDONE = 16,   // [m-tile]
+    B_PVDONE = 16,   // [m-tile]: the piece's last PV has completed (O_i is final)
     B_FINAL = 18,
     B_COUNT = 19
 };
@@ -302,29 +302,28 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
             if (ne == 1) umma_commit_warp(bar(B_QFREE));
             for (int j = 0; ok && j < ne; ++j) {
                 const int Jj = J + j, s = Jj % kVStages, kn = (Jj + 1) % kKStages;
+                const bool more = j + 1 < ne;
+                // The tile's V and the next K landed long before the softmax publishes P, so their
+                // waits come first; between P and the next QK^T there is then one wait, one fence
+                // and the MMAs, and every release is committed after them. (An idle warp still
+                // waits for each tile it releases, so it never arrives twice on one phase.)
+                if (!wait_w(B_VFULL + s, (Jj / kVStages) & 1, 63) ||
+                    (more && !wait_w(B_KFULL + kn, ((Jj + 1) / kKStages) & 1, 64))) { ok = false; break; }
                 if (act) {
-                    if (!wait_w(B_PFULL + mi, ci & 1, 62) || !wait_w(B_VFULL + s, (Jj / kVStages) & 1, 63)) { ok = false; break; }
+                    if (!wait_w(B_PFULL + mi, ci & 1, 62)) { ok = false; break; }
                     tc_fence_after();
                     const uint64_t db = dv0 + (uint64_t)(s * (kTile >> 4));
 #pragma unroll
                     for (int kk = 0; kk < 8; ++kk)
                         umma_bf16_ts_warp(tO, tS + kk * 8, db + kk * (2048 >> 4), idPV, (j > 0 || kk > 0));
-                    umma_commit_warp(bar(B_PVDONE + mi));
                     ++ci;
-                } else if (!wait_w(B_VFULL + s, (Jj / kVStages) & 1, 63)) {
-                    // an idle warp releases a V tile only once it has landed, so that it never
-                    // arrives twice on one phase of the release barrier (K and query releases are
-                    // gated the same way by the waits on the next K tile and the queries)
-                    ok = false;
-                    break;
+                    // S_i of the next tile overwrites P_i only after this PV has read it (one
+                    // thread's MMAs run in issue order)
+                    if (more) issue_s(kn);
+                    else umma_commit_warp(bar(B_PVDONE + mi));   // O_i of the piece is complete
                 }
                 umma_commit_warp(bar(B_VEMPTY + s));
-                if (j + 1 < ne) {
-                    if (!wait_w(B_KFULL + kn, ((Jj + 1) / kKStages) & 1, 64)) { ok = false; break; }
-                    if (act) {
-                        tc_fence_after();
-                        issue_s(kn);
-                    }
+                if (more) {
                     umma_commit_warp(bar(B_KEMPTY + kn));
                     if (j + 2 == ne) umma_commit_warp(bar(B_QFREE));
                 }
@@ -358,6 +357,7 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
             return o;
         };
         int cnt0 = 0, cnt1 = 0;   // tiles of M-tile 0 / 1 so far
+        int pd0 = 0, pd1 = 0;     // pieces of M-tile 0 / 1 with tiles so far
         bool ok = true;
         // The next piece's fields are read while the current piece runs (its item at the piece's
         // start, the rows' cutoffs after its first tile), so no global load latency sits between
@@ -490,10 +490,12 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
 #pragma unroll
             for (int mi = 0; mi < 2; ++mi) {
                 if (mi >= mt) break;
-                const int cnt = mi ? cnt1 : cnt0;
                 const float m_ref = mi ? m1 : m0;
                 float l = mi ? l1 : l0;
-                if (ne > 0) ok = ok && wait_all(B_PVDONE + mi, (cnt - 1) & 1, 71);
+                if (ne > 0) {
+                    ok = ok && wait_all(B_PVDONE + mi, (mi ? pd1 : pd0) & 1, 71);
+                    if (mi) ++pd1; else ++pd0;
+                }
                 l += swap_row(l);   // plus the other column half's sum
                 if (!ok) continue;
                 tc_fence_after();
