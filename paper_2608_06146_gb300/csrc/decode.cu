@@ -279,20 +279,23 @@ struct UniformSlots {  // public combine: part_row = split * rows + row
 
 // Decode merge: one CTA per (stream, KV head), 16 dim chunks x its 8 query heads, each thread 8 of
 // the 128 dims of one head. One pass over the slots with an online reference (the running max of lse_s): four
-// partials' LSE and O loads are in flight per thread at a time.
-__global__ void __launch_bounds__(128) decode_combine_kernel(const int32_t *__restrict__ slot_ptr,
+// partials' LSE and O loads are in flight per thread at a time. Registers are capped so that nine CTAs
+// fit on an SM: the serving batch's 1344 (stream, KV head) pairs then start in one wave.
+__global__ void __launch_bounds__(128, 9) decode_combine_kernel(const int32_t *__restrict__ slot_ptr,
                                                              const float *__restrict__ part_o,
                                                              const float *__restrict__ part_lse,
                                                              __nv_bfloat16 *__restrict__ out, float *__restrict__ lse_out)
 {
-    // launched programmatically after the decode kernels: wait for them (and their partials), then
-    // let the next step's first kernel launch (it waits for this grid before touching memory)
+    // The slot range comes from the plan, which no kernel of the step writes, so it is read before
+    // the wait. Launched programmatically after the decode kernels: wait for them (and their
+    // partials), then let the next step's first kernel launch (it waits for this grid before
+    // touching memory).
+    const int key = blockIdx.x;                      // s * Hkv + g; output rows key * 8 + h
+    const int p0 = slot_ptr[key], n = slot_ptr[key + 1] - p0;
     pdl_wait_prerequisite();
     pdl_launch_dependents();
-    const int key = blockIdx.x;                      // s * Hkv + g; output rows key * 8 + h
     const int tid = threadIdx.x;
     const int h = tid & 7, part = tid >> 3;          // head, 8-dim chunk: a warp reads 4 chunks x 8 heads, contiguous
-    const int p0 = slot_ptr[key], n = slot_ptr[key + 1] - p0;
     const float *bo = part_o + (size_t)p0 * kGroup * kD + (part * kGroup + h) * 8;   // chunk `part` of head h
     const float *bl = part_lse + (size_t)p0 * kGroup + h;
     constexpr size_t kSlotO = (size_t)kGroup * kD;

@@ -8,6 +8,7 @@
 #include <cstdint>
 #include <cstring>
 #include <numeric>
+#include <queue>
 #include <vector>
 
 #include <cuda_runtime.h>
@@ -284,6 +285,7 @@ padoc_status build_parts(const padoc_page *pages, int32_t num_pages, const padoc
         max_piece = std::max(max_piece, piece_cost(sg));
         max_w = std::max<int64_t>(max_w, sg.weight);
     }
+    std::vector<int64_t> tc_load;   // planned load of each tensor-core CTA (emitting walk)
     auto walk = [&](int64_t T, bool emit) {
         int64_t used = 0, load = 0;
         for (const Segment &sg : segs) {
@@ -292,7 +294,10 @@ padoc_status build_parts(const padoc_page *pages, int32_t num_pages, const padoc
                 const int64_t piece_w = piece_cost(sg);
                 int64_t room = used > 0 ? (T - load - piece_w) / sg.weight : 0;
                 if (room < 1) {   // close the current CTA, open the next
-                    if (emit) pp.cta_ptr.push_back((int32_t)tc_items.size());
+                    if (emit) {
+                        if (used > 0) tc_load.push_back(load);
+                        pp.cta_ptr.push_back((int32_t)tc_items.size());
+                    }
                     ++used;
                     load = 0;
                     room = std::max<int64_t>(1, (T - piece_w) / sg.weight);
@@ -308,6 +313,7 @@ padoc_status build_parts(const padoc_page *pages, int32_t num_pages, const padoc
                 t = t1;
             }
         }
+        if (emit && used > 0) tc_load.push_back(load);
         return used;
     };
     int32_t ctas = 0;
@@ -352,9 +358,8 @@ padoc_status build_parts(const padoc_page *pages, int32_t num_pages, const padoc
     for (size_t i = 0; i < (size_t)S * Hkv; ++i) pp.slot_ptr[i + 1] = pp.slot_ptr[i] + cnt[i];
 
     // The warp grid runs as one wave. Items are taken longest first (LPT; a counting sort on the
-    // block count keeps ties in plan order) and each goes to the least loaded CTA (an SM's warps
-    // share its memory bandwidth, so CTA totals are what must match), then within each CTA to its
-    // least loaded warp. Cost: 16-token blocks plus a fixed start-up cost per item.
+    // block count keeps ties in plan order) and each goes to the warp with the most capacity left
+    // (below). Cost: 16-token blocks plus a fixed start-up cost per item.
     const int32_t nitems = (int32_t)warp_items.size();
     std::vector<int32_t> cost((size_t)nitems), order((size_t)nitems);
     int32_t maxb = 0;
@@ -378,51 +383,61 @@ padoc_status build_parts(const padoc_page *pages, int32_t num_pages, const padoc
     pp.items.resize(tc_items.size() + (size_t)nitems);
     std::copy(tc_items.begin(), tc_items.end(), pp.items.begin());
     if (nwarps > 0) {
-        // least loaded CTA: loads only grow and the minimum never falls, so CTAs sit in FIFO buckets
-        // by load and a cursor walks up to the lowest non-empty bucket (O(1) per item)
+        // Warp CTAs start at different times: the first (SMs - tensor-core CTAs) of them on SMs the
+        // tensor-core grid leaves free, soon after launch; the others, in index order, on the SMs
+        // that tensor-core CTAs free as they finish (predicted from their planned loads). A warp's
+        // share of the work is sized to the time it has: its capacity is its rate times
+        // (T - its CTA's start - the time to its first block), with T such that the capacities add
+        // up to the work. Taking items longest first, each to the warp with the most capacity left,
+        // puts the longest items on the warps that start first. Without tensor-core work every warp
+        // starts at once and the capacities are equal.
         int64_t total = 0;
         for (int32_t i = 0; i < nitems; ++i) total += cost[(size_t)i];
-        const int64_t nbuckets = total / wctas + maxb + PADOC_WARP_ITEM_COST + 2;
-        std::vector<int32_t> head((size_t)nbuckets, -1), tail((size_t)nbuckets, -1), next((size_t)wctas, -1);
-        auto push = [&](int64_t load, int32_t c) {
-            next[(size_t)c] = -1;
-            if (tail[(size_t)load] < 0) head[(size_t)load] = c; else next[(size_t)tail[(size_t)load]] = c;
-            tail[(size_t)load] = c;
-        };
-        for (int32_t c = 0; c < wctas; ++c) push(0, c);
-        std::vector<int32_t> cta_of((size_t)nitems), cstart((size_t)wctas + 1, 0);
-        int64_t cur = 0;
-        for (int32_t k : order) {
-            while (head[(size_t)cur] < 0) ++cur;
-            const int32_t c = head[(size_t)cur];
-            head[(size_t)cur] = next[(size_t)c];
-            if (head[(size_t)cur] < 0) tail[(size_t)cur] = -1;
-            cta_of[(size_t)k] = c;
-            ++cstart[(size_t)c + 1];
-            push(cur + cost[(size_t)k], c);
-        }
-        for (int32_t c = 0; c < wctas; ++c) cstart[(size_t)c + 1] += cstart[(size_t)c];
-        std::vector<int32_t> by_cta((size_t)nitems), cpos(cstart.begin(), cstart.end() - 1);
-        for (int32_t k : order) by_cta[(size_t)cpos[(size_t)cta_of[(size_t)k]]++] = k;   // LPT order per CTA
-        std::vector<int32_t> warp_of((size_t)nitems);
-        for (int32_t c = 0; c < wctas; ++c) {
-            const int32_t w0 = c * PADOC_WARP_KERNEL_WARPS;
-            const int32_t nw = std::min<int32_t>(PADOC_WARP_KERNEL_WARPS, nwarps - w0);
-            int64_t load[PADOC_WARP_KERNEL_WARPS] = {0};
-            for (int32_t j = cstart[(size_t)c]; j < cstart[(size_t)c + 1]; ++j) {
-                const int32_t k = by_cta[(size_t)j];
-                int32_t best = 0;
-                for (int32_t w = 1; w < nw; ++w)
-                    if (load[w] < load[best]) best = w;
-                warp_of[(size_t)k] = w0 + best;
-                load[best] += cost[(size_t)k];
-                ++pp.warp_ptr[(size_t)(w0 + best) + 1];
+        std::vector<double> start((size_t)nwarps, 0.0), rate((size_t)nwarps, PADOC_WARP_RATE);
+        if (!tc_load.empty()) {
+            std::vector<double> tend(tc_load.size());
+            for (size_t c = 0; c < tc_load.size(); ++c) tend[c] = PADOC_TC_END_US0 + PADOC_TC_US_PER_UNIT * (double)tc_load[c];
+            std::sort(tend.begin(), tend.end());
+            const int32_t nfree = std::max<int32_t>(0, padoc_default_ctas() - (int32_t)tc_load.size());
+            for (int32_t w = 0; w < nwarps; ++w) {
+                const int32_t c = w / PADOC_WARP_KERNEL_WARPS;
+                if (c < nfree) {
+                    start[(size_t)w] = PADOC_WARP_EARLY_START_US;
+                    rate[(size_t)w] = PADOC_WARP_EARLY_RATE;
+                } else {
+                    const size_t k = std::min<size_t>((size_t)(c - nfree), tend.size() - 1);
+                    start[(size_t)w] = tend[k] + PADOC_WARP_START_DELAY_US;
+                }
             }
+        }
+        for (int32_t w = 0; w < nwarps; ++w) start[(size_t)w] += PADOC_WARP_FIRST_US;
+        // T by bisection on sum_w rate_w * max(0, T - start_w) = total
+        auto cap_sum = [&](double T) {
+            double s = 0.0;
+            for (int32_t w = 0; w < nwarps; ++w) s += rate[(size_t)w] * std::max(0.0, T - start[(size_t)w]);
+            return s;
+        };
+        double lo = 0.0, hi = 1.0;
+        while (cap_sum(hi) < (double)total) hi *= 2.0;
+        for (int it = 0; it < 60; ++it) {
+            const double mid = 0.5 * (lo + hi);
+            if (cap_sum(mid) < (double)total) lo = mid; else hi = mid;
+        }
+        std::priority_queue<std::pair<double, int32_t>> room;   // (capacity left, -warp)
+        for (int32_t w = 0; w < nwarps; ++w) room.push({rate[(size_t)w] * std::max(0.0, hi - start[(size_t)w]), -w});
+        std::vector<int32_t> warp_of((size_t)nitems);
+        for (int32_t k : order) {
+            auto top = room.top();
+            room.pop();
+            const int32_t w = -top.second;
+            warp_of[(size_t)k] = w;
+            ++pp.warp_ptr[(size_t)w + 1];
+            room.push({top.first - (double)cost[(size_t)k], top.second});
         }
         for (int32_t w = 0; w < nwarps; ++w) pp.warp_ptr[(size_t)w + 1] += pp.warp_ptr[(size_t)w];
         std::vector<int32_t> wpos(pp.warp_ptr.begin(), pp.warp_ptr.end() - 1);
         padoc_item *dst = pp.items.data() + tc_items.size();
-        for (int32_t k : by_cta) dst[wpos[(size_t)warp_of[(size_t)k]]++] = warp_items[(size_t)k];
+        for (int32_t k : order) dst[wpos[(size_t)warp_of[(size_t)k]]++] = warp_items[(size_t)k];   // longest first per warp
     }
     pp.num_warps = nwarps;
     return PADOC_OK;

@@ -193,13 +193,21 @@ def test_decode_plan_covers_every_visible_token_once(wl_name, layout, tc_ctas, w
     assert wp[0] == 0 and wp[-1] == nw_items and np.all(np.diff(wp) >= 0)
     cost = [-(-(te - tb) // 16) + 2 for _, _, _, tb, te, *_ in items[ntc:]]
     loads = np.array([sum(cost[wp[w]:wp[w + 1]]) for w in range(info.num_warps)])
-    # CTA totals (LPT over CTAs) and the warps inside each CTA (LPT again) are balanced
-    cta_loads = [loads[c * W:(c + 1) * W].sum() for c in range(-(-info.num_warps // W))]
-    assert max(cta_loads) - min(cta_loads) <= max(cost) or len(cta_loads) == 1
-    for c in range(len(cta_loads)):
-        wl_ = loads[c * W:(c + 1) * W]
-        if len(wl_) == W and wl_.min() > 0:
+    # Each warp's share follows the time it has (LPT over warps by capacity left). Without
+    # tensor-core work every warp starts at once, so the shares are equal up to one item; with it,
+    # the warps of one CTA start together, so their shares are equal up to one item, and the
+    # longest items go to the warps that start first.
+    if ntc == 0:
+        assert loads.max() - loads.min() <= max(cost)
+    else:
+        for c in range(-(-info.num_warps // W)):
+            wl_ = loads[c * W:(c + 1) * W]
             assert wl_.max() - wl_.min() <= max(cost)
+        first = np.array([cost[wp[w]] if wp[w + 1] > wp[w] else 0 for w in range(info.num_warps)])
+        nfree = max(0, 152 - info.tc_ctas)   # the planner's SM count on a host without a GPU
+        if 0 < nfree * W < info.num_warps:
+            assert first[:nfree * W].min() >= first[nfree * W:].max() - 2
+    assert loads.sum() == sum(cost)
     # a warp item never reaches past its stream's cutoff (the warp kernel reads none)
     for kind, idx, g, tb, te, fs, ns, slot in items[ntc:]:
         assert te <= (sh[fs] if kind == 0 else pl[fs])
