@@ -406,11 +406,10 @@ padoc_status build_parts(const padoc_page *pages, int32_t num_pages, const padoc
                     rate[(size_t)w] = PADOC_WARP_EARLY_RATE;
                 } else {
                     const size_t k = std::min<size_t>((size_t)(c - nfree), tend.size() - 1);
-                    start[(size_t)w] = tend[k] + PADOC_WARP_START_DELAY_US;
+                    start[(size_t)w] = tend[k] + PADOC_WARP_START_DELAY_US + PADOC_WARP_FIRST_US;
                 }
             }
         }
-        for (int32_t w = 0; w < nwarps; ++w) start[(size_t)w] += PADOC_WARP_FIRST_US;
         // T by bisection on sum_w rate_w * max(0, T - start_w) = total
         auto cap_sum = [&](double T) {
             double s = 0.0;

@@ -38,18 +38,18 @@
 // batch (times in microseconds from the start of the tensor-core grid), used to size each warp's
 // share: a tensor-core CTA with a planned load of L units (the weights above) ends at about
 // PADOC_TC_END_US0 + PADOC_TC_US_PER_UNIT * L; a warp CTA on an SM the tensor-core grid leaves free
-// starts at PADOC_WARP_EARLY_START_US, one that waits for a tensor-core CTA starts
-// PADOC_WARP_START_DELAY_US after it ends; a warp then needs PADOC_WARP_FIRST_US before its first
-// block lands and works through PADOC_WARP_RATE cost units (16-token blocks plus
-// PADOC_WARP_ITEM_COST per item) per microsecond, or PADOC_WARP_EARLY_RATE while tensor-core CTAs
-// still run beside it.
+// starts at PADOC_WARP_EARLY_START_US and works through PADOC_WARP_EARLY_RATE cost units (16-token
+// blocks plus PADOC_WARP_ITEM_COST per item) per microsecond; one that waits for a tensor-core CTA
+// starts PADOC_WARP_START_DELAY_US after it ends, needs PADOC_WARP_FIRST_US before its first block
+// lands (the memory system is busiest then) and then works through PADOC_WARP_RATE units per
+// microsecond.
 #define PADOC_TC_END_US0 5.6
 #define PADOC_TC_US_PER_UNIT 0.238
 #define PADOC_WARP_EARLY_START_US 5.2
 #define PADOC_WARP_START_DELAY_US 0.4
-#define PADOC_WARP_FIRST_US 6.3
-#define PADOC_WARP_RATE 1.72
-#define PADOC_WARP_EARLY_RATE 1.2
+#define PADOC_WARP_FIRST_US 5.3
+#define PADOC_WARP_RATE 1.53
+#define PADOC_WARP_EARLY_RATE 1.21
 
 #define PADOC_ITEM_INTS 8
 enum { PADOC_ITEM_SHARED = 0, PADOC_ITEM_PRIVATE = 1, PADOC_ITEM_SHARED_TC = 2 };
