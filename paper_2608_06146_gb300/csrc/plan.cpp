@@ -5,6 +5,7 @@
 // sees [page_begin, page_begin + P + f_k) and [ybase_k, q]. Everything here is exact integer
 // arithmetic; outputs are bit-exact and canonical (see padoc_attn.h).
 #include <algorithm>
+#include <atomic>
 #include <cstdint>
 #include <cstring>
 #include <numeric>
@@ -181,14 +182,26 @@ namespace {
 
 struct Stream { int32_t page, shared_len, private_len; };
 
-// Multiprocessor count of the current CUDA device, or 152 (one GB300) when none is visible.
+// Multiprocessor count of the current CUDA device, or 152 (one GB300) when none is visible; the
+// device attribute is read once per device (a plan is built for every decode step).
 int32_t padoc_default_ctas()
 {
+    constexpr int kMaxDevices = 64;
+    static std::atomic<int32_t> cached[kMaxDevices];   // 0: not read yet
     int dev = 0, n = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n < 1) {
+    if (cudaGetDevice(&dev) != cudaSuccess) {
         cudaGetLastError();
         return 152;
     }
+    if (dev >= 0 && dev < kMaxDevices) {
+        const int32_t c = cached[dev].load(std::memory_order_relaxed);
+        if (c > 0) return c;
+    }
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n < 1) {
+        cudaGetLastError();
+        n = 152;
+    }
+    if (dev >= 0 && dev < kMaxDevices) cached[dev].store(n, std::memory_order_relaxed);
     return n;
 }
 
@@ -391,47 +404,74 @@ padoc_status build_parts(const padoc_page *pages, int32_t num_pages, const padoc
         // up to the work. Taking items longest first, each to the warp with the most capacity left,
         // puts the longest items on the warps that start first. Without tensor-core work every warp
         // starts at once and the capacities are equal.
-        int64_t total = 0;
-        for (int32_t i = 0; i < nitems; ++i) total += cost[(size_t)i];
-        std::vector<double> start((size_t)nwarps, 0.0), rate((size_t)nwarps, PADOC_WARP_RATE);
+        // the warps of a CTA start together: start, rate and warp count per CTA
+        std::vector<double> start((size_t)wctas, 0.0), rate((size_t)wctas, PADOC_WARP_RATE);
+        std::vector<int32_t> nw_of((size_t)wctas);
+        for (int32_t c = 0; c < wctas; ++c)
+            nw_of[(size_t)c] = std::min<int32_t>(PADOC_WARP_KERNEL_WARPS, nwarps - c * PADOC_WARP_KERNEL_WARPS);
         if (!tc_load.empty()) {
             std::vector<double> tend(tc_load.size());
             for (size_t c = 0; c < tc_load.size(); ++c) tend[c] = PADOC_TC_END_US0 + PADOC_TC_US_PER_UNIT * (double)tc_load[c];
             std::sort(tend.begin(), tend.end());
             const int32_t nfree = std::max<int32_t>(0, padoc_default_ctas() - (int32_t)tc_load.size());
-            for (int32_t w = 0; w < nwarps; ++w) {
-                const int32_t c = w / PADOC_WARP_KERNEL_WARPS;
+            for (int32_t c = 0; c < wctas; ++c) {
                 if (c < nfree) {
-                    start[(size_t)w] = PADOC_WARP_EARLY_START_US;
-                    rate[(size_t)w] = PADOC_WARP_EARLY_RATE;
+                    start[(size_t)c] = PADOC_WARP_EARLY_START_US;
+                    rate[(size_t)c] = PADOC_WARP_EARLY_RATE;
                 } else {
                     const size_t k = std::min<size_t>((size_t)(c - nfree), tend.size() - 1);
-                    start[(size_t)w] = tend[k] + PADOC_WARP_START_DELAY_US + PADOC_WARP_FIRST_US;
+                    start[(size_t)c] = tend[k] + PADOC_WARP_START_DELAY_US + PADOC_WARP_FIRST_US;
                 }
             }
         }
-        // T by bisection on sum_w rate_w * max(0, T - start_w) = total
-        auto cap_sum = [&](double T) {
-            double s = 0.0;
-            for (int32_t w = 0; w < nwarps; ++w) s += rate[(size_t)w] * std::max(0.0, T - start[(size_t)w]);
-            return s;
-        };
-        double lo = 0.0, hi = 1.0;
-        while (cap_sum(hi) < (double)total) hi *= 2.0;
-        for (int it = 0; it < 60; ++it) {
-            const double mid = 0.5 * (lo + hi);
-            if (cap_sum(mid) < (double)total) lo = mid; else hi = mid;
+        int64_t total = 0;
+        for (int32_t i = 0; i < nitems; ++i) total += cost[(size_t)i];
+        // T solves sum_c nw_c rate_c max(0, T - start_c) = total, which is piecewise linear in T:
+        // walk the CTAs in order of start, adding each one's slope, until the line reaches total
+        std::vector<int32_t> by_start((size_t)wctas);
+        std::iota(by_start.begin(), by_start.end(), 0);
+        std::sort(by_start.begin(), by_start.end(), [&](int32_t x, int32_t y) { return start[(size_t)x] < start[(size_t)y]; });
+        double T = 0.0, slope = 0.0, icpt = 0.0;   // capacity at T = slope * T - icpt
+        for (size_t j = 0; j < by_start.size(); ++j) {
+            const int32_t c = by_start[j];
+            slope += nw_of[(size_t)c] * rate[(size_t)c];
+            icpt += nw_of[(size_t)c] * rate[(size_t)c] * start[(size_t)c];
+            T = (icpt + (double)total) / slope;
+            if (j + 1 == by_start.size() || T <= start[(size_t)by_start[j + 1]]) break;
         }
-        std::priority_queue<std::pair<double, int32_t>> room;   // (capacity left, -warp)
-        for (int32_t w = 0; w < nwarps; ++w) room.push({rate[(size_t)w] * std::max(0.0, hi - start[(size_t)w]), -w});
+        // Longest item first, each to the warp with the most capacity left (integer cost units). The
+        // largest capacity left never grows, so the warps sit in FIFO buckets by capacity left and a
+        // cursor walks down to the highest non-empty bucket (O(1) per item). A warp's capacity left
+        // never falls more than one item below the largest, so the buckets start at -(longest
+        // item + 2).
+        int64_t max_cost = 0, max_room = 0;
+        for (int32_t i = 0; i < nitems; ++i) max_cost = std::max<int64_t>(max_cost, cost[(size_t)i]);
+        std::vector<int64_t> room((size_t)nwarps);
+        for (int32_t w = 0; w < nwarps; ++w) {
+            const int32_t c = w / PADOC_WARP_KERNEL_WARPS;
+            room[(size_t)w] = (int64_t)(rate[(size_t)c] * std::max(0.0, T - start[(size_t)c]));
+            max_room = std::max(max_room, room[(size_t)w]);
+        }
+        const int64_t off = max_cost + 2, nbuckets = max_room + off + 1;
+        std::vector<int32_t> head((size_t)nbuckets, -1), tail((size_t)nbuckets, -1), next((size_t)nwarps, -1);
+        auto push = [&](int32_t w) {
+            const int64_t b = std::max<int64_t>(0, room[(size_t)w] + off);
+            next[(size_t)w] = -1;
+            if (tail[(size_t)b] < 0) head[(size_t)b] = w; else next[(size_t)tail[(size_t)b]] = w;
+            tail[(size_t)b] = w;
+        };
+        for (int32_t w = 0; w < nwarps; ++w) push(w);
         std::vector<int32_t> warp_of((size_t)nitems);
+        int64_t cur = nbuckets - 1;
         for (int32_t k : order) {
-            auto top = room.top();
-            room.pop();
-            const int32_t w = -top.second;
+            while (head[(size_t)cur] < 0) --cur;
+            const int32_t w = head[(size_t)cur];
+            head[(size_t)cur] = next[(size_t)w];
+            if (head[(size_t)cur] < 0) tail[(size_t)cur] = -1;
             warp_of[(size_t)k] = w;
             ++pp.warp_ptr[(size_t)w + 1];
-            room.push({top.first - (double)cost[(size_t)k], top.second});
+            room[(size_t)w] -= cost[(size_t)k];
+            push(w);
         }
         for (int32_t w = 0; w < nwarps; ++w) pp.warp_ptr[(size_t)w + 1] += pp.warp_ptr[(size_t)w];
         std::vector<int32_t> wpos(pp.warp_ptr.begin(), pp.warp_ptr.end() - 1);
