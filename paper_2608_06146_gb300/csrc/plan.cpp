@@ -205,6 +205,9 @@ int32_t padoc_default_ctas()
     return n;
 }
 
+struct PlanParts;
+int32_t choose_tc_ctas(const PlanParts &pp, const padoc_decode_config *cfg, int64_t total_w, int64_t max_piece);
+
 struct PlanParts {
     std::vector<Stream> streams;
     std::vector<int32_t> page_len, page_first_stream, page_num_streams;
@@ -331,7 +334,7 @@ padoc_status build_parts(const padoc_page *pages, int32_t num_pages, const padoc
     };
     int32_t ctas = 0;
     if (!segs.empty()) {
-        const int64_t want = cfg->tc_ctas > 0 ? cfg->tc_ctas : padoc_default_ctas();
+        const int64_t want = cfg->tc_ctas > 0 ? cfg->tc_ctas : choose_tc_ctas(pp, cfg, total_w, max_piece);
         int64_t lo = max_w + max_piece, hi = total_w + max_w;   // walk(hi) needs one CTA
         while (lo < hi) {
             const int64_t mid = lo + (hi - lo) / 2;
@@ -480,6 +483,59 @@ padoc_status build_parts(const padoc_page *pages, int32_t num_pages, const padoc
     }
     pp.num_warps = nwarps;
     return PADOC_OK;
+}
+
+// How many SMs the tensor-core grid gets when the caller leaves it to the planner. Fewer tensor-core
+// CTAs make that grid run longer but leave SMs to warp CTAs from the start, where they use the
+// memory bandwidth the tensor-core CTAs (bound by their softmax and MMA chain) leave unused. With
+// the timing model above, each candidate count n (the SM count, then down in steps of 8 to half of
+// it) gets a predicted end of step: the tensor-core CTAs end on average at
+// PADOC_TC_END_US0 + PADOC_TC_US_PER_UNIT * (total load / n + one piece) and the last of them
+// PADOC_TC_END_SPREAD_US later, and the warp work, sized to each warp's start as in the planner
+// (warp CTAs that wait for a tensor-core CTA start at the average end), ends at T; the count whose
+// later of the two ends is earliest wins (the larger count on a tie).
+int32_t choose_tc_ctas(const PlanParts &pp, const padoc_decode_config *cfg, int64_t total_w, int64_t max_piece)
+{
+    const int32_t nsm = padoc_default_ctas();
+    const int32_t group = cfg->num_q_heads / cfg->num_kv_heads;
+    const int32_t split = std::min(cfg->split_tokens > 0 ? cfg->split_tokens : PADOC_DEFAULT_SPLIT_TOKENS,
+                                   PADOC_WARP_MAX_ITEM_TOKENS);
+    // the warp work: its items and their cost, as the planner will cut them
+    int64_t wcost = 0, witems = 0;
+    auto add = [&](int32_t len, int32_t step) {
+        for (int32_t tb = 0; tb < len; tb += step) {
+            wcost += (std::min(len, tb + step) - tb + 15) / 16 + PADOC_WARP_ITEM_COST;
+            ++witems;
+        }
+    };
+    for (int32_t g = 0; g < cfg->num_kv_heads; ++g) {
+        for (size_t p = 0; p < pp.page_len.size(); ++p) {
+            const int32_t f0 = pp.page_first_stream[p], ns = pp.page_num_streams[p];
+            if ((int64_t)ns * group >= PADOC_TC_MIN_ROWS) continue;
+            for (int32_t st = f0; st < f0 + ns; ++st) add(pp.streams[(size_t)st].shared_len, split);
+        }
+        for (const Stream &st : pp.streams) add(st.private_len, PADOC_PRIVATE_SPLIT_TOKENS);
+    }
+    const int64_t wctas = std::min<int64_t>(cfg->warp_ctas > 0 ? cfg->warp_ctas : nsm,
+                                            (witems + PADOC_WARP_KERNEL_WARPS - 1) / PADOC_WARP_KERNEL_WARPS);
+    if (wcost == 0 || wctas == 0) return nsm;
+    int32_t best_n = nsm;
+    double best = 1e300;
+    for (int32_t n = nsm; n >= std::max(1, nsm / 2); n -= 8) {
+        const double tc_end = PADOC_TC_END_US0 + PADOC_TC_US_PER_UNIT * ((double)total_w / n + (double)max_piece);
+        const double ne = (double)std::min<int64_t>(std::max(0, nsm - n), wctas), nl = (double)wctas - ne;
+        const double se = PADOC_WARP_EARLY_START_US, sl = tc_end + PADOC_WARP_START_DELAY_US + PADOC_WARP_FIRST_US;
+        const double ae = PADOC_WARP_KERNEL_WARPS * PADOC_WARP_EARLY_RATE * ne, al = PADOC_WARP_KERNEL_WARPS * PADOC_WARP_RATE * nl;
+        // capacity at T: ae (T - se) + al max(0, T - sl) (se < sl); solve for T = the warp work
+        double T = ae > 0 ? se + (double)wcost / ae : 1e300;
+        if (T > sl) T = (ae * se + al * sl + (double)wcost) / (ae + al);
+        const double end = std::max(tc_end + PADOC_TC_END_SPREAD_US, T);
+        if (end < best - 1e-9) {
+            best = end;
+            best_n = n;
+        }
+    }
+    return best_n;
 }
 
 // int32 words of the plan blob: stream_page, shared_len, private_len [S], slot_ptr [S Hkv + 1],

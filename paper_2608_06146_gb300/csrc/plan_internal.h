@@ -45,11 +45,13 @@
 // microsecond.
 #define PADOC_TC_END_US0 5.6
 #define PADOC_TC_US_PER_UNIT 0.238
+// the last tensor-core CTA of a step ends about this long after the average one
+#define PADOC_TC_END_SPREAD_US 2.5
 #define PADOC_WARP_EARLY_START_US 5.2
 #define PADOC_WARP_START_DELAY_US 0.4
 #define PADOC_WARP_FIRST_US 5.3
 #define PADOC_WARP_RATE 1.53
-#define PADOC_WARP_EARLY_RATE 1.21
+#define PADOC_WARP_EARLY_RATE 1.28
 
 #define PADOC_ITEM_INTS 8
 enum { PADOC_ITEM_SHARED = 0, PADOC_ITEM_PRIVATE = 1, PADOC_ITEM_SHARED_TC = 2 };
