@@ -38,7 +38,7 @@ FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustain
 # dram__bytes_read.sum + dram__bytes_write.sum per launch from the ncu captures summarised under
 # profiles/ (None until a capture of the current kernel exists). Decode: one step = the three
 # kernels' captures added up (profiles/decode_*_serving_batch.md), cold caches.
-TRAFFIC_BYTES = {"decode": 230_266_000, "prefill": 260_600_000}   # prefill: profiles/prefill_tc_packed_32k.md
+TRAFFIC_BYTES = {"decode": 227_310_000, "prefill": 260_600_000}   # prefill: profiles/prefill_tc_packed_32k.md
 
 
 def load_peaks():
