@@ -9,7 +9,8 @@ Every function follows the paper's definition of the visibility (Sec. 3.2 ancest
 App. C.1 packed statement; App. E.1 additive-bias softmax and Algorithm 1); the C source states
 the readings taken where the paper is silent. Parity of all functions is pinned by
 tests/test_oracle_pins.py against closed forms, torch's SDPA, a simulator of Algorithm 1's mask
-recurrence and hand-derived fixtures.
+recurrence and hand-derived fixtures; the backward against central differences of the forward,
+torch autograd through the per-branch gather, and closed forms.
 """
 from __future__ import annotations
 
@@ -64,6 +65,10 @@ def _load():
                                          _f64p, _f64p]
             lib.oracle_tile_kinds.argtypes = [_i32p, ctypes.c_int32, _i32p, _i32p, ctypes.c_int32,
                                               ctypes.c_int32, _i8p]
+            lib.oracle_prefill_bwd.argtypes = [_i32p, ctypes.c_int32, _i32p, _i32p, _f32p, _f32p, _f32p,
+                                               _f32p, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32,
+                                               ctypes.c_double, ctypes.c_int64, _i64p, ctypes.c_int64,
+                                               _i64p, _f64p, _f64p, _f64p]
             _lib = lib
     return _lib
 
@@ -189,3 +194,27 @@ def tile_kinds(pages, q_tile: int, k_tile: int) -> np.ndarray:
     _load().oracle_tile_kinds(_ptr(pln, _i32p), n, _ptr(f, _i32p), _ptr(b, _i32p), q_tile, k_tile,
                               _ptr(out, _i8p))
     return out[:nq, :nk]
+
+
+def prefill_bwd(pages, q, k, v, dout, scale, q_rows=None, k_rows=None):
+    """Gradients of the packed prefill for upstream gradient ``dout`` (Sec. 3.2 visibility,
+    App. C.1 scatter-add of shared rows). Returns fp64 (dQ [nq][Hq][d], dK [nk][Hkv][d],
+    dV [nk][Hkv][d]) for the packed query rows ``q_rows`` and key rows ``k_rows`` (default: all)."""
+    pln, n, f, b = _flat(pages)
+    q, k, v, g = _f32(q), _f32(k), _f32(v), _f32(dout)
+    T, Hq, d = q.shape
+    Hkv = k.shape[1]
+    assert k.shape == (T, Hkv, d) and v.shape == (T, Hkv, d) and g.shape == q.shape and Hq % Hkv == 0
+    qs = np.ascontiguousarray(np.arange(T) if q_rows is None else np.asarray(q_rows), np.int64)
+    ks = np.ascontiguousarray(np.arange(T) if k_rows is None else np.asarray(k_rows), np.int64)
+    assert ((qs >= 0) & (qs < T)).all() and ((ks >= 0) & (ks < T)).all()
+    dq = np.zeros((len(qs), Hq, d), np.float64)
+    dk = np.zeros((len(ks), Hkv, d), np.float64)
+    dv = np.zeros((len(ks), Hkv, d), np.float64)
+    guard = lambda a: a if a.size else np.zeros(1, a.dtype)
+    if T:
+        _load().oracle_prefill_bwd(_ptr(pln, _i32p), n, _ptr(f, _i32p), _ptr(b, _i32p), _ptr(q, _f32p),
+                                   _ptr(k, _f32p), _ptr(v, _f32p), _ptr(g, _f32p), Hq, Hkv, d, float(scale),
+                                   len(qs), _ptr(guard(qs), _i64p), len(ks), _ptr(guard(ks), _i64p),
+                                   _ptr(guard(dq), _f64p), _ptr(guard(dk), _f64p), _ptr(guard(dv), _f64p))
+    return dq, dk, dv

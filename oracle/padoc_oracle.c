@@ -25,6 +25,10 @@
  * ("Dense SDPA", the paper's reference implementation), and a per-branch gather of
  * [M_<=f_k ; Y_k] with bottom-right-aligned causal attention ("Tree-varlen").
  *
+ * The backward (oracle_prefill_bwd) is the chain rule of that softmax attention for an upstream
+ * gradient dO: dQ, dK, dV under the same visibility, with every shared-stream key's gradient summed
+ * over all queries that see it (the scatter-add of the tree-varlen gather's backward, App. C.1).
+ *
  * Readings of the paper used here (each also listed in the design notes):
  *   - f_k is the number of layout-stream tokens visible to branch k (Alg. 1 copies the layout
  *     row before the boundary output is appended; Sec. E.1). Any f_k in [0, L], in any order.
@@ -425,4 +429,191 @@ void oracle_tile_kinds(const int32_t *pln, int32_t num_pages, const int32_t *for
         }
     }
     free(pg); free(loc); free(boffs);
+}
+
+/* ------------------------------------------------------------------------------------------ */
+/* Packed prefill backward: gradients of the ancestor-masked attention                          */
+/* ------------------------------------------------------------------------------------------ */
+
+/* The forward of every query row and head is s_j = scale * q.k_j over its visible keys j,
+ * P_j = exp(s_j - lse), O = sum_j P_j v_j (Sec. 3.2 visibility, App. E.1 softmax). For an upstream
+ * gradient dO of O, the chain rule through the softmax gives, per query row and head,
+ *   dP_j = dO . v_j,   D = sum_j P_j dP_j,   dS_j = P_j (dP_j - D),   dQ = scale * sum_j dS_j k_j,
+ * and every key j of KV head g collects over the queries i that see it and the query heads h that
+ * read KV head g:
+ *   dK_j = scale * sum_{i,h} dS_ij q_ih,   dV_j = sum_{i,h} P_ij dO_ih.
+ * A shared-stream key is seen by the stream's later tokens and by every branch forked after it, so
+ * its dK and dV sum over all of them: the scatter-add back onto the shared rows that the backward
+ * of the tree-varlen gather performs (App. C.1). Visibility is the dense ancestor test above; lse
+ * and D are recomputed here in fp64 from the inputs (nothing is taken from a forward output).
+ *
+ * q: [T][Hq][d], k, v: [T][Hkv][d], dout: [T][Hq][d] (packed order, fp32 holding exact values).
+ * Only the selected rows are produced: q_sel[0..nq) (packed query rows) -> dq [nq][Hq][d];
+ * k_sel[0..nk) (packed key rows) -> dk, dv [nk][Hkv][d]. Sums run over keys (dQ) or queries then
+ * heads (dK, dV) in ascending order. */
+
+typedef struct {
+    int32_t *pg;        /* page of each packed token */
+    int64_t *loc;       /* page-local position */
+    int64_t *pbase;     /* first packed token of each page */
+    int64_t *boffs;     /* first branch of each page in fork[] / blen[] */
+    int64_t *ptok;      /* tokens of each page */
+} page_index;
+
+static void page_index_build(const int32_t *pln, int32_t num_pages, const int32_t *blen, int64_t T, page_index *ix)
+{
+    ix->pg = (int32_t *)malloc(sizeof(int32_t) * (size_t)(T > 0 ? T : 1));
+    ix->loc = (int64_t *)malloc(sizeof(int64_t) * (size_t)(T > 0 ? T : 1));
+    ix->pbase = (int64_t *)malloc(sizeof(int64_t) * (size_t)(num_pages > 0 ? num_pages : 1));
+    ix->boffs = (int64_t *)malloc(sizeof(int64_t) * (size_t)(num_pages > 0 ? num_pages : 1));
+    ix->ptok = (int64_t *)malloc(sizeof(int64_t) * (size_t)(num_pages > 0 ? num_pages : 1));
+    int64_t t = 0, boff = 0;
+    for (int p = 0; p < num_pages; ++p) {
+        ix->pbase[p] = t;
+        ix->boffs[p] = boff;
+        ix->ptok[p] = page_tokens(pln, blen, boff, p);
+        for (int64_t i = 0; i < ix->ptok[p]; ++i) { ix->pg[t] = p; ix->loc[t] = i; ++t; }
+        boff += pln[3 * p + 2];
+    }
+}
+
+static void page_index_free(page_index *ix)
+{
+    free(ix->pg); free(ix->loc); free(ix->pbase); free(ix->boffs); free(ix->ptok);
+}
+
+static double dot_fd(const float *a, const float *b, int d)
+{
+    double acc = 0.0;
+    for (int c = 0; c < d; ++c) acc += (double)a[c] * (double)b[c];
+    return acc;
+}
+
+/* Softmax statistics of query (page p, local qi), head h: lse and D = sum_j P_j dP_j. With dq
+ * non-null, also dq[c] = scale * sum_j dS_j k_j[c]. sbuf/pbuf: scratch of the page's size. */
+static void row_backward(const int32_t *pln, const int32_t *fork, const int32_t *blen, const page_index *ix, int p,
+                         int64_t qi, int h, const float *q, const float *k, const float *v, const float *dout,
+                         int32_t Hq, int32_t Hkv, int32_t d, double scale, int64_t *vis, double *sbuf,
+                         double *dpbuf, double *lse_out, double *D_out, double *dq)
+{
+    const int32_t *pp = pln + 3 * p;
+    const int32_t *fk = fork + ix->boffs[p], *bl = blen + ix->boffs[p];
+    const int64_t S = ix->ptok[p], pb = ix->pbase[p];
+    const int g = h / (Hq / Hkv);
+    const float *qr = q + ((pb + qi) * Hq + h) * d;
+    const float *gr = dout + ((pb + qi) * Hq + h) * d;
+    int64_t nv = 0;
+    double mx = -INFINITY;
+    for (int64_t j = 0; j < S; ++j) {
+        if (!visible_by_ancestors(pp, fk, bl, qi, j)) continue;
+        vis[nv] = j;
+        sbuf[nv] = scale * dot_fd(qr, k + ((pb + j) * Hkv + g) * d, d);
+        if (sbuf[nv] > mx) mx = sbuf[nv];
+        ++nv;
+    }
+    double sum = 0.0;
+    for (int64_t c = 0; c < nv; ++c) sum += exp(sbuf[c] - mx);
+    const double lse = nv ? mx + log(sum) : -INFINITY;
+    double D = 0.0;
+    for (int64_t c = 0; c < nv; ++c) {
+        sbuf[c] = exp(sbuf[c] - lse);                                   /* P_j */
+        dpbuf[c] = dot_fd(gr, v + ((pb + vis[c]) * Hkv + g) * d, d);    /* dP_j */
+        D += sbuf[c] * dpbuf[c];
+    }
+    *lse_out = lse;
+    *D_out = D;
+    if (dq) {
+        for (int c = 0; c < d; ++c) dq[c] = 0.0;
+        for (int64_t c = 0; c < nv; ++c) {
+            const double ds = sbuf[c] * (dpbuf[c] - D);
+            const float *kr = k + ((pb + vis[c]) * Hkv + g) * d;
+            for (int e = 0; e < d; ++e) dq[e] += ds * (double)kr[e];
+        }
+        for (int c = 0; c < d; ++c) dq[c] *= scale;
+    }
+}
+
+void oracle_prefill_bwd(const int32_t *pln, int32_t num_pages, const int32_t *fork, const int32_t *blen,
+                        const float *q, const float *k, const float *v, const float *dout, int32_t Hq, int32_t Hkv,
+                        int32_t d, double scale, int64_t nq, const int64_t *q_sel, int64_t nk, const int64_t *k_sel,
+                        double *dq, double *dk, double *dv)
+{
+    const int64_t T = oracle_total_tokens(pln, num_pages, blen);
+    page_index ix;
+    page_index_build(pln, num_pages, blen, T, &ix);
+    int64_t smax = 1;
+    for (int p = 0; p < num_pages; ++p) if (ix.ptok[p] > smax) smax = ix.ptok[p];
+
+    /* dQ of the selected query rows */
+#pragma omp parallel
+    {
+        int64_t *vis = (int64_t *)malloc(sizeof(int64_t) * (size_t)smax);
+        double *sb = (double *)malloc(sizeof(double) * (size_t)smax);
+        double *db = (double *)malloc(sizeof(double) * (size_t)smax);
+#pragma omp for collapse(2) schedule(dynamic, 4)
+        for (int64_t r = 0; r < nq; ++r) {
+            for (int h = 0; h < Hq; ++h) {
+                const int64_t t = q_sel[r];
+                double lse, D;
+                row_backward(pln, fork, blen, &ix, ix.pg[t], ix.loc[t], h, q, k, v, dout, Hq, Hkv, d, scale, vis, sb,
+                             db, &lse, &D, dq + (r * Hq + h) * d);
+            }
+        }
+        free(vis); free(sb); free(db);
+    }
+
+    /* dK, dV of the selected key rows: the softmax statistics of every query of a touched page */
+    uint8_t *touched = (uint8_t *)calloc((size_t)(num_pages > 0 ? num_pages : 1), 1);
+    for (int64_t r = 0; r < nk; ++r) touched[ix.pg[k_sel[r]]] = 1;
+    double *lse_all = (double *)malloc(sizeof(double) * (size_t)(T > 0 ? T : 1) * (size_t)Hq);
+    double *D_all = (double *)malloc(sizeof(double) * (size_t)(T > 0 ? T : 1) * (size_t)Hq);
+    for (int p = 0; p < num_pages; ++p) {
+        if (!touched[p]) continue;
+        const int64_t S = ix.ptok[p];
+#pragma omp parallel
+        {
+            int64_t *vis = (int64_t *)malloc(sizeof(int64_t) * (size_t)smax);
+            double *sb = (double *)malloc(sizeof(double) * (size_t)smax);
+            double *db = (double *)malloc(sizeof(double) * (size_t)smax);
+#pragma omp for collapse(2) schedule(dynamic, 4)
+            for (int64_t qi = 0; qi < S; ++qi) {
+                for (int h = 0; h < Hq; ++h) {
+                    const int64_t row = (ix.pbase[p] + qi) * Hq + h;
+                    row_backward(pln, fork, blen, &ix, p, qi, h, q, k, v, dout, Hq, Hkv, d, scale, vis, sb, db,
+                                 &lse_all[row], &D_all[row], NULL);
+                }
+            }
+            free(vis); free(sb); free(db);
+        }
+    }
+    const int group = Hq / Hkv;
+#pragma omp parallel for collapse(2) schedule(dynamic, 1)
+    for (int64_t r = 0; r < nk; ++r) {
+        for (int g = 0; g < Hkv; ++g) {
+            const int64_t t = k_sel[r];
+            const int p = ix.pg[t];
+            const int64_t j = ix.loc[t], pb = ix.pbase[p], S = ix.ptok[p];
+            const int32_t *pp = pln + 3 * p;
+            const int32_t *fk = fork + ix.boffs[p], *bl = blen + ix.boffs[p];
+            const float *kr = k + (t * Hkv + g) * d, *vr = v + (t * Hkv + g) * d;
+            double *dkr = dk + (r * Hkv + g) * d, *dvr = dv + (r * Hkv + g) * d;
+            for (int c = 0; c < d; ++c) { dkr[c] = 0.0; dvr[c] = 0.0; }
+            for (int64_t qi = 0; qi < S; ++qi) {
+                if (!visible_by_ancestors(pp, fk, bl, qi, j)) continue;
+                for (int h = g * group; h < (g + 1) * group; ++h) {
+                    const int64_t row = (pb + qi) * Hq + h;
+                    const float *qr = q + row * d, *gr = dout + row * d;
+                    const double pij = exp(scale * dot_fd(qr, kr, d) - lse_all[row]);
+                    const double ds = pij * (dot_fd(gr, vr, d) - D_all[row]);
+                    for (int c = 0; c < d; ++c) {
+                        dkr[c] += ds * (double)qr[c];
+                        dvr[c] += pij * (double)gr[c];
+                    }
+                }
+            }
+            for (int c = 0; c < d; ++c) dkr[c] *= scale;
+        }
+    }
+    free(touched); free(lse_all); free(D_all);
+    page_index_free(&ix);
 }

@@ -13,6 +13,9 @@ Each test ties one oracle function to something the paper or the mathematics fix
     disjoint key sets);
   * decode of a branch's newest token equals the matching prefill row (Algorithm 1 appends before
     it decodes).
+  * the backward: central differences of the forward, torch autograd through the per-branch
+    gather (whose backward scatter-adds onto the shared rows, App. C.1), the page sums that the
+    softmax fixes (sum of dK is zero, sum of dV is the sum of dO) and the K = 0 closed form.
 """
 import math
 import os
@@ -343,3 +346,176 @@ def test_dense_and_gather_agree_on_workload_shapes():
     b = oracle.prefill_gather(pages, q, k, v, 0.25)
     np.testing.assert_allclose(a[0], b[0], rtol=0, atol=1e-12)
     np.testing.assert_allclose(a[1], b[1], rtol=0, atol=1e-12)
+
+
+# --------------------------------------------------------------------------------------------
+# Backward (gradients of the packed prefill)
+# --------------------------------------------------------------------------------------------
+
+def _grid_inputs(rng, T, Hq, Hkv, d, step=2.0 ** -12):
+    """Inputs on a 2^-12 grid in [-1, 1): x +- 2^-10 stays exact in fp32, so central differences
+    of the fp64 forward see exactly the perturbed values."""
+    f = lambda *s: (np.round(rng.uniform(-1, 1, s) / step) * step).astype(np.float32)
+    return f(T, Hq, d), f(T, Hkv, d), f(T, Hkv, d), f(T, Hq, d)
+
+
+def test_prefill_bwd_matches_central_differences_of_forward():
+    """dQ, dK, dV are the derivatives of L = sum(dO * O) with O from the (separately pinned)
+    forward: central differences with h = 2^-10 (error O(h^2) ~ 1e-6)."""
+    pages = [(3, 2, [1, 2], [2, 1]), (2, 1, [0], [2])]
+    rng = np.random.default_rng(7)
+    T = oracle.total_tokens(pages)
+    Hq, Hkv, d, scale = 4, 2, 3, 0.7
+    q, k, v, g = _grid_inputs(rng, T, Hq, Hkv, d)
+    dq, dk, dv = oracle.prefill_bwd(pages, q, k, v, g, scale)
+    h = 2.0 ** -10
+
+    def loss(qq, kk, vv):
+        o, _ = oracle.prefill_dense(pages, qq, kk, vv, scale)
+        return float((o * g.astype(np.float64)).sum())
+
+    for name, arr, got in (("q", q, dq), ("k", k, dk), ("v", v, dv)):
+        fd = np.zeros(arr.shape)
+        for idx in np.ndindex(arr.shape):
+            a = arr.copy(); a[idx] += np.float32(h)
+            b = arr.copy(); b[idx] -= np.float32(h)
+            args = {"q": (q, k, v), "k": (q, k, v), "v": (q, k, v)}[name]
+            pa = [a if x is arr else x for x in args]
+            pb = [b if x is arr else x for x in args]
+            fd[idx] = (loss(*pa) - loss(*pb)) / (2 * h)
+        np.testing.assert_allclose(got, fd, rtol=0, atol=2e-5 * max(1.0, np.abs(fd).max()), err_msg=name)
+
+
+def _gather_autograd(pages, q, k, v, g, scale):
+    """The paper's tree-varlen formulation in torch fp64 with autograd: the shared stream is one
+    causal problem; branch k gathers [M_<P+f_k ; Y_k] with index_select and runs bottom-right
+    causal attention; the gather's backward scatter-adds onto the shared rows (App. C.1). The
+    masks are built here from (P, L, f, n) alone."""
+    Q = torch.tensor(q, dtype=torch.float64, requires_grad=True)
+    K = torch.tensor(k, dtype=torch.float64, requires_grad=True)
+    V = torch.tensor(v, dtype=torch.float64, requires_grad=True)
+    G = torch.tensor(g, dtype=torch.float64)
+    T, Hq, d = q.shape
+    rep = Hq // k.shape[1]
+    out = torch.zeros(T, Hq, d, dtype=torch.float64)
+
+    def attend(qrows, krows, n_q, n_k):
+        qq = Q.index_select(0, qrows).transpose(0, 1)                           # [Hq, n_q, d]
+        kk = K.index_select(0, krows).repeat_interleave(rep, 1).transpose(0, 1)  # [Hq, n_k, d]
+        vv = V.index_select(0, krows).repeat_interleave(rep, 1).transpose(0, 1)
+        i = torch.arange(n_q)[:, None]
+        j = torch.arange(n_k)[None, :]
+        allowed = j <= i + (n_k - n_q)                                           # bottom-right causal
+        s = (qq @ kk.transpose(1, 2)) * scale
+        s = s.masked_fill(~allowed, float("-inf"))
+        return (torch.softmax(s, -1) @ vv).transpose(0, 1)
+
+    base = 0
+    for P, L, f, n in pages:
+        M = P + L
+        rows = []
+        if M:
+            idx = torch.arange(base, base + M)
+            rows.append((idx, attend(idx, idx, M, M)))
+        y = base + M
+        for fk, nk in zip(f, n):
+            qi = torch.arange(y, y + nk)
+            ki = torch.cat([torch.arange(base, base + P + fk), qi])
+            rows.append((qi, attend(qi, ki, nk, P + fk + nk)))
+            y += nk
+        for idx, o in rows:
+            out = out.index_put((idx,), o)
+        base = y
+    (out * G).sum().backward()
+    return Q.grad.numpy(), K.grad.numpy(), V.grad.numpy()
+
+
+@pytest.mark.parametrize("seed", range(6))
+def test_prefill_bwd_matches_torch_autograd_of_gather(seed):
+    rng = np.random.default_rng(100 + seed)
+    pages = [_rand_page(rng, P_max=12, L_max=8, N_max=4, n_max=5) for _ in range(3)]
+    T = oracle.total_tokens(pages)
+    Hq, Hkv, d = [(2, 1, 8), (4, 2, 4), (6, 3, 5)][seed % 3]
+    q = rng.standard_normal((T, Hq, d)).astype(np.float32)
+    k = rng.standard_normal((T, Hkv, d)).astype(np.float32)
+    v = rng.standard_normal((T, Hkv, d)).astype(np.float32)
+    g = rng.standard_normal((T, Hq, d)).astype(np.float32)
+    scale = 1 / math.sqrt(d)
+    dq, dk, dv = oracle.prefill_bwd(pages, q, k, v, g, scale)
+    tq, tk, tv = _gather_autograd(pages, q, k, v, g, scale)
+    for got, want in ((dq, tq), (dk, tk), (dv, tv)):
+        np.testing.assert_allclose(got, want, rtol=1e-10, atol=1e-11)
+
+
+def test_prefill_bwd_page_sums_and_first_token():
+    """Per page and KV head: sum_j dK_j = 0 (every query's dS row sums to zero) and
+    sum_j dV_j = sum of the group's dO rows (every query's P row sums to one); a page's first
+    token sees only itself, so its dQ is zero."""
+    rng = np.random.default_rng(5)
+    pages = [(9, 6, [2, 6, 0], [4, 3, 2]), (1, 0, [], []), (5, 3, [3, 1], [1, 6])]
+    T = oracle.total_tokens(pages)
+    Hq, Hkv, d = 4, 2, 6
+    q = rng.standard_normal((T, Hq, d)).astype(np.float32)
+    k = rng.standard_normal((T, Hkv, d)).astype(np.float32)
+    v = rng.standard_normal((T, Hkv, d)).astype(np.float32)
+    g = rng.standard_normal((T, Hq, d)).astype(np.float32)
+    dq, dk, dv = oracle.prefill_bwd(pages, q, k, v, g, 0.5)
+    base = 0
+    for P, L, f, n in pages:
+        S = P + L + sum(n)
+        sl = slice(base, base + S)
+        np.testing.assert_allclose(dk[sl].sum(0), 0.0, atol=1e-12)
+        want = g[sl].astype(np.float64).reshape(S, Hkv, Hq // Hkv, d).sum((0, 2))
+        np.testing.assert_allclose(dv[sl].sum(0), want, rtol=1e-12, atol=1e-12)
+        np.testing.assert_array_equal(dq[base], 0.0)
+        base += S
+
+
+def test_prefill_bwd_zero_keys_closed_form():
+    """K = 0 makes every visible weight 1/n_i: dV_j = sum over queries i that see j of dO_i / n_i
+    (summed over the group's heads), dQ = 0, and
+    dK_j = scale * sum_i (1/n_i) (dO_i.v_j - mean over i's visible keys of dO_i.v) q_i."""
+    rng = np.random.default_rng(11)
+    pages = [(6, 4, [4, 1], [3, 2]), (3, 2, [2], [3])]
+    T = oracle.total_tokens(pages)
+    Hq, Hkv, d, scale = 2, 1, 5, 0.3
+    q = rng.standard_normal((T, Hq, d)).astype(np.float32)
+    k = np.zeros((T, Hkv, d), np.float32)
+    v = rng.standard_normal((T, Hkv, d)).astype(np.float32)
+    g = rng.standard_normal((T, Hq, d)).astype(np.float32)
+    dq, dk, dv = oracle.prefill_bwd(pages, q, k, v, g, scale)
+    sp = oracle.spans(pages)
+    vis = np.zeros((T, T), bool)
+    for t in range(T):
+        vis[t, sp[t, 0]:sp[t, 1]] = True
+        vis[t, sp[t, 2]:sp[t, 3]] = True
+    n = vis.sum(1)
+    q64, v64, g64 = (x.astype(np.float64) for x in (q, v, g))
+    want_dv = np.zeros((T, Hkv, d))
+    want_dk = np.zeros((T, Hkv, d))
+    for i in range(T):
+        for h in range(Hq):
+            dp = v64[:, 0, :] @ g64[i, h]                 # dO_i . v_j for every j
+            mean = dp[vis[i]].mean()
+            for j in np.nonzero(vis[i])[0]:
+                want_dv[j, 0] += g64[i, h] / n[i]
+                want_dk[j, 0] += scale * (dp[j] - mean) / n[i] * q64[i, h]
+    np.testing.assert_array_equal(dq, 0.0)
+    np.testing.assert_allclose(dv, want_dv, rtol=1e-12, atol=1e-13)
+    np.testing.assert_allclose(dk, want_dk, rtol=1e-10, atol=1e-12)
+
+
+def test_prefill_bwd_row_selection_matches_full():
+    rng = np.random.default_rng(3)
+    pages = [(7, 4, [1, 4], [3, 2]), (4, 2, [2, 0], [2, 2])]
+    T = oracle.total_tokens(pages)
+    q = rng.standard_normal((T, 2, 4)).astype(np.float32)
+    k = rng.standard_normal((T, 1, 4)).astype(np.float32)
+    v = rng.standard_normal((T, 1, 4)).astype(np.float32)
+    g = rng.standard_normal((T, 2, 4)).astype(np.float32)
+    full = oracle.prefill_bwd(pages, q, k, v, g, 0.5)
+    qr, kr = [T - 1, 0, 5, 12], [3, T - 2, 0]
+    part = oracle.prefill_bwd(pages, q, k, v, g, 0.5, q_rows=qr, k_rows=kr)
+    np.testing.assert_array_equal(part[0], full[0][qr])
+    np.testing.assert_array_equal(part[1], full[1][kr])
+    np.testing.assert_array_equal(part[2], full[2][kr])
