@@ -119,6 +119,26 @@ padoc_status padoc_tile_map_size(const padoc_page *pages, int32_t num_pages, int
 padoc_status padoc_build_tile_map(const padoc_page *pages, int32_t num_pages, int32_t q_tile, int32_t k_tile,
                                   int32_t *row_ptr, int32_t *k_tiles, int8_t *kinds, int64_t capacity_nnz);
 
+/* Key-major (CSC) form of the same work list, for the dK/dV pass of the prefill backward, where
+ * every key's gradient sums over all queries that see it (App. C.1: the backward of the
+ * tree-varlen gather scatter-adds onto the shared rows). For k-tile c, entries
+ * [col_ptr[c], col_ptr[c+1]) list the q-tiles holding a visible pair in ascending order, with the
+ * kinds padoc_build_tile_map gives the same (q-tile, k-tile) pair. k_order lists every k-tile once,
+ * those with more entries first (ties in ascending order): the order the dK/dV pass takes them.
+ * col_ptr: (host) int32 [ceil(T / k_tile) + 1]; q_tiles: (host) int32 [capacity_nnz];
+ * kinds: (host) int8 [capacity_nnz]; k_order: (host) int32 [ceil(T / k_tile)].
+ * nnz is the one padoc_tile_map_size reports. Errors: INVALID_ARGUMENT; CAPACITY. */
+padoc_status padoc_build_key_tile_map(const padoc_page *pages, int32_t num_pages, int32_t q_tile, int32_t k_tile,
+                                      int32_t *col_ptr, int32_t *q_tiles, int8_t *kinds, int32_t *k_order,
+                                      int64_t capacity_nnz);
+
+/* Tile shapes the prefill backward for (dtype, head_dim) consumes: the dQ pass reads a query-major
+ * map (padoc_build_tile_map) of dq_q_tile x dq_k_tile tiles, the dK/dV pass a key-major map
+ * (padoc_build_key_tile_map) of dkv_q_tile x dkv_k_tile tiles. Errors: INVALID_ARGUMENT,
+ * UNSUPPORTED. */
+padoc_status padoc_prefill_bwd_tile_shapes(padoc_dtype dtype, int32_t head_dim, int32_t *dq_q_tile,
+                                           int32_t *dq_k_tile, int32_t *dkv_q_tile, int32_t *dkv_k_tile);
+
 /* ============================================================================================
  * C5 + C2 + C4: paged KV cache and one decode step for every live stream (App. E.1, Alg. 1)
  * ========================================================================================== */
@@ -279,6 +299,48 @@ padoc_status padoc_ancestor_prefill_attn(const void *q, const void *k, const voi
                                          const int32_t *tile_row_ptr_dev, const int32_t *tile_k_dev,
                                          const int8_t *tile_kind_dev, int32_t q_tile, int32_t k_tile,
                                          float scale, void *out, float *lse, padoc_stream_t stream);
+
+/* ============================================================================================
+ * Prefill backward: gradients of C3 (training backward of the tree-varlen attention)
+ * ========================================================================================== */
+
+/* A tile map in device memory (host struct of device pointers). Query-major maps come from
+ * padoc_build_tile_map (ptr = row_ptr, idx = k_tiles, order = NULL); key-major maps from
+ * padoc_build_key_tile_map (ptr = col_ptr, idx = q_tiles, order = k_order). */
+typedef struct {
+    const int32_t *ptr;
+    const int32_t *idx;
+    const int8_t *kind;
+    const int32_t *order;
+    int32_t q_tile, k_tile;
+} padoc_tile_map_dev;
+
+/* Workspace of padoc_ancestor_prefill_bwd: two fp32 arrays [Hq][ceil(T/128)*128] (the forward's
+ * log-sum-exp in base 2 and D = rowsum(dO * O) per head), 256-byte aligned. */
+padoc_status padoc_prefill_bwd_workspace_size(int64_t total_tokens, int32_t num_q_heads, size_t *bytes);
+
+/* Gradients of the packed ancestor prefill for an upstream gradient dO (App. C.1; Sec. 3.2
+ * visibility). Per query row and head, with P_j = exp(scale * q.k_j - lse) over the visible keys:
+ *   D = sum_c dO[c] O[c],  dS_j = P_j (dO.v_j - D),  dQ = scale * sum_j dS_j k_j;
+ * every key of KV head g collects over the queries that see it and the query heads reading g:
+ *   dK_j = scale * sum dS_ij q_i,  dV_j = sum P_ij dO_i,
+ * so a shared-stream key's gradient sums over the stream's later tokens and over every branch
+ * forked after it (the scatter-add of the gather's backward), with no gather and no atomics.
+ *   q, out, dout: (device) [T][Hq][head_dim]; k, v: (device) [T][Hkv][head_dim]; all in dtype,
+ *   16-byte aligned; out and lse are the forward's outputs (lse natural log, fp32 [T][Hq]).
+ *   spans_dev: (device) int32 [T][4] from padoc_build_query_spans.
+ *   q_map: query-major map, k_map: key-major map, built with padoc_prefill_bwd_tile_shapes.
+ *   dq: (device) [T][Hq][head_dim]; dk, dv: (device) [T][Hkv][head_dim]; in dtype. Every row is
+ *   written (a key no query sees would get zeros; in the packed layout every token sees itself).
+ *   workspace: (device) padoc_prefill_bwd_workspace_size bytes, 256-byte aligned.
+ * bf16 path: head_dim 128, tensor cores. f32 path: head_dim 64 or 128 (bring-up, CUDA cores).
+ * Errors: INVALID_ARGUMENT, UNSUPPORTED, WORKSPACE_TOO_SMALL, CUDA. */
+padoc_status padoc_ancestor_prefill_bwd(const void *q, const void *k, const void *v, const void *out,
+                                        const void *dout, const float *lse, padoc_dtype dtype, int64_t total_tokens,
+                                        int32_t num_q_heads, int32_t num_kv_heads, int32_t head_dim,
+                                        const int32_t *spans_dev, const padoc_tile_map_dev *q_map,
+                                        const padoc_tile_map_dev *k_map, float scale, void *dq, void *dk, void *dv,
+                                        void *workspace, size_t workspace_bytes, padoc_stream_t stream);
 
 /* ============================================================================================
  * Status

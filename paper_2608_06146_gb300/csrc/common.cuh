@@ -134,6 +134,15 @@ __device__ __forceinline__ void tma_load_4d(uint32_t dst, const CUtensorMap *map
         : "memory");
 }
 
+// Contiguous bulk copy global -> shared (both addresses 16-byte aligned, bytes a multiple of 16),
+// completion on an mbarrier.
+__device__ __forceinline__ void bulk_load(uint32_t dst, const void *src, uint32_t bytes, uint32_t bar)
+{
+    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
+                 "l"(src), "r"(bytes), "r"(bar)
+                 : "memory");
+}
+
 // Pulls a 2-D box into L2 without a destination or completion signal (out-of-range parts fetch nothing).
 __device__ __forceinline__ void tma_prefetch_l2_2d(const CUtensorMap *map, int32_t c0, int32_t c1)
 {
@@ -279,6 +288,13 @@ padoc_status padoc_launch_decode_tc(const CUtensorMap *kmap, const CUtensorMap *
                                     const padoc_decode_plan *info, const int32_t *page_table, int32_t page_stride,
                                     int32_t num_blocks, float *part_o, float *part_lse, float scale_log2, int *err,
                                     cudaStream_t stream);
+// tcgen05 prefill backward (prefill_bwd_tc.cu): the dK/dV pass and the dQ pass; arguments validated
+// by the caller. lt / dt: [Hq][t_pad] base-2 log-sum-exp and rowsum(dO * O).
+padoc_status padoc_launch_prefill_bwd_tc(const void *q, const void *k, const void *v, const void *dout,
+                                         int64_t total_tokens, int32_t num_q_heads, int32_t num_kv_heads,
+                                         const int32_t *spans_dev, const padoc_tile_map_dev *q_map,
+                                         const padoc_tile_map_dev *k_map, const float *lt, const float *dt,
+                                         int64_t t_pad, float scale, void *dq, void *dk, void *dv, cudaStream_t stream);
 int padoc_num_sms();
 
 #define PADOC_CUDA_TRY(expr)                                   \

@@ -174,6 +174,55 @@ extern "C" padoc_status padoc_build_tile_map(const padoc_page *pages, int32_t nu
     return PADOC_OK;
 }
 
+extern "C" padoc_status padoc_build_key_tile_map(const padoc_page *pages, int32_t num_pages, int32_t q_tile,
+                                                 int32_t k_tile, int32_t *col_ptr, int32_t *q_tiles, int8_t *kinds,
+                                                 int32_t *k_order, int64_t capacity_nnz)
+{
+    int64_t T = 0;
+    padoc_status st = validate_pages(pages, num_pages, &T);
+    if (st != PADOC_OK) return st;
+    if (q_tile < 1 || k_tile < 1 || !col_ptr || !k_order) return PADOC_ERR_INVALID_ARGUMENT;
+    std::vector<int32_t> spans((size_t)std::max<int64_t>(T, 1) * 4);
+    fill_spans(pages, num_pages, spans.data());
+    const int64_t nkt = (T + k_tile - 1) / k_tile;
+    std::vector<int64_t> cnt((size_t)nkt + 1, 0);
+    int64_t n = 0;
+    walk_tiles(spans.data(), T, q_tile, k_tile, [&](int64_t, int32_t kt, int8_t) { ++cnt[(size_t)kt + 1]; ++n; });
+    if (n > capacity_nnz) return PADOC_ERR_CAPACITY;
+    if (n > 0 && (!q_tiles || !kinds)) return PADOC_ERR_INVALID_ARGUMENT;
+    for (int64_t c = 0; c < nkt; ++c) cnt[(size_t)c + 1] += cnt[(size_t)c];
+    for (int64_t c = 0; c <= nkt; ++c) col_ptr[c] = (int32_t)cnt[(size_t)c];
+    // the walk visits q-tiles in ascending order, so each column's entries come out ascending
+    std::vector<int64_t> fill(cnt.begin(), cnt.end() - 1);
+    walk_tiles(spans.data(), T, q_tile, k_tile, [&](int64_t qt, int32_t kt, int8_t kind) {
+        const int64_t e = fill[(size_t)kt]++;
+        q_tiles[e] = (int32_t)qt;
+        kinds[e] = kind;
+    });
+    // processing order: most entries first (a k-tile's work grows with the q-tiles that see it)
+    std::vector<int32_t> ord((size_t)nkt);
+    std::iota(ord.begin(), ord.end(), 0);
+    std::stable_sort(ord.begin(), ord.end(), [&](int32_t a, int32_t b) {
+        return col_ptr[a + 1] - col_ptr[a] > col_ptr[b + 1] - col_ptr[b];
+    });
+    std::copy(ord.begin(), ord.end(), k_order);
+    return PADOC_OK;
+}
+
+extern "C" padoc_status padoc_prefill_bwd_tile_shapes(padoc_dtype dtype, int32_t head_dim, int32_t *dq_q_tile,
+                                                      int32_t *dq_k_tile, int32_t *dkv_q_tile, int32_t *dkv_k_tile)
+{
+    if (!dq_q_tile || !dq_k_tile || !dkv_q_tile || !dkv_k_tile) return PADOC_ERR_INVALID_ARGUMENT;
+    const bool ok = (dtype == PADOC_DTYPE_BF16 && head_dim == 128) ||
+                    (dtype == PADOC_DTYPE_F32 && (head_dim == 64 || head_dim == 128));
+    if (!ok) return PADOC_ERR_UNSUPPORTED;
+    *dq_q_tile = PADOC_BWD_DQ_Q_TILE;
+    *dq_k_tile = PADOC_BWD_DQ_K_TILE;
+    *dkv_q_tile = PADOC_BWD_DKV_Q_TILE;
+    *dkv_k_tile = PADOC_BWD_DKV_K_TILE;
+    return PADOC_OK;
+}
+
 // ------------------------------------------------------------------------------------------------
 // Decode plan
 // ------------------------------------------------------------------------------------------------

@@ -8,6 +8,15 @@
 #define PADOC_PREFILL_Q_TILE 128
 #define PADOC_PREFILL_K_TILE 128
 
+// Prefill backward tiles. The dQ pass keeps 128 query rows (the M of its MMAs) and walks 64-key
+// k-tiles; the dK/dV pass keeps 128 keys (the M of its MMAs) and walks 64-row q-tiles. 64-wide
+// steps let two steps' scores sit in tensor memory beside the accumulators, so the exponentials
+// of one step overlap the MMAs of the next.
+#define PADOC_BWD_DQ_Q_TILE 128
+#define PADOC_BWD_DQ_K_TILE 64
+#define PADOC_BWD_DKV_Q_TILE 64
+#define PADOC_BWD_DKV_K_TILE 128
+
 // Decode split-K: shared-stream tokens per partial result and private tokens per partial result.
 #define PADOC_DEFAULT_SPLIT_TOKENS 512
 // Longest warp item: a warp keeps one block id per lane, so an item spans at most 32 blocks.

@@ -1,0 +1,626 @@
+// prefill_bwd_tc.cu -- gradients of the packed ancestor prefill on the 5th-generation tensor cores
+// (App. C.1: the backward of the tree-varlen attention; Sec. 3.2 visibility), in two passes that
+// need neither a gather nor atomics.
+//
+// With c = scale * log2(e), lse2 = lse * log2(e) and D = rowsum(dO * O) per query row and head
+// (both precomputed per head, [Hq][t_pad], padded rows lse2 = +inf so that their P is 0):
+//   P = exp2(S c - lse2),  dS = P (dP - D),  S = Q K^T,  dP = dO V^T.
+//
+// dK/dV pass: one CTA per (128-key k-tile, KV head), k-tiles taken in the key-major map's order
+//   (most work first). The CTA walks every (64-row q-tile that sees the k-tile, query head reading
+//   the KV head) step: S^T = K Q^T and dP^T = V dO^T (M = 128 keys, N = 64 queries), the softmax
+//   warps write P^T and dS^T back into tensor memory as bf16, and dV += P^T dO, dK += dS^T Q
+//   accumulate in tensor memory over the whole walk. Every query that sees a shared-stream key
+//   (the stream's later tokens and each branch forked after it) therefore adds into that key's
+//   gradient inside one CTA: the scatter-add of the gather's backward, with nothing scattered.
+// dQ pass: one CTA per (128-row q-tile, query head), heavier q-tiles first. It walks the query-major
+//   map of 64-key k-tiles: S = Q K^T, dP = dO V^T, dS written back as bf16, dQ += dS K.
+//
+// Both passes keep two steps' scores in tensor memory: columns [0,128) hold S (or S^T) of steps
+// with parity 0 / 1 at 0 / 64, [128,256) dP likewise, [256,512) the accumulators. While the
+// softmax warps turn step u into P and dS, the tensor cores run step u-1's accumulating MMAs and
+// step u+1's S and dP. A softmax warp owns 32 TMEM lanes (rows) and one 32-column half of a
+// 64-wide step and packs its 32 bf16 results into the first 16 columns of its own half, so no warp
+// overwrites a column another warp still has to read; the accumulating MMAs read the 64-wide
+// operand as k-slices at columns {0, 8, 32, 40}.
+//
+// Warp roles (320 threads): warps 0-7 softmax and epilogue, warp 8 TMA producer, warp 9 TMEM
+// allocation and MMA issue (converged warp, one elected lane issues). Every wait is bounded; a wait
+// that runs out records an error and all roles leave their loops, the MMA warp waits for its MMAs,
+// the producer for its copies, and tensor memory is released.
+#include <math.h>
+
+#include "common.cuh"
+#include "tc.cuh"
+
+namespace {
+
+constexpr int kD = 128;
+constexpr int kThreads = 320;
+constexpr uint32_t kTmemCols = 512;
+constexpr uint32_t kColS = 0, kColDP = 128, kColAcc0 = 256, kColAcc1 = 384;
+
+struct BwdParams {
+    const int32_t *spans, *ptr, *idx, *order;
+    const int8_t *kind;
+    const float *lt, *dt;   // [Hq][t_pad]
+    int64_t T, t_pad;
+    int32_t num_q_heads, num_kv_heads, num_tiles;
+    float scale_log2, scale;
+    __nv_bfloat16 *out0, *out1;   // dK/dV pass: dK, dV; dQ pass: dQ
+    int *err;
+};
+
+__device__ __forceinline__ bool wait_or_abort(uint32_t bar, uint32_t parity, int *err, int site, volatile int *abort_flag)
+{
+    if (*abort_flag) return false;
+    if (mbar_wait_bounded(bar, parity, err, site)) return true;
+    *abort_flag = 1;
+    return false;
+}
+
+// TMEM column of k-slice kk (16 values) of a 64-wide bf16 operand written by the softmax warps.
+__device__ __forceinline__ uint32_t slice_col(int kk) { return (uint32_t)((kk >> 1) * 32 + (kk & 1) * 8); }
+
+__device__ __forceinline__ void store_row_bf16(__nv_bfloat16 *dst, const uint32_t (&o)[32], float mul)
+{
+#pragma unroll
+    for (int i = 0; i < 32; i += 8) {
+        uint4 w;
+        w.x = pack_bf16x2(__uint_as_float(o[i]) * mul, __uint_as_float(o[i + 1]) * mul);
+        w.y = pack_bf16x2(__uint_as_float(o[i + 2]) * mul, __uint_as_float(o[i + 3]) * mul);
+        w.z = pack_bf16x2(__uint_as_float(o[i + 4]) * mul, __uint_as_float(o[i + 5]) * mul);
+        w.w = pack_bf16x2(__uint_as_float(o[i + 6]) * mul, __uint_as_float(o[i + 7]) * mul);
+        *reinterpret_cast<uint4 *>(dst + i) = w;
+    }
+}
+
+// ================================================================================================
+// dK/dV pass
+// ================================================================================================
+namespace dkv {
+constexpr int kKT = PADOC_BWD_DKV_K_TILE;   // 128 keys: the M of every MMA
+constexpr int kQT = PADOC_BWD_DKV_Q_TILE;   // 64 queries per step
+constexpr int kStages = 3;
+constexpr int kKPanel = kKT * 128;           // [128 rows][64 bf16]
+constexpr int kQPanel = kQT * 128;           // [64 rows][64 bf16]
+constexpr int kKTile = 2 * kKPanel;
+constexpr int kQTile = 2 * kQPanel;
+constexpr int kAuxBytes = 2 * kQT * 4 + kQT * 16;   // lse2[64], D[64], spans[64][4]
+enum {
+    B_KV = 0,
+    B_QFULL = 1,                  // [stage]
+    B_QEMPTY = 1 + kStages,       // [stage]
+    B_SFULL = 1 + 2 * kStages,    // [step parity]
+    B_PFULL = 3 + 2 * kStages,    // [step parity], 256 arrivals
+    B_FINAL = 5 + 2 * kStages,
+    B_COUNT = 6 + 2 * kStages
+};
+constexpr size_t kSmemBytes = 1024 + 2 * (size_t)kKTile + 2 * (size_t)kStages * kQTile + (size_t)kStages * kAuxBytes +
+                              B_COUNT * 8 + 64;
+}  // namespace dkv
+
+__global__ void __launch_bounds__(kThreads, 1)
+prefill_bwd_dkv_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__ CUtensorMap gmap,
+                       const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap,
+                       const BwdParams prm)
+{
+    using namespace dkv;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+    uint8_t *sk = smem;
+    uint8_t *sv = sk + kKTile;
+    uint8_t *sq = sv + kKTile;                 // [stage] Q step tiles
+    uint8_t *sg = sq + kStages * kQTile;       // [stage] dO step tiles
+    uint8_t *aux = sg + kStages * kQTile;      // [stage] lse2, D, spans
+    uint64_t *bars = (uint64_t *)(aux + kStages * kAuxBytes);
+    uint32_t *tmem_slot = (uint32_t *)(bars + B_COUNT);
+    volatile int *abort_flag = (volatile int *)(tmem_slot + 1);
+
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int hkv = prm.num_kv_heads, group = prm.num_q_heads / hkv;
+    const int kt = prm.order[blockIdx.x / hkv], g = (int)(blockIdx.x % hkv);
+    const int e0 = prm.ptr[kt], ne = prm.ptr[kt + 1] - e0;
+    const int nu = ne * group;
+    auto bar = [&](int i) { return smem_u32(&bars[i]); };
+
+    if (tid == 0) {
+        for (int i = 0; i < B_COUNT; ++i) mbar_init(bar(i), (i == B_PFULL || i == B_PFULL + 1) ? 256 : 1);
+        *abort_flag = 0;
+        fence_barrier_init();
+    }
+    if (warp == 9) {
+        tmem_alloc(smem_u32(tmem_slot), kTmemCols);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
+
+    if (warp == 8) {
+        // ---------------------------------------------------------------- TMA producer
+        if (lane == 0 && nu > 0) {
+            tma_prefetch_desc(&qmap);
+            tma_prefetch_desc(&gmap);
+            tma_prefetch_desc(&kmap);
+            tma_prefetch_desc(&vmap);
+            mbar_arrive_expect_tx(bar(B_KV), 2 * kKTile);
+            tma_load_2d(smem_u32(sk), &kmap, g * kD, kt * kKT, bar(B_KV));
+            tma_load_2d(smem_u32(sk) + kKPanel, &kmap, g * kD + 64, kt * kKT, bar(B_KV));
+            tma_load_2d(smem_u32(sv), &vmap, g * kD, kt * kKT, bar(B_KV));
+            tma_load_2d(smem_u32(sv) + kKPanel, &vmap, g * kD + 64, kt * kKT, bar(B_KV));
+            int issued = 0;
+            for (int u = 0; u < nu; ++u) {
+                const int s = u % kStages;
+                if (u >= kStages && !wait_or_abort(bar(B_QEMPTY + s), (u / kStages - 1) & 1, prm.err, 50, abort_flag))
+                    break;
+                const int e = e0 + u / group, h = g * group + u % group;
+                const int q0 = prm.idx[e] * kQT;
+                const int nsp = prm.kind[e] == PADOC_TILE_FULL ? 0 : min(kQT, (int)(prm.T - q0)) * 16;
+                const uint32_t fb = bar(B_QFULL + s);
+                const uint32_t qb = smem_u32(sq + s * kQTile), gb = smem_u32(sg + s * kQTile);
+                const uint32_t ab = smem_u32(aux + s * kAuxBytes);
+                mbar_arrive_expect_tx(fb, 2 * kQTile + 2 * kQT * 4 + nsp);
+                tma_load_2d(qb, &qmap, h * kD, q0, fb);
+                tma_load_2d(qb + kQPanel, &qmap, h * kD + 64, q0, fb);
+                tma_load_2d(gb, &gmap, h * kD, q0, fb);
+                tma_load_2d(gb + kQPanel, &gmap, h * kD + 64, q0, fb);
+                bulk_load(ab, prm.lt + (size_t)h * prm.t_pad + q0, kQT * 4, fb);
+                bulk_load(ab + kQT * 4, prm.dt + (size_t)h * prm.t_pad + q0, kQT * 4, fb);
+                if (nsp) bulk_load(ab + 2 * kQT * 4, prm.spans + 4 * (size_t)q0, (uint32_t)nsp, fb);
+                issued = u + 1;
+            }
+            // copies still in flight must land before the CTA's shared memory is released
+            mbar_wait_bounded(bar(B_KV), 0, prm.err, 51);
+            for (int u = (issued > kStages ? issued - kStages : 0); u < issued; ++u)
+                mbar_wait_bounded(bar(B_QFULL + u % kStages), (u / kStages) & 1, prm.err, 52);
+        }
+    } else if (warp == 9) {
+        // ---------------------------------------------------------------- MMA issuer (whole warp)
+        if (nu > 0) {
+            constexpr uint32_t idS = umma_idesc_bf16(128, kQT, false);
+            constexpr uint32_t idAcc = umma_idesc_bf16(128, kD, true);
+            const uint64_t dK = umma_desc_sw128(smem_u32(sk), 16, 1024);
+            const uint64_t dV = umma_desc_sw128(smem_u32(sv), 16, 1024);
+            auto wait_w = [&](int b, uint32_t parity, int site) {
+                const bool r = wait_or_abort(bar(b), parity, prm.err, site, abort_flag);
+                return __all_sync(0xffffffffu, r);
+            };
+            // S^T and dP^T of step u into the parity-(u & 1) columns
+            auto issue_s = [&](int u) {
+                const int s = u % kStages;
+                const uint32_t b = (uint32_t)(u & 1) * 64;
+                const uint64_t dq = umma_desc_sw128(smem_u32(sq + s * kQTile), 16, 1024);
+                const uint64_t dg = umma_desc_sw128(smem_u32(sg + s * kQTile), 16, 1024);
+#pragma unroll
+                for (int ks = 0; ks < 8; ++ks) {
+                    const uint32_t oa = ((ks >> 2) * kKPanel + (ks & 3) * 32) >> 4;
+                    const uint32_t ob = ((ks >> 2) * kQPanel + (ks & 3) * 32) >> 4;
+                    umma_bf16_ss_warp(tmem + kColS + b, dK + oa, dq + ob, idS, ks > 0);
+                }
+#pragma unroll
+                for (int ks = 0; ks < 8; ++ks) {
+                    const uint32_t oa = ((ks >> 2) * kKPanel + (ks & 3) * 32) >> 4;
+                    const uint32_t ob = ((ks >> 2) * kQPanel + (ks & 3) * 32) >> 4;
+                    umma_bf16_ss_warp(tmem + kColDP + b, dV + oa, dg + ob, idS, ks > 0);
+                }
+                umma_commit_warp(bar(B_SFULL + (u & 1)));
+            };
+            bool ok = wait_w(B_KV, 0, 60);
+            for (int u = 0; ok && u < 2 && u < nu; ++u) {
+                ok = wait_w(B_QFULL + u % kStages, (u / kStages) & 1, 61);
+                if (ok) {
+                    tc_fence_after();
+                    issue_s(u);
+                }
+            }
+            for (int u = 0; ok && u < nu; ++u) {
+                const int s = u % kStages;
+                const uint32_t b = (uint32_t)(u & 1) * 64;
+                if (!wait_w(B_PFULL + (u & 1), (u >> 1) & 1, 62)) { ok = false; break; }
+                tc_fence_after();
+                // the step's Q and dO as MN-major B operands (N = head dim, K = the 64 queries)
+                const uint64_t gmn = umma_desc_sw128(smem_u32(sg + s * kQTile), kQPanel, 1024);
+                const uint64_t qmn = umma_desc_sw128(smem_u32(sq + s * kQTile), kQPanel, 1024);
+#pragma unroll
+                for (int kk = 0; kk < 4; ++kk)
+                    umma_bf16_ts_warp(tmem + kColAcc0, tmem + kColS + b + slice_col(kk), gmn + kk * (2048 >> 4), idAcc,
+                                      (u > 0 || kk > 0));
+#pragma unroll
+                for (int kk = 0; kk < 4; ++kk)
+                    umma_bf16_ts_warp(tmem + kColAcc1, tmem + kColDP + b + slice_col(kk), qmn + kk * (2048 >> 4), idAcc,
+                                      (u > 0 || kk > 0));
+                umma_commit_warp(bar(B_QEMPTY + s));
+                if (u + 2 < nu) {
+                    if (!wait_w(B_QFULL + (u + 2) % kStages, ((u + 2) / kStages) & 1, 63)) { ok = false; break; }
+                    tc_fence_after();
+                    issue_s(u + 2);
+                }
+            }
+            // every MMA issued above must complete before tensor memory is read or released
+            umma_commit_warp(bar(B_FINAL));
+            mbar_wait_bounded(bar(B_FINAL), 0, prm.err, 64);
+        }
+    } else {
+        // ---------------------------------------------------------------- softmax + epilogue
+        const int lq = warp & 3, ch = warp >> 2;          // TMEM lane quarter, column half
+        const int key = kt * kKT + lq * 32 + lane;
+        const uint32_t lanes = (uint32_t)(lq * 32) << 16;
+        const float c = prm.scale_log2;
+        auto wait_all = [&](int b, uint32_t parity, int site) {
+            const bool r = wait_or_abort(bar(b), parity, prm.err, site, abort_flag);
+            return __all_sync(0xffffffffu, r);
+        };
+        bool ok = true;
+        for (int u = 0; u < nu; ++u) {
+            const int s = u % kStages;
+            const uint32_t b = (uint32_t)(u & 1) * 64 + 32 * ch;
+            const int e = e0 + u / group;
+            const bool partial = prm.kind[e] != PADOC_TILE_FULL;
+            const int qbase = prm.idx[e] * kQT + 32 * ch;
+            if (!wait_all(B_SFULL + (u & 1), (u >> 1) & 1, 70) || !wait_all(B_QFULL + s, (u / kStages) & 1, 71)) {
+                ok = false;
+                break;
+            }
+            tc_fence_after();
+            uint32_t sr[32], dr[32];
+            tmem_ld32(tmem + lanes + kColS + b, sr);
+            tmem_ld32(tmem + lanes + kColDP + b, dr);
+            const float4 *la = reinterpret_cast<const float4 *>(aux + s * kAuxBytes) + 8 * ch;
+            const float4 *da = reinterpret_cast<const float4 *>(aux + s * kAuxBytes + kQT * 4) + 8 * ch;
+            const int4 *sp = reinterpret_cast<const int4 *>(aux + s * kAuxBytes + 2 * kQT * 4) + 32 * ch;
+            uint32_t vis = 0xffffffffu;
+            if (partial) {
+                vis = 0u;
+                const int64_t rem = prm.T - qbase;   // query columns past T hold no spans
+                const int nvalid = rem <= 0 ? 0 : (rem >= 32 ? 32 : (int)rem);
+                for (int i = 0; i < nvalid; ++i) {
+                    const int4 w = sp[i];
+                    const bool in = (key >= w.x && key < w.y) || (key >= w.z && key < w.w);
+                    vis |= (uint32_t)in << i;
+                }
+            }
+            tmem_ld_wait();
+            uint32_t pk[16], dk[16];
+#pragma unroll
+            for (int i4 = 0; i4 < 8; ++i4) {
+                const float4 l4 = la[i4], d4 = da[i4];
+                const float lv[4] = {l4.x, l4.y, l4.z, l4.w}, dv[4] = {d4.x, d4.y, d4.z, d4.w};
+                float p[4], ds[4];
+#pragma unroll
+                for (int j = 0; j < 4; ++j) {
+                    const int i = 4 * i4 + j;
+                    const float pe = fast_exp2(fmaf(__uint_as_float(sr[i]), c, -lv[j]));
+                    p[j] = (vis >> i) & 1u ? pe : 0.f;
+                    ds[j] = p[j] * (__uint_as_float(dr[i]) - dv[j]);
+                }
+                pk[2 * i4] = pack_bf16x2(p[0], p[1]);
+                pk[2 * i4 + 1] = pack_bf16x2(p[2], p[3]);
+                dk[2 * i4] = pack_bf16x2(ds[0], ds[1]);
+                dk[2 * i4 + 1] = pack_bf16x2(ds[2], ds[3]);
+            }
+            tmem_st16(tmem + lanes + kColS + b, pk);
+            tmem_st16(tmem + lanes + kColDP + b, dk);
+            tmem_st_wait();
+            tc_fence_before();
+            mbar_arrive(bar(B_PFULL + (u & 1)));
+        }
+        // epilogue: column half 0 writes dV, half 1 writes dK (times scale), one key row per thread
+        if (ok && (nu == 0 || wait_all(B_FINAL, 0, 72))) {
+            tc_fence_after();
+            const bool isk = ch == 1;
+            __nv_bfloat16 *dst = (isk ? prm.out0 : prm.out1) + ((size_t)(key < prm.T ? key : 0) * hkv + g) * kD;
+            const float mul = isk ? prm.scale : 1.f;
+#pragma unroll
+            for (int cc = 0; cc < 4; ++cc) {
+                uint32_t o[32];
+                if (nu > 0) {
+                    tmem_ld32(tmem + lanes + (isk ? kColAcc1 : kColAcc0) + 32 * cc, o);
+                    tmem_ld_wait();
+                } else {
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) o[i] = 0u;
+                }
+                if (key < prm.T) store_row_bf16(dst + 32 * cc, o, mul);
+            }
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 9) {
+        tc_fence_after();
+        tmem_dealloc(tmem, kTmemCols);
+    }
+}
+
+// ================================================================================================
+// dQ pass
+// ================================================================================================
+namespace dqp {
+constexpr int kQT = PADOC_BWD_DQ_Q_TILE;    // 128 query rows: the M of every MMA
+constexpr int kKT = PADOC_BWD_DQ_K_TILE;    // 64 keys per step
+constexpr int kStages = 4;
+constexpr int kQPanel = kQT * 128;
+constexpr int kKPanel = kKT * 128;
+constexpr int kQTile = 2 * kQPanel;
+constexpr int kKTile = 2 * kKPanel;
+enum {
+    B_QG = 0,
+    B_KFULL = 1,                  // [stage]
+    B_KEMPTY = 1 + kStages,       // [stage]
+    B_SFULL = 1 + 2 * kStages,    // [step parity]
+    B_PFULL = 3 + 2 * kStages,    // [step parity], 256 arrivals
+    B_FINAL = 5 + 2 * kStages,
+    B_COUNT = 6 + 2 * kStages
+};
+constexpr size_t kSmemBytes = 1024 + 2 * (size_t)kQTile + 2 * (size_t)kStages * kKTile + B_COUNT * 8 + 64;
+}  // namespace dqp
+
+__device__ __forceinline__ int clamp32(int x) { return min(max(x, 0), 32); }
+
+__global__ void __launch_bounds__(kThreads, 1)
+prefill_bwd_dq_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__ CUtensorMap gmap,
+                      const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap,
+                      const BwdParams prm)
+{
+    using namespace dqp;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+    uint8_t *sq = smem;
+    uint8_t *sg = sq + kQTile;
+    uint8_t *sk = sg + kQTile;                 // [stage] K step tiles
+    uint8_t *sv = sk + kStages * kKTile;       // [stage] V step tiles
+    uint64_t *bars = (uint64_t *)(sv + kStages * kKTile);
+    uint32_t *tmem_slot = (uint32_t *)(bars + B_COUNT);
+    volatile int *abort_flag = (volatile int *)(tmem_slot + 1);
+
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int hq = prm.num_q_heads, group = hq / prm.num_kv_heads;
+    const int qt = prm.num_tiles - 1 - (int)(blockIdx.x / hq);   // heavier q-tiles (later in a page) first
+    const int h = (int)(blockIdx.x % hq), g = h / group;
+    const int e0 = prm.ptr[qt], nu = prm.ptr[qt + 1] - e0;
+    auto bar = [&](int i) { return smem_u32(&bars[i]); };
+
+    if (tid == 0) {
+        for (int i = 0; i < B_COUNT; ++i) mbar_init(bar(i), (i == B_PFULL || i == B_PFULL + 1) ? 256 : 1);
+        *abort_flag = 0;
+        fence_barrier_init();
+    }
+    if (warp == 9) {
+        tmem_alloc(smem_u32(tmem_slot), kTmemCols);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
+
+    if (warp == 8) {
+        // ---------------------------------------------------------------- TMA producer
+        if (lane == 0 && nu > 0) {
+            tma_prefetch_desc(&qmap);
+            tma_prefetch_desc(&gmap);
+            tma_prefetch_desc(&kmap);
+            tma_prefetch_desc(&vmap);
+            mbar_arrive_expect_tx(bar(B_QG), 2 * kQTile);
+            tma_load_2d(smem_u32(sq), &qmap, h * kD, qt * kQT, bar(B_QG));
+            tma_load_2d(smem_u32(sq) + kQPanel, &qmap, h * kD + 64, qt * kQT, bar(B_QG));
+            tma_load_2d(smem_u32(sg), &gmap, h * kD, qt * kQT, bar(B_QG));
+            tma_load_2d(smem_u32(sg) + kQPanel, &gmap, h * kD + 64, qt * kQT, bar(B_QG));
+            int issued = 0;
+            for (int u = 0; u < nu; ++u) {
+                const int s = u % kStages;
+                if (u >= kStages && !wait_or_abort(bar(B_KEMPTY + s), (u / kStages - 1) & 1, prm.err, 80, abort_flag))
+                    break;
+                const int k0 = prm.idx[e0 + u] * kKT;
+                const uint32_t fb = bar(B_KFULL + s);
+                const uint32_t kb = smem_u32(sk + s * kKTile), vb = smem_u32(sv + s * kKTile);
+                mbar_arrive_expect_tx(fb, 2 * kKTile);
+                tma_load_2d(kb, &kmap, g * kD, k0, fb);
+                tma_load_2d(kb + kKPanel, &kmap, g * kD + 64, k0, fb);
+                tma_load_2d(vb, &vmap, g * kD, k0, fb);
+                tma_load_2d(vb + kKPanel, &vmap, g * kD + 64, k0, fb);
+                issued = u + 1;
+            }
+            mbar_wait_bounded(bar(B_QG), 0, prm.err, 81);
+            for (int u = (issued > kStages ? issued - kStages : 0); u < issued; ++u)
+                mbar_wait_bounded(bar(B_KFULL + u % kStages), (u / kStages) & 1, prm.err, 82);
+        }
+    } else if (warp == 9) {
+        // ---------------------------------------------------------------- MMA issuer (whole warp)
+        if (nu > 0) {
+            constexpr uint32_t idS = umma_idesc_bf16(128, kKT, false);
+            constexpr uint32_t idAcc = umma_idesc_bf16(128, kD, true);
+            const uint64_t dQ = umma_desc_sw128(smem_u32(sq), 16, 1024);
+            const uint64_t dG = umma_desc_sw128(smem_u32(sg), 16, 1024);
+            auto wait_w = [&](int b, uint32_t parity, int site) {
+                const bool r = wait_or_abort(bar(b), parity, prm.err, site, abort_flag);
+                return __all_sync(0xffffffffu, r);
+            };
+            auto issue_s = [&](int u) {
+                const int s = u % kStages;
+                const uint32_t b = (uint32_t)(u & 1) * 64;
+                const uint64_t dk = umma_desc_sw128(smem_u32(sk + s * kKTile), 16, 1024);
+                const uint64_t dv = umma_desc_sw128(smem_u32(sv + s * kKTile), 16, 1024);
+#pragma unroll
+                for (int ks = 0; ks < 8; ++ks) {
+                    const uint32_t oa = ((ks >> 2) * kQPanel + (ks & 3) * 32) >> 4;
+                    const uint32_t ob = ((ks >> 2) * kKPanel + (ks & 3) * 32) >> 4;
+                    umma_bf16_ss_warp(tmem + kColS + b, dQ + oa, dk + ob, idS, ks > 0);
+                }
+#pragma unroll
+                for (int ks = 0; ks < 8; ++ks) {
+                    const uint32_t oa = ((ks >> 2) * kQPanel + (ks & 3) * 32) >> 4;
+                    const uint32_t ob = ((ks >> 2) * kKPanel + (ks & 3) * 32) >> 4;
+                    umma_bf16_ss_warp(tmem + kColDP + b, dG + oa, dv + ob, idS, ks > 0);
+                }
+                umma_commit_warp(bar(B_SFULL + (u & 1)));
+            };
+            bool ok = wait_w(B_QG, 0, 90);
+            for (int u = 0; ok && u < 2 && u < nu; ++u) {
+                ok = wait_w(B_KFULL + u % kStages, (u / kStages) & 1, 91);
+                if (ok) {
+                    tc_fence_after();
+                    issue_s(u);
+                }
+            }
+            for (int u = 0; ok && u < nu; ++u) {
+                const int s = u % kStages;
+                const uint32_t b = (uint32_t)(u & 1) * 64;
+                if (!wait_w(B_PFULL + (u & 1), (u >> 1) & 1, 92)) { ok = false; break; }
+                tc_fence_after();
+                // the step's K as an MN-major B operand (N = head dim, K = the 64 keys)
+                const uint64_t kmn = umma_desc_sw128(smem_u32(sk + s * kKTile), kKPanel, 1024);
+#pragma unroll
+                for (int kk = 0; kk < 4; ++kk)
+                    umma_bf16_ts_warp(tmem + kColAcc0, tmem + kColDP + b + slice_col(kk), kmn + kk * (2048 >> 4), idAcc,
+                                      (u > 0 || kk > 0));
+                umma_commit_warp(bar(B_KEMPTY + s));
+                if (u + 2 < nu) {
+                    if (!wait_w(B_KFULL + (u + 2) % kStages, ((u + 2) / kStages) & 1, 93)) { ok = false; break; }
+                    tc_fence_after();
+                    issue_s(u + 2);
+                }
+            }
+            umma_commit_warp(bar(B_FINAL));
+            mbar_wait_bounded(bar(B_FINAL), 0, prm.err, 94);
+        }
+    } else {
+        // ---------------------------------------------------------------- softmax + epilogue
+        const int lq = warp & 3, ch = warp >> 2;
+        const int row = lq * 32 + lane;
+        const int64_t t = (int64_t)qt * kQT + row;
+        const uint32_t lanes = (uint32_t)(lq * 32) << 16;
+        const float c = prm.scale_log2;
+        int a0 = 0, a1 = 0, b0 = 0, b1 = 0;
+        if (t < prm.T) {
+            const int4 w = *reinterpret_cast<const int4 *>(prm.spans + 4 * t);
+            a0 = w.x; a1 = w.y; b0 = w.z; b1 = w.w;
+        }
+        // rows past T read the padding (lse2 = +inf, D = 0): their P and dS are 0
+        const float lrow = prm.lt[(size_t)h * prm.t_pad + t], drow = prm.dt[(size_t)h * prm.t_pad + t];
+        auto wait_all = [&](int b, uint32_t parity, int site) {
+            const bool r = wait_or_abort(bar(b), parity, prm.err, site, abort_flag);
+            return __all_sync(0xffffffffu, r);
+        };
+        bool ok = true;
+        for (int u = 0; u < nu; ++u) {
+            const uint32_t b = (uint32_t)(u & 1) * 64 + 32 * ch;
+            const bool partial = prm.kind[e0 + u] != PADOC_TILE_FULL;
+            const int cb = prm.idx[e0 + u] * kKT + 32 * ch;
+            if (!wait_all(B_SFULL + (u & 1), (u >> 1) & 1, 95)) { ok = false; break; }
+            tc_fence_after();
+            uint32_t sr[32], dr[32];
+            tmem_ld32(tmem + lanes + kColS + b, sr);
+            tmem_ld32(tmem + lanes + kColDP + b, dr);
+            uint32_t vis = 0xffffffffu;
+            if (partial) {
+                const int lo0 = clamp32(a0 - cb), lo1 = clamp32(b0 - cb);
+                vis = interval_bits(lo0, max(clamp32(a1 - cb) - lo0, 0), 0) |
+                      interval_bits(lo1, max(clamp32(b1 - cb) - lo1, 0), 0);
+            }
+            tmem_ld_wait();
+            uint32_t dk[16];
+#pragma unroll
+            for (int i = 0; i < 32; i += 2) {
+                const float pe0 = fast_exp2(fmaf(__uint_as_float(sr[i]), c, -lrow));
+                const float pe1 = fast_exp2(fmaf(__uint_as_float(sr[i + 1]), c, -lrow));
+                const float p0 = (vis >> i) & 1u ? pe0 : 0.f;
+                const float p1 = (vis >> (i + 1)) & 1u ? pe1 : 0.f;
+                dk[i >> 1] = pack_bf16x2(p0 * (__uint_as_float(dr[i]) - drow), p1 * (__uint_as_float(dr[i + 1]) - drow));
+            }
+            tmem_st16(tmem + lanes + kColDP + b, dk);
+            tmem_st_wait();
+            tc_fence_before();
+            mbar_arrive(bar(B_PFULL + (u & 1)));
+        }
+        // epilogue: dQ times scale, columns 64 ch .. 64 ch + 63 of the thread's row
+        if (ok && (nu == 0 || wait_all(B_FINAL, 0, 96))) {
+            tc_fence_after();
+            __nv_bfloat16 *dst = prm.out0 + ((size_t)(t < prm.T ? t : 0) * hq + h) * kD + 64 * ch;
+#pragma unroll
+            for (int cc = 0; cc < 2; ++cc) {
+                uint32_t o[32];
+                if (nu > 0) {
+                    tmem_ld32(tmem + lanes + kColAcc0 + 64 * ch + 32 * cc, o);
+                    tmem_ld_wait();
+                } else {
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) o[i] = 0u;
+                }
+                if (t < prm.T) store_row_bf16(dst + 32 * cc, o, prm.scale);
+            }
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 9) {
+        tc_fence_after();
+        tmem_dealloc(tmem, kTmemCols);
+    }
+}
+
+}  // namespace
+
+padoc_status padoc_launch_prefill_bwd_tc(const void *q, const void *k, const void *v, const void *dout,
+                                         int64_t total_tokens, int32_t num_q_heads, int32_t num_kv_heads,
+                                         const int32_t *spans_dev, const padoc_tile_map_dev *q_map,
+                                         const padoc_tile_map_dev *k_map, const float *lt, const float *dt,
+                                         int64_t t_pad, float scale, void *dq, void *dk, void *dv, cudaStream_t stream)
+{
+    int *err = padoc_device_error_word();
+    if (!err) return PADOC_ERR_CUDA;
+    const int64_t T = total_tokens;
+    const int64_t nkt = (T + dkv::kKT - 1) / dkv::kKT, nqt = (T + dqp::kQT - 1) / dqp::kQT;
+    if (nkt * num_kv_heads > INT32_MAX || nqt * num_q_heads > INT32_MAX) return PADOC_ERR_UNSUPPORTED;
+    const uint64_t qcols = (uint64_t)num_q_heads * kD, kcols = (uint64_t)num_kv_heads * kD;
+    CUtensorMap q64, g64, k128, v128, q128, g128, k64, v64;
+    if (!padoc_make_tmap_bf16(&q64, q, qcols, T, qcols * 2, 64, dkv::kQT) ||
+        !padoc_make_tmap_bf16(&g64, dout, qcols, T, qcols * 2, 64, dkv::kQT) ||
+        !padoc_make_tmap_bf16(&k128, k, kcols, T, kcols * 2, 64, dkv::kKT) ||
+        !padoc_make_tmap_bf16(&v128, v, kcols, T, kcols * 2, 64, dkv::kKT) ||
+        !padoc_make_tmap_bf16(&q128, q, qcols, T, qcols * 2, 64, dqp::kQT) ||
+        !padoc_make_tmap_bf16(&g128, dout, qcols, T, qcols * 2, 64, dqp::kQT) ||
+        !padoc_make_tmap_bf16(&k64, k, kcols, T, kcols * 2, 64, dqp::kKT) ||
+        !padoc_make_tmap_bf16(&v64, v, kcols, T, kcols * 2, 64, dqp::kKT))
+        return PADOC_ERR_CUDA;
+    BwdParams prm;
+    prm.spans = spans_dev;
+    prm.lt = lt;
+    prm.dt = dt;
+    prm.T = T;
+    prm.t_pad = t_pad;
+    prm.num_q_heads = num_q_heads;
+    prm.num_kv_heads = num_kv_heads;
+    prm.scale_log2 = scale * PADOC_LOG2E;
+    prm.scale = scale;
+    prm.err = err;
+
+    BwdParams pk = prm;   // dK/dV pass over the key-major map
+    pk.ptr = k_map->ptr;
+    pk.idx = k_map->idx;
+    pk.kind = k_map->kind;
+    pk.order = k_map->order;
+    pk.num_tiles = (int32_t)nkt;
+    pk.out0 = (__nv_bfloat16 *)dk;
+    pk.out1 = (__nv_bfloat16 *)dv;
+    PADOC_CUDA_TRY(cudaFuncSetAttribute(prefill_bwd_dkv_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                        (int)dkv::kSmemBytes));
+    prefill_bwd_dkv_kernel<<<(unsigned)(nkt * num_kv_heads), kThreads, dkv::kSmemBytes, stream>>>(q64, g64, k128, v128, pk);
+    padoc_status st = padoc_launch_status();
+    if (st != PADOC_OK) return st;
+
+    BwdParams pq = prm;   // dQ pass over the query-major map
+    pq.ptr = q_map->ptr;
+    pq.idx = q_map->idx;
+    pq.kind = q_map->kind;
+    pq.order = nullptr;
+    pq.num_tiles = (int32_t)nqt;
+    pq.out0 = (__nv_bfloat16 *)dq;
+    pq.out1 = nullptr;
+    PADOC_CUDA_TRY(cudaFuncSetAttribute(prefill_bwd_dq_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                        (int)dqp::kSmemBytes));
+    prefill_bwd_dq_kernel<<<(unsigned)(nqt * num_q_heads), kThreads, dqp::kSmemBytes, stream>>>(q128, g128, k64, v64, pq);
+    return padoc_launch_status();
+}

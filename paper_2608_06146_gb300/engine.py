@@ -57,6 +57,31 @@ class PrefillPlan:
                                        self.q_tile, self.k_tile, stream)
 
 
+class PrefillBwdPlan:
+    """Spans, the query-major and key-major tile maps (C1) and the workspace of a packed prefill's
+    backward, on the device."""
+
+    def __init__(self, pages, dtype: torch.dtype, head_dim: int, num_q_heads: int, device):
+        code = pa.PADOC_DTYPE_BF16 if dtype == torch.bfloat16 else pa.PADOC_DTYPE_F32
+        (qq, qk), (kq, kk) = pa.padoc_prefill_bwd_tile_shapes(code, head_dim)
+        spans = pa.padoc_build_query_spans(pages)
+        self.T = int(spans.shape[0])
+        up = lambda a, dt: torch.from_numpy(np.ascontiguousarray(a if len(a) else np.zeros(1, dt))).to(device)
+        self.spans = torch.from_numpy(spans.copy()).to(device)
+        row_ptr, k_tiles, kinds = pa.padoc_build_tile_map(pages, qq, qk)
+        col_ptr, q_tiles, kkinds, order = pa.padoc_build_key_tile_map(pages, kq, kk)
+        self._keep = [up(row_ptr, np.int32), up(k_tiles, np.int32), up(kinds, np.int8),
+                      up(col_ptr, np.int32), up(q_tiles, np.int32), up(kkinds, np.int8), up(order, np.int32)]
+        self.q_map = pa.make_tile_map_dev(*self._keep[:3], qq, qk)
+        self.k_map = pa.make_tile_map_dev(*self._keep[3:6], kq, kk, order=self._keep[6])
+        ws = pa.padoc_prefill_bwd_workspace_size(self.T, num_q_heads)
+        self.workspace = torch.empty(max(ws, 256), dtype=torch.uint8, device=device)
+
+    def run(self, q, k, v, out, dout, lse, scale, dq, dk, dv, stream=None):
+        pa.padoc_ancestor_prefill_bwd(q, k, v, out, dout, lse, self.spans, self.q_map, self.k_map, scale, dq, dk, dv,
+                                      self.workspace, stream)
+
+
 def visible_pairs(pages) -> int:
     """Visible (query, key) pairs of a packed prefill, summed in closed form per page."""
     n = 0

@@ -175,6 +175,12 @@ def packed_qkv(wl: Workload, seed: int, scale: float = 1.0):
     return q, k, v
 
 
+def packed_dout(wl: Workload, seed: int, scale: float = 1.0) -> torch.Tensor:
+    """Upstream gradient dO [T][Hq][d] of a packed prefill, in ``wl.dtype`` on the CPU."""
+    T = sum(p.packed_len for p in wl.pages)
+    return randn((T, wl.num_q_heads, wl.head_dim), wl.dtype, seed * 1000 + 4, scale)
+
+
 @dataclass
 class DecodeInputs:
     """Logical (unpaged) decode-step state plus its paged layout.

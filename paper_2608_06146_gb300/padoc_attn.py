@@ -49,6 +49,11 @@ class padoc_decode_config(ctypes.Structure):
                 ("tc_ctas", ctypes.c_int32), ("warp_ctas", ctypes.c_int32)]
 
 
+class padoc_tile_map_dev(ctypes.Structure):
+    _fields_ = [("ptr", ctypes.c_void_p), ("idx", ctypes.c_void_p), ("kind", ctypes.c_void_p),
+                ("order", ctypes.c_void_p), ("q_tile", ctypes.c_int32), ("k_tile", ctypes.c_int32)]
+
+
 class padoc_decode_plan(ctypes.Structure):
     _fields_ = [("cfg", padoc_decode_config), ("num_pages", ctypes.c_int32), ("num_streams", ctypes.c_int32),
                 ("num_items", ctypes.c_int32), ("num_tc_items", ctypes.c_int32), ("tc_ctas", ctypes.c_int32),
@@ -99,6 +104,14 @@ def load_library(path: Optional[str] = None):
         "padoc_ancestor_prefill_attn": [_vp, _vp, _vp, ctypes.c_int, ctypes.c_int64, ctypes.c_int32, ctypes.c_int32,
                                         ctypes.c_int32, _vp, _vp, _vp, _vp, ctypes.c_int32, ctypes.c_int32,
                                         ctypes.c_float, _vp, _vp, _vp],
+        "padoc_build_key_tile_map": [P, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32, _i32p, _i32p, _i8p, _i32p,
+                                     ctypes.c_int64],
+        "padoc_prefill_bwd_tile_shapes": [ctypes.c_int, ctypes.c_int32, _i32p, _i32p, _i32p, _i32p],
+        "padoc_prefill_bwd_workspace_size": [ctypes.c_int64, ctypes.c_int32, ctypes.POINTER(ctypes.c_size_t)],
+        "padoc_ancestor_prefill_bwd": [_vp, _vp, _vp, _vp, _vp, _vp, ctypes.c_int, ctypes.c_int64, ctypes.c_int32,
+                                       ctypes.c_int32, ctypes.c_int32, _vp, ctypes.POINTER(padoc_tile_map_dev),
+                                       ctypes.POINTER(padoc_tile_map_dev), ctypes.c_float, _vp, _vp, _vp, _vp,
+                                       ctypes.c_size_t, _vp],
         "padoc_selftest_tcgen05": [_vp, _vp, _vp, _vp, _vp, _vp, _vp],
         "padoc_check_device_errors": [_vp],
         "padoc_last_device_error": [_i32p, _i32p],
@@ -120,7 +133,9 @@ def exported_symbols() -> Sequence[str]:
                         "padoc_tile_map_size", "padoc_build_tile_map", "padoc_decode_plan_size",
                         "padoc_build_decode_plan", "padoc_decode_workspace_size", "padoc_branch_decode_attn",
                         "padoc_branch_decode_attn_noalloc",
-                        "padoc_splitk_combine", "padoc_ancestor_prefill_attn", "padoc_selftest_tcgen05",
+                        "padoc_splitk_combine", "padoc_ancestor_prefill_attn", "padoc_build_key_tile_map",
+                        "padoc_prefill_bwd_tile_shapes", "padoc_prefill_bwd_workspace_size",
+                        "padoc_ancestor_prefill_bwd", "padoc_selftest_tcgen05",
                         "padoc_check_device_errors",
                         "padoc_last_device_error", "padoc_status_string", "padoc_version")]
 
@@ -232,6 +247,33 @@ def padoc_build_tile_map(pages, q_tile: int, k_tile: int):
     return row_ptr, kt[:nnz], kind[:nnz]
 
 
+def padoc_build_key_tile_map(pages, q_tile: int, k_tile: int):
+    """Returns (col_ptr int32 [k_tiles+1], q_tiles int32 [nnz], kinds int8 [nnz], k_order int32 [k_tiles])."""
+    lib, P = load_library(), _Pages(pages)
+    T = padoc_packed_size(pages)
+    _, nnz = padoc_tile_map_size(pages, q_tile, k_tile)
+    nkt = -(-T // k_tile)
+    col_ptr = np.zeros(nkt + 1, np.int32)
+    qt = np.zeros(max(nnz, 1), np.int32)
+    kind = np.zeros(max(nnz, 1), np.int8)
+    order = np.zeros(max(nkt, 1), np.int32)
+    _check("padoc_build_key_tile_map",
+           lib.padoc_build_key_tile_map(P.arr, P.n, q_tile, k_tile, col_ptr.ctypes.data_as(_i32p),
+                                        qt.ctypes.data_as(_i32p), kind.ctypes.data_as(_i8p),
+                                        order.ctypes.data_as(_i32p), nnz))
+    return col_ptr, qt[:nnz], kind[:nnz], order[:nkt]
+
+
+def padoc_prefill_bwd_tile_shapes(dtype: int, head_dim: int):
+    """Returns ((dq_q_tile, dq_k_tile), (dkv_q_tile, dkv_k_tile))."""
+    lib = load_library()
+    a, b, c, d = (ctypes.c_int32() for _ in range(4))
+    _check("padoc_prefill_bwd_tile_shapes",
+           lib.padoc_prefill_bwd_tile_shapes(dtype, head_dim, ctypes.byref(a), ctypes.byref(b), ctypes.byref(c),
+                                             ctypes.byref(d)))
+    return (a.value, b.value), (c.value, d.value)
+
+
 # ------------------------------------------------------------------------------------------------
 # Decode
 # ------------------------------------------------------------------------------------------------
@@ -334,6 +376,36 @@ def padoc_ancestor_prefill_attn(q, k, v, spans_dev, row_ptr_dev, k_tiles_dev, ki
                                          _dev(k_tiles_dev, "k_tiles"), _dev(kinds_dev, "kinds"), q_tile, k_tile,
                                          float(scale), _dev(out, "out"), _dev(lse, "lse"), _stream_ptr(stream))
     _check("padoc_ancestor_prefill_attn", st)
+
+
+def make_tile_map_dev(ptr, idx, kind, q_tile: int, k_tile: int, order=None) -> padoc_tile_map_dev:
+    """A padoc_tile_map_dev over device tensors (the caller keeps them alive)."""
+    return padoc_tile_map_dev(_dev(ptr, "ptr"), _dev(idx, "idx"), _dev(kind, "kind"),
+                              _dev(order, "order") if order is not None else None, q_tile, k_tile)
+
+
+def padoc_prefill_bwd_workspace_size(total_tokens: int, num_q_heads: int) -> int:
+    lib = load_library()
+    n = ctypes.c_size_t()
+    _check("padoc_prefill_bwd_workspace_size",
+           lib.padoc_prefill_bwd_workspace_size(total_tokens, num_q_heads, ctypes.byref(n)))
+    return n.value
+
+
+def padoc_ancestor_prefill_bwd(q, k, v, out, dout, lse, spans_dev, q_map: padoc_tile_map_dev,
+                               k_map: padoc_tile_map_dev, scale, dq, dk, dv, workspace, stream=None):
+    """Gradients of the packed prefill: q/out/dout/dq [T][Hq][d]; k/v/dk/dv [T][Hkv][d]; lse fp32 [T][Hq];
+    workspace a uint8 device tensor of padoc_prefill_bwd_workspace_size bytes."""
+    lib = load_library()
+    T, Hq, d = q.shape
+    Hkv = k.shape[1]
+    st = lib.padoc_ancestor_prefill_bwd(_dev(q, "q"), _dev(k, "k"), _dev(v, "v"), _dev(out, "out"),
+                                        _dev(dout, "dout"), _dev(lse, "lse"), _dtype_code(q), T, Hq, Hkv, d,
+                                        _dev(spans_dev, "spans"), ctypes.byref(q_map), ctypes.byref(k_map),
+                                        float(scale), _dev(dq, "dq"), _dev(dk, "dk"), _dev(dv, "dv"),
+                                        _dev(workspace, "workspace"), workspace.numel() * workspace.element_size(),
+                                        _stream_ptr(stream))
+    _check("padoc_ancestor_prefill_bwd", st)
 
 
 def padoc_selftest_tcgen05(a, bk, v, c1, c2, c3, stream=None):

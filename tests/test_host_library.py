@@ -83,6 +83,43 @@ def test_tile_map_bit_exact_vs_oracle_brute_force(seed, qb, kb):
     assert T > 0
 
 
+@pytest.mark.parametrize("seed", range(6))
+@pytest.mark.parametrize("qb,kb", [(64, 128), (16, 32), (32, 16)])
+def test_key_tile_map_is_the_transpose_with_brute_force_kinds(seed, qb, kb):
+    # the key-major map of the backward's dK/dV pass: every (q-tile, k-tile) pair of the oracle's
+    # brute-force classification, listed per k-tile in ascending q-tile order; the order lists every
+    # k-tile once, the longest columns first
+    rng = np.random.default_rng(200 + seed)
+    pages = _rand_pages(rng, int(rng.integers(1, 5)))
+    col_ptr, qt, kind, order = pa.padoc_build_key_tile_map(pages, qb, kb)
+    want = oracle.tile_kinds(pages, qb, kb)
+    nqt, nkt = want.shape
+    assert len(col_ptr) == nkt + 1 and col_ptr[0] == 0 and col_ptr[-1] == len(qt)
+    got = np.zeros((nqt, nkt), np.int8)
+    for c in range(nkt):
+        assert np.all(np.diff(qt[col_ptr[c]:col_ptr[c + 1]]) > 0)
+        got[qt[col_ptr[c]:col_ptr[c + 1]], c] = kind[col_ptr[c]:col_ptr[c + 1]]
+    np.testing.assert_array_equal(got, want)
+    assert sorted(order.tolist()) == list(range(nkt))
+    counts = np.diff(col_ptr)[order]
+    assert np.all(np.diff(counts) <= 0)
+    for a, b in zip(order[:-1], order[1:]):   # ties keep ascending k-tile order
+        if counts[list(order).index(a)] == counts[list(order).index(b)]:
+            assert a < b
+    assert pa.padoc_tile_map_size(pages, qb, kb)[1] == len(qt)
+
+
+def test_prefill_bwd_tile_shapes_and_workspace():
+    assert pa.padoc_prefill_bwd_tile_shapes(pa.PADOC_DTYPE_BF16, 128) == ((128, 64), (64, 128))
+    assert pa.padoc_prefill_bwd_tile_shapes(pa.PADOC_DTYPE_F32, 64) == ((128, 64), (64, 128))
+    with pytest.raises(pa.PadocError):
+        pa.padoc_prefill_bwd_tile_shapes(pa.PADOC_DTYPE_BF16, 64)
+    # lse2 and D per head, rows padded to 128
+    assert pa.padoc_prefill_bwd_workspace_size(1, 16) == 2 * 16 * 128 * 4
+    assert pa.padoc_prefill_bwd_workspace_size(32768, 16) == 2 * 16 * 32768 * 4
+    assert pa.padoc_prefill_bwd_workspace_size(0, 4) == 0
+
+
 def test_tile_map_full_size_packed_prefill_matches_interval_count():
     # 32768 tokens is too large for the quadratic brute force; count visible pairs per tile from the
     # oracle's spans with interval arithmetic instead.
