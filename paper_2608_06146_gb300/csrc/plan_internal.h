@@ -8,10 +8,10 @@
 #define PADOC_PREFILL_Q_TILE 128
 #define PADOC_PREFILL_K_TILE 128
 
-// Prefill backward tiles. The dQ pass keeps 128 query rows (the M of its MMAs) and walks 64-key
-// k-tiles; the dK/dV pass keeps 128 keys (the M of its MMAs) and walks 64-row q-tiles. 64-wide
-// steps let two steps' scores sit in tensor memory beside the accumulators, so the exponentials
-// of one step overlap the MMAs of the next.
+// Prefill backward tiles. The dQ pass keeps 128 query rows (the M of its MMAs) and walks 32-key
+// k-tiles; the dK/dV pass keeps 128 keys (the M of its MMAs) and walks 32-row q-tiles. Narrow
+// steps let several steps' scores sit in tensor memory beside the accumulators and the resident
+// A operands, so the exponentials of one step overlap the MMAs of the next ones.
 #define PADOC_BWD_DQ_Q_TILE 128
 #define PADOC_BWD_DQ_K_TILE 64
 #define PADOC_BWD_DKV_Q_TILE 64

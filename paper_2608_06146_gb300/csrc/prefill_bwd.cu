@@ -4,9 +4,10 @@
 // (prefill_bwd_tc.cu).
 //
 // Per query row and head the backward needs lse (from the forward) and D = sum_c dO[c] O[c]
-// (the softmax's chain-rule term, equal to sum_j P_j dP_j). The statistics pass writes both per
-// head in base 2, [Hq][t_pad] with t_pad = ceil(T / 128) * 128, padded rows lse2 = +inf and D = 0,
-// so that a padded row's P = exp2(S c - lse2) is exactly 0 and the tile passes need no row test.
+// (the softmax's chain-rule term, equal to sum_j P_j dP_j). The statistics pass writes, per head,
+// [Hq][t_pad] with t_pad = ceil(T / 128) * 128, the negated base-2 log-sum-exp -lse2 (so that
+// P = exp2(S c + (-lse2)) is one fused multiply-add and an exponential) and D; padded rows hold
+// -lse2 = -inf and D = 0, so that their P is exactly 0 and the tile passes need no row test.
 #include <math.h>
 
 #include "common.cuh"
@@ -22,7 +23,7 @@ __device__ __forceinline__ float ld_f32<float>(const float *p) { return *p; }
 template <>
 __device__ __forceinline__ float ld_f32<__nv_bfloat16>(const __nv_bfloat16 *p) { return __bfloat162float(*p); }
 
-// One warp per (row, head): D = dO . O (fp32) and lse2 = lse * log2(e), transposed to [Hq][t_pad].
+// One warp per (row, head): D = dO . O (fp32) and -lse * log2(e), transposed to [Hq][t_pad].
 template <typename T, int D>
 __global__ void __launch_bounds__(256) prefill_bwd_stats_kernel(const T *__restrict__ out, const T *__restrict__ dout,
                                                                 const float *__restrict__ lse, int64_t total_tokens,
@@ -48,10 +49,10 @@ __global__ void __launch_bounds__(256) prefill_bwd_stats_kernel(const T *__restr
         const size_t w = (size_t)h * t_pad + t;
         if (t < total_tokens) {
             const float l = lse[r];
-            lt[w] = l == -INFINITY ? INFINITY : l * PADOC_LOG2E;   // a row that sees nothing has P = 0
+            lt[w] = l == -INFINITY ? -INFINITY : -l * PADOC_LOG2E;   // a row that sees nothing has P = 0
             dt[w] = acc;
         } else {
-            lt[w] = INFINITY;
+            lt[w] = -INFINITY;
             dt[w] = 0.f;
         }
     }
@@ -95,7 +96,7 @@ __global__ void __launch_bounds__(128) prefill_bwd_dq_f32_kernel(const float *__
                 s += __shfl_xor_sync(0xffffffffu, s, sh);
                 dp += __shfl_xor_sync(0xffffffffu, dp, sh);
             }
-            const float ds = exp2f(fmaf(s, c, -l2)) * (dp - dd);
+            const float ds = exp2f(fmaf(s, c, l2)) * (dp - dd);
 #pragma unroll
             for (int e = 0; e < E; ++e) acc[e] = fmaf(ds, k[kr + lane + 32 * e], acc[e]);
         }
@@ -148,7 +149,7 @@ __global__ void __launch_bounds__(128) prefill_bwd_dkv_f32_kernel(
                     s += __shfl_xor_sync(0xffffffffu, s, sh);
                     dp += __shfl_xor_sync(0xffffffffu, dp, sh);
                 }
-                const float p = exp2f(fmaf(s, c, -lt[(size_t)h * t_pad + i]));
+                const float p = exp2f(fmaf(s, c, lt[(size_t)h * t_pad + i]));
                 const float ds = p * (dp - dt[(size_t)h * t_pad + i]);
 #pragma unroll
                 for (int e = 0; e < E; ++e) {

@@ -3,32 +3,40 @@
 // need neither a gather nor atomics.
 //
 // With c = scale * log2(e), lse2 = lse * log2(e) and D = rowsum(dO * O) per query row and head
-// (both precomputed per head, [Hq][t_pad], padded rows lse2 = +inf so that their P is 0):
+// (-lse2 and D precomputed per head, [Hq][t_pad], padded rows -lse2 = -inf so that their P is 0):
 //   P = exp2(S c - lse2),  dS = P (dP - D),  S = Q K^T,  dP = dO V^T.
 //
 // dK/dV pass: one CTA per (128-key k-tile, KV head), k-tiles taken in the key-major map's order
-//   (most work first). The CTA walks every (64-row q-tile that sees the k-tile, query head reading
-//   the KV head) step: S^T = K Q^T and dP^T = V dO^T (M = 128 keys, N = 64 queries), the softmax
-//   warps write P^T and dS^T back into tensor memory as bf16, and dV += P^T dO, dK += dS^T Q
-//   accumulate in tensor memory over the whole walk. Every query that sees a shared-stream key
-//   (the stream's later tokens and each branch forked after it) therefore adds into that key's
-//   gradient inside one CTA: the scatter-add of the gather's backward, with nothing scattered.
-// dQ pass: one CTA per (128-row q-tile, query head), heavier q-tiles first. It walks the query-major
-//   map of 64-key k-tiles: S = Q K^T, dP = dO V^T, dS written back as bf16, dQ += dS K.
+//   (most work first). K and V of the tile sit in tensor memory as A operands for the whole walk.
+//   For every (32-row q-tile that sees the k-tile, query head reading the KV head) step the tensor
+//   cores form S^T = K Q^T and dP^T = V dO^T (M = 128 keys, N = 32 queries, B from shared memory),
+//   the softmax warps write P^T and dS^T back into tensor memory as bf16, and dV += P^T dO,
+//   dK += dS^T Q accumulate in tensor memory over the whole walk. Every query that sees a
+//   shared-stream key (the stream's later tokens and each branch forked after it) therefore adds
+//   into that key's gradient inside one CTA: the scatter-add of the gather's backward, with nothing
+//   scattered.
+// dQ pass: one CTA per (128-row q-tile, query head), heavier q-tiles first, Q and dO resident in
+//   tensor memory. It walks the query-major map of 32-key k-tiles: S = Q K^T, dP = dO V^T, dS written
+//   back as bf16, dQ += dS K.
 //
-// Both passes keep two steps' scores in tensor memory: columns [0,128) hold S (or S^T) of steps
-// with parity 0 / 1 at 0 / 64, [128,256) dP likewise, [256,512) the accumulators. While the
-// softmax warps turn step u into P and dS, the tensor cores run step u-1's accumulating MMAs and
-// step u+1's S and dP. A softmax warp owns 32 TMEM lanes (rows) and one 32-column half of a
-// 64-wide step and packs its 32 bf16 results into the first 16 columns of its own half, so no warp
-// overwrites a column another warp still has to read; the accumulating MMAs read the 64-wide
-// operand as k-slices at columns {0, 8, 32, 40}.
+// Every MMA reads at most one operand from shared memory (the other lives in tensor memory), which
+// keeps the narrow steps at the tensor cores' rate instead of shared memory's. Tensor memory holds
+// the resident A operands (128 columns), the accumulators (dV and dK: 256; dQ: 128) and, in what
+// is left, as many step buffers (S and dP, 2 x 32 columns each) as fit: 2 in the dK/dV pass, 4 in
+// the dQ pass. While the softmax warps turn step u into P and dS, the tensor cores run the
+// accumulating MMAs of step u-1 and the S and dP of the steps after u. A softmax warp owns 32 TMEM
+// lanes (rows) and one 16-column half of a step and packs its 16 bf16 results into the first 8
+// columns of its own half, so no warp overwrites a column another warp still has to read; the
+// accumulating MMAs read the two k-slices at columns 0 and 16 of the buffer.
 //
-// Warp roles (320 threads): warps 0-7 softmax and epilogue, warp 8 TMA producer, warp 9 TMEM
-// allocation and MMA issue (converged warp, one elected lane issues). Every wait is bounded; a wait
-// that runs out records an error and all roles leave their loops, the MMA warp waits for its MMAs,
-// the producer for its copies, and tensor memory is released.
+// Warp roles (320 threads): warps 0-7 softmax and epilogue (they also store the resident operands
+// into tensor memory), warp 8 TMA producer, warp 9 TMEM allocation and MMA issue (converged warp,
+// one elected lane issues). Every wait is bounded; a wait that runs out records an error and all
+// roles leave their loops, the MMA warp waits for its MMAs, the producer for its copies, and tensor
+// memory is released.
 #include <math.h>
+
+#include <type_traits>
 
 #include "common.cuh"
 #include "tc.cuh"
@@ -38,16 +46,16 @@ namespace {
 constexpr int kD = 128;
 constexpr int kThreads = 320;
 constexpr uint32_t kTmemCols = 512;
-constexpr uint32_t kColS = 0, kColDP = 128, kColAcc0 = 256, kColAcc1 = 384;
 
 struct BwdParams {
     const int32_t *spans, *ptr, *idx, *order;
     const int8_t *kind;
-    const float *lt, *dt;   // [Hq][t_pad]
+    const float *lt, *dt;               // [Hq][t_pad]: -lse2 and D
+    const __nv_bfloat16 *a0, *a1;       // the pass's tensor-memory operands: dQ pass Q, dO; dK/dV pass K, V
     int64_t T, t_pad;
     int32_t num_q_heads, num_kv_heads, num_tiles;
     float scale_log2, scale;
-    __nv_bfloat16 *out0, *out1;   // dK/dV pass: dK, dV; dQ pass: dQ
+    __nv_bfloat16 *out0, *out1;         // dK/dV pass: dK, dV; dQ pass: dQ
     int *err;
 };
 
@@ -59,8 +67,27 @@ __device__ __forceinline__ bool wait_or_abort(uint32_t bar, uint32_t parity, int
     return false;
 }
 
-// TMEM column of k-slice kk (16 values) of a 64-wide bf16 operand written by the softmax warps.
-__device__ __forceinline__ uint32_t slice_col(int kk) { return (uint32_t)((kk >> 1) * 32 + (kk & 1) * 8); }
+// TMEM column of k-slice k (16 values) of a W-wide bf16 operand written by the softmax warps: column
+// half c packs its W/2 values into the first W/4 columns of its own half.
+template <int W>
+__device__ __forceinline__ uint32_t slice_col(int k)
+{
+    constexpr int per_half = W / 32;
+    return (uint32_t)((k / per_half) * (W / 2) + (k % per_half) * 8);
+}
+
+template <int N>
+__device__ __forceinline__ void tmem_ld_cols(uint32_t taddr, uint32_t (&r)[N])
+{
+    static_assert(N == 16 || N == 32, "16 or 32 columns");
+    if constexpr (N == 32) tmem_ld32(taddr, r); else tmem_ld16(taddr, r);
+}
+template <int N>
+__device__ __forceinline__ void tmem_st_cols(uint32_t taddr, const uint32_t (&r)[N])
+{
+    static_assert(N == 8 || N == 16, "8 or 16 columns");
+    if constexpr (N == 16) tmem_st16(taddr, r); else tmem_st8(taddr, r);
+}
 
 __device__ __forceinline__ void store_row_bf16(__nv_bfloat16 *dst, const uint32_t (&o)[32], float mul)
 {
@@ -75,6 +102,19 @@ __device__ __forceinline__ void store_row_bf16(__nv_bfloat16 *dst, const uint32_
     }
 }
 
+// Stores 64 bf16 of a row (global, 16-byte aligned; zeros when src is null) into 32 TMEM columns of
+// the calling thread's lane: the K-major A-operand layout (column c holds elements 2c, 2c+1).
+__device__ __forceinline__ void row_to_tmem(uint32_t taddr, const __nv_bfloat16 *src)
+{
+    uint32_t w[32];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+        const uint4 x = src ? reinterpret_cast<const uint4 *>(src)[i] : make_uint4(0u, 0u, 0u, 0u);
+        w[4 * i] = x.x; w[4 * i + 1] = x.y; w[4 * i + 2] = x.z; w[4 * i + 3] = x.w;
+    }
+    tmem_st32(taddr, w);
+}
+
 // ================================================================================================
 // dK/dV pass
 // ================================================================================================
@@ -82,6 +122,7 @@ namespace dkv {
 constexpr int kKT = PADOC_BWD_DKV_K_TILE;   // 128 keys: the M of every MMA
 constexpr int kQT = PADOC_BWD_DKV_Q_TILE;   // 64 queries per step
 constexpr int kStages = 3;
+constexpr uint32_t kColS = 0, kColDP = 128, kColAcc0 = 256, kColAcc1 = 384;
 constexpr int kKPanel = kKT * 128;           // [128 rows][64 bf16]
 constexpr int kQPanel = kQT * 128;           // [64 rows][64 bf16]
 constexpr int kKTile = 2 * kKPanel;
@@ -225,11 +266,11 @@ prefill_bwd_dkv_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_co
                 const uint64_t qmn = umma_desc_sw128(smem_u32(sq + s * kQTile), kQPanel, 1024);
 #pragma unroll
                 for (int kk = 0; kk < 4; ++kk)
-                    umma_bf16_ts_warp(tmem + kColAcc0, tmem + kColS + b + slice_col(kk), gmn + kk * (2048 >> 4), idAcc,
+                    umma_bf16_ts_warp(tmem + kColAcc0, tmem + kColS + b + slice_col<kQT>(kk), gmn + kk * (2048 >> 4), idAcc,
                                       (u > 0 || kk > 0));
 #pragma unroll
                 for (int kk = 0; kk < 4; ++kk)
-                    umma_bf16_ts_warp(tmem + kColAcc1, tmem + kColDP + b + slice_col(kk), qmn + kk * (2048 >> 4), idAcc,
+                    umma_bf16_ts_warp(tmem + kColAcc1, tmem + kColDP + b + slice_col<kQT>(kk), qmn + kk * (2048 >> 4), idAcc,
                                       (u > 0 || kk > 0));
                 umma_commit_warp(bar(B_QEMPTY + s));
                 if (u + 2 < nu) {
@@ -283,23 +324,33 @@ prefill_bwd_dkv_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_co
             }
             tmem_ld_wait();
             uint32_t pk[16], dk[16];
+            const uint64_t c2 = f2_pack(c, c);
+            // two query columns per packed instruction: P = exp2(S c - lse2), dS = P (dP - D)
+            auto column_pairs = [&](auto masked) {
 #pragma unroll
-            for (int i4 = 0; i4 < 8; ++i4) {
-                const float4 l4 = la[i4], d4 = da[i4];
-                const float lv[4] = {l4.x, l4.y, l4.z, l4.w}, dv[4] = {d4.x, d4.y, d4.z, d4.w};
-                float p[4], ds[4];
+                for (int i4 = 0; i4 < 8; ++i4) {
+                    const float4 l4 = la[i4], d4 = da[i4];
 #pragma unroll
-                for (int j = 0; j < 4; ++j) {
-                    const int i = 4 * i4 + j;
-                    const float pe = fast_exp2(fmaf(__uint_as_float(sr[i]), c, -lv[j]));
-                    p[j] = (vis >> i) & 1u ? pe : 0.f;
-                    ds[j] = p[j] * (__uint_as_float(dr[i]) - dv[j]);
+                    for (int j = 0; j < 2; ++j) {
+                        const int i = 4 * i4 + 2 * j;
+                        float x0, x1;
+                        f2_unpack(f2_fma(f2_pack(__uint_as_float(sr[i]), __uint_as_float(sr[i + 1])), c2,
+                                         j ? f2_pack(l4.z, l4.w) : f2_pack(l4.x, l4.y)), x0, x1);
+                        float p0 = fast_exp2(x0), p1 = fast_exp2(x1);
+                        if (decltype(masked)::value) {
+                            p0 = (vis >> i) & 1u ? p0 : 0.f;
+                            p1 = (vis >> (i + 1)) & 1u ? p1 : 0.f;
+                        }
+                        const uint64_t t = f2_sub(f2_pack(__uint_as_float(dr[i]), __uint_as_float(dr[i + 1])),
+                                                  j ? f2_pack(d4.z, d4.w) : f2_pack(d4.x, d4.y));
+                        float d0, d1;
+                        f2_unpack(f2_mul(f2_pack(p0, p1), t), d0, d1);
+                        pk[i >> 1] = pack_bf16x2(p0, p1);
+                        dk[i >> 1] = pack_bf16x2(d0, d1);
+                    }
                 }
-                pk[2 * i4] = pack_bf16x2(p[0], p[1]);
-                pk[2 * i4 + 1] = pack_bf16x2(p[2], p[3]);
-                dk[2 * i4] = pack_bf16x2(ds[0], ds[1]);
-                dk[2 * i4 + 1] = pack_bf16x2(ds[2], ds[3]);
-            }
+            };
+            if (partial) column_pairs(std::true_type{}); else column_pairs(std::false_type{});
             tmem_st16(tmem + lanes + kColS + b, pk);
             tmem_st16(tmem + lanes + kColDP + b, dk);
             tmem_st_wait();
@@ -337,42 +388,44 @@ prefill_bwd_dkv_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_co
 // ================================================================================================
 // dQ pass
 // ================================================================================================
-namespace dqp {
-constexpr int kQT = PADOC_BWD_DQ_Q_TILE;    // 128 query rows: the M of every MMA
-constexpr int kKT = PADOC_BWD_DQ_K_TILE;    // 64 keys per step
-constexpr int kStages = 4;
-constexpr int kQPanel = kQT * 128;
-constexpr int kKPanel = kKT * 128;
-constexpr int kQTile = 2 * kQPanel;
-constexpr int kKTile = 2 * kKPanel;
-enum {
-    B_QG = 0,
-    B_KFULL = 1,                  // [stage]
-    B_KEMPTY = 1 + kStages,       // [stage]
-    B_SFULL = 1 + 2 * kStages,    // [step parity]
-    B_PFULL = 3 + 2 * kStages,    // [step parity], 256 arrivals
-    B_FINAL = 5 + 2 * kStages,
-    B_COUNT = 6 + 2 * kStages
+// TMEM: Q at [0,64) and dO at [64,128) as A operands, the step buffers at 128 + 2W i (S, then dP),
+// dQ at [384,512).
+template <int W>
+struct DqCfg {
+    static constexpr int kQT = PADOC_BWD_DQ_Q_TILE;    // 128 query rows: the M of every MMA
+    static constexpr int kDepth = 256 / (2 * W);
+    static constexpr int kStages = W == 32 ? 8 : 5;
+    static constexpr int kPanel = W * 128;
+    static constexpr int kTile = 2 * kPanel;            // K or V of one step
+    static constexpr uint32_t kColQ = 0, kColG = 64, kColBuf = 128, kColDQ = 384;
+    enum {
+        B_QG = 0,                       // 256 arrivals: Q and dO stored into tensor memory
+        B_KFULL = 1,                    // [stage]
+        B_KEMPTY = 1 + kStages,         // [stage]
+        B_SFULL = 1 + 2 * kStages,      // [buffer]
+        B_PFULL = 1 + 2 * kStages + kDepth,   // [buffer], 256 arrivals
+        B_FINAL = 1 + 2 * kStages + 2 * kDepth,
+        B_COUNT = 2 + 2 * kStages + 2 * kDepth
+    };
+    static constexpr size_t kSmemBytes = 1024 + (size_t)kStages * 2 * kTile + B_COUNT * 8 + 64;
+    static_assert(kDepth >= 1 && W % 32 == 0, "step width");
 };
-constexpr size_t kSmemBytes = 1024 + 2 * (size_t)kQTile + 2 * (size_t)kStages * kKTile + B_COUNT * 8 + 64;
-}  // namespace dqp
 
-__device__ __forceinline__ int clamp32(int x) { return min(max(x, 0), 32); }
+__device__ __forceinline__ int clamp_w(int x, int w) { return min(max(x, 0), w); }
 
+template <int W>
 __global__ void __launch_bounds__(kThreads, 1)
-prefill_bwd_dq_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__ CUtensorMap gmap,
-                      const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap,
+prefill_bwd_dq_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap,
                       const BwdParams prm)
 {
-    using namespace dqp;
+    using C = DqCfg<W>;
+    constexpr int S = C::kStages, DEPTH = C::kDepth;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
-    uint8_t *sq = smem;
-    uint8_t *sg = sq + kQTile;
-    uint8_t *sk = sg + kQTile;                 // [stage] K step tiles
-    uint8_t *sv = sk + kStages * kKTile;       // [stage] V step tiles
-    uint64_t *bars = (uint64_t *)(sv + kStages * kKTile);
-    uint32_t *tmem_slot = (uint32_t *)(bars + B_COUNT);
+    uint8_t *sk = smem;                        // [stage] K step tiles
+    uint8_t *sv = sk + S * C::kTile;           // [stage] V step tiles
+    uint64_t *bars = (uint64_t *)(sv + S * C::kTile);
+    uint32_t *tmem_slot = (uint32_t *)(bars + C::B_COUNT);
     volatile int *abort_flag = (volatile int *)(tmem_slot + 1);
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -383,7 +436,8 @@ prefill_bwd_dq_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_con
     auto bar = [&](int i) { return smem_u32(&bars[i]); };
 
     if (tid == 0) {
-        for (int i = 0; i < B_COUNT; ++i) mbar_init(bar(i), (i == B_PFULL || i == B_PFULL + 1) ? 256 : 1);
+        for (int i = 0; i < C::B_COUNT; ++i)
+            mbar_init(bar(i), (i == C::B_QG || (i >= C::B_PFULL && i < C::B_PFULL + DEPTH)) ? 256 : 1);
         *abort_flag = 0;
         fence_barrier_init();
     }
@@ -399,98 +453,79 @@ prefill_bwd_dq_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_con
     if (warp == 8) {
         // ---------------------------------------------------------------- TMA producer
         if (lane == 0 && nu > 0) {
-            tma_prefetch_desc(&qmap);
-            tma_prefetch_desc(&gmap);
             tma_prefetch_desc(&kmap);
             tma_prefetch_desc(&vmap);
-            mbar_arrive_expect_tx(bar(B_QG), 2 * kQTile);
-            tma_load_2d(smem_u32(sq), &qmap, h * kD, qt * kQT, bar(B_QG));
-            tma_load_2d(smem_u32(sq) + kQPanel, &qmap, h * kD + 64, qt * kQT, bar(B_QG));
-            tma_load_2d(smem_u32(sg), &gmap, h * kD, qt * kQT, bar(B_QG));
-            tma_load_2d(smem_u32(sg) + kQPanel, &gmap, h * kD + 64, qt * kQT, bar(B_QG));
             int issued = 0;
             for (int u = 0; u < nu; ++u) {
-                const int s = u % kStages;
-                if (u >= kStages && !wait_or_abort(bar(B_KEMPTY + s), (u / kStages - 1) & 1, prm.err, 80, abort_flag))
-                    break;
-                const int k0 = prm.idx[e0 + u] * kKT;
-                const uint32_t fb = bar(B_KFULL + s);
-                const uint32_t kb = smem_u32(sk + s * kKTile), vb = smem_u32(sv + s * kKTile);
-                mbar_arrive_expect_tx(fb, 2 * kKTile);
+                const int s = u % S;
+                if (u >= S && !wait_or_abort(bar(C::B_KEMPTY + s), (u / S - 1) & 1, prm.err, 80, abort_flag)) break;
+                const int k0 = prm.idx[e0 + u] * W;
+                const uint32_t fb = bar(C::B_KFULL + s);
+                const uint32_t kb = smem_u32(sk + s * C::kTile), vb = smem_u32(sv + s * C::kTile);
+                mbar_arrive_expect_tx(fb, 2 * C::kTile);
                 tma_load_2d(kb, &kmap, g * kD, k0, fb);
-                tma_load_2d(kb + kKPanel, &kmap, g * kD + 64, k0, fb);
+                tma_load_2d(kb + C::kPanel, &kmap, g * kD + 64, k0, fb);
                 tma_load_2d(vb, &vmap, g * kD, k0, fb);
-                tma_load_2d(vb + kKPanel, &vmap, g * kD + 64, k0, fb);
+                tma_load_2d(vb + C::kPanel, &vmap, g * kD + 64, k0, fb);
                 issued = u + 1;
             }
-            mbar_wait_bounded(bar(B_QG), 0, prm.err, 81);
-            for (int u = (issued > kStages ? issued - kStages : 0); u < issued; ++u)
-                mbar_wait_bounded(bar(B_KFULL + u % kStages), (u / kStages) & 1, prm.err, 82);
+            for (int u = (issued > S ? issued - S : 0); u < issued; ++u)
+                mbar_wait_bounded(bar(C::B_KFULL + u % S), (u / S) & 1, prm.err, 82);
         }
     } else if (warp == 9) {
         // ---------------------------------------------------------------- MMA issuer (whole warp)
         if (nu > 0) {
-            constexpr uint32_t idS = umma_idesc_bf16(128, kKT, false);
+            constexpr uint32_t idS = umma_idesc_bf16(128, W, false);
             constexpr uint32_t idAcc = umma_idesc_bf16(128, kD, true);
-            const uint64_t dQ = umma_desc_sw128(smem_u32(sq), 16, 1024);
-            const uint64_t dG = umma_desc_sw128(smem_u32(sg), 16, 1024);
             auto wait_w = [&](int b, uint32_t parity, int site) {
                 const bool r = wait_or_abort(bar(b), parity, prm.err, site, abort_flag);
                 return __all_sync(0xffffffffu, r);
             };
+            // S = Q K^T and dP = dO V^T of step u into buffer u % DEPTH (A from tensor memory)
             auto issue_s = [&](int u) {
-                const int s = u % kStages;
-                const uint32_t b = (uint32_t)(u & 1) * 64;
-                const uint64_t dk = umma_desc_sw128(smem_u32(sk + s * kKTile), 16, 1024);
-                const uint64_t dv = umma_desc_sw128(smem_u32(sv + s * kKTile), 16, 1024);
-#pragma unroll
-                for (int ks = 0; ks < 8; ++ks) {
-                    const uint32_t oa = ((ks >> 2) * kQPanel + (ks & 3) * 32) >> 4;
-                    const uint32_t ob = ((ks >> 2) * kKPanel + (ks & 3) * 32) >> 4;
-                    umma_bf16_ss_warp(tmem + kColS + b, dQ + oa, dk + ob, idS, ks > 0);
-                }
-#pragma unroll
-                for (int ks = 0; ks < 8; ++ks) {
-                    const uint32_t oa = ((ks >> 2) * kQPanel + (ks & 3) * 32) >> 4;
-                    const uint32_t ob = ((ks >> 2) * kKPanel + (ks & 3) * 32) >> 4;
-                    umma_bf16_ss_warp(tmem + kColDP + b, dG + oa, dv + ob, idS, ks > 0);
-                }
-                umma_commit_warp(bar(B_SFULL + (u & 1)));
-            };
-            bool ok = wait_w(B_QG, 0, 90);
-            for (int u = 0; ok && u < 2 && u < nu; ++u) {
-                ok = wait_w(B_KFULL + u % kStages, (u / kStages) & 1, 91);
-                if (ok) {
-                    tc_fence_after();
-                    issue_s(u);
-                }
-            }
-            for (int u = 0; ok && u < nu; ++u) {
-                const int s = u % kStages;
-                const uint32_t b = (uint32_t)(u & 1) * 64;
-                if (!wait_w(B_PFULL + (u & 1), (u >> 1) & 1, 92)) { ok = false; break; }
+                const int s = u % S;
+                const uint32_t b = C::kColBuf + (uint32_t)(u % DEPTH) * 2 * W;
+                if (!wait_w(C::B_KFULL + s, (u / S) & 1, 91)) return false;
                 tc_fence_after();
-                // the step's K as an MN-major B operand (N = head dim, K = the 64 keys)
-                const uint64_t kmn = umma_desc_sw128(smem_u32(sk + s * kKTile), kKPanel, 1024);
+                const uint64_t dk = umma_desc_sw128(smem_u32(sk + s * C::kTile), 16, 1024);
+                const uint64_t dv = umma_desc_sw128(smem_u32(sv + s * C::kTile), 16, 1024);
 #pragma unroll
-                for (int kk = 0; kk < 4; ++kk)
-                    umma_bf16_ts_warp(tmem + kColAcc0, tmem + kColDP + b + slice_col(kk), kmn + kk * (2048 >> 4), idAcc,
-                                      (u > 0 || kk > 0));
-                umma_commit_warp(bar(B_KEMPTY + s));
-                if (u + 2 < nu) {
-                    if (!wait_w(B_KFULL + (u + 2) % kStages, ((u + 2) / kStages) & 1, 93)) { ok = false; break; }
-                    tc_fence_after();
-                    issue_s(u + 2);
-                }
+                for (int ks = 0; ks < 8; ++ks)
+                    umma_bf16_ts_warp(tmem + b, tmem + C::kColQ + 8 * ks,
+                                      dk + (((ks >> 2) * C::kPanel + (ks & 3) * 32) >> 4), idS, ks > 0);
+#pragma unroll
+                for (int ks = 0; ks < 8; ++ks)
+                    umma_bf16_ts_warp(tmem + b + W, tmem + C::kColG + 8 * ks,
+                                      dv + (((ks >> 2) * C::kPanel + (ks & 3) * 32) >> 4), idS, ks > 0);
+                umma_commit_warp(bar(C::B_SFULL + u % DEPTH));
+                return true;
+            };
+            bool ok = wait_w(C::B_QG, 0, 90);
+            if (ok) tc_fence_after();
+            for (int u = 0; ok && u < DEPTH && u < nu; ++u) ok = issue_s(u);
+            for (int u = 0; ok && u < nu; ++u) {
+                const int s = u % S;
+                const uint32_t b = C::kColBuf + (uint32_t)(u % DEPTH) * 2 * W;
+                if (!wait_w(C::B_PFULL + u % DEPTH, (u / DEPTH) & 1, 92)) { ok = false; break; }
+                tc_fence_after();
+                // the step's K as an MN-major B operand (N = head dim, K = the W keys)
+                const uint64_t kmn = umma_desc_sw128(smem_u32(sk + s * C::kTile), C::kPanel, 1024);
+#pragma unroll
+                for (int k = 0; k < W / 16; ++k)
+                    umma_bf16_ts_warp(tmem + C::kColDQ, tmem + b + W + slice_col<W>(k), kmn + k * (2048 >> 4), idAcc,
+                                      (u > 0 || k > 0));
+                umma_commit_warp(bar(C::B_KEMPTY + s));
+                if (u + DEPTH < nu && !issue_s(u + DEPTH)) { ok = false; break; }
             }
-            umma_commit_warp(bar(B_FINAL));
-            mbar_wait_bounded(bar(B_FINAL), 0, prm.err, 94);
+            umma_commit_warp(bar(C::B_FINAL));
+            mbar_wait_bounded(bar(C::B_FINAL), 0, prm.err, 94);
         }
     } else {
         // ---------------------------------------------------------------- softmax + epilogue
+        constexpr int HW = W / 2;
         const int lq = warp & 3, ch = warp >> 2;
         const int row = lq * 32 + lane;
-        const int64_t t = (int64_t)qt * kQT + row;
+        const int64_t t = (int64_t)qt * C::kQT + row;
         const uint32_t lanes = (uint32_t)(lq * 32) << 16;
         const float c = prm.scale_log2;
         int a0 = 0, a1 = 0, b0 = 0, b1 = 0;
@@ -498,52 +533,73 @@ prefill_bwd_dq_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_con
             const int4 w = *reinterpret_cast<const int4 *>(prm.spans + 4 * t);
             a0 = w.x; a1 = w.y; b0 = w.z; b1 = w.w;
         }
-        // rows past T read the padding (lse2 = +inf, D = 0): their P and dS are 0
-        const float lrow = prm.lt[(size_t)h * prm.t_pad + t], drow = prm.dt[(size_t)h * prm.t_pad + t];
+        // rows past T read the padding (-lse2 = -inf, D = 0): their P and dS are 0
+        const uint64_t c2 = f2_pack(c, c);
+        const float nlrow = prm.lt[(size_t)h * prm.t_pad + t], drow = prm.dt[(size_t)h * prm.t_pad + t];
+        const uint64_t nl2 = f2_pack(nlrow, nlrow), d2 = f2_pack(drow, drow);
         auto wait_all = [&](int b, uint32_t parity, int site) {
             const bool r = wait_or_abort(bar(b), parity, prm.err, site, abort_flag);
             return __all_sync(0xffffffffu, r);
         };
-        bool ok = true;
-        for (int u = 0; u < nu; ++u) {
-            const uint32_t b = (uint32_t)(u & 1) * 64 + 32 * ch;
-            const bool partial = prm.kind[e0 + u] != PADOC_TILE_FULL;
-            const int cb = prm.idx[e0 + u] * kKT + 32 * ch;
-            if (!wait_all(B_SFULL + (u & 1), (u >> 1) & 1, 95)) { ok = false; break; }
-            tc_fence_after();
-            uint32_t sr[32], dr[32];
-            tmem_ld32(tmem + lanes + kColS + b, sr);
-            tmem_ld32(tmem + lanes + kColDP + b, dr);
-            uint32_t vis = 0xffffffffu;
-            if (partial) {
-                const int lo0 = clamp32(a0 - cb), lo1 = clamp32(b0 - cb);
-                vis = interval_bits(lo0, max(clamp32(a1 - cb) - lo0, 0), 0) |
-                      interval_bits(lo1, max(clamp32(b1 - cb) - lo1, 0), 0);
-            }
-            tmem_ld_wait();
-            uint32_t dk[16];
-#pragma unroll
-            for (int i = 0; i < 32; i += 2) {
-                const float pe0 = fast_exp2(fmaf(__uint_as_float(sr[i]), c, -lrow));
-                const float pe1 = fast_exp2(fmaf(__uint_as_float(sr[i + 1]), c, -lrow));
-                const float p0 = (vis >> i) & 1u ? pe0 : 0.f;
-                const float p1 = (vis >> (i + 1)) & 1u ? pe1 : 0.f;
-                dk[i >> 1] = pack_bf16x2(p0 * (__uint_as_float(dr[i]) - drow), p1 * (__uint_as_float(dr[i + 1]) - drow));
-            }
-            tmem_st16(tmem + lanes + kColDP + b, dk);
+        // Q and dO rows of this query into tensor memory (dims 64 ch .. 64 ch + 63)
+        {
+            const size_t off = ((size_t)(t < prm.T ? t : 0) * hq + h) * kD + 64 * ch;
+            row_to_tmem(tmem + lanes + C::kColQ + 32 * ch, t < prm.T ? prm.a0 + off : nullptr);
+            row_to_tmem(tmem + lanes + C::kColG + 32 * ch, t < prm.T ? prm.a1 + off : nullptr);
             tmem_st_wait();
             tc_fence_before();
-            mbar_arrive(bar(B_PFULL + (u & 1)));
+            mbar_arrive(bar(C::B_QG));
+        }
+        bool ok = true;
+        for (int u = 0; u < nu; ++u) {
+            const uint32_t b = C::kColBuf + (uint32_t)(u % DEPTH) * 2 * W + HW * ch;
+            const bool partial = prm.kind[e0 + u] != PADOC_TILE_FULL;
+            const int cb = prm.idx[e0 + u] * W + HW * ch;
+            if (!wait_all(C::B_SFULL + u % DEPTH, (u / DEPTH) & 1, 95)) { ok = false; break; }
+            tc_fence_after();
+            uint32_t sr[HW], dr[HW];
+            tmem_ld_cols<HW>(tmem + lanes + b, sr);
+            tmem_ld_cols<HW>(tmem + lanes + b + W, dr);
+            uint32_t vis = 0xffffffffu;
+            if (partial) {
+                const int lo0 = clamp_w(a0 - cb, HW), lo1 = clamp_w(b0 - cb, HW);
+                vis = interval_bits(lo0, max(clamp_w(a1 - cb, HW) - lo0, 0), 0) |
+                      interval_bits(lo1, max(clamp_w(b1 - cb, HW) - lo1, 0), 0);
+            }
+            tmem_ld_wait();
+            uint32_t dk[HW / 2];
+            // two key columns per packed instruction: P = exp2(S c - lse2), dS = P (dP - D)
+            auto column_pairs = [&](auto masked) {
+#pragma unroll
+                for (int i = 0; i < HW; i += 2) {
+                    float x0, x1;
+                    f2_unpack(f2_fma(f2_pack(__uint_as_float(sr[i]), __uint_as_float(sr[i + 1])), c2, nl2), x0, x1);
+                    float p0 = fast_exp2(x0), p1 = fast_exp2(x1);
+                    if (decltype(masked)::value) {
+                        p0 = (vis >> i) & 1u ? p0 : 0.f;
+                        p1 = (vis >> (i + 1)) & 1u ? p1 : 0.f;
+                    }
+                    const uint64_t t = f2_sub(f2_pack(__uint_as_float(dr[i]), __uint_as_float(dr[i + 1])), d2);
+                    float d0, d1;
+                    f2_unpack(f2_mul(f2_pack(p0, p1), t), d0, d1);
+                    dk[i >> 1] = pack_bf16x2(d0, d1);
+                }
+            };
+            if (partial) column_pairs(std::true_type{}); else column_pairs(std::false_type{});
+            tmem_st_cols<HW / 2>(tmem + lanes + b + W, dk);
+            tmem_st_wait();
+            tc_fence_before();
+            mbar_arrive(bar(C::B_PFULL + u % DEPTH));
         }
         // epilogue: dQ times scale, columns 64 ch .. 64 ch + 63 of the thread's row
-        if (ok && (nu == 0 || wait_all(B_FINAL, 0, 96))) {
+        if (ok && (nu == 0 || wait_all(C::B_FINAL, 0, 96))) {
             tc_fence_after();
             __nv_bfloat16 *dst = prm.out0 + ((size_t)(t < prm.T ? t : 0) * hq + h) * kD + 64 * ch;
 #pragma unroll
             for (int cc = 0; cc < 2; ++cc) {
                 uint32_t o[32];
                 if (nu > 0) {
-                    tmem_ld32(tmem + lanes + kColAcc0 + 64 * ch + 32 * cc, o);
+                    tmem_ld32(tmem + lanes + C::kColDQ + 64 * ch + 32 * cc, o);
                     tmem_ld_wait();
                 } else {
 #pragma unroll
@@ -569,21 +625,21 @@ padoc_status padoc_launch_prefill_bwd_tc(const void *q, const void *k, const voi
                                          const padoc_tile_map_dev *k_map, const float *lt, const float *dt,
                                          int64_t t_pad, float scale, void *dq, void *dk, void *dv, cudaStream_t stream)
 {
+    constexpr int WQ = PADOC_BWD_DQ_K_TILE;
+    using CQ = DqCfg<WQ>;
     int *err = padoc_device_error_word();
     if (!err) return PADOC_ERR_CUDA;
     const int64_t T = total_tokens;
-    const int64_t nkt = (T + dkv::kKT - 1) / dkv::kKT, nqt = (T + dqp::kQT - 1) / dqp::kQT;
+    const int64_t nkt = (T + dkv::kKT - 1) / dkv::kKT, nqt = (T + CQ::kQT - 1) / CQ::kQT;
     if (nkt * num_kv_heads > INT32_MAX || nqt * num_q_heads > INT32_MAX) return PADOC_ERR_UNSUPPORTED;
     const uint64_t qcols = (uint64_t)num_q_heads * kD, kcols = (uint64_t)num_kv_heads * kD;
-    CUtensorMap q64, g64, k128, v128, q128, g128, k64, v64;
+    CUtensorMap q64, g64, k128, v128, kmap, vmap;
     if (!padoc_make_tmap_bf16(&q64, q, qcols, T, qcols * 2, 64, dkv::kQT) ||
         !padoc_make_tmap_bf16(&g64, dout, qcols, T, qcols * 2, 64, dkv::kQT) ||
         !padoc_make_tmap_bf16(&k128, k, kcols, T, kcols * 2, 64, dkv::kKT) ||
         !padoc_make_tmap_bf16(&v128, v, kcols, T, kcols * 2, 64, dkv::kKT) ||
-        !padoc_make_tmap_bf16(&q128, q, qcols, T, qcols * 2, 64, dqp::kQT) ||
-        !padoc_make_tmap_bf16(&g128, dout, qcols, T, qcols * 2, 64, dqp::kQT) ||
-        !padoc_make_tmap_bf16(&k64, k, kcols, T, kcols * 2, 64, dqp::kKT) ||
-        !padoc_make_tmap_bf16(&v64, v, kcols, T, kcols * 2, 64, dqp::kKT))
+        !padoc_make_tmap_bf16(&kmap, k, kcols, T, kcols * 2, 64, WQ) ||
+        !padoc_make_tmap_bf16(&vmap, v, kcols, T, kcols * 2, 64, WQ))
         return PADOC_ERR_CUDA;
     BwdParams prm;
     prm.spans = spans_dev;
@@ -611,16 +667,18 @@ padoc_status padoc_launch_prefill_bwd_tc(const void *q, const void *k, const voi
     padoc_status st = padoc_launch_status();
     if (st != PADOC_OK) return st;
 
-    BwdParams pq = prm;   // dQ pass over the query-major map
+    BwdParams pq = prm;   // dQ pass over the query-major map; Q and dO go to tensor memory
     pq.ptr = q_map->ptr;
     pq.idx = q_map->idx;
     pq.kind = q_map->kind;
     pq.order = nullptr;
+    pq.a0 = (const __nv_bfloat16 *)q;
+    pq.a1 = (const __nv_bfloat16 *)dout;
     pq.num_tiles = (int32_t)nqt;
     pq.out0 = (__nv_bfloat16 *)dq;
     pq.out1 = nullptr;
-    PADOC_CUDA_TRY(cudaFuncSetAttribute(prefill_bwd_dq_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                        (int)dqp::kSmemBytes));
-    prefill_bwd_dq_kernel<<<(unsigned)(nqt * num_q_heads), kThreads, dqp::kSmemBytes, stream>>>(q128, g128, k64, v64, pq);
+    PADOC_CUDA_TRY(cudaFuncSetAttribute(prefill_bwd_dq_kernel<WQ>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                        (int)CQ::kSmemBytes));
+    prefill_bwd_dq_kernel<WQ><<<(unsigned)(nqt * num_q_heads), kThreads, CQ::kSmemBytes, stream>>>(kmap, vmap, pq);
     return padoc_launch_status();
 }

@@ -84,7 +84,7 @@ def test_tile_map_bit_exact_vs_oracle_brute_force(seed, qb, kb):
 
 
 @pytest.mark.parametrize("seed", range(6))
-@pytest.mark.parametrize("qb,kb", [(64, 128), (16, 32), (32, 16)])
+@pytest.mark.parametrize("qb,kb", [(32, 128), (16, 32), (64, 16)])
 def test_key_tile_map_is_the_transpose_with_brute_force_kinds(seed, qb, kb):
     # the key-major map of the backward's dK/dV pass: every (q-tile, k-tile) pair of the oracle's
     # brute-force classification, listed per k-tile in ascending q-tile order; the order lists every
