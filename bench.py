@@ -4,7 +4,9 @@ A step is one pass of the hot path over one batch:
   decode  -- one decode step for every branch of the 32-page concurrent serving batch (prefix
              uniform in [1024,4096], Poisson(20) branches per page, log-normal private lengths):
              the decode plan's split-K kernel over the paged bf16 cache plus the split-K merge;
-  prefill -- the packed ancestor prefill of 8 pages x 4096 tokens (reported in "prefill").
+  prefill -- the packed ancestor prefill of 8 pages x 4096 tokens (reported in "prefill");
+  prefill_bwd -- its gradients dQ, dK, dV for a seeded upstream gradient (reported in
+             "prefill_bwd").
 Headline metric: decode queries/s (one query = one branch's newest token, all 16 query heads).
 
 Timing: W untimed warm-up steps, then K steps between CUDA events on the launching stream, with
@@ -38,7 +40,8 @@ FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustain
 # dram__bytes_read.sum + dram__bytes_write.sum per launch from the ncu captures summarised under
 # profiles/ (None until a capture of the current kernel exists). Decode: one step = the three
 # kernels' captures added up (profiles/decode_*_serving_batch.md), cold caches.
-TRAFFIC_BYTES = {"decode": 227_310_000, "prefill": 260_600_000}   # prefill: profiles/prefill_tc_packed_32k.md
+TRAFFIC_BYTES = {"decode": 227_310_000, "prefill": 260_600_000,   # prefill: profiles/prefill_tc_packed_32k.md
+                 "prefill_bwd": None}
 
 
 def load_peaks():
@@ -279,6 +282,46 @@ def bench_prefill(args, torch, dev, rank, world):
     return dict(ms=ms, flops=prefill_flops(wl), tokens=plan.T, steps=steps)
 
 
+def bench_prefill_bwd(args, torch, dev, rank, world):
+    """The gradients of the packed prefill (dQ, dK, dV) for a seeded upstream gradient, after one
+    forward that supplies O and lse; each timed step is one padoc_ancestor_prefill_bwd call."""
+    from paper_2608_06146_gb300 import inputs
+    from paper_2608_06146_gb300 import padoc_attn as pa
+    from paper_2608_06146_gb300.engine import PrefillBwdPlan, PrefillPlan
+
+    wl = inputs.packed_prefill(seed=4 + 1000 * rank)
+    q, k, v = (x.to(dev) for x in inputs.packed_qkv(wl, 4 + 1000 * rank))
+    g = inputs.packed_dout(wl, 4 + 1000 * rank).to(dev)
+    scale = 1.0 / math.sqrt(wl.head_dim)
+    fwd = PrefillPlan(wl.pages, wl.dtype, wl.head_dim, dev)
+    out = torch.empty(q.shape, dtype=q.dtype, device=dev)
+    lse = torch.empty(q.shape[:2], dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream()
+    fwd.run(q, k, v, scale, out, lse, stream)
+    plan = PrefillBwdPlan(wl.pages, wl.dtype, wl.head_dim, wl.num_q_heads, dev)
+    dq, dk, dv = torch.empty_like(q), torch.empty_like(k), torch.empty_like(v)
+    flush = torch.empty(2 * l2_bytes(torch), dtype=torch.uint8, device=dev)
+    steps = max(3, min(args.steps, 20))
+    for _ in range(max(args.warmup, 3)):
+        plan.run(q, k, v, out, g, lse, scale, dq, dk, dv, stream)
+    pa.padoc_check_device_errors(stream)
+    barrier(torch, world)
+    times = []
+    for _ in range(steps):
+        flush.fill_(1)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        plan.run(q, k, v, out, g, lse, scale, dq, dk, dv, stream)
+        e1.record(stream)
+        e1.synchronize()
+        times.append(e0.elapsed_time(e1))
+    pa.padoc_check_device_errors(stream)
+    barrier(torch, world)
+    ms = sum(times) / len(times)
+    # five T x T x d products per visible pair (S, dP, dV, dK, dQ): 2.5x the forward's two
+    return dict(ms=ms, flops=2.5 * prefill_flops(wl), tokens=plan.T, steps=steps)
+
+
 # ------------------------------------------------------------------------------------------------
 # Distributed plumbing (one process per GPU; no data-path collective: pages are independent)
 # ------------------------------------------------------------------------------------------------
@@ -378,7 +421,7 @@ def main():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="padoc", choices=["padoc", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--only", default="all", choices=["all", "decode", "prefill"])
+    ap.add_argument("--only", default="all", choices=["all", "decode", "prefill", "prefill_bwd"])
     ap.add_argument("--replicas", type=int, default=0, help="decode input replicas (0: enough to exceed 4x L2)")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--tc-ctas", type=int, default=0, help="tensor-core decode CTAs (0: one per SM)")
@@ -406,14 +449,16 @@ def main():
 
     from paper_2608_06146_gb300 import build as pbuild
     pbuild.build()
-    if args.only == "prefill":
-        p = bench_prefill(args, torch, dev, rank, world)
+    if args.only in ("prefill", "prefill_bwd"):
+        fn = bench_prefill if args.only == "prefill" else bench_prefill_bwd
+        p = fn(args, torch, dev, rank, world)
         pms = max_over_ranks(torch, world, p["ms"])
         if rank == 0:
-            print(json.dumps({"prefill_ms": pms, "tflops": p["flops"] * world / (pms * 1e-3) / 1e12}))
+            print(json.dumps({f"{args.only}_ms": pms, "tflops": p["flops"] * world / (pms * 1e-3) / 1e12}))
         return 0
     d = bench_decode(args, torch, dev, rank, world)
     p = None if args.only == "decode" else bench_prefill(args, torch, dev, rank, world)
+    pb = None if args.only == "decode" else bench_prefill_bwd(args, torch, dev, rank, world)
 
     peaks, peak_src = load_peaks()
     ms = max_over_ranks(torch, world, d["ms"])
@@ -450,6 +495,19 @@ def main():
                                         "traffic": TRAFFIC_BYTES["prefill"],
                                         "peak_source": f"{peak_src} bf16_tflops (burst)",
                                         "algorithmic_flops": p["flops"]}}
+    if pb is not None:
+        bms = max_over_ranks(torch, world, pb["ms"])
+        achieved = pb["flops"] / (pb["ms"] * 1e-3) / 1e12
+        line["prefill_bwd"] = {"value": pb["flops"] * world / (bms * 1e-3) / 1e12, "unit": "TFLOP/s", "ms_per_step": bms,
+                               "steps": pb["steps"],
+                               "workload": "gradients (dQ, dK, dV) of the packed ancestor prefill, 8 pages x 4096 "
+                                           "tokens, 2.5x the forward's unmasked-entry FLOPs",
+                               "l2": "flushed between steps",
+                               "roofline": {"bound": "tensor", "achieved": achieved, "peak": peaks["bf16_tflops"],
+                                            "unit": "TFLOP/s", "frac": achieved / peaks["bf16_tflops"],
+                                            "traffic": TRAFFIC_BYTES["prefill_bwd"],
+                                            "peak_source": f"{peak_src} bf16_tflops (burst)",
+                                            "algorithmic_flops": pb["flops"]}}
     if rank == 0:
         print(json.dumps(line))
     if world > 1:

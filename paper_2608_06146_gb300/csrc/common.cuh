@@ -288,13 +288,14 @@ padoc_status padoc_launch_decode_tc(const CUtensorMap *kmap, const CUtensorMap *
                                     const padoc_decode_plan *info, const int32_t *page_table, int32_t page_stride,
                                     int32_t num_blocks, float *part_o, float *part_lse, float scale_log2, int *err,
                                     cudaStream_t stream);
-// tcgen05 prefill backward (prefill_bwd_tc.cu): the dK/dV pass and the dQ pass; arguments validated
-// by the caller. lt / dt: [Hq][t_pad] base-2 log-sum-exp and rowsum(dO * O).
-padoc_status padoc_launch_prefill_bwd_tc(const void *q, const void *k, const void *v, const void *dout,
-                                         int64_t total_tokens, int32_t num_q_heads, int32_t num_kv_heads,
-                                         const int32_t *spans_dev, const padoc_tile_map_dev *q_map,
-                                         const padoc_tile_map_dev *k_map, const float *lt, const float *dt,
-                                         int64_t t_pad, float scale, void *dq, void *dk, void *dv, cudaStream_t stream);
+// tcgen05 prefill backward (prefill_bwd_tc.cu): the dQ pass, which also writes lt / dt (per head
+// [Hq][t_pad]: -lse2 and rowsum(dO * O)), then the dK/dV pass; arguments validated by the caller.
+padoc_status padoc_launch_prefill_bwd_tc(const void *q, const void *k, const void *v, const void *out,
+                                         const void *dout, const float *lse, int64_t total_tokens,
+                                         int32_t num_q_heads, int32_t num_kv_heads, const int32_t *spans_dev,
+                                         const padoc_tile_map_dev *q_map, const padoc_tile_map_dev *k_map, float *lt,
+                                         float *dt, int64_t t_pad, float scale, void *dq, void *dk, void *dv,
+                                         cudaStream_t stream);
 int padoc_num_sms();
 
 #define PADOC_CUDA_TRY(expr)                                   \

@@ -1,10 +1,10 @@
 // prefill_bwd.cu -- gradients of C3, the packed ancestor prefill (App. C.1: training through the
-// tree-varlen attention; Sec. 3.2 visibility): the host entry point, its validation, the per-row
-// statistics pass, and the fp32 bring-up kernels. The bf16 passes run on the tensor cores
-// (prefill_bwd_tc.cu).
+// tree-varlen attention; Sec. 3.2 visibility): the host entry point, its validation and the fp32
+// bring-up kernels (a per-row statistics pass, dQ and dK/dV). The bf16 passes run on the tensor
+// cores (prefill_bwd_tc.cu).
 //
 // Per query row and head the backward needs lse (from the forward) and D = sum_c dO[c] O[c]
-// (the softmax's chain-rule term, equal to sum_j P_j dP_j). The statistics pass writes, per head,
+// (the softmax's chain-rule term, equal to sum_j P_j dP_j). Both paths write, per head,
 // [Hq][t_pad] with t_pad = ceil(T / 128) * 128, the negated base-2 log-sum-exp -lse2 (so that
 // P = exp2(S c + (-lse2)) is one fused multiply-add and an exponential) and D; padded rows hold
 // -lse2 = -inf and D = 0, so that their P is exactly 0 and the tile passes need no row test.
@@ -16,16 +16,10 @@ namespace {
 
 constexpr int64_t kPad = 128;
 
-template <typename T>
-__device__ __forceinline__ float ld_f32(const T *p);
-template <>
-__device__ __forceinline__ float ld_f32<float>(const float *p) { return *p; }
-template <>
-__device__ __forceinline__ float ld_f32<__nv_bfloat16>(const __nv_bfloat16 *p) { return __bfloat162float(*p); }
-
-// One warp per (row, head): D = dO . O (fp32) and -lse * log2(e), transposed to [Hq][t_pad].
-template <typename T, int D>
-__global__ void __launch_bounds__(256) prefill_bwd_stats_kernel(const T *__restrict__ out, const T *__restrict__ dout,
+// fp32 path: one warp per (row, head): D = dO . O and -lse * log2(e), transposed to [Hq][t_pad].
+// (The bf16 path computes both inside its dQ pass.)
+template <int D>
+__global__ void __launch_bounds__(256) prefill_bwd_stats_kernel(const float *__restrict__ out, const float *__restrict__ dout,
                                                                 const float *__restrict__ lse, int64_t total_tokens,
                                                                 int64_t t_pad, int32_t hq, float *__restrict__ lt,
                                                                 float *__restrict__ dt)
@@ -38,10 +32,10 @@ __global__ void __launch_bounds__(256) prefill_bwd_stats_kernel(const T *__restr
     const int h = (int)(r % hq);
     float acc = 0.f;
     if (t < total_tokens) {
-        const T *o = out + r * D + lane * E;
-        const T *g = dout + r * D + lane * E;
+        const float *o = out + r * D + lane * E;
+        const float *g = dout + r * D + lane * E;
 #pragma unroll
-        for (int e = 0; e < E; ++e) acc = fmaf(ld_f32(o + e), ld_f32(g + e), acc);
+        for (int e = 0; e < E; ++e) acc = fmaf(o[e], g[e], acc);
 #pragma unroll
         for (int sh = 16; sh > 0; sh >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, sh);
     }
@@ -215,18 +209,13 @@ extern "C" padoc_status padoc_ancestor_prefill_bwd(const void *q, const void *k,
     float *dt = lt + (size_t)num_q_heads * t_pad;
     const float c = scale * PADOC_LOG2E;
     const unsigned sgrid = (unsigned)((t_pad * num_q_heads + 7) / 8);
-    if (dtype == PADOC_DTYPE_BF16) {
-        prefill_bwd_stats_kernel<__nv_bfloat16, 128><<<sgrid, 256, 0, cs>>>(
-            (const __nv_bfloat16 *)out, (const __nv_bfloat16 *)dout, lse, T, t_pad, num_q_heads, lt, dt);
-        padoc_status st = padoc_launch_status();
-        if (st != PADOC_OK) return st;
-        return padoc_launch_prefill_bwd_tc(q, k, v, dout, T, num_q_heads, num_kv_heads, spans_dev, q_map, k_map, lt,
-                                           dt, t_pad, scale, dq, dk, dv, cs);
-    }
+    if (dtype == PADOC_DTYPE_BF16)   // the tensor-core dQ pass computes the statistics itself
+        return padoc_launch_prefill_bwd_tc(q, k, v, out, dout, lse, T, num_q_heads, num_kv_heads, spans_dev, q_map,
+                                           k_map, lt, dt, t_pad, scale, dq, dk, dv, cs);
     const unsigned qgrid = (unsigned)((T * num_q_heads + 3) / 4), kgrid = (unsigned)((T * num_kv_heads + 3) / 4);
 #define PADOC_BWD_F32(D)                                                                                              \
     do {                                                                                                              \
-        prefill_bwd_stats_kernel<float, D><<<sgrid, 256, 0, cs>>>((const float *)out, (const float *)dout, lse, T,    \
+        prefill_bwd_stats_kernel<D><<<sgrid, 256, 0, cs>>>((const float *)out, (const float *)dout, lse, T,    \
                                                                   t_pad, num_q_heads, lt, dt);                        \
         prefill_bwd_dq_f32_kernel<D><<<qgrid, 128, 0, cs>>>((const float *)q, (const float *)k, (const float *)v,     \
                                                             (const float *)dout, spans_dev, lt, dt, T, t_pad,          \

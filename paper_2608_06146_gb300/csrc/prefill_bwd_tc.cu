@@ -50,7 +50,9 @@ constexpr uint32_t kTmemCols = 512;
 struct BwdParams {
     const int32_t *spans, *ptr, *idx, *order;
     const int8_t *kind;
-    const float *lt, *dt;               // [Hq][t_pad]: -lse2 and D
+    float *lt, *dt;                     // [Hq][t_pad]: -lse2 and D (written by the dQ pass, read by the dK/dV pass)
+    const __nv_bfloat16 *o;             // the forward's output (dQ pass: D = dO . O)
+    const float *lse;                   // the forward's log-sum-exp, natural log, [T][Hq]
     const __nv_bfloat16 *a0, *a1;       // the pass's tensor-memory operands: dQ pass Q, dO; dK/dV pass K, V
     int64_t T, t_pad;
     int32_t num_q_heads, num_kv_heads, num_tiles;
@@ -407,7 +409,7 @@ struct DqCfg {
         B_FINAL = 1 + 2 * kStages + 2 * kDepth,
         B_COUNT = 2 + 2 * kStages + 2 * kDepth
     };
-    static constexpr size_t kSmemBytes = 1024 + (size_t)kStages * 2 * kTile + B_COUNT * 8 + 64;
+    static constexpr size_t kSmemBytes = 1024 + (size_t)kStages * 2 * kTile + B_COUNT * 8 + 64 + 2 * kQT * 4;
     static_assert(kDepth >= 1 && W % 32 == 0, "step width");
 };
 
@@ -427,6 +429,7 @@ prefill_bwd_dq_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_con
     uint64_t *bars = (uint64_t *)(sv + S * C::kTile);
     uint32_t *tmem_slot = (uint32_t *)(bars + C::B_COUNT);
     volatile int *abort_flag = (volatile int *)(tmem_slot + 1);
+    float *dsum = (float *)(tmem_slot + 16);   // [2][128]: the two column halves' parts of D
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int hq = prm.num_q_heads, group = hq / prm.num_kv_heads;
@@ -533,23 +536,52 @@ prefill_bwd_dq_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_con
             const int4 w = *reinterpret_cast<const int4 *>(prm.spans + 4 * t);
             a0 = w.x; a1 = w.y; b0 = w.z; b1 = w.w;
         }
-        // rows past T read the padding (-lse2 = -inf, D = 0): their P and dS are 0
         const uint64_t c2 = f2_pack(c, c);
-        const float nlrow = prm.lt[(size_t)h * prm.t_pad + t], drow = prm.dt[(size_t)h * prm.t_pad + t];
-        const uint64_t nl2 = f2_pack(nlrow, nlrow), d2 = f2_pack(drow, drow);
         auto wait_all = [&](int b, uint32_t parity, int site) {
             const bool r = wait_or_abort(bar(b), parity, prm.err, site, abort_flag);
             return __all_sync(0xffffffffu, r);
         };
-        // Q and dO rows of this query into tensor memory (dims 64 ch .. 64 ch + 63)
+        // Q and dO rows of this query into tensor memory (dims 64 ch .. 64 ch + 63), and the row's
+        // statistics: D = dO . O (fp32, the two column halves added through shared memory) and
+        // -lse2; rows past T get -lse2 = -inf and D = 0, so that their P and dS are 0. Every
+        // (row, head) of [0, t_pad) belongs to exactly one CTA, which writes them for the dK/dV pass.
+        float nlrow, drow;
         {
-            const size_t off = ((size_t)(t < prm.T ? t : 0) * hq + h) * kD + 64 * ch;
-            row_to_tmem(tmem + lanes + C::kColQ + 32 * ch, t < prm.T ? prm.a0 + off : nullptr);
-            row_to_tmem(tmem + lanes + C::kColG + 32 * ch, t < prm.T ? prm.a1 + off : nullptr);
+            const bool in = t < prm.T;
+            const size_t off = ((size_t)(in ? t : 0) * hq + h) * kD + 64 * ch;
+            row_to_tmem(tmem + lanes + C::kColQ + 32 * ch, in ? prm.a0 + off : nullptr);
+            uint32_t w[32];
+            uint64_t acc2 = f2_pack(0.f, 0.f);
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+                const uint4 x = in ? reinterpret_cast<const uint4 *>(prm.a1 + off)[i] : make_uint4(0u, 0u, 0u, 0u);
+                const uint4 y = in ? reinterpret_cast<const uint4 *>(prm.o + off)[i] : make_uint4(0u, 0u, 0u, 0u);
+                const uint32_t xs[4] = {x.x, x.y, x.z, x.w}, ys[4] = {y.x, y.y, y.z, y.w};
+#pragma unroll
+                for (int j = 0; j < 4; ++j) {
+                    w[4 * i + j] = xs[j];
+                    acc2 = f2_fma(f2_pack(__uint_as_float(xs[j] << 16), __uint_as_float(xs[j] & 0xffff0000u)),
+                                  f2_pack(__uint_as_float(ys[j] << 16), __uint_as_float(ys[j] & 0xffff0000u)), acc2);
+                }
+            }
+            tmem_st32(tmem + lanes + C::kColG + 32 * ch, w);
             tmem_st_wait();
             tc_fence_before();
             mbar_arrive(bar(C::B_QG));
+            float lo, hi;
+            f2_unpack(acc2, lo, hi);
+            dsum[ch * C::kQT + row] = lo + hi;
+            named_bar_sync(1, 256);   // the eight softmax warps
+            drow = dsum[row] + dsum[C::kQT + row];
+            const float l = in ? prm.lse[(size_t)t * hq + h] : -INFINITY;
+            nlrow = l == -INFINITY ? -INFINITY : -l * PADOC_LOG2E;
+            if (!in) drow = 0.f;
+            if (ch == 0) {
+                prm.lt[(size_t)h * prm.t_pad + t] = nlrow;
+                prm.dt[(size_t)h * prm.t_pad + t] = drow;
+            }
         }
+        const uint64_t nl2 = f2_pack(nlrow, nlrow), d2 = f2_pack(drow, drow);
         bool ok = true;
         for (int u = 0; u < nu; ++u) {
             const uint32_t b = C::kColBuf + (uint32_t)(u % DEPTH) * 2 * W + HW * ch;
@@ -619,11 +651,12 @@ prefill_bwd_dq_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_con
 
 }  // namespace
 
-padoc_status padoc_launch_prefill_bwd_tc(const void *q, const void *k, const void *v, const void *dout,
-                                         int64_t total_tokens, int32_t num_q_heads, int32_t num_kv_heads,
-                                         const int32_t *spans_dev, const padoc_tile_map_dev *q_map,
-                                         const padoc_tile_map_dev *k_map, const float *lt, const float *dt,
-                                         int64_t t_pad, float scale, void *dq, void *dk, void *dv, cudaStream_t stream)
+padoc_status padoc_launch_prefill_bwd_tc(const void *q, const void *k, const void *v, const void *out,
+                                         const void *dout, const float *lse, int64_t total_tokens,
+                                         int32_t num_q_heads, int32_t num_kv_heads, const int32_t *spans_dev,
+                                         const padoc_tile_map_dev *q_map, const padoc_tile_map_dev *k_map, float *lt,
+                                         float *dt, int64_t t_pad, float scale, void *dq, void *dk, void *dv,
+                                         cudaStream_t stream)
 {
     constexpr int WQ = PADOC_BWD_DQ_K_TILE;
     using CQ = DqCfg<WQ>;
@@ -652,6 +685,27 @@ padoc_status padoc_launch_prefill_bwd_tc(const void *q, const void *k, const voi
     prm.scale_log2 = scale * PADOC_LOG2E;
     prm.scale = scale;
     prm.err = err;
+    prm.o = nullptr;
+    prm.lse = nullptr;
+
+    // the dQ pass first: it also writes -lse2 and D of every row for the dK/dV pass
+    BwdParams pq = prm;   // dQ pass over the query-major map; Q and dO go to tensor memory
+    pq.ptr = q_map->ptr;
+    pq.idx = q_map->idx;
+    pq.kind = q_map->kind;
+    pq.order = nullptr;
+    pq.a0 = (const __nv_bfloat16 *)q;
+    pq.a1 = (const __nv_bfloat16 *)dout;
+    pq.num_tiles = (int32_t)nqt;
+    pq.out0 = (__nv_bfloat16 *)dq;
+    pq.out1 = nullptr;
+    pq.o = (const __nv_bfloat16 *)out;
+    pq.lse = lse;
+    PADOC_CUDA_TRY(cudaFuncSetAttribute(prefill_bwd_dq_kernel<WQ>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                        (int)CQ::kSmemBytes));
+    prefill_bwd_dq_kernel<WQ><<<(unsigned)(nqt * num_q_heads), kThreads, CQ::kSmemBytes, stream>>>(kmap, vmap, pq);
+    padoc_status st = padoc_launch_status();
+    if (st != PADOC_OK) return st;
 
     BwdParams pk = prm;   // dK/dV pass over the key-major map
     pk.ptr = k_map->ptr;
@@ -664,21 +718,6 @@ padoc_status padoc_launch_prefill_bwd_tc(const void *q, const void *k, const voi
     PADOC_CUDA_TRY(cudaFuncSetAttribute(prefill_bwd_dkv_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                         (int)dkv::kSmemBytes));
     prefill_bwd_dkv_kernel<<<(unsigned)(nkt * num_kv_heads), kThreads, dkv::kSmemBytes, stream>>>(q64, g64, k128, v128, pk);
-    padoc_status st = padoc_launch_status();
-    if (st != PADOC_OK) return st;
 
-    BwdParams pq = prm;   // dQ pass over the query-major map; Q and dO go to tensor memory
-    pq.ptr = q_map->ptr;
-    pq.idx = q_map->idx;
-    pq.kind = q_map->kind;
-    pq.order = nullptr;
-    pq.a0 = (const __nv_bfloat16 *)q;
-    pq.a1 = (const __nv_bfloat16 *)dout;
-    pq.num_tiles = (int32_t)nqt;
-    pq.out0 = (__nv_bfloat16 *)dq;
-    pq.out1 = nullptr;
-    PADOC_CUDA_TRY(cudaFuncSetAttribute(prefill_bwd_dq_kernel<WQ>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                        (int)CQ::kSmemBytes));
-    prefill_bwd_dq_kernel<WQ><<<(unsigned)(nqt * num_q_heads), kThreads, CQ::kSmemBytes, stream>>>(kmap, vmap, pq);
     return padoc_launch_status();
 }
