@@ -41,7 +41,7 @@ FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustain
 # profiles/ (None until a capture of the current kernel exists). Decode: one step = the three
 # kernels' captures added up (profiles/decode_*_serving_batch.md), cold caches.
 TRAFFIC_BYTES = {"decode": 227_310_000, "prefill": 260_600_000,   # prefill: profiles/prefill_tc_packed_32k.md
-                 "prefill_bwd": None}
+                 "prefill_bwd": 1_459_570_000}  # both passes: profiles/prefill_bwd_packed_32k.md
 
 
 def load_peaks():
