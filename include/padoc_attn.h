@@ -22,7 +22,8 @@
  * Conventions for every call
  *   - Ownership: the caller owns every buffer. The library never allocates device memory, never
  *     keeps a pointer after a call returns and never synchronizes, except
- *     padoc_check_device_errors.
+ *     padoc_check_device_errors. The one object it allocates is the decoding loop's host-side
+ *     scheduler state (padoc_mpd_create / padoc_mpd_destroy).
  *   - Host pointers are marked (host); device pointers (device). Device calls are asynchronous on
  *     the given stream (a cudaStream_t; NULL is the legacy default stream).
  *   - Every argument is validated on the host before any launch; a failed check returns
@@ -217,6 +218,31 @@ padoc_status padoc_decode_plan_size(const padoc_page *pages, int32_t num_pages, 
 padoc_status padoc_build_decode_plan(const padoc_page *pages, int32_t num_pages, const padoc_decode_config *cfg,
                                      int32_t *plan, int64_t capacity_ints, padoc_decode_plan *info);
 
+/* One stream of an explicit stream list (the per-branch plan {page, shared_len = P + f_k,
+ * private_len} of C1, given directly instead of derived from padoc_page records). */
+typedef struct {
+    int32_t page;         /* index into the list's pages; streams are grouped page by page, pages ascending */
+    int32_t shared_len;   /* cutoff on the page's shared stream: P + f_k for a branch, the page's whole
+                             shared length for its layout stream; 0 <= shared_len <= page_len[page] */
+    int32_t private_len;  /* private rows, the newest being the token decoded; 0 for a layout stream */
+} padoc_stream_desc;
+
+/* padoc_decode_plan_size / padoc_build_decode_plan for an explicit stream list, as the decoding loop
+ * of Algorithm 1 has it at each step: a page's layout stream may have retired while its branches
+ * live on, and branches join and leave the batch one by one (App. E.1: a completed stream's row is
+ * removed). page_len: (host) int32 [num_pages], the shared-stream tokens of each page in the cache;
+ * streams: (host) [num_streams]; cfg->layout_streams must be 0 (the list names every stream). The
+ * plan is the one padoc_build_decode_plan gives for the same streams in the same order; Q, out and
+ * lse rows follow the list. A page with no stream is skipped.
+ * Errors: INVALID_ARGUMENT (also for streams out of page order or a cutoff past page_len);
+ * UNSUPPORTED; CAPACITY. */
+padoc_status padoc_decode_plan_size_streams(const int32_t *page_len, int32_t num_pages, const padoc_stream_desc *streams,
+                                            int32_t num_streams, const padoc_decode_config *cfg, int64_t *plan_ints);
+padoc_status padoc_build_decode_plan_streams(const int32_t *page_len, int32_t num_pages,
+                                             const padoc_stream_desc *streams, int32_t num_streams,
+                                             const padoc_decode_config *cfg, int32_t *plan, int64_t capacity_ints,
+                                             padoc_decode_plan *info);
+
 /* Workspace (device) bytes padoc_branch_decode_attn needs for this plan (split-K partials). */
 padoc_status padoc_decode_workspace_size(const padoc_decode_plan *info, size_t *bytes);
 
@@ -277,6 +303,124 @@ padoc_status padoc_branch_decode_attn_noalloc(const padoc_kv_pool *pool, const p
 padoc_status padoc_splitk_combine(const float *part_o, const float *part_lse, int32_t num_splits, int64_t rows,
                                   int32_t head_dim, padoc_dtype out_dtype, void *out, float *lse,
                                   padoc_stream_t stream);
+
+/* ============================================================================================
+ * Algorithm 1 (App. E.1): the masked parallel decoding loop over the paged cache
+ * ========================================================================================== */
+
+/* Host-side scheduler state of the loop for a batch of pages sharing one KV pool (opaque; created by
+ * padoc_mpd_create, freed by padoc_mpd_destroy: the one object this library allocates, in host
+ * memory). It keeps, per page, the shared stream's blocks (prefix X, then the layout stream's
+ * tokens) and, per stream, its cutoff on the shared stream and its private blocks, and it hands out
+ * and takes back pool blocks. It realises the logical mask M of App. E.1 without materialising it:
+ *   - each step appends one input per live stream (M <- [M I_C]): the layout stream's input extends
+ *     the page's shared stream, a branch's input extends its private rows;
+ *   - a fork copies the layout stream's pre-boundary row: the new branch's cutoff is the page's
+ *     shared length at that moment (P + the layout tokens in the cache), and it appends its
+ *     branch-initialization input at the next step;
+ *   - a retired branch's private blocks return to the pool; a page's shared blocks return when its
+ *     last stream retires (a completed stream's row is removed and its positions are never read
+ *     again).
+ * Streams of a step are ordered page by page (pages in admission order), within a page its live
+ * branches in fork order, then its layout stream while it is live. Stream ids count up from 0 in
+ * creation order over the object's life. Not thread-safe: one caller at a time. */
+typedef struct padoc_mpd padoc_mpd;
+
+/* num_blocks pool blocks of block_size (16) tokens, handed out first in the order of block_order
+ * ((host) int32 [num_blocks], a permutation of 0..num_blocks-1; NULL = ascending); returned blocks
+ * are handed out again after those (first in, first out). Errors: INVALID_ARGUMENT, UNSUPPORTED. */
+padoc_status padoc_mpd_create(int32_t num_blocks, int32_t block_size, const int32_t *block_order, padoc_mpd **mpd);
+void padoc_mpd_destroy(padoc_mpd *mpd);
+
+/* Admits a page whose prefix X has prefix_len tokens (Algorithm 1: "Prefill X; initialize the
+ * layout stream"). prefix_slots: (host) int32 [prefix_len] receives the pool slot
+ * (block * block_size + offset) of each prefix token; the caller writes the prefix K/V there
+ * (padoc_append_inputs) before the first step that decodes the page. The prefill's output decides
+ * the first events: num_forks branches forked from the prefill (f = 0: they see X only) and
+ * layout_eos = 1 when the layout stream ends at once. new_streams: (host) int32 [1 + num_forks]
+ * receives the layout stream's id (-1 with layout_eos) and then the new branches' ids.
+ * page_id: (host) the page's id (admission counter). Errors: INVALID_ARGUMENT (also during a step,
+ * between padoc_mpd_begin_step and padoc_mpd_end_step); CAPACITY when the pool has too few free
+ * blocks (nothing changes). */
+padoc_status padoc_mpd_add_page(padoc_mpd *mpd, int32_t prefix_len, int32_t num_forks, int32_t layout_eos,
+                                int32_t *page_id, int32_t *prefix_slots, int32_t *new_streams);
+
+/* Begins one step: "Let C be the live-stream count and i their next inputs. Append i to the cache"
+ * (Algorithm 1). Every live stream gets the pool slot of its next input (a new block when its next
+ * row starts one); its length counts that input from now on. stream_ids, append_slots: (host) int32
+ * [capacity] receive the step's streams in order and their slots; num_streams: C.
+ * Errors: INVALID_ARGUMENT (null pointers, a step already begun); CAPACITY when capacity < C or the
+ * pool has too few free blocks (nothing changes). */
+padoc_status padoc_mpd_begin_step(padoc_mpd *mpd, int32_t *num_streams, int32_t *stream_ids, int32_t *append_slots,
+                                  int32_t capacity);
+
+/* Sizes of the current step's decode tables: live pages, live streams, the widest page and stream
+ * block lists. Valid between padoc_mpd_begin_step and padoc_mpd_end_step. */
+padoc_status padoc_mpd_step_shape(const padoc_mpd *mpd, int32_t *num_pages, int32_t *num_streams,
+                                  int32_t *max_page_blocks, int32_t *max_stream_blocks);
+
+/* The current step's decode inputs, in step order: page_len (host) int32 [num_pages] and streams
+ * (host) [num_streams] for padoc_build_decode_plan_streams, and the block tables for
+ * padoc_branch_decode_attn: page_table (host) int32 [num_pages][page_stride], stream_table (host)
+ * int32 [num_streams][stream_stride], unused entries -1. Strides at least the step_shape widths
+ * (stream_stride >= 1). Errors: INVALID_ARGUMENT (also outside a step). */
+padoc_status padoc_mpd_step_tables(const padoc_mpd *mpd, int32_t *page_len, padoc_stream_desc *streams,
+                                   int32_t *page_table, int32_t page_stride, int32_t *stream_table,
+                                   int32_t stream_stride);
+
+/* Ends the step with each stream's output event, in step order ((host) arrays [num_streams], the
+ * C of padoc_mpd_begin_step): num_forks[i] branches forked from stream i's output ("the layout
+ * output completes region B_k": only a layout stream forks; NULL = none), eos[i] != 0 when stream
+ * i's output is EOS (it retires; NULL = none). A layout stream may fork and retire on the same
+ * output. new_streams: (host) int32 [capacity] receives the new branches' ids (in step order, a
+ * stream's forks consecutively), num_new their count. Errors: INVALID_ARGUMENT (no step begun, a
+ * wrong count, a branch that forks); CAPACITY when capacity is below the new branches (nothing
+ * changes). */
+padoc_status padoc_mpd_end_step(padoc_mpd *mpd, const int32_t *num_forks, const uint8_t *eos, int32_t num_streams,
+                                int32_t *new_streams, int32_t capacity, int32_t *num_new);
+
+/* Layout of one step prepared by padoc_mpd_prepare_step in the caller's int32 staging buffer
+ * (offsets in int32 words, each a multiple of 32, so every part starts on a 128-byte boundary). */
+typedef struct {
+    int32_t num_streams;       /* C: the step's streams */
+    int32_t num_pages;         /* live pages (rows of the page table) */
+    int32_t page_stride;       /* page-table row width (>= 1) */
+    int32_t stream_stride;     /* stream-table row width (>= 1) */
+    int64_t off_plan;          /* the decode plan blob (plan.plan_ints words) */
+    int64_t off_page_table;    /* int32 [num_pages][page_stride], unused entries -1 */
+    int64_t off_stream_table;  /* int32 [num_streams][stream_stride], unused entries -1 */
+    int64_t off_slots;         /* int32 [num_streams]: each stream's append slot */
+    int64_t off_rows;          /* int32 [num_streams]: left for the caller (e.g. the source rows of the
+                                  inputs for padoc_append_inputs), not written */
+    int64_t off_stream_ids;    /* int32 [num_streams]: the step's stream ids (host use) */
+    int64_t upload_words;      /* [0, upload_words) is what the device needs: everything but the ids */
+    int64_t total_words;       /* words the step needs in the staging buffer */
+    padoc_decode_plan plan;    /* host summary of the step's decode plan */
+} padoc_mpd_step;
+
+/* One call for a step's host work: padoc_mpd_begin_step, padoc_mpd_step_tables and
+ * padoc_build_decode_plan_streams (with cfg; cfg->layout_streams 0) in one planner pass, written
+ * into stage ((host) int32 [capacity_words], e.g. pinned memory for one host->device copy) in the
+ * layout `step` describes. With too small a capacity it returns CAPACITY with step->total_words
+ * set and begins nothing; so does a pool without enough free blocks (step->total_words = 0).
+ * Errors: INVALID_ARGUMENT (also a step already begun), UNSUPPORTED, CAPACITY. */
+padoc_status padoc_mpd_prepare_step(padoc_mpd *mpd, const padoc_decode_config *cfg, int32_t *stage,
+                                    int64_t capacity_words, padoc_mpd_step *step);
+
+/* Live pages, live streams and free pool blocks. */
+padoc_status padoc_mpd_status(const padoc_mpd *mpd, int32_t *live_pages, int32_t *live_streams, int32_t *free_blocks);
+
+/* Writes one step's inputs (device): for i < count, the K and V rows src_rows[i] of k_src / v_src
+ * ([src_total][Hkv][head_dim]) go to pool slot slots[i] (block slots[i] / block_size, row
+ * slots[i] % block_size, every KV head), and, when q_src is not NULL, Q row src_rows[i] of q_src
+ * ([src_total][num_q_heads][head_dim]) goes to row i of q_dst ([count][num_q_heads][head_dim]), the
+ * decode call's query order. src_rows NULL means row i. The pool's K and V arrays are written;
+ * everything is in the pool's dtype, 16-byte aligned. Used for the prefix of a new page and for
+ * every step's inputs (Algorithm 1's append). A slot or source row out of range sets the device
+ * error word (code 1) and that row is skipped. Errors: INVALID_ARGUMENT, UNSUPPORTED, CUDA. */
+padoc_status padoc_append_inputs(const padoc_kv_pool *pool, const void *k_src, const void *v_src, const void *q_src,
+                                 int64_t src_total, int32_t num_q_heads, void *q_dst, const int32_t *src_rows,
+                                 const int32_t *slots, int32_t count, padoc_stream_t stream);
 
 /* ============================================================================================
  * C3: packed variable-length ancestor prefill (training forward / branch prefill)

@@ -16,6 +16,7 @@
 
 #include "padoc_attn.h"
 #include "plan_internal.h"
+#include "plan_build.h"
 
 namespace {
 
@@ -229,7 +230,6 @@ extern "C" padoc_status padoc_prefill_bwd_tile_shapes(padoc_dtype dtype, int32_t
 
 namespace {
 
-struct Stream { int32_t page, shared_len, private_len; };
 
 // Multiprocessor count of the current CUDA device, or 152 (one GB300) when none is visible; the
 // device attribute is read once per device (a plan is built for every decode step).
@@ -254,38 +254,26 @@ int32_t padoc_default_ctas()
     return n;
 }
 
-struct PlanParts;
 int32_t choose_tc_ctas(const PlanParts &pp, const padoc_decode_config *cfg, int64_t total_w, int64_t max_piece);
 
-struct PlanParts {
-    std::vector<Stream> streams;
-    std::vector<int32_t> page_len, page_first_stream, page_num_streams;
-    std::vector<int32_t> slot_ptr;      // [S * Hkv + 1]: partial slots of each (stream, KV head)
-    std::vector<int32_t> cta_ptr;       // [tc_ctas + 1]: tensor-core items of each CTA
-    std::vector<int32_t> warp_ptr;      // [num_warps + 1]: warp items of each warp (from the first)
-    std::vector<padoc_item> items;
-    int32_t num_tc_items = 0, tc_ctas = 0, num_warps = 0;
-    int32_t max_page_blocks = 0, max_stream_blocks = 0;
-    int64_t kv_tokens = 0;
-};
-
-padoc_status build_parts(const padoc_page *pages, int32_t num_pages, const padoc_decode_config *cfg, PlanParts &pp)
+padoc_status check_config(const padoc_decode_config *cfg)
 {
     if (!cfg) return PADOC_ERR_INVALID_ARGUMENT;
-    if (num_pages < 0 || (num_pages > 0 && !pages)) return PADOC_ERR_INVALID_ARGUMENT;
     if (cfg->num_q_heads < 1 || cfg->num_kv_heads < 1 || cfg->num_q_heads % cfg->num_kv_heads != 0)
         return PADOC_ERR_INVALID_ARGUMENT;
     if (cfg->head_dim < 1 || cfg->block_size < 1) return PADOC_ERR_INVALID_ARGUMENT;
     if (cfg->block_size != 16) return PADOC_ERR_UNSUPPORTED;
     if (cfg->split_tokens < 0 || (cfg->split_tokens > 0 && cfg->split_tokens % cfg->block_size != 0))
         return PADOC_ERR_INVALID_ARGUMENT;
-    const int32_t bs = cfg->block_size;
     if (cfg->tc_ctas < 0 || cfg->warp_ctas < 0) return PADOC_ERR_INVALID_ARGUMENT;
-    const int32_t split = std::min(cfg->split_tokens > 0 ? cfg->split_tokens : PADOC_DEFAULT_SPLIT_TOKENS,
-                                   PADOC_WARP_MAX_ITEM_TOKENS);
-    const int32_t psplit = PADOC_PRIVATE_SPLIT_TOKENS;
-    const int32_t group = cfg->num_q_heads / cfg->num_kv_heads;
+    return PADOC_OK;
+}
 
+// Streams of the pages (each page's branches, then its layout stream when cfg->layout_streams).
+padoc_status streams_of_pages(const padoc_page *pages, int32_t num_pages, const padoc_decode_config *cfg,
+                              PlanParts &pp)
+{
+    if (num_pages < 0 || (num_pages > 0 && !pages)) return PADOC_ERR_INVALID_ARGUMENT;
     for (int32_t p = 0; p < num_pages; ++p) {
         const padoc_page &pg = pages[p];
         if (pg.prefix_len < 0 || pg.layout_len < 0 || pg.num_branches < 0) return PADOC_ERR_INVALID_ARGUMENT;
@@ -304,11 +292,54 @@ padoc_status build_parts(const padoc_page *pages, int32_t num_pages, const padoc
             pp.streams.push_back({p, (int32_t)plen, 0});
         }
         pp.page_num_streams.push_back((int32_t)pp.streams.size() - pp.page_first_stream.back());
+    }
+    return PADOC_OK;
+}
+
+// An explicit stream list: page_len[p] shared-stream tokens of page p, streams grouped by page in
+// ascending page order, each cutting the page's shared stream at shared_len <= page_len.
+padoc_status streams_of_list(const int32_t *page_len, int32_t num_pages, const padoc_stream_desc *streams,
+                             int32_t num_streams, PlanParts &pp)
+{
+    if (num_pages < 0 || num_streams < 0 || (num_pages > 0 && !page_len) || (num_streams > 0 && !streams))
+        return PADOC_ERR_INVALID_ARGUMENT;
+    for (int32_t p = 0; p < num_pages; ++p) {
+        if (page_len[p] < 0 || page_len[p] >= (1 << 30)) return PADOC_ERR_INVALID_ARGUMENT;
+        pp.page_len.push_back(page_len[p]);
+    }
+    pp.page_first_stream.assign(num_pages, 0);
+    pp.page_num_streams.assign(num_pages, 0);
+    int32_t prev = 0;
+    for (int32_t s = 0; s < num_streams; ++s) {
+        const padoc_stream_desc &d = streams[s];
+        if (d.page < prev || d.page >= num_pages) return PADOC_ERR_INVALID_ARGUMENT;  // grouped, ascending
+        if (d.shared_len < 0 || d.shared_len > page_len[d.page]) return PADOC_ERR_INVALID_ARGUMENT;
+        if (d.private_len < 0 || d.private_len >= (1 << 30)) return PADOC_ERR_INVALID_ARGUMENT;
+        if (pp.page_num_streams[d.page]++ == 0) pp.page_first_stream[d.page] = s;
+        prev = d.page;
+        pp.streams.push_back({d.page, d.shared_len, d.private_len});
+    }
+    for (int32_t p = 0; p < num_pages; ++p)
+        if (pp.page_num_streams[p] == 0) pp.page_first_stream[p] = p > 0 ? pp.page_first_stream[p - 1] + pp.page_num_streams[p - 1] : 0;
+    return PADOC_OK;
+}
+
+// The split-K work of a stream list (pp.streams, page_len, page_first_stream, page_num_streams).
+padoc_status build_work(int32_t num_pages, const padoc_decode_config *cfg, PlanParts &pp)
+{
+    const int32_t bs = cfg->block_size;
+    const int32_t split = std::min(cfg->split_tokens > 0 ? cfg->split_tokens : PADOC_DEFAULT_SPLIT_TOKENS,
+                                   PADOC_WARP_MAX_ITEM_TOKENS);
+    const int32_t psplit = PADOC_PRIVATE_SPLIT_TOKENS;
+    const int32_t group = cfg->num_q_heads / cfg->num_kv_heads;
+
+    for (int32_t p = 0; p < num_pages; ++p) {
+        const int64_t plen = pp.page_len[p];
         pp.max_page_blocks = std::max<int32_t>(pp.max_page_blocks, (int32_t)((plen + bs - 1) / bs));
-        if (pp.page_num_streams.back() > 0) pp.kv_tokens += plen;
+        if (pp.page_num_streams[p] > 0) pp.kv_tokens += plen;
     }
     const int32_t S = (int32_t)pp.streams.size();
-    for (const Stream &s : pp.streams) {
+    for (const PlanStream &s : pp.streams) {
         if (s.shared_len + s.private_len < 1) return PADOC_ERR_INVALID_ARGUMENT;
         pp.max_stream_blocks = std::max<int32_t>(pp.max_stream_blocks, (s.private_len + bs - 1) / bs);
         pp.kv_tokens += s.private_len;
@@ -563,7 +594,7 @@ int32_t choose_tc_ctas(const PlanParts &pp, const padoc_decode_config *cfg, int6
             if ((int64_t)ns * group >= PADOC_TC_MIN_ROWS) continue;
             for (int32_t st = f0; st < f0 + ns; ++st) add(pp.streams[(size_t)st].shared_len, split);
         }
-        for (const Stream &st : pp.streams) add(st.private_len, PADOC_PRIVATE_SPLIT_TOKENS);
+        for (const PlanStream &st : pp.streams) add(st.private_len, PADOC_PRIVATE_SPLIT_TOKENS);
     }
     const int64_t wctas = std::min<int64_t>(cfg->warp_ctas > 0 ? cfg->warp_ctas : nsm,
                                             (witems + PADOC_WARP_KERNEL_WARPS - 1) / PADOC_WARP_KERNEL_WARPS);
@@ -587,38 +618,45 @@ int32_t choose_tc_ctas(const PlanParts &pp, const padoc_decode_config *cfg, int6
     return best_n;
 }
 
+}  // namespace
+
 // int32 words of the plan blob: stream_page, shared_len, private_len [S], slot_ptr [S Hkv + 1],
 // items [num_items][8], page_len [num_pages], cta_ptr [tc_ctas + 1], warp_ptr [num_warps + 1]
-int64_t blob_ints(const PlanParts &pp, int32_t num_pages, int32_t hkv)
+int64_t padoc_plan_blob_ints(const PlanParts &pp, int32_t num_pages, int32_t hkv)
 {
     const int64_t S = (int64_t)pp.streams.size();
     return 3 * S + (S * hkv + 1) + (int64_t)pp.items.size() * PADOC_ITEM_INTS + num_pages + (int64_t)pp.cta_ptr.size() +
            (int64_t)pp.warp_ptr.size();
 }
 
-}  // namespace
+namespace {
 
-extern "C" padoc_status padoc_decode_plan_size(const padoc_page *pages, int32_t num_pages,
-                                               const padoc_decode_config *cfg, int64_t *plan_ints)
+padoc_status parts_of_pages(const padoc_page *pages, int32_t num_pages, const padoc_decode_config *cfg,
+                           PlanParts &pp)
 {
-    if (!plan_ints) return PADOC_ERR_INVALID_ARGUMENT;
-    PlanParts pp;
-    padoc_status st = build_parts(pages, num_pages, cfg, pp);
-    if (st != PADOC_OK) return st;
-    *plan_ints = blob_ints(pp, num_pages, cfg->num_kv_heads);
-    return PADOC_OK;
+    padoc_status st = check_config(cfg);
+    if (st == PADOC_OK) st = streams_of_pages(pages, num_pages, cfg, pp);
+    if (st == PADOC_OK) st = build_work(num_pages, cfg, pp);
+    return st;
 }
 
-extern "C" padoc_status padoc_build_decode_plan(const padoc_page *pages, int32_t num_pages,
-                                                const padoc_decode_config *cfg, int32_t *plan,
-                                                int64_t capacity_ints, padoc_decode_plan *info)
+}  // namespace
+
+padoc_status padoc_plan_parts_of_list(const int32_t *page_len, int32_t num_pages, const padoc_stream_desc *streams,
+                                      int32_t num_streams, const padoc_decode_config *cfg, PlanParts &pp)
 {
-    if (!info) return PADOC_ERR_INVALID_ARGUMENT;
-    PlanParts pp;
-    padoc_status st = build_parts(pages, num_pages, cfg, pp);
-    if (st != PADOC_OK) return st;
+    padoc_status st = check_config(cfg);
+    if (st == PADOC_OK && cfg->layout_streams) st = PADOC_ERR_INVALID_ARGUMENT;  // the list names every stream
+    if (st == PADOC_OK) st = streams_of_list(page_len, num_pages, streams, num_streams, pp);
+    if (st == PADOC_OK) st = build_work(num_pages, cfg, pp);
+    return st;
+}
+
+padoc_status padoc_plan_write_blob(const PlanParts &pp, int32_t num_pages, const padoc_decode_config *cfg, int32_t *plan,
+                                   int64_t capacity_ints, padoc_decode_plan *info)
+{
     const int64_t S = (int64_t)pp.streams.size();
-    const int64_t need = blob_ints(pp, num_pages, cfg->num_kv_heads);
+    const int64_t need = padoc_plan_blob_ints(pp, num_pages, cfg->num_kv_heads);
     if (capacity_ints < need) return PADOC_ERR_CAPACITY;
     if (need > 0 && !plan) return PADOC_ERR_INVALID_ARGUMENT;
     std::memset(info, 0, sizeof(*info));
@@ -656,6 +694,52 @@ extern "C" padoc_status padoc_build_decode_plan(const padoc_page *pages, int32_t
     if (!pp.cta_ptr.empty()) std::memcpy(plan + info->off_cta_ptr, pp.cta_ptr.data(), pp.cta_ptr.size() * sizeof(int32_t));
     std::memcpy(plan + info->off_warp_ptr, pp.warp_ptr.data(), pp.warp_ptr.size() * sizeof(int32_t));
     return PADOC_OK;
+}
+
+extern "C" padoc_status padoc_decode_plan_size(const padoc_page *pages, int32_t num_pages,
+                                               const padoc_decode_config *cfg, int64_t *plan_ints)
+{
+    if (!plan_ints) return PADOC_ERR_INVALID_ARGUMENT;
+    PlanParts pp;
+    padoc_status st = parts_of_pages(pages, num_pages, cfg, pp);
+    if (st != PADOC_OK) return st;
+    *plan_ints = padoc_plan_blob_ints(pp, num_pages, cfg->num_kv_heads);
+    return PADOC_OK;
+}
+
+extern "C" padoc_status padoc_build_decode_plan(const padoc_page *pages, int32_t num_pages,
+                                                const padoc_decode_config *cfg, int32_t *plan,
+                                                int64_t capacity_ints, padoc_decode_plan *info)
+{
+    if (!info) return PADOC_ERR_INVALID_ARGUMENT;
+    PlanParts pp;
+    padoc_status st = parts_of_pages(pages, num_pages, cfg, pp);
+    if (st != PADOC_OK) return st;
+    return padoc_plan_write_blob(pp, num_pages, cfg, plan, capacity_ints, info);
+}
+
+extern "C" padoc_status padoc_decode_plan_size_streams(const int32_t *page_len, int32_t num_pages,
+                                                       const padoc_stream_desc *streams, int32_t num_streams,
+                                                       const padoc_decode_config *cfg, int64_t *plan_ints)
+{
+    if (!plan_ints) return PADOC_ERR_INVALID_ARGUMENT;
+    PlanParts pp;
+    padoc_status st = padoc_plan_parts_of_list(page_len, num_pages, streams, num_streams, cfg, pp);
+    if (st != PADOC_OK) return st;
+    *plan_ints = padoc_plan_blob_ints(pp, num_pages, cfg->num_kv_heads);
+    return PADOC_OK;
+}
+
+extern "C" padoc_status padoc_build_decode_plan_streams(const int32_t *page_len, int32_t num_pages,
+                                                        const padoc_stream_desc *streams, int32_t num_streams,
+                                                        const padoc_decode_config *cfg, int32_t *plan,
+                                                        int64_t capacity_ints, padoc_decode_plan *info)
+{
+    if (!info) return PADOC_ERR_INVALID_ARGUMENT;
+    PlanParts pp;
+    padoc_status st = padoc_plan_parts_of_list(page_len, num_pages, streams, num_streams, cfg, pp);
+    if (st != PADOC_OK) return st;
+    return padoc_plan_write_blob(pp, num_pages, cfg, plan, capacity_ints, info);
 }
 
 extern "C" padoc_status padoc_decode_workspace_size(const padoc_decode_plan *info, size_t *bytes)

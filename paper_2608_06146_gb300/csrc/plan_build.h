@@ -1,0 +1,33 @@
+// plan_build.h -- host-only internals of the decode planner (plan.cpp), shared with the decoding
+// loop's scheduler (mpd.cpp), which plans each step from its stream list in one pass.
+#pragma once
+
+#include <stdint.h>
+
+#include <vector>
+
+#include "padoc_attn.h"
+#include "plan_internal.h"
+
+struct PlanStream { int32_t page, shared_len, private_len; };
+
+struct PlanParts {
+    std::vector<PlanStream> streams;
+    std::vector<int32_t> page_len, page_first_stream, page_num_streams;
+    std::vector<int32_t> slot_ptr;      // [S * Hkv + 1]: partial slots of each (stream, KV head)
+    std::vector<int32_t> cta_ptr;       // [tc_ctas + 1]: tensor-core items of each CTA
+    std::vector<int32_t> warp_ptr;      // [num_warps + 1]: warp items of each warp (from the first)
+    std::vector<padoc_item> items;
+    int32_t num_tc_items = 0, tc_ctas = 0, num_warps = 0;
+    int32_t max_page_blocks = 0, max_stream_blocks = 0;
+    int64_t kv_tokens = 0;
+};
+
+// The split-K work of an explicit stream list (padoc_build_decode_plan_streams' rules).
+padoc_status padoc_plan_parts_of_list(const int32_t *page_len, int32_t num_pages, const padoc_stream_desc *streams,
+                                      int32_t num_streams, const padoc_decode_config *cfg, PlanParts &pp);
+// int32 words of the plan blob of pp.
+int64_t padoc_plan_blob_ints(const PlanParts &pp, int32_t num_pages, int32_t hkv);
+// Writes the blob and its host summary (CAPACITY when capacity_ints is too small).
+padoc_status padoc_plan_write_blob(const PlanParts &pp, int32_t num_pages, const padoc_decode_config *cfg, int32_t *plan,
+                                   int64_t capacity_ints, padoc_decode_plan *info);

@@ -82,6 +82,140 @@ class PrefillBwdPlan:
                                       self.workspace, stream)
 
 
+class MaskedParallelLoop:
+    """Algorithm 1 (App. E.1) over the library: the host scheduler (padoc_mpd_*), the append kernel
+    and the decode step on one paged KV pool, with device memory from torch.
+
+    Per step the host asks the scheduler for the live streams and their input slots, builds the
+    step's decode plan from the stream list, and sends slots, source rows, block tables and plan to
+    the device in one copy from pinned memory (two staging buffers, so the host fills one while
+    the previous step's copy may still read the other). The device then appends every input's K/V
+    into the pool, lays out the queries and decodes every stream, all on one CUDA stream."""
+
+    def __init__(self, num_blocks: int, num_q_heads: int, num_kv_heads: int, head_dim: int, dtype: torch.dtype,
+                 device, block_order=None, block_size: int = 16, tc_ctas: int = 0, warp_ctas: int = 0):
+        self.mpd = pa.Mpd(num_blocks, block_size, block_order)
+        self.k_pool = torch.zeros((num_blocks, num_kv_heads, block_size, head_dim), dtype=dtype, device=device)
+        self.v_pool = torch.zeros_like(self.k_pool)
+        self.cfg = pa.make_decode_config(num_q_heads, num_kv_heads, head_dim, block_size, False, 0, tc_ctas,
+                                         warp_ctas)
+        self.device, self.dtype = device, dtype
+        self.num_q_heads, self.head_dim = num_q_heads, head_dim
+        self._stage = [None, None]
+        self._stage_free = [torch.cuda.Event(), torch.cuda.Event()]
+        self._turn = 0
+        self._ints = torch.empty(1024, dtype=torch.int32, device=device)
+        self.workspace = torch.empty(256, dtype=torch.uint8, device=device)
+        self.q_step = torch.empty((64, num_q_heads, head_dim), dtype=dtype, device=device)
+        self.last_info = None
+        self.last_step = None
+        self.last_stage = None
+        self.h2d_bytes = 0
+
+    def _upload(self, parts, stream):
+        """Copies int32 host arrays to the device in one transfer, each starting on a 128-byte
+        boundary; returns device views."""
+        offs, n = [], 0
+        for a in parts:
+            offs.append(n)
+            n += (int(a.size) + 31) // 32 * 32
+        b = self._turn & 1
+        self._turn += 1
+        self._stage_free[b].synchronize()
+        if self._stage[b] is None or self._stage[b].numel() < n:
+            self._stage[b] = torch.empty(max(n, 2 * (0 if self._stage[b] is None else self._stage[b].numel()), 4096),
+                                         dtype=torch.int32).pin_memory()
+        host = self._stage[b].numpy()
+        for a, o in zip(parts, offs):
+            host[o:o + a.size] = a.reshape(-1)
+        if self._ints.numel() < n:
+            self._ints = torch.empty(max(n, 2 * self._ints.numel()), dtype=torch.int32, device=self.device)
+        with torch.cuda.stream(stream):
+            self._ints[:n].copy_(self._stage[b][:n], non_blocking=True)
+        self._stage_free[b].record(stream)
+        self.h2d_bytes = 4 * n
+        return [self._ints[o:o + a.size] for a, o in zip(parts, offs)]
+
+    def add_page(self, prefix_len: int, num_forks: int, layout_eos: bool, k_src, v_src, src_rows, stream=None):
+        """Admits a page: its prefix K/V (rows src_rows of k_src / v_src, device tensors [rows][Hkv][d])
+        go into the blocks the scheduler gives it. Returns (page id, new stream ids)."""
+        stream = stream or torch.cuda.current_stream()
+        pid, slots, new = self.mpd.add_page(prefix_len, num_forks, layout_eos)
+        if prefix_len > 0:
+            slots_d, rows_d = self._upload([slots, np.asarray(src_rows, np.int32)], stream)
+            pa.padoc_append_inputs(self.k_pool, self.v_pool, k_src, v_src, slots_d, src_rows=rows_d, count=prefix_len,
+                                   stream=stream)
+        return pid, new
+
+    def step(self, k_src, v_src, q_src, rows_of, scale: float, out=None, lse=None, stream=None):
+        """One iteration: every live stream appends its next input (rows_of(stream ids) gives the rows
+        of k_src / v_src / q_src that hold them) and is decoded. Returns (stream ids, out [C][Hq][d],
+        lse fp32 [C][Hq]); the caller ends the step with end_step. The host work is one library call
+        (padoc_mpd_prepare_step) into a pinned staging buffer and one copy of it to the device."""
+        stream = stream or torch.cuda.current_stream()
+        b = self._turn & 1
+        self._turn += 1
+        self._stage_free[b].synchronize()
+        if self._stage[b] is None:
+            self._stage[b] = torch.empty(1 << 16, dtype=torch.int32).pin_memory()
+        while True:
+            try:
+                st = self.mpd.prepare_step(self.cfg, self._stage[b].numpy())
+                break
+            except pa.PadocError as e:
+                need = getattr(e, "step", None)
+                if e.status != 6 or need is None or need.total_words <= self._stage[b].numel():
+                    raise
+                self._stage[b] = torch.empty(2 * int(need.total_words), dtype=torch.int32).pin_memory()
+        host = self._stage[b].numpy()
+        C = int(st.num_streams)
+        ids = host[st.off_stream_ids:st.off_stream_ids + C].copy()
+        host[st.off_rows:st.off_rows + C] = rows_of(ids)
+        n = int(st.upload_words)
+        if self._ints.numel() < n:
+            self._ints = torch.empty(max(n, 2 * self._ints.numel()), dtype=torch.int32, device=self.device)
+        with torch.cuda.stream(stream):
+            self._ints[:n].copy_(self._stage[b][:n], non_blocking=True)
+        self._stage_free[b].record(stream)
+        self.h2d_bytes = 4 * n
+        info = st.plan
+        self.last_info = info
+        self.last_step = st
+        self.last_stage = host
+        if C == 0:
+            empty = torch.empty((0, self.num_q_heads), dtype=torch.float32, device=self.device)
+            return ids, torch.empty((0, self.num_q_heads, self.head_dim), dtype=self.dtype, device=self.device), empty
+        d = self._ints
+        plan_d = d[st.off_plan:st.off_plan + info.plan_ints]
+        pt_d = d[st.off_page_table:st.off_page_table + st.num_pages * st.page_stride].view(st.num_pages, st.page_stride)
+        st_d = d[st.off_stream_table:st.off_stream_table + C * st.stream_stride].view(C, st.stream_stride)
+        slots_d = d[st.off_slots:st.off_slots + C]
+        rows_d = d[st.off_rows:st.off_rows + C]
+        if self.q_step.shape[0] < C:
+            self.q_step = torch.empty((max(C, 2 * self.q_step.shape[0]), self.num_q_heads, self.head_dim),
+                                      dtype=self.dtype, device=self.device)
+        q_step = self.q_step[:C]
+        pa.padoc_append_inputs(self.k_pool, self.v_pool, k_src, v_src, slots_d, q_src=q_src, q_dst=q_step,
+                               src_rows=rows_d, count=C, stream=stream)
+        ws = pa.padoc_decode_workspace_size(info)
+        if self.workspace.numel() < ws:
+            self.workspace = torch.empty(max(ws, 2 * self.workspace.numel()), dtype=torch.uint8, device=self.device)
+        if out is None:
+            out = torch.empty((C, self.num_q_heads, self.head_dim), dtype=self.dtype, device=self.device)
+        if lse is None:
+            lse = torch.empty((C, self.num_q_heads), dtype=torch.float32, device=self.device)
+        pa.padoc_branch_decode_attn(self.k_pool, self.v_pool, info, plan_d, pt_d, st_d, q_step, scale, out, lse,
+                                    self.workspace, stream)
+        return ids, out, lse
+
+    def end_step(self, num_forks=None, eos=None, num_streams=None):
+        """Each stream's output event (forks, EOS) in step order; returns the new branches' ids."""
+        return self.mpd.end_step(num_forks, eos, num_streams)
+
+    def status(self):
+        return self.mpd.status()
+
+
 def visible_pairs(pages) -> int:
     """Visible (query, key) pairs of a packed prefill, summed in closed form per page."""
     n = 0

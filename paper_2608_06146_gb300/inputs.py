@@ -154,6 +154,125 @@ WORKLOADS = {
 
 
 # --------------------------------------------------------------------------------------------
+# A synthetic token source for the decoding loop (Algorithm 1)
+# --------------------------------------------------------------------------------------------
+
+class LoopTokenSource:
+    """Stands in for the decoder inside Algorithm 1's loop over ``pages``: each output's event comes
+    from the page structure alone, never from the attention outputs. The layout stream of a page
+    completes region B_k (a fork) when its c-th token is in the cache and f_k = c, and outputs EOS
+    after its L-th token; branch k outputs EOS after its n_k-th token; branches with f_k = 0 fork
+    from the prefill's output. Every input's Q/K/V is the row of the packed tensors (pages back to
+    back, each [X | layout | Y_1 | ... | Y_N], as ``packed_qkv`` draws them) of the token it is, so a
+    loop run decodes exactly the tokens of the packed pages.
+
+    Stream ids are the scheduler's; the source learns them from ``admitted`` and ``forked``.
+    Per-stream state is kept in arrays indexed by stream id, so a step costs a few numpy calls."""
+
+    def __init__(self, pages: Sequence[PageSpec]):
+        self.pages = list(pages)
+        n = len(self.pages)
+        lens = [pg.packed_len for pg in self.pages]
+        self.base = np.concatenate([[0], np.cumsum(lens)[:-1]]).astype(np.int64) if lens else np.zeros(0, np.int64)
+        self.ybase = [[pg.prefix_len + pg.layout_len + int(sum(pg.branch_len[:k])) for k in range(pg.num_branches)]
+                      for pg in self.pages]
+        self._P = np.asarray([pg.prefix_len for pg in self.pages], np.int64)
+        self._L = np.asarray([pg.layout_len for pg in self.pages], np.int64)
+        nb = [pg.num_branches for pg in self.pages]
+        self._kbase = np.concatenate([[0], np.cumsum(nb)[:-1]]).astype(np.int64) if n else np.zeros(0, np.int64)
+        self._yabs = np.asarray([self.base[p] + y for p in range(n) for y in self.ybase[p]], np.int64)
+        self._nlen = np.asarray([x for pg in self.pages for x in pg.branch_len], np.int64)
+        self._forks_by_count = []
+        for pg in self.pages:
+            d = {}
+            for k, f in enumerate(pg.fork_offset):
+                d.setdefault(int(f), []).append(k)
+            self._forks_by_count.append(d)
+        cap = n + int(sum(nb))           # every stream ever: one layout stream and N branches per page
+        self._page = np.full(max(cap, 1), -1, np.int64)
+        self._flat = np.full(max(cap, 1), -1, np.int64)   # -1: layout stream, else flat branch index
+        self._count = np.zeros(max(cap, 1), np.int64)
+        self._pending = {}
+
+    def _grow(self, sid: int) -> None:
+        if sid >= self._page.size:
+            extra = sid + 1 - self._page.size
+            self._page = np.concatenate([self._page, np.full(extra, -1, np.int64)])
+            self._flat = np.concatenate([self._flat, np.full(extra, -1, np.int64)])
+            self._count = np.concatenate([self._count, np.zeros(extra, np.int64)])
+
+    def _set(self, sid: int, p: int, k: int) -> None:
+        self._grow(sid)
+        self._page[sid] = p
+        self._flat[sid] = -1 if k < 0 else self._kbase[p] + k
+        self._count[sid] = 0
+
+    def _forks_at(self, p: int, c: int) -> List[int]:
+        return self._forks_by_count[p].get(int(c), [])
+
+    def stream_of(self, sid: int):
+        """(page, branch index or -1 for the layout stream) of a stream."""
+        p = int(self._page[sid])
+        f = int(self._flat[sid])
+        return p, (-1 if f < 0 else f - int(self._kbase[p]))
+
+    def admission(self, p: int):
+        """(prefix_len, num_forks, layout_eos, prefix rows int64 [P]) of page p's prefill output."""
+        pg = self.pages[p]
+        rows = self.base[p] + np.arange(pg.prefix_len, dtype=np.int64)
+        return pg.prefix_len, len(self._forks_at(p, 0)), pg.layout_len == 0, rows
+
+    def admitted(self, p: int, new_streams) -> None:
+        if int(new_streams[0]) >= 0:
+            self._set(int(new_streams[0]), p, -1)
+        for sid, k in zip(new_streams[1:], self._forks_at(p, 0)):
+            self._set(int(sid), p, k)
+
+    def rows(self, ids) -> np.ndarray:
+        """Packed rows of the inputs the given streams append now (each stream's next token)."""
+        ids = np.asarray(ids, np.int64)
+        pg, fl, c = self._page[ids], self._flat[ids], self._count[ids]
+        lay = fl < 0
+        out = np.where(lay, self.base[pg] + self._P[pg] + c, self._yabs[np.where(lay, 0, fl)] + c)
+        self._count[ids] = c + 1
+        return out
+
+    def events(self, ids):
+        """(num_forks int32 [C], eos uint8 [C]) of the outputs of this step's streams."""
+        ids = np.asarray(ids, np.int64)
+        pg, fl, c = self._page[ids], self._flat[ids], self._count[ids]
+        lay = fl < 0
+        eos = np.where(lay, c == self._L[pg], c == self._nlen[np.where(lay, 0, fl)]).astype(np.uint8)
+        nf = np.zeros(len(ids), np.int32)
+        for i in np.nonzero(lay)[0]:
+            ks = self._forks_at(int(pg[i]), int(c[i]))
+            if ks:
+                self._pending[int(ids[i])] = ks
+                nf[i] = len(ks)
+        return nf, eos
+
+    def forked(self, ids, num_forks, new_streams) -> None:
+        """Records the ids the scheduler gave the branches forked at this step (in step order)."""
+        j = 0
+        for i in np.nonzero(np.asarray(num_forks))[0]:
+            sid = int(ids[i])
+            p = int(self._page[sid])
+            for k in self._pending.pop(sid):
+                self._set(int(new_streams[j]), p, k)
+                j += 1
+
+    def token_rows(self, ids) -> np.ndarray:
+        """Packed rows of the tokens the given streams appended last."""
+        ids = np.asarray(ids, np.int64)
+        pg, fl, c = self._page[ids], self._flat[ids], self._count[ids]
+        lay = fl < 0
+        return np.where(lay, self.base[pg] + self._P[pg] + c - 1, self._yabs[np.where(lay, 0, fl)] + c - 1)
+
+    def token_row(self, sid: int) -> int:
+        return int(self.token_rows([sid])[0])
+
+
+# --------------------------------------------------------------------------------------------
 # Tensors
 # --------------------------------------------------------------------------------------------
 

@@ -49,6 +49,10 @@ class padoc_decode_config(ctypes.Structure):
                 ("tc_ctas", ctypes.c_int32), ("warp_ctas", ctypes.c_int32)]
 
 
+class padoc_stream_desc(ctypes.Structure):
+    _fields_ = [("page", ctypes.c_int32), ("shared_len", ctypes.c_int32), ("private_len", ctypes.c_int32)]
+
+
 class padoc_tile_map_dev(ctypes.Structure):
     _fields_ = [("ptr", ctypes.c_void_p), ("idx", ctypes.c_void_p), ("kind", ctypes.c_void_p),
                 ("order", ctypes.c_void_p), ("q_tile", ctypes.c_int32), ("k_tile", ctypes.c_int32)]
@@ -65,6 +69,14 @@ class padoc_decode_plan(ctypes.Structure):
                 ("off_private_len", ctypes.c_int64), ("off_slot_ptr", ctypes.c_int64), ("off_items", ctypes.c_int64),
                 ("off_page_len", ctypes.c_int64), ("off_cta_ptr", ctypes.c_int64), ("off_warp_ptr", ctypes.c_int64),
                 ("kv_tokens", ctypes.c_int64)]
+
+
+class padoc_mpd_step(ctypes.Structure):
+    _fields_ = [("num_streams", ctypes.c_int32), ("num_pages", ctypes.c_int32), ("page_stride", ctypes.c_int32),
+                ("stream_stride", ctypes.c_int32), ("off_plan", ctypes.c_int64), ("off_page_table", ctypes.c_int64),
+                ("off_stream_table", ctypes.c_int64), ("off_slots", ctypes.c_int64), ("off_rows", ctypes.c_int64),
+                ("off_stream_ids", ctypes.c_int64), ("upload_words", ctypes.c_int64), ("total_words", ctypes.c_int64),
+                ("plan", padoc_decode_plan)]
 
 
 _lib = None
@@ -112,6 +124,25 @@ def load_library(path: Optional[str] = None):
                                        ctypes.c_int32, ctypes.c_int32, _vp, ctypes.POINTER(padoc_tile_map_dev),
                                        ctypes.POINTER(padoc_tile_map_dev), ctypes.c_float, _vp, _vp, _vp, _vp,
                                        ctypes.c_size_t, _vp],
+        "padoc_decode_plan_size_streams": [_i32p, ctypes.c_int32, ctypes.POINTER(padoc_stream_desc), ctypes.c_int32,
+                                           ctypes.POINTER(padoc_decode_config), _i64p],
+        "padoc_build_decode_plan_streams": [_i32p, ctypes.c_int32, ctypes.POINTER(padoc_stream_desc), ctypes.c_int32,
+                                            ctypes.POINTER(padoc_decode_config), _i32p, ctypes.c_int64,
+                                            ctypes.POINTER(padoc_decode_plan)],
+        "padoc_mpd_create": [ctypes.c_int32, ctypes.c_int32, _i32p, ctypes.POINTER(_vp)],
+        "padoc_mpd_destroy": [_vp],
+        "padoc_mpd_add_page": [_vp, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32, _i32p, _i32p, _i32p],
+        "padoc_mpd_begin_step": [_vp, _i32p, _i32p, _i32p, ctypes.c_int32],
+        "padoc_mpd_step_shape": [_vp, _i32p, _i32p, _i32p, _i32p],
+        "padoc_mpd_step_tables": [_vp, _i32p, ctypes.POINTER(padoc_stream_desc), _i32p, ctypes.c_int32, _i32p,
+                                  ctypes.c_int32],
+        "padoc_mpd_end_step": [_vp, _i32p, ctypes.POINTER(ctypes.c_uint8), ctypes.c_int32, _i32p, ctypes.c_int32,
+                               _i32p],
+        "padoc_mpd_status": [_vp, _i32p, _i32p, _i32p],
+        "padoc_mpd_prepare_step": [_vp, ctypes.POINTER(padoc_decode_config), _i32p, ctypes.c_int64,
+                                   ctypes.POINTER(padoc_mpd_step)],
+        "padoc_append_inputs": [ctypes.POINTER(padoc_kv_pool), _vp, _vp, _vp, ctypes.c_int64, ctypes.c_int32, _vp, _vp,
+                                _vp, ctypes.c_int32, _vp],
         "padoc_selftest_tcgen05": [_vp, _vp, _vp, _vp, _vp, _vp, _vp],
         "padoc_check_device_errors": [_vp],
         "padoc_last_device_error": [_i32p, _i32p],
@@ -124,6 +155,7 @@ def load_library(path: Optional[str] = None):
         f.restype = ctypes.c_int
     lib.padoc_status_string.restype = ctypes.c_char_p
     lib.padoc_last_device_error.restype = None
+    lib.padoc_mpd_destroy.restype = None
     _lib = lib
     return lib
 
@@ -135,7 +167,12 @@ def exported_symbols() -> Sequence[str]:
                         "padoc_branch_decode_attn_noalloc",
                         "padoc_splitk_combine", "padoc_ancestor_prefill_attn", "padoc_build_key_tile_map",
                         "padoc_prefill_bwd_tile_shapes", "padoc_prefill_bwd_workspace_size",
-                        "padoc_ancestor_prefill_bwd", "padoc_selftest_tcgen05",
+                        "padoc_ancestor_prefill_bwd", "padoc_decode_plan_size_streams",
+                        "padoc_build_decode_plan_streams", "padoc_mpd_create", "padoc_mpd_destroy",
+                        "padoc_mpd_add_page", "padoc_mpd_begin_step", "padoc_mpd_step_shape",
+                        "padoc_mpd_step_tables", "padoc_mpd_end_step", "padoc_mpd_status", "padoc_mpd_prepare_step",
+                        "padoc_append_inputs",
+                        "padoc_selftest_tcgen05",
                         "padoc_check_device_errors",
                         "padoc_last_device_error", "padoc_status_string", "padoc_version")]
 
@@ -312,6 +349,51 @@ def padoc_build_decode_plan(pages, cfg: padoc_decode_config, out=None):
     return out[:n], info
 
 
+_STREAM_DTYPE = np.dtype([("page", np.int32), ("shared_len", np.int32), ("private_len", np.int32)])
+
+
+def _stream_arr(streams):
+    """streams: numpy array of _STREAM_DTYPE (or an int32 [S][3] array)."""
+    a = np.ascontiguousarray(streams)
+    if a.dtype != _STREAM_DTYPE:
+        a = np.ascontiguousarray(np.asarray(a, np.int32).reshape(-1, 3)).view(_STREAM_DTYPE).reshape(-1)
+    return a, ctypes.cast(a.ctypes.data, ctypes.POINTER(padoc_stream_desc))
+
+
+def padoc_decode_plan_size_streams(page_len, streams, cfg: padoc_decode_config) -> int:
+    lib = load_library()
+    pl = np.ascontiguousarray(page_len, np.int32)
+    sa, sp = _stream_arr(streams)
+    n = ctypes.c_int64()
+    _check("padoc_decode_plan_size_streams",
+           lib.padoc_decode_plan_size_streams(pl.ctypes.data_as(_i32p), pl.size, sp, sa.size, ctypes.byref(cfg),
+                                              ctypes.byref(n)))
+    return n.value
+
+
+def padoc_build_decode_plan_streams(page_len, streams, cfg: padoc_decode_config, out=None):
+    """The decode plan of an explicit stream list (page_len int32 [pages]; streams [S] of
+    (page, shared_len, private_len)). Returns (plan blob, padoc_decode_plan); ``out`` as in
+    padoc_build_decode_plan."""
+    lib = load_library()
+    pl = np.ascontiguousarray(page_len, np.int32)
+    sa, sp = _stream_arr(streams)
+    info = padoc_decode_plan()
+    if out is not None:
+        st = lib.padoc_build_decode_plan_streams(pl.ctypes.data_as(_i32p), pl.size, sp, sa.size, ctypes.byref(cfg),
+                                                 out.ctypes.data_as(_i32p), out.size, ctypes.byref(info))
+        if st == PADOC_OK:
+            return out[:info.plan_ints], info
+        if st != 6:
+            _check("padoc_build_decode_plan_streams", st)
+    n = padoc_decode_plan_size_streams(pl, sa, cfg)
+    out = np.zeros(max(n, 1), np.int32)
+    _check("padoc_build_decode_plan_streams",
+           lib.padoc_build_decode_plan_streams(pl.ctypes.data_as(_i32p), pl.size, sp, sa.size, ctypes.byref(cfg),
+                                               out.ctypes.data_as(_i32p), n, ctypes.byref(info)))
+    return out[:n], info
+
+
 def padoc_decode_workspace_size(info: padoc_decode_plan) -> int:
     lib = load_library()
     b = ctypes.c_size_t()
@@ -359,6 +441,135 @@ def padoc_splitk_combine(part_o, part_lse, out, lse=None, stream=None):
     st = lib.padoc_splitk_combine(_dev(part_o, "part_o"), _dev(part_lse, "part_lse"), S, R, d, _dtype_code(out),
                                   _dev(out, "out"), _dev(lse, "lse"), _stream_ptr(stream))
     _check("padoc_splitk_combine", st)
+
+
+# ------------------------------------------------------------------------------------------------
+# Algorithm 1: the masked parallel decoding loop
+# ------------------------------------------------------------------------------------------------
+
+class Mpd:
+    """The loop's host-side scheduler (padoc_mpd_*). Methods return numpy int32 arrays."""
+
+    def __init__(self, num_blocks: int, block_size: int = 16, block_order=None):
+        self._lib = load_library()
+        h = _vp()
+        order = None if block_order is None else np.ascontiguousarray(block_order, np.int32)
+        _check("padoc_mpd_create", self._lib.padoc_mpd_create(num_blocks, block_size,
+                                                              None if order is None else order.ctypes.data_as(_i32p),
+                                                              ctypes.byref(h)))
+        self._h = h
+        self.block_size = block_size
+        self._cap = 0
+        self._ids = self._slots = None
+
+    def close(self):
+        if self._h:
+            self._lib.padoc_mpd_destroy(self._h)
+            self._h = _vp()
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def add_page(self, prefix_len: int, num_forks: int = 0, layout_eos: bool = False):
+        """Returns (page id, prefix slots int32 [P], new stream ids int32 [1 + num_forks]; the first
+        is the layout stream's, -1 with layout_eos)."""
+        pid = ctypes.c_int32()
+        slots = np.zeros(max(prefix_len, 1), np.int32)
+        new = np.zeros(1 + num_forks, np.int32)
+        _check("padoc_mpd_add_page", self._lib.padoc_mpd_add_page(self._h, prefix_len, num_forks, int(bool(layout_eos)),
+                                                                  ctypes.byref(pid), slots.ctypes.data_as(_i32p),
+                                                                  new.ctypes.data_as(_i32p)))
+        return pid.value, slots[:prefix_len], new
+
+    def begin_step(self):
+        """Returns (stream ids, append slots) of the step, both int32 [C]."""
+        lp, ls, fb = self.status()
+        if ls > self._cap:
+            self._cap = max(ls, 2 * self._cap, 64)
+            self._ids = np.zeros(self._cap, np.int32)
+            self._slots = np.zeros(self._cap, np.int32)
+        c = ctypes.c_int32()
+        ids = self._ids if self._ids is not None else np.zeros(1, np.int32)
+        slots = self._slots if self._slots is not None else np.zeros(1, np.int32)
+        _check("padoc_mpd_begin_step", self._lib.padoc_mpd_begin_step(self._h, ctypes.byref(c), ids.ctypes.data_as(_i32p),
+                                                                      slots.ctypes.data_as(_i32p), max(self._cap, 0)))
+        return ids[:c.value].copy(), slots[:c.value].copy()
+
+    def step_shape(self):
+        a, b, c, d = (ctypes.c_int32() for _ in range(4))
+        _check("padoc_mpd_step_shape", self._lib.padoc_mpd_step_shape(self._h, ctypes.byref(a), ctypes.byref(b),
+                                                                      ctypes.byref(c), ctypes.byref(d)))
+        return a.value, b.value, c.value, d.value
+
+    def step_tables(self, page_stride=None, stream_stride=None):
+        """Returns (page_len int32 [pages], streams [S] of _STREAM_DTYPE, page_table int32 [pages][stride],
+        stream_table int32 [S][stride])."""
+        npg, ns, mp, ms = self.step_shape()
+        page_stride = max(mp, 1) if page_stride is None else page_stride
+        stream_stride = max(ms, 1) if stream_stride is None else stream_stride
+        page_len = np.zeros(max(npg, 1), np.int32)
+        streams = np.zeros(max(ns, 1), _STREAM_DTYPE)
+        pt = np.zeros((max(npg, 1), page_stride), np.int32)
+        stt = np.zeros((max(ns, 1), stream_stride), np.int32)
+        _check("padoc_mpd_step_tables",
+               self._lib.padoc_mpd_step_tables(self._h, page_len.ctypes.data_as(_i32p),
+                                               ctypes.cast(streams.ctypes.data, ctypes.POINTER(padoc_stream_desc)),
+                                               pt.ctypes.data_as(_i32p), page_stride, stt.ctypes.data_as(_i32p),
+                                               stream_stride))
+        return page_len[:npg], streams[:ns], pt[:npg], stt[:ns]
+
+    def end_step(self, num_forks=None, eos=None, num_streams=None):
+        """num_forks int32 [C], eos bool/uint8 [C] (None = all zero). Returns the new branches' ids."""
+        n = num_streams
+        if n is None:
+            n = len(num_forks) if num_forks is not None else len(eos) if eos is not None else 0
+        f = None if num_forks is None else np.ascontiguousarray(num_forks, np.int32)
+        e = None if eos is None else np.ascontiguousarray(eos, np.uint8)
+        total = int(f.sum()) if f is not None else 0
+        new = np.zeros(max(total, 1), np.int32)
+        k = ctypes.c_int32()
+        _check("padoc_mpd_end_step",
+               self._lib.padoc_mpd_end_step(self._h, None if f is None else f.ctypes.data_as(_i32p),
+                                            None if e is None else e.ctypes.data_as(ctypes.POINTER(ctypes.c_uint8)),
+                                            n, new.ctypes.data_as(_i32p), new.size, ctypes.byref(k)))
+        return new[:k.value]
+
+    def prepare_step(self, cfg: padoc_decode_config, stage: np.ndarray) -> padoc_mpd_step:
+        """padoc_mpd_prepare_step into ``stage`` (int32 numpy array, e.g. a view of pinned memory).
+        Raises PadocError (status 6) when the stage is too small; step.total_words is then set on
+        the error's ``step`` attribute."""
+        st = padoc_mpd_step()
+        code = self._lib.padoc_mpd_prepare_step(self._h, ctypes.byref(cfg), stage.ctypes.data_as(_i32p), stage.size,
+                                                ctypes.byref(st))
+        if code != PADOC_OK:
+            err = PadocError("padoc_mpd_prepare_step", code)
+            err.step = st
+            raise err
+        return st
+
+    def status(self):
+        """(live pages, live streams, free blocks)."""
+        a, b, c = ctypes.c_int32(), ctypes.c_int32(), ctypes.c_int32()
+        _check("padoc_mpd_status", self._lib.padoc_mpd_status(self._h, ctypes.byref(a), ctypes.byref(b), ctypes.byref(c)))
+        return a.value, b.value, c.value
+
+
+def padoc_append_inputs(k_pool, v_pool, k_src, v_src, slots, q_src=None, q_dst=None, src_rows=None, count=None,
+                        stream=None):
+    """K/V rows (src_rows or 0..count-1) of k_src/v_src [rows][Hkv][d] into pool slots (int32 CUDA tensor);
+    with q_src [rows][Hq][d], the same rows' queries into q_dst [count][Hq][d]."""
+    lib = load_library()
+    pool = padoc_kv_pool(_dev(k_pool, "k_pool"), _dev(v_pool, "v_pool"), k_pool.shape[0], k_pool.shape[2],
+                         k_pool.shape[1], k_pool.shape[3], _dtype_code(k_pool))
+    n = slots.shape[0] if count is None else count
+    hq = q_src.shape[1] if q_src is not None else 0
+    st = lib.padoc_append_inputs(ctypes.byref(pool), _dev(k_src, "k_src"), _dev(v_src, "v_src"), _dev(q_src, "q_src"),
+                                 k_src.shape[0], hq, _dev(q_dst, "q_dst"), _dev(src_rows, "src_rows"),
+                                 _dev(slots, "slots"), n, _stream_ptr(stream))
+    _check("padoc_append_inputs", st)
 
 
 # ------------------------------------------------------------------------------------------------
