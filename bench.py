@@ -153,7 +153,7 @@ def bench_decode(args, torch, dev, rank, world):
     scale = 1.0 / math.sqrt(wl.head_dim)
     di = inputs.decode_inputs(wl, 3 + 1000 * rank, pool_slack=1.0)
     plan = DecodePlan(wl.pages, wl.num_q_heads, wl.num_kv_heads, wl.head_dim, dev, tc_ctas=args.tc_ctas,
-                      warp_ctas=args.warp_ctas)
+                      warp_ctas=args.warp_ctas, split_tokens=args.split_tokens)
     S = plan.num_streams
     per_replica = (di.k_pool.numel() + di.v_pool.numel()) * 2
     R = args.replicas if args.replicas > 0 else max(2, math.ceil(4 * l2_bytes(torch) / per_replica) + 1)
@@ -347,7 +347,7 @@ def bench_loop(args, torch, dev, rank, world):
     def admit_all():
         src = inputs.LoopTokenSource(wl.pages)
         loop = MaskedParallelLoop(nb, Hq, Hkv, d, wl.dtype, dev, block_order=order, tc_ctas=args.tc_ctas,
-                                  warp_ctas=args.warp_ctas)
+                                  warp_ctas=args.warp_ctas, split_tokens=args.split_tokens)
         for p in range(len(wl.pages)):
             P, nf, leos, rows = src.admission(p)
             _, new = loop.add_page(P, nf, leos, kd, vd, rows)
@@ -556,6 +556,7 @@ def main():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--tc-ctas", type=int, default=0, help="tensor-core decode CTAs (0: one per SM)")
     ap.add_argument("--warp-ctas", type=int, default=0, help="warp-kernel decode CTAs (0: one per SM)")
+    ap.add_argument("--split-tokens", type=int, default=0, help="decode shared-stream split (0: library default)")
     args = ap.parse_args()
     if args.impl == "reference":
         return run_reference(args)

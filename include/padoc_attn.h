@@ -169,7 +169,7 @@ typedef struct {
     int32_t layout_streams;  /* 1: also decode each page's layout stream (Alg. 1 decodes every live
                                 stream): cutoff P + L over the shared stream, no private rows */
     int32_t split_tokens;    /* shared-stream tokens per split-K partial of the warp kernel (pages with
-                                too few streams for the tensor cores); 0 = library default (512);
+                                too few streams for the tensor cores); 0 = library default (256);
                                 a positive value must be a multiple of block_size; values above
                                 512 act as 512 */
     int32_t tc_ctas;         /* CTAs the tensor-core shared-stream work is balanced over (one range of

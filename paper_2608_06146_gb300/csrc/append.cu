@@ -18,6 +18,12 @@ __global__ void __launch_bounds__(kThreads) append_kernel(const uint4 *__restric
                                                           int32_t block_size, int32_t hkv, int32_t hq, int32_t vec_per_head,
                                                           int *err)
 {
+    // Launched as a programmatic dependent of the previous kernel in the stream (the previous
+    // step's merge, whose step may still be reading the pool and the queries): wait for it before
+    // any global access, then let the decode kernels launch (each of them waits for this grid
+    // before it reads anything).
+    pdl_wait_prerequisite();
+    pdl_launch_dependents();
     const int64_t i = blockIdx.x;
     const int64_t row = src_rows ? (int64_t)src_rows[i] : i;
     const int64_t slot = slots[i];
@@ -67,9 +73,19 @@ extern "C" padoc_status padoc_append_inputs(const padoc_kv_pool *pool, const voi
     if (align & 15) return PADOC_ERR_INVALID_ARGUMENT;
     int *err = padoc_device_error_word();
     if (!err) return PADOC_ERR_CUDA;
-    append_kernel<<<(unsigned)count, kThreads, 0, (cudaStream_t)stream>>>(
-        (const uint4 *)k_src, (const uint4 *)v_src, (const uint4 *)q_src, src_total, (uint4 *)q_dst, src_rows, slots,
-        (uint4 *)pool->k_pool, (uint4 *)pool->v_pool, (int64_t)pool->num_blocks * pool->block_size, pool->block_size,
-        pool->num_kv_heads, q_src ? num_q_heads : 0, (int32_t)(row_bytes / 16), err);
+    cudaLaunchConfig_t lc = {};
+    lc.gridDim = dim3((unsigned)count);
+    lc.blockDim = dim3(kThreads);
+    lc.stream = (cudaStream_t)stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;   // see the kernel's wait
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    lc.attrs = attr;
+    lc.numAttrs = 1;
+    PADOC_CUDA_TRY(cudaLaunchKernelEx(&lc, append_kernel, (const uint4 *)k_src, (const uint4 *)v_src,
+                                      (const uint4 *)q_src, src_total, (uint4 *)q_dst, src_rows, slots,
+                                      (uint4 *)pool->k_pool, (uint4 *)pool->v_pool,
+                                      (int64_t)pool->num_blocks * pool->block_size, pool->block_size,
+                                      pool->num_kv_heads, q_src ? num_q_heads : 0, (int32_t)(row_bytes / 16), err));
     return padoc_launch_status();
 }

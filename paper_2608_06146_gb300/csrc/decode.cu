@@ -67,6 +67,11 @@ decode_warp_kernel(const DecodeParams prm)
 {
     // the merge that follows waits for this whole grid before it reads anything, so it may launch now
     pdl_launch_dependents();
+    // Without a tensor-core grid this grid is a programmatic dependent of whatever kernel precedes
+    // it in the stream (the previous step's merge, which may still read partials, or the kernel
+    // that wrote the queries and the new K/V rows): it waits for that kernel before any global
+    // access, so only its launch overlaps the previous kernel.
+    if (!prm.after_tc) pdl_wait_prerequisite();
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -558,7 +563,7 @@ extern "C" padoc_status padoc_branch_decode_attn(const padoc_kv_pool *pool, cons
         attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
         attr[0].val.programmaticStreamSerializationAllowed = 1;
         lc.attrs = attr;
-        lc.numAttrs = prm.after_tc ? 1 : 0;
+        lc.numAttrs = 1;
         PADOC_CUDA_TRY(cudaLaunchKernelEx(&lc, decode_warp_kernel, prm));
         st = padoc_launch_status();
         if (st != PADOC_OK) return st;

@@ -18,7 +18,10 @@
 #define PADOC_BWD_DKV_K_TILE 128
 
 // Decode split-K: shared-stream tokens per partial result and private tokens per partial result.
-#define PADOC_DEFAULT_SPLIT_TOKENS 512
+// 256 rather than 512: in decoding-loop steps with few streams the warp items on a page's shared
+// stream are the critical path (measured on GB300: 31 -> 21 us per step at 1-2 live streams), and
+// the one-shot serving batch, whose shared streams go to the tensor cores, does not change.
+#define PADOC_DEFAULT_SPLIT_TOKENS 256
 // Longest warp item: a warp keeps one block id per lane, so an item spans at most 32 blocks.
 #define PADOC_WARP_MAX_ITEM_TOKENS 512
 #define PADOC_PRIVATE_SPLIT_TOKENS 256

@@ -93,12 +93,13 @@ class MaskedParallelLoop:
     into the pool, lays out the queries and decodes every stream, all on one CUDA stream."""
 
     def __init__(self, num_blocks: int, num_q_heads: int, num_kv_heads: int, head_dim: int, dtype: torch.dtype,
-                 device, block_order=None, block_size: int = 16, tc_ctas: int = 0, warp_ctas: int = 0):
+                 device, block_order=None, block_size: int = 16, tc_ctas: int = 0, warp_ctas: int = 0,
+                 split_tokens: int = 0):
         self.mpd = pa.Mpd(num_blocks, block_size, block_order)
         self.k_pool = torch.zeros((num_blocks, num_kv_heads, block_size, head_dim), dtype=dtype, device=device)
         self.v_pool = torch.zeros_like(self.k_pool)
-        self.cfg = pa.make_decode_config(num_q_heads, num_kv_heads, head_dim, block_size, False, 0, tc_ctas,
-                                         warp_ctas)
+        self.cfg = pa.make_decode_config(num_q_heads, num_kv_heads, head_dim, block_size, False, split_tokens,
+                                         tc_ctas, warp_ctas)
         self.device, self.dtype = device, dtype
         self.num_q_heads, self.head_dim = num_q_heads, head_dim
         self._stage = [None, None]
