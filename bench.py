@@ -6,7 +6,10 @@ A step is one pass of the hot path over one batch:
              the decode plan's split-K kernel over the paged bf16 cache plus the split-K merge;
   prefill -- the packed ancestor prefill of 8 pages x 4096 tokens (reported in "prefill");
   prefill_bwd -- its gradients dQ, dK, dV for a seeded upstream gradient (reported in
-             "prefill_bwd").
+             "prefill_bwd");
+  loop    -- Algorithm 1 over the serving batch's 32 pages, from admission to the last EOS
+             (reported in "loop": end to end through the engine, and the device time of the same
+             steps replayed from a CUDA graph).
 Headline metric: decode queries/s (one query = one branch's newest token, all 16 query heads).
 
 Timing: W untimed warm-up steps, then K steps between CUDA events on the launching stream, with
