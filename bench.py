@@ -7,6 +7,8 @@ A step is one pass of the hot path over one batch:
   prefill -- the packed ancestor prefill of 8 pages x 4096 tokens (reported in "prefill");
   prefill_bwd -- its gradients dQ, dK, dV for a seeded upstream gradient (reported in
              "prefill_bwd");
+  chunk_prefill -- branch prefill over the paged cache of the serving batch's pages, every branch
+             as one chunk (reported in "branch_prefill");
   loop    -- Algorithm 1 over the serving batch's 32 pages, from admission to the last EOS
              (reported in "loop": end to end through the engine, and the device time of the same
              steps replayed from a CUDA graph).
@@ -325,6 +327,62 @@ def bench_prefill_bwd(args, torch, dev, rank, world):
     return dict(ms=ms, flops=2.5 * prefill_flops(wl), tokens=plan.T, steps=steps)
 
 
+def bench_chunk_prefill(args, torch, dev, rank, world):
+    """Branch prefill over the paged cache of the 32 serving-batch pages: every branch's tokens as one
+    chunk from its branch-initialization token (private rows 0 .. n_k - 1 against the page's shared
+    stream up to P + f_k) and every page's layout stream as one shared-stream chunk; each timed step
+    is one decode-kernel pass over the chunk plan, with L2 flushed between steps."""
+    from paper_2608_06146_gb300 import inputs
+    from paper_2608_06146_gb300 import padoc_attn as pa
+    from paper_2608_06146_gb300.engine import ChunkPrefillPlan
+
+    seed = 3 + 1000 * rank
+    wl = inputs.serving_batch(seed=seed)
+    di = inputs.decode_inputs(wl, seed, pool_slack=1.0)
+    chunks, table, b = [], [], 0
+    pairs = 0
+    for p, pg in enumerate(wl.pages):
+        for f, n in zip(pg.fork_offset, pg.branch_len):
+            chunks.append((p, pg.prefix_len + f, 0, n))
+            table.append(di.stream_table[b])
+            b += 1
+            pairs += n * (pg.prefix_len + f) + n * (n + 1) // 2
+        chunks.append((p, pg.prefix_len, -1, pg.layout_len))
+        table.append(np.full(di.stream_table.shape[1], -1, np.int32))
+        pairs += pg.layout_len * pg.prefix_len + pg.layout_len * (pg.layout_len + 1) // 2
+    page_len = np.array([pg.stream_len for pg in wl.pages], np.int32)
+    plan = ChunkPrefillPlan(page_len, chunks, np.stack(table), wl.num_q_heads, wl.num_kv_heads, wl.head_dim, dev,
+                            tc_ctas=args.tc_ctas, warp_ctas=args.warp_ctas)
+    T = plan.num_tokens
+    q = inputs.randn((T, wl.num_q_heads, wl.head_dim), wl.dtype, seed * 1000 + 98).to(dev)
+    out = torch.empty_like(q)
+    lse = torch.empty((T, wl.num_q_heads), dtype=torch.float32, device=dev)
+    k_pool, v_pool = di.k_pool.to(dev), di.v_pool.to(dev)
+    page_table = torch.from_numpy(di.page_table).to(dev)
+    scale = 1.0 / math.sqrt(wl.head_dim)
+    flush = torch.empty(2 * l2_bytes(torch), dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream()
+    steps = max(3, min(args.steps, 20))
+    for _ in range(max(args.warmup, 3)):
+        plan.run(k_pool, v_pool, page_table, q, scale, out, lse, stream)
+    pa.padoc_check_device_errors(stream)
+    barrier(torch, world)
+    times = []
+    for _ in range(steps):
+        flush.fill_(1)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        plan.run(k_pool, v_pool, page_table, q, scale, out, lse, stream)
+        e1.record(stream)
+        e1.synchronize()
+        times.append(e0.elapsed_time(e1))
+    pa.padoc_check_device_errors(stream)
+    barrier(torch, world)
+    info = plan.info
+    return dict(ms=sum(times) / len(times), flops=4.0 * wl.head_dim * wl.num_q_heads * pairs, tokens=T, steps=steps,
+                chunks=len(chunks), tc_items=int(info.num_tc_items), warp_items=int(info.num_items - info.num_tc_items))
+
+
 def bench_loop(args, torch, dev, rank, world):
     """Algorithm 1 over the serving batch's 32 pages: every page is admitted (its prefix K/V appended
     into the pool, untimed), then the loop runs every layout stream and branch from its first input
@@ -554,7 +612,8 @@ def main():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="padoc", choices=["padoc", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--only", default="all", choices=["all", "decode", "prefill", "prefill_bwd", "loop"])
+    ap.add_argument("--only", default="all", choices=["all", "decode", "prefill", "prefill_bwd", "loop",
+                                                      "chunk_prefill"])
     ap.add_argument("--replicas", type=int, default=0, help="decode input replicas (0: enough to exceed 4x L2)")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--tc-ctas", type=int, default=0, help="tensor-core decode CTAs (0: one per SM)")
@@ -590,8 +649,9 @@ def main():
                               "loop_tokens_per_s_device": lp["tokens"] / lp["dev_s"], **{k: lp[k] for k in
                               ("steps", "tokens", "e2e_s", "dev_s", "eager_s", "bytes", "h2d", "launches")}}))
         return 0
-    if args.only in ("prefill", "prefill_bwd"):
-        fn = bench_prefill if args.only == "prefill" else bench_prefill_bwd
+    if args.only in ("prefill", "prefill_bwd", "chunk_prefill"):
+        fn = {"prefill": bench_prefill, "prefill_bwd": bench_prefill_bwd,
+              "chunk_prefill": bench_chunk_prefill}[args.only]
         p = fn(args, torch, dev, rank, world)
         pms = max_over_ranks(torch, world, p["ms"])
         if rank == 0:
@@ -600,6 +660,7 @@ def main():
     d = bench_decode(args, torch, dev, rank, world)
     p = None if args.only == "decode" else bench_prefill(args, torch, dev, rank, world)
     pb = None if args.only == "decode" else bench_prefill_bwd(args, torch, dev, rank, world)
+    cp = None if args.only == "decode" else bench_chunk_prefill(args, torch, dev, rank, world)
     lp = None if args.only == "decode" else bench_loop(args, torch, dev, rank, world)
 
     peaks, peak_src = load_peaks()
@@ -650,6 +711,19 @@ def main():
                                             "traffic": TRAFFIC_BYTES["prefill_bwd"],
                                             "peak_source": f"{peak_src} bf16_tflops (burst)",
                                             "algorithmic_flops": pb["flops"]}}
+    if cp is not None:
+        cms = max_over_ranks(torch, world, cp["ms"])
+        achieved = cp["flops"] / (cp["ms"] * 1e-3) / 1e12
+        line["branch_prefill"] = {
+            "value": cp["flops"] * world / (cms * 1e-3) / 1e12, "unit": "TFLOP/s", "ms_per_step": cms,
+            "tokens_per_s": cp["tokens"] * world / (cms * 1e-3), "steps": cp["steps"],
+            "workload": "branch prefill over the paged cache of the 32 serving-batch pages: every branch's tokens as "
+                        "one chunk from its branch-initialization token, every layout stream as one shared-stream "
+                        f"chunk ({cp['chunks']} chunks, {cp['tokens']} query tokens), unmasked-entry FLOPs",
+            "l2": "flushed between steps",
+            "roofline": {"bound": "tensor", "achieved": achieved, "peak": peaks["bf16_tflops"], "unit": "TFLOP/s",
+                         "frac": achieved / peaks["bf16_tflops"], "traffic": None,
+                         "peak_source": f"{peak_src} bf16_tflops (burst)", "algorithmic_flops": cp["flops"]}}
     if lp is not None:
         tokens = lp["tokens"] * world
         e2e_s = max_over_ranks(torch, world, lp["e2e_s"])

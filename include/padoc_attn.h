@@ -305,6 +305,50 @@ padoc_status padoc_splitk_combine(const float *part_o, const float *part_lse, in
                                   padoc_stream_t stream);
 
 /* ============================================================================================
+ * Branch prefill over the paged cache: chunks of several query tokens per stream
+ * ========================================================================================== */
+
+/* A chunk of consecutive query tokens of one stream whose K/V rows are already in the paged cache
+ * (App. E.2: a child's branch-initialization input and its residual prefill; Sec. 3.2 visibility).
+ * Chunks are processed by the decode kernels with the chunk's tokens as streams of its page: each
+ * page's shared stream is read once per group of up to 32 tokens of a chunk, and a chunk's own
+ * private rows once per group on the tensor cores (8 or more tokens) instead of once per token. */
+typedef struct {
+    int32_t page;           /* index into the call's pages; chunks grouped page by page, pages ascending */
+    int32_t shared_len;     /* branch chunk: the stream's cutoff on the page's shared stream (P + f_k);
+                               shared-stream chunk: the shared rows before the chunk's first token */
+    int32_t private_start;  /* branch chunk: the stream's private rows before the chunk (its first token
+                               is private row private_start); -1: the chunk's tokens are the shared-stream
+                               rows shared_len .. shared_len + num_tokens - 1 (prefix or layout tokens) */
+    int32_t num_tokens;     /* >= 1 */
+} padoc_prefill_chunk;
+
+/* Plan for a chunked prefill, run by padoc_branch_decode_attn (the same kernels, Q / out / lse rows =
+ * the chunks' tokens in order). Token i of a branch chunk attends to shared rows [0, shared_len) and
+ * private rows [0, private_start + i + 1) (causal inside the chunk); token i of a shared-stream chunk
+ * to shared rows [0, shared_len + i + 1). page_len: (host) int32 [num_pages], each page's shared rows
+ * in the cache; chunks: (host) [num_chunks]. The stream block table passed to the decode call has
+ * one row per token, every token of a branch chunk carrying its stream's private blocks
+ * (padoc_expand_chunk_table writes it from one row per chunk). cfg->layout_streams must be 0.
+ * Errors: INVALID_ARGUMENT (also chunks out of page order, a cutoff past page_len, a shared-stream
+ * chunk reaching past page_len); UNSUPPORTED; CAPACITY. */
+padoc_status padoc_chunk_prefill_plan_size(const int32_t *page_len, int32_t num_pages, const padoc_prefill_chunk *chunks,
+                                           int32_t num_chunks, const padoc_decode_config *cfg, int64_t *plan_ints);
+padoc_status padoc_build_chunk_prefill_plan(const int32_t *page_len, int32_t num_pages,
+                                            const padoc_prefill_chunk *chunks, int32_t num_chunks,
+                                            const padoc_decode_config *cfg, int32_t *plan, int64_t capacity_ints,
+                                            padoc_decode_plan *info);
+
+/* Writes the per-token stream block table of a chunked prefill: chunk_table (host) int32
+ * [num_chunks][chunk_stride] holds each chunk's private block ids (any content for a shared-stream
+ * chunk); row r of stream_table (host) int32 [capacity_rows][stream_stride] gets the row of the
+ * chunk that token r belongs to, padded with -1. Errors: INVALID_ARGUMENT; CAPACITY when
+ * capacity_rows is below the chunks' token count. */
+padoc_status padoc_expand_chunk_table(const padoc_prefill_chunk *chunks, int32_t num_chunks, const int32_t *chunk_table,
+                                      int32_t chunk_stride, int32_t *stream_table, int32_t stream_stride,
+                                      int64_t capacity_rows);
+
+/* ============================================================================================
  * Algorithm 1 (App. E.1): the masked parallel decoding loop over the paged cache
  * ========================================================================================== */
 

@@ -286,7 +286,7 @@ padoc_status padoc_launch_prefill_tc(const void *q, const void *k, const void *v
 // tcgen05 shared-stream decode (decode_tc.cu): the plan's tensor-core items.
 padoc_status padoc_launch_decode_tc(const CUtensorMap *kmap, const CUtensorMap *vmap, const CUtensorMap *qmap, const int32_t *plan,
                                     const padoc_decode_plan *info, const int32_t *page_table, int32_t page_stride,
-                                    int32_t num_blocks, float *part_o, float *part_lse, float scale_log2, int *err,
+                                    const int32_t *stream_table, int32_t stream_stride, int32_t num_blocks, float *part_o, float *part_lse, float scale_log2, int *err,
                                     cudaStream_t stream);
 // tcgen05 prefill backward (prefill_bwd_tc.cu): the dQ pass, which also writes lt / dt (per head
 // [Hq][t_pad]: -lse2 and rowsum(dO * O)), then the dK/dV pass; arguments validated by the caller.

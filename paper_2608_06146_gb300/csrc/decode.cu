@@ -523,6 +523,7 @@ extern "C" padoc_status padoc_branch_decode_attn(const padoc_kv_pool *pool, cons
         if (info->num_tc_items > 0 && !padoc_make_tmap_bf16_4d(&qmap, q, dims, strides, box)) return PADOC_ERR_CUDA;
     }
     padoc_status st = padoc_launch_decode_tc(&kmap, &vmap, &qmap, plan, info, page_block_table, page_table_stride,
+                                             stream_block_table, stream_table_stride,
                                              pool->num_blocks, part_o, part_lse, sl2, err, cs);
     if (st != PADOC_OK) return st;
 

@@ -69,11 +69,11 @@ constexpr size_t kSmemBytes = kTilesBytes + 256 + kXchBytes;
 static_assert(kSmemBytes <= 232448, "shared memory per CTA");
 
 struct TcDecodeParams {
-    const int32_t *shared_len, *slot_ptr, *cta_ptr;
+    const int32_t *shared_len, *private_len, *slot_ptr, *cta_ptr;
     const padoc_item *items;
-    int32_t num_tc_items, num_pages;
-    const int32_t *page_table;
-    int32_t page_stride;
+    int32_t num_tc_items, num_pages, num_streams;
+    const int32_t *page_table, *stream_table;
+    int32_t page_stride, stream_stride;
     int32_t num_blocks, num_kv_heads;
     int32_t pool_rows;           // num_blocks * num_kv_heads * 16: first out-of-range row
     float *part_o, *part_lse;
@@ -95,6 +95,19 @@ __device__ __forceinline__ int piece_tiles(const padoc_item &it)
 }
 
 __device__ __forceinline__ int piece_mtiles(const padoc_item &it) { return it.num_streams > 16 ? 2 : 1; }
+
+// The block-table row an item walks: a page's shared stream (PADOC_ITEM_SHARED_TC, index = page) or
+// the private rows of a chunk of one stream's consecutive query tokens (PADOC_ITEM_PRIVATE_TC, index
+// = the chunk's first stream, whose row every token of the chunk shares). Returns null when the
+// row is out of range.
+__device__ __forceinline__ const int32_t *item_row(const TcDecodeParams &prm, const padoc_item &it, int32_t &stride)
+{
+    const bool priv = it.kind == PADOC_ITEM_PRIVATE_TC;
+    stride = priv ? prm.stream_stride : prm.page_stride;
+    const int32_t rows = priv ? prm.num_streams : prm.num_pages;
+    if (it.index < 0 || it.index >= rows) return nullptr;
+    return (priv ? prm.stream_table : prm.page_table) + (size_t)it.index * stride;
+}
 
 __global__ void __launch_bounds__(kThreads, 1)
 decode_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap,
@@ -126,9 +139,10 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
             const CUtensorMap *map = warp == 8 ? &kmap : &vmap;
             const int j = lane >> 3, b = lane & 7;   // lanes 0-15: tiles 0-1, blocks 0-7
             const int tok0 = it.tok_begin + j * kKT + b * kBlk;
-            if (lane < 16 && it.index >= 0 && it.index < prm.num_pages && tok0 >= 0 && tok0 < it.tok_end &&
-                tok0 / kBlk < prm.page_stride) {
-                const int32_t id = prm.page_table[(size_t)it.index * prm.page_stride + tok0 / kBlk];
+            int32_t stride = 0;
+            const int32_t *trow = item_row(prm, it, stride);
+            if (lane < 16 && trow && tok0 >= 0 && tok0 < it.tok_end && tok0 / kBlk < stride) {
+                const int32_t id = trow[tok0 / kBlk];
                 if (id >= 0 && id < prm.num_blocks) {
                     const int32_t row = (id * prm.num_kv_heads + it.kv_head) * kBlk;
                     tma_prefetch_l2_2d(map, 0, row);
@@ -187,8 +201,12 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
         auto fetch_id = [&](int uu, int jj) {
             const padoc_item &p = prm.items[uu];
             const int tok0 = p.tok_begin + jj * kKT + lane * kBlk;
+            int32_t stride = 0;
+            const int32_t *trow = item_row(prm, p, stride);
             in_next = lane < kKT / kBlk && tok0 < p.tok_end;
-            id_next = in_next ? prm.page_table[(size_t)p.index * prm.page_stride + tok0 / kBlk] : 0;
+            // a table row or block index the plan never produces reads as block -1, which the range
+            // check below reports and skips
+            id_next = !in_next ? 0 : (trow != nullptr && tok0 / kBlk < stride) ? trow[tok0 / kBlk] : -1;
         };
         // a piece's queries: one 4-D box per 64-column panel gathers 16 streams x the 8 heads of the
         // KV head; the next piece's boxes are pulled into L2 meanwhile, so that its reload (which
@@ -365,6 +383,7 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
         // columns before their cutoff.
         const int b0 = row / kGroup, b1 = 16 + row / kGroup;
         int n_tb = 0, n_te = 0, n_nstr = 0, n_first = 0, n_kvh = 0, n_slot = 0, n_cut0 = 0, n_cut1 = 0;
+        bool n_priv = false;
         auto fetch_item = [&](int uu) {
             const padoc_item *p = prm.items + uu;
             n_tb = p->tok_begin;
@@ -373,10 +392,13 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
             n_first = p->first_stream;
             n_kvh = p->kv_head;
             n_slot = p->slot;
+            n_priv = p->kind == PADOC_ITEM_PRIVATE_TC;
         };
+        // a row's cutoff: its stream's shared length, or for a chunk's private rows its private length
         auto fetch_cut = [&]() {
-            n_cut0 = b0 < n_nstr ? min(prm.shared_len[n_first + b0], n_te) : n_tb;
-            n_cut1 = b1 < n_nstr ? min(prm.shared_len[n_first + b1], n_te) : n_tb;
+            const int32_t *cut = n_priv ? prm.private_len : prm.shared_len;
+            n_cut0 = b0 < n_nstr ? min(cut[n_first + b0], n_te) : n_tb;
+            n_cut1 = b1 < n_nstr ? min(cut[n_first + b1], n_te) : n_tb;
         };
         if (u0 < u1) {
             fetch_item(u0);
@@ -540,19 +562,24 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
 
 padoc_status padoc_launch_decode_tc(const CUtensorMap *kmap, const CUtensorMap *vmap, const CUtensorMap *qmap, const int32_t *plan,
                                     const padoc_decode_plan *info, const int32_t *page_table, int32_t page_stride,
+                                    const int32_t *stream_table, int32_t stream_stride,
                                     int32_t num_blocks, float *part_o, float *part_lse, float scale_log2, int *err,
                                     cudaStream_t stream)
 {
     if (info->num_tc_items == 0 || info->tc_ctas == 0) return PADOC_OK;
     TcDecodeParams prm;
     prm.shared_len = plan + info->off_shared_len;
+    prm.private_len = plan + info->off_private_len;
     prm.slot_ptr = plan + info->off_slot_ptr;
     prm.cta_ptr = plan + info->off_cta_ptr;
     prm.items = reinterpret_cast<const padoc_item *>(plan + info->off_items);
     prm.num_tc_items = info->num_tc_items;
     prm.num_pages = info->num_pages;
+    prm.num_streams = info->num_streams;
     prm.page_table = page_table;
     prm.page_stride = page_stride;
+    prm.stream_table = stream_table;
+    prm.stream_stride = stream_stride;
     prm.num_blocks = num_blocks;
     prm.num_kv_heads = info->cfg.num_kv_heads;
     prm.pool_rows = num_blocks * info->cfg.num_kv_heads * kBlk;

@@ -324,6 +324,41 @@ padoc_status streams_of_list(const int32_t *page_len, int32_t num_pages, const p
     return PADOC_OK;
 }
 
+// A chunked prefill: each chunk's tokens become consecutive streams. A branch chunk (private_start
+// >= 0) of n tokens: token i sees the page's shared stream before shared_len and its private rows
+// [0, private_start + i + 1). A shared-stream chunk (private_start = -1): token i is shared row
+// shared_len + i and sees the shared rows up to and including itself.
+padoc_status streams_of_chunks(const int32_t *page_len, int32_t num_pages, const padoc_prefill_chunk *chunks,
+                               int32_t num_chunks, PlanParts &pp)
+{
+    if (num_pages < 0 || num_chunks < 0 || (num_pages > 0 && !page_len) || (num_chunks > 0 && !chunks))
+        return PADOC_ERR_INVALID_ARGUMENT;
+    std::vector<padoc_stream_desc> list;
+    int32_t prev = 0;
+    for (int32_t c = 0; c < num_chunks; ++c) {
+        const padoc_prefill_chunk &k = chunks[c];
+        if (k.page < prev || k.page >= num_pages || k.num_tokens < 1 || k.shared_len < 0 || k.private_start < -1)
+            return PADOC_ERR_INVALID_ARGUMENT;
+        const int32_t pl = page_len[k.page];
+        if (pl < 0 || k.shared_len > pl) return PADOC_ERR_INVALID_ARGUMENT;
+        if (k.private_start < 0 && (int64_t)k.shared_len + k.num_tokens > pl) return PADOC_ERR_INVALID_ARGUMENT;
+        if (k.private_start >= 0 && (int64_t)k.private_start + k.num_tokens >= (1 << 30)) return PADOC_ERR_INVALID_ARGUMENT;
+        if ((int64_t)list.size() + k.num_tokens >= (1 << 30)) return PADOC_ERR_INVALID_ARGUMENT;
+        prev = k.page;
+        pp.chunk_first.push_back((int32_t)list.size());
+        pp.chunk_len.push_back(k.num_tokens);
+        pp.chunk_private.push_back(k.private_start >= 0 ? 1 : 0);
+        for (int32_t i = 0; i < k.num_tokens; ++i) {
+            pp.chunk_of.push_back(c);
+            if (k.private_start >= 0)
+                list.push_back({k.page, k.shared_len, k.private_start + i + 1});
+            else
+                list.push_back({k.page, k.shared_len + i + 1, 0});
+        }
+    }
+    return streams_of_list(page_len, num_pages, list.data(), (int32_t)list.size(), pp);
+}
+
 // The split-K work of a stream list (pp.streams, page_len, page_first_stream, page_num_streams).
 padoc_status build_work(int32_t num_pages, const padoc_decode_config *cfg, PlanParts &pp)
 {
@@ -350,21 +385,48 @@ padoc_status build_work(int32_t num_pages, const padoc_decode_config *cfg, PlanP
     // the group can see. The segments are laid end to end and cut into one contiguous range per CTA
     // (a tile weighs PADOC_TC_WEIGHT_2M for a group of two M-tiles and PADOC_TC_WEIGHT_1M for one);
     // a range becomes the pieces where it overlaps segments.
-    struct Segment { int32_t g, p, first, ns, vis, ntiles, weight; };
+    // A chunked prefill groups streams within a chunk only, and a chunk whose tokens have private
+    // rows and are many enough also gets private segments over those rows (PADOC_ITEM_PRIVATE_TC)
+    // with the same groups, so that every stream of a group receives the same items and therefore
+    // the same partial-slot numbers.
+    struct Segment { int32_t kind, g, p, first, ns, vis, ntiles, weight; };
     std::vector<Segment> segs;
-    for (int32_t g = 0; g < cfg->num_kv_heads; ++g)
+    const bool chunked = !pp.chunk_of.empty();
+    std::vector<uint8_t> priv_tc(chunked ? (size_t)S : 0, 0);
+    auto weight_of = [](int32_t nb) { return nb > PADOC_TC_ITEM_STREAMS / 2 ? PADOC_TC_WEIGHT_2M : PADOC_TC_WEIGHT_1M; };
+    for (int32_t g = 0; g < cfg->num_kv_heads; ++g) {
         for (int32_t p = 0; p < num_pages; ++p) {
             const int32_t f0 = pp.page_first_stream[p], ns = pp.page_num_streams[p];
             if ((int64_t)ns * group < PADOC_TC_MIN_ROWS) continue;
-            for (int32_t r = 0; r < ns; r += PADOC_TC_ITEM_STREAMS) {
-                const int32_t nb = std::min(PADOC_TC_ITEM_STREAMS, ns - r);
+            for (int32_t r = 0; r < ns;) {
+                int32_t nb = std::min(PADOC_TC_ITEM_STREAMS, ns - r);
+                if (chunked)
+                    for (int32_t j = 1; j < nb; ++j)
+                        if (pp.chunk_of[f0 + r + j] != pp.chunk_of[f0 + r] ||
+                            (f0 + r + j - pp.chunk_first[pp.chunk_of[f0 + r + j]]) % PADOC_TC_ITEM_STREAMS == 0) {
+                            nb = j;
+                            break;
+                        }
                 int32_t vis = 0;
                 for (int32_t st = f0 + r; st < f0 + r + nb; ++st) vis = std::max(vis, pp.streams[st].shared_len);
-                if (vis <= 0) continue;
-                segs.push_back({g, p, f0 + r, nb, vis, (vis + PADOC_TC_TILE_TOKENS - 1) / PADOC_TC_TILE_TOKENS,
-                                nb > PADOC_TC_ITEM_STREAMS / 2 ? PADOC_TC_WEIGHT_2M : PADOC_TC_WEIGHT_1M});
+                if (vis > 0)
+                    segs.push_back({PADOC_ITEM_SHARED_TC, g, p, f0 + r, nb, vis,
+                                    (vis + PADOC_TC_TILE_TOKENS - 1) / PADOC_TC_TILE_TOKENS, weight_of(nb)});
+                r += nb;
             }
         }
+        for (size_t c = 0; c < pp.chunk_first.size(); ++c) {
+            const int32_t first = pp.chunk_first[c], len = pp.chunk_len[c];
+            if (!pp.chunk_private[c] || (int64_t)len * group < PADOC_TC_MIN_ROWS) continue;
+            for (int32_t r = 0; r < len; r += PADOC_TC_ITEM_STREAMS) {
+                const int32_t nb = std::min(PADOC_TC_ITEM_STREAMS, len - r);
+                const int32_t vis = pp.streams[first + r + nb - 1].private_len;   // increasing within a chunk
+                for (int32_t st = first + r; st < first + r + nb; ++st) priv_tc[st] = 1;
+                segs.push_back({PADOC_ITEM_PRIVATE_TC, g, first, first + r, nb, vis,
+                                (vis + PADOC_TC_TILE_TOKENS - 1) / PADOC_TC_TILE_TOKENS, weight_of(nb)});
+            }
+        }
+    }
     const int32_t Hkv = cfg->num_kv_heads;
     std::vector<int32_t> cnt((size_t)S * Hkv, 0);   // partial slots handed out per (stream, KV head)
     std::vector<padoc_item> tc_items;
@@ -404,7 +466,7 @@ padoc_status build_work(int32_t num_pages, const padoc_decode_config *cfg, PlanP
                     const int32_t tb = t * PADOC_TC_TILE_TOKENS, te = std::min(sg.vis, t1 * PADOC_TC_TILE_TOKENS);
                     const int32_t slot = cnt[(size_t)sg.first * Hkv + sg.g];
                     for (int32_t st = sg.first; st < sg.first + sg.ns; ++st) ++cnt[(size_t)st * Hkv + sg.g];
-                    tc_items.push_back({PADOC_ITEM_SHARED_TC, sg.p, sg.g, tb, te, sg.first, sg.ns, slot});
+                    tc_items.push_back({sg.kind, sg.p, sg.g, tb, te, sg.first, sg.ns, slot});
                 }
                 t = t1;
             }
@@ -437,6 +499,7 @@ padoc_status build_work(int32_t num_pages, const padoc_decode_config *cfg, PlanP
                                           st, 1, cnt[(size_t)st * Hkv + g]++});
         }
         for (int32_t st = 0; st < S; ++st) {
+            if (chunked && priv_tc[st]) continue;   // the chunk's private rows go to the tensor cores
             const int32_t L = pp.streams[st].private_len;
             for (int32_t tb = 0; tb < L; tb += psplit)
                 warp_items.push_back({PADOC_ITEM_PRIVATE, st, g, tb, std::min(L, tb + psplit), st, 1,
@@ -652,6 +715,16 @@ padoc_status padoc_plan_parts_of_list(const int32_t *page_len, int32_t num_pages
     return st;
 }
 
+padoc_status padoc_plan_parts_of_chunks(const int32_t *page_len, int32_t num_pages, const padoc_prefill_chunk *chunks,
+                                        int32_t num_chunks, const padoc_decode_config *cfg, PlanParts &pp)
+{
+    padoc_status st = check_config(cfg);
+    if (st == PADOC_OK && cfg->layout_streams) st = PADOC_ERR_INVALID_ARGUMENT;
+    if (st == PADOC_OK) st = streams_of_chunks(page_len, num_pages, chunks, num_chunks, pp);
+    if (st == PADOC_OK) st = build_work(num_pages, cfg, pp);
+    return st;
+}
+
 padoc_status padoc_plan_write_blob(const PlanParts &pp, int32_t num_pages, const padoc_decode_config *cfg, int32_t *plan,
                                    int64_t capacity_ints, padoc_decode_plan *info)
 {
@@ -747,5 +820,52 @@ extern "C" padoc_status padoc_decode_workspace_size(const padoc_decode_plan *inf
     if (!info || !bytes) return PADOC_ERR_INVALID_ARGUMENT;
     *bytes = padoc_decode_workspace_bytes(info->num_slots, info->cfg.num_q_heads / info->cfg.num_kv_heads,
                                           info->cfg.head_dim);
+    return PADOC_OK;
+}
+
+extern "C" padoc_status padoc_chunk_prefill_plan_size(const int32_t *page_len, int32_t num_pages,
+                                                      const padoc_prefill_chunk *chunks, int32_t num_chunks,
+                                                      const padoc_decode_config *cfg, int64_t *plan_ints)
+{
+    if (!plan_ints) return PADOC_ERR_INVALID_ARGUMENT;
+    PlanParts pp;
+    padoc_status st = padoc_plan_parts_of_chunks(page_len, num_pages, chunks, num_chunks, cfg, pp);
+    if (st != PADOC_OK) return st;
+    *plan_ints = padoc_plan_blob_ints(pp, num_pages, cfg->num_kv_heads);
+    return PADOC_OK;
+}
+
+extern "C" padoc_status padoc_build_chunk_prefill_plan(const int32_t *page_len, int32_t num_pages,
+                                                       const padoc_prefill_chunk *chunks, int32_t num_chunks,
+                                                       const padoc_decode_config *cfg, int32_t *plan,
+                                                       int64_t capacity_ints, padoc_decode_plan *info)
+{
+    if (!info) return PADOC_ERR_INVALID_ARGUMENT;
+    PlanParts pp;
+    padoc_status st = padoc_plan_parts_of_chunks(page_len, num_pages, chunks, num_chunks, cfg, pp);
+    if (st != PADOC_OK) return st;
+    return padoc_plan_write_blob(pp, num_pages, cfg, plan, capacity_ints, info);
+}
+
+extern "C" padoc_status padoc_expand_chunk_table(const padoc_prefill_chunk *chunks, int32_t num_chunks,
+                                                 const int32_t *chunk_table, int32_t chunk_stride,
+                                                 int32_t *stream_table, int32_t stream_stride, int64_t capacity_rows)
+{
+    if (num_chunks < 0 || (num_chunks > 0 && (!chunks || !chunk_table || !stream_table)) || chunk_stride < 1 ||
+        stream_stride < chunk_stride)
+        return PADOC_ERR_INVALID_ARGUMENT;
+    int64_t rows = 0;
+    for (int32_t c = 0; c < num_chunks; ++c) {
+        if (chunks[c].num_tokens < 1) return PADOC_ERR_INVALID_ARGUMENT;
+        rows += chunks[c].num_tokens;
+    }
+    if (rows > capacity_rows) return PADOC_ERR_CAPACITY;
+    int64_t r = 0;
+    for (int32_t c = 0; c < num_chunks; ++c)
+        for (int32_t i = 0; i < chunks[c].num_tokens; ++i, ++r) {
+            int32_t *dst = stream_table + r * stream_stride;
+            std::memcpy(dst, chunk_table + (int64_t)c * chunk_stride, sizeof(int32_t) * (size_t)chunk_stride);
+            std::fill(dst + chunk_stride, dst + stream_stride, -1);
+        }
     return PADOC_OK;
 }

@@ -21,11 +21,18 @@ struct PlanParts {
     int32_t num_tc_items = 0, tc_ctas = 0, num_warps = 0;
     int32_t max_page_blocks = 0, max_stream_blocks = 0;
     int64_t kv_tokens = 0;
+    // chunked prefill plans only (empty otherwise): the chunk of each stream, and per chunk its
+    // first stream, its token count and whether its tokens have private rows
+    std::vector<int32_t> chunk_of, chunk_first, chunk_len;
+    std::vector<uint8_t> chunk_private;
 };
 
 // The split-K work of an explicit stream list (padoc_build_decode_plan_streams' rules).
 padoc_status padoc_plan_parts_of_list(const int32_t *page_len, int32_t num_pages, const padoc_stream_desc *streams,
                                       int32_t num_streams, const padoc_decode_config *cfg, PlanParts &pp);
+// The streams of a chunked prefill (padoc_build_chunk_prefill_plan's rules) and their work.
+padoc_status padoc_plan_parts_of_chunks(const int32_t *page_len, int32_t num_pages, const padoc_prefill_chunk *chunks,
+                                        int32_t num_chunks, const padoc_decode_config *cfg, PlanParts &pp);
 // int32 words of the plan blob of pp.
 int64_t padoc_plan_blob_ints(const PlanParts &pp, int32_t num_pages, int32_t hkv);
 // Writes the blob and its host summary (CAPACITY when capacity_ints is too small).

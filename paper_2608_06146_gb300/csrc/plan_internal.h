@@ -66,7 +66,7 @@
 #define PADOC_WARP_EARLY_RATE 1.28
 
 #define PADOC_ITEM_INTS 8
-enum { PADOC_ITEM_SHARED = 0, PADOC_ITEM_PRIVATE = 1, PADOC_ITEM_SHARED_TC = 2 };
+enum { PADOC_ITEM_SHARED = 0, PADOC_ITEM_PRIVATE = 1, PADOC_ITEM_SHARED_TC = 2, PADOC_ITEM_PRIVATE_TC = 3 };
 
 // One split-K work item of the decode kernels (8 int32 words in the plan blob). The blob holds
 // the tensor-core items first ([0, num_tc_items)), CTA c of the tensor-core grid owning items
@@ -77,7 +77,11 @@ enum { PADOC_ITEM_SHARED = 0, PADOC_ITEM_PRIVATE = 1, PADOC_ITEM_SHARED_TC = 2 }
 //               streams [first_stream, first_stream + num_streams) (<= 32) of that page, each with
 //               its own column cutoff shared_len (tensor-core kernel);
 //               PADOC_ITEM_SHARED: the same for the one stream first_stream (warp kernel);
-//               PADOC_ITEM_PRIVATE: private tokens [tok_begin, tok_end) of stream `index` (warp kernel).
+//               PADOC_ITEM_PRIVATE: private tokens [tok_begin, tok_end) of stream `index` (warp kernel);
+//               PADOC_ITEM_PRIVATE_TC: private tokens [tok_begin, tok_end) of a chunk of consecutive query
+//               tokens of one stream: streams [first_stream, first_stream + num_streams) (<= 32), each
+//               with its own cutoff private_len, all reading the private block-table row of stream
+//               `index`, the chunk's first token (tensor-core kernel).
 //   kv_head     the KV head; the item covers that head's Hq/Hkv query heads of every stream.
 //   slot        partial-result slot of each covered stream s: slot_ptr[s * Hkv + kv_head] + slot.
 typedef struct {

@@ -82,6 +82,33 @@ class PrefillBwdPlan:
                                       self.workspace, stream)
 
 
+class ChunkPrefillPlan:
+    """Plan (C1) of a chunked prefill over the paged cache, uploaded: chunks of consecutive query
+    tokens per stream (padoc_prefill_chunk rows), run by the decode kernels with the chunks' tokens
+    as streams; ``chunk_table`` holds each chunk's private block ids (one row per chunk)."""
+
+    def __init__(self, page_len, chunks, chunk_table, num_q_heads: int, num_kv_heads: int, head_dim: int, device,
+                 block_size: int = 16, tc_ctas: int = 0, warp_ctas: int = 0):
+        self.cfg = pa.make_decode_config(num_q_heads, num_kv_heads, head_dim, block_size, False, 0, tc_ctas, warp_ctas)
+        self.chunks = np.ascontiguousarray(np.asarray(chunks, np.int32).reshape(-1, 4))
+        plan, self.info = pa.padoc_build_chunk_prefill_plan(page_len, self.chunks, self.cfg)
+        self.plan_dev = torch.from_numpy(plan.copy()).to(device)
+        table = pa.padoc_expand_chunk_table(self.chunks, chunk_table,
+                                            max(int(self.info.max_stream_blocks), np.asarray(chunk_table).shape[1], 1))
+        self.stream_table = torch.from_numpy(table.copy()).to(device)
+        ws = pa.padoc_decode_workspace_size(self.info)
+        self.workspace = torch.empty(max(ws, 256), dtype=torch.uint8, device=device)
+
+    @property
+    def num_tokens(self) -> int:
+        return self.info.num_streams
+
+    def run(self, k_pool, v_pool, page_table, q, scale, out, lse, stream=None):
+        """q / out: [tokens][Hq][d] in the chunks' token order; lse fp32 [tokens][Hq]."""
+        pa.padoc_branch_decode_attn(k_pool, v_pool, self.info, self.plan_dev, page_table, self.stream_table, q, scale,
+                                    out, lse, self.workspace, stream)
+
+
 class MaskedParallelLoop:
     """Algorithm 1 (App. E.1) over the library: the host scheduler (padoc_mpd_*), the append kernel
     and the decode step on one paged KV pool, with device memory from torch.

@@ -53,6 +53,11 @@ class padoc_stream_desc(ctypes.Structure):
     _fields_ = [("page", ctypes.c_int32), ("shared_len", ctypes.c_int32), ("private_len", ctypes.c_int32)]
 
 
+class padoc_prefill_chunk(ctypes.Structure):
+    _fields_ = [("page", ctypes.c_int32), ("shared_len", ctypes.c_int32), ("private_start", ctypes.c_int32),
+                ("num_tokens", ctypes.c_int32)]
+
+
 class padoc_tile_map_dev(ctypes.Structure):
     _fields_ = [("ptr", ctypes.c_void_p), ("idx", ctypes.c_void_p), ("kind", ctypes.c_void_p),
                 ("order", ctypes.c_void_p), ("q_tile", ctypes.c_int32), ("k_tile", ctypes.c_int32)]
@@ -129,6 +134,13 @@ def load_library(path: Optional[str] = None):
         "padoc_build_decode_plan_streams": [_i32p, ctypes.c_int32, ctypes.POINTER(padoc_stream_desc), ctypes.c_int32,
                                             ctypes.POINTER(padoc_decode_config), _i32p, ctypes.c_int64,
                                             ctypes.POINTER(padoc_decode_plan)],
+        "padoc_chunk_prefill_plan_size": [_i32p, ctypes.c_int32, ctypes.POINTER(padoc_prefill_chunk), ctypes.c_int32,
+                                          ctypes.POINTER(padoc_decode_config), _i64p],
+        "padoc_build_chunk_prefill_plan": [_i32p, ctypes.c_int32, ctypes.POINTER(padoc_prefill_chunk), ctypes.c_int32,
+                                           ctypes.POINTER(padoc_decode_config), _i32p, ctypes.c_int64,
+                                           ctypes.POINTER(padoc_decode_plan)],
+        "padoc_expand_chunk_table": [ctypes.POINTER(padoc_prefill_chunk), ctypes.c_int32, _i32p, ctypes.c_int32, _i32p,
+                                     ctypes.c_int32, ctypes.c_int64],
         "padoc_mpd_create": [ctypes.c_int32, ctypes.c_int32, _i32p, ctypes.POINTER(_vp)],
         "padoc_mpd_destroy": [_vp],
         "padoc_mpd_add_page": [_vp, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32, _i32p, _i32p, _i32p],
@@ -168,7 +180,9 @@ def exported_symbols() -> Sequence[str]:
                         "padoc_splitk_combine", "padoc_ancestor_prefill_attn", "padoc_build_key_tile_map",
                         "padoc_prefill_bwd_tile_shapes", "padoc_prefill_bwd_workspace_size",
                         "padoc_ancestor_prefill_bwd", "padoc_decode_plan_size_streams",
-                        "padoc_build_decode_plan_streams", "padoc_mpd_create", "padoc_mpd_destroy",
+                        "padoc_build_decode_plan_streams", "padoc_chunk_prefill_plan_size",
+                        "padoc_build_chunk_prefill_plan", "padoc_expand_chunk_table",
+                        "padoc_mpd_create", "padoc_mpd_destroy",
                         "padoc_mpd_add_page", "padoc_mpd_begin_step", "padoc_mpd_step_shape",
                         "padoc_mpd_step_tables", "padoc_mpd_end_step", "padoc_mpd_status", "padoc_mpd_prepare_step",
                         "padoc_append_inputs",
@@ -392,6 +406,47 @@ def padoc_build_decode_plan_streams(page_len, streams, cfg: padoc_decode_config,
            lib.padoc_build_decode_plan_streams(pl.ctypes.data_as(_i32p), pl.size, sp, sa.size, ctypes.byref(cfg),
                                                out.ctypes.data_as(_i32p), n, ctypes.byref(info)))
     return out[:n], info
+
+
+_CHUNK_DTYPE = np.dtype([("page", np.int32), ("shared_len", np.int32), ("private_start", np.int32),
+                         ("num_tokens", np.int32)])
+
+
+def _chunk_arr(chunks):
+    a = np.ascontiguousarray(np.asarray(chunks, np.int32).reshape(-1, 4)).view(_CHUNK_DTYPE).reshape(-1)
+    return a, ctypes.cast(a.ctypes.data, ctypes.POINTER(padoc_prefill_chunk))
+
+
+def padoc_build_chunk_prefill_plan(page_len, chunks, cfg: padoc_decode_config):
+    """Plan of a chunked prefill: page_len int32 [pages]; chunks [C] of (page, shared_len, private_start,
+    num_tokens). Returns (plan blob, padoc_decode_plan)."""
+    lib = load_library()
+    pl = np.ascontiguousarray(page_len, np.int32)
+    ca, cp = _chunk_arr(chunks)
+    n = ctypes.c_int64()
+    _check("padoc_chunk_prefill_plan_size",
+           lib.padoc_chunk_prefill_plan_size(pl.ctypes.data_as(_i32p), pl.size, cp, ca.size, ctypes.byref(cfg),
+                                             ctypes.byref(n)))
+    out = np.zeros(max(n.value, 1), np.int32)
+    info = padoc_decode_plan()
+    _check("padoc_build_chunk_prefill_plan",
+           lib.padoc_build_chunk_prefill_plan(pl.ctypes.data_as(_i32p), pl.size, cp, ca.size, ctypes.byref(cfg),
+                                              out.ctypes.data_as(_i32p), n.value, ctypes.byref(info)))
+    return out[:n.value], info
+
+
+def padoc_expand_chunk_table(chunks, chunk_table, stream_stride=None):
+    """Per-token stream block table [tokens][stride] from one row per chunk ([chunks][chunk_stride])."""
+    lib = load_library()
+    ca, cp = _chunk_arr(chunks)
+    ct = np.ascontiguousarray(chunk_table, np.int32)
+    stride = ct.shape[1] if stream_stride is None else stream_stride
+    rows = int(ca["num_tokens"].sum())
+    out = np.zeros((max(rows, 1), stride), np.int32)
+    _check("padoc_expand_chunk_table",
+           lib.padoc_expand_chunk_table(cp, ca.size, ct.ctypes.data_as(_i32p), ct.shape[1], out.ctypes.data_as(_i32p),
+                                        stride, rows))
+    return out[:rows]
 
 
 def padoc_decode_workspace_size(info: padoc_decode_plan) -> int:
