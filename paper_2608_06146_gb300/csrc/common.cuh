@@ -115,6 +115,13 @@ __device__ __forceinline__ uint64_t l2_evict_first_policy()
     return p;
 }
 
+__device__ __forceinline__ uint64_t l2_evict_normal_policy()
+{
+    uint64_t p;
+    asm volatile("createpolicy.fractional.L2::evict_normal.b64 %0, 1.0;" : "=l"(p));
+    return p;
+}
+
 // tma_load_2d with an L2 cache policy.
 __device__ __forceinline__ void tma_load_2d_hint(uint32_t dst, const CUtensorMap *map, int32_t x, int32_t y, uint32_t bar,
                                                  uint64_t policy)

@@ -102,7 +102,7 @@ __device__ __forceinline__ int piece_mtiles(const padoc_item &it) { return it.nu
 // row is out of range.
 __device__ __forceinline__ const int32_t *item_row(const TcDecodeParams &prm, const padoc_item &it, int32_t &stride)
 {
-    const bool priv = it.kind == PADOC_ITEM_PRIVATE_TC;
+    const bool priv = PADOC_ITEM_KIND(it.kind) == PADOC_ITEM_PRIVATE_TC;
     stride = priv ? prm.stream_stride : prm.page_stride;
     const int32_t rows = priv ? prm.num_streams : prm.num_pages;
     if (it.index < 0 || it.index >= rows) return nullptr;
@@ -195,7 +195,8 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
         const CUtensorMap *map = is_k ? &kmap : &vmap;
         uint8_t *ring = is_k ? sk : sv;
         const int b_full = is_k ? B_KFULL : B_VFULL, b_empty = is_k ? B_KEMPTY : B_VEMPTY;
-        const uint64_t kv_policy = l2_evict_first_policy();   // K/V tiles are read once per call
+        // K/V tiles read by one group only are evict-first; see PADOC_ITEM_REREAD
+        const uint64_t once_policy = l2_evict_first_policy(), shared_policy = l2_evict_normal_policy();
         int32_t id_next = 0;
         bool in_next = false;
         auto fetch_id = [&](int uu, int jj) {
@@ -259,6 +260,7 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
                 __syncwarp();
                 if (lane < kKT / kBlk) {
                     const uint32_t dst = smem_u32(ring + s * kTile) + (uint32_t)lane * (kBlk * 128);
+                    const uint64_t kv_policy = (it.kind & PADOC_ITEM_REREAD) ? shared_policy : once_policy;
                     tma_load_2d_hint(dst, map, 0, row, bar(b_full + s), kv_policy);
                     tma_load_2d_hint(dst + kPanel, map, 64, row, bar(b_full + s), kv_policy);
                 }
@@ -392,7 +394,7 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
             n_first = p->first_stream;
             n_kvh = p->kv_head;
             n_slot = p->slot;
-            n_priv = p->kind == PADOC_ITEM_PRIVATE_TC;
+            n_priv = PADOC_ITEM_KIND(p->kind) == PADOC_ITEM_PRIVATE_TC;
         };
         // a row's cutoff: its stream's shared length, or for a chunk's private rows its private length
         auto fetch_cut = [&]() {

@@ -410,7 +410,7 @@ padoc_status build_work(int32_t num_pages, const padoc_decode_config *cfg, PlanP
                 int32_t vis = 0;
                 for (int32_t st = f0 + r; st < f0 + r + nb; ++st) vis = std::max(vis, pp.streams[st].shared_len);
                 if (vis > 0)
-                    segs.push_back({PADOC_ITEM_SHARED_TC, g, p, f0 + r, nb, vis,
+                    segs.push_back({PADOC_ITEM_SHARED_TC | (nb < ns ? PADOC_ITEM_REREAD : 0), g, p, f0 + r, nb, vis,
                                     (vis + PADOC_TC_TILE_TOKENS - 1) / PADOC_TC_TILE_TOKENS, weight_of(nb)});
                 r += nb;
             }
@@ -422,7 +422,7 @@ padoc_status build_work(int32_t num_pages, const padoc_decode_config *cfg, PlanP
                 const int32_t nb = std::min(PADOC_TC_ITEM_STREAMS, len - r);
                 const int32_t vis = pp.streams[first + r + nb - 1].private_len;   // increasing within a chunk
                 for (int32_t st = first + r; st < first + r + nb; ++st) priv_tc[st] = 1;
-                segs.push_back({PADOC_ITEM_PRIVATE_TC, g, first, first + r, nb, vis,
+                segs.push_back({PADOC_ITEM_PRIVATE_TC | (nb < len ? PADOC_ITEM_REREAD : 0), g, first, first + r, nb, vis,
                                 (vis + PADOC_TC_TILE_TOKENS - 1) / PADOC_TC_TILE_TOKENS, weight_of(nb)});
             }
         }

@@ -67,6 +67,12 @@
 
 #define PADOC_ITEM_INTS 8
 enum { PADOC_ITEM_SHARED = 0, PADOC_ITEM_PRIVATE = 1, PADOC_ITEM_SHARED_TC = 2, PADOC_ITEM_PRIVATE_TC = 3 };
+// Flag added to the kind of a tensor-core item whose rows other groups read too (a page with more
+// than 32 streams, a chunk of more than 32 tokens): its tiles are loaded with the normal L2 policy
+// so that the groups running at the same time share them; rows read by one group only are loaded
+// evict-first, which keeps the split-K partials in L2 for the merge.
+#define PADOC_ITEM_REREAD 16
+#define PADOC_ITEM_KIND(k) ((k) & 15)
 
 // One split-K work item of the decode kernels (8 int32 words in the plan blob). The blob holds
 // the tensor-core items first ([0, num_tc_items)), CTA c of the tensor-core grid owning items

@@ -60,12 +60,16 @@ def test_chunk_plan_covers_every_visible_row_once(seed, tc_ctas):
     slot_ptr = plan[info.off_slot_ptr:info.off_slot_ptr + S * Hkv + 1]
     items = plan[info.off_items:info.off_items + 8 * info.num_items].reshape(-1, 8)
     ntc = info.num_tc_items
-    assert np.isin(items[:ntc, 0], [2, 3]).all() and np.isin(items[ntc:, 0], [0, 1]).all()
+    assert np.isin(items[:ntc, 0] & 15, [2, 3]).all() and np.isin(items[ntc:, 0], [0, 1]).all()
     first_of = {c: int(np.nonzero(ch == c)[0][0]) for c in range(len(chunks))}
     cov_sh = {(s, g): np.zeros(sh[s], np.int32) for s in range(S) for g in range(Hkv)}
     cov_pv = {(s, g): np.zeros(pl[s], np.int32) for s in range(S) for g in range(Hkv)}
     slots = {(s, g): [] for s in range(S) for g in range(Hkv)}
     for kind, idx, g, tb, te, fs, ns, slot in items:
+        reread = bool(kind & 16)
+        kind &= 15
+        if kind == 3:   # reread exactly when the chunk has more than one group
+            assert reread == (chunks[ch[fs]][3] > 32)
         if kind in (2, 3):
             assert 1 <= ns <= 32 and tb % 128 == 0 and te > tb
             assert len(set(ch[fs:fs + ns])) == 1, "a tensor-core group never crosses a chunk"

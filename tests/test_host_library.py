@@ -182,9 +182,14 @@ def test_decode_plan_covers_every_visible_token_once(wl_name, layout, tc_ctas, w
     cov_pv = {(s, g): np.zeros(pl[s], np.int32) for s in range(S) for g in range(Hkv)}
     slots_used = {(s, g): [] for s in range(S) for g in range(Hkv)}
     ntc = info.num_tc_items
-    assert all(items[:ntc, 0] == 2) and not any(items[ntc:, 0] == 2)
+    kinds = items[:, 0] & 15
+    assert all(kinds[:ntc] == 2) and not any(kinds[ntc:] == 2)
+    # the reread flag marks exactly the pieces of pages with more than one group of 32 streams
+    assert np.all((items[:ntc, 0] & 16 != 0) == (np.bincount(sp, minlength=len(wl.pages))[items[:ntc, 1]] > 32))
+    assert not np.any(items[ntc:, 0] & 16)
     page_streams = np.bincount(sp, minlength=len(wl.pages))
     for kind, idx, g, tb, te, fs, ns, slot in items:
+        kind &= 15
         assert tb % 16 == 0
         if kind == 2:      # tensor-core piece: whole 128-token tiles of up to 32 streams of a page
             assert 1 <= ns <= 32 and te > tb and page_streams[idx] * 8 >= 64 and tb % 128 == 0
