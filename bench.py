@@ -44,8 +44,9 @@ METRIC = "ancestor-attn decode queries/s, % of HBM roofline; packed prefill TFLO
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 # dram__bytes_read.sum + dram__bytes_write.sum per launch from the ncu captures summarised under
 # profiles/ (None until a capture of the current kernel exists). Decode: one step = the three
-# kernels' captures added up (profiles/decode_*_serving_batch.md), cold caches.
-TRAFFIC_BYTES = {"decode": 227_310_000, "prefill": 260_600_000,   # prefill: profiles/prefill_tc_packed_32k.md
+# kernels' counters added up (profiles/decode_traffic_serving_batch.md), cold caches.
+TRAFFIC_BYTES = {"decode": 224_800_000,    # profiles/decode_traffic_serving_batch.md
+                 "prefill": 260_600_000,   # profiles/prefill_tc_packed_32k.md
                  "prefill_bwd": 1_459_570_000}  # both passes: profiles/prefill_bwd_packed_32k.md
 
 

@@ -451,6 +451,22 @@ typedef struct {
 padoc_status padoc_mpd_prepare_step(padoc_mpd *mpd, const padoc_decode_config *cfg, int32_t *stage,
                                     int64_t capacity_words, padoc_mpd_step *step);
 
+/* Runs a step prepared by padoc_mpd_prepare_step, all on `stream`, with no host synchronization:
+ * copies stage[0, step->upload_words) (host; pinned memory makes the copy asynchronous, and the
+ * stage must stay unchanged until the copy has run) to dev_ints ((device) int32
+ * [dev_capacity_words], 256-byte aligned), appends every input (padoc_append_inputs with the step's
+ * slots and the source rows the caller wrote at stage[step->off_rows]; k_src / v_src
+ * [src_total][Hkv][d], q_src [src_total][Hq][d], q_dst (device) [C][Hq][d] receives the step's
+ * queries) and decodes every stream (padoc_branch_decode_attn: out [C][Hq][d], lse fp32 [C][Hq],
+ * workspace >= padoc_decode_workspace_size(&step->plan) bytes). Nothing is launched for C = 0.
+ * Errors: INVALID_ARGUMENT (also dev_capacity_words < upload_words), UNSUPPORTED,
+ * WORKSPACE_TOO_SMALL, CUDA. */
+padoc_status padoc_mpd_launch_step(const padoc_mpd_step *step, const int32_t *stage, int32_t *dev_ints,
+                                   int64_t dev_capacity_words, const padoc_kv_pool *pool, const void *k_src,
+                                   const void *v_src, const void *q_src, int64_t src_total, void *q_dst, float scale,
+                                   void *out, float *lse, void *workspace, size_t workspace_bytes,
+                                   padoc_stream_t stream);
+
 /* Live pages, live streams and free pool blocks. */
 padoc_status padoc_mpd_status(const padoc_mpd *mpd, int32_t *live_pages, int32_t *live_streams, int32_t *free_blocks);
 

@@ -410,7 +410,7 @@ padoc_status build_work(int32_t num_pages, const padoc_decode_config *cfg, PlanP
                 int32_t vis = 0;
                 for (int32_t st = f0 + r; st < f0 + r + nb; ++st) vis = std::max(vis, pp.streams[st].shared_len);
                 if (vis > 0)
-                    segs.push_back({PADOC_ITEM_SHARED_TC | (nb < ns ? PADOC_ITEM_REREAD : 0), g, p, f0 + r, nb, vis,
+                    segs.push_back({PADOC_ITEM_SHARED_TC | (chunked && nb < ns ? PADOC_ITEM_REREAD : 0), g, p, f0 + r, nb, vis,
                                     (vis + PADOC_TC_TILE_TOKENS - 1) / PADOC_TC_TILE_TOKENS, weight_of(nb)});
                 r += nb;
             }

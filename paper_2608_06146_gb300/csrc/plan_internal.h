@@ -67,10 +67,11 @@
 
 #define PADOC_ITEM_INTS 8
 enum { PADOC_ITEM_SHARED = 0, PADOC_ITEM_PRIVATE = 1, PADOC_ITEM_SHARED_TC = 2, PADOC_ITEM_PRIVATE_TC = 3 };
-// Flag added to the kind of a tensor-core item whose rows other groups read too (a page with more
-// than 32 streams, a chunk of more than 32 tokens): its tiles are loaded with the normal L2 policy
-// so that the groups running at the same time share them; rows read by one group only are loaded
-// evict-first, which keeps the split-K partials in L2 for the merge.
+// Flag added to the kind of a tensor-core item of a chunked prefill whose rows other groups read
+// too (a page with more than 32 chunk tokens, a chunk of more than 32 tokens): its tiles are loaded
+// with the normal L2 policy so that the groups running at the same time share them. Decode plans
+// never set it: their tiles are loaded evict-first, which keeps the split-K partials in L2 for the
+// merge (measured: flagging the decode step's pages of more than 32 streams was no faster).
 #define PADOC_ITEM_REREAD 16
 #define PADOC_ITEM_KIND(k) ((k) & 15)
 

@@ -125,6 +125,7 @@ class MaskedParallelLoop:
         self.mpd = pa.Mpd(num_blocks, block_size, block_order)
         self.k_pool = torch.zeros((num_blocks, num_kv_heads, block_size, head_dim), dtype=dtype, device=device)
         self.v_pool = torch.zeros_like(self.k_pool)
+        self._pool = pa.make_kv_pool(self.k_pool, self.v_pool)
         self.cfg = pa.make_decode_config(num_q_heads, num_kv_heads, head_dim, block_size, False, split_tokens,
                                          tc_ctas, warp_ctas)
         self.device, self.dtype = device, dtype
@@ -178,8 +179,9 @@ class MaskedParallelLoop:
     def step(self, k_src, v_src, q_src, rows_of, scale: float, out=None, lse=None, stream=None):
         """One iteration: every live stream appends its next input (rows_of(stream ids) gives the rows
         of k_src / v_src / q_src that hold them) and is decoded. Returns (stream ids, out [C][Hq][d],
-        lse fp32 [C][Hq]); the caller ends the step with end_step. The host work is one library call
-        (padoc_mpd_prepare_step) into a pinned staging buffer and one copy of it to the device."""
+        lse fp32 [C][Hq]); the caller ends the step with end_step. The host work is two library calls:
+        padoc_mpd_prepare_step into a pinned staging buffer, and padoc_mpd_launch_step, which copies it
+        to the device and launches the append and the decode."""
         stream = stream or torch.cuda.current_stream()
         b = self._turn & 1
         self._turn += 1
@@ -202,38 +204,30 @@ class MaskedParallelLoop:
         n = int(st.upload_words)
         if self._ints.numel() < n:
             self._ints = torch.empty(max(n, 2 * self._ints.numel()), dtype=torch.int32, device=self.device)
-        with torch.cuda.stream(stream):
-            self._ints[:n].copy_(self._stage[b][:n], non_blocking=True)
-        self._stage_free[b].record(stream)
         self.h2d_bytes = 4 * n
         info = st.plan
         self.last_info = info
         self.last_step = st
         self.last_stage = host
         if C == 0:
+            self._stage_free[b].record(stream)
             empty = torch.empty((0, self.num_q_heads), dtype=torch.float32, device=self.device)
             return ids, torch.empty((0, self.num_q_heads, self.head_dim), dtype=self.dtype, device=self.device), empty
-        d = self._ints
-        plan_d = d[st.off_plan:st.off_plan + info.plan_ints]
-        pt_d = d[st.off_page_table:st.off_page_table + st.num_pages * st.page_stride].view(st.num_pages, st.page_stride)
-        st_d = d[st.off_stream_table:st.off_stream_table + C * st.stream_stride].view(C, st.stream_stride)
-        slots_d = d[st.off_slots:st.off_slots + C]
-        rows_d = d[st.off_rows:st.off_rows + C]
         if self.q_step.shape[0] < C:
             self.q_step = torch.empty((max(C, 2 * self.q_step.shape[0]), self.num_q_heads, self.head_dim),
                                       dtype=self.dtype, device=self.device)
-        q_step = self.q_step[:C]
-        pa.padoc_append_inputs(self.k_pool, self.v_pool, k_src, v_src, slots_d, q_src=q_src, q_dst=q_step,
-                               src_rows=rows_d, count=C, stream=stream)
-        ws = pa.padoc_decode_workspace_size(info)
+        group = self.cfg.num_q_heads // self.cfg.num_kv_heads   # padoc_decode_workspace_size, computed here
+        ws = int(info.num_slots) * group * (self.head_dim + 1) * 4 + 512
         if self.workspace.numel() < ws:
             self.workspace = torch.empty(max(ws, 2 * self.workspace.numel()), dtype=torch.uint8, device=self.device)
         if out is None:
             out = torch.empty((C, self.num_q_heads, self.head_dim), dtype=self.dtype, device=self.device)
         if lse is None:
             lse = torch.empty((C, self.num_q_heads), dtype=torch.float32, device=self.device)
-        pa.padoc_branch_decode_attn(self.k_pool, self.v_pool, info, plan_d, pt_d, st_d, q_step, scale, out, lse,
-                                    self.workspace, stream)
+        # one library call: the stage's copy to the device, the append and the decode
+        pa.padoc_mpd_launch_step(st, self._stage[b], self._ints, self._pool, k_src, v_src, q_src, self.q_step, scale,
+                                 out, lse, self.workspace, stream)
+        self._stage_free[b].record(stream)
         return ids, out, lse
 
     def end_step(self, num_forks=None, eos=None, num_streams=None):

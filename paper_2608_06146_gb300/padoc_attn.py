@@ -155,6 +155,9 @@ def load_library(path: Optional[str] = None):
                                    ctypes.POINTER(padoc_mpd_step)],
         "padoc_append_inputs": [ctypes.POINTER(padoc_kv_pool), _vp, _vp, _vp, ctypes.c_int64, ctypes.c_int32, _vp, _vp,
                                 _vp, ctypes.c_int32, _vp],
+        "padoc_mpd_launch_step": [ctypes.POINTER(padoc_mpd_step), _vp, _vp, ctypes.c_int64,
+                                  ctypes.POINTER(padoc_kv_pool), _vp, _vp, _vp, ctypes.c_int64, _vp, ctypes.c_float, _vp,
+                                  _vp, _vp, ctypes.c_size_t, _vp],
         "padoc_selftest_tcgen05": [_vp, _vp, _vp, _vp, _vp, _vp, _vp],
         "padoc_check_device_errors": [_vp],
         "padoc_last_device_error": [_i32p, _i32p],
@@ -185,6 +188,7 @@ def exported_symbols() -> Sequence[str]:
                         "padoc_mpd_create", "padoc_mpd_destroy",
                         "padoc_mpd_add_page", "padoc_mpd_begin_step", "padoc_mpd_step_shape",
                         "padoc_mpd_step_tables", "padoc_mpd_end_step", "padoc_mpd_status", "padoc_mpd_prepare_step",
+                        "padoc_mpd_launch_step",
                         "padoc_append_inputs",
                         "padoc_selftest_tcgen05",
                         "padoc_check_device_errors",
@@ -610,6 +614,25 @@ class Mpd:
         a, b, c = ctypes.c_int32(), ctypes.c_int32(), ctypes.c_int32()
         _check("padoc_mpd_status", self._lib.padoc_mpd_status(self._h, ctypes.byref(a), ctypes.byref(b), ctypes.byref(c)))
         return a.value, b.value, c.value
+
+
+def padoc_mpd_launch_step(step: padoc_mpd_step, stage, dev_ints, pool: padoc_kv_pool, k_src, v_src, q_src, q_dst,
+                          scale, out, lse, workspace, stream=None):
+    """stage: pinned int32 CPU tensor holding the prepared step; dev_ints: int32 CUDA tensor; pool: a
+    padoc_kv_pool (make_kv_pool); other tensors as in padoc_append_inputs / padoc_branch_decode_attn."""
+    lib = load_library()
+    st = lib.padoc_mpd_launch_step(ctypes.byref(step), stage.data_ptr(), _dev(dev_ints, "dev_ints"), dev_ints.numel(),
+                                   ctypes.byref(pool), _dev(k_src, "k_src"), _dev(v_src, "v_src"), _dev(q_src, "q_src"),
+                                   k_src.shape[0], _dev(q_dst, "q_dst"), float(scale), _dev(out, "out"),
+                                   _dev(lse, "lse"), _dev(workspace, "workspace"),
+                                   workspace.numel() * workspace.element_size(), _stream_ptr(stream))
+    _check("padoc_mpd_launch_step", st)
+
+
+def make_kv_pool(k_pool, v_pool) -> padoc_kv_pool:
+    """padoc_kv_pool over pool tensors [num_blocks][Hkv][16][d] (the caller keeps them alive)."""
+    return padoc_kv_pool(_dev(k_pool, "k_pool"), _dev(v_pool, "v_pool"), k_pool.shape[0], k_pool.shape[2],
+                         k_pool.shape[1], k_pool.shape[3], _dtype_code(k_pool))
 
 
 def padoc_append_inputs(k_pool, v_pool, k_src, v_src, slots, q_src=None, q_dst=None, src_rows=None, count=None,

@@ -70,6 +70,8 @@ def test_chunk_plan_covers_every_visible_row_once(seed, tc_ctas):
         kind &= 15
         if kind == 3:   # reread exactly when the chunk has more than one group
             assert reread == (chunks[ch[fs]][3] > 32)
+        if kind == 2:   # reread exactly when the page's chunk tokens form more than one group
+            assert reread == (np.count_nonzero(sp == idx) > ns)
         if kind in (2, 3):
             assert 1 <= ns <= 32 and tb % 128 == 0 and te > tb
             assert len(set(ch[fs:fs + ns])) == 1, "a tensor-core group never crosses a chunk"

@@ -184,9 +184,7 @@ def test_decode_plan_covers_every_visible_token_once(wl_name, layout, tc_ctas, w
     ntc = info.num_tc_items
     kinds = items[:, 0] & 15
     assert all(kinds[:ntc] == 2) and not any(kinds[ntc:] == 2)
-    # the reread flag marks exactly the pieces of pages with more than one group of 32 streams
-    assert np.all((items[:ntc, 0] & 16 != 0) == (np.bincount(sp, minlength=len(wl.pages))[items[:ntc, 1]] > 32))
-    assert not np.any(items[ntc:, 0] & 16)
+    assert not np.any(items[:, 0] & 16), "decode plans load every tile evict-first"
     page_streams = np.bincount(sp, minlength=len(wl.pages))
     for kind, idx, g, tb, te, fs, ns, slot in items:
         kind &= 15
