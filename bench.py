@@ -219,11 +219,15 @@ def bench_decode(args, torch, dev, rank, world):
     blob_np = [b.numpy() for b in blob_pinned]
     blob_free = [torch.cuda.Event(), torch.cuda.Event()]
 
+    # the page records stay in one native array (a serving loop updates its lengths in place); the
+    # planner runs every step
+    page_array = pa.PageArray(wl.pages)
+
     def e2e_step(i):
         r = i % R
         b = i & 1
         blob_free[b].synchronize()
-        blob, info = pa.padoc_build_decode_plan(wl.pages, cfg, out=blob_np[b])
+        blob, info = pa.padoc_build_decode_plan(page_array, cfg, out=blob_np[b])
         blob_t = blob_pinned[b][: blob.size]
         plan_dev[: blob.size].copy_(blob_t, non_blocking=True)
         blob_free[b].record(stream)

@@ -274,6 +274,12 @@ padoc_status streams_of_pages(const padoc_page *pages, int32_t num_pages, const 
                               PlanParts &pp)
 {
     if (num_pages < 0 || (num_pages > 0 && !pages)) return PADOC_ERR_INVALID_ARGUMENT;
+    int64_t ns = 0;
+    for (int32_t p = 0; p < num_pages; ++p) ns += std::max(pages[p].num_branches, 0) + (cfg->layout_streams ? 1 : 0);
+    pp.streams.reserve((size_t)ns);
+    pp.page_len.reserve((size_t)num_pages);
+    pp.page_first_stream.reserve((size_t)num_pages);
+    pp.page_num_streams.reserve((size_t)num_pages);
     for (int32_t p = 0; p < num_pages; ++p) {
         const padoc_page &pg = pages[p];
         if (pg.prefix_len < 0 || pg.layout_len < 0 || pg.num_branches < 0) return PADOC_ERR_INVALID_ARGUMENT;
@@ -430,6 +436,7 @@ padoc_status build_work(int32_t num_pages, const padoc_decode_config *cfg, PlanP
     const int32_t Hkv = cfg->num_kv_heads;
     std::vector<int32_t> cnt((size_t)S * Hkv, 0);   // partial slots handed out per (stream, KV head)
     std::vector<padoc_item> tc_items;
+    tc_items.reserve(segs.size() * 2 + 64);
     // CTA loads count every piece's own cost too (its epilogue, and the query reload before it):
     // the smallest bound T for which a greedy walk along the sequences needs at most `want` CTAs
     // is found by bisection, then the walk is made once more to emit the pieces.
@@ -489,6 +496,16 @@ padoc_status build_work(int32_t num_pages, const padoc_decode_config *cfg, PlanP
 
     // ---- warp work: shared streams of sparse pages (per stream) and every private history ------
     std::vector<padoc_item> warp_items;
+    {
+        int64_t n = 0;   // exact count, so the list is allocated once
+        for (int32_t p = 0; p < num_pages; ++p) {
+            const int32_t f0 = pp.page_first_stream[p], ns = pp.page_num_streams[p];
+            if ((int64_t)ns * group >= PADOC_TC_MIN_ROWS) continue;
+            for (int32_t st = f0; st < f0 + ns; ++st) n += (pp.streams[st].shared_len + split - 1) / split;
+        }
+        for (int32_t st = 0; st < S; ++st) n += (pp.streams[st].private_len + psplit - 1) / psplit + 1;
+        warp_items.reserve((size_t)(n * Hkv));
+    }
     for (int32_t g = 0; g < Hkv; ++g) {
         for (int32_t p = 0; p < num_pages; ++p) {
             const int32_t f0 = pp.page_first_stream[p], ns = pp.page_num_streams[p];

@@ -207,7 +207,12 @@ _PAGE_DTYPE = np.dtype({"names": ["prefix_len", "layout_len", "num_branches", "f
 
 class _Pages:
     """C array of padoc_page built with vectorized numpy (one pass over the pages); keeps the
-    concatenated fork-offset and branch-length arrays alive."""
+    concatenated fork-offset and branch-length arrays alive.
+
+    Public as PageArray: a caller that plans every step (a decode loop whose branches grow by one
+    token per step) keeps one and updates its arrays in place (``lens``: every page's branch lengths
+    back to back; ``forks``: their fork offsets; ``rec["prefix_len"]`` / ``rec["layout_len"]``) instead
+    of marshalling Python page objects again; the page and branch counts are fixed."""
 
     def __init__(self, pages):
         import itertools
@@ -231,6 +236,13 @@ class _Pages:
         self.rec = rec
         self.arr = ctypes.cast(rec.ctypes.data, ctypes.POINTER(padoc_page))
         self.n = n
+
+
+PageArray = _Pages
+
+
+def _as_pages(pages) -> _Pages:
+    return pages if isinstance(pages, _Pages) else _Pages(pages)
 
 
 def _stream_ptr(stream):
@@ -262,14 +274,14 @@ def _dev(t, name):
 # ------------------------------------------------------------------------------------------------
 
 def padoc_packed_size(pages) -> int:
-    lib, P = load_library(), _Pages(pages)
+    lib, P = load_library(), _as_pages(pages)
     t = ctypes.c_int64()
     _check("padoc_packed_size", lib.padoc_packed_size(P.arr, P.n, ctypes.byref(t)))
     return t.value
 
 
 def padoc_build_query_spans(pages) -> np.ndarray:
-    lib, P = load_library(), _Pages(pages)
+    lib, P = load_library(), _as_pages(pages)
     T = padoc_packed_size(pages)
     out = np.zeros((max(T, 1), 4), np.int32)
     _check("padoc_build_query_spans", lib.padoc_build_query_spans(P.arr, P.n, out.ctypes.data_as(_i32p), T))
@@ -284,7 +296,7 @@ def padoc_prefill_tile_shape(dtype: int, head_dim: int):
 
 
 def padoc_tile_map_size(pages, q_tile: int, k_tile: int):
-    lib, P = load_library(), _Pages(pages)
+    lib, P = load_library(), _as_pages(pages)
     a, b = ctypes.c_int64(), ctypes.c_int64()
     _check("padoc_tile_map_size", lib.padoc_tile_map_size(P.arr, P.n, q_tile, k_tile, ctypes.byref(a), ctypes.byref(b)))
     return a.value, b.value
@@ -292,7 +304,7 @@ def padoc_tile_map_size(pages, q_tile: int, k_tile: int):
 
 def padoc_build_tile_map(pages, q_tile: int, k_tile: int):
     """Returns (row_ptr int32 [q_tiles+1], k_tiles int32 [nnz], kinds int8 [nnz])."""
-    lib, P = load_library(), _Pages(pages)
+    lib, P = load_library(), _as_pages(pages)
     nqt, nnz = padoc_tile_map_size(pages, q_tile, k_tile)
     row_ptr = np.zeros(nqt + 1, np.int32)
     kt = np.zeros(max(nnz, 1), np.int32)
@@ -304,7 +316,7 @@ def padoc_build_tile_map(pages, q_tile: int, k_tile: int):
 
 def padoc_build_key_tile_map(pages, q_tile: int, k_tile: int):
     """Returns (col_ptr int32 [k_tiles+1], q_tiles int32 [nnz], kinds int8 [nnz], k_order int32 [k_tiles])."""
-    lib, P = load_library(), _Pages(pages)
+    lib, P = load_library(), _as_pages(pages)
     T = padoc_packed_size(pages)
     _, nnz = padoc_tile_map_size(pages, q_tile, k_tile)
     nkt = -(-T // k_tile)
@@ -340,7 +352,7 @@ def make_decode_config(num_q_heads, num_kv_heads, head_dim, block_size=16, layou
 
 
 def padoc_decode_plan_size(pages, cfg: padoc_decode_config) -> int:
-    lib, P = load_library(), _Pages(pages)
+    lib, P = load_library(), _as_pages(pages)
     n = ctypes.c_int64()
     _check("padoc_decode_plan_size", lib.padoc_decode_plan_size(P.arr, P.n, ctypes.byref(cfg), ctypes.byref(n)))
     return n.value
@@ -349,7 +361,7 @@ def padoc_decode_plan_size(pages, cfg: padoc_decode_config) -> int:
 def padoc_build_decode_plan(pages, cfg: padoc_decode_config, out=None):
     """Returns (plan blob int32 numpy array, padoc_decode_plan host summary). ``out`` may be an int32
     numpy array (e.g. a view of pinned host memory) that receives the blob; a view of it is returned."""
-    lib, P = load_library(), _Pages(pages)
+    lib, P = load_library(), _as_pages(pages)
     info = padoc_decode_plan()
     if out is not None:   # one planner pass when the caller's buffer is large enough
         st = lib.padoc_build_decode_plan(P.arr, P.n, ctypes.byref(cfg), out.ctypes.data_as(_i32p), out.size,

@@ -264,3 +264,20 @@ def test_decode_plan_rejects_bad_config():
     with pytest.raises(pa.PadocError) as e:
         pa.padoc_build_decode_plan(wl.pages, pa.make_decode_config(16, 2, 128, block_size=32))
     assert e.value.status == 2
+
+
+def test_page_array_plans_like_page_objects():
+    """A persistent PageArray, updated in place between steps (every branch one token longer), plans
+    exactly like page objects marshalled afresh."""
+    wl = inputs.serving_batch(seed=3)
+    cfg = pa.make_decode_config(16, 2, 128, tc_ctas=96, warp_ctas=152)
+    arr = pa.PageArray(wl.pages)
+    a, ia = pa.padoc_build_decode_plan(arr, cfg)
+    b, ib = pa.padoc_build_decode_plan(wl.pages, cfg)
+    np.testing.assert_array_equal(a, b)
+    arr.lens += 1
+    grown = [PageSpec(pg.prefix_len, pg.layout_len, list(pg.fork_offset), [n + 1 for n in pg.branch_len])
+             for pg in wl.pages]
+    a, _ = pa.padoc_build_decode_plan(arr, cfg)
+    b, _ = pa.padoc_build_decode_plan(grown, cfg)
+    np.testing.assert_array_equal(a, b)
