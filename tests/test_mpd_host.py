@@ -285,3 +285,24 @@ def test_prepare_step_equals_granular_calls(seed):
         np.testing.assert_array_equal(a.end_step(nf, eos), new)
         src.forked(ids, nf, new)
     assert a.status() == b.status() == (0, 0, nb)
+
+
+def test_launch_step_validates_before_any_device_work(lib):
+    """padoc_mpd_launch_step rejects a device buffer too small for the stage or not 256-byte aligned,
+    and a null stage or pool, before it touches the device (these checks need no GPU)."""
+    import ctypes
+    m = pa.Mpd(64)
+    m.add_page(40, 2)
+    cfg = pa.make_decode_config(16, 2, 128)
+    stage = np.zeros(1 << 16, np.int32)
+    st = m.prepare_step(cfg, stage)
+    assert st.num_streams == 3 and st.upload_words > 0
+    pool = pa.padoc_kv_pool(256, 512, 64, 16, 2, 128, pa.PADOC_DTYPE_BF16)   # never dereferenced here
+    sp = stage.ctypes.data
+    call = lambda stage_p, dev, cap, pool_p: lib.padoc_mpd_launch_step(
+        ctypes.byref(st), stage_p, dev, cap, pool_p, 1024, 1024, 1024, 10, 1024, 0.1, 1024, 1024, 1024, 1 << 20, None)
+    assert call(sp, 4096, st.upload_words - 1, ctypes.byref(pool)) == 1   # too small
+    assert call(sp, 4096 + 4, st.upload_words, ctypes.byref(pool)) == 1   # not 256-byte aligned
+    assert call(None, 4096, st.upload_words, ctypes.byref(pool)) == 1     # no stage
+    assert call(sp, 4096, st.upload_words, None) == 1                     # no pool
+    m.end_step(np.zeros(3, np.int32), np.zeros(3, np.uint8))
