@@ -150,16 +150,18 @@ def l2_bytes(torch):
         return 129 * 1024 * 1024
 
 
-def bench_decode(args, torch, dev, rank, world):
+def bench_decode(args, torch, dev, rank, world, layout_streams=False):
+    """The serving-batch decode step (with ``layout_streams``, every page's layout stream is decoded
+    too, as Algorithm 1 decodes every live stream)."""
     from paper_2608_06146_gb300 import inputs
     from paper_2608_06146_gb300 import padoc_attn as pa
     from paper_2608_06146_gb300.engine import DecodePlan
 
     wl = inputs.serving_batch(seed=3 + 1000 * rank)
     scale = 1.0 / math.sqrt(wl.head_dim)
-    di = inputs.decode_inputs(wl, 3 + 1000 * rank, pool_slack=1.0)
+    di = inputs.decode_inputs(wl, 3 + 1000 * rank, pool_slack=1.0, layout_streams=layout_streams)
     plan = DecodePlan(wl.pages, wl.num_q_heads, wl.num_kv_heads, wl.head_dim, dev, tc_ctas=args.tc_ctas,
-                      warp_ctas=args.warp_ctas, split_tokens=args.split_tokens)
+                      warp_ctas=args.warp_ctas, split_tokens=args.split_tokens, layout_streams=layout_streams)
     S = plan.num_streams
     per_replica = (di.k_pool.numel() + di.v_pool.numel()) * 2
     R = args.replicas if args.replicas > 0 else max(2, math.ceil(4 * l2_bytes(torch) / per_replica) + 1)
@@ -192,13 +194,13 @@ def bench_decode(args, torch, dev, rank, world):
     pa.padoc_check_device_errors(stream)
     ms = ev0.elapsed_time(ev1) / args.steps
 
-    sp, sh, pl = inputs.decode_streams(wl)
+    sp, sh, pl = inputs.decode_streams(wl, layout_streams)
     nbytes = decode_bytes(wl, sp, sh, pl)
     info = plan.info
     launches = (1 if info.num_tc_items > 0 else 0) + (1 if info.num_warps > 0 else 0) + 1   # + the merge
     res = dict(ms=ms, streams=S, bytes=nbytes, launches=launches, clocks=clk.summary(), replicas=R,
                pages=len(wl.pages), e2e_ms=None, h2d=0, d2h=0)
-    if args.no_e2e:
+    if args.no_e2e or layout_streams:
         return res
 
     # end to end through the public API: host C1 plan, host->device copies of the step's inputs
@@ -258,12 +260,14 @@ def bench_decode(args, torch, dev, rank, world):
     return res
 
 
-def bench_prefill(args, torch, dev, rank, world):
+def bench_prefill(args, torch, dev, rank, world, shuffle=False):
+    """The packed prefill of 8 pages x 4096 tokens (with ``shuffle``, each page's branches permuted
+    so that the fork offsets are not monotone in the branch index)."""
     from paper_2608_06146_gb300 import inputs
     from paper_2608_06146_gb300 import padoc_attn as pa
     from paper_2608_06146_gb300.engine import PrefillPlan
 
-    wl = inputs.packed_prefill(seed=4 + 1000 * rank)
+    wl = inputs.packed_prefill(seed=4 + 1000 * rank, shuffle_branches=shuffle)
     q, k, v = inputs.packed_qkv(wl, 4 + 1000 * rank)
     plan = PrefillPlan(wl.pages, wl.dtype, wl.head_dim, dev)
     q, k, v = q.to(dev), k.to(dev), v.to(dev)
@@ -618,7 +622,7 @@ def main():
     ap.add_argument("--impl", default="padoc", choices=["padoc", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--only", default="all", choices=["all", "decode", "prefill", "prefill_bwd", "loop",
-                                                      "chunk_prefill"])
+                                                      "chunk_prefill", "variants"])
     ap.add_argument("--replicas", type=int, default=0, help="decode input replicas (0: enough to exceed 4x L2)")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--tc-ctas", type=int, default=0, help="tensor-core decode CTAs (0: one per SM)")
@@ -647,6 +651,13 @@ def main():
 
     from paper_2608_06146_gb300 import build as pbuild
     pbuild.build()
+    if args.only == "variants":   # the two extra report lines alone
+        a = bench_decode(args, torch, dev, rank, world, layout_streams=True)
+        b = bench_prefill(args, torch, dev, rank, world, shuffle=True)
+        if rank == 0:
+            print(json.dumps({"decode_with_layout_streams_us": a["ms"] * 1e3, "streams": a["streams"],
+                              "prefill_shuffled_ms": b["ms"], "prefill_shuffled_tflops": b["flops"] / (b["ms"] * 1e-3) / 1e12}))
+        return 0
     if args.only == "loop":
         lp = bench_loop(args, torch, dev, rank, world)
         if rank == 0:
@@ -665,6 +676,14 @@ def main():
     d = bench_decode(args, torch, dev, rank, world)
     p = None if args.only == "decode" else bench_prefill(args, torch, dev, rank, world)
     pb = None if args.only == "decode" else bench_prefill_bwd(args, torch, dev, rank, world)
+    def variant(fn, **kw):   # an extra report line: a failure is recorded, the headline stands
+        try:
+            return fn(args, torch, dev, rank, world, **kw)
+        except Exception as e:  # noqa: BLE001
+            return {"error": f"{type(e).__name__}: {e}"[:300]}
+
+    dl = None if args.only == "decode" else variant(bench_decode, layout_streams=True)
+    ps = None if args.only == "decode" else variant(bench_prefill, shuffle=True)
     cp = None if args.only == "decode" else bench_chunk_prefill(args, torch, dev, rank, world)
     lp = None if args.only == "decode" else bench_loop(args, torch, dev, rank, world)
 
@@ -716,6 +735,29 @@ def main():
                                             "traffic": TRAFFIC_BYTES["prefill_bwd"],
                                             "peak_source": f"{peak_src} bf16_tflops (burst)",
                                             "algorithmic_flops": pb["flops"]}}
+    if dl is not None:
+        if "error" in dl:
+            line["decode_with_layout_streams"] = dl
+        else:
+            dms = max_over_ranks(torch, world, dl["ms"])
+            ach = dl["bytes"] / (dl["ms"] * 1e-3) / 1e9
+            line["decode_with_layout_streams"] = {
+                "value": dl["streams"] * world / (dms * 1e-3), "unit": "queries/s", "ms_per_step": dms,
+                "streams_per_gpu": dl["streams"],
+                "workload": "the serving-batch decode step with every page's layout stream decoded too "
+                            "(branches + layout streams; the headline counts branches only)",
+                "roofline": {"bound": "hbm", "achieved": ach, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                             "frac": ach / peaks["hbm_gbs"], "traffic": None, "algorithmic_bytes": dl["bytes"]}}
+    if ps is not None and p is not None:
+        if "error" in ps:
+            line["prefill"]["shuffled_branches"] = ps
+        else:
+            sms = max_over_ranks(torch, world, ps["ms"])
+            line["prefill"]["shuffled_branches"] = {
+                "value": ps["flops"] * world / (sms * 1e-3) / 1e12, "unit": "TFLOP/s", "ms_per_step": sms,
+                "workload": "the same packed prefill with each page's branches permuted (fork offsets not "
+                            "monotone in the branch index)",
+                "frac": ps["flops"] / (ps["ms"] * 1e-3) / 1e12 / peaks["bf16_tflops"]}
     if cp is not None:
         cms = max_over_ranks(torch, world, cp["ms"])
         achieved = cp["flops"] / (cp["ms"] * 1e-3) / 1e12
