@@ -484,7 +484,13 @@ padoc_status build_work(int32_t num_pages, const padoc_decode_config *cfg, PlanP
     int32_t ctas = 0;
     if (!segs.empty()) {
         const int64_t want = cfg->tc_ctas > 0 ? cfg->tc_ctas : choose_tc_ctas(pp, cfg, total_w, max_piece);
-        int64_t lo = max_w + max_piece, hi = total_w + max_w;   // walk(hi) needs one CTA
+        // Every CTA's load stays within T (T >= max_w + max_piece), so T below total_w / want needs
+        // more than `want` CTAs: that is a lower bound. A CTA is closed only once less than a piece
+        // and a tile fit, and cutting adds at most one piece per CTA, so T = total_w / (want - 1) +
+        // 2 max_piece + max_w fits in `want`; it is checked, with the one-CTA bound behind it.
+        int64_t lo = std::max<int64_t>(max_w + max_piece, (total_w + want - 1) / want);
+        int64_t hi = (want > 1 ? (total_w + want - 2) / (want - 1) : total_w) + 2 * max_piece + max_w + 1;
+        if (hi < lo || walk(hi, false) > want) hi = std::max(lo, total_w + max_w);   // walk(total_w + max_w) needs one CTA
         while (lo < hi) {
             const int64_t mid = lo + (hi - lo) / 2;
             if (walk(mid, false) <= want) hi = mid; else lo = mid + 1;
