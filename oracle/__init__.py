@@ -10,7 +10,9 @@ App. C.1 packed statement; App. E.1 additive-bias softmax and Algorithm 1); the 
 the readings taken where the paper is silent. Parity of all functions is pinned by
 tests/test_oracle_pins.py against closed forms, torch's SDPA, a simulator of Algorithm 1's mask
 recurrence and hand-derived fixtures; the backward against central differences of the forward,
-torch autograd through the per-branch gather, and closed forms.
+torch autograd through the per-branch gather, and closed forms. The FP8 (E4M3) KV-cache
+definitions (encode, decode, per-block quantization) are pinned against torch's float8_e4m3fn on
+every code and on every tie between neighbouring codes, and by the format's error bound.
 """
 from __future__ import annotations
 
@@ -69,6 +71,12 @@ def _load():
                                                _f32p, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32,
                                                ctypes.c_double, ctypes.c_int64, _i64p, ctypes.c_int64,
                                                _i64p, _f64p, _f64p, _f64p]
+            lib.oracle_e4m3_encode.argtypes = [_f32p, ctypes.c_int64, _u8p]
+            lib.oracle_e4m3_decode.argtypes = [_u8p, ctypes.c_int64, _f64p]
+            lib.oracle_quantize_kv_blocks.argtypes = [_f32p, ctypes.c_int64, ctypes.c_int32, ctypes.c_int32,
+                                                      ctypes.c_int32, _u8p, _f32p]
+            lib.oracle_dequantize_kv_blocks.argtypes = [_u8p, _f32p, ctypes.c_int64, ctypes.c_int32, ctypes.c_int32,
+                                                        ctypes.c_int32, _f64p]
             _lib = lib
     return _lib
 
@@ -218,3 +226,43 @@ def prefill_bwd(pages, q, k, v, dout, scale, q_rows=None, k_rows=None):
                                    len(qs), _ptr(guard(qs), _i64p), len(ks), _ptr(guard(ks), _i64p),
                                    _ptr(guard(dq), _f64p), _ptr(guard(dk), _f64p), _ptr(guard(dv), _f64p))
     return dq, dk, dv
+
+
+# --------------------------------------------------------------------------------------------
+# FP8 (E4M3) KV cache: see padoc_oracle.c, "FP8 (E4M3) KV cache"
+# --------------------------------------------------------------------------------------------
+
+def e4m3_encode(x) -> np.ndarray:
+    """E4M3 codes (uint8) of fp32 values: nearest, ties to even, saturating at 448, NaN -> 0x7F."""
+    a = np.ascontiguousarray(np.asarray(x, np.float32))
+    out = np.zeros(a.shape, np.uint8)
+    _load().oracle_e4m3_encode(_ptr(a, _f32p), a.size, _ptr(out, _u8p))
+    return out
+
+
+def e4m3_decode(codes) -> np.ndarray:
+    """fp64 values of E4M3 codes (NaN for 0x7F / 0xFF)."""
+    c = np.ascontiguousarray(np.asarray(codes, np.uint8))
+    out = np.zeros(c.shape, np.float64)
+    _load().oracle_e4m3_decode(_ptr(c, _u8p), c.size, _ptr(out, _f64p))
+    return out
+
+
+def quantize_kv_blocks(pool):
+    """pool fp32 [num_blocks][Hkv][block][d] -> (codes uint8 same shape, scales fp32 [num_blocks][Hkv])."""
+    x = _f32(pool)
+    nb, hkv, bs, d = x.shape
+    codes = np.zeros(x.shape, np.uint8)
+    scales = np.zeros((nb, hkv), np.float32)
+    _load().oracle_quantize_kv_blocks(_ptr(x, _f32p), nb, hkv, bs, d, _ptr(codes, _u8p), _ptr(scales, _f32p))
+    return codes, scales
+
+
+def dequantize_kv_blocks(codes, scales) -> np.ndarray:
+    """code_value * scale per (block, head), exact in fp64."""
+    c = np.ascontiguousarray(np.asarray(codes, np.uint8))
+    sc = np.ascontiguousarray(np.asarray(scales, np.float32))
+    nb, hkv, bs, d = c.shape
+    out = np.zeros(c.shape, np.float64)
+    _load().oracle_dequantize_kv_blocks(_ptr(c, _u8p), _ptr(sc, _f32p), nb, hkv, bs, d, _ptr(out, _f64p))
+    return out

@@ -617,3 +617,84 @@ void oracle_prefill_bwd(const int32_t *pln, int32_t num_pages, const int32_t *fo
     free(touched); free(lse_all); free(D_all);
     page_index_free(&ix);
 }
+
+/* ============================================================================================
+ * FP8 (E4M3) KV cache. The paper serves a bf16 cache; this is the definition the FP8 cache
+ * variant of the decode step is checked against: K and V stored as E4M3 codes with one fp32 scale
+ * per (block, KV head), and attention over the dequantized values code_value * scale.
+ *
+ * E4M3 (the OCP 8-bit floating point format): sign bit, 4 exponent bits with bias 7, 3 mantissa
+ * bits; exponent field 0 is subnormal (value m * 2^-9); no infinities; S.1111.111 is NaN, so the
+ * largest finite magnitude is 1.75 * 2^8 = 448.
+ * ========================================================================================== */
+
+double oracle_e4m3_value(uint8_t code)
+{
+    const int s = code >> 7, e = (code >> 3) & 15, m = code & 7;
+    if (e == 15 && m == 7) return NAN;
+    const double v = e == 0 ? ldexp((double)m, -9) : ldexp((double)(8 + m), e - 10);
+    return s ? -v : v;
+}
+
+/* Nearest E4M3 code to x, ties to the even code (the one whose mantissa's last bit is 0),
+ * magnitudes of 448 and above saturated to 448, NaN to the NaN code 0x7F. The search runs over
+ * every finite positive code, which is slow and plainly correct. */
+uint8_t oracle_e4m3_encode_one(double x)
+{
+    if (isnan(x)) return 0x7F;
+    const int s = signbit(x) ? 1 : 0;
+    const double a = fabs(x);
+    int best = 0;
+    if (a >= 448.0) {
+        best = 0x7E;
+    } else {
+        double best_err = INFINITY;
+        for (int c = 0; c <= 0x7E; ++c) {
+            const double err = fabs(oracle_e4m3_value((uint8_t)c) - a);
+            if (err < best_err || (err == best_err && (c & 1) == 0)) {
+                best_err = err;
+                best = c;
+            }
+        }
+    }
+    return (uint8_t)(best | (s << 7));
+}
+
+void oracle_e4m3_encode(const float *x, int64_t n, uint8_t *codes)
+{
+    for (int64_t i = 0; i < n; ++i) codes[i] = oracle_e4m3_encode_one((double)x[i]);
+}
+
+void oracle_e4m3_decode(const uint8_t *codes, int64_t n, double *x)
+{
+    for (int64_t i = 0; i < n; ++i) x[i] = oracle_e4m3_value(codes[i]);
+}
+
+/* Quantizes a pool [num_blocks][hkv][bs][d] of fp32 K or V: per (block, head) the scale is
+ * amax / 448 in fp32 (1 for an all-zero block) and each element's code is the E4M3 code of
+ * x / scale, the division taken in fp32, the precision a kernel that quantizes on write uses. */
+void oracle_quantize_kv_blocks(const float *x, int64_t num_blocks, int32_t hkv, int32_t bs, int32_t d, uint8_t *codes,
+                               float *scales)
+{
+    const int64_t per = (int64_t)bs * d;
+    for (int64_t u = 0; u < num_blocks * hkv; ++u) {
+        const float *src = x + u * per;
+        float amax = 0.0f;
+        for (int64_t i = 0; i < per; ++i) amax = fmaxf(amax, fabsf(src[i]));
+        const float scale = amax > 0.0f ? amax / 448.0f : 1.0f;
+        scales[u] = scale;
+        for (int64_t i = 0; i < per; ++i) {
+            const float y = src[i] / scale;
+            codes[u * per + i] = oracle_e4m3_encode_one((double)y);
+        }
+    }
+}
+
+/* The dequantized pool: code_value * scale, exact in fp64. */
+void oracle_dequantize_kv_blocks(const uint8_t *codes, const float *scales, int64_t num_blocks, int32_t hkv,
+                                 int32_t bs, int32_t d, double *x)
+{
+    const int64_t per = (int64_t)bs * d;
+    for (int64_t u = 0; u < num_blocks * hkv; ++u)
+        for (int64_t i = 0; i < per; ++i) x[u * per + i] = oracle_e4m3_value(codes[u * per + i]) * (double)scales[u];
+}

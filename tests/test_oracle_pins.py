@@ -519,3 +519,72 @@ def test_prefill_bwd_row_selection_matches_full():
     np.testing.assert_array_equal(part[0], full[0][qr])
     np.testing.assert_array_equal(part[1], full[1][kr])
     np.testing.assert_array_equal(part[2], full[2][kr])
+
+
+# ------------------------------------------------------------------------------------------------
+# FP8 (E4M3) KV cache
+# ------------------------------------------------------------------------------------------------
+
+def test_e4m3_decode_matches_torch_on_every_code():
+    """All 256 codes against torch's float8_e4m3fn (a library decoder of the same format)."""
+    codes = np.arange(256, dtype=np.uint8)
+    ref = torch.from_numpy(codes.copy()).view(torch.float8_e4m3fn).to(torch.float64).numpy()
+    got = oracle.e4m3_decode(codes)
+    assert np.array_equal(np.isnan(got), np.isnan(ref))
+    ok = ~np.isnan(ref)
+    np.testing.assert_array_equal(got[ok], ref[ok])
+    np.testing.assert_array_equal(np.signbit(got[ok]), np.signbit(ref[ok]))
+    assert np.nanmax(got) == 448.0 and got[1] == 2.0 ** -9
+
+
+def test_e4m3_encode_matches_torch_rounding_in_range():
+    """Nearest-even encoding against torch's conversion wherever torch's result is finite (|x| < 464):
+    random values over the whole range, exact midpoints between neighbouring codes (ties), the
+    subnormal range and signed zeros."""
+    rng = np.random.default_rng(0)
+    vals = oracle.e4m3_decode(np.arange(0, 0x7E, dtype=np.uint8))
+    mids = (vals[:-1] + vals[1:]) / 2
+    x = np.concatenate([rng.uniform(-463, 463, 20000), np.exp(rng.uniform(-14, 6, 20000)) * rng.choice([-1, 1], 20000),
+                        mids, -mids, vals, [0.0, -0.0, 2.0 ** -10, 3 * 2.0 ** -10, 447.9, 463.9]]).astype(np.float32)
+    got = oracle.e4m3_encode(x)
+    ref = torch.from_numpy(x).to(torch.float8_e4m3fn).view(torch.uint8).numpy()
+    bad = np.nonzero(got != ref)[0]
+    assert bad.size == 0, f"{bad.size} codes differ, first x = {x[bad[0]]!r}: {got[bad[0]]:#x} vs {ref[bad[0]]:#x}"
+
+
+def test_e4m3_encode_saturates_and_keeps_nan():
+    x = np.array([464.0, 480.0, 1e6, np.inf, -464.0, -1e9, -np.inf, np.nan], np.float32)
+    got = oracle.e4m3_encode(x)
+    np.testing.assert_array_equal(got[:4], 0x7E)
+    np.testing.assert_array_equal(got[4:7], 0xFE)
+    assert np.isnan(oracle.e4m3_decode(got[7:]))[0]
+
+
+def test_quantize_kv_blocks_scale_bound_and_exact_values():
+    """Per (block, head): the largest magnitude maps to 448; every element is within half a code step
+    of its value (relative 2^-4 for normal codes, 2^-10 * scale below the normal range); a block
+    whose values are already codes times a power-of-two scale comes back exactly; a zero block
+    keeps scale 1 and codes 0."""
+    rng = np.random.default_rng(1)
+    x = rng.standard_normal((6, 2, 16, 128)).astype(np.float32) * rng.uniform(0.01, 50, (6, 2, 1, 1)).astype(np.float32)
+    x[5, 1] = 0.0
+    codes, scales = oracle.quantize_kv_blocks(x)
+    deq = oracle.dequantize_kv_blocks(codes, scales)
+    for b in range(6):
+        for h in range(2):
+            blk, s = x[b, h].astype(np.float64), float(scales[b, h])
+            if b == 5 and h == 1:
+                assert s == 1.0 and not codes[b, h].any()
+                continue
+            assert np.isclose(s, np.float32(np.abs(x[b, h]).max() / np.float32(448.0)), rtol=0, atol=0)
+            assert np.abs(oracle.e4m3_decode(codes[b, h])).max() == 448.0
+            y = np.abs(blk) / s
+            bound = np.where(y >= 2.0 ** -6, 2.0 ** -4 * y, 2.0 ** -10) * s * (1 + 1e-6)
+            assert np.all(np.abs(deq[b, h] - blk) <= bound + 1e-30)
+    # exact round trip: values that are codes times a power-of-two scale with the largest code present
+    c = rng.integers(0, 0x7E, (1, 1, 16, 128)).astype(np.uint8)
+    c[0, 0, 0, 0] = 0x7E
+    exact = (oracle.e4m3_decode(c) * 2.0 ** -3).astype(np.float32)
+    codes2, scales2 = oracle.quantize_kv_blocks(exact)
+    assert scales2[0, 0] == np.float32(2.0 ** -3)
+    np.testing.assert_array_equal(oracle.dequantize_kv_blocks(codes2, scales2), exact.astype(np.float64))
