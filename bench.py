@@ -684,8 +684,8 @@ def main():
 
     dl = None if args.only == "decode" else variant(bench_decode, layout_streams=True)
     ps = None if args.only == "decode" else variant(bench_prefill, shuffle=True)
-    cp = None if args.only == "decode" else bench_chunk_prefill(args, torch, dev, rank, world)
-    lp = None if args.only == "decode" else bench_loop(args, torch, dev, rank, world)
+    cp = None if args.only == "decode" else variant(bench_chunk_prefill)
+    lp = None if args.only == "decode" else variant(bench_loop)
 
     peaks, peak_src = load_peaks()
     ms = max_over_ranks(torch, world, d["ms"])
@@ -758,7 +758,9 @@ def main():
                 "workload": "the same packed prefill with each page's branches permuted (fork offsets not "
                             "monotone in the branch index)",
                 "frac": ps["flops"] / (ps["ms"] * 1e-3) / 1e12 / peaks["bf16_tflops"]}
-    if cp is not None:
+    if cp is not None and "error" in cp:
+        line["branch_prefill"] = cp
+    elif cp is not None:
         cms = max_over_ranks(torch, world, cp["ms"])
         achieved = cp["flops"] / (cp["ms"] * 1e-3) / 1e12
         line["branch_prefill"] = {
@@ -771,7 +773,9 @@ def main():
             "roofline": {"bound": "tensor", "achieved": achieved, "peak": peaks["bf16_tflops"], "unit": "TFLOP/s",
                          "frac": achieved / peaks["bf16_tflops"], "traffic": None,
                          "peak_source": f"{peak_src} bf16_tflops (burst)", "algorithmic_flops": cp["flops"]}}
-    if lp is not None:
+    if lp is not None and "error" in lp:
+        line["loop"] = lp
+    elif lp is not None:
         tokens = lp["tokens"] * world
         e2e_s = max_over_ranks(torch, world, lp["e2e_s"])
         dev_s = max_over_ranks(torch, world, lp["dev_s"])
