@@ -188,6 +188,13 @@ class LoopTokenSource:
             for k, f in enumerate(pg.fork_offset):
                 d.setdefault(int(f), []).append(k)
             self._forks_by_count.append(d)
+        # forks per (page, layout tokens in the cache), flattened: page p's counts c = 0..L start at _fbase[p]
+        self._fbase = np.concatenate([[0], np.cumsum([pg.layout_len + 1 for pg in self.pages])[:-1]]).astype(np.int64) \
+            if n else np.zeros(0, np.int64)
+        self._fcount = np.zeros(int(sum(pg.layout_len + 1 for pg in self.pages)) + 1, np.int32)
+        for p, pg in enumerate(self.pages):
+            for f in pg.fork_offset:
+                self._fcount[self._fbase[p] + int(f)] += 1
         cap = n + int(sum(nb))           # every stream ever: one layout stream and N branches per page
         self._page = np.full(max(cap, 1), -1, np.int64)
         self._flat = np.full(max(cap, 1), -1, np.int64)   # -1: layout stream, else flat branch index
@@ -243,12 +250,9 @@ class LoopTokenSource:
         pg, fl, c = self._page[ids], self._flat[ids], self._count[ids]
         lay = fl < 0
         eos = np.where(lay, c == self._L[pg], c == self._nlen[np.where(lay, 0, fl)]).astype(np.uint8)
-        nf = np.zeros(len(ids), np.int32)
-        for i in np.nonzero(lay)[0]:
-            ks = self._forks_at(int(pg[i]), int(c[i]))
-            if ks:
-                self._pending[int(ids[i])] = ks
-                nf[i] = len(ks)
+        nf = np.where(lay, self._fcount[np.where(lay, self._fbase[pg] + np.minimum(c, self._L[pg]), 0)], 0).astype(np.int32)
+        for i in np.nonzero(nf)[0]:
+            self._pending[int(ids[i])] = self._forks_at(int(pg[i]), int(c[i]))
         return nf, eos
 
     def forked(self, ids, num_forks, new_streams) -> None:
