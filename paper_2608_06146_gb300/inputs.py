@@ -180,8 +180,10 @@ class LoopTokenSource:
         self._L = np.asarray([pg.layout_len for pg in self.pages], np.int64)
         nb = [pg.num_branches for pg in self.pages]
         self._kbase = np.concatenate([[0], np.cumsum(nb)[:-1]]).astype(np.int64) if n else np.zeros(0, np.int64)
-        self._yabs = np.asarray([self.base[p] + y for p in range(n) for y in self.ybase[p]], np.int64)
-        self._nlen = np.asarray([x for pg in self.pages for x in pg.branch_len], np.int64)
+        # one unused element at the end: np.where evaluates both of its arms, so a layout stream's
+        # lookup of these per-branch arrays needs an index even when no page has a branch
+        self._yabs = np.asarray([self.base[p] + y for p in range(n) for y in self.ybase[p]] + [0], np.int64)
+        self._nlen = np.asarray([x for pg in self.pages for x in pg.branch_len] + [0], np.int64)
         self._forks_by_count = []
         for pg in self.pages:
             d = {}
