@@ -47,8 +47,12 @@ def test_chunk_plan_covers_every_visible_row_once(seed, tc_ctas):
     page_len, chunks = rand_chunks(rng, int(rng.integers(1, 5)))
     if len(chunks) == 0:
         chunks = np.array([[0, 0, 0, 1]], np.int32)
+    check_chunk_plan(page_len, chunks, tc_ctas)
+
+
+def check_chunk_plan(page_len, chunks, tc_ctas, warp_ctas=0):
     Hkv = 2
-    cfg = pa.make_decode_config(16, Hkv, 128, tc_ctas=tc_ctas, warp_ctas=0)
+    cfg = pa.make_decode_config(16, Hkv, 128, tc_ctas=tc_ctas, warp_ctas=warp_ctas)
     plan, info = pa.padoc_build_chunk_prefill_plan(page_len, chunks, cfg)
     ex = expand(chunks)
     S = len(ex)
@@ -112,3 +116,35 @@ def test_chunk_plan_validation_and_table():
     chunks = np.array([[0, 5, 0, 2], [0, 5, -1, 1], [1, 3, 7, 3]], np.int32)
     t = pa.padoc_expand_chunk_table(chunks, np.array([[4, 5], [0, 0], [9, 8]], np.int32), 3)
     np.testing.assert_array_equal(t, [[4, 5, -1], [4, 5, -1], [0, 0, -1], [9, 8, -1], [9, 8, -1], [9, 8, -1]])
+
+
+def test_chunk_plan_properties():
+    """hypothesis draws pages and chunks (1 to 70 tokens, branch chunks anywhere in a branch,
+    shared-stream chunks up to the page's end, cutoffs 0 and page_len) and CTA counts; every plan
+    reads each token's visible rows exactly once with consistent slots."""
+    hyp = pytest.importorskip("hypothesis")
+    st = pytest.importorskip("hypothesis.strategies")
+
+    @st.composite
+    def cases(draw):
+        n_pages = draw(st.integers(1, 3))
+        page_len = [draw(st.integers(0, 700)) for _ in range(n_pages)]
+        chunks = []
+        for p in range(n_pages):
+            for _ in range(draw(st.integers(0, 4))):
+                n = draw(st.integers(1, 70))
+                if page_len[p] >= n and draw(st.booleans()):
+                    chunks.append((p, draw(st.integers(0, page_len[p] - n)), -1, n))
+                else:
+                    chunks.append((p, draw(st.integers(0, page_len[p])), draw(st.integers(0, 300)), n))
+        if not chunks:
+            chunks = [(0, 0, 0, 1)]
+        return (np.asarray(page_len, np.int32), np.asarray(chunks, np.int32).reshape(-1, 4),
+                draw(st.sampled_from([0, 1, 2, 7])), draw(st.sampled_from([0, 1, 3])))
+
+    @hyp.settings(max_examples=80, deadline=None)
+    @hyp.given(cases())
+    def run(case):
+        check_chunk_plan(*case)
+
+    run()
