@@ -163,7 +163,10 @@ def _plan_items(plan, info):
 @pytest.mark.parametrize("wl_name,layout", [("decode_page", False), ("dense_page", False), ("serving_batch", True),
                                             ("serving_batch", False), ("tiny", False)])
 def test_decode_plan_covers_every_visible_token_once(wl_name, layout, tc_ctas, warp_ctas):
-    wl = inputs.WORKLOADS[wl_name]()
+    check_decode_plan(inputs.WORKLOADS[wl_name](), layout, tc_ctas, warp_ctas)
+
+
+def check_decode_plan(wl, layout, tc_ctas, warp_ctas):
     Hkv = wl.num_kv_heads
     cfg = pa.make_decode_config(wl.num_q_heads, Hkv, wl.head_dim, 16, layout, 0, tc_ctas, warp_ctas)
     plan, info = pa.padoc_build_decode_plan(wl.pages, cfg)
@@ -253,6 +256,37 @@ def test_decode_plan_covers_every_visible_token_once(wl_name, layout, tc_ctas, w
         assert te <= (sh[fs] if kind == 0 else pl[fs])
     need = pa.padoc_decode_workspace_size(info)
     assert need >= info.num_slots * (wl.num_q_heads // Hkv) * (wl.head_dim + 1) * 4
+
+
+def test_decode_plan_properties():
+    """hypothesis draws the pages (prefixes 0-3000, 0-40 branches with any fork offsets and private
+    lengths 1-900, layout streams or not) and the CTA counts; every plan passes the coverage,
+    slot, balance and cutoff checks above."""
+    hyp = pytest.importorskip("hypothesis")
+    st = pytest.importorskip("hypothesis.strategies")
+
+    @st.composite
+    def cases(draw):
+        pages = []
+        for _ in range(draw(st.integers(1, 8))):
+            P, L, N = draw(st.integers(0, 3000)), draw(st.integers(0, 300)), draw(st.integers(0, 40))
+            if P + L == 0:
+                P = 1
+            forks = draw(st.lists(st.integers(0, L), min_size=N, max_size=N))
+            lens = draw(st.lists(st.integers(1, 900), min_size=N, max_size=N))
+            pages.append(PageSpec(P, L, forks, lens))
+        wl = inputs.Workload("drawn", pages, 16, 2, 128, None, "decode")
+        return wl, draw(st.booleans()), draw(st.sampled_from([0, 1, 5, 96])), draw(st.sampled_from([0, 1, 4, 152]))
+
+    @hyp.settings(max_examples=60, deadline=None)
+    @hyp.given(cases())
+    def run(case):
+        wl, layout, tc, wc = case
+        if not layout and all(pg.num_branches == 0 for pg in wl.pages):
+            return   # no stream at all
+        check_decode_plan(wl, layout, tc, wc)
+
+    run()
 
 
 def test_decode_plan_rejects_bad_config():
