@@ -315,3 +315,41 @@ def test_page_array_plans_like_page_objects():
     a, _ = pa.padoc_build_decode_plan(arr, cfg)
     b, _ = pa.padoc_build_decode_plan(grown, cfg)
     np.testing.assert_array_equal(a, b)
+
+
+C_PROGRAM = r"""
+#include <stdio.h>
+#include "padoc_attn.h"
+int main(void) {
+    int32_t forks[2] = {3, 8}, lens[2] = {5, 20};
+    padoc_page pg = {40, 8, 2, forks, lens};
+    int64_t T = 0;
+    padoc_status st = padoc_packed_size(&pg, 1, &T);
+    padoc_mpd *m = NULL;
+    st |= padoc_mpd_create(64, 16, NULL, &m);
+    int32_t pid, slots[40], news[3], lp, ls, fb;
+    st |= padoc_mpd_add_page(m, 40, 2, 0, &pid, slots, news);
+    st |= padoc_mpd_status(m, &lp, &ls, &fb);
+    padoc_mpd_destroy(m);
+    printf("%d %lld %d %d %d %s\n", (int)st, (long long)T, lp, ls, fb, padoc_status_string(PADOC_OK));
+    return st != PADOC_OK;
+}
+"""
+
+
+def test_header_is_plain_c_and_links_from_c(tmp_path):
+    """The C ABI is C: the header compiles as strict C11 without CUDA's headers, and a C program
+    links against the library and runs its host calls."""
+    import shutil
+    import subprocess
+    if shutil.which("gcc") is None:
+        pytest.skip("no C compiler")
+    src = tmp_path / "t.c"
+    src.write_text(C_PROGRAM)
+    inc = os.path.dirname(HEADER)
+    libdir = os.path.dirname(pbuild.LIB)
+    exe = tmp_path / "t"
+    subprocess.check_call(["gcc", "-std=c11", "-Wall", "-Wextra", "-Werror", "-pedantic", "-I", inc, str(src), "-L", libdir,
+                           "-lpadoc_attn", f"-Wl,-rpath,{libdir}", "-o", str(exe)])
+    out = subprocess.run([str(exe)], capture_output=True, text=True, check=True).stdout.split()
+    assert out == ["0", "73", "1", "3", "61", "ok"]   # 40 + 8 + 5 + 20 tokens; one page, 3 streams; 3 prefix blocks taken
