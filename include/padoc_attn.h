@@ -46,7 +46,9 @@
 extern "C" {
 #endif
 
-#define PADOC_ATTN_VERSION 1
+/* 1: descriptors, decode, prefill, combine, prefill backward, no-alloc decode. 2 adds the
+ * stream-list and chunked-prefill planners, Algorithm 1's loop (padoc_mpd_*) and the append call. */
+#define PADOC_ATTN_VERSION 2
 
 /* A CUDA stream handle; identical to cudaStream_t. */
 typedef struct CUstream_st *padoc_stream_t;
