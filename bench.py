@@ -42,12 +42,12 @@ sys.path.insert(0, ROOT)
 
 METRIC = "ancestor-attn decode queries/s, % of HBM roofline; packed prefill TFLOP/s"
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
-# dram__bytes_read.sum + dram__bytes_write.sum per launch from the ncu captures summarised under
-# profiles/ (None until a capture of the current kernel exists). Decode: one step = the three
-# kernels' counters added up (profiles/decode_traffic_serving_batch.md), cold caches.
-TRAFFIC_BYTES = {"decode": 224_800_000,    # profiles/decode_traffic_serving_batch.md
-                 "prefill": 260_600_000,   # profiles/prefill_tc_packed_32k.md
-                 "prefill_bwd": 1_459_570_000}  # both passes: profiles/prefill_bwd_packed_32k.md
+# DRAM traffic per launch, dram__bytes_read.sum + dram__bytes_write.sum, copied from one ncu capture
+# of each kernel as it stands (cold caches); None where no capture of the current kernel exists.
+# Decode: one step = its three kernels' counters added up. Prefill backward: both passes.
+TRAFFIC_BYTES = {"decode": 224_800_000,
+                 "prefill": 260_600_000,
+                 "prefill_bwd": 1_459_570_000}
 
 
 def load_peaks():
@@ -123,23 +123,39 @@ class ClockSampler:
 # Workloads
 # ------------------------------------------------------------------------------------------------
 
-def decode_bytes(wl, streams_sp, streams_sh, streams_pl):
-    """Minimum HBM bytes of one decode step: each page's visible shared stream once per KV head,
-    every private row once, Q in, O and LSE out."""
+def decode_bytes(wl, layout_streams=False, kv_bytes=2, scale_bytes=0):
+    """Minimum HBM bytes of one decode step: each page's shared stream once per KV head up to the
+    last row any of its streams sees (P + max f_k, or P + L when the layout stream is decoded),
+    every private row once, Q in, O and LSE out. ``kv_bytes`` per K/V element; ``scale_bytes`` per
+    (16-token block, KV head) for K and for V each (a quantized cache's scales)."""
     Hq, Hkv, d = wl.num_q_heads, wl.num_kv_heads, wl.head_dim
-    esz = 2
-    shared = 0
-    for p in range(len(wl.pages)):
-        mask = streams_sp == p
-        if mask.any():
-            shared += int(streams_sh[mask].max())
-    priv = int(streams_pl.sum())
-    S = len(streams_sp)
-    return (shared + priv) * Hkv * d * 2 * esz + S * Hq * d * esz * 2 + S * Hq * 4
+    shared = priv = S = sblk = 0
+    for pg in wl.pages:
+        n = pg.num_branches + (1 if layout_streams else 0)
+        if n == 0:
+            continue
+        cut = pg.prefix_len + (pg.layout_len if layout_streams else max(pg.fork_offset))
+        shared += cut
+        priv += int(sum(pg.branch_len))
+        sblk += -(-cut // 16) + sum(-(-b // 16) for b in pg.branch_len)
+        S += n
+    return ((shared + priv) * Hkv * d * 2 * kv_bytes + sblk * Hkv * 2 * scale_bytes
+            + S * Hq * d * 2 * 2 + S * Hq * 4)
+
+
+def visible_pairs(pages) -> int:
+    """Visible (query, key) pairs of a packed prefill, summed in closed form per page."""
+    n = 0
+    for pg in pages:
+        P, L = pg.prefix_len, pg.layout_len
+        M = P + L
+        n += M * (M + 1) // 2
+        for f, b in zip(pg.fork_offset, pg.branch_len):
+            n += b * (P + f) + b * (b + 1) // 2
+    return n
 
 
 def prefill_flops(wl):
-    from paper_2608_06146_gb300.engine import visible_pairs
     return 4.0 * wl.head_dim * wl.num_q_heads * visible_pairs(wl.pages)
 
 
@@ -148,6 +164,80 @@ def l2_bytes(torch):
         return int(torch.cuda.get_device_properties(torch.cuda.current_device()).L2_cache_size)
     except Exception:
         return 129 * 1024 * 1024
+
+
+class StepGraphs:
+    """Decode steps captured in CUDA graphs: graph g holds ``n`` consecutive steps starting at step
+    ``first``. A step's kernels are programmatic dependents of the previous step's, and capture keeps
+    those dependencies as programmatic edges, so consecutive steps inside a graph overlap exactly as
+    they do when launched one by one; what the graph removes is the host's per-launch cost."""
+
+    def __init__(self, torch, step, first, n, stream):
+        self.g = torch.cuda.CUDAGraph()
+        cap = torch.cuda.Stream()
+        cap.wait_stream(stream)
+        with torch.cuda.graph(self.g, stream=cap):
+            s = torch.cuda.current_stream()
+            for i in range(n):
+                step(first + i, s)
+        stream.wait_stream(cap)
+        self.n = n
+
+    def replay(self):
+        self.g.replay()
+
+
+def time_steps(args, torch, world, stream, step, steady=True, steady_steps=25000, steady_graph=1000):
+    """W eager warm-up steps; then exactly K steps from CUDA graphs between one pair of CUDA events,
+    bracketed by a barrier and a synchronize; then (``steady``) a long run of back-to-back steps,
+    each graph replay of ``steady_graph`` steps timed with its own events, whose median, minimum and
+    maximum per-step times are reported. nvidia-smi samples clocks over both timed regions."""
+    for i in range(args.warmup):
+        step(i, stream)
+    torch.cuda.synchronize()
+    import paper_2608_06146_gb300.padoc_attn as pa
+    pa.padoc_check_device_errors(stream)
+    K = args.steps
+    G = min(K, 500)
+    graphs = [StepGraphs(torch, step, args.warmup, G, stream)]
+    if K % G:
+        graphs.append(StepGraphs(torch, step, args.warmup + (K // G) * G, K % G, stream))
+    plan = [graphs[0]] * (K // G) + graphs[1:]
+    for g in graphs:           # first replays upload the graphs
+        g.replay()
+    torch.cuda.synchronize()
+    pa.padoc_check_device_errors(stream)
+    barrier(torch, world)
+    torch.cuda.synchronize()
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    res = {}
+    with ClockSampler(physical_gpu_index(torch.cuda.current_device())) as clk:
+        ev0.record(stream)
+        with torch.cuda.stream(stream):
+            for g in plan:
+                g.replay()
+        ev1.record(stream)
+        torch.cuda.synchronize()
+        barrier(torch, world)
+        res["ms"] = ev0.elapsed_time(ev1) / K
+        if steady and not args.no_steady:
+            sg = StepGraphs(torch, step, args.warmup, steady_graph, stream)
+            reps = max(1, steady_steps // steady_graph)
+            evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(reps + 1)]
+            with torch.cuda.stream(stream):
+                sg.replay()
+                for a, b in evs:
+                    a.record(stream)
+                    sg.replay()
+                    b.record(stream)
+            torch.cuda.synchronize()
+            per = sorted(a.elapsed_time(b) / steady_graph for a, b in evs[1:])
+            res["steady"] = dict(steps=reps * steady_graph, graph_steps=steady_graph, replays=reps,
+                                 median_ms=statistics.median(per), min_ms=per[0], max_ms=per[-1],
+                                 mean_ms=sum(per) / len(per))
+    pa.padoc_check_device_errors(stream)
+    res["clocks"] = clk.summary()
+    return res
 
 
 def bench_decode(args, torch, dev, rank, world, layout_streams=False):
@@ -174,32 +264,16 @@ def bench_decode(args, torch, dev, rank, world, layout_streams=False):
     lses = [torch.empty((S, wl.num_q_heads), dtype=torch.float32, device=dev) for _ in range(R)]
     stream = torch.cuda.current_stream()
 
-    def step(i):
+    def step(i, s):
         r = i % R
-        plan.run(k_pools[r], v_pools[r], page_table, stream_table, qs[r], scale, outs[r], lses[r], stream)
+        plan.run(k_pools[r], v_pools[r], page_table, stream_table, qs[r], scale, outs[r], lses[r], s)
 
-    for i in range(args.warmup):
-        step(i)
-    pa.padoc_check_device_errors(stream)
-    barrier(torch, world)
-    torch.cuda.synchronize()
-    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    with ClockSampler(physical_gpu_index(torch.cuda.current_device())) as clk:
-        ev0.record(stream)
-        for i in range(args.steps):
-            step(args.warmup + i)
-        ev1.record(stream)
-        torch.cuda.synchronize()
-    barrier(torch, world)
-    pa.padoc_check_device_errors(stream)
-    ms = ev0.elapsed_time(ev1) / args.steps
-
-    sp, sh, pl = inputs.decode_streams(wl, layout_streams)
-    nbytes = decode_bytes(wl, sp, sh, pl)
+    timing = time_steps(args, torch, world, stream, step, steady=not layout_streams)
+    nbytes = decode_bytes(wl, layout_streams)
     info = plan.info
     launches = (1 if info.num_tc_items > 0 else 0) + (1 if info.num_warps > 0 else 0) + 1   # + the merge
-    res = dict(ms=ms, streams=S, bytes=nbytes, launches=launches, clocks=clk.summary(), replicas=R,
-               pages=len(wl.pages), e2e_ms=None, h2d=0, d2h=0)
+    res = dict(ms=timing["ms"], streams=S, bytes=nbytes, launches=launches, clocks=timing["clocks"], replicas=R,
+               pages=len(wl.pages), e2e_ms=None, h2d=0, d2h=0, steady=timing.get("steady"))
     if args.no_e2e or layout_streams:
         return res
 
@@ -563,8 +637,7 @@ def cpu_baseline_decode(max_seconds=20.0):
         wl = inputs.Workload("sample", [wl_full.pages[p]], 16, 2, 128, wl_full.dtype, "decode")
         di = inputs.decode_inputs(wl, 3)
         t0 = time.perf_counter()
-        oracle.decode(di.stream_page, di.shared_len, di.priv_len, di.page_off, di.priv_off, di.stream_k, di.stream_v,
-                      di.priv_k, di.priv_v, di.q, scale)
+        oracle.decode_pages(wl.pages, di, scale)
         elapsed += time.perf_counter() - t0
         done_streams += len(di.stream_page)
         pages_used += 1
@@ -575,24 +648,31 @@ def cpu_baseline_decode(max_seconds=20.0):
                       f"queries x 16 heads), fp64, OpenMP, {elapsed:.2f} s"}
 
 
+def decode_config(pages, streams, world):
+    """The headline workload, as both arms name it."""
+    return {"workload": "concurrent serving batch decode step: 32 pages, prefix U[1024,4096], Poisson(20) "
+                        "branches/page, log-normal private KV (median 96, cap 2048)",
+            "pages": pages, "streams_per_gpu": streams, "num_q_heads": 16, "num_kv_heads": 2, "head_dim": 128,
+            "block_size": 16, "parallelism": f"replicas x{world} (pages per GPU)",
+            "l2": "inputs rotate over replicas in distinct memory totalling more than 4x L2"}
+
+
 def run_reference(args):
-    """The oracle as the reference arm: each step is the decode of a bounded sample of the serving
-    batch (the first 2 pages) on the host cores."""
+    """The oracle as the reference arm: each step is the decode step of the whole 32-page serving
+    batch (the headline's workload), fp64 on the host cores."""
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
         return 0
     import oracle
     from paper_2608_06146_gb300 import inputs
     oracle.build()
-    wl_full = inputs.serving_batch(seed=3)
-    wl = inputs.Workload("sample", wl_full.pages[:2], 16, 2, 128, wl_full.dtype, "decode")
-    di = inputs.decode_inputs(wl, 3)
+    wl = inputs.serving_batch(seed=3)
+    di = inputs.decode_inputs(wl, 3, pool_slack=1.0)
     scale = 1.0 / math.sqrt(wl.head_dim)
     S = len(di.stream_page)
 
     def step():
-        oracle.decode(di.stream_page, di.shared_len, di.priv_len, di.page_off, di.priv_off, di.stream_k, di.stream_v,
-                      di.priv_k, di.priv_v, di.q, scale)
+        oracle.decode_pages(wl.pages, di, scale)
 
     for _ in range(args.warmup):
         step()
@@ -605,10 +685,9 @@ def run_reference(args):
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "queries/s", "n_gpus": args.gpus,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": dt * 1e3, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": {"workload": "concurrent serving batch decode step (sample: first 2 of 32 pages)",
-                       "streams": S, "num_q_heads": 16, "num_kv_heads": 2, "head_dim": 128, "block_size": 16},
+            "config": decode_config(len(wl.pages), S, args.gpus),
             "cpu_baseline": {"value": value, "unit": "queries/s", "cores": cores, "kind": "oracle",
-                             "sample": f"first 2 of 32 serving-batch pages, {S} branch queries per step"},
+                             "sample": f"the whole 32-page serving batch, {S} branch queries x 16 heads per step"},
             "e2e": {"value": value, "unit": "queries/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line))
     return 0
@@ -617,7 +696,7 @@ def run_reference(args):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=4000)
+    ap.add_argument("--steps", type=int, default=200)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="padoc", choices=["padoc", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -625,6 +704,7 @@ def main():
                                                       "chunk_prefill", "variants"])
     ap.add_argument("--replicas", type=int, default=0, help="decode input replicas (0: enough to exceed 4x L2)")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-steady", action="store_true", help="skip the long back-to-back decode run")
     ap.add_argument("--tc-ctas", type=int, default=0, help="tensor-core decode CTAs (0: one per SM)")
     ap.add_argument("--warp-ctas", type=int, default=0, help="warp-kernel decode CTAs (0: one per SM)")
     ap.add_argument("--split-tokens", type=int, default=0, help="decode shared-stream split (0: library default)")
@@ -700,14 +780,24 @@ def main():
     line = {"metric": METRIC, "value": value, "unit": "queries/s", "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-            "config": {"workload": "concurrent serving batch decode step: 32 pages, prefix U[1024,4096], "
-                                   "Poisson(20) branches/page, log-normal private KV (median 96, cap 2048)",
-                       "pages": d["pages"], "streams_per_gpu": d["streams"], "num_q_heads": 16, "num_kv_heads": 2,
-                       "head_dim": 128, "block_size": 16, "parallelism": f"replicas x{world} (pages per GPU)",
-                       "l2": f"{d['replicas']} rotating input replicas > 4x L2"},
+            "config": decode_config(d["pages"], d["streams"], world),
+            "l2_replicas": d["replicas"],
+            "timing": "the K steps replayed from CUDA graphs (steps as programmatic dependents of one another, as "
+                      "when launched one by one) between one pair of CUDA events",
             "roofline": roof, "gpu_launches": d["launches"] * args.steps, "clocks": d["clocks"],
             "e2e": {"value": total_streams / (e2e_ms * 1e-3), "unit": "queries/s", "h2d_bytes_per_step": d["h2d"],
                     "d2h_bytes_per_step": d["d2h"]}}
+    if d.get("steady"):
+        sd = d["steady"]
+        sach = d["bytes"] / (sd["median_ms"] * 1e-3) / 1e9
+        line["decode_steady"] = {
+            "value": total_streams / (max_over_ranks(torch, world, sd["median_ms"]) * 1e-3), "unit": "queries/s",
+            "median_ms_per_step": sd["median_ms"], "min_ms_per_step": sd["min_ms"], "max_ms_per_step": sd["max_ms"],
+            "mean_ms_per_step": sd["mean_ms"], "steps": sd["steps"],
+            "how": f"{sd['replays']} replays of a CUDA graph of {sd['graph_steps']} back-to-back decode steps over the "
+                   "same rotating replicas, each replay between its own CUDA events; per-step median over replays",
+            "roofline": {"bound": "hbm", "achieved": sach, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                         "frac": sach / peaks["hbm_gbs"], "algorithmic_bytes": d["bytes"]}}
     if cpu is not None:
         line["cpu_baseline"] = cpu
     if p is not None:

@@ -283,7 +283,9 @@ padoc_status padoc_branch_decode_attn(const padoc_kv_pool *pool, const padoc_dec
  * PADOC_STATIC_WORKSPACE_BYTES (32 MiB) that every GPU which loads this library holds until the
  * process exits; the call allocates nothing (no cudaMalloc, cudaFree or allocating library call).
  *   - The first call on a device looks up that device's address of the array (once per device,
- *     with that device current); make that first call before any stream capture.
+ *     with that device current); make that first call before any stream capture. The address is
+ *     kept for the life of the process, so the library must not be used on a device after a
+ *     cudaDeviceReset of it (the same holds for the device error word of every call).
  *   - Every call shares the one array, and it keeps the last call's contents. The decode writes
  *     every partial it later reads, so nothing needs clearing, but calls that overlap on the GPU
  *     (other streams, other host threads, concurrent graph launches) race on it: serialize them.
@@ -560,6 +562,16 @@ padoc_status padoc_ancestor_prefill_bwd(const void *q, const void *k, const void
  * compares them with its own product. Errors: INVALID_ARGUMENT, CUDA. */
 padoc_status padoc_selftest_tcgen05(const void *a, const void *bk, const void *v, float *c1, float *c2, float *c3,
                                     padoc_stream_t stream);
+
+/* Self-check of the failure path every kernel's waits share (no counterpart in the paper: the
+ * library's own failure detection). One CTA of 64 threads waits, with the same bounded mbarrier
+ * wait the kernels use but a limit of limit_us microseconds (1 .. 100000), on a barrier that nothing
+ * ever arrives at. The wait gives up, records code 2 (bounded wait ran out) with `site` as the
+ * detail in the device error word, and every thread that gave up adds 1 to *gave_up ((device)
+ * int32, which the caller zeroes first); the kernel then returns, nothing being in flight, and the
+ * context stays usable. Read the error with padoc_check_device_errors.
+ * Errors: INVALID_ARGUMENT, CUDA. */
+padoc_status padoc_selftest_wait_timeout(int32_t limit_us, int32_t site, int32_t *gave_up, padoc_stream_t stream);
 
 /* Synchronizes `stream`, then reads and clears the current device's error word. Returns
  * PADOC_ERR_DEVICE_CHECK if a kernel recorded a failed check since the last call (code and detail

@@ -159,6 +159,39 @@ def prefill_gather(pages, q, k, v, scale):
     return _prefill("oracle_prefill_gather", pages, q, k, v, scale)
 
 
+def decode_streams(pages, layout_streams: bool = False):
+    """The per-stream decode plan {page, shared_len, private_len} of a decode step, in stream order
+    (each page's branches in order, then with ``layout_streams`` its layout stream).
+
+    Sec. 3.2 gives branch k the ancestors {X, B_<=k}: the whole prefix X and the layout-stream
+    tokens written before it forked, f_k of them (Algorithm 1 copies the layout row before the
+    region's boundary output is appended), so its cutoff on the page's shared stream [X | layout]
+    is P + f_k and its private rows are its own n_k tokens, the newest being the one decoded
+    (Algorithm 1 appends before it decodes). The layout stream sees the prefix and all L of its own
+    tokens and has no private rows: cutoff P + L, private 0."""
+    sp, sh, pl = [], [], []
+    for p, pg in enumerate(pages):
+        if isinstance(pg, tuple):
+            P, L, forks, lens = pg
+        else:
+            P, L, forks, lens = pg.prefix_len, pg.layout_len, pg.fork_offset, pg.branch_len
+        for f, n in zip(forks, lens):
+            assert 0 <= f <= L and n >= 1
+            sp.append(p); sh.append(P + f); pl.append(n)
+        if layout_streams:
+            sp.append(p); sh.append(P + L); pl.append(0)
+    return np.asarray(sp, np.int32), np.asarray(sh, np.int32), np.asarray(pl, np.int32)
+
+
+def decode_pages(pages, di, scale, layout_streams: bool = False):
+    """``decode`` of every stream of ``pages`` over the logical rows of ``di`` (an object with the
+    fields page_off, priv_off, stream_k, stream_v, priv_k, priv_v and q laid out as the seeded
+    input generator does), each stream's cutoff and private length taken from ``decode_streams``."""
+    sp, sh, pl = decode_streams(pages, layout_streams)
+    assert np.array_equal(sp, np.asarray(di.stream_page)) and np.array_equal(pl, np.asarray(di.priv_len))
+    return decode(sp, sh, pl, di.page_off, di.priv_off, di.stream_k, di.stream_v, di.priv_k, di.priv_v, di.q, scale)
+
+
 def decode(stream_page, shared_len, priv_len, page_off, priv_off, stream_k, stream_v, priv_k, priv_v,
            q, scale):
     """One decode step over logical (unpaged) K/V; see padoc_oracle.c:oracle_decode."""

@@ -79,19 +79,26 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity)
     return ok != 0;
 }
 
-// Waits for the phase with the given parity to complete; false (and the error word set) if it
-// does not complete within PADOC_WAIT_LIMIT_NS.
-__device__ __forceinline__ bool mbar_wait_bounded(uint32_t bar, uint32_t parity, int *err, int site)
+// Waits for the phase with the given parity to complete; false (and the error word set to
+// PADOC_DEVERR_TIMEOUT with `site` as the detail) if it does not complete within limit_ns.
+__device__ __forceinline__ bool mbar_wait_bounded_ns(uint32_t bar, uint32_t parity, int *err, int site,
+                                                     uint64_t limit_ns)
 {
     if (mbar_try_wait(bar, parity)) return true;
     const uint64_t t0 = padoc_globaltimer();
     for (uint32_t i = 1;; ++i) {
         if (mbar_try_wait(bar, parity)) return true;
-        if ((i & 255u) == 0 && padoc_globaltimer() - t0 > PADOC_WAIT_LIMIT_NS) {
+        if ((i & 255u) == 0 && padoc_globaltimer() - t0 > limit_ns) {
             padoc_record_error(err, PADOC_DEVERR_TIMEOUT, site);
             return false;
         }
     }
+}
+
+// The kernels' wait: mbar_wait_bounded_ns with the library's limit, PADOC_WAIT_LIMIT_NS.
+__device__ __forceinline__ bool mbar_wait_bounded(uint32_t bar, uint32_t parity, int *err, int site)
+{
+    return mbar_wait_bounded_ns(bar, parity, err, site, PADOC_WAIT_LIMIT_NS);
 }
 
 // ------------------------------------------------------------------------------------------------

@@ -499,7 +499,8 @@ extern "C" padoc_status padoc_branch_decode_attn(const padoc_kv_pool *pool, cons
     if (cfg.head_dim != kD || cfg.num_q_heads != kGroup * cfg.num_kv_heads || cfg.block_size != kBlk)
         return PADOC_ERR_UNSUPPORTED;
     size_t need = 0;
-    padoc_decode_workspace_size(info, &need);
+    const padoc_status ws_st = padoc_decode_workspace_size(info, &need);
+    if (ws_st != PADOC_OK) return ws_st;
     if (!workspace || workspace_bytes < need) return PADOC_ERR_WORKSPACE_TOO_SMALL;
     if (((uintptr_t)workspace) & 255) return PADOC_ERR_INVALID_ARGUMENT;
 

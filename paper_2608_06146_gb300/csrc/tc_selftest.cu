@@ -95,7 +95,35 @@ tc_selftest_kernel(const __nv_bfloat16 *__restrict__ a, const __nv_bfloat16 *__r
     if (warp == 0) tmem_dealloc(tmem, 512);
 }
 
+// One CTA waits, with the kernels' bounded wait and a limit of limit_ns, on an mbarrier that
+// nothing arrives at. Nothing else is in flight (no copy, no MMA, no tensor memory), so the CTA
+// leaves cleanly once the wait gives up; every thread checks that it did give up.
+__global__ void __launch_bounds__(64, 1) wait_timeout_selftest_kernel(uint64_t limit_ns, int site, int *err,
+                                                                      int *gave_up)
+{
+    __shared__ uint64_t bar;
+    if (threadIdx.x == 0) {
+        mbar_init(smem_u32(&bar), 1);
+        fence_barrier_init();
+    }
+    __syncthreads();
+    // phase 0 never completes: its one expected arrival is never made
+    const bool done = mbar_wait_bounded_ns(smem_u32(&bar), 0, err, site, limit_ns);
+    if (!done) atomicAdd(gave_up, 1);
+}
+
 }  // namespace
+
+extern "C" padoc_status padoc_selftest_wait_timeout(int32_t limit_us, int32_t site, int32_t *gave_up,
+                                                    padoc_stream_t stream)
+{
+    if (limit_us < 1 || limit_us > 100000 || site < 0 || !gave_up) return PADOC_ERR_INVALID_ARGUMENT;
+    int *err = padoc_device_error_word();
+    if (!err) return PADOC_ERR_CUDA;
+    wait_timeout_selftest_kernel<<<1, 64, 0, (cudaStream_t)stream>>>((uint64_t)limit_us * 1000ull, site, err,
+                                                                     (int *)gave_up);
+    return padoc_launch_status();
+}
 
 extern "C" padoc_status padoc_selftest_tcgen05(const void *a, const void *bk, const void *v, float *c1, float *c2,
                                                float *c3, padoc_stream_t stream)

@@ -216,8 +216,7 @@ class MaskedParallelLoop:
         if self.q_step.shape[0] < C:
             self.q_step = torch.empty((max(C, 2 * self.q_step.shape[0]), self.num_q_heads, self.head_dim),
                                       dtype=self.dtype, device=self.device)
-        group = self.cfg.num_q_heads // self.cfg.num_kv_heads   # padoc_decode_workspace_size, computed here
-        ws = int(info.num_slots) * group * (self.head_dim + 1) * 4 + 512
+        ws = pa.padoc_decode_workspace_size(info)
         if self.workspace.numel() < ws:
             self.workspace = torch.empty(max(ws, 2 * self.workspace.numel()), dtype=torch.uint8, device=self.device)
         if out is None:
@@ -236,18 +235,6 @@ class MaskedParallelLoop:
 
     def status(self):
         return self.mpd.status()
-
-
-def visible_pairs(pages) -> int:
-    """Visible (query, key) pairs of a packed prefill, summed in closed form per page."""
-    n = 0
-    for pg in pages:
-        P, L = pg.prefix_len, pg.layout_len
-        M = P + L
-        n += M * (M + 1) // 2
-        for f, b in zip(pg.fork_offset, pg.branch_len):
-            n += b * (P + f) + b * (b + 1) // 2
-    return n
 
 
 def shard_pages(num_pages: int, rank: int, world: int) -> List[int]:

@@ -324,7 +324,6 @@ class DecodeInputs:
     page_off: np.ndarray
     priv_off: np.ndarray
     stream_page: np.ndarray
-    shared_len: np.ndarray
     priv_len: np.ndarray
     k_pool: torch.Tensor
     v_pool: torch.Tensor
@@ -333,15 +332,18 @@ class DecodeInputs:
     num_blocks: int
 
 
-def decode_streams(wl: Workload, layout_streams: bool = False):
-    """(stream_page, shared_len, priv_len) in the stream order described in ``DecodeInputs``."""
-    sp, sh, pl = [], [], []
+def decode_stream_order(wl: Workload, layout_streams: bool = False):
+    """(stream_page, priv_len) in the stream order described in ``DecodeInputs``: each page's
+    branches with their private lengths as drawn, then (with ``layout_streams``) its layout stream,
+    which has no private rows. Where each stream's view of the shared stream ends is not decided
+    here."""
+    sp, pl = [], []
     for p, pg in enumerate(wl.pages):
-        for f, n in zip(pg.fork_offset, pg.branch_len):
-            sp.append(p); sh.append(pg.prefix_len + f); pl.append(n)
+        for n in pg.branch_len:
+            sp.append(p); pl.append(n)
         if layout_streams:
-            sp.append(p); sh.append(pg.prefix_len + pg.layout_len); pl.append(0)
-    return (np.asarray(sp, np.int32), np.asarray(sh, np.int32), np.asarray(pl, np.int32))
+            sp.append(p); pl.append(0)
+    return np.asarray(sp, np.int32), np.asarray(pl, np.int32)
 
 
 def decode_inputs(wl: Workload, seed: int, layout_streams: bool = False, scale: float = 1.0,
@@ -349,7 +351,7 @@ def decode_inputs(wl: Workload, seed: int, layout_streams: bool = False, scale: 
     """Random logical cache and queries for one decode step, scattered into a block pool whose
     block ids are a seeded random permutation (the pool holds ``pool_slack`` x the needed blocks)."""
     bs, Hkv, d, Hq = wl.block_size, wl.num_kv_heads, wl.head_dim, wl.num_q_heads
-    stream_page, shared_len, priv_len = decode_streams(wl, layout_streams)
+    stream_page, priv_len = decode_stream_order(wl, layout_streams)
     S = len(stream_page)
     page_rows = np.asarray([pg.stream_len for pg in wl.pages], np.int64)
     page_off = np.concatenate([[0], np.cumsum(page_rows)[:-1]]).astype(np.int64)
@@ -392,4 +394,4 @@ def decode_inputs(wl: Workload, seed: int, layout_streams: bool = False, scale: 
         lo = int(priv_off[s]); n = int(priv_len[s])
         scatter(priv_k[lo:lo + n], priv_v[lo:lo + n], n, stream_table[s])
     return DecodeInputs(q, stream_k, stream_v, priv_k, priv_v, page_off, priv_off, stream_page,
-                        shared_len, priv_len, k_pool, v_pool, page_table, stream_table, num_blocks)
+                        priv_len, k_pool, v_pool, page_table, stream_table, num_blocks)

@@ -159,6 +159,7 @@ def load_library(path: Optional[str] = None):
                                   ctypes.POINTER(padoc_kv_pool), _vp, _vp, _vp, ctypes.c_int64, _vp, ctypes.c_float, _vp,
                                   _vp, _vp, ctypes.c_size_t, _vp],
         "padoc_selftest_tcgen05": [_vp, _vp, _vp, _vp, _vp, _vp, _vp],
+        "padoc_selftest_wait_timeout": [ctypes.c_int32, ctypes.c_int32, _vp, _vp],
         "padoc_check_device_errors": [_vp],
         "padoc_last_device_error": [_i32p, _i32p],
         "padoc_status_string": [ctypes.c_int],
@@ -190,7 +191,7 @@ def exported_symbols() -> Sequence[str]:
                         "padoc_mpd_step_tables", "padoc_mpd_end_step", "padoc_mpd_status", "padoc_mpd_prepare_step",
                         "padoc_mpd_launch_step",
                         "padoc_append_inputs",
-                        "padoc_selftest_tcgen05",
+                        "padoc_selftest_tcgen05", "padoc_selftest_wait_timeout",
                         "padoc_check_device_errors",
                         "padoc_last_device_error", "padoc_status_string", "padoc_version")]
 
@@ -716,6 +717,16 @@ def padoc_selftest_tcgen05(a, bk, v, c1, c2, c3, stream=None):
     _check("padoc_selftest_tcgen05", lib.padoc_selftest_tcgen05(_dev(a, "a"), _dev(bk, "bk"), _dev(v, "v"),
                                                                 _dev(c1, "c1"), _dev(c2, "c2"), _dev(c3, "c3"),
                                                                 _stream_ptr(stream)))
+
+
+def padoc_selftest_wait_timeout(limit_us: int, site: int, gave_up, stream=None):
+    """One CTA's bounded wait on an mbarrier nothing arrives at, with a limit of limit_us; the
+    device error word then holds code 2 with ``site``; gave_up (int32 CUDA tensor, zeroed by the
+    caller) counts the threads whose wait gave up."""
+    lib = load_library()
+    _check("padoc_selftest_wait_timeout", lib.padoc_selftest_wait_timeout(int(limit_us), int(site),
+                                                                          _dev(gave_up, "gave_up"),
+                                                                          _stream_ptr(stream)))
 
 
 def padoc_check_device_errors(stream=None):

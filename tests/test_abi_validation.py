@@ -98,3 +98,9 @@ def test_combine_rejects_malformed_calls(lib):
     assert call(S=-1) == 1 and call(R=-1) == 1 and call(d=130) == 1 and call(d=512) == 1
     assert call(R=0) == 0
     assert call(out=None) == 1 and call(po=MIS) == 1
+
+
+def test_wait_timeout_selftest_rejects_malformed_calls(lib):
+    call = lambda limit=1000, site=5, gave_up=A: lib.padoc_selftest_wait_timeout(limit, site, gave_up, None)
+    assert call(limit=0) == 1 and call(limit=100001) == 1   # limits outside 1 us .. 0.1 s
+    assert call(site=-1) == 1 and call(gave_up=None) == 1

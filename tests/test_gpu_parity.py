@@ -47,8 +47,7 @@ def run_decode(wl: Workload, seed: int, layout_streams=False, split_tokens=0, sc
     plan.run(di.k_pool.to(DEV), di.v_pool.to(DEV), torch.from_numpy(di.page_table).to(DEV),
              torch.from_numpy(di.stream_table).to(DEV), q, scale, out, lse)
     pa.padoc_check_device_errors()
-    ref_o, ref_lse = oracle.decode(di.stream_page, di.shared_len, di.priv_len, di.page_off, di.priv_off,
-                                   di.stream_k, di.stream_v, di.priv_k, di.priv_v, di.q, scale)
+    ref_o, ref_lse = oracle.decode_pages(wl.pages, di, scale, layout_streams)
     return out.float().cpu().numpy(), lse.cpu().numpy(), ref_o, ref_lse
 
 
@@ -148,8 +147,7 @@ def test_decode_repeated_calls_on_one_workspace():
         plan.run(di.k_pool.to(DEV), di.v_pool.to(DEV), torch.from_numpy(di.page_table).to(DEV),
                  torch.from_numpy(di.stream_table).to(DEV), di.q.to(DEV), scale, out, lse)
         pa.padoc_check_device_errors()
-        ref_o, ref_lse = oracle.decode(di.stream_page, di.shared_len, di.priv_len, di.page_off, di.priv_off,
-                                       di.stream_k, di.stream_v, di.priv_k, di.priv_v, di.q, scale)
+        ref_o, ref_lse = oracle.decode_pages(wl.pages, di, scale)
         assert_close(out.float().cpu().numpy(), lse.cpu().numpy(), ref_o, ref_lse, torch.bfloat16)
 
 

@@ -170,7 +170,7 @@ def check_decode_plan(wl, layout, tc_ctas, warp_ctas):
     Hkv = wl.num_kv_heads
     cfg = pa.make_decode_config(wl.num_q_heads, Hkv, wl.head_dim, 16, layout, 0, tc_ctas, warp_ctas)
     plan, info = pa.padoc_build_decode_plan(wl.pages, cfg)
-    sp, sh, pl = inputs.decode_streams(wl, layout)
+    sp, sh, pl = oracle.decode_streams(wl.pages, layout)
     S = len(sp)
     assert info.num_streams == S
     np.testing.assert_array_equal(plan[info.off_stream_page: info.off_stream_page + S], sp)

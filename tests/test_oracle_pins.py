@@ -325,15 +325,45 @@ def test_decode_of_newest_token_equals_prefill_row():
     o_pre, l_pre = oracle.prefill_gather([page], q, k, v, 0.35)
     ybase = [P + L + sum(lens[:i]) for i in range(3)]
     rows = [ybase[i] + lens[i] - 1 for i in range(3)] + [P + L - 1]
-    sp = np.zeros(4, np.int32)
-    sh = np.array([P + f for f in forks] + [P + L])
-    pl = np.array(lens + [0])
+    sp, sh, pl = oracle.decode_streams([page], layout_streams=True)
+    np.testing.assert_array_equal(sp, np.zeros(4, np.int32))
     po = np.array([0])
     priv_rows = sum([list(range(ybase[i], ybase[i] + lens[i])) for i in range(3)], [])
     vo = np.array([0, lens[0], lens[0] + lens[1], 0])
     o, lse = oracle.decode(sp, sh, pl, po, vo, k[:P + L], v[:P + L], k[priv_rows], v[priv_rows], q[rows], 0.35)
     np.testing.assert_allclose(o, o_pre[rows], rtol=0, atol=1e-13)
     np.testing.assert_allclose(lse, l_pre[rows], rtol=0, atol=1e-13)
+
+
+@pytest.mark.parametrize("seed", range(6))
+def test_decode_streams_equal_dense_mask_rows_of_newest_tokens(seed):
+    # The per-stream decode plan {page, shared_len, private_len} against the dense visibility built
+    # from node membership: the newest token of branch k sees exactly the first shared_len columns
+    # of its page's shared stream and private_len columns of its own segment; the layout stream's
+    # newest token sees the whole shared stream and nothing else.
+    rng = np.random.default_rng(seed)
+    pages = []
+    for _ in range(3):
+        P, L, n = int(rng.integers(0, 20)), int(rng.integers(0, 9)), int(rng.integers(1, 5))
+        if P + L == 0:
+            P = 1
+        pages.append((P, L, [int(x) for x in rng.integers(0, L + 1, size=n)], [int(x) for x in rng.integers(1, 6, size=n)]))
+    sp, sh, pl = oracle.decode_streams(pages, layout_streams=True)
+    s = 0
+    for p, (P, L, forks, lens) in enumerate(pages):
+        m = oracle.dense_mask(pages, p)
+        ybase = P + L
+        for k, n in enumerate(lens):
+            row = m[ybase + n - 1]
+            assert sp[s] == p and pl[s] == n
+            assert row[:P + L].sum() == sh[s] and row[:sh[s]].all()
+            assert row[ybase:ybase + n].all() and row.sum() == sh[s] + n
+            ybase += n
+            s += 1
+        row = m[P + L - 1]
+        assert sp[s] == p and pl[s] == 0 and sh[s] == P + L and row.sum() == P + L
+        s += 1
+    assert s == len(sp)
 
 
 def test_dense_and_gather_agree_on_workload_shapes():
