@@ -188,53 +188,54 @@ class StepGraphs:
 
 
 def time_steps(args, torch, world, stream, step, steady=True, steady_steps=25000, steady_graph=1000):
-    """W eager warm-up steps; then exactly K steps from CUDA graphs between one pair of CUDA events,
-    bracketed by a barrier and a synchronize; then (``steady``) a long run of back-to-back steps,
-    each graph replay of ``steady_graph`` steps timed with its own events, whose median, minimum and
-    maximum per-step times are reported. nvidia-smi samples clocks over both timed regions."""
+    """W eager warm-up steps, then the graphs are captured and uploaded. Inside the clock sampler:
+    a long run of back-to-back steps (``steady_steps``, replays of a ``steady_graph``-step graph,
+    each replay between its own CUDA events; median, minimum and maximum per step), and right after
+    it, with no idle gap, exactly K steps from CUDA graphs between one pair of CUDA events,
+    bracketed by a barrier and a synchronize. The long run comes first so that the K steps are
+    measured at the clocks the GPU holds under this load, not while it ramps up from idle. With
+    --no-steady the long-run graph is replayed once, untimed, instead."""
+    import paper_2608_06146_gb300.padoc_attn as pa
     for i in range(args.warmup):
         step(i, stream)
     torch.cuda.synchronize()
-    import paper_2608_06146_gb300.padoc_attn as pa
     pa.padoc_check_device_errors(stream)
     K = args.steps
     G = min(K, 500)
     graphs = [StepGraphs(torch, step, args.warmup, G, stream)]
     if K % G:
         graphs.append(StepGraphs(torch, step, args.warmup + (K // G) * G, K % G, stream))
-    plan = [graphs[0]] * (K // G) + graphs[1:]
-    for g in graphs:           # first replays upload the graphs
+    timed = [graphs[0]] * (K // G) + graphs[1:]
+    sg = StepGraphs(torch, step, args.warmup, steady_graph, stream)
+    for g in graphs + [sg]:    # first replays upload the graphs
         g.replay()
     torch.cuda.synchronize()
     pa.padoc_check_device_errors(stream)
-    barrier(torch, world)
-    torch.cuda.synchronize()
+    reps = max(1, steady_steps // steady_graph) if (steady and not args.no_steady) else 0
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(reps)]
     ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     res = {}
     with ClockSampler(physical_gpu_index(torch.cuda.current_device())) as clk:
-        ev0.record(stream)
+        barrier(torch, world)
+        torch.cuda.synchronize()
         with torch.cuda.stream(stream):
-            for g in plan:
+            sg.replay()
+            for a, b in evs:
+                a.record(stream)
+                sg.replay()
+                b.record(stream)
+            ev0.record(stream)
+            for g in timed:
                 g.replay()
-        ev1.record(stream)
+            ev1.record(stream)
         torch.cuda.synchronize()
         barrier(torch, world)
-        res["ms"] = ev0.elapsed_time(ev1) / K
-        if steady and not args.no_steady:
-            sg = StepGraphs(torch, step, args.warmup, steady_graph, stream)
-            reps = max(1, steady_steps // steady_graph)
-            evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(reps + 1)]
-            with torch.cuda.stream(stream):
-                sg.replay()
-                for a, b in evs:
-                    a.record(stream)
-                    sg.replay()
-                    b.record(stream)
-            torch.cuda.synchronize()
-            per = sorted(a.elapsed_time(b) / steady_graph for a, b in evs[1:])
-            res["steady"] = dict(steps=reps * steady_graph, graph_steps=steady_graph, replays=reps,
-                                 median_ms=statistics.median(per), min_ms=per[0], max_ms=per[-1],
-                                 mean_ms=sum(per) / len(per))
+    res["ms"] = ev0.elapsed_time(ev1) / K
+    if reps:
+        per = sorted(a.elapsed_time(b) / steady_graph for a, b in evs)
+        res["steady"] = dict(steps=reps * steady_graph, graph_steps=steady_graph, replays=reps,
+                             median_ms=statistics.median(per), min_ms=per[0], max_ms=per[-1],
+                             mean_ms=sum(per) / len(per))
     pa.padoc_check_device_errors(stream)
     res["clocks"] = clk.summary()
     return res
@@ -783,7 +784,8 @@ def main():
             "config": decode_config(d["pages"], d["streams"], world),
             "l2_replicas": d["replicas"],
             "timing": "the K steps replayed from CUDA graphs (steps as programmatic dependents of one another, as "
-                      "when launched one by one) between one pair of CUDA events",
+                      "when launched one by one) between one pair of CUDA events, right after the long run "
+                      "(decode_steady) with no idle gap",
             "roofline": roof, "gpu_launches": d["launches"] * args.steps, "clocks": d["clocks"],
             "e2e": {"value": total_streams / (e2e_ms * 1e-3), "unit": "queries/s", "h2d_bytes_per_step": d["h2d"],
                     "d2h_bytes_per_step": d["d2h"]}}
