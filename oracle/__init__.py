@@ -77,6 +77,11 @@ def _load():
                                                       ctypes.c_int32, _u8p, _f32p]
             lib.oracle_dequantize_kv_blocks.argtypes = [_u8p, _f32p, ctypes.c_int64, ctypes.c_int32, ctypes.c_int32,
                                                         ctypes.c_int32, _f64p]
+            lib.oracle_append_kv_quantized.argtypes = [_u8p, _f32p, ctypes.c_int64, ctypes.c_int32, ctypes.c_int32,
+                                                       ctypes.c_int32, _i32p, ctypes.c_int32, _f32p]
+            lib.oracle_decode_f64.argtypes = [ctypes.c_int32, _i32p, _i32p, _i32p, _i64p, _i64p, _f64p, _f64p,
+                                              _f64p, _f64p, _f32p, ctypes.c_int32, ctypes.c_int32,
+                                              ctypes.c_int32, ctypes.c_double, _f64p, _f64p]
             _lib = lib
     return _lib
 
@@ -282,7 +287,8 @@ def e4m3_decode(codes) -> np.ndarray:
 
 
 def quantize_kv_blocks(pool):
-    """pool fp32 [num_blocks][Hkv][block][d] -> (codes uint8 same shape, scales fp32 [num_blocks][Hkv])."""
+    """pool fp32 [num_blocks][Hkv][block][d] -> (codes uint8 same shape, scales fp32 [num_blocks][Hkv]);
+    scale = amax / 448 per (block, head), 0 for an all-zero one."""
     x = _f32(pool)
     nb, hkv, bs, d = x.shape
     codes = np.zeros(x.shape, np.uint8)
@@ -299,3 +305,69 @@ def dequantize_kv_blocks(codes, scales) -> np.ndarray:
     out = np.zeros(c.shape, np.float64)
     _load().oracle_dequantize_kv_blocks(_ptr(c, _u8p), _ptr(sc, _f32p), nb, hkv, bs, d, _ptr(out, _f64p))
     return out
+
+
+def append_kv_quantized(codes, scales, slots, rows):
+    """Appends rows [count][Hkv][d] (fp32 values) to slots (block * block + row) of a quantized pool,
+    one at a time in order, with the scale rule of padoc_oracle.c:oracle_append_kv_quantized (the
+    scale grows to amax / 448 of the rows so far; earlier rows are re-encoded when it grows; a
+    block's row 0 starts it afresh). Returns new (codes, scales); the inputs are not changed."""
+    c = np.ascontiguousarray(np.array(codes, np.uint8, copy=True))
+    sc = np.ascontiguousarray(np.array(scales, np.float32, copy=True))
+    nb, hkv, bs, d = c.shape
+    sl = np.ascontiguousarray(np.asarray(slots, np.int32))
+    x = _f32(rows)
+    assert x.shape == (len(sl), hkv, d)
+    if len(sl):
+        _load().oracle_append_kv_quantized(_ptr(c, _u8p), _ptr(sc, _f32p), nb, hkv, bs, d, _ptr(sl, _i32p), len(sl),
+                                           _ptr(x, _f32p))
+    return c, sc
+
+
+def decode_f64(stream_page, shared_len, priv_len, page_off, priv_off, stream_k, stream_v, priv_k, priv_v, q, scale):
+    """``decode`` over fp64 K/V rows (e.g. a dequantized cache); q fp32-exact (bf16 or fp32)."""
+    sp = np.ascontiguousarray(np.asarray(stream_page, np.int32))
+    sh = np.ascontiguousarray(np.asarray(shared_len, np.int32))
+    pl = np.ascontiguousarray(np.asarray(priv_len, np.int32))
+    po = np.ascontiguousarray(np.asarray(page_off, np.int64))
+    vo = np.ascontiguousarray(np.asarray(priv_off, np.int64))
+    sk, sv, pk, pv = (np.ascontiguousarray(np.asarray(a, np.float64)) for a in (stream_k, stream_v, priv_k, priv_v))
+    qq = _f32(q)
+    S, Hq, d = qq.shape
+    Hkv = sk.shape[1] if sk.size else pk.shape[1]
+    guard = lambda a: a if a.size else np.zeros((1, Hkv, d), np.float64)
+    sk, sv, pk, pv = guard(sk), guard(sv), guard(pk), guard(pv)
+    o = np.zeros((S, Hq, d), np.float64)
+    lse = np.zeros((S, Hq), np.float64)
+    if S:
+        _load().oracle_decode_f64(S, _ptr(sp, _i32p), _ptr(sh, _i32p), _ptr(pl, _i32p), _ptr(po, _i64p),
+                                  _ptr(vo, _i64p), _ptr(sk, _f64p), _ptr(sv, _f64p), _ptr(pk, _f64p),
+                                  _ptr(pv, _f64p), _ptr(qq, _f32p), Hq, Hkv, d, float(scale),
+                                  _ptr(o, _f64p), _ptr(lse, _f64p))
+    return o, lse
+
+
+def decode_paged(pages, pool_k, pool_v, page_table, stream_table, q, scale, layout_streams: bool = False,
+                 block_size: int = 16):
+    """One decode step read through the paged layout: pool_k / pool_v [num_blocks][Hkv][block][d]
+    (any real dtype; fp64 for a dequantized cache), page_table [pages][stride] (the block of each
+    block_size rows of the page's shared stream), stream_table [streams][stride] (each stream's
+    private rows from block offset 0). Streams and their cutoffs as ``decode_streams``; the rows each
+    stream sees are gathered block by block and attended in fp64 with ``decode_f64``."""
+    sp, sh, pl = decode_streams(pages, layout_streams)
+    pk_ = np.asarray(pool_k, np.float64) if not hasattr(pool_k, "numpy") else pool_k.double().numpy()
+    pv_ = np.asarray(pool_v, np.float64) if not hasattr(pool_v, "numpy") else pool_v.double().numpy()
+    pt, st = np.asarray(page_table), np.asarray(stream_table)
+
+    def rows(pool, table_row, n):
+        out = [pool[int(table_row[t // block_size]), :, t % block_size, :] for t in range(n)]
+        return np.stack(out) if out else np.zeros((0,) + pool.shape[1:2] + pool.shape[3:], np.float64)
+
+    plen = [(pg[0] + pg[1]) if isinstance(pg, tuple) else pg.prefix_len + pg.layout_len for pg in pages]
+    page_off = np.concatenate([[0], np.cumsum(plen)[:-1]]).astype(np.int64)
+    priv_off = np.concatenate([[0], np.cumsum(pl.astype(np.int64))[:-1]]).astype(np.int64) if len(pl) else np.zeros(0, np.int64)
+    sk = np.concatenate([rows(pk_, pt[p], plen[p]) for p in range(len(pages))]) if pages else np.zeros((0,))
+    sv = np.concatenate([rows(pv_, pt[p], plen[p]) for p in range(len(pages))]) if pages else np.zeros((0,))
+    prk = np.concatenate([rows(pk_, st[i], int(pl[i])) for i in range(len(pl))]) if len(pl) else np.zeros((0,))
+    prv = np.concatenate([rows(pv_, st[i], int(pl[i])) for i in range(len(pl))]) if len(pl) else np.zeros((0,))
+    return decode_f64(sp, sh, pl, page_off, priv_off, sk, sv, prk, prv, q, scale)

@@ -360,6 +360,70 @@ void oracle_decode(int32_t num_streams, const int32_t *stream_page, const int32_
     }
 }
 
+/* The same decode step over fp64 K/V rows (a dequantized cache, whose values code_value * scale
+ * need more bits than fp32 holds); q stays fp32. Arguments as oracle_decode. */
+static double attend_rows_f64(const float *q, const double *const *k_rows, const double *const *v_rows, int64_t nk,
+                              int d, double scale, double *s_buf, double *o)
+{
+    for (int c = 0; c < d; ++c) o[c] = 0.0;
+    if (nk == 0) return -INFINITY;
+    double mx = -INFINITY;
+    for (int64_t j = 0; j < nk; ++j) {
+        double acc = 0.0;
+        for (int c = 0; c < d; ++c) acc += (double)q[c] * k_rows[j][c];
+        s_buf[j] = scale * acc;
+        if (s_buf[j] > mx) mx = s_buf[j];
+    }
+    double sum = 0.0;
+    for (int64_t j = 0; j < nk; ++j) sum += exp(s_buf[j] - mx);
+    const double lse = mx + log(sum);
+    for (int64_t j = 0; j < nk; ++j) {
+        const double w = exp(s_buf[j] - lse);
+        for (int c = 0; c < d; ++c) o[c] += w * v_rows[j][c];
+    }
+    return lse;
+}
+
+void oracle_decode_f64(int32_t num_streams, const int32_t *stream_page, const int32_t *shared_len,
+                       const int32_t *priv_len, const int64_t *page_off, const int64_t *priv_off,
+                       const double *stream_k, const double *stream_v, const double *priv_k, const double *priv_v,
+                       const float *q, int32_t Hq, int32_t Hkv, int32_t d, double scale, double *o, double *lse)
+{
+    const int group = Hq / Hkv;
+#pragma omp parallel
+    {
+        int64_t cap = 0;
+        const double **kr = NULL, **vr = NULL;
+        double *sb = NULL;
+#pragma omp for schedule(dynamic, 1) collapse(2)
+        for (int s = 0; s < num_streams; ++s) {
+            for (int h = 0; h < Hq; ++h) {
+                const int g = h / group;
+                const int64_t nk = (int64_t)shared_len[s] + priv_len[s];
+                if (nk > cap) {
+                    cap = nk;
+                    kr = (const double **)realloc((void *)kr, sizeof(double *) * (size_t)cap);
+                    vr = (const double **)realloc((void *)vr, sizeof(double *) * (size_t)cap);
+                    sb = (double *)realloc(sb, sizeof(double) * (size_t)cap);
+                }
+                int64_t c = 0;
+                const int64_t po = page_off[stream_page[s]];
+                for (int64_t j = 0; j < shared_len[s]; ++j, ++c) {
+                    kr[c] = stream_k + ((po + j) * Hkv + g) * d;
+                    vr[c] = stream_v + ((po + j) * Hkv + g) * d;
+                }
+                for (int64_t j = 0; j < priv_len[s]; ++j, ++c) {
+                    kr[c] = priv_k + ((priv_off[s] + j) * Hkv + g) * d;
+                    vr[c] = priv_v + ((priv_off[s] + j) * Hkv + g) * d;
+                }
+                const int64_t row = (int64_t)s * Hq + h;
+                lse[row] = attend_rows_f64(q + row * d, kr, vr, nk, d, scale, sb, o + row * d);
+            }
+        }
+        free((void *)kr); free((void *)vr); free(sb);
+    }
+}
+
 /* ------------------------------------------------------------------------------------------ */
 /* Merge of partial softmax results over a partition of the visible set                         */
 /* ------------------------------------------------------------------------------------------ */
@@ -671,8 +735,11 @@ void oracle_e4m3_decode(const uint8_t *codes, int64_t n, double *x)
 }
 
 /* Quantizes a pool [num_blocks][hkv][bs][d] of fp32 K or V: per (block, head) the scale is
- * amax / 448 in fp32 (1 for an all-zero block) and each element's code is the E4M3 code of
- * x / scale, the division taken in fp32, the precision a kernel that quantizes on write uses. */
+ * amax / 448 in fp32 and each element's code is the E4M3 code of x / scale, the division taken in
+ * fp32, the precision a kernel that quantizes on write uses. An all-zero (block, head) gets scale 0
+ * and codes 0: a zero scale marks a (block, head) that holds no nonzero value, the state the
+ * row-by-row append below starts from, so a block quantized whole and then extended row by row
+ * follows one rule. */
 void oracle_quantize_kv_blocks(const float *x, int64_t num_blocks, int32_t hkv, int32_t bs, int32_t d, uint8_t *codes,
                                float *scales)
 {
@@ -681,11 +748,63 @@ void oracle_quantize_kv_blocks(const float *x, int64_t num_blocks, int32_t hkv, 
         const float *src = x + u * per;
         float amax = 0.0f;
         for (int64_t i = 0; i < per; ++i) amax = fmaxf(amax, fabsf(src[i]));
-        const float scale = amax > 0.0f ? amax / 448.0f : 1.0f;
+        const float scale = amax / 448.0f;
         scales[u] = scale;
         for (int64_t i = 0; i < per; ++i) {
+            if (scale == 0.0f) { codes[u * per + i] = 0; continue; }
             const float y = src[i] / scale;
             codes[u * per + i] = oracle_e4m3_encode_one((double)y);
+        }
+    }
+}
+
+/* Appends rows to a quantized pool one at a time, in the order given, as a decoding loop writes
+ * its cache (Algorithm 1 appends one input per live stream per step). Row i, for every KV head g,
+ * goes to block b = slots[i] / bs, row r = slots[i] % bs:
+ *   1. a = max_c |x_c| over the new row (fp32); s_old = the block's scale, taken as 0 when r = 0
+ *      (a block's first row starts it afresh: a block handed out again keeps a former owner's
+ *      scale and rows, which no one reads);
+ *   2. s_new = max(s_old, a / 448), the division in fp32: the scale stays amax / 448 over the rows
+ *      written so far;
+ *   3. if s_new > s_old > 0, each earlier row r' < r is re-encoded against the new scale: the value
+ *      its code stood for, code_value * s_old (fp32 product), divided by s_new (fp32), is encoded
+ *      again (nearest even, saturating);
+ *   4. the new row's codes are the codes of x_c / s_new (fp32 division), or 0 when s_new = 0;
+ *   5. the block's scale becomes s_new.
+ * Rows r' > r are left as they are. rows: [count][hkv][d] fp32; codes [num_blocks][hkv][bs][d];
+ * scales [num_blocks][hkv]. */
+void oracle_append_kv_quantized(uint8_t *codes, float *scales, int64_t num_blocks, int32_t hkv, int32_t bs, int32_t d,
+                                const int32_t *slots, int32_t count, const float *rows)
+{
+    for (int32_t i = 0; i < count; ++i) {
+        const int64_t b = slots[i] / bs;
+        const int32_t r = slots[i] % bs;
+        if (b < 0 || b >= num_blocks) continue;
+        for (int32_t g = 0; g < hkv; ++g) {
+            const float *x = rows + ((int64_t)i * hkv + g) * d;
+            uint8_t *blk = codes + (b * hkv + g) * (int64_t)bs * d;
+            float *sc = scales + b * hkv + g;
+            float a = 0.0f;
+            for (int32_t c = 0; c < d; ++c) a = fmaxf(a, fabsf(x[c]));
+            const float s_old = r == 0 ? 0.0f : *sc;
+            const float cand = a / 448.0f;
+            const float s_new = cand > s_old ? cand : s_old;
+            if (s_new > s_old && s_old > 0.0f) {
+                for (int32_t rr = 0; rr < r; ++rr)
+                    for (int32_t c = 0; c < d; ++c) {
+                        uint8_t *cp = blk + (int64_t)rr * d + c;
+                        const float y = (float)oracle_e4m3_value(*cp) * s_old;
+                        const float z = y / s_new;
+                        *cp = oracle_e4m3_encode_one((double)z);
+                    }
+            }
+            for (int32_t c = 0; c < d; ++c) {
+                uint8_t *cp = blk + (int64_t)r * d + c;
+                if (s_new == 0.0f) { *cp = 0; continue; }
+                const float z = x[c] / s_new;
+                *cp = oracle_e4m3_encode_one((double)z);
+            }
+            *sc = s_new;
         }
     }
 }

@@ -594,7 +594,7 @@ def test_quantize_kv_blocks_scale_bound_and_exact_values():
     """Per (block, head): the largest magnitude maps to 448; every element is within half a code step
     of its value (relative 2^-4 for normal codes, 2^-10 * scale below the normal range); a block
     whose values are already codes times a power-of-two scale comes back exactly; a zero block
-    keeps scale 1 and codes 0."""
+    gets scale 0 (no nonzero value yet) and codes 0."""
     rng = np.random.default_rng(1)
     x = rng.standard_normal((6, 2, 16, 128)).astype(np.float32) * rng.uniform(0.01, 50, (6, 2, 1, 1)).astype(np.float32)
     x[5, 1] = 0.0
@@ -604,7 +604,7 @@ def test_quantize_kv_blocks_scale_bound_and_exact_values():
         for h in range(2):
             blk, s = x[b, h].astype(np.float64), float(scales[b, h])
             if b == 5 and h == 1:
-                assert s == 1.0 and not codes[b, h].any()
+                assert s == 0.0 and not codes[b, h].any()
                 continue
             assert np.isclose(s, np.float32(np.abs(x[b, h]).max() / np.float32(448.0)), rtol=0, atol=0)
             assert np.abs(oracle.e4m3_decode(codes[b, h])).max() == 448.0
@@ -618,3 +618,125 @@ def test_quantize_kv_blocks_scale_bound_and_exact_values():
     codes2, scales2 = oracle.quantize_kv_blocks(exact)
     assert scales2[0, 0] == np.float32(2.0 ** -3)
     np.testing.assert_array_equal(oracle.dequantize_kv_blocks(codes2, scales2), exact.astype(np.float64))
+
+
+# ------------------------------------------------------------------------------------------------
+# FP8 (E4M3) cache written row by row (a decoding loop's append)
+# ------------------------------------------------------------------------------------------------
+
+def _rows_into_block(rows, bs=16):
+    """slots 0 .. n-1 of block 0 and the rows as [n][Hkv][d]"""
+    return np.arange(len(rows), dtype=np.int32), np.ascontiguousarray(rows, np.float32)
+
+
+def test_append_rows_equal_whole_block_quantization_when_the_first_row_holds_the_max():
+    # the scale never grows after row 0, so no row is re-encoded: every row's codes are those of
+    # the whole block quantized at once (itself pinned against torch's float8_e4m3fn)
+    rng = np.random.default_rng(3)
+    x = rng.standard_normal((1, 2, 16, 64)).astype(np.float32)
+    x[0, :, 0, 5] = 9.0          # row 0 of each head holds the block's largest magnitude
+    x[0, 1, 0, 7] = -11.0
+    want_c, want_s = oracle.quantize_kv_blocks(x)
+    c0 = np.zeros_like(want_c)
+    s0 = np.zeros_like(want_s)
+    slots, rows = _rows_into_block(x[0].transpose(1, 0, 2))
+    got_c, got_s = oracle.append_kv_quantized(c0, s0, slots, rows)
+    np.testing.assert_array_equal(got_s, want_s)
+    np.testing.assert_array_equal(got_c, want_c)
+
+
+def test_append_scale_is_amax_over_rows_so_far_and_power_of_two_growth_is_exact():
+    # rows 0..3 each double the block's largest magnitude (scales 2^-2 .. 2^1, exact in fp32), with
+    # every value a normal code times its row's scale, at least 2^-2 of a unit: every re-encoding
+    # divides by exactly 2 and stays in the normal range, so after all appends the dequantized block
+    # is the written rows exactly; the scale after row r is amax(rows <= r) / 448 (the whole-block
+    # quantizer's scale of the block truncated to those rows).
+    rng = np.random.default_rng(4)
+    d = 32
+    normal = oracle.e4m3_decode(np.arange(0x28, 0x7F, dtype=np.uint8))      # codes 0.25 .. 448
+    rows = np.zeros((16, 1, d), np.float32)
+    for r in range(16):
+        s_r = 2.0 ** (min(r, 3) - 2)
+        vals = rng.choice(normal[normal <= 448.0 / (2.0 if r > 3 else 1.0)], size=d) * rng.choice([-1, 1], size=d)
+        vals[rng.integers(0, d)] = 0.0
+        if r <= 3:
+            vals[0] = 448.0
+        rows[r, 0] = (vals * s_r).astype(np.float32)
+    c = np.zeros((1, 1, 16, d), np.uint8)
+    s = np.zeros((1, 1), np.float32)
+    for r in range(16):
+        c, s = oracle.append_kv_quantized(c, s, [r], rows[r:r + 1])
+        trunc = np.zeros((1, 1, 16, d), np.float32)
+        trunc[0, 0, :r + 1] = rows[:r + 1, 0]
+        assert s[0, 0] == oracle.quantize_kv_blocks(trunc)[1][0, 0]
+    assert s[0, 0] == 2.0
+    np.testing.assert_array_equal(oracle.dequantize_kv_blocks(c, s)[0, 0], rows[:, 0].astype(np.float64))
+
+
+def test_append_re_encoding_stays_within_the_accumulated_rounding_bound():
+    # each re-encoding moves a value by at most half a code step at the new scale (relative 2^-4 in
+    # the normal range, 2^-10 * scale below it) plus fp32 roundings; a row re-encoded k times is
+    # within k + 1 such steps of its value at the final scale
+    rng = np.random.default_rng(5)
+    d = 128
+    rows = (rng.standard_normal((16, 2, d)) * np.exp(rng.uniform(-2, 2, (16, 2, 1)))).astype(np.float32)
+    c = np.zeros((1, 2, 16, d), np.uint8)
+    s = np.zeros((1, 2), np.float32)
+    grown = np.zeros((16, 2), np.int64)
+    for r in range(16):
+        s_before = s.copy()
+        c, s = oracle.append_kv_quantized(c, s, [r], rows[r:r + 1])
+        for g in range(2):
+            if r > 0 and s[0, g] > s_before[0, g]:
+                grown[:r, g] += 1
+    deq = oracle.dequantize_kv_blocks(c, s)
+    for g in range(2):
+        sf = float(s[0, g])
+        x = rows[:, g].astype(np.float64)
+        step = np.where(np.abs(x) >= 2.0 ** -6 * sf, 2.0 ** -4 * np.abs(x) * 1.07, 2.0 ** -10 * sf)
+        bound = (grown[:, g, None] + 1) * step + 1e-7 * sf
+        assert np.all(np.abs(deq[0, g] - x) <= bound)
+        assert sf == np.float32(np.abs(rows[:, g]).max()) / np.float32(448.0)
+
+
+def test_append_row_zero_starts_a_reused_block_afresh_and_zero_rows_keep_scale_zero():
+    rng = np.random.default_rng(6)
+    d = 16
+    # a block handed out again: stale codes and scale from a former owner
+    c = rng.integers(0, 0x7E, (2, 1, 16, d)).astype(np.uint8)
+    s = np.array([[3.5], [0.25]], np.float32)
+    x = rng.standard_normal((1, 1, d)).astype(np.float32)
+    c2, s2 = oracle.append_kv_quantized(c, s, [16], x)          # block 1, row 0
+    assert s2[1, 0] == np.float32(np.abs(x).max()) / np.float32(448.0)
+    np.testing.assert_array_equal(c2[1, 0, 1:], c[1, 0, 1:])    # later rows untouched
+    np.testing.assert_array_equal(c2[0], c[0])                  # other blocks untouched
+    ref = torch.from_numpy(x[0, 0] / s2[1, 0]).to(torch.float8_e4m3fn).view(torch.uint8).numpy()
+    np.testing.assert_array_equal(c2[1, 0, 0], ref)
+    # zero rows: the scale stays 0 and the codes 0 until a nonzero row arrives, which does not
+    # touch them
+    c = np.zeros((1, 1, 16, d), np.uint8)
+    s = np.zeros((1, 1), np.float32)
+    c, s = oracle.append_kv_quantized(c, s, [0, 1, 2], np.zeros((3, 1, d), np.float32))
+    assert s[0, 0] == 0.0 and not c.any()
+    c, s = oracle.append_kv_quantized(c, s, [3], x)
+    assert s[0, 0] == np.float32(np.abs(x).max()) / np.float32(448.0) and not c[0, 0, :3].any()
+
+
+def test_decode_f64_and_paged_decode_equal_the_fp32_row_decode():
+    # the fp64-row decode is the same arithmetic as oracle.decode on fp32-exact rows, and the paged
+    # form, which gathers each stream's rows through the block tables, reads exactly those rows
+    from paper_2608_06146_gb300 import inputs
+    pages = [inputs.PageSpec(40, 9, [0, 9, 4], [3, 20, 17]), inputs.PageSpec(5, 16, [16, 2], [1, 33])]
+    wl = inputs.Workload("pin", pages, 8, 2, 16, torch.bfloat16, "decode")
+    di = inputs.decode_inputs(wl, 9, layout_streams=True)
+    o32, l32 = oracle.decode_pages(pages, di, 0.3, layout_streams=True)
+    sp, sh, pl = oracle.decode_streams(pages, layout_streams=True)
+    f64 = lambda t: t.double().numpy()
+    o64, l64 = oracle.decode_f64(sp, sh, pl, di.page_off, di.priv_off, f64(di.stream_k), f64(di.stream_v),
+                                 f64(di.priv_k), f64(di.priv_v), di.q, 0.3)
+    np.testing.assert_array_equal(o64, o32)
+    np.testing.assert_array_equal(l64, l32)
+    op, lp = oracle.decode_paged(pages, di.k_pool, di.v_pool, di.page_table, di.stream_table, di.q, 0.3,
+                                 layout_streams=True)
+    np.testing.assert_array_equal(op, o32)
+    np.testing.assert_array_equal(lp, l32)
