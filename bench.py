@@ -335,6 +335,48 @@ def bench_decode(args, torch, dev, rank, world, layout_streams=False):
     return res
 
 
+def bench_decode_e4m3(args, torch, dev, rank, world):
+    """The serving-batch decode step over the FP8 (E4M3) cache: the same pages, plan and queries, the
+    pool quantized from the bf16 one (whole blocks) in R replicas in distinct memory."""
+    from paper_2608_06146_gb300 import inputs
+    from paper_2608_06146_gb300 import padoc_attn as pa
+    from paper_2608_06146_gb300.engine import DecodePlan
+
+    wl = inputs.serving_batch(seed=3 + 1000 * rank)
+    scale = 1.0 / math.sqrt(wl.head_dim)
+    di = inputs.decode_inputs(wl, 3 + 1000 * rank, pool_slack=1.0)
+    plan = DecodePlan(wl.pages, wl.num_q_heads, wl.num_kv_heads, wl.head_dim, dev, tc_ctas=args.tc_ctas,
+                      warp_ctas=args.warp_ctas, split_tokens=args.split_tokens)
+    S = plan.num_streams
+    per_replica = di.k_pool.numel() * 2 + di.num_blocks * wl.num_kv_heads * 8
+    R = max(2, math.ceil(4 * l2_bytes(torch) / per_replica) + 1)
+    k_bf, v_bf = di.k_pool.to(dev), di.v_pool.to(dev)
+    blocks = torch.arange(di.num_blocks, dtype=torch.int32, device=dev)
+    pools = []
+    for _ in range(R):
+        pool = pa.E4M3Pool(di.num_blocks, wl.num_kv_heads, wl.head_dim, dev)
+        pa.padoc_quantize_kv_blocks(pool, k_bf, v_bf, blocks)
+        pools.append(pool)
+    del k_bf, v_bf
+    qs = [di.q.to(dev) for _ in range(R)]
+    page_table = torch.from_numpy(di.page_table).to(dev)
+    stream_table = torch.from_numpy(di.stream_table).to(dev)
+    outs = [torch.empty((S, wl.num_q_heads, wl.head_dim), dtype=torch.bfloat16, device=dev) for _ in range(R)]
+    lses = [torch.empty((S, wl.num_q_heads), dtype=torch.float32, device=dev) for _ in range(R)]
+    stream = torch.cuda.current_stream()
+
+    def step(i, s):
+        r = i % R
+        pa.padoc_branch_decode_attn_e4m3(pools[r], plan.info, plan.plan_dev, page_table, stream_table, qs[r], scale,
+                                         outs[r], lses[r], plan.workspace, s)
+
+    timing = time_steps(args, torch, world, stream, step, steady=False)
+    info = plan.info
+    launches = (1 if info.num_tc_items > 0 else 0) + (1 if info.num_warps > 0 else 0) + 1
+    return dict(ms=timing["ms"], streams=S, bytes=decode_bytes(wl, kv_bytes=1, scale_bytes=4), launches=launches,
+                clocks=timing["clocks"], replicas=R)
+
+
 def bench_prefill(args, torch, dev, rank, world, shuffle=False):
     """The packed prefill of 8 pages x 4096 tokens (with ``shuffle``, each page's branches permuted
     so that the fork offsets are not monotone in the branch index)."""
@@ -702,7 +744,7 @@ def main():
     ap.add_argument("--impl", default="padoc", choices=["padoc", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--only", default="all", choices=["all", "decode", "prefill", "prefill_bwd", "loop",
-                                                      "chunk_prefill", "variants"])
+                                                      "chunk_prefill", "variants", "decode_e4m3"])
     ap.add_argument("--replicas", type=int, default=0, help="decode input replicas (0: enough to exceed 4x L2)")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-steady", action="store_true", help="skip the long back-to-back decode run")
@@ -739,6 +781,12 @@ def main():
             print(json.dumps({"decode_with_layout_streams_us": a["ms"] * 1e3, "streams": a["streams"],
                               "prefill_shuffled_ms": b["ms"], "prefill_shuffled_tflops": b["flops"] / (b["ms"] * 1e-3) / 1e12}))
         return 0
+    if args.only == "decode_e4m3":
+        e = bench_decode_e4m3(args, torch, dev, rank, world)
+        if rank == 0:
+            print(json.dumps({"decode_e4m3_us": e["ms"] * 1e3, "queries_per_s": e["streams"] / (e["ms"] * 1e-3),
+                              "hbm_gbs": e["bytes"] / (e["ms"] * 1e-3) / 1e9, "bytes": e["bytes"]}))
+        return 0
     if args.only == "loop":
         lp = bench_loop(args, torch, dev, rank, world)
         if rank == 0:
@@ -764,6 +812,7 @@ def main():
             return {"error": f"{type(e).__name__}: {e}"[:300]}
 
     dl = None if args.only == "decode" else variant(bench_decode, layout_streams=True)
+    d8 = None if args.only == "decode" else variant(bench_decode_e4m3)
     ps = None if args.only == "decode" else variant(bench_prefill, shuffle=True)
     cp = None if args.only == "decode" else variant(bench_chunk_prefill)
     lp = None if args.only == "decode" else variant(bench_loop)
@@ -840,6 +889,22 @@ def main():
                             "(branches + layout streams; the headline counts branches only)",
                 "roofline": {"bound": "hbm", "achieved": ach, "peak": peaks["hbm_gbs"], "unit": "GB/s",
                              "frac": ach / peaks["hbm_gbs"], "traffic": None, "algorithmic_bytes": dl["bytes"]}}
+    if d8 is not None and "error" in d8:
+        line["decode_e4m3"] = d8
+    elif d8 is not None:
+        ems = max_over_ranks(torch, world, d8["ms"])
+        ach = d8["bytes"] / (d8["ms"] * 1e-3) / 1e9
+        line["decode_e4m3"] = {
+            "value": d8["streams"] * world / (ems * 1e-3), "unit": "queries/s", "ms_per_step": ems,
+            "streams_per_gpu": d8["streams"], "replicas": d8["replicas"], "clocks": d8["clocks"],
+            "workload": "the serving-batch decode step over the FP8 (E4M3) KV cache (codes + one fp32 scale per "
+                        "(block, KV head)), quantized from the same bf16 cache",
+            "roofline": {"bound": "hbm", "achieved": ach, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                         "frac": ach / peaks["hbm_gbs"], "traffic": None,
+                         "algorithmic_bytes": d8["bytes"],
+                         "bytes_rule": "each page's visible shared stream once and every private row once at 1 byte "
+                                       "per K/V element, plus a 4-byte K and V scale per (16-token block, KV head), Q "
+                                       "in, O and LSE out"}}
     if ps is not None and p is not None:
         if "error" in ps:
             line["prefill"]["shuffled_branches"] = ps

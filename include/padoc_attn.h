@@ -47,8 +47,10 @@ extern "C" {
 #endif
 
 /* 1: descriptors, decode, prefill, combine, prefill backward, no-alloc decode. 2 adds the
- * stream-list and chunked-prefill planners, Algorithm 1's loop (padoc_mpd_*) and the append call. */
-#define PADOC_ATTN_VERSION 2
+ * stream-list and chunked-prefill planners, Algorithm 1's loop (padoc_mpd_*) and the append call.
+ * 3 adds the FP8 (E4M3) KV cache (padoc_kv_pool_e4m3 and its quantize, append and decode calls)
+ * and the bounded-wait self-test. */
+#define PADOC_ATTN_VERSION 3
 
 /* A CUDA stream handle; identical to cudaStream_t. */
 typedef struct CUstream_st *padoc_stream_t;
@@ -307,6 +309,66 @@ padoc_status padoc_branch_decode_attn_noalloc(const padoc_kv_pool *pool, const p
 padoc_status padoc_splitk_combine(const float *part_o, const float *part_lse, int32_t num_splits, int64_t rows,
                                   int32_t head_dim, padoc_dtype out_dtype, void *out, float *lse,
                                   padoc_stream_t stream);
+
+/* ============================================================================================
+ * FP8 (E4M3) variant of the paged KV cache (C5) and of the decode step (C2)
+ * ========================================================================================== */
+
+/* The paper serves a bf16 cache (Sec. 4 serving setup); this variant halves the bytes a decode
+ * step reads. K and V are stored as E4M3 codes (the OCP 8-bit format: 4 exponent bits with bias 7,
+ * 3 mantissa bits, largest finite 448) with one fp32 scale per (block, KV head); an element's value
+ * is code_value * scale. The scale is amax / 448 over the rows the block holds (0 while it holds no
+ * nonzero value), so a block's largest magnitude maps to 448. Layouts as padoc_kv_pool:
+ *   k_codes, v_codes:   (device) uint8 [num_blocks][num_kv_heads][block_size][head_dim], 16-byte aligned
+ *   k_scales, v_scales: (device) fp32 [num_blocks][num_kv_heads]
+ * Supported: block_size 16, head_dim 128. */
+typedef struct {
+    const void *k_codes;
+    const void *v_codes;
+    const float *k_scales;
+    const float *v_scales;
+    int32_t num_blocks;
+    int32_t block_size;
+    int32_t num_kv_heads;
+    int32_t head_dim;
+} padoc_kv_pool_e4m3;
+
+/* Quantizes whole blocks (a page's prefix after its prefill): (block i, head g) of k_src / v_src
+ * ((device) bf16 [count][num_kv_heads][block_size][head_dim]) becomes (block dst_blocks[i], head g)
+ * of the pool: scale = amax / 448 (fp32), code = the E4M3 code of x / scale (fp32 division,
+ * nearest even, saturating at 448); an all-zero one gets scale 0 and codes 0. dst_blocks: (device)
+ * int32 [count]; an id out of range sets the device error word (code 1) and that block is skipped.
+ * Errors: INVALID_ARGUMENT, UNSUPPORTED, CUDA. */
+padoc_status padoc_quantize_kv_blocks(const padoc_kv_pool_e4m3 *pool, const void *k_src, const void *v_src,
+                                      const int32_t *dst_blocks, int32_t count, padoc_stream_t stream);
+
+/* padoc_append_inputs for an E4M3 pool (Algorithm 1's append; sources bf16 [src_total][Hkv][d],
+ * queries bf16 as there). Input i goes to row r = slots[i] % block_size of block
+ * slots[i] / block_size, every KV head, by the scale rule: the block's scale becomes
+ * max(old scale, amax(row) / 448), the old scale taken as 0 when r = 0 (a block's first row starts
+ * it afresh; a block handed out again keeps a former owner's scale and rows, which no one reads);
+ * when the scale grows from a nonzero old scale, rows 0 .. r-1 are re-encoded (code value x old
+ * scale, divided by the new scale, each step rounded to fp32, then encoded nearest even); the row's
+ * codes are those of x / new scale. Rows past r are left as they are. The inputs of one call must
+ * lie in distinct blocks (Algorithm 1 appends one input per stream, each stream to its own
+ * blocks); two inputs in one block race. Errors: INVALID_ARGUMENT, UNSUPPORTED, CUDA. */
+padoc_status padoc_append_inputs_e4m3(const padoc_kv_pool_e4m3 *pool, const void *k_src, const void *v_src,
+                                      const void *q_src, int64_t src_total, int32_t num_q_heads, void *q_dst,
+                                      const int32_t *src_rows, const int32_t *slots, int32_t count,
+                                      padoc_stream_t stream);
+
+/* padoc_branch_decode_attn over an E4M3 pool: the same plans (padoc_build_decode_plan and the other
+ * planners, built with the same padoc_decode_config), tables, workspace and results; q, out bf16
+ * [num_streams][Hq][128], lse fp32. Attention is over the dequantized values code_value * scale:
+ * codes become bf16 exactly in shared memory, the K scale multiplies each 16-token block's scores
+ * and the V scale the block's probabilities in fp32 before they are rounded to bf16. Hq / Hkv = 8,
+ * block_size 16, head_dim 128. Errors: INVALID_ARGUMENT, UNSUPPORTED, WORKSPACE_TOO_SMALL, CUDA. */
+padoc_status padoc_branch_decode_attn_e4m3(const padoc_kv_pool_e4m3 *pool, const padoc_decode_plan *info,
+                                           const int32_t *plan_dev, const int32_t *page_block_table,
+                                           int32_t page_table_stride, const int32_t *stream_block_table,
+                                           int32_t stream_table_stride, const void *q, float scale, void *out,
+                                           float *lse, void *workspace, size_t workspace_bytes,
+                                           padoc_stream_t stream);
 
 /* ============================================================================================
  * Branch prefill over the paged cache: chunks of several query tokens per stream

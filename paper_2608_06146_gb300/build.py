@@ -13,7 +13,7 @@ INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(BUILD, "libpadoc_attn.so")
 SOURCES = ["plan.cpp", "api.cu", "decode.cu", "prefill.cu", "prefill_tc.cu", "prefill_bwd.cu", "prefill_bwd_tc.cu",
-           "decode_tc.cu", "tc_selftest.cu", "mpd.cpp", "append.cu"]
+           "decode_tc.cu", "tc_selftest.cu", "mpd.cpp", "append.cu", "e4m3.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

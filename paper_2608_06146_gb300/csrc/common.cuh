@@ -4,6 +4,7 @@
 
 #include <cuda.h>
 #include <cuda_bf16.h>
+#include <cuda_fp16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -193,6 +194,11 @@ __device__ __forceinline__ void cp_async_16_hint(uint32_t dst, const void *src, 
                  "l"(policy)
                  : "memory");
 }
+// 4 bytes through L1 (cp.async of fewer than 16 bytes takes the .ca form); src_bytes 0 writes zeros.
+__device__ __forceinline__ void cp_async_4(uint32_t dst, const void *src, uint32_t src_bytes)
+{
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;" ::"r"(dst), "l"(src), "r"(src_bytes) : "memory");
+}
 __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
 template <int N>
 __device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
@@ -255,6 +261,46 @@ __device__ __forceinline__ float fast_exp2(float x)
     return y;
 }
 
+// ------------------------------------------------------------------------------------------------
+// E4M3 (the OCP 8-bit floating point format, 4 exponent bits with bias 7, 3 mantissa bits, no
+// infinities, largest finite 448) conversions of the FP8 KV cache.
+// ------------------------------------------------------------------------------------------------
+// Two codes (low byte first) to an f16x2: exact (every E4M3 value is an f16 normal or zero).
+__device__ __forceinline__ uint32_t e4m3x2_to_f16x2(uint16_t c)
+{
+    uint32_t h;
+    asm("cvt.rn.f16x2.e4m3x2 %0, %1;" : "=r"(h) : "h"(c));
+    return h;
+}
+
+// Two codes to a bf16x2 holding code_value * 2^-112, exactly: the f16 bits with the exponent and
+// the top 7 mantissa bits moved down three places (E4M3 values use only the top 3 of f16's 10
+// mantissa bits) read as bf16 with exponent field 0..23 instead of f16's biased exponent, i.e.
+// the value times 2^(15 - 127); every nonzero result is a bf16 normal (no subnormal operand
+// reaches the tensor cores). Callers fold 2^112 into the scale they apply.
+#define PADOC_E4M3_BF16_SHIFT_LOG2 112
+__device__ __forceinline__ uint32_t e4m3x2_to_bf16x2_shifted(uint16_t c)
+{
+    const uint32_t h = e4m3x2_to_f16x2(c);
+    const uint32_t mag = (h & 0x7FFF7FFFu) >> 3;   // the high half's low mantissa bits are zero
+    return mag | (h & 0x80008000u);
+}
+
+// The exact fp32 value of one code.
+__device__ __forceinline__ float e4m3_to_f32(uint8_t c)
+{
+    const uint32_t h = e4m3x2_to_f16x2((uint16_t)c);
+    return __half2float(__ushort_as_half((unsigned short)(h & 0xFFFFu)));
+}
+
+// Codes of two fp32 values (lo -> low byte), nearest even, magnitudes past 448 saturated to 448.
+__device__ __forceinline__ uint16_t f32x2_to_e4m3x2(float lo, float hi)
+{
+    uint16_t c;
+    asm("cvt.rn.satfinite.e4m3x2.f32 %0, %1, %2;" : "=h"(c) : "f"(hi), "f"(lo));
+    return c;
+}
+
 // Programmatic dependent launch: a grid lets the next grid in its stream start launching, and a
 // dependent grid waits until its prerequisite grid has completed and its writes are visible.
 // One 32-byte store of eight floats (p 32-byte aligned): a whole sector per lane.
@@ -287,6 +333,10 @@ int *padoc_device_error_word();
 // box_rows x 64 columns, 128-byte swizzle. Returns false if the driver rejects it.
 bool padoc_make_tmap_bf16(CUtensorMap *map, const void *base, uint64_t cols, uint64_t rows,
                           uint64_t row_stride_bytes, uint32_t box_cols, uint32_t box_rows);
+// 2-D uint8 tensor map (E4M3 codes): rows x cols bytes with a row pitch of `row_stride_bytes`, box of
+// box_rows x box_cols bytes (box_cols <= 128), 128-byte swizzle.
+bool padoc_make_tmap_u8(CUtensorMap *map, const void *base, uint64_t cols, uint64_t rows, uint64_t row_stride_bytes,
+                        uint32_t box_cols, uint32_t box_rows);
 // 4-D bf16 tensor map (dims[0] innermost, strides of dims 1..3 in bytes), 128-byte swizzle.
 bool padoc_make_tmap_bf16_4d(CUtensorMap *map, const void *base, const uint64_t dims[4], const uint64_t strides_bytes[3],
                              const uint32_t box[4]);
@@ -298,10 +348,12 @@ padoc_status padoc_launch_prefill_tc(const void *q, const void *k, const void *v
                                      const int8_t *tile_kind_dev, float scale_log2, void *out, float *lse,
                                      cudaStream_t stream);
 // tcgen05 shared-stream decode (decode_tc.cu): the plan's tensor-core items.
+// k_scales / v_scales non-null: an E4M3 pool (kmap / vmap are padoc_make_tmap_u8 maps of the codes).
 padoc_status padoc_launch_decode_tc(const CUtensorMap *kmap, const CUtensorMap *vmap, const CUtensorMap *qmap, const int32_t *plan,
                                     const padoc_decode_plan *info, const int32_t *page_table, int32_t page_stride,
-                                    const int32_t *stream_table, int32_t stream_stride, int32_t num_blocks, float *part_o, float *part_lse, float scale_log2, int *err,
-                                    cudaStream_t stream);
+                                    const int32_t *stream_table, int32_t stream_stride, int32_t num_blocks,
+                                    const float *k_scales, const float *v_scales, float *part_o, float *part_lse,
+                                    float scale_log2, int *err, cudaStream_t stream);
 // tcgen05 prefill backward (prefill_bwd_tc.cu): the dQ pass, which also writes lt / dt (per head
 // [Hq][t_pad]: -lse2 and rowsum(dO * O)), then the dK/dV pass; arguments validated by the caller.
 padoc_status padoc_launch_prefill_bwd_tc(const void *q, const void *k, const void *v, const void *out,

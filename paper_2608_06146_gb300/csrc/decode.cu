@@ -36,6 +36,15 @@ constexpr int kBoxBytes = kBlk * 128;  // one 16-row x 64-column box
 constexpr int kWStageBytes = 4 * kBoxBytes;   // K lo, K hi, V lo, V hi
 constexpr int kWarpRing = kWStages * kWStageBytes;
 constexpr size_t kDecodeSmem = 1024 + (size_t)kWarps * kWarpRing;
+// E4M3 pool: a stage holds a block's K and V codes ([16 rows][128 bytes] each, 16-byte chunks
+// swizzled by row) and its two scales; each warp expands the block it works on into one bf16
+// buffer laid out as a bf16 stage, which the MMAs read.
+constexpr int kE8Rows = kBlk * 128;                  // 2 KB of codes per tensor
+constexpr int kE8StageBytes = 2 * kE8Rows + 128;     // K codes, V codes, scales (k, v)
+constexpr int kE8WarpBytes = kWStages * kE8StageBytes + kWStageBytes;
+constexpr size_t kDecodeSmemE4M3 = 1024 + (size_t)kWarps * kE8WarpBytes;
+constexpr float kTwo112 = 5.192296858534828e33f;     // 2^112: the bf16 expansion's factor
+static_assert(PADOC_E4M3_BF16_SHIFT_LOG2 == 112, "expansion factor");
 
 struct DecodeParams {
     const int32_t *stream_page, *shared_len, *private_len, *slot_ptr;
@@ -49,6 +58,8 @@ struct DecodeParams {
     int32_t num_blocks, num_kv_heads, num_q_heads, pool_rows;
     int32_t after_tc;    // launched as a programmatic dependent of the tensor-core grid
     const __nv_bfloat16 *k_pool, *v_pool;
+    const uint8_t *k_codes, *v_codes;     // E4M3 pool (k_pool / v_pool unused)
+    const float *k_scales, *v_scales;
     const __nv_bfloat16 *q;
     float *part_o, *part_lse;
     float scale_log2;
@@ -62,6 +73,7 @@ __device__ __forceinline__ void finish_warp(const DecodeParams &prm)
     if (prm.after_tc) pdl_wait_prerequisite();
 }
 
+template <bool kE4M3>
 __global__ void __launch_bounds__(kWarps * 32, 1)
 decode_warp_kernel(const DecodeParams prm)
 {
@@ -77,7 +89,8 @@ decode_warp_kernel(const DecodeParams prm)
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int wi = blockIdx.x * kWarps + warp;
     if (wi >= prm.num_warps) { finish_warp(prm); return; }   // warps are independent: no CTA barrier follows
-    uint8_t *wbuf = smem + (size_t)warp * kWarpRing;
+    uint8_t *wbuf = smem + (size_t)warp * (kE4M3 ? kE8WarpBytes : kWarpRing);
+    uint8_t *cbuf = wbuf + kWStages * kE8StageBytes;   // E4M3: the expanded bf16 block
     const padoc_item *items = prm.items + prm.first_item;
     const int i0 = prm.warp_ptr[wi], i1 = prm.warp_ptr[wi + 1];
     // Every global read the loop depends on is issued at least one item ahead: item headers two
@@ -128,15 +141,35 @@ decode_warp_kernel(const DecodeParams prm)
             const bool okid = id >= 0 && id < prm.num_blocks;
             if (!okid && lane == 0) padoc_record_error(prm.err, PADOC_DEVERR_BLOCK_ID, id);
             const size_t rowbase = okid ? ((size_t)id * prm.num_kv_heads + pc.g) * kBlk : 0;
-            const uint32_t base = smem_u32(wbuf + (ring % kWStages) * kWStageBytes);
+            if constexpr (kE4M3) {
+                // chunk q = lane + 32k of the block's 256 16-byte chunks of codes: tensor q / 128,
+                // row (q / 8) % 16, chunk q % 8 (swizzled by row); lanes 0 and 1 also copy the K and
+                // V scales of the (block, KV head) (zeros for a bad id, whose codes are zeros too)
+                const uint32_t base = smem_u32(wbuf + (ring % kWStages) * kE8StageBytes);
 #pragma unroll
-            for (int k = 0; k < 16; ++k) {
-                const int q = lane + 32 * k;
-                const int panel = q >> 7, r = (q >> 3) & 15, cc = q & 7;
-                const __nv_bfloat16 *src = (panel < 2 ? prm.k_pool : prm.v_pool) +
-                                           (rowbase + r) * kD + (panel & 1) * 64 + cc * 8;
-                cp_async_16_hint(base + panel * kBoxBytes + r * 128 + ((cc ^ (r & 7)) << 4), src, okid ? 16u : 0u,
-                                 kv_policy);
+                for (int k = 0; k < 8; ++k) {
+                    const int q = lane + 32 * k;
+                    const int tn = q >> 7, r = (q >> 3) & 15, cc = q & 7;
+                    const uint8_t *src = (tn == 0 ? prm.k_codes : prm.v_codes) + (rowbase + r) * kD + cc * 16;
+                    cp_async_16_hint(base + tn * kE8Rows + r * 128 + ((cc ^ (r & 7)) << 4), src, okid ? 16u : 0u,
+                                     kv_policy);
+                }
+                if (lane < 2) {
+                    const size_t si = okid ? (size_t)id * prm.num_kv_heads + pc.g : 0;
+                    cp_async_4(base + 2 * kE8Rows + lane * 4, (lane == 0 ? prm.k_scales : prm.v_scales) + si,
+                               okid ? 4u : 0u);
+                }
+            } else {
+                const uint32_t base = smem_u32(wbuf + (ring % kWStages) * kWStageBytes);
+#pragma unroll
+                for (int k = 0; k < 16; ++k) {
+                    const int q = lane + 32 * k;
+                    const int panel = q >> 7, r = (q >> 3) & 15, cc = q & 7;
+                    const __nv_bfloat16 *src = (panel < 2 ? prm.k_pool : prm.v_pool) +
+                                               (rowbase + r) * kD + (panel & 1) * 64 + cc * 8;
+                    cp_async_16_hint(base + panel * kBoxBytes + r * 128 + ((cc ^ (r & 7)) << 4), src, okid ? 16u : 0u,
+                                     kv_policy);
+                }
             }
             ++pb;
             ++ring;
@@ -185,7 +218,45 @@ decode_warp_kernel(const DecodeParams prm)
         for (int bi = 0; bi < nblk; ++bi, ++gc) {
             cp_async_wait<kWStages - 1>();   // block gc has landed (one group per block)
             __syncwarp();
-            const uint32_t base = smem_u32(wbuf + (gc % kWStages) * kWStageBytes);
+            // per block: the multiplier of the raw scores (scale in log2 units) and, for an E4M3
+            // pool, the factor folded into P (the V scale; both carry the expansion's 2^112)
+            float kmul = prm.scale_log2, vfac = 1.f;
+            uint32_t base;
+            if constexpr (kE4M3) {
+                const uint8_t *stg = wbuf + (gc % kWStages) * kE8StageBytes;
+                const float ks = *reinterpret_cast<const float *>(stg + 2 * kE8Rows);
+                const float vs = *reinterpret_cast<const float *>(stg + 2 * kE8Rows + 4);
+                // a zero scale marks a block without a nonzero value (its codes are all zero):
+                // any positive factor then gives the same scores and keeps masked ones at -inf
+                kmul = prm.scale_log2 * (ks > 0.f ? ks : 1.f) * kTwo112;
+                vfac = (vs > 0.f ? vs : 1.f) * kTwo112;
+                // lane l expands row l % 16 of tensor l / 16 (K, V) into the bf16 panels
+                const int tn = lane >> 4, r = lane & 15;
+                uint4 raw[8];
+#pragma unroll
+                for (int c = 0; c < 8; ++c)
+                    raw[c] = *reinterpret_cast<const uint4 *>(stg + tn * kE8Rows + r * 128 + ((c ^ (r & 7)) << 4));
+                __syncwarp();   // every lane has its row: the stage may be refilled
+                issue_next();
+#pragma unroll
+                for (int c = 0; c < 8; ++c) {
+                    const uint32_t w[4] = {raw[c].x, raw[c].y, raw[c].z, raw[c].w};
+#pragma unroll
+                    for (int hh = 0; hh < 2; ++hh) {   // dims 16c + 8hh .. + 7: bf16 chunk 2c + hh
+                        const int k = 2 * c + hh, panel = 2 * tn + (k >> 3), kk = k & 7;
+                        uint4 o;
+                        o.x = e4m3x2_to_bf16x2_shifted((uint16_t)(w[2 * hh] & 0xFFFFu));
+                        o.y = e4m3x2_to_bf16x2_shifted((uint16_t)(w[2 * hh] >> 16));
+                        o.z = e4m3x2_to_bf16x2_shifted((uint16_t)(w[2 * hh + 1] & 0xFFFFu));
+                        o.w = e4m3x2_to_bf16x2_shifted((uint16_t)(w[2 * hh + 1] >> 16));
+                        *reinterpret_cast<uint4 *>(cbuf + panel * kBoxBytes + r * 128 + ((kk ^ (r & 7)) << 4)) = o;
+                    }
+                }
+                __syncwarp();
+                base = smem_u32(cbuf);
+            } else {
+                base = smem_u32(wbuf + (gc % kWStages) * kWStageBytes);
+            }
             const int tokbase = (blk0 + bi) * kBlk;
             // S^T = K . Q^T, as two independent MMA chains (even / odd k-steps) added at the end
             float acc[4] = {0.f, 0.f, 0.f, 0.f}, acc2[4] = {0.f, 0.f, 0.f, 0.f};
@@ -201,10 +272,10 @@ decode_warp_kernel(const DecodeParams prm)
             for (int i = 0; i < 4; ++i) acc[i] += acc2[i];
             const int t0 = tokbase + (lane >> 2), t1 = t0 + 8;
             float sc[4];
-            sc[0] = t0 < cutoff ? acc[0] * prm.scale_log2 : -INFINITY;
-            sc[1] = t0 < cutoff ? acc[1] * prm.scale_log2 : -INFINITY;
-            sc[2] = t1 < cutoff ? acc[2] * prm.scale_log2 : -INFINITY;
-            sc[3] = t1 < cutoff ? acc[3] * prm.scale_log2 : -INFINITY;
+            sc[0] = t0 < cutoff ? acc[0] * kmul : -INFINITY;
+            sc[1] = t0 < cutoff ? acc[1] * kmul : -INFINITY;
+            sc[2] = t1 < cutoff ? acc[2] * kmul : -INFINITY;
+            sc[3] = t1 < cutoff ? acc[3] * kmul : -INFINITY;
             float mx0 = fmaxf(sc[0], sc[2]), mx1 = fmaxf(sc[1], sc[3]);
 #pragma unroll
             for (int sh = 4; sh < 32; sh <<= 1) {
@@ -221,8 +292,9 @@ decode_warp_kernel(const DecodeParams prm)
             m[0] = mn0; m[1] = mn1;
             l[0] = l[0] * al0 + p0 + p2;
             l[1] = l[1] * al1 + p1 + p3;
-            const uint32_t b0 = movmatrix_trans(pack_bf16x2(p0, p1));
-            const uint32_t b1 = movmatrix_trans(pack_bf16x2(p2, p3));
+            // the V scale rides on P (E4M3); l keeps the plain probabilities
+            const uint32_t b0 = movmatrix_trans(kE4M3 ? pack_bf16x2(p0 * vfac, p1 * vfac) : pack_bf16x2(p0, p1));
+            const uint32_t b1 = movmatrix_trans(kE4M3 ? pack_bf16x2(p2 * vfac, p3 * vfac) : pack_bf16x2(p2, p3));
             if (__any_sync(0xffffffffu, al0 != 1.f || al1 != 1.f)) {   // a head's running max moved
 #pragma unroll
                 for (int mt = 0; mt < 8; ++mt) {
@@ -238,8 +310,8 @@ decode_warp_kernel(const DecodeParams prm)
                 ldmatrix_x4_trans(a, base + (2 + (mt >> 2)) * kBoxBytes + sw128_offset(row, col));
                 mma_bf16_16816(o[mt], a, b0, b1);
             }
-            __syncwarp();   // every lane is done with the stage before it is refilled
-            issue_next();
+            __syncwarp();   // every lane is done with the stage (bf16) or the expanded block (E4M3)
+            if constexpr (!kE4M3) issue_next();   // (E4M3: the stage was refilled after its expansion)
         }
         // complete the row sums over the 8 token lanes of each head
 #pragma unroll
@@ -449,6 +521,122 @@ __global__ void __launch_bounds__(128) decode_f32_kernel(const float *__restrict
     if (lane == 0) lse[row] = empty ? -INFINITY : (m + log2f(l)) * PADOC_LN2;
 }
 
+// The bf16 path's split-K decode over either pool: the tensor-core grid for the shared streams of
+// dense pages, the warp grid for the rest, and the merge; arguments validated by the caller.
+struct DecodePool {
+    bool e4m3;
+    const void *k, *v;                    // bf16 pools or E4M3 codes
+    const float *k_scales, *v_scales;     // E4M3 scales
+    int32_t num_blocks;
+};
+
+padoc_status decode_split_k(const DecodePool &pl, const padoc_decode_plan *info, const int32_t *plan,
+                            const int32_t *page_block_table, int32_t page_table_stride,
+                            const int32_t *stream_block_table, int32_t stream_table_stride, const void *q, float scale,
+                            void *out, float *lse, void *workspace, size_t workspace_bytes, cudaStream_t cs)
+{
+    const padoc_decode_config &cfg = info->cfg;
+    if (cfg.head_dim != kD || cfg.num_q_heads != kGroup * cfg.num_kv_heads || cfg.block_size != kBlk)
+        return PADOC_ERR_UNSUPPORTED;
+    size_t need = 0;
+    const padoc_status ws_st = padoc_decode_workspace_size(info, &need);
+    if (ws_st != PADOC_OK) return ws_st;
+    if (!workspace || workspace_bytes < need) return PADOC_ERR_WORKSPACE_TOO_SMALL;
+    if (((uintptr_t)workspace) & 255) return PADOC_ERR_INVALID_ARGUMENT;
+    int *err = padoc_device_error_word();   // the first CUDA call: every check above is on the host
+    if (!err) return PADOC_ERR_CUDA;
+
+    const uint64_t rows = (uint64_t)pl.num_blocks * cfg.num_kv_heads * kBlk;
+    CUtensorMap kmap, vmap;   // bf16: 16-row x 64-column boxes; E4M3: 16-row x 128-byte boxes of codes
+    if (pl.e4m3 ? (!padoc_make_tmap_u8(&kmap, pl.k, kD, rows, kD, kD, kBlk) ||
+                   !padoc_make_tmap_u8(&vmap, pl.v, kD, rows, kD, kD, kBlk))
+                : (!padoc_make_tmap_bf16(&kmap, pl.k, kD, rows, kD * 2, 64, kBlk) ||
+                   !padoc_make_tmap_bf16(&vmap, pl.v, kD, rows, kD * 2, 64, kBlk)))
+        return PADOC_ERR_CUDA;
+
+    if ((int64_t)pl.num_blocks * cfg.num_kv_heads * kBlk >= INT32_MAX) return PADOC_ERR_UNSUPPORTED;
+    float *part_o = (float *)workspace;
+    float *part_lse = (float *)((uint8_t *)workspace + padoc_align256((size_t)info->num_slots * kGroup * kD * 4));
+    const float sl2 = scale * PADOC_LOG2E;
+
+    // shared streams of dense pages on the tensor cores
+    CUtensorMap qmap;   // Q [S][Hq][d] as [S][Hkv][8][d]: a box is 16 streams x the 8 heads of one KV head
+    {
+        const uint64_t dims[4] = {(uint64_t)kD, (uint64_t)kGroup, (uint64_t)cfg.num_kv_heads, (uint64_t)info->num_streams};
+        const uint64_t strides[3] = {(uint64_t)kD * 2, (uint64_t)kGroup * kD * 2, (uint64_t)cfg.num_q_heads * kD * 2};
+        const uint32_t box[4] = {64, (uint32_t)kGroup, 1, 16};
+        if (info->num_tc_items > 0 && !padoc_make_tmap_bf16_4d(&qmap, q, dims, strides, box)) return PADOC_ERR_CUDA;
+    }
+    padoc_status st = padoc_launch_decode_tc(&kmap, &vmap, &qmap, plan, info, page_block_table, page_table_stride,
+                                             stream_block_table, stream_table_stride,
+                                             pl.num_blocks, pl.e4m3 ? pl.k_scales : nullptr,
+                                             pl.e4m3 ? pl.v_scales : nullptr, part_o, part_lse, sl2, err, cs);
+    if (st != PADOC_OK) return st;
+
+    // private histories and the shared streams of sparse pages, one warp per item
+    DecodeParams prm;
+    prm.stream_page = plan + info->off_stream_page;
+    prm.shared_len = plan + info->off_shared_len;
+    prm.private_len = plan + info->off_private_len;
+    prm.slot_ptr = plan + info->off_slot_ptr;
+    prm.items = reinterpret_cast<const padoc_item *>(plan + info->off_items);
+    prm.first_item = info->num_tc_items;
+    prm.warp_ptr = plan + info->off_warp_ptr;
+    prm.num_warps = info->num_warps;
+    prm.page_table = page_block_table;
+    prm.stream_table = stream_block_table;
+    prm.page_stride = page_table_stride;
+    prm.stream_stride = stream_table_stride;
+    prm.num_blocks = pl.num_blocks;
+    prm.num_kv_heads = cfg.num_kv_heads;
+    prm.num_q_heads = cfg.num_q_heads;
+    prm.pool_rows = pl.num_blocks * cfg.num_kv_heads * kBlk;
+    prm.k_pool = pl.e4m3 ? nullptr : (const __nv_bfloat16 *)pl.k;
+    prm.v_pool = pl.e4m3 ? nullptr : (const __nv_bfloat16 *)pl.v;
+    prm.k_codes = pl.e4m3 ? (const uint8_t *)pl.k : nullptr;
+    prm.v_codes = pl.e4m3 ? (const uint8_t *)pl.v : nullptr;
+    prm.k_scales = pl.k_scales;
+    prm.v_scales = pl.v_scales;
+    prm.q = (const __nv_bfloat16 *)q;
+    prm.part_o = part_o;
+    prm.part_lse = part_lse;
+    prm.scale_log2 = sl2;
+    prm.err = err;
+    prm.after_tc = info->num_tc_items > 0 ? 1 : 0;
+    if (prm.num_warps > 0) {
+        const size_t smem = pl.e4m3 ? kDecodeSmemE4M3 : kDecodeSmem;
+        auto kern = pl.e4m3 ? decode_warp_kernel<true> : decode_warp_kernel<false>;
+        PADOC_CUDA_TRY(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
+        cudaLaunchConfig_t lc = {};
+        lc.gridDim = dim3((unsigned)((prm.num_warps + kWarps - 1) / kWarps));
+        lc.blockDim = dim3(kWarps * 32);
+        lc.dynamicSmemBytes = smem;
+        lc.stream = cs;
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        attr[0].val.programmaticStreamSerializationAllowed = 1;
+        lc.attrs = attr;
+        lc.numAttrs = 1;
+        PADOC_CUDA_TRY(cudaLaunchKernelEx(&lc, kern, prm));
+        st = padoc_launch_status();
+        if (st != PADOC_OK) return st;
+    }
+    {
+        cudaLaunchConfig_t lc = {};
+        lc.gridDim = dim3((unsigned)((int64_t)info->num_streams * cfg.num_kv_heads));
+        lc.blockDim = dim3(128);
+        lc.stream = cs;
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;   // see the kernel's wait
+        attr[0].val.programmaticStreamSerializationAllowed = 1;
+        lc.attrs = attr;
+        lc.numAttrs = 1;
+        PADOC_CUDA_TRY(cudaLaunchKernelEx(&lc, decode_combine_kernel, prm.slot_ptr, (const float *)part_o,
+                                          (const float *)part_lse, (__nv_bfloat16 *)out, lse));
+    }
+    return padoc_launch_status();
+}
+
 }  // namespace
 
 // ------------------------------------------------------------------------------------------------
@@ -476,11 +664,11 @@ extern "C" padoc_status padoc_branch_decode_attn(const padoc_kv_pool *pool, cons
     if ((((uintptr_t)pool->k_pool) | ((uintptr_t)pool->v_pool) | ((uintptr_t)q) | ((uintptr_t)out)) & 15)
         return PADOC_ERR_INVALID_ARGUMENT;
     const int32_t *plan = plan_dev;
-    int *err = padoc_device_error_word();
-    if (!err) return PADOC_ERR_CUDA;
     cudaStream_t cs = (cudaStream_t)stream;
 
     if (pool->dtype == PADOC_DTYPE_F32) {
+        int *err = padoc_device_error_word();
+        if (!err) return PADOC_ERR_CUDA;
         if (cfg.head_dim != 64 && cfg.head_dim != 128) return PADOC_ERR_UNSUPPORTED;
         const int64_t rows = (int64_t)info->num_streams * cfg.num_q_heads;
         const unsigned grid = (unsigned)((rows + 3) / 4);
@@ -496,94 +684,36 @@ extern "C" padoc_status padoc_branch_decode_attn(const padoc_kv_pool *pool, cons
         return padoc_launch_status();
     }
     if (pool->dtype != PADOC_DTYPE_BF16) return PADOC_ERR_UNSUPPORTED;
-    if (cfg.head_dim != kD || cfg.num_q_heads != kGroup * cfg.num_kv_heads || cfg.block_size != kBlk)
-        return PADOC_ERR_UNSUPPORTED;
-    size_t need = 0;
-    const padoc_status ws_st = padoc_decode_workspace_size(info, &need);
-    if (ws_st != PADOC_OK) return ws_st;
-    if (!workspace || workspace_bytes < need) return PADOC_ERR_WORKSPACE_TOO_SMALL;
-    if (((uintptr_t)workspace) & 255) return PADOC_ERR_INVALID_ARGUMENT;
+    const DecodePool dp{false, pool->k_pool, pool->v_pool, nullptr, nullptr, pool->num_blocks};
+    return decode_split_k(dp, info, plan, page_block_table, page_table_stride, stream_block_table, stream_table_stride,
+                          q, scale, out, lse, workspace, workspace_bytes, cs);
+}
 
-    const uint64_t rows = (uint64_t)pool->num_blocks * cfg.num_kv_heads * kBlk;
-    CUtensorMap kmap, vmap;
-    if (!padoc_make_tmap_bf16(&kmap, pool->k_pool, kD, rows, kD * 2, 64, kBlk) ||
-        !padoc_make_tmap_bf16(&vmap, pool->v_pool, kD, rows, kD * 2, 64, kBlk))
-        return PADOC_ERR_CUDA;
-
-    if ((int64_t)pool->num_blocks * cfg.num_kv_heads * kBlk >= INT32_MAX) return PADOC_ERR_UNSUPPORTED;
-    float *part_o = (float *)workspace;
-    float *part_lse = (float *)((uint8_t *)workspace + padoc_align256((size_t)info->num_slots * kGroup * kD * 4));
-    const float sl2 = scale * PADOC_LOG2E;
-
-    // shared streams of dense pages on the tensor cores
-    CUtensorMap qmap;   // Q [S][Hq][d] as [S][Hkv][8][d]: a box is 16 streams x the 8 heads of one KV head
-    {
-        const uint64_t dims[4] = {(uint64_t)kD, (uint64_t)kGroup, (uint64_t)cfg.num_kv_heads, (uint64_t)info->num_streams};
-        const uint64_t strides[3] = {(uint64_t)kD * 2, (uint64_t)kGroup * kD * 2, (uint64_t)cfg.num_q_heads * kD * 2};
-        const uint32_t box[4] = {64, (uint32_t)kGroup, 1, 16};
-        if (info->num_tc_items > 0 && !padoc_make_tmap_bf16_4d(&qmap, q, dims, strides, box)) return PADOC_ERR_CUDA;
-    }
-    padoc_status st = padoc_launch_decode_tc(&kmap, &vmap, &qmap, plan, info, page_block_table, page_table_stride,
-                                             stream_block_table, stream_table_stride,
-                                             pool->num_blocks, part_o, part_lse, sl2, err, cs);
-    if (st != PADOC_OK) return st;
-
-    // private histories and the shared streams of sparse pages, one warp per item
-    DecodeParams prm;
-    prm.stream_page = plan + info->off_stream_page;
-    prm.shared_len = plan + info->off_shared_len;
-    prm.private_len = plan + info->off_private_len;
-    prm.slot_ptr = plan + info->off_slot_ptr;
-    prm.items = reinterpret_cast<const padoc_item *>(plan + info->off_items);
-    prm.first_item = info->num_tc_items;
-    prm.warp_ptr = plan + info->off_warp_ptr;
-    prm.num_warps = info->num_warps;
-    prm.page_table = page_block_table;
-    prm.stream_table = stream_block_table;
-    prm.page_stride = page_table_stride;
-    prm.stream_stride = stream_table_stride;
-    prm.num_blocks = pool->num_blocks;
-    prm.num_kv_heads = cfg.num_kv_heads;
-    prm.num_q_heads = cfg.num_q_heads;
-    prm.pool_rows = pool->num_blocks * cfg.num_kv_heads * kBlk;
-    prm.k_pool = (const __nv_bfloat16 *)pool->k_pool;
-    prm.v_pool = (const __nv_bfloat16 *)pool->v_pool;
-    prm.q = (const __nv_bfloat16 *)q;
-    prm.part_o = part_o;
-    prm.part_lse = part_lse;
-    prm.scale_log2 = sl2;
-    prm.err = err;
-    prm.after_tc = info->num_tc_items > 0 ? 1 : 0;
-    if (prm.num_warps > 0) {
-        PADOC_CUDA_TRY(cudaFuncSetAttribute(decode_warp_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kDecodeSmem));
-        cudaLaunchConfig_t lc = {};
-        lc.gridDim = dim3((unsigned)((prm.num_warps + kWarps - 1) / kWarps));
-        lc.blockDim = dim3(kWarps * 32);
-        lc.dynamicSmemBytes = kDecodeSmem;
-        lc.stream = cs;
-        cudaLaunchAttribute attr[1];
-        attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-        attr[0].val.programmaticStreamSerializationAllowed = 1;
-        lc.attrs = attr;
-        lc.numAttrs = 1;
-        PADOC_CUDA_TRY(cudaLaunchKernelEx(&lc, decode_warp_kernel, prm));
-        st = padoc_launch_status();
-        if (st != PADOC_OK) return st;
-    }
-    {
-        cudaLaunchConfig_t lc = {};
-        lc.gridDim = dim3((unsigned)((int64_t)info->num_streams * cfg.num_kv_heads));
-        lc.blockDim = dim3(128);
-        lc.stream = cs;
-        cudaLaunchAttribute attr[1];
-        attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;   // see the kernel's wait
-        attr[0].val.programmaticStreamSerializationAllowed = 1;
-        lc.attrs = attr;
-        lc.numAttrs = 1;
-        PADOC_CUDA_TRY(cudaLaunchKernelEx(&lc, decode_combine_kernel, prm.slot_ptr, (const float *)part_o,
-                                          (const float *)part_lse, (__nv_bfloat16 *)out, lse));
-    }
-    return padoc_launch_status();
+extern "C" padoc_status padoc_branch_decode_attn_e4m3(const padoc_kv_pool_e4m3 *pool, const padoc_decode_plan *info,
+                                                      const int32_t *plan_dev, const int32_t *page_block_table,
+                                                      int32_t page_table_stride, const int32_t *stream_block_table,
+                                                      int32_t stream_table_stride, const void *q, float scale,
+                                                      void *out, float *lse, void *workspace, size_t workspace_bytes,
+                                                      padoc_stream_t stream)
+{
+    if (!pool || !info || !plan_dev || !q || !out || !lse) return PADOC_ERR_INVALID_ARGUMENT;
+    const padoc_decode_config &cfg = info->cfg;
+    if (pool->block_size != cfg.block_size || pool->num_kv_heads != cfg.num_kv_heads || pool->head_dim != cfg.head_dim)
+        return PADOC_ERR_INVALID_ARGUMENT;
+    if (!pool->k_codes || !pool->v_codes || !pool->k_scales || !pool->v_scales || pool->num_blocks < 1)
+        return PADOC_ERR_INVALID_ARGUMENT;
+    if (!(scale > 0.f) || !isfinite(scale)) return PADOC_ERR_INVALID_ARGUMENT;
+    if (info->num_pages > 0 && (!page_block_table || page_table_stride < info->max_page_blocks))
+        return PADOC_ERR_INVALID_ARGUMENT;
+    if (info->num_streams > 0 && (!stream_block_table || stream_table_stride < info->max_stream_blocks))
+        return PADOC_ERR_INVALID_ARGUMENT;
+    if (info->num_streams == 0) return PADOC_OK;
+    if ((((uintptr_t)pool->k_codes) | ((uintptr_t)pool->v_codes) | ((uintptr_t)q) | ((uintptr_t)out)) & 15)
+        return PADOC_ERR_INVALID_ARGUMENT;
+    if ((((uintptr_t)pool->k_scales) | ((uintptr_t)pool->v_scales)) & 3) return PADOC_ERR_INVALID_ARGUMENT;
+    const DecodePool dp{true, pool->k_codes, pool->v_codes, pool->k_scales, pool->v_scales, pool->num_blocks};
+    return decode_split_k(dp, info, plan_dev, page_block_table, page_table_stride, stream_block_table,
+                          stream_table_stride, q, scale, out, lse, workspace, workspace_bytes, (cudaStream_t)stream);
 }
 
 extern "C" padoc_status padoc_splitk_combine(const float *part_o, const float *part_lse, int32_t num_splits,

@@ -27,6 +27,15 @@
 // allocates TMEM; warps 9 and 11 issue the MMAs of M-tile 0 and M-tile 1, each as a converged warp.
 // TMEM: S_i / P_i at columns 128i, O_i at 256 + 128i. The next piece's first PV overwrites O_i; it
 // waits for P_i of that piece, which the softmax warps publish only after reading O_i out.
+//
+// FP8 (E4M3) pool (kE4M3): each paged block's codes (16 rows x 128 bytes) land by TMA in the upper
+// half of the tile's ring slot, and the producer warp that loaded them expands them in place into
+// the bf16 panels the MMAs read (each lane owns whole rows, reads a row's codes before writing it;
+// codes times 2^-112 are exact bf16 values), then marks the slot full. A producer expands tile n - 2
+// (K) or n - 1 (V) before it issues tile n, so loads stay in flight while it converts. The K
+// producer also copies each block's K and V scales into a ring of 8 entries, one per tile; the
+// softmax applies the K scale to the block's scores and folds the V scale into the block's
+// probabilities before they are rounded to bf16, and removes it again from their row sum.
 #include <math.h>
 
 #include "common.cuh"
@@ -56,17 +65,27 @@ enum {
     B_PFULL = 14,    // [m-tile], one arrival per softmax warp
     B_PVDONE = 16,   // [m-tile]: the piece's last PV has completed (O_i is final)
     B_FINAL = 18,
-    B_COUNT = 19
+    B_KSTG = 19,     // [K stage] E4M3: the tile's codes have landed
+    B_VSTG = 22,     // [V stage] E4M3
+    B_SCL = 24,      // [scale entry] E4M3: the tile's scales have landed (one arrival per loading lane)
+    B_COUNT = 32
 };
+constexpr int kSclEntries = 8;   // scale ring: entry n % 8 for tile n
 
 constexpr int kSoftmaxWarps = 8;
 constexpr int kXchBytes = 2 * 2 * 128 * 4;   // row max / sum swap: [buffer][column half][row] floats
-// Q (two M-tiles), the K and V rings, then barriers and the swap buffer: 231,680 bytes, so there is
-// no room to align the start by hand; the kernel checks that the driver placed it on a 1024-byte
-// boundary (the base of a CTA's dynamic shared memory is) and refuses to run otherwise.
+// Q (two M-tiles), the K and V rings, then barriers (256 bytes), the TMEM address and abort flag,
+// the scale ring (E4M3: [8 entries][8 K scales, 8 V scales]) and the swap buffer: 232,448 bytes,
+// the most a CTA may have, so there is no room to align the start by hand; the kernel checks that
+// the driver placed it on a 1024-byte boundary (the base of a CTA's dynamic shared memory is) and
+// refuses to run otherwise.
 constexpr size_t kTilesBytes = (size_t)kTile * (2 + kKStages + kVStages);
-constexpr size_t kSmemBytes = kTilesBytes + 256 + kXchBytes;
+constexpr int kMiscScl = 320, kMiscXch = 1024;
+constexpr size_t kSmemBytes = kTilesBytes + kMiscXch + kXchBytes;
 static_assert(kSmemBytes <= 232448, "shared memory per CTA");
+static_assert(B_COUNT * 8 <= 256 && kMiscScl + kSclEntries * 16 * 4 <= kMiscXch, "misc layout");
+constexpr float kTwo112 = 5.192296858534828e33f;   // 2^112: the bf16 expansion's factor
+static_assert(PADOC_E4M3_BF16_SHIFT_LOG2 == 112, "expansion factor");
 
 struct TcDecodeParams {
     const int32_t *shared_len, *private_len, *slot_ptr, *cta_ptr;
@@ -76,6 +95,7 @@ struct TcDecodeParams {
     int32_t page_stride, stream_stride;
     int32_t num_blocks, num_kv_heads;
     int32_t pool_rows;           // num_blocks * num_kv_heads * 16: first out-of-range row
+    const float *k_scales, *v_scales;   // E4M3 pool: [num_blocks][num_kv_heads]
     float *part_o, *part_lse;
     float scale_log2;
     int *err;
@@ -109,6 +129,37 @@ __device__ __forceinline__ const int32_t *item_row(const TcDecodeParams &prm, co
     return (priv ? prm.stream_table : prm.page_table) + (size_t)it.index * stride;
 }
 
+// E4M3: expands one landed tile of codes in place into the slot's two bf16 panels. Lane l owns
+// rows l, l + 32, l + 64, l + 96; it reads a row's eight 16-byte chunks of codes (swizzled by row,
+// in the upper half of the slot, where the row's panel-1 bytes go) before it writes the row.
+__device__ __forceinline__ void expand_tile(uint8_t *slot, int lane)
+{
+    const uint8_t *codes = slot + kPanel;
+#pragma unroll 1
+    for (int k = 0; k < 4; ++k) {
+        const int r = lane + 32 * k;
+        uint4 raw[8];
+#pragma unroll
+        for (int c = 0; c < 8; ++c) raw[c] = *reinterpret_cast<const uint4 *>(codes + r * 128 + ((c ^ (r & 7)) << 4));
+#pragma unroll
+        for (int c = 0; c < 8; ++c) {
+            const uint32_t w[4] = {raw[c].x, raw[c].y, raw[c].z, raw[c].w};
+#pragma unroll
+            for (int hh = 0; hh < 2; ++hh) {   // dims 16c + 8hh .. + 7: chunk 2c + hh of the row
+                const int kk = 2 * c + hh;
+                uint4 o;
+                o.x = e4m3x2_to_bf16x2_shifted((uint16_t)(w[2 * hh] & 0xFFFFu));
+                o.y = e4m3x2_to_bf16x2_shifted((uint16_t)(w[2 * hh] >> 16));
+                o.z = e4m3x2_to_bf16x2_shifted((uint16_t)(w[2 * hh + 1] & 0xFFFFu));
+                o.w = e4m3x2_to_bf16x2_shifted((uint16_t)(w[2 * hh + 1] >> 16));
+                *reinterpret_cast<uint4 *>(slot + (kk >> 3) * kPanel + r * 128 + (((kk & 7) ^ (r & 7)) << 4)) = o;
+            }
+        }
+    }
+    fence_proxy_async_smem();   // the MMAs read the panels through the async proxy
+}
+
+template <bool kE4M3>
 __global__ void __launch_bounds__(kThreads, 1)
 decode_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap,
                  const __grid_constant__ CUtensorMap qmap, const TcDecodeParams prm)
@@ -123,9 +174,10 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
     uint8_t *sv = sk + kKStages * kTile;
     uint8_t *misc = smem + kTilesBytes;
     uint64_t *bars = (uint64_t *)misc;
-    uint32_t *tmem_slot = (uint32_t *)(misc + 192);
-    volatile int *abort_flag = (volatile int *)(misc + 196);
-    float *xch = (float *)(misc + 256);
+    uint32_t *tmem_slot = (uint32_t *)(misc + 256);
+    volatile int *abort_flag = (volatile int *)(misc + 260);
+    float *scl = (float *)(misc + kMiscScl);   // E4M3: [entry][K scales of 8 blocks, V scales of 8 blocks]
+    float *xch = (float *)(misc + kMiscXch);
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     auto bar = [&](int i) { return smem_u32(&bars[i]); };
     if (warp == 8 || warp == 10) {
@@ -146,7 +198,7 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
                 if (id >= 0 && id < prm.num_blocks) {
                     const int32_t row = (id * prm.num_kv_heads + it.kv_head) * kBlk;
                     tma_prefetch_l2_2d(map, 0, row);
-                    tma_prefetch_l2_2d(map, 64, row);
+                    if (!kE4M3) tma_prefetch_l2_2d(map, 64, row);   // (an E4M3 box holds the whole row)
                 }
             }
             if (warp == 8 && lane == 16)
@@ -162,6 +214,7 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
                                           : (i == B_QFREE || (i >= B_KEMPTY && i < B_KEMPTY + kKStages) ||
                                              (i >= B_VEMPTY && i < B_VEMPTY + kVStages) || i == B_FINAL)
                                                 ? 2     // one commit from each MMA warp
+                                          : (i >= B_SCL) ? kKT / kBlk   // one per lane that loads a block
                                                 : 1);
         *abort_flag = 0;
         fence_barrier_init();
@@ -229,6 +282,23 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
         };
         if (u0 < u1) fetch_id(u0, 0);
         int n = 0, nq = 0;   // tiles and query sets issued
+        // E4M3: tiles expanded so far; a tile is expanded `lag` tiles after it is issued (K runs
+        // further ahead: its ring has three slots)
+        int nc = 0;
+        const int lag = is_k ? 2 : 1;
+        const int b_stg = is_k ? B_KSTG : B_VSTG;
+        auto expand_next = [&]() {   // whole warp; nc counts only tiles whose codes have landed
+            const int t = nc;
+            const int st = t % nst;
+            bool r = wait_or_abort(bar(b_stg + st), (t / nst) & 1, prm.err, is_k ? 56 : 57, abort_flag);
+            r = __all_sync(0xffffffffu, r);
+            if (!r) return false;
+            ++nc;
+            expand_tile(ring + st * kTile, lane);
+            __syncwarp();
+            if (lane == 0) mbar_arrive(bar(b_full + st));
+            return true;
+        };
         // the first piece's queries go out before anything else (they wait for nothing)
         const bool q_first = is_k && u0 < u1 && piece_tiles(prm.items[u0]) > 0;
         if (q_first) {
@@ -254,18 +324,45 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
                     else if (is_k) padoc_record_error(prm.err, PADOC_DEVERR_BLOCK_ID, id);
                 }
                 const int s = n % nst, use = n / nst;
+                if (kE4M3)
+                    while (ok && nc <= n - lag) ok = expand_next();
+                if (!ok) break;
                 if (use > 0) ok = wait_or_abort(bar(b_empty + s), (use - 1) & 1, prm.err, is_k ? 50 : 53, abort_flag);
                 if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
-                if (lane == 0) mbar_arrive_expect_tx(bar(b_full + s), kTile);
-                __syncwarp();
-                if (lane < kKT / kBlk) {
-                    const uint32_t dst = smem_u32(ring + s * kTile) + (uint32_t)lane * (kBlk * 128);
-                    const uint64_t kv_policy = (it.kind & PADOC_ITEM_REREAD) ? shared_policy : once_policy;
-                    tma_load_2d_hint(dst, map, 0, row, bar(b_full + s), kv_policy);
-                    tma_load_2d_hint(dst + kPanel, map, 64, row, bar(b_full + s), kv_policy);
+                const uint64_t kv_policy = (it.kind & PADOC_ITEM_REREAD) ? shared_policy : once_policy;
+                if constexpr (kE4M3) {
+                    // the block's codes (16 rows x 128 bytes) into the slot's upper half; the K warp also
+                    // copies the block's two scales into the tile's scale entry (zeros past the piece
+                    // or for a bad id, whose codes are zeros too)
+                    if (lane == 0) mbar_arrive_expect_tx(bar(b_stg + s), kTile / 2);
+                    __syncwarp();
+                    if (lane < kKT / kBlk) {
+                        const uint32_t dst = smem_u32(ring + s * kTile) + kPanel + (uint32_t)lane * (kBlk * 128);
+                        tma_load_2d_hint(dst, map, 0, row, bar(b_stg + s), kv_policy);
+                        if (is_k) {
+                            const bool okid = row != prm.pool_rows;
+                            const size_t si = okid ? (size_t)id * prm.num_kv_heads + it.kv_head : 0;
+                            float *e = scl + (n % kSclEntries) * 16;
+                            cp_async_4(smem_u32(e + lane), prm.k_scales + si, okid ? 4u : 0u);
+                            cp_async_4(smem_u32(e + 8 + lane), prm.v_scales + si, okid ? 4u : 0u);
+                            cp_async_mbar_arrive(bar(B_SCL + n % kSclEntries));
+                        }
+                    }
+                } else {
+                    if (lane == 0) mbar_arrive_expect_tx(bar(b_full + s), kTile);
+                    __syncwarp();
+                    if (lane < kKT / kBlk) {
+                        const uint32_t dst = smem_u32(ring + s * kTile) + (uint32_t)lane * (kBlk * 128);
+                        tma_load_2d_hint(dst, map, 0, row, bar(b_full + s), kv_policy);
+                        tma_load_2d_hint(dst + kPanel, map, 64, row, bar(b_full + s), kv_policy);
+                    }
                 }
                 ++n;
                 if (is_k && j == 0 && !(q_first && u == u0)) {
+                    // E4M3: the previous piece's tiles must be expanded before its last QK^T can run
+                    if (kE4M3)
+                        while (ok && nc < n - 1) ok = expand_next();
+                    if (!ok) break;
                     // this piece's queries, once the previous piece's last QK^T has read the buffer
                     if (nq > 0) ok = wait_or_abort(bar(B_QFREE), (nq - 1) & 1, prm.err, 55, abort_flag);
                     if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
@@ -274,8 +371,16 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
                 }
             }
         }
-        // copies still in flight must land before the CTA's shared memory is released
-        if (lane == 0) {
+        if constexpr (kE4M3) {
+            // the last tiles' expansion; after a failed wait only their copies are waited for
+            while (ok && nc < n) ok = expand_next();
+            if (lane == 0)
+                for (int J = nc; J < n; ++J)
+                    mbar_wait_bounded(bar(b_stg + J % nst), (J / nst) & 1, prm.err, is_k ? 51 : 52);
+            if (is_k) cp_async_wait<0>();
+            if (lane == 0 && nq > 0) mbar_wait_bounded(bar(B_Q), (nq - 1) & 1, prm.err, 54);
+        } else if (lane == 0) {
+            // copies still in flight must land before the CTA's shared memory is released
             if (nq > 0) mbar_wait_bounded(bar(B_Q), (nq - 1) & 1, prm.err, 54);
             for (int J = (n > nst ? n - nst : 0); J < n; ++J)
                 mbar_wait_bounded(bar(b_full + J % nst), (J / nst) & 1, prm.err, is_k ? 51 : 52);
@@ -360,6 +465,7 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
         const int hl = row % kGroup;
         const uint32_t lanes = (uint32_t)(quad * 32) << 16;
         const float c = prm.scale_log2;
+        const float cm = kE4M3 ? 1.f : c;   // E4M3: the row maxima are already scaled by the multipliers
         auto wait_all = [&](int bb, uint32_t parity, int site) {
             const bool r = wait_or_abort(bar(bb), parity, prm.err, site, abort_flag);
             return __all_sync(0xffffffffu, r);
@@ -421,6 +527,24 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
             for (int j = 0; j < ne; ++j) {
                 if (j == 1 && u + 1 < u1) fetch_cut();
                 if (j == ne - 1) fetch_slots();
+                // E4M3: for the 16-column blocks 4 hc .. 4 hc + 3 of this thread's column half, the
+                // multiplier of the raw scores (log2 units, K scale and 2^112 folded in), the V factor
+                // folded into P (as a log2 offset of the exponent) and its inverse for the row sum. A
+                // zero scale marks a block without a nonzero value (its codes are zeros): any positive
+                // factor gives the same result there.
+                float kcb[4], vlb[4], vib[4];
+                if constexpr (kE4M3) {
+                    const int e = cnt0 % kSclEntries;   // cnt0: tiles so far (every piece has M-tile 0)
+                    ok = ok && wait_all(B_SCL + e, (cnt0 / kSclEntries) & 1, 72);
+#pragma unroll
+                    for (int b = 0; b < 4; ++b) {
+                        const float ks = scl[e * 16 + 4 * hc + b], vs = scl[e * 16 + 8 + 4 * hc + b];
+                        kcb[b] = c * (ks > 0.f ? ks : 1.f) * kTwo112;
+                        const float vf = (vs > 0.f ? vs : 1.f) * kTwo112;
+                        vlb[b] = __log2f(vf);
+                        vib[b] = fast_exp2(-vlb[b]);
+                    }
+                }
 #pragma unroll
                 for (int mi = 0; mi < 2; ++mi) {
                     if (mi >= mt) break;
@@ -451,44 +575,77 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
                         }
                     }
                     float mx4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+                    float mx;
+                    if constexpr (kE4M3) {
+                        // block b = columns 16b .. 16b + 15 of the half: its max, then times its multiplier
 #pragma unroll
-                    for (int uu = 0; uu < 2; ++uu)
+                        for (int uu = 0; uu < 2; ++uu)
 #pragma unroll
-                        for (int i = 0; i < 32; i += 8) {
-                            mx4[0] = fmax3f(mx4[0], __uint_as_float(sr[uu][i]), __uint_as_float(sr[uu][i + 1]));
-                            mx4[1] = fmax3f(mx4[1], __uint_as_float(sr[uu][i + 2]), __uint_as_float(sr[uu][i + 3]));
-                            mx4[2] = fmax3f(mx4[2], __uint_as_float(sr[uu][i + 4]), __uint_as_float(sr[uu][i + 5]));
-                            mx4[3] = fmax3f(mx4[3], __uint_as_float(sr[uu][i + 6]), __uint_as_float(sr[uu][i + 7]));
-                        }
-                    float mx = fmaxf(fmax3f(mx4[0], mx4[1], mx4[2]), mx4[3]);
+                            for (int i = 0; i < 32; i += 4) {
+                                const int b = 2 * uu + (i >> 4);
+                                mx4[b] = fmax3f(mx4[b], __uint_as_float(sr[uu][i]), __uint_as_float(sr[uu][i + 1]));
+                                mx4[b] = fmax3f(mx4[b], __uint_as_float(sr[uu][i + 2]), __uint_as_float(sr[uu][i + 3]));
+                            }
+                        mx = fmaxf(fmaxf(mx4[0] * kcb[0], mx4[1] * kcb[1]), fmaxf(mx4[2] * kcb[2], mx4[3] * kcb[3]));
+                    } else {
+#pragma unroll
+                        for (int uu = 0; uu < 2; ++uu)
+#pragma unroll
+                            for (int i = 0; i < 32; i += 8) {
+                                mx4[0] = fmax3f(mx4[0], __uint_as_float(sr[uu][i]), __uint_as_float(sr[uu][i + 1]));
+                                mx4[1] = fmax3f(mx4[1], __uint_as_float(sr[uu][i + 2]), __uint_as_float(sr[uu][i + 3]));
+                                mx4[2] = fmax3f(mx4[2], __uint_as_float(sr[uu][i + 4]), __uint_as_float(sr[uu][i + 5]));
+                                mx4[3] = fmax3f(mx4[3], __uint_as_float(sr[uu][i + 6]), __uint_as_float(sr[uu][i + 7]));
+                            }
+                        mx = fmaxf(fmax3f(mx4[0], mx4[1], mx4[2]), mx4[3]);
+                    }
                     // every P store below lands after both halves have read their S columns
                     mx = fmaxf(mx, swap_row(mx));
                     const float m_new = fmaxf(m_ref, mx);
                     // lazy rescaling: the reference max moves only when the row max grew by more
-                    // than 2^8 in probability
-                    const bool rescale = m_ref != -INFINITY && (m_new - m_ref) * c > 8.f;
+                    // than 2^8 in probability (E4M3: maxima are kept already in log2 units)
+                    const bool rescale = m_ref != -INFINITY && (m_new - m_ref) * cm > 8.f;
                     if (m_ref == -INFINITY) m_ref = m_new;
                     float alpha = 1.f;
                     if (rescale) {
-                        alpha = fast_exp2((m_ref - m_new) * c);
+                        alpha = fast_exp2((m_ref - m_new) * cm);
                         l *= alpha;
                         m_ref = m_new;
                     }
-                    const float moff = m_ref == -INFINITY ? 0.f : m_ref * c;
+                    const float moff = m_ref == -INFINITY ? 0.f : m_ref * cm;
                     float rs[4] = {0.f, 0.f, 0.f, 0.f};
                     uint32_t pk[32];
+                    if constexpr (kE4M3) {
+                        // P of block b carries its V factor (the exponent's log2 offset); rs[b] sums the
+                        // block's carried values, and the factor comes off again in the row sum
 #pragma unroll
-                    for (int qq = 0; qq < 2; ++qq) {
+                        for (int qq = 0; qq < 2; ++qq) {
 #pragma unroll
-                        for (int i = 0; i < 32; i += 2) {
-                            const float p0 = fast_exp2(fmaf(__uint_as_float(sr[qq][i]), c, -moff));
-                            const float p1 = fast_exp2(fmaf(__uint_as_float(sr[qq][i + 1]), c, -moff));
-                            rs[(i >> 1) & 3] += p0 + p1;
-                            pk[qq * 16 + (i >> 1)] = pack_bf16x2(p0, p1);
+                            for (int i = 0; i < 32; i += 2) {
+                                const int b = 2 * qq + (i >> 4);
+                                const float off = vlb[b] - moff;
+                                const float p0 = fast_exp2(fmaf(__uint_as_float(sr[qq][i]), kcb[b], off));
+                                const float p1 = fast_exp2(fmaf(__uint_as_float(sr[qq][i + 1]), kcb[b], off));
+                                rs[b] += p0 + p1;
+                                pk[qq * 16 + (i >> 1)] = pack_bf16x2(p0, p1);
+                            }
                         }
+                        tmem_st32(tS + 32 * hc, pk);
+                        l += (rs[0] * vib[0] + rs[1] * vib[1]) + (rs[2] * vib[2] + rs[3] * vib[3]);
+                    } else {
+#pragma unroll
+                        for (int qq = 0; qq < 2; ++qq) {
+#pragma unroll
+                            for (int i = 0; i < 32; i += 2) {
+                                const float p0 = fast_exp2(fmaf(__uint_as_float(sr[qq][i]), c, -moff));
+                                const float p1 = fast_exp2(fmaf(__uint_as_float(sr[qq][i + 1]), c, -moff));
+                                rs[(i >> 1) & 3] += p0 + p1;
+                                pk[qq * 16 + (i >> 1)] = pack_bf16x2(p0, p1);
+                            }
+                        }
+                        tmem_st32(tS + 32 * hc, pk);   // P (bf16 pairs) of columns [64 hc, 64 hc + 64)
+                        l += (rs[0] + rs[1]) + (rs[2] + rs[3]);
                     }
-                    tmem_st32(tS + 32 * hc, pk);   // P (bf16 pairs) of columns [64 hc, 64 hc + 64)
-                    l += (rs[0] + rs[1]) + (rs[2] + rs[3]);
                     if (__any_sync(0xffffffffu, rescale)) {
                         // PV_i(j-1) completed before S_i(j) (issue order) and PV_i(j) waits for this
                         // warp's P, so O_i is quiescent here
@@ -548,7 +705,7 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
                         }
                     }
                 }
-                if (valid && hc == 0) prm.part_lse[prow] = empty ? -INFINITY : (m_ref * c + log2f(l)) * PADOC_LN2;
+                if (valid && hc == 0) prm.part_lse[prow] = empty ? -INFINITY : (m_ref * cm + log2f(l)) * PADOC_LN2;
             }
         }
     }
@@ -564,9 +721,9 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
 
 padoc_status padoc_launch_decode_tc(const CUtensorMap *kmap, const CUtensorMap *vmap, const CUtensorMap *qmap, const int32_t *plan,
                                     const padoc_decode_plan *info, const int32_t *page_table, int32_t page_stride,
-                                    const int32_t *stream_table, int32_t stream_stride,
-                                    int32_t num_blocks, float *part_o, float *part_lse, float scale_log2, int *err,
-                                    cudaStream_t stream)
+                                    const int32_t *stream_table, int32_t stream_stride, int32_t num_blocks,
+                                    const float *k_scales, const float *v_scales, float *part_o, float *part_lse,
+                                    float scale_log2, int *err, cudaStream_t stream)
 {
     if (info->num_tc_items == 0 || info->tc_ctas == 0) return PADOC_OK;
     TcDecodeParams prm;
@@ -585,11 +742,15 @@ padoc_status padoc_launch_decode_tc(const CUtensorMap *kmap, const CUtensorMap *
     prm.num_blocks = num_blocks;
     prm.num_kv_heads = info->cfg.num_kv_heads;
     prm.pool_rows = num_blocks * info->cfg.num_kv_heads * kBlk;
+    prm.k_scales = k_scales;
+    prm.v_scales = v_scales;
     prm.part_o = part_o;
     prm.part_lse = part_lse;
     prm.scale_log2 = scale_log2;
     prm.err = err;
-    PADOC_CUDA_TRY(cudaFuncSetAttribute(decode_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes));
+    const bool e4m3 = k_scales != nullptr;   // an E4M3 pool: the maps hold codes
+    auto kern = e4m3 ? decode_tc_kernel<true> : decode_tc_kernel<false>;
+    PADOC_CUDA_TRY(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes));
     cudaLaunchConfig_t lc = {};
     lc.gridDim = dim3((unsigned)info->tc_ctas);
     lc.blockDim = dim3(kThreads);
@@ -600,6 +761,6 @@ padoc_status padoc_launch_decode_tc(const CUtensorMap *kmap, const CUtensorMap *
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     lc.attrs = attr;
     lc.numAttrs = 1;
-    PADOC_CUDA_TRY(cudaLaunchKernelEx(&lc, decode_tc_kernel, *kmap, *vmap, *qmap, prm));
+    PADOC_CUDA_TRY(cudaLaunchKernelEx(&lc, kern, *kmap, *vmap, *qmap, prm));
     return padoc_launch_status();
 }

@@ -49,6 +49,12 @@ class padoc_decode_config(ctypes.Structure):
                 ("tc_ctas", ctypes.c_int32), ("warp_ctas", ctypes.c_int32)]
 
 
+class padoc_kv_pool_e4m3(ctypes.Structure):
+    _fields_ = [("k_codes", ctypes.c_void_p), ("v_codes", ctypes.c_void_p), ("k_scales", ctypes.c_void_p),
+                ("v_scales", ctypes.c_void_p), ("num_blocks", ctypes.c_int32), ("block_size", ctypes.c_int32),
+                ("num_kv_heads", ctypes.c_int32), ("head_dim", ctypes.c_int32)]
+
+
 class padoc_stream_desc(ctypes.Structure):
     _fields_ = [("page", ctypes.c_int32), ("shared_len", ctypes.c_int32), ("private_len", ctypes.c_int32)]
 
@@ -160,6 +166,12 @@ def load_library(path: Optional[str] = None):
                                   _vp, _vp, ctypes.c_size_t, _vp],
         "padoc_selftest_tcgen05": [_vp, _vp, _vp, _vp, _vp, _vp, _vp],
         "padoc_selftest_wait_timeout": [ctypes.c_int32, ctypes.c_int32, _vp, _vp],
+        "padoc_quantize_kv_blocks": [ctypes.POINTER(padoc_kv_pool_e4m3), _vp, _vp, _vp, ctypes.c_int32, _vp],
+        "padoc_append_inputs_e4m3": [ctypes.POINTER(padoc_kv_pool_e4m3), _vp, _vp, _vp, ctypes.c_int64, ctypes.c_int32,
+                                     _vp, _vp, _vp, ctypes.c_int32, _vp],
+        "padoc_branch_decode_attn_e4m3": [ctypes.POINTER(padoc_kv_pool_e4m3), ctypes.POINTER(padoc_decode_plan), _vp,
+                                          _vp, ctypes.c_int32, _vp, ctypes.c_int32, _vp, ctypes.c_float, _vp, _vp,
+                                          _vp, ctypes.c_size_t, _vp],
         "padoc_check_device_errors": [_vp],
         "padoc_last_device_error": [_i32p, _i32p],
         "padoc_status_string": [ctypes.c_int],
@@ -192,6 +204,7 @@ def exported_symbols() -> Sequence[str]:
                         "padoc_mpd_launch_step",
                         "padoc_append_inputs",
                         "padoc_selftest_tcgen05", "padoc_selftest_wait_timeout",
+                        "padoc_quantize_kv_blocks", "padoc_append_inputs_e4m3", "padoc_branch_decode_attn_e4m3",
                         "padoc_check_device_errors",
                         "padoc_last_device_error", "padoc_status_string", "padoc_version")]
 
@@ -646,6 +659,59 @@ def make_kv_pool(k_pool, v_pool) -> padoc_kv_pool:
     """padoc_kv_pool over pool tensors [num_blocks][Hkv][16][d] (the caller keeps them alive)."""
     return padoc_kv_pool(_dev(k_pool, "k_pool"), _dev(v_pool, "v_pool"), k_pool.shape[0], k_pool.shape[2],
                          k_pool.shape[1], k_pool.shape[3], _dtype_code(k_pool))
+
+
+class E4M3Pool:
+    """An FP8 (E4M3) paged KV pool on the device: codes uint8 [num_blocks][Hkv][16][d] for K and V and
+    fp32 scales [num_blocks][Hkv] (torch tensors owned here), and its padoc_kv_pool_e4m3."""
+
+    def __init__(self, num_blocks: int, num_kv_heads: int, head_dim: int, device, block_size: int = 16):
+        import torch
+        shape = (num_blocks, num_kv_heads, block_size, head_dim)
+        self.k_codes = torch.zeros(shape, dtype=torch.uint8, device=device)
+        self.v_codes = torch.zeros(shape, dtype=torch.uint8, device=device)
+        self.k_scales = torch.zeros((num_blocks, num_kv_heads), dtype=torch.float32, device=device)
+        self.v_scales = torch.zeros((num_blocks, num_kv_heads), dtype=torch.float32, device=device)
+        self.c = padoc_kv_pool_e4m3(_dev(self.k_codes, "k_codes"), _dev(self.v_codes, "v_codes"),
+                                    _dev(self.k_scales, "k_scales"), _dev(self.v_scales, "v_scales"), num_blocks,
+                                    block_size, num_kv_heads, head_dim)
+
+    @property
+    def num_blocks(self) -> int:
+        return self.c.num_blocks
+
+
+def padoc_quantize_kv_blocks(pool: E4M3Pool, k_src, v_src, dst_blocks, stream=None):
+    """Whole bf16 blocks k_src / v_src [count][Hkv][16][d] into pool blocks dst_blocks (int32 CUDA tensor)."""
+    lib = load_library()
+    _check("padoc_quantize_kv_blocks", lib.padoc_quantize_kv_blocks(ctypes.byref(pool.c), _dev(k_src, "k_src"),
+                                                                    _dev(v_src, "v_src"), _dev(dst_blocks, "dst_blocks"),
+                                                                    dst_blocks.shape[0], _stream_ptr(stream)))
+
+
+def padoc_append_inputs_e4m3(pool: E4M3Pool, k_src, v_src, slots, q_src=None, q_dst=None, src_rows=None, count=None,
+                             stream=None):
+    """padoc_append_inputs into an E4M3 pool (bf16 sources); the slots of one call in distinct blocks."""
+    lib = load_library()
+    n = slots.shape[0] if count is None else count
+    hq = q_src.shape[1] if q_src is not None else 0
+    st = lib.padoc_append_inputs_e4m3(ctypes.byref(pool.c), _dev(k_src, "k_src"), _dev(v_src, "v_src"),
+                                      _dev(q_src, "q_src"), k_src.shape[0], hq, _dev(q_dst, "q_dst"),
+                                      _dev(src_rows, "src_rows"), _dev(slots, "slots"), n, _stream_ptr(stream))
+    _check("padoc_append_inputs_e4m3", st)
+
+
+def padoc_branch_decode_attn_e4m3(pool: E4M3Pool, info: padoc_decode_plan, plan_dev, page_table, stream_table, q,
+                                  scale, out, lse, workspace, stream=None):
+    """padoc_branch_decode_attn over an E4M3 pool (q / out bf16 [streams][Hq][128], lse fp32)."""
+    lib = load_library()
+    st = lib.padoc_branch_decode_attn_e4m3(ctypes.byref(pool.c), ctypes.byref(info), _dev(plan_dev, "plan_dev"),
+                                           _dev(page_table, "page_table"), page_table.shape[1],
+                                           _dev(stream_table, "stream_table"), stream_table.shape[1], _dev(q, "q"),
+                                           float(scale), _dev(out, "out"), _dev(lse, "lse"),
+                                           _dev(workspace, "workspace"), workspace.numel() * workspace.element_size(),
+                                           _stream_ptr(stream))
+    _check("padoc_branch_decode_attn_e4m3", st)
 
 
 def padoc_append_inputs(k_pool, v_pool, k_src, v_src, slots, q_src=None, q_dst=None, src_rows=None, count=None,

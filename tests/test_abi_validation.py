@@ -104,3 +104,31 @@ def test_wait_timeout_selftest_rejects_malformed_calls(lib):
     call = lambda limit=1000, site=5, gave_up=A: lib.padoc_selftest_wait_timeout(limit, site, gave_up, None)
     assert call(limit=0) == 1 and call(limit=100001) == 1   # limits outside 1 us .. 0.1 s
     assert call(site=-1) == 1 and call(gave_up=None) == 1
+
+
+def _pool8(block_size=16, hkv=2, d=128, k=A, v=A, ks=A, vs=A):
+    return pa.padoc_kv_pool_e4m3(k, v, ks, vs, 64, block_size, hkv, d)
+
+
+def test_e4m3_calls_reject_malformed_calls(lib):
+    info = _decode_info(lib)
+    dec = lambda pool, q=A, ws=1 << 20: lib.padoc_branch_decode_attn_e4m3(
+        ctypes.byref(pool) if pool is not None else None, ctypes.byref(info), A, A, 8, A, 8, q, 0.1, A, A, A, ws, None)
+    assert dec(None) == 1
+    assert dec(_pool8(ks=None)) == 1 and dec(_pool8(k=None)) == 1       # codes and scales are required
+    assert dec(_pool8(hkv=4)) == 1 and dec(_pool8(block_size=32)) == 1  # pool and plan disagree
+    assert dec(_pool8(k=MIS)) == 1 and dec(_pool8(vs=A + 2)) == 1       # 16-byte codes, 4-byte scales
+    assert dec(_pool8(), q=MIS) == 1
+    assert dec(_pool8(), ws=16) == 3                                    # workspace below the plan's need
+    quant = lambda pool, k=A, v=A, blocks=A, count=3: lib.padoc_quantize_kv_blocks(
+        ctypes.byref(pool) if pool is not None else None, k, v, blocks, count, None)
+    assert quant(None) == 1 and quant(_pool8(), count=-1) == 1
+    assert quant(_pool8(), count=0) == 0                                # nothing to do
+    assert quant(_pool8(), blocks=None) == 1 and quant(_pool8(), k=MIS) == 1
+    assert quant(_pool8(d=64)) == 2 and quant(_pool8(block_size=8)) == 2
+    app = lambda pool, slots=A, qs=None, qd=None, count=4: lib.padoc_append_inputs_e4m3(
+        ctypes.byref(pool) if pool is not None else None, A, A, qs, 10, 16, qd, None, slots, count, None)
+    assert app(None) == 1 and app(_pool8(), count=-1) == 1
+    assert app(_pool8(), count=0) == 0
+    assert app(_pool8(), slots=None) == 1 and app(_pool8(), qs=A, qd=None) == 1
+    assert app(_pool8(d=64)) == 2
