@@ -335,6 +335,44 @@ def bench_decode(args, torch, dev, rank, world, layout_streams=False):
     return res
 
 
+def bench_decode_replicas(args, torch, dev, rank, world, shape):
+    """A decode step over R replicas of one page shape, decoded together (one decode call per step):
+    ``shape`` "decode_page" (P = 2048, L = 256, 16 branches) or "dense_page" (P = 4096, L = 512,
+    64 branches); each replica has its own seeded K/V/Q in distinct memory, R chosen so that the
+    batch's cache exceeds 4x L2 (every step reads the whole batch, so no step is served from L2)."""
+    from paper_2608_06146_gb300 import inputs
+    from paper_2608_06146_gb300 import padoc_attn as pa
+    from paper_2608_06146_gb300.engine import DecodePlan
+
+    base = inputs.WORKLOADS[shape](seed=1 if shape == "decode_page" else 2)
+    pg = base.pages[0]
+    page_bytes = (pg.stream_len + sum(pg.branch_len)) * base.num_kv_heads * base.head_dim * 2 * 2
+    R = math.ceil(4 * l2_bytes(torch) / page_bytes) + 1
+    wl = inputs.Workload(f"{R} x {shape}", [pg] * R, base.num_q_heads, base.num_kv_heads, base.head_dim,
+                         base.dtype, "decode")
+    seed = 7 + 1000 * rank
+    di = inputs.decode_inputs(wl, seed, pool_slack=1.0)
+    plan = DecodePlan(wl.pages, wl.num_q_heads, wl.num_kv_heads, wl.head_dim, dev, tc_ctas=args.tc_ctas,
+                      warp_ctas=args.warp_ctas, split_tokens=args.split_tokens)
+    S = plan.num_streams
+    k_pool, v_pool, q = di.k_pool.to(dev), di.v_pool.to(dev), di.q.to(dev)
+    page_table = torch.from_numpy(di.page_table).to(dev)
+    stream_table = torch.from_numpy(di.stream_table).to(dev)
+    out = torch.empty((S, wl.num_q_heads, wl.head_dim), dtype=torch.bfloat16, device=dev)
+    lse = torch.empty((S, wl.num_q_heads), dtype=torch.float32, device=dev)
+    scale = 1.0 / math.sqrt(wl.head_dim)
+    stream = torch.cuda.current_stream()
+
+    def step(i, s):
+        plan.run(k_pool, v_pool, page_table, stream_table, q, scale, out, lse, s)
+
+    timing = time_steps(args, torch, world, stream, step, steady=False)
+    info = plan.info
+    launches = (1 if info.num_tc_items > 0 else 0) + (1 if info.num_warps > 0 else 0) + 1
+    return dict(ms=timing["ms"], streams=S, pages=R, bytes=decode_bytes(wl), launches=launches,
+                clocks=timing["clocks"], tc_items=int(info.num_tc_items), warp_items=int(info.num_items - info.num_tc_items))
+
+
 def bench_decode_e4m3(args, torch, dev, rank, world):
     """The serving-batch decode step over the FP8 (E4M3) cache: the same pages, plan and queries, the
     pool quantized from the bf16 one (whole blocks) in R replicas in distinct memory."""
@@ -744,7 +782,7 @@ def main():
     ap.add_argument("--impl", default="padoc", choices=["padoc", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--only", default="all", choices=["all", "decode", "prefill", "prefill_bwd", "loop",
-                                                      "chunk_prefill", "variants", "decode_e4m3"])
+                                                      "chunk_prefill", "variants", "decode_e4m3", "replicas"])
     ap.add_argument("--replicas", type=int, default=0, help="decode input replicas (0: enough to exceed 4x L2)")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-steady", action="store_true", help="skip the long back-to-back decode run")
@@ -781,6 +819,15 @@ def main():
             print(json.dumps({"decode_with_layout_streams_us": a["ms"] * 1e3, "streams": a["streams"],
                               "prefill_shuffled_ms": b["ms"], "prefill_shuffled_tflops": b["flops"] / (b["ms"] * 1e-3) / 1e12}))
         return 0
+    if args.only == "replicas":
+        for shape in ("decode_page", "dense_page"):
+            r = bench_decode_replicas(args, torch, dev, rank, world, shape)
+            if rank == 0:
+                print(json.dumps({"shape": shape, "pages": r["pages"], "streams": r["streams"], "us": r["ms"] * 1e3,
+                                  "queries_per_s": r["streams"] / (r["ms"] * 1e-3),
+                                  "hbm_frac": r["bytes"] / (r["ms"] * 1e-3) / 1e9 / load_peaks()[0]["hbm_gbs"],
+                                  "tc_items": r["tc_items"], "warp_items": r["warp_items"]}))
+        return 0
     if args.only == "decode_e4m3":
         e = bench_decode_e4m3(args, torch, dev, rank, world)
         if rank == 0:
@@ -813,6 +860,8 @@ def main():
 
     dl = None if args.only == "decode" else variant(bench_decode, layout_streams=True)
     d8 = None if args.only == "decode" else variant(bench_decode_e4m3)
+    reps = {} if args.only == "decode" else {k: variant(bench_decode_replicas, shape=k)
+                                               for k in ("decode_page", "dense_page")}
     ps = None if args.only == "decode" else variant(bench_prefill, shuffle=True)
     cp = None if args.only == "decode" else variant(bench_chunk_prefill)
     lp = None if args.only == "decode" else variant(bench_loop)
@@ -889,6 +938,27 @@ def main():
                             "(branches + layout streams; the headline counts branches only)",
                 "roofline": {"bound": "hbm", "achieved": ach, "peak": peaks["hbm_gbs"], "unit": "GB/s",
                              "frac": ach / peaks["hbm_gbs"], "traffic": None, "algorithmic_bytes": dl["bytes"]}}
+    for shape, key, desc in (("decode_page", "decode_one_page_replicas",
+                              "one-page decode shape (P = 2048 = 1792 visual + 256 prompt, layout stream 256, 16 "
+                              "branches, private KV U[16,256])"),
+                             ("dense_page", "decode_dense_page_replicas",
+                              "dense-page decode shape (P = 4096, layout stream 512, 64 branches, log-normal private "
+                              "KV, median 64, cap 1024)")):
+        r = reps.get(shape)
+        if r is None:
+            continue
+        if "error" in r:
+            line[key] = r
+            continue
+        rms = max_over_ranks(torch, world, r["ms"])
+        ach = r["bytes"] / (r["ms"] * 1e-3) / 1e9
+        line[key] = {"value": r["streams"] * world / (rms * 1e-3), "unit": "queries/s", "ms_per_step": rms,
+                     "pages": r["pages"], "streams_per_gpu": r["streams"], "clocks": r["clocks"],
+                     "tc_items": r["tc_items"], "warp_items": r["warp_items"],
+                     "workload": f"{r['pages']} replicas of the {desc}, each with its own K/V/Q in distinct memory, "
+                                 "decoded as one batch per step (the batch's cache > 4x L2)",
+                     "roofline": {"bound": "hbm", "achieved": ach, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                                  "frac": ach / peaks["hbm_gbs"], "traffic": None, "algorithmic_bytes": r["bytes"]}}
     if d8 is not None and "error" in d8:
         line["decode_e4m3"] = d8
     elif d8 is not None:

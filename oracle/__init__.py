@@ -77,6 +77,9 @@ def _load():
                                                       ctypes.c_int32, _u8p, _f32p]
             lib.oracle_dequantize_kv_blocks.argtypes = [_u8p, _f32p, ctypes.c_int64, ctypes.c_int32, ctypes.c_int32,
                                                         ctypes.c_int32, _f64p]
+            lib.oracle_prefill_dense_rows.argtypes = [_i32p, ctypes.c_int32, _i32p, _i32p, _f32p, _f32p, _f32p,
+                                                      ctypes.c_int32, ctypes.c_int32, ctypes.c_int32, ctypes.c_double,
+                                                      ctypes.c_int64, _i64p, _f64p, _f64p]
             lib.oracle_append_kv_quantized.argtypes = [_u8p, _f32p, ctypes.c_int64, ctypes.c_int32, ctypes.c_int32,
                                                        ctypes.c_int32, _i32p, ctypes.c_int32, _f32p]
             lib.oracle_decode_f64.argtypes = [ctypes.c_int32, _i32p, _i32p, _i32p, _i64p, _i64p, _f64p, _f64p,
@@ -157,6 +160,24 @@ def _prefill(fn_name, pages, q, k, v, scale):
 def prefill_dense(pages, q, k, v, scale):
     """Packed prefill via the dense ancestor visibility. Returns fp64 (O [T][Hq][d], LSE [T][Hq])."""
     return _prefill("oracle_prefill_dense", pages, q, k, v, scale)
+
+
+def prefill_dense_rows(pages, q_rows, k, v, scale, rows):
+    """``prefill_dense`` on the absolute packed rows ``rows`` only: q_rows [n][Hq][d] are those rows'
+    queries, k / v the whole packed [T][Hkv][d]. Returns fp64 (O [n][Hq][d], LSE [n][Hq])."""
+    pln, n, f, b = _flat(pages)
+    qs, k, v = _f32(q_rows), _f32(k), _f32(v)
+    r = np.ascontiguousarray(np.asarray(rows, np.int64))
+    T = total_tokens(pages)
+    assert k.shape[0] == T and v.shape == k.shape and qs.shape[0] == len(r) and ((r >= 0) & (r < T)).all()
+    Hq, d = qs.shape[1], qs.shape[2]
+    o = np.zeros((len(r), Hq, d), np.float64)
+    lse = np.zeros((len(r), Hq), np.float64)
+    if len(r):
+        _load().oracle_prefill_dense_rows(_ptr(pln, _i32p), n, _ptr(f, _i32p), _ptr(b, _i32p), _ptr(qs, _f32p),
+                                          _ptr(k, _f32p), _ptr(v, _f32p), Hq, k.shape[1], d, float(scale), len(r),
+                                          _ptr(r, _i64p), _ptr(o, _f64p), _ptr(lse, _f64p))
+    return o, lse
 
 
 def prefill_gather(pages, q, k, v, scale):

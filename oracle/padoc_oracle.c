@@ -234,6 +234,59 @@ void oracle_prefill_dense(const int32_t *pln, int32_t num_pages, const int32_t *
     }
 }
 
+/* The dense formulation on selected query rows only (sampled checks of large packed batches):
+ * rows[i] is an absolute packed row; q_sel: [n_rows][Hq][d] holds those rows' queries; k, v the whole
+ * packed [T][Hkv][d]; o: [n_rows][Hq][d], lse: [n_rows][Hq]. Each row's visible keys come from
+ * visible_by_ancestors exactly as in oracle_prefill_dense, so a selected row's result is that
+ * function's row bit for bit. */
+void oracle_prefill_dense_rows(const int32_t *pln, int32_t num_pages, const int32_t *fork, const int32_t *blen,
+                               const float *q_sel, const float *k, const float *v, int32_t Hq, int32_t Hkv, int32_t d,
+                               double scale, int64_t n_rows, const int64_t *rows, double *o, double *lse)
+{
+    const int group = Hq / Hkv;
+    /* page of each row: page starts and branch offsets */
+    int64_t *pstart = (int64_t *)malloc(sizeof(int64_t) * (size_t)(num_pages + 1));
+    int64_t *bstart = (int64_t *)malloc(sizeof(int64_t) * (size_t)(num_pages + 1));
+    pstart[0] = 0; bstart[0] = 0;
+    for (int p = 0; p < num_pages; ++p) {
+        pstart[p + 1] = pstart[p] + page_tokens(pln, blen, bstart[p], p);
+        bstart[p + 1] = bstart[p] + pln[3 * p + 2];
+    }
+#pragma omp parallel
+    {
+        int64_t cap = 0;
+        const float **kr = NULL, **vr = NULL;
+        double *sb = NULL;
+        int64_t *vis = NULL;
+#pragma omp for schedule(dynamic, 1)
+        for (int64_t i = 0; i < n_rows; ++i) {
+            int p = 0;
+            while (p + 1 < num_pages && rows[i] >= pstart[p + 1]) ++p;
+            const int64_t S = pstart[p + 1] - pstart[p], qi = rows[i] - pstart[p];
+            if (S > cap) {
+                cap = S;
+                kr = (const float **)realloc((void *)kr, sizeof(float *) * (size_t)cap);
+                vr = (const float **)realloc((void *)vr, sizeof(float *) * (size_t)cap);
+                sb = (double *)realloc(sb, sizeof(double) * (size_t)cap);
+                vis = (int64_t *)realloc(vis, sizeof(int64_t) * (size_t)cap);
+            }
+            int64_t nk = 0;
+            for (int64_t j = 0; j < S; ++j)
+                if (visible_by_ancestors(pln + 3 * p, fork + bstart[p], blen + bstart[p], qi, j)) vis[nk++] = j;
+            for (int h = 0; h < Hq; ++h) {
+                const int g = h / group;
+                for (int64_t c = 0; c < nk; ++c) {
+                    kr[c] = k + ((pstart[p] + vis[c]) * Hkv + g) * d;
+                    vr[c] = v + ((pstart[p] + vis[c]) * Hkv + g) * d;
+                }
+                lse[i * Hq + h] = attend_rows(q_sel + (i * Hq + h) * d, kr, vr, nk, d, scale, sb, o + (i * Hq + h) * d);
+            }
+        }
+        free((void *)kr); free((void *)vr); free(sb); free(vis);
+    }
+    free(pstart); free(bstart);
+}
+
 /* ------------------------------------------------------------------------------------------ */
 /* Packed prefill, formulation 2: tree-varlen gather with bottom-right causal alignment          */
 /* ------------------------------------------------------------------------------------------ */

@@ -111,3 +111,53 @@ def test_chunk_prefill_fp32_tiny():
     pg = wl.pages[0]
     spec = [(0, k, 0, pg.branch_len[k]) for k in range(pg.num_branches)] + [(0, -1, 250, 38)]
     assert_close(*run_chunks(wl, 0, spec, scale_in=1 / 8), torch.float32)
+
+
+def test_chunk_prefill_serving_batch_at_benchmark_size_sampled_rows():
+    # the benchmarked branch prefill: the 32 serving-batch pages, every branch as one chunk from its
+    # branch-initialization token and every layout stream as one shared-stream chunk (704 chunks,
+    # 115,034 query tokens), in the launch configuration the benchmark times; the first, a middle
+    # and the last token of every chunk (every page, every branch, every layout stream) against the
+    # dense oracle's rows of those tokens of the packed pages
+    wl = inputs.serving_batch(seed=3)
+    di = inputs.decode_inputs(wl, 3, pool_slack=1.0)
+    ks, vs, chunks, table, packed = [], [], [], [], []
+    base, b = 0, 0
+    for p, pg in enumerate(wl.pages):
+        lo = int(di.page_off[p])
+        ks.append(di.stream_k[lo:lo + pg.stream_len]); vs.append(di.stream_v[lo:lo + pg.stream_len])
+        yb = base + pg.stream_len
+        for f, n in zip(pg.fork_offset, pg.branch_len):
+            plo = int(di.priv_off[b])
+            ks.append(di.priv_k[plo:plo + n]); vs.append(di.priv_v[plo:plo + n])
+            chunks.append((p, pg.prefix_len + f, 0, n))
+            table.append(di.stream_table[b])
+            packed.append(np.arange(yb, yb + n))
+            yb += n
+            b += 1
+        chunks.append((p, pg.prefix_len, -1, pg.layout_len))
+        table.append(np.full(di.stream_table.shape[1], -1, np.int32))
+        packed.append(np.arange(base + pg.prefix_len, base + pg.stream_len))
+        base += pg.packed_len
+    K, V = torch.cat(ks), torch.cat(vs)
+    page_len = np.array([pg.stream_len for pg in wl.pages], np.int32)
+    plan = ChunkPrefillPlan(page_len, chunks, np.stack(table), 16, 2, 128, DEV)
+    T = plan.num_tokens
+    assert len(chunks) == 704 and T == 115034
+    q = inputs.randn((T, 16, 128), torch.bfloat16, 3 * 1000 + 98)
+    out = torch.full((T, 16, 128), float("nan"), dtype=torch.bfloat16, device=DEV)
+    lse = torch.full((T, 16), float("nan"), dtype=torch.float32, device=DEV)
+    scale = 1.0 / math.sqrt(128)
+    plan.run(di.k_pool.to(DEV), di.v_pool.to(DEV), torch.from_numpy(di.page_table).to(DEV), q.to(DEV), scale, out, lse)
+    pa.padoc_check_device_errors()
+    tok, rows, t0 = [], [], 0
+    for c, rr in zip(chunks, packed):
+        n = c[3]
+        for i in sorted({0, n // 2, n - 1}):
+            tok.append(t0 + i)
+            rows.append(int(rr[i]))
+        t0 += n
+    tok = np.array(tok)
+    ref_o, ref_l = oracle.prefill_dense_rows(wl.pages, q[torch.from_numpy(tok)], K, V, scale, np.array(rows))
+    got_o, got_l = out[torch.from_numpy(tok).to(DEV)].float().cpu().numpy(), lse[torch.from_numpy(tok).to(DEV)].cpu().numpy()
+    assert_close(got_o, got_l, ref_o, ref_l, torch.bfloat16)

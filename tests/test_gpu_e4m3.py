@@ -117,8 +117,8 @@ def test_quantize_ties_saturation_and_subnormals_bit_exact():
 def test_append_rows_bit_exact_against_oracle_rule():
     # 12 blocks filled over 20 steps; each step appends one row to each of a subset of the blocks
     # (distinct blocks within a call), rows in order inside a block; magnitudes grow and shrink so
-    # that scales grow (re-encoding earlier rows) and stay; blocks 0-3 hold stale codes and scales
-    # from a former owner and are started afresh at row 0; a zero row and a block of zero rows
+    # that scales grow (re-encoding earlier rows) and stay; every block starts with stale codes and
+    # scales from a former owner and is started afresh at row 0; a zero row and a block of zero rows
     rng = np.random.default_rng(12)
     nb, hkv, d = 12, 2, 128
     kc0 = rng.integers(0, 0x7E, (nb, hkv, 16, d)).astype(np.uint8)
@@ -204,15 +204,19 @@ def test_decode_e4m3_tensor_core_ctas_walk_many_pieces(tc_ctas, warp_ctas):
 
 
 def test_decode_e4m3_scales_that_differ_block_by_block():
-    # every block of the cache gets its own magnitude (scales over four orders of magnitude), and
-    # some blocks are all zero (scale 0): the per-block K multipliers and V factors must follow
+    # every block of the cache gets its own magnitude, so scales differ block by block (K over e^-3
+    # .. e^1, V over e^-3 .. 1, independently), and some K blocks are all zero (scale 0): the per-
+    # block K multipliers and V factors must follow. Magnitudes stay at most those of the N(0,1)
+    # workloads' (|V| up to ~4.5) so that the bf16 path's absolute tolerances still apply: the
+    # outputs' own bf16 rounding grows with |V|.
     wl = inputs.dense_page()
     di = inputs.decode_inputs(wl, 65)
     rng = np.random.default_rng(65)
-    mag = torch.from_numpy(np.exp(rng.uniform(-4, 4, (di.num_blocks, 1, 1, 1))).astype(np.float32))
-    zero = torch.from_numpy(rng.random((di.num_blocks, 1, 1, 1)) < 0.05)
-    di.k_pool = (di.k_pool.float() * mag).masked_fill(zero, 0.0).to(torch.bfloat16)
-    di.v_pool = (di.v_pool.float() * mag.flip(0)).to(torch.bfloat16)
+    kmag = torch.from_numpy(np.exp(rng.uniform(-3, 1, (di.num_blocks, 2, 1, 1))).astype(np.float32))
+    vmag = torch.from_numpy(np.exp(rng.uniform(-3, 0, (di.num_blocks, 2, 1, 1))).astype(np.float32))
+    zero = torch.from_numpy(rng.random((di.num_blocks, 2, 1, 1)) < 0.05)
+    di.k_pool = (di.k_pool.float() * kmag).masked_fill(zero, 0.0).to(torch.bfloat16)
+    di.v_pool = (di.v_pool.float() * vmag).to(torch.bfloat16)
     pool = pa.E4M3Pool(di.num_blocks, 2, 128, DEV)
     pa.padoc_quantize_kv_blocks(pool, di.k_pool.to(DEV), di.v_pool.to(DEV),
                                 torch.arange(di.num_blocks, dtype=torch.int32, device=DEV))

@@ -740,3 +740,16 @@ def test_decode_f64_and_paged_decode_equal_the_fp32_row_decode():
                                  layout_streams=True)
     np.testing.assert_array_equal(op, o32)
     np.testing.assert_array_equal(lp, l32)
+
+
+def test_prefill_dense_rows_is_the_dense_prefill_on_those_rows():
+    # the row-selected form reads the same visibility and does the same arithmetic per row, so its
+    # rows are bit-identical to the full function's (itself pinned above)
+    pages = [(13, 9, [3, 9, 0], [4, 6, 2]), (0, 5, [5, 1], [3, 7]), (20, 0, [0], [5])]
+    T = oracle.total_tokens(pages)
+    q, k, v = _qkv(T, 4, 2, 8, seed=21)
+    o_all, l_all = oracle.prefill_dense(pages, q, k, v, 0.3)
+    rows = np.array([0, 5, 21, 22, 25, 33, T - 1, 40, 41], np.int64)
+    o, l = oracle.prefill_dense_rows(pages, q[rows], k, v, 0.3, rows)
+    np.testing.assert_array_equal(o, o_all[rows])
+    np.testing.assert_array_equal(l, l_all[rows])
