@@ -278,58 +278,58 @@ def bench_decode(args, torch, dev, rank, world, layout_streams=False):
     if args.no_e2e or layout_streams:
         return res
 
-    # end to end through the public API: host C1 plan, host->device copies of the step's inputs
-    # (plan blob, block tables, queries, from pinned memory), the decode, and the read-back of O/LSE
+    # end to end through the public API, every step: the plan brought to the step's lengths
+    # (padoc_advance_decode_plan, which checks and patches the host plan in place; this batch's
+    # lengths do not change from step to step, so nothing moves), and one library call that copies
+    # the step's integers (plan blob, page and stream block tables) and queries from pinned host
+    # memory to the device, decodes, and copies O and LSE back to pinned host memory. Two staging
+    # buffers: the host prepares step i+1 while step i's copies may still read the other one.
+    PT, STW = di.page_table.shape[1], di.stream_table.shape[1]
+    align = lambda n: (n + 31) // 32 * 32
+    plan_ints = int(plan.info.plan_ints)
+    off_pt = align(plan_ints)
+    off_st = off_pt + align(len(wl.pages) * PT)
+    words = off_st + align(S * STW)
+    stages = [torch.zeros(words, dtype=torch.int32).pin_memory() for _ in range(2)]
+    infos = []
+    for st in stages:
+        h = st.numpy()
+        h[:plan_ints] = plan.plan_host
+        h[off_pt:off_pt + len(wl.pages) * PT] = di.page_table.reshape(-1)
+        h[off_st:off_st + S * STW] = di.stream_table.reshape(-1)
+        infos.append(pa.padoc_decode_plan.from_buffer_copy(plan.info))
+    stage_free = [torch.cuda.Event(), torch.cuda.Event()]
+    dev_ints = torch.empty(words, dtype=torch.int32, device=dev)
     q_host = di.q.pin_memory()
-    pt_host = torch.from_numpy(di.page_table).pin_memory()
-    st_host = torch.from_numpy(di.stream_table).pin_memory()
+    q_dev = torch.empty_like(qs[0])
     o_host = torch.empty((S, wl.num_q_heads, wl.head_dim), dtype=torch.bfloat16).pin_memory()
     l_host = torch.empty((S, wl.num_q_heads), dtype=torch.float32).pin_memory()
-    q_dev = torch.empty_like(qs[0])
-    pt_dev, st_dev = torch.empty_like(page_table), torch.empty_like(stream_table)
-    cfg = plan.cfg
-    plan_dev = torch.empty(int(plan.info.plan_ints), dtype=torch.int32, device=dev)
-
-    # two pinned plan buffers: the host builds step i+1's plan into one while step i's copy from the
-    # other may still be in flight (an event per buffer says when it may be overwritten)
-    blob_pinned = [torch.empty(int(plan.info.plan_ints) + 4096, dtype=torch.int32).pin_memory() for _ in range(2)]
-    blob_np = [b.numpy() for b in blob_pinned]
-    blob_free = [torch.cuda.Event(), torch.cuda.Event()]
-
-    # the page records stay in one native array (a serving loop updates its lengths in place); the
-    # planner runs every step
-    page_array = pa.PageArray(wl.pages)
+    lens = np.ascontiguousarray(plan.plan_host[plan.info.off_private_len:plan.info.off_private_len + S])
 
     def e2e_step(i):
         r = i % R
         b = i & 1
-        blob_free[b].synchronize()
-        blob, info = pa.padoc_build_decode_plan(page_array, cfg, out=blob_np[b])
-        blob_t = blob_pinned[b][: blob.size]
-        plan_dev[: blob.size].copy_(blob_t, non_blocking=True)
-        blob_free[b].record(stream)
-        q_dev.copy_(q_host, non_blocking=True)
-        pt_dev.copy_(pt_host, non_blocking=True)
-        st_dev.copy_(st_host, non_blocking=True)
-        pa.padoc_branch_decode_attn(k_pools[r], v_pools[r], info, plan_dev, pt_dev, st_dev, q_dev, scale, outs[r],
-                                    lses[r], plan.workspace, stream)
-        o_host.copy_(outs[r], non_blocking=True)
-        l_host.copy_(lses[r], non_blocking=True)
-        return blob_t.numel() * 4
+        stage_free[b].synchronize()
+        h = stages[b].numpy()
+        if not pa.padoc_advance_decode_plan(h[:plan_ints], infos[b], lens):
+            raise RuntimeError("plan advance refused")
+        pa.padoc_launch_decode_step(k_pools[r], v_pools[r], infos[b], stages[b], words, off_pt, PT, off_st, STW,
+                                    dev_ints, q_host, q_dev, scale, outs[r], lses[r], o_host, l_host, plan.workspace,
+                                    stream)
+        stage_free[b].record(stream)
 
     for i in range(max(args.warmup, 1)):
         e2e_step(i)
     torch.cuda.synchronize()
     barrier(torch, world)
     t0 = time.perf_counter()
-    blob_bytes = 0
-    e2e_steps = min(args.steps, 500)
+    e2e_steps = min(args.steps, 2000)
     for i in range(e2e_steps):
-        blob_bytes = e2e_step(i)
+        e2e_step(i)
     torch.cuda.synchronize()
     e2e_ms = (time.perf_counter() - t0) * 1e3 / e2e_steps
     barrier(torch, world)
-    h2d = blob_bytes + q_host.numel() * 2 + pt_host.numel() * 4 + st_host.numel() * 4
+    h2d = words * 4 + q_host.numel() * 2
     d2h = o_host.numel() * 2 + l_host.numel() * 4
     res.update(e2e_ms=e2e_ms, h2d=h2d, d2h=d2h)
     return res

@@ -48,8 +48,8 @@ extern "C" {
 
 /* 1: descriptors, decode, prefill, combine, prefill backward, no-alloc decode. 2 adds the
  * stream-list and chunked-prefill planners, Algorithm 1's loop (padoc_mpd_*) and the append call.
- * 3 adds the FP8 (E4M3) KV cache (padoc_kv_pool_e4m3 and its quantize, append and decode calls)
- * and the bounded-wait self-test. */
+ * 3 adds the FP8 (E4M3) KV cache (padoc_kv_pool_e4m3 and its quantize, append and decode calls),
+ * the bounded-wait self-test, the in-place plan advance and the one-call decode step. */
 #define PADOC_ATTN_VERSION 3
 
 /* A CUDA stream handle; identical to cudaStream_t. */
@@ -272,6 +272,35 @@ padoc_status padoc_branch_decode_attn(const padoc_kv_pool *pool, const padoc_dec
                                       int32_t stream_table_stride, const void *q, float scale, void *out,
                                       float *lse, void *workspace, size_t workspace_bytes,
                                       padoc_stream_t stream);
+
+/* Patches a plan built by the planners above, and its host summary, for new private lengths of
+ * the same streams (a decoding loop's steady state: every stream appends one token per step and
+ * nothing forks or retires): private_len (host) int32 [num_streams] with num_streams =
+ * info->num_streams. Each stream keeps its work items and partial slots; the private item that
+ * ended at its old length (one per KV head) now ends at the new one, so the plan covers every
+ * visible row exactly once as before. O(streams + items). plan is the host copy of the blob (copy
+ * it to the device again). Returns CAPACITY, changing nothing, when the patch does not apply (a
+ * length below the old one, a stream that had no private rows, an item that would exceed the warp
+ * kernel's item length, a chunked-prefill plan): then build a new plan. The stream block table must
+ * cover the new lengths (info->max_stream_blocks is updated). Errors: INVALID_ARGUMENT, CAPACITY. */
+padoc_status padoc_advance_decode_plan(int32_t *plan, padoc_decode_plan *info, const int32_t *private_len,
+                                       int32_t num_streams);
+
+/* One decode step for a caller whose step inputs live in host memory, all on `stream` with no host
+ * synchronization: copies stage[0, stage_words) ((host) int32, pinned for an asynchronous copy: the
+ * plan blob at word 0, the page block table at off_page_table and the stream block table at
+ * off_stream_table, each offset a multiple of 32 words past the blob) to dev_ints ((device) int32
+ * [dev_capacity_words], 256-byte aligned) and q_host ((host) [num_streams][Hq][head_dim] in the pool
+ * dtype) to q_dev (device, same size), runs padoc_branch_decode_attn on them, then copies out_dev and
+ * lse_dev into out_host and lse_host ((host), same sizes). The host buffers must stay unchanged
+ * (inputs) or unread (results) until the stream has run the copies.
+ * Errors: INVALID_ARGUMENT, and those of padoc_branch_decode_attn. */
+padoc_status padoc_launch_decode_step(const padoc_kv_pool *pool, const padoc_decode_plan *info, const int32_t *stage,
+                                      int64_t stage_words, int64_t off_page_table, int32_t page_table_stride,
+                                      int64_t off_stream_table, int32_t stream_table_stride, int32_t *dev_ints,
+                                      int64_t dev_capacity_words, const void *q_host, void *q_dev, float scale,
+                                      void *out_dev, float *lse_dev, void *out_host, float *lse_host, void *workspace,
+                                      size_t workspace_bytes, padoc_stream_t stream);
 
 /* Size of the device array that padoc_branch_decode_attn_noalloc uses as its workspace. */
 #define PADOC_STATIC_WORKSPACE_BYTES (32u << 20)

@@ -716,6 +716,45 @@ extern "C" padoc_status padoc_branch_decode_attn_e4m3(const padoc_kv_pool_e4m3 *
                           stream_table_stride, q, scale, out, lse, workspace, workspace_bytes, (cudaStream_t)stream);
 }
 
+extern "C" padoc_status padoc_launch_decode_step(const padoc_kv_pool *pool, const padoc_decode_plan *info,
+                                                 const int32_t *stage, int64_t stage_words, int64_t off_page_table,
+                                                 int32_t page_table_stride, int64_t off_stream_table,
+                                                 int32_t stream_table_stride, int32_t *dev_ints,
+                                                 int64_t dev_capacity_words, const void *q_host, void *q_dev,
+                                                 float scale, void *out_dev, float *lse_dev, void *out_host,
+                                                 float *lse_host, void *workspace, size_t workspace_bytes,
+                                                 padoc_stream_t stream)
+{
+    if (!pool || !info || !stage || !dev_ints || !q_host || !q_dev || !out_dev || !lse_dev || !out_host || !lse_host)
+        return PADOC_ERR_INVALID_ARGUMENT;
+    const int64_t P = info->num_pages, S = info->num_streams;
+    if (stage_words < info->plan_ints || dev_capacity_words < stage_words) return PADOC_ERR_INVALID_ARGUMENT;
+    if ((((uintptr_t)dev_ints) & 255) || (off_page_table & 31) || (off_stream_table & 31)) return PADOC_ERR_INVALID_ARGUMENT;
+    if (page_table_stride < 1 || stream_table_stride < 1) return PADOC_ERR_INVALID_ARGUMENT;
+    if (off_page_table < info->plan_ints || off_page_table + P * page_table_stride > stage_words ||
+        off_stream_table < info->plan_ints || off_stream_table + S * stream_table_stride > stage_words)
+        return PADOC_ERR_INVALID_ARGUMENT;
+    const bool overlap = off_page_table < off_stream_table ? off_page_table + P * page_table_stride > off_stream_table
+                                                           : off_stream_table + S * stream_table_stride > off_page_table;
+    if (P > 0 && S > 0 && overlap) return PADOC_ERR_INVALID_ARGUMENT;
+    const size_t esz = pool->dtype == PADOC_DTYPE_BF16 ? 2 : 4;
+    const size_t q_bytes = (size_t)S * info->cfg.num_q_heads * info->cfg.head_dim * esz;
+    const size_t lse_bytes = (size_t)S * info->cfg.num_q_heads * sizeof(float);
+    if (S == 0) return PADOC_OK;
+    cudaStream_t cs = (cudaStream_t)stream;
+    // the step's integers and queries in (pinned host memory makes both copies asynchronous)
+    PADOC_CUDA_TRY(cudaMemcpyAsync(dev_ints, stage, (size_t)stage_words * sizeof(int32_t), cudaMemcpyHostToDevice, cs));
+    PADOC_CUDA_TRY(cudaMemcpyAsync(q_dev, q_host, q_bytes, cudaMemcpyHostToDevice, cs));
+    const padoc_status st = padoc_branch_decode_attn(pool, info, dev_ints, dev_ints + off_page_table, page_table_stride,
+                                                     dev_ints + off_stream_table, stream_table_stride, q_dev, scale,
+                                                     out_dev, lse_dev, workspace, workspace_bytes, stream);
+    if (st != PADOC_OK) return st;
+    // and the results out
+    PADOC_CUDA_TRY(cudaMemcpyAsync(out_host, out_dev, q_bytes, cudaMemcpyDeviceToHost, cs));
+    PADOC_CUDA_TRY(cudaMemcpyAsync(lse_host, lse_dev, lse_bytes, cudaMemcpyDeviceToHost, cs));
+    return PADOC_OK;
+}
+
 extern "C" padoc_status padoc_splitk_combine(const float *part_o, const float *part_lse, int32_t num_splits,
                                              int64_t rows, int32_t head_dim, padoc_dtype out_dtype, void *out,
                                              float *lse, padoc_stream_t stream)

@@ -846,6 +846,60 @@ extern "C" padoc_status padoc_decode_workspace_size(const padoc_decode_plan *inf
     return PADOC_OK;
 }
 
+// Patches a decode plan for new private lengths (the decoding loop's steady state: every stream
+// appends one token per step, nothing forks or retires). Each stream's work stays where it is; the
+// private item that ends at a stream's old length (one per KV head) is extended to the new one,
+// which is allowed while the item stays within PADOC_WARP_MAX_ITEM_TOKENS (the planner cuts private
+// histories at PADOC_PRIVATE_SPLIT_TOKENS, which leaves that much room to grow). Anything else
+// (a shorter length, a stream that had no private rows, an item past the limit, a chunked-prefill
+// plan) asks for a new plan.
+extern "C" padoc_status padoc_advance_decode_plan(int32_t *plan, padoc_decode_plan *info, const int32_t *private_len,
+                                                  int32_t num_streams)
+{
+    if (!plan || !info || (num_streams > 0 && !private_len)) return PADOC_ERR_INVALID_ARGUMENT;
+    if (num_streams != info->num_streams) return PADOC_ERR_INVALID_ARGUMENT;
+    const int32_t S = info->num_streams;
+    const int32_t Hkv = info->cfg.num_kv_heads;
+    if (Hkv < 1 || info->num_items < info->num_tc_items || info->num_tc_items < 0) return PADOC_ERR_INVALID_ARGUMENT;
+    int32_t *old_len = plan + info->off_private_len;
+    padoc_item *items = reinterpret_cast<padoc_item *>(plan + info->off_items);
+    int64_t grow = 0;
+    int32_t max_blocks = info->max_stream_blocks;
+    for (int32_t s = 0; s < S; ++s) {
+        const int32_t n = private_len[s], o = old_len[s];
+        if (n < o || n >= (1 << 30)) return PADOC_ERR_CAPACITY;
+        if (n > o && o == 0) return PADOC_ERR_CAPACITY;   // no private item to extend
+        grow += n - o;
+        max_blocks = std::max(max_blocks, (n + info->cfg.block_size - 1) / info->cfg.block_size);
+    }
+    for (int32_t i = 0; i < info->num_tc_items; ++i)
+        if (PADOC_ITEM_KIND(items[i].kind) == PADOC_ITEM_PRIVATE_TC) return PADOC_ERR_CAPACITY;
+    if (grow == 0) return PADOC_OK;
+    // the items to extend: a private item of stream s whose end is s's old length (checked first,
+    // changed after, so that a refusal leaves the plan as it was)
+    int64_t extended = 0;
+    for (int32_t i = info->num_tc_items; i < info->num_items; ++i) {
+        const padoc_item &it = items[i];
+        if (it.kind != PADOC_ITEM_PRIVATE || it.index < 0 || it.index >= S) continue;
+        const int32_t s = it.index;
+        if (it.tok_end != old_len[s] || private_len[s] == old_len[s]) continue;
+        if (private_len[s] - it.tok_begin > PADOC_WARP_MAX_ITEM_TOKENS) return PADOC_ERR_CAPACITY;
+        ++extended;
+    }
+    int64_t want = 0;
+    for (int32_t s = 0; s < S; ++s) want += (private_len[s] != old_len[s]) ? Hkv : 0;
+    if (extended != want) return PADOC_ERR_CAPACITY;
+    for (int32_t i = info->num_tc_items; i < info->num_items; ++i) {
+        padoc_item &it = items[i];
+        if (it.kind == PADOC_ITEM_PRIVATE && it.index >= 0 && it.index < S && it.tok_end == old_len[it.index])
+            it.tok_end = private_len[it.index];
+    }
+    for (int32_t s = 0; s < S; ++s) old_len[s] = private_len[s];
+    info->max_stream_blocks = max_blocks;
+    info->kv_tokens += grow;
+    return PADOC_OK;
+}
+
 extern "C" padoc_status padoc_chunk_prefill_plan_size(const int32_t *page_len, int32_t num_pages,
                                                       const padoc_prefill_chunk *chunks, int32_t num_chunks,
                                                       const padoc_decode_config *cfg, int64_t *plan_ints)

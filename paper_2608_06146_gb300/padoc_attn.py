@@ -166,6 +166,11 @@ def load_library(path: Optional[str] = None):
                                   _vp, _vp, ctypes.c_size_t, _vp],
         "padoc_selftest_tcgen05": [_vp, _vp, _vp, _vp, _vp, _vp, _vp],
         "padoc_selftest_wait_timeout": [ctypes.c_int32, ctypes.c_int32, _vp, _vp],
+        "padoc_advance_decode_plan": [_i32p, ctypes.POINTER(padoc_decode_plan), _i32p, ctypes.c_int32],
+        "padoc_launch_decode_step": [ctypes.POINTER(padoc_kv_pool), ctypes.POINTER(padoc_decode_plan), _vp,
+                                     ctypes.c_int64, ctypes.c_int64, ctypes.c_int32, ctypes.c_int64, ctypes.c_int32,
+                                     _vp, ctypes.c_int64, _vp, _vp, ctypes.c_float, _vp, _vp, _vp, _vp, _vp,
+                                     ctypes.c_size_t, _vp],
         "padoc_quantize_kv_blocks": [ctypes.POINTER(padoc_kv_pool_e4m3), _vp, _vp, _vp, ctypes.c_int32, _vp],
         "padoc_append_inputs_e4m3": [ctypes.POINTER(padoc_kv_pool_e4m3), _vp, _vp, _vp, ctypes.c_int64, ctypes.c_int32,
                                      _vp, _vp, _vp, ctypes.c_int32, _vp],
@@ -205,6 +210,7 @@ def exported_symbols() -> Sequence[str]:
                         "padoc_append_inputs",
                         "padoc_selftest_tcgen05", "padoc_selftest_wait_timeout",
                         "padoc_quantize_kv_blocks", "padoc_append_inputs_e4m3", "padoc_branch_decode_attn_e4m3",
+                        "padoc_advance_decode_plan", "padoc_launch_decode_step",
                         "padoc_check_device_errors",
                         "padoc_last_device_error", "padoc_status_string", "padoc_version")]
 
@@ -500,6 +506,37 @@ def padoc_branch_decode_attn(k_pool, v_pool, info: padoc_decode_plan, plan_dev, 
                                       _dev(stream_table, "stream_table"), stream_table.shape[1], _dev(q, "q"),
                                       float(scale), _dev(out, "out"), _dev(lse, "lse"), ws, wsb, _stream_ptr(stream))
     _check("padoc_branch_decode_attn", st)
+
+
+def padoc_advance_decode_plan(plan, info: padoc_decode_plan, private_len) -> bool:
+    """Patches ``plan`` (int32 numpy host blob) and ``info`` in place for new private lengths of the
+    same streams; False (nothing changed) when a new plan is needed."""
+    lib = load_library()
+    pl = np.ascontiguousarray(np.asarray(private_len, np.int32))
+    st = lib.padoc_advance_decode_plan(plan.ctypes.data_as(_i32p), ctypes.byref(info), pl.ctypes.data_as(_i32p),
+                                       pl.size)
+    if st == 6:
+        return False
+    _check("padoc_advance_decode_plan", st)
+    return True
+
+
+def padoc_launch_decode_step(k_pool, v_pool, info: padoc_decode_plan, stage, stage_words: int, off_page_table: int,
+                             page_stride: int, off_stream_table: int, stream_stride: int, dev_ints, q_host, q_dev,
+                             scale, out_dev, lse_dev, out_host, lse_host, workspace, stream=None):
+    """One decode step from host inputs: stage (pinned int32 CPU tensor: plan blob, page table, stream
+    table), q_host (pinned) -> device, decode, out / lse -> out_host / lse_host (pinned); no sync."""
+    lib = load_library()
+    pool = padoc_kv_pool(_dev(k_pool, "k_pool"), _dev(v_pool, "v_pool"), k_pool.shape[0], k_pool.shape[2],
+                         k_pool.shape[1], k_pool.shape[3], _dtype_code(k_pool))
+    st = lib.padoc_launch_decode_step(ctypes.byref(pool), ctypes.byref(info), stage.data_ptr(), int(stage_words),
+                                      int(off_page_table), int(page_stride), int(off_stream_table), int(stream_stride),
+                                      _dev(dev_ints, "dev_ints"), dev_ints.numel(), q_host.data_ptr(),
+                                      _dev(q_dev, "q_dev"), float(scale), _dev(out_dev, "out_dev"),
+                                      _dev(lse_dev, "lse_dev"), out_host.data_ptr(), lse_host.data_ptr(),
+                                      _dev(workspace, "workspace"), workspace.numel() * workspace.element_size(),
+                                      _stream_ptr(stream))
+    _check("padoc_launch_decode_step", st)
 
 
 PADOC_STATIC_WORKSPACE_BYTES = 32 << 20

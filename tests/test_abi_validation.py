@@ -132,3 +132,19 @@ def test_e4m3_calls_reject_malformed_calls(lib):
     assert app(_pool8(), count=0) == 0
     assert app(_pool8(), slots=None) == 1 and app(_pool8(), qs=A, qd=None) == 1
     assert app(_pool8(d=64)) == 2
+
+
+def test_launch_decode_step_rejects_malformed_calls(lib):
+    info = _decode_info(lib)
+    words = 4096
+    call = lambda stage=A, sw=words, opt=2048, pts=8, ost=3072, sts=8, dev=A, dcap=words, qh=A: lib.padoc_launch_decode_step(
+        ctypes.byref(_pool()), ctypes.byref(info), stage, sw, opt, pts, ost, sts, dev, dcap, qh, A, 0.1, A, A, A, A, A,
+        1 << 20, None)
+    assert call(stage=None) == 1 and call(qh=None) == 1 and call(dev=None) == 1
+    assert call(sw=info.plan_ints - 1) == 1                  # the stage must hold the blob
+    assert call(dcap=words - 1) == 1                         # the device buffer must hold the stage
+    assert call(dev=A + 128) == 1                            # 256-byte aligned device buffer
+    assert call(opt=2047) == 1 and call(ost=3073) == 1       # tables on 128-byte boundaries
+    assert call(opt=0) == 1                                  # tables after the blob
+    assert call(ost=2048) == 1                               # tables must not overlap
+    assert call(opt=4064, pts=64) == 1                       # a table past the stage

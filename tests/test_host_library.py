@@ -353,3 +353,82 @@ def test_header_is_plain_c_and_links_from_c(tmp_path):
                            "-lpadoc_attn", f"-Wl,-rpath,{libdir}", "-o", str(exe)])
     out = subprocess.run([str(exe)], capture_output=True, text=True, check=True).stdout.split()
     assert out == ["0", "73", "1", "3", "61", "ok"]   # 40 + 8 + 5 + 20 tokens; one page, 3 streams; 3 prefix blocks taken
+
+
+def _coverage(plan, info, sp, sh, pl, Hkv):
+    """every visible (stream, KV head) row read exactly once; slots 0..n-1 of each key used once"""
+    S = len(sp)
+    items = _plan_items(plan, info)
+    slot_ptr = plan[info.off_slot_ptr: info.off_slot_ptr + S * Hkv + 1]
+    cov_sh = {(s, g): np.zeros(sh[s], np.int32) for s in range(S) for g in range(Hkv)}
+    cov_pv = {(s, g): np.zeros(pl[s], np.int32) for s in range(S) for g in range(Hkv)}
+    used = {(s, g): [] for s in range(S) for g in range(Hkv)}
+    for kind, idx, g, tb, te, fs, ns, slot in items:
+        for s in range(fs, fs + ns):
+            if (kind & 15) in (0, 2):
+                hi = min(te, sh[s])
+                if hi > tb:
+                    cov_sh[(s, g)][tb:hi] += 1
+            else:
+                assert te <= pl[s] and te - tb <= 512
+                cov_pv[(s, g)][tb:te] += 1
+            used[(s, g)].append(slot)
+    for (s, g) in cov_sh:
+        assert np.all(cov_sh[(s, g)] == 1) and np.all(cov_pv[(s, g)] == 1)
+        assert sorted(used[(s, g)]) == list(range(slot_ptr[s * Hkv + g + 1] - slot_ptr[s * Hkv + g]))
+
+
+def test_advance_decode_plan_patches_lengths_and_keeps_the_work_in_place():
+    wl = inputs.serving_batch(num_pages=8)
+    cfg = pa.make_decode_config(16, 2, 128, 16, True, 0, 40, 40)
+    plan, info = pa.padoc_build_decode_plan(wl.pages, cfg)
+    plan = plan.copy()
+    sp, sh, pl = oracle.decode_streams(wl.pages, True)
+    before, info0 = plan.copy(), pa.padoc_decode_plan.from_buffer_copy(info)
+    # nothing changed: the plan is the planner's, bit for bit
+    assert pa.padoc_advance_decode_plan(plan, info, pl)
+    np.testing.assert_array_equal(plan, before)
+    assert bytes(info) == bytes(info0)
+    # every branch grows by 1 .. 200 tokens over several steps; the layout streams keep no private rows
+    rng = np.random.default_rng(3)
+    cur = pl.copy()
+    for step in range(6):
+        grow = np.where(cur > 0, rng.integers(1, 40, size=len(cur)), 0).astype(np.int32)
+        new = cur + grow
+        assert pa.padoc_advance_decode_plan(plan, info, new)
+        cur = new
+        np.testing.assert_array_equal(plan[info.off_private_len: info.off_private_len + len(sp)], cur)
+        _coverage(plan, info, sp, sh, cur, 2)
+        assert info.max_stream_blocks == max(-(-int(x) // 16) for x in cur)
+        assert info.kv_tokens == info0.kv_tokens + int((cur - pl).sum())
+    # only the private items' ends and the private lengths moved
+    items0, items1 = _plan_items(before, info0), _plan_items(plan, info)
+    assert np.array_equal(items0[:, [0, 1, 2, 3, 5, 6, 7]], items1[:, [0, 1, 2, 3, 5, 6, 7]])
+    moved = items0[:, 4] != items1[:, 4]
+    assert np.all(items0[moved, 0] == 1)
+    # the same lengths again after a full build of the grown batch: coverage holds for both
+    grown = [inputs.PageSpec(pg.prefix_len, pg.layout_len, pg.fork_offset, []) for pg in wl.pages]
+    s = 0
+    for g, pg in zip(grown, wl.pages):
+        g.branch_len = [int(x) for x in cur[s:s + pg.num_branches]]
+        s += pg.num_branches + 1
+    fresh, finfo = pa.padoc_build_decode_plan(grown, cfg)
+    _coverage(fresh, finfo, sp, sh, cur, 2)
+
+
+def test_advance_decode_plan_refuses_and_changes_nothing():
+    wl = inputs.serving_batch(num_pages=4)
+    cfg = pa.make_decode_config(16, 2, 128, 16, True, 0, 16, 16)
+    plan, info = pa.padoc_build_decode_plan(wl.pages, cfg)
+    plan = plan.copy()
+    sp, sh, pl = oracle.decode_streams(wl.pages, True)
+    before, info0 = plan.copy(), bytes(info)
+    shorter = pl.copy(); shorter[0] -= 1
+    lay = pl.copy(); lay[np.nonzero(pl == 0)[0][0]] = 1            # a layout stream has no private item
+    long_ = pl.copy(); long_[0] = pl[0] + 600                        # past the warp kernel's item length
+    for bad in (shorter, lay, long_):
+        assert not pa.padoc_advance_decode_plan(plan, info, bad)
+        np.testing.assert_array_equal(plan, before)
+        assert bytes(info) == info0
+    with pytest.raises(pa.PadocError):
+        pa.padoc_advance_decode_plan(plan, info, pl[:-1])           # a wrong stream count
