@@ -282,43 +282,49 @@ def bench_decode(args, torch, dev, rank, world, layout_streams=False):
     # (padoc_advance_decode_plan, which checks and patches the host plan in place; this batch's
     # lengths do not change from step to step, so nothing moves), and one library call that copies
     # the step's integers (plan blob, page and stream block tables) and queries from pinned host
-    # memory to the device, decodes, and copies O and LSE back to pinned host memory. Two staging
-    # buffers: the host prepares step i+1 while step i's copies may still read the other one.
+    # memory to the device, decodes, and copies O and LSE back to pinned host memory. Two buffer
+    # sets used in turn and two copy streams: a step's copies in overlap the previous step's decode,
+    # its copies out the next step's (the library orders them with the set's events).
     PT, STW = di.page_table.shape[1], di.stream_table.shape[1]
     align = lambda n: (n + 31) // 32 * 32
     plan_ints = int(plan.info.plan_ints)
     off_pt = align(plan_ints)
     off_st = off_pt + align(len(wl.pages) * PT)
     words = off_st + align(S * STW)
-    stages = [torch.zeros(words, dtype=torch.int32).pin_memory() for _ in range(2)]
-    infos = []
-    for st in stages:
-        h = st.numpy()
+    copy_in, copy_out = torch.cuda.Stream(), torch.cuda.Stream()
+    sets = []
+    for _ in range(2):
+        stage = torch.zeros(words, dtype=torch.int32).pin_memory()
+        h = stage.numpy()
         h[:plan_ints] = plan.plan_host
         h[off_pt:off_pt + len(wl.pages) * PT] = di.page_table.reshape(-1)
         h[off_st:off_st + S * STW] = di.stream_table.reshape(-1)
-        infos.append(pa.padoc_decode_plan.from_buffer_copy(plan.info))
-    stage_free = [torch.cuda.Event(), torch.cuda.Event()]
-    dev_ints = torch.empty(words, dtype=torch.int32, device=dev)
-    q_host = di.q.pin_memory()
-    q_dev = torch.empty_like(qs[0])
-    o_host = torch.empty((S, wl.num_q_heads, wl.head_dim), dtype=torch.bfloat16).pin_memory()
-    l_host = torch.empty((S, wl.num_q_heads), dtype=torch.float32).pin_memory()
+        evs = [torch.cuda.Event() for _ in range(3)]
+        for e in evs:            # created (and ev_free set) before the first step
+            e.record(stream)
+        sets.append(dict(stage=stage, info=pa.padoc_decode_plan.from_buffer_copy(plan.info),
+                         dev_ints=torch.empty(words, dtype=torch.int32, device=dev),
+                         q_host=di.q.pin_memory(), q_dev=torch.empty_like(qs[0]),
+                         out=torch.empty_like(outs[0]), lse=torch.empty_like(lses[0]),
+                         o_host=torch.empty((S, wl.num_q_heads, wl.head_dim), dtype=torch.bfloat16).pin_memory(),
+                         l_host=torch.empty((S, wl.num_q_heads), dtype=torch.float32).pin_memory(), ev=evs))
+    ws2 = [plan.workspace, torch.empty_like(plan.workspace)]
     lens = np.ascontiguousarray(plan.plan_host[plan.info.off_private_len:plan.info.off_private_len + S])
 
     def e2e_step(i):
         r = i % R
         b = i & 1
-        stage_free[b].synchronize()
-        h = stages[b].numpy()
-        if not pa.padoc_advance_decode_plan(h[:plan_ints], infos[b], lens):
+        st_ = sets[b]
+        st_["ev"][1].synchronize()     # this set's previous copies in have run: its stage may change
+        h = st_["stage"].numpy()
+        if not pa.padoc_advance_decode_plan(h[:plan_ints], st_["info"], lens):
             raise RuntimeError("plan advance refused")
-        pa.padoc_launch_decode_step(k_pools[r], v_pools[r], infos[b], stages[b], words, off_pt, PT, off_st, STW,
-                                    dev_ints, q_host, q_dev, scale, outs[r], lses[r], o_host, l_host, plan.workspace,
-                                    stream)
-        stage_free[b].record(stream)
+        pa.padoc_launch_decode_step(k_pools[r], v_pools[r], st_["info"], st_["stage"], words, off_pt, PT, off_st, STW,
+                                    st_["dev_ints"], st_["q_host"], st_["q_dev"], scale, st_["out"], st_["lse"],
+                                    st_["o_host"], st_["l_host"], ws2[b], stream, copy_in, copy_out,
+                                    st_["ev"][0], st_["ev"][1], st_["ev"][2])
 
-    for i in range(max(args.warmup, 1)):
+    for i in range(max(args.warmup, 2)):
         e2e_step(i)
     torch.cuda.synchronize()
     barrier(torch, world)
@@ -329,8 +335,8 @@ def bench_decode(args, torch, dev, rank, world, layout_streams=False):
     torch.cuda.synchronize()
     e2e_ms = (time.perf_counter() - t0) * 1e3 / e2e_steps
     barrier(torch, world)
-    h2d = words * 4 + q_host.numel() * 2
-    d2h = o_host.numel() * 2 + l_host.numel() * 4
+    h2d = words * 4 + sets[0]["q_host"].numel() * 2
+    d2h = sets[0]["o_host"].numel() * 2 + sets[0]["l_host"].numel() * 4
     res.update(e2e_ms=e2e_ms, h2d=h2d, d2h=d2h)
     return res
 

@@ -54,6 +54,8 @@ extern "C" {
 
 /* A CUDA stream handle; identical to cudaStream_t. */
 typedef struct CUstream_st *padoc_stream_t;
+/* A CUDA event handle; identical to cudaEvent_t. */
+typedef struct CUevent_st *padoc_event_t;
 
 typedef enum {
     PADOC_OK = 0,
@@ -286,21 +288,30 @@ padoc_status padoc_branch_decode_attn(const padoc_kv_pool *pool, const padoc_dec
 padoc_status padoc_advance_decode_plan(int32_t *plan, padoc_decode_plan *info, const int32_t *private_len,
                                        int32_t num_streams);
 
-/* One decode step for a caller whose step inputs live in host memory, all on `stream` with no host
+/* One decode step for a caller whose step inputs live in host memory, with no host
  * synchronization: copies stage[0, stage_words) ((host) int32, pinned for an asynchronous copy: the
  * plan blob at word 0, the page block table at off_page_table and the stream block table at
  * off_stream_table, each offset a multiple of 32 words past the blob) to dev_ints ((device) int32
  * [dev_capacity_words], 256-byte aligned) and q_host ((host) [num_streams][Hq][head_dim] in the pool
- * dtype) to q_dev (device, same size), runs padoc_branch_decode_attn on them, then copies out_dev and
- * lse_dev into out_host and lse_host ((host), same sizes). The host buffers must stay unchanged
- * (inputs) or unread (results) until the stream has run the copies.
+ * dtype) to q_dev (device, same size), runs padoc_branch_decode_attn on them on `stream`, then
+ * copies out_dev and lse_dev into out_host and lse_host ((host), same sizes).
+ *   copy_in NULL: everything runs on `stream` (copy_out and the events are not used).
+ *   copy_in, copy_out non-NULL (streams) with three events (created by the caller, e.g. with
+ *   cudaEventDisableTiming) of the buffer set this call uses: copy_in waits for ev_free (the set's
+ *   previous step has copied its results out; record it once before the first use), copies the
+ *   inputs in and records ev_in; `stream` waits for ev_in and decodes, and records ev_dec; copy_out
+ *   waits for ev_dec, copies the results out and records ev_free. With two buffer sets used in
+ *   turn, one step's copies in overlap the previous step's decode and its copies out the next one's.
+ * The host buffers must stay unchanged (inputs) or unread (results) until their copies have run.
  * Errors: INVALID_ARGUMENT, and those of padoc_branch_decode_attn. */
 padoc_status padoc_launch_decode_step(const padoc_kv_pool *pool, const padoc_decode_plan *info, const int32_t *stage,
                                       int64_t stage_words, int64_t off_page_table, int32_t page_table_stride,
                                       int64_t off_stream_table, int32_t stream_table_stride, int32_t *dev_ints,
                                       int64_t dev_capacity_words, const void *q_host, void *q_dev, float scale,
                                       void *out_dev, float *lse_dev, void *out_host, float *lse_host, void *workspace,
-                                      size_t workspace_bytes, padoc_stream_t stream);
+                                      size_t workspace_bytes, padoc_stream_t stream, padoc_stream_t copy_in,
+                                      padoc_stream_t copy_out, padoc_event_t ev_free, padoc_event_t ev_in,
+                                      padoc_event_t ev_dec);
 
 /* Size of the device array that padoc_branch_decode_attn_noalloc uses as its workspace. */
 #define PADOC_STATIC_WORKSPACE_BYTES (32u << 20)

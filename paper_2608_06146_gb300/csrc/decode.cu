@@ -723,10 +723,14 @@ extern "C" padoc_status padoc_launch_decode_step(const padoc_kv_pool *pool, cons
                                                  int64_t dev_capacity_words, const void *q_host, void *q_dev,
                                                  float scale, void *out_dev, float *lse_dev, void *out_host,
                                                  float *lse_host, void *workspace, size_t workspace_bytes,
-                                                 padoc_stream_t stream)
+                                                 padoc_stream_t stream, padoc_stream_t copy_in,
+                                                 padoc_stream_t copy_out, padoc_event_t ev_free, padoc_event_t ev_in,
+                                                 padoc_event_t ev_dec)
 {
     if (!pool || !info || !stage || !dev_ints || !q_host || !q_dev || !out_dev || !lse_dev || !out_host || !lse_host)
         return PADOC_ERR_INVALID_ARGUMENT;
+    const bool piped = copy_in != nullptr;
+    if (piped && (!copy_out || !ev_free || !ev_in || !ev_dec)) return PADOC_ERR_INVALID_ARGUMENT;
     const int64_t P = info->num_pages, S = info->num_streams;
     if (stage_words < info->plan_ints || dev_capacity_words < stage_words) return PADOC_ERR_INVALID_ARGUMENT;
     if ((((uintptr_t)dev_ints) & 255) || (off_page_table & 31) || (off_stream_table & 31)) return PADOC_ERR_INVALID_ARGUMENT;
@@ -742,16 +746,28 @@ extern "C" padoc_status padoc_launch_decode_step(const padoc_kv_pool *pool, cons
     const size_t lse_bytes = (size_t)S * info->cfg.num_q_heads * sizeof(float);
     if (S == 0) return PADOC_OK;
     cudaStream_t cs = (cudaStream_t)stream;
-    // the step's integers and queries in (pinned host memory makes both copies asynchronous)
-    PADOC_CUDA_TRY(cudaMemcpyAsync(dev_ints, stage, (size_t)stage_words * sizeof(int32_t), cudaMemcpyHostToDevice, cs));
-    PADOC_CUDA_TRY(cudaMemcpyAsync(q_dev, q_host, q_bytes, cudaMemcpyHostToDevice, cs));
+    cudaStream_t cin = piped ? (cudaStream_t)copy_in : cs, cout = piped ? (cudaStream_t)copy_out : cs;
+    // the step's integers and queries in (pinned host memory makes both copies asynchronous), once
+    // this buffer set's previous step has copied its results out
+    if (piped) PADOC_CUDA_TRY(cudaStreamWaitEvent(cin, (cudaEvent_t)ev_free, 0));
+    PADOC_CUDA_TRY(cudaMemcpyAsync(dev_ints, stage, (size_t)stage_words * sizeof(int32_t), cudaMemcpyHostToDevice, cin));
+    PADOC_CUDA_TRY(cudaMemcpyAsync(q_dev, q_host, q_bytes, cudaMemcpyHostToDevice, cin));
+    if (piped) {
+        PADOC_CUDA_TRY(cudaEventRecord((cudaEvent_t)ev_in, cin));
+        PADOC_CUDA_TRY(cudaStreamWaitEvent(cs, (cudaEvent_t)ev_in, 0));
+    }
     const padoc_status st = padoc_branch_decode_attn(pool, info, dev_ints, dev_ints + off_page_table, page_table_stride,
                                                      dev_ints + off_stream_table, stream_table_stride, q_dev, scale,
                                                      out_dev, lse_dev, workspace, workspace_bytes, stream);
     if (st != PADOC_OK) return st;
     // and the results out
-    PADOC_CUDA_TRY(cudaMemcpyAsync(out_host, out_dev, q_bytes, cudaMemcpyDeviceToHost, cs));
-    PADOC_CUDA_TRY(cudaMemcpyAsync(lse_host, lse_dev, lse_bytes, cudaMemcpyDeviceToHost, cs));
+    if (piped) {
+        PADOC_CUDA_TRY(cudaEventRecord((cudaEvent_t)ev_dec, cs));
+        PADOC_CUDA_TRY(cudaStreamWaitEvent(cout, (cudaEvent_t)ev_dec, 0));
+    }
+    PADOC_CUDA_TRY(cudaMemcpyAsync(out_host, out_dev, q_bytes, cudaMemcpyDeviceToHost, cout));
+    PADOC_CUDA_TRY(cudaMemcpyAsync(lse_host, lse_dev, lse_bytes, cudaMemcpyDeviceToHost, cout));
+    if (piped) PADOC_CUDA_TRY(cudaEventRecord((cudaEvent_t)ev_free, cout));
     return PADOC_OK;
 }
 

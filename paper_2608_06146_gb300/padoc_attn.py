@@ -170,7 +170,7 @@ def load_library(path: Optional[str] = None):
         "padoc_launch_decode_step": [ctypes.POINTER(padoc_kv_pool), ctypes.POINTER(padoc_decode_plan), _vp,
                                      ctypes.c_int64, ctypes.c_int64, ctypes.c_int32, ctypes.c_int64, ctypes.c_int32,
                                      _vp, ctypes.c_int64, _vp, _vp, ctypes.c_float, _vp, _vp, _vp, _vp, _vp,
-                                     ctypes.c_size_t, _vp],
+                                     ctypes.c_size_t, _vp, _vp, _vp, _vp, _vp, _vp],
         "padoc_quantize_kv_blocks": [ctypes.POINTER(padoc_kv_pool_e4m3), _vp, _vp, _vp, ctypes.c_int32, _vp],
         "padoc_append_inputs_e4m3": [ctypes.POINTER(padoc_kv_pool_e4m3), _vp, _vp, _vp, ctypes.c_int64, ctypes.c_int32,
                                      _vp, _vp, _vp, ctypes.c_int32, _vp],
@@ -523,9 +523,13 @@ def padoc_advance_decode_plan(plan, info: padoc_decode_plan, private_len) -> boo
 
 def padoc_launch_decode_step(k_pool, v_pool, info: padoc_decode_plan, stage, stage_words: int, off_page_table: int,
                              page_stride: int, off_stream_table: int, stream_stride: int, dev_ints, q_host, q_dev,
-                             scale, out_dev, lse_dev, out_host, lse_host, workspace, stream=None):
+                             scale, out_dev, lse_dev, out_host, lse_host, workspace, stream=None, copy_in=None,
+                             copy_out=None, ev_free=None, ev_in=None, ev_dec=None):
     """One decode step from host inputs: stage (pinned int32 CPU tensor: plan blob, page table, stream
-    table), q_host (pinned) -> device, decode, out / lse -> out_host / lse_host (pinned); no sync."""
+    table), q_host (pinned) -> device, decode, out / lse -> out_host / lse_host (pinned); no sync.
+    With copy_in / copy_out (torch streams) and the buffer set's three torch events, the copies run
+    on those streams, ordered by the events (see the C header)."""
+    ev = lambda e: None if e is None else e.cuda_event
     lib = load_library()
     pool = padoc_kv_pool(_dev(k_pool, "k_pool"), _dev(v_pool, "v_pool"), k_pool.shape[0], k_pool.shape[2],
                          k_pool.shape[1], k_pool.shape[3], _dtype_code(k_pool))
@@ -535,7 +539,9 @@ def padoc_launch_decode_step(k_pool, v_pool, info: padoc_decode_plan, stage, sta
                                       _dev(q_dev, "q_dev"), float(scale), _dev(out_dev, "out_dev"),
                                       _dev(lse_dev, "lse_dev"), out_host.data_ptr(), lse_host.data_ptr(),
                                       _dev(workspace, "workspace"), workspace.numel() * workspace.element_size(),
-                                      _stream_ptr(stream))
+                                      _stream_ptr(stream), None if copy_in is None else _stream_ptr(copy_in),
+                                      None if copy_out is None else _stream_ptr(copy_out), ev(ev_free), ev(ev_in),
+                                      ev(ev_dec))
     _check("padoc_launch_decode_step", st)
 
 

@@ -139,7 +139,7 @@ def test_launch_decode_step_rejects_malformed_calls(lib):
     words = 4096
     call = lambda stage=A, sw=words, opt=2048, pts=8, ost=3072, sts=8, dev=A, dcap=words, qh=A: lib.padoc_launch_decode_step(
         ctypes.byref(_pool()), ctypes.byref(info), stage, sw, opt, pts, ost, sts, dev, dcap, qh, A, 0.1, A, A, A, A, A,
-        1 << 20, None)
+        1 << 20, None, None, None, None, None, None)
     assert call(stage=None) == 1 and call(qh=None) == 1 and call(dev=None) == 1
     assert call(sw=info.plan_ints - 1) == 1                  # the stage must hold the blob
     assert call(dcap=words - 1) == 1                         # the device buffer must hold the stage
@@ -148,3 +148,6 @@ def test_launch_decode_step_rejects_malformed_calls(lib):
     assert call(opt=0) == 1                                  # tables after the blob
     assert call(ost=2048) == 1                               # tables must not overlap
     assert call(opt=4064, pts=64) == 1                       # a table past the stage
+    piped = lambda ev: lib.padoc_launch_decode_step(ctypes.byref(_pool()), ctypes.byref(info), A, words, 2048, 8, 3072, 8,
+                                                    A, words, A, A, 0.1, A, A, A, A, A, 1 << 20, None, A, A, ev, A, A)
+    assert piped(None) == 1                                  # copy streams need the three events

@@ -57,7 +57,8 @@ def test_advanced_plan_decodes_the_grown_batch():
     _check(out.float().cpu().numpy(), lse.cpu().numpy(), ref_o, ref_l)
 
 
-def test_one_call_step_from_host_memory():
+@pytest.mark.parametrize("piped", [False, True])
+def test_one_call_step_from_host_memory(piped):
     wl = inputs.dense_page()
     di = inputs.decode_inputs(wl, 71)
     cfg = pa.make_decode_config(16, 2, 128, 16, False, 0, 0, 0)
@@ -82,8 +83,16 @@ def test_one_call_step_from_host_memory():
     l_host = torch.full((S, 16), float("nan"), dtype=torch.float32).pin_memory()
     ws = torch.empty(pa.padoc_decode_workspace_size(info), dtype=torch.uint8, device=DEV)
     scale = 1.0 / math.sqrt(128)
+    kw = {}
+    if piped:   # copies on their own streams, ordered by the buffer set's events
+        evs = [torch.cuda.Event() for _ in range(3)]
+        for e in evs:
+            e.record()
+        kw = dict(copy_in=torch.cuda.Stream(), copy_out=torch.cuda.Stream(), ev_free=evs[0], ev_in=evs[1], ev_dec=evs[2])
     pa.padoc_launch_decode_step(di.k_pool.to(DEV), di.v_pool.to(DEV), info, stage, words, off_pt, PT, off_st, STW,
-                                dev_ints, q_host, q_dev, scale, out, lse, o_host, l_host, ws)
+                                dev_ints, q_host, q_dev, scale, out, lse, o_host, l_host, ws, **kw)
+    if piped:
+        kw["ev_free"].synchronize()         # the results' copies out have run
     pa.padoc_check_device_errors()          # synchronizes the stream: the results are in host memory
     ref_o, ref_l = oracle.decode_pages(wl.pages, di, scale)
     _check(o_host.float().numpy(), l_host.numpy(), ref_o, ref_l)
