@@ -558,9 +558,13 @@ def bench_loop(args, torch, dev, rank, world):
     into the pool, untimed), then the loop runs every layout stream and branch from its first input
     to its EOS. Timed twice: (a) end to end through the engine, as a caller runs it (host scheduler
     and planner in one library call, one host->device copy and the append + decode launches per
-    step; the synthetic token source needs no outputs, so no step waits for the device); (b) the
-    device work alone: the same steps' launches, captured once in a CUDA graph from per-step inputs
-    already on the device, replayed."""
+    step, the step's events handed to the scheduler); the synthetic token source stands in for the
+    decoder's sampled outputs, and its events depend only on the pages and the scheduler's stream
+    order, so they are drawn once, before the timed region (a warm-up pass records each step's
+    stream ids, source rows, forks and EOS flags; the timed pass replays them and checks that the
+    scheduler hands out the same stream ids); no step waits for the device; (b) the device work
+    alone: the same steps' launches, captured once in a CUDA graph from per-step inputs already on
+    the device, replayed."""
     from paper_2608_06146_gb300 import inputs
     from paper_2608_06146_gb300 import padoc_attn as pa
     from paper_2608_06146_gb300.engine import MaskedParallelLoop
@@ -589,10 +593,11 @@ def bench_loop(args, torch, dev, rank, world):
         src, loop = admit_all()
         torch.cuda.synchronize()
         steps = toks = h2d = 0
-        rec = []
+        rec, traj = [], []
         t0 = time.perf_counter()
         while loop.status()[1] > 0:
-            ids, out, lse = loop.step(kd, vd, qd, src.rows, scale)
+            rows_now = []
+            ids, out, lse = loop.step(kd, vd, qd, lambda x: rows_now.append(src.rows(x)) or rows_now[0], scale)
             steps += 1
             toks += len(ids)
             h2d += loop.h2d_bytes
@@ -600,15 +605,38 @@ def bench_loop(args, torch, dev, rank, world):
                 stp = loop.last_step
                 rec.append((loop.last_stage[:int(stp.upload_words)].copy(), stp))
             nf, eos = src.events(ids)
+            traj.append((ids.copy(), np.asarray(rows_now[0], np.int32).copy(), nf.copy(), eos.copy()))
             src.forked(ids, nf, loop.end_step(nf, eos))
         torch.cuda.synchronize()
-        return time.perf_counter() - t0, steps, toks, h2d, rec
+        return time.perf_counter() - t0, steps, toks, h2d, rec, traj
 
-    run(False)   # warm-up pass (first launches, the pool's first touch, the staging buffers)
+    def run_replay(traj):
+        _, loop = admit_all()
+        cmax = max(len(t[0]) for t in traj)
+        outs_ = [torch.empty((cmax, Hq, d), dtype=wl.dtype, device=dev) for _ in range(2)]
+        lses_ = [torch.empty((cmax, Hq), dtype=torch.float32, device=dev) for _ in range(2)]
+        torch.cuda.synchronize()
+        toks = h2d = 0
+        same = True
+        t0 = time.perf_counter()
+        for i, (ids_r, rows_r, nf_r, eos_r) in enumerate(traj):
+            C = len(ids_r)
+            ids, out, lse = loop.step(kd, vd, qd, lambda x: rows_r, scale, out=outs_[i & 1][:C], lse=lses_[i & 1][:C])
+            same = same and np.array_equal(ids, ids_r)
+            toks += C
+            h2d += loop.h2d_bytes
+            loop.end_step(nf_r, eos_r)
+        torch.cuda.synchronize()
+        el = time.perf_counter() - t0
+        if not same or loop.status()[1] != 0:
+            raise RuntimeError("the replayed loop diverged from the recorded one")
+        return el, len(traj), toks, h2d
+
+    _, _, _, _, _, traj = run(False)   # warm-up pass (first launches, the pool's first touch, staging), recorded
     pa.padoc_check_device_errors(stream)
-    e2e_s, steps, toks, h2d, _ = run(False)
+    e2e_s, steps, toks, h2d = run_replay(traj)
     pa.padoc_check_device_errors(stream)
-    _, _, _, _, rec = run(True)
+    _, _, _, _, rec, _ = run(True)
 
     # algorithmic bytes of the loop: per step the decode minimum (each page's visible shared stream
     # once, private rows, Q in, O and LSE out) plus the append (the inputs' K and V rows written,
