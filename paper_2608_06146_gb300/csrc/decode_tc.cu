@@ -28,6 +28,10 @@
 // TMEM: S_i / P_i at columns 128i, O_i at 256 + 128i. The next piece's first PV overwrites O_i; it
 // waits for P_i of that piece, which the softmax warps publish only after reading O_i out.
 //
+// A piece may span two items (chunked prefill: a group's shared tiles, then its private ones; the
+// first item flagged PADOC_ITEM_CONT): the second item keeps the queries, the softmax state and O
+// (its first PV accumulates), and only it writes the partial.
+//
 // FP8 (E4M3) pool (kE4M3): each paged block's codes (16 rows x 128 bytes) land by TMA in the upper
 // half of the tile's ring slot, and the producer warp that loaded them expands them in place into
 // the bf16 panels the MMAs read (each lane owns whole rows, reads a row's codes before writing it;
@@ -309,6 +313,8 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
         for (int u = u0; ok && u < u1; ++u) {
             const padoc_item it = prm.items[u];
             const int ne = piece_tiles(it);
+            // an item that continues the previous one keeps its queries
+            const bool cont_in = u > u0 && (prm.items[u - 1].kind & PADOC_ITEM_CONT);
             if (ne == 0) {
                 if (u + 1 < u1) fetch_id(u + 1, 0);
                 continue;
@@ -358,7 +364,7 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
                     }
                 }
                 ++n;
-                if (is_k && j == 0 && !(q_first && u == u0)) {
+                if (is_k && j == 0 && !(q_first && u == u0) && !cont_in) {
                     // E4M3: the previous piece's tiles must be expanded before its last QK^T can run
                     if (kE4M3)
                         while (ok && nc < n - 1) ok = expand_next();
@@ -418,13 +424,20 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
             const padoc_item it = prm.items[u];
             const int ne = piece_tiles(it);
             const bool act = mi < piece_mtiles(it);   // this warp's M-tile is part of the piece
+            // a piece over two items: the second keeps the queries and accumulates into O; only the
+            // last item of a piece releases the queries and reports O complete
+            const bool cont_in = u > u0 && (prm.items[u - 1].kind & PADOC_ITEM_CONT);
+            const bool cont_out = (it.kind & PADOC_ITEM_CONT) != 0;
             if (ne == 0) continue;
-            if (!wait_w(B_Q, nq & 1, 60) || !wait_w(B_KFULL + J % kKStages, (J / kKStages) & 1, 61)) { ok = false; break; }
-            ++nq;
+            if ((!cont_in && !wait_w(B_Q, nq & 1, 60)) || !wait_w(B_KFULL + J % kKStages, (J / kKStages) & 1, 61)) {
+                ok = false;
+                break;
+            }
+            if (!cont_in) ++nq;
             tc_fence_after();
             if (act) issue_s(J % kKStages);
             umma_commit_warp(bar(B_KEMPTY + J % kKStages));
-            if (ne == 1) umma_commit_warp(bar(B_QFREE));
+            if (ne == 1 && !cont_out) umma_commit_warp(bar(B_QFREE));
             for (int j = 0; ok && j < ne; ++j) {
                 const int Jj = J + j, s = Jj % kVStages, kn = (Jj + 1) % kKStages;
                 const bool more = j + 1 < ne;
@@ -440,17 +453,17 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
                     const uint64_t db = dv0 + (uint64_t)(s * (kTile >> 4));
 #pragma unroll
                     for (int kk = 0; kk < 8; ++kk)
-                        umma_bf16_ts_warp(tO, tS + kk * 8, db + kk * (2048 >> 4), idPV, (j > 0 || kk > 0));
+                        umma_bf16_ts_warp(tO, tS + kk * 8, db + kk * (2048 >> 4), idPV, (cont_in || j > 0 || kk > 0));
                     ++ci;
                     // S_i of the next tile overwrites P_i only after this PV has read it (one
                     // thread's MMAs run in issue order)
                     if (more) issue_s(kn);
-                    else umma_commit_warp(bar(B_PVDONE + mi));   // O_i of the piece is complete
+                    else if (!cont_out) umma_commit_warp(bar(B_PVDONE + mi));   // O_i of the piece is complete
                 }
                 umma_commit_warp(bar(B_VEMPTY + s));
                 if (more) {
                     umma_commit_warp(bar(B_KEMPTY + kn));
-                    if (j + 2 == ne) umma_commit_warp(bar(B_QFREE));
+                    if (j + 2 == ne && !cont_out) umma_commit_warp(bar(B_QFREE));
                 }
             }
             J += ne;
@@ -491,7 +504,7 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
         // columns before their cutoff.
         const int b0 = row / kGroup, b1 = 16 + row / kGroup;
         int n_tb = 0, n_te = 0, n_nstr = 0, n_first = 0, n_kvh = 0, n_slot = 0, n_cut0 = 0, n_cut1 = 0;
-        bool n_priv = false;
+        bool n_priv = false, n_cont = false;
         auto fetch_item = [&](int uu) {
             const padoc_item *p = prm.items + uu;
             n_tb = p->tok_begin;
@@ -501,6 +514,7 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
             n_kvh = p->kv_head;
             n_slot = p->slot;
             n_priv = PADOC_ITEM_KIND(p->kind) == PADOC_ITEM_PRIVATE_TC;
+            n_cont = (p->kind & PADOC_ITEM_CONT) != 0;
         };
         // a row's cutoff: its stream's shared length, or for a chunk's private rows its private length
         auto fetch_cut = [&]() {
@@ -512,9 +526,12 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
             fetch_item(u0);
             fetch_cut();
         }
+        float m0 = -INFINITY, l0 = 0.f, m1 = -INFINITY, l1 = 0.f;   // running softmax state of the piece
+        bool cont_in = false;   // the previous item continues into this one
         for (int u = u0; u < u1; ++u) {
             const int tb = n_tb, te = n_te, nstr = n_nstr, first = n_first, kvh = n_kvh, slot = n_slot;
             const int cut0 = n_cut0, cut1 = n_cut1;
+            const bool cont_out = n_cont;
             const int ne = te > tb ? (te - tb + kKT - 1) / kKT : 0, mt = nstr > 16 ? 2 : 1;
             if (u + 1 < u1) fetch_item(u + 1);
             // first partial slot of each row's (stream, KV head), read during the piece's last tile
@@ -523,7 +540,9 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
                 pb0 = prm.slot_ptr[(size_t)(first + (b0 < nstr ? b0 : 0)) * prm.num_kv_heads + kvh] + slot;
                 if (mt == 2) pb1 = prm.slot_ptr[(size_t)(first + (b1 < nstr ? b1 : 0)) * prm.num_kv_heads + kvh] + slot;
             };
-            float m0 = -INFINITY, l0 = 0.f, m1 = -INFINITY, l1 = 0.f;
+            if (!cont_in) {   // a new piece (an item continuing the previous one keeps the state)
+                m0 = -INFINITY; l0 = 0.f; m1 = -INFINITY; l1 = 0.f;
+            }
             for (int j = 0; j < ne; ++j) {
                 if (j == 1 && u + 1 < u1) fetch_cut();
                 if (j == ne - 1) fetch_slots();
@@ -667,6 +686,8 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
             }
             if (ne < 2 && u + 1 < u1) fetch_cut();
             if (ne == 0) fetch_slots();
+            cont_in = cont_out;
+            if (cont_out) continue;   // the piece goes on in the next item
             // partials of this piece: O / l (fp32) and the natural-log LSE of every row
 #pragma unroll
             for (int mi = 0; mi < 2; ++mi) {

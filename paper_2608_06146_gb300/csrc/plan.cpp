@@ -391,11 +391,16 @@ padoc_status build_work(int32_t num_pages, const padoc_decode_config *cfg, PlanP
     // the group can see. The segments are laid end to end and cut into one contiguous range per CTA
     // (a tile weighs PADOC_TC_WEIGHT_2M for a group of two M-tiles and PADOC_TC_WEIGHT_1M for one);
     // a range becomes the pieces where it overlaps segments.
-    // A chunked prefill groups streams within a chunk only, and a chunk whose tokens have private
-    // rows and are many enough also gets private segments over those rows (PADOC_ITEM_PRIVATE_TC)
-    // with the same groups, so that every stream of a group receives the same items and therefore
-    // the same partial-slot numbers.
-    struct Segment { int32_t kind, g, p, first, ns, vis, ntiles, weight; };
+    // A chunked prefill groups streams within a chunk only, and a group of a chunk whose tokens have
+    // private rows and are many enough continues its segment over those rows (PADOC_ITEM_PRIVATE_TC,
+    // through the chunk's first token's block-table row): the shared tiles, then the private ones,
+    // one sequence with one running softmax, so that a piece covering both writes one partial. A
+    // piece that crosses from the shared to the private tiles becomes two items, the first flagged
+    // PADOC_ITEM_CONT; every stream of a group receives the same items and partial-slot numbers.
+    struct Segment {
+        int32_t kind, g, p, first, ns, vis, ntiles, weight;
+        int32_t kind2, p2, vis2, ntiles2;   // the private continuation (ntiles2 = 0: none)
+    };
     std::vector<Segment> segs;
     const bool chunked = !pp.chunk_of.empty();
     std::vector<uint8_t> priv_tc(chunked ? (size_t)S : 0, 0);
@@ -415,21 +420,22 @@ padoc_status build_work(int32_t num_pages, const padoc_decode_config *cfg, PlanP
                         }
                 int32_t vis = 0;
                 for (int32_t st = f0 + r; st < f0 + r + nb; ++st) vis = std::max(vis, pp.streams[st].shared_len);
-                if (vis > 0)
-                    segs.push_back({PADOC_ITEM_SHARED_TC | (chunked && nb < ns ? PADOC_ITEM_REREAD : 0), g, p, f0 + r, nb, vis,
-                                    (vis + PADOC_TC_TILE_TOKENS - 1) / PADOC_TC_TILE_TOKENS, weight_of(nb)});
+                Segment sg{PADOC_ITEM_SHARED_TC | (chunked && nb < ns ? PADOC_ITEM_REREAD : 0), g, p, f0 + r, nb, vis,
+                           (vis + PADOC_TC_TILE_TOKENS - 1) / PADOC_TC_TILE_TOKENS, weight_of(nb), 0, 0, 0, 0};
+                if (chunked) {
+                    // a group of a chunk with private rows on the tensor cores continues over them
+                    const int32_t c = pp.chunk_of[f0 + r], first = pp.chunk_first[c], len = pp.chunk_len[c];
+                    if (pp.chunk_private[c] && (int64_t)len * group >= PADOC_TC_MIN_ROWS) {
+                        const int32_t vis2 = pp.streams[f0 + r + nb - 1].private_len;   // increasing within a chunk
+                        for (int32_t st = f0 + r; st < f0 + r + nb; ++st) priv_tc[st] = 1;
+                        sg.kind2 = PADOC_ITEM_PRIVATE_TC | (nb < len ? PADOC_ITEM_REREAD : 0);
+                        sg.p2 = first;
+                        sg.vis2 = vis2;
+                        sg.ntiles2 = (vis2 + PADOC_TC_TILE_TOKENS - 1) / PADOC_TC_TILE_TOKENS;
+                    }
+                }
+                if (sg.ntiles + sg.ntiles2 > 0) segs.push_back(sg);
                 r += nb;
-            }
-        }
-        for (size_t c = 0; c < pp.chunk_first.size(); ++c) {
-            const int32_t first = pp.chunk_first[c], len = pp.chunk_len[c];
-            if (!pp.chunk_private[c] || (int64_t)len * group < PADOC_TC_MIN_ROWS) continue;
-            for (int32_t r = 0; r < len; r += PADOC_TC_ITEM_STREAMS) {
-                const int32_t nb = std::min(PADOC_TC_ITEM_STREAMS, len - r);
-                const int32_t vis = pp.streams[first + r + nb - 1].private_len;   // increasing within a chunk
-                for (int32_t st = first + r; st < first + r + nb; ++st) priv_tc[st] = 1;
-                segs.push_back({PADOC_ITEM_PRIVATE_TC | (nb < len ? PADOC_ITEM_REREAD : 0), g, first, first + r, nb, vis,
-                                (vis + PADOC_TC_TILE_TOKENS - 1) / PADOC_TC_TILE_TOKENS, weight_of(nb)});
             }
         }
     }
@@ -446,7 +452,7 @@ padoc_status build_work(int32_t num_pages, const padoc_decode_config *cfg, PlanP
     int64_t max_piece = 0;
     int64_t total_w = 0, max_w = 0;
     for (const Segment &sg : segs) {
-        total_w += (int64_t)sg.ntiles * sg.weight + piece_cost(sg);
+        total_w += (int64_t)(sg.ntiles + sg.ntiles2) * sg.weight + piece_cost(sg);
         max_piece = std::max(max_piece, piece_cost(sg));
         max_w = std::max<int64_t>(max_w, sg.weight);
     }
@@ -455,7 +461,8 @@ padoc_status build_work(int32_t num_pages, const padoc_decode_config *cfg, PlanP
         int64_t used = 0, load = 0;
         for (const Segment &sg : segs) {
             int32_t t = 0;
-            while (t < sg.ntiles) {
+            const int32_t ntot = sg.ntiles + sg.ntiles2;
+            while (t < ntot) {
                 const int64_t piece_w = piece_cost(sg);
                 int64_t room = used > 0 ? (T - load - piece_w) / sg.weight : 0;
                 if (room < 1) {   // close the current CTA, open the next
@@ -467,13 +474,23 @@ padoc_status build_work(int32_t num_pages, const padoc_decode_config *cfg, PlanP
                     load = 0;
                     room = std::max<int64_t>(1, (T - piece_w) / sg.weight);
                 }
-                const int32_t t1 = (int32_t)std::min<int64_t>(sg.ntiles, t + room);
+                const int32_t t1 = (int32_t)std::min<int64_t>(ntot, t + room);
                 load += piece_w + (int64_t)(t1 - t) * sg.weight;
                 if (emit) {
-                    const int32_t tb = t * PADOC_TC_TILE_TOKENS, te = std::min(sg.vis, t1 * PADOC_TC_TILE_TOKENS);
+                    // one partial slot per piece; a piece over shared and private tiles is two items
                     const int32_t slot = cnt[(size_t)sg.first * Hkv + sg.g];
                     for (int32_t st = sg.first; st < sg.first + sg.ns; ++st) ++cnt[(size_t)st * Hkv + sg.g];
-                    tc_items.push_back({sg.kind, sg.p, sg.g, tb, te, sg.first, sg.ns, slot});
+                    if (t < sg.ntiles) {
+                        const int32_t e = std::min(t1, sg.ntiles);
+                        const int32_t tb = t * PADOC_TC_TILE_TOKENS, te = std::min(sg.vis, e * PADOC_TC_TILE_TOKENS);
+                        tc_items.push_back({sg.kind | (t1 > sg.ntiles ? PADOC_ITEM_CONT : 0), sg.p, sg.g, tb, te,
+                                            sg.first, sg.ns, slot});
+                    }
+                    if (t1 > sg.ntiles) {
+                        const int32_t b = std::max(t, sg.ntiles) - sg.ntiles, e = t1 - sg.ntiles;
+                        const int32_t tb = b * PADOC_TC_TILE_TOKENS, te = std::min(sg.vis2, e * PADOC_TC_TILE_TOKENS);
+                        tc_items.push_back({sg.kind2, sg.p2, sg.g, tb, te, sg.first, sg.ns, slot});
+                    }
                 }
                 t = t1;
             }

@@ -73,6 +73,10 @@ enum { PADOC_ITEM_SHARED = 0, PADOC_ITEM_PRIVATE = 1, PADOC_ITEM_SHARED_TC = 2, 
 // never set it: their tiles are loaded evict-first, which keeps the split-K partials in L2 for the
 // merge (measured: flagging the decode step's pages of more than 32 streams was no faster).
 #define PADOC_ITEM_REREAD 16
+// Flag of a tensor-core item that the next item of the same CTA continues (a chunked prefill's
+// piece over a group's shared tiles and then its private ones): the same streams, KV head and
+// partial slot, one running softmax over both, one partial written after the second item.
+#define PADOC_ITEM_CONT 32
 #define PADOC_ITEM_KIND(k) ((k) & 15)
 
 // One split-K work item of the decode kernels (8 int32 words in the plan blob). The blob holds

@@ -65,12 +65,24 @@ def check_chunk_plan(page_len, chunks, tc_ctas, warp_ctas=0):
     items = plan[info.off_items:info.off_items + 8 * info.num_items].reshape(-1, 8)
     ntc = info.num_tc_items
     assert np.isin(items[:ntc, 0] & 15, [2, 3]).all() and np.isin(items[ntc:, 0], [0, 1]).all()
+    assert not np.any(items[:, 0] & ~(15 | 16 | 32))
     first_of = {c: int(np.nonzero(ch == c)[0][0]) for c in range(len(chunks))}
     cov_sh = {(s, g): np.zeros(sh[s], np.int32) for s in range(S) for g in range(Hkv)}
     cov_pv = {(s, g): np.zeros(pl[s], np.int32) for s in range(S) for g in range(Hkv)}
     slots = {(s, g): [] for s in range(S) for g in range(Hkv)}
-    for kind, idx, g, tb, te, fs, ns, slot in items:
+    # a piece over a group's shared and then its private rows is two items, the first flagged CONT:
+    # the second is the group's private item with the same head, streams and slot, in the same CTA
+    cta = plan[info.off_cta_ptr:info.off_cta_ptr + info.tc_ctas + 1] if ntc else np.zeros(1, np.int32)
+    cont = (items[:, 0] & 32) != 0
+    assert not cont[ntc:].any() and (ntc == 0 or not cont[ntc - 1])
+    for u in np.nonzero(cont)[0]:
+        a, b = items[u], items[u + 1]
+        assert a[0] & 15 == 2 and b[0] & 15 == 3 and (a[2], a[5], a[6], a[7]) == (b[2], b[5], b[6], b[7])
+        assert b[3] == 0, "the private part of a piece starts at the chunk's first private tile"
+        assert not np.isin(u + 1, cta), "both items of a piece belong to one CTA"
+    for i, (kind, idx, g, tb, te, fs, ns, slot) in enumerate(items):
         reread = bool(kind & 16)
+        continued = i > 0 and cont[i - 1]
         kind &= 15
         if kind == 3:   # reread exactly when the chunk has more than one group
             assert reread == (chunks[ch[fs]][3] > 32)
@@ -93,7 +105,8 @@ def check_chunk_plan(page_len, chunks, tc_ctas, warp_ctas=0):
                 hi = min(te, sh[s])
                 if hi > tb:
                     cov_sh[(s, g)][tb:hi] += 1
-            slots[(s, g)].append(slot)
+            if not continued:    # one partial per piece
+                slots[(s, g)].append(slot)
     for key in cov_sh:
         s, g = key
         assert np.all(cov_sh[key] == 1), f"shared rows of token {s} head {g}"
