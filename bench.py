@@ -272,7 +272,7 @@ def bench_decode(args, torch, dev, rank, world, layout_streams=False):
     timing = time_steps(args, torch, world, stream, step, steady=not layout_streams)
     nbytes = decode_bytes(wl, layout_streams)
     info = plan.info
-    launches = (1 if info.num_tc_items > 0 else 0) + (1 if info.num_warps > 0 else 0) + 1   # + the merge
+    launches = (1 if info.num_tc_items > 0 or info.num_warps > 0 else 0) + 1   # the decode grid + the merge
     res = dict(ms=timing["ms"], streams=S, bytes=nbytes, launches=launches, clocks=timing["clocks"], replicas=R,
                pages=len(wl.pages), e2e_ms=None, h2d=0, d2h=0, steady=timing.get("steady"))
     if args.no_e2e or layout_streams:
@@ -374,7 +374,7 @@ def bench_decode_replicas(args, torch, dev, rank, world, shape):
 
     timing = time_steps(args, torch, world, stream, step, steady=False)
     info = plan.info
-    launches = (1 if info.num_tc_items > 0 else 0) + (1 if info.num_warps > 0 else 0) + 1
+    launches = (1 if info.num_tc_items > 0 or info.num_warps > 0 else 0) + 1
     return dict(ms=timing["ms"], streams=S, pages=R, bytes=decode_bytes(wl), launches=launches,
                 clocks=timing["clocks"], tc_items=int(info.num_tc_items), warp_items=int(info.num_items - info.num_tc_items))
 
@@ -416,6 +416,7 @@ def bench_decode_e4m3(args, torch, dev, rank, world):
 
     timing = time_steps(args, torch, world, stream, step, steady=False)
     info = plan.info
+    # the tensor-core grid, the warp grid (the E4M3 pool runs them apart) and the merge
     launches = (1 if info.num_tc_items > 0 else 0) + (1 if info.num_warps > 0 else 0) + 1
     return dict(ms=timing["ms"], streams=S, bytes=decode_bytes(wl, kv_bytes=1, scale_bytes=4), launches=launches,
                 clocks=timing["clocks"], replicas=R)
@@ -705,8 +706,8 @@ def bench_loop(args, torch, dev, rank, world):
         torch.cuda.synchronize()
     pa.padoc_check_device_errors(stream)
     dev_s = e0.elapsed_time(e1) * 1e-3
-    launches = sum(1 + (1 if stp.plan.num_tc_items > 0 else 0) + (1 if stp.plan.num_warps > 0 else 0) + 1
-                   for _, stp in rec)
+    # per step: the append kernel, the decode grid and the merge
+    launches = sum(1 + (1 if stp.plan.num_tc_items > 0 or stp.plan.num_warps > 0 else 0) + 1 for _, stp in rec)
     return dict(e2e_s=e2e_s, dev_s=dev_s, eager_s=eager_s, steps=steps, tokens=toks, bytes=nbytes, h2d=h2d,
                 launches=launches, clocks=clk.summary(), pages=len(wl.pages), pool_blocks=nb)
 

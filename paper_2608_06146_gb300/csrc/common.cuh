@@ -318,6 +318,19 @@ __device__ __forceinline__ void named_bar_sync(int id, int count)
     asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(count) : "memory");
 }
 
+// Per-thread register budget of the executing warpgroup (all four warps run the same instruction):
+// inc waits until the CTA's pool (what its threads were launched with) has the registers; dec
+// returns registers to it. N is a multiple of 8 in [24, 256].
+template <uint32_t N>
+__device__ __forceinline__ void setmaxnreg_inc()
+{
+    asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(N));
+}
+template <uint32_t N>
+__device__ __forceinline__ void setmaxnreg_dec()
+{
+    asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(N));
+}
 __device__ __forceinline__ void pdl_launch_dependents() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
 __device__ __forceinline__ void pdl_wait_prerequisite() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 
@@ -347,13 +360,19 @@ padoc_status padoc_launch_prefill_tc(const void *q, const void *k, const void *v
                                      const int32_t *tile_row_ptr_dev, const int32_t *tile_k_dev,
                                      const int8_t *tile_kind_dev, float scale_log2, void *out, float *lse,
                                      cudaStream_t stream);
-// tcgen05 shared-stream decode (decode_tc.cu): the plan's tensor-core items.
-// k_scales / v_scales non-null: an E4M3 pool (kmap / vmap are padoc_make_tmap_u8 maps of the codes).
+namespace padoc_warp {
+struct DecodeParams;
+}
+// The decode grid (decode_tc.cu): the plan's tensor-core items, then its warp lists (wprm, the
+// warp path's arguments). k_scales / v_scales non-null: an E4M3 pool (kmap / vmap are
+// padoc_make_tmap_u8 maps of the codes), whose grid runs the tensor-core items only (the caller
+// launches decode_warp_kernel after it).
 padoc_status padoc_launch_decode_tc(const CUtensorMap *kmap, const CUtensorMap *vmap, const CUtensorMap *qmap, const int32_t *plan,
                                     const padoc_decode_plan *info, const int32_t *page_table, int32_t page_stride,
                                     const int32_t *stream_table, int32_t stream_stride, int32_t num_blocks,
                                     const float *k_scales, const float *v_scales, float *part_o, float *part_lse,
-                                    float scale_log2, int *err, cudaStream_t stream);
+                                    float scale_log2, int *err, const padoc_warp::DecodeParams *wprm,
+                                    cudaStream_t stream);
 // tcgen05 prefill backward (prefill_bwd_tc.cu): the dQ pass, which also writes lt / dt (per head
 // [Hq][t_pad]: -lse2 and rowsum(dO * O)), then the dK/dV pass; arguments validated by the caller.
 padoc_status padoc_launch_prefill_bwd_tc(const void *q, const void *k, const void *v, const void *out,
@@ -363,6 +382,8 @@ padoc_status padoc_launch_prefill_bwd_tc(const void *q, const void *k, const voi
                                          float *dt, int64_t t_pad, float scale, void *dq, void *dk, void *dv,
                                          cudaStream_t stream);
 int padoc_num_sms();
+// SM count the planner sizes grids for (the current device's, read once; 152 without a device)
+int32_t padoc_default_ctas();
 
 #define PADOC_CUDA_TRY(expr)                                   \
     do {                                                       \

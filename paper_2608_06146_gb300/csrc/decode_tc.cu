@@ -43,6 +43,7 @@
 #include <math.h>
 
 #include "common.cuh"
+#include "decode_warp.cuh"
 #include "tc.cuh"
 
 namespace {
@@ -103,6 +104,9 @@ struct TcDecodeParams {
     float *part_o, *part_lse;
     float scale_log2;
     int *err;
+    // the fused grid (plan_internal.h): CTAs [0, tc_ctas) run pieces, then warp CTA early_ctas + c;
+    // CTAs from tc_ctas on run warp CTA c - tc_ctas; warp CTAs at or past warp_ctas do not exist
+    int32_t tc_ctas, early_ctas, warp_ctas;
 };
 
 __device__ __forceinline__ bool wait_or_abort(uint32_t bar, uint32_t parity, int *err, int site, volatile int *abort_flag)
@@ -163,16 +167,41 @@ __device__ __forceinline__ void expand_tile(uint8_t *slot, int lane)
     fence_proxy_async_smem();   // the MMAs read the panels through the async proxy
 }
 
+// Pulls into L2 the first paged blocks (up to 4) of the first item of each of warp CTA wc's warp
+// lists, which this CTA runs once its pieces end, so that they land from L2 rather than from a
+// memory system under full load. Lane l takes block l % 4 of warp l / 4's first item; it reads the
+// same plan words and block-table entries that warp reads, and skips out-of-range block ids.
 template <bool kE4M3>
-__global__ void __launch_bounds__(kThreads, 1)
-decode_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap,
-                 const __grid_constant__ CUtensorMap qmap, const TcDecodeParams prm)
+__device__ __forceinline__ void prefetch_warp_lists(const padoc_warp::DecodeParams &w, const CUtensorMap &kmap,
+                                                    const CUtensorMap &vmap, int wc, int lane)
 {
-    extern __shared__ __align__(1024) uint8_t smem[];
-    if (smem_u32(smem) & 1023u) {
-        if (threadIdx.x == 0) padoc_record_error(prm.err, PADOC_DEVERR_SMEM_ALIGN, (int)(smem_u32(smem) & 1023u));
-        return;
+    const int wi = wc * padoc_warp::kWarps + (lane >> 2), b = lane & 3;
+    if (wi >= w.num_warps) return;
+    const int i0 = w.warp_ptr[wi], i1 = w.warp_ptr[wi + 1];
+    if (i0 >= i1) return;
+    const padoc_item it = w.items[w.first_item + i0];
+    const int tok = it.tok_begin + b * kBlk;
+    if (tok >= it.tok_end) return;
+    const int32_t *table = it.kind == PADOC_ITEM_SHARED ? w.page_table + (size_t)it.index * w.page_stride
+                                                        : w.stream_table + (size_t)it.first_stream * w.stream_stride;
+    const int32_t id = table[tok / kBlk];
+    if (id < 0 || id >= w.num_blocks) return;
+    const int32_t row = (id * w.num_kv_heads + it.kv_head) * kBlk;
+    tma_prefetch_l2_2d(&kmap, 0, row);
+    tma_prefetch_l2_2d(&vmap, 0, row);
+    if (!kE4M3) {   // (an E4M3 box holds the whole row)
+        tma_prefetch_l2_2d(&kmap, 64, row);
+        tma_prefetch_l2_2d(&vmap, 64, row);
     }
+}
+
+// The pieces of tensor-core CTA blockIdx.x (every thread of the CTA; smem 1024-byte aligned).
+// kFused: the CTA runs warp lists next (their first blocks are pulled into L2 meanwhile).
+template <bool kE4M3, bool kFused>
+__device__ __forceinline__ void decode_tc_role(const CUtensorMap &kmap, const CUtensorMap &vmap, const CUtensorMap &qmap,
+                                               const TcDecodeParams &prm, const padoc_warp::DecodeParams &wprm,
+                                               uint8_t *smem)
+{
     uint8_t *sq = smem;
     uint8_t *sk = sq + 2 * kTile;
     uint8_t *sv = sk + kKStages * kTile;
@@ -377,9 +406,14 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
                 }
             }
         }
+        // the K producer is done first (its ring runs two tiles ahead): it warms L2 for the warp lists
+        // this CTA runs next (E4M3: after the last expansions below)
+        const int wc = prm.early_ctas + (int)blockIdx.x;
+        if (kFused && !kE4M3 && is_k && wc < prm.warp_ctas) prefetch_warp_lists<kE4M3>(wprm, kmap, vmap, wc, lane);
         if constexpr (kE4M3) {
             // the last tiles' expansion; after a failed wait only their copies are waited for
             while (ok && nc < n) ok = expand_next();
+            if (kFused && is_k && wc < prm.warp_ctas) prefetch_warp_lists<kE4M3>(wprm, kmap, vmap, wc, lane);
             if (lane == 0)
                 for (int J = nc; J < n; ++J)
                     mbar_wait_bounded(bar(b_stg + J % nst), (J / nst) & 1, prm.err, is_k ? 51 : 52);
@@ -738,15 +772,70 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
     }
 }
 
+// Registers per thread of the warp path's eight warps (warpgroups 0 and 1) and of warpgroup 2, which
+// idles there: 256 x 232 + 128 x 24 = 62,464, within the 384 x 168 = 64,512 the CTA is launched
+// with (an increase beyond what the CTA holds would wait forever).
+constexpr uint32_t kWarpPathRegs = 232, kIdleRegs = 24;
+static_assert(2 * 128 * kWarpPathRegs + 128 * kIdleRegs <= (uint32_t)kThreads * 168, "register split");
+static_assert(padoc_warp::kRingBytes <= kSmemBytes && padoc_warp::kRingBytesE4M3 <= kSmemBytes, "warp rings");
+static_assert(padoc_warp::kWarps * 32 == 256, "the warp path runs on warpgroups 0 and 1");
+
+
+// The decode grid (kFused): a CTA runs its tensor-core pieces (CTAs below tc_ctas), then one warp
+// CTA's lists on warps 0-7 with the larger register budget (decode_warp.cuh); warps 8-11 give their
+// registers back and end. A plan without tensor-core work runs warp CTAs only. Without kFused the
+// grid runs the tensor-core pieces only (the E4M3 pool, whose warp lists run in a grid of their own:
+// there the warp path needs more registers than the split leaves it).
+template <bool kE4M3, bool kFused>
+__global__ void __launch_bounds__(kThreads, 1)
+decode_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap,
+                 const __grid_constant__ CUtensorMap qmap, const TcDecodeParams prm,
+                 const padoc_warp::DecodeParams wprm)
+{
+    extern __shared__ __align__(1024) uint8_t smem[];
+    if (smem_u32(smem) & 1023u) {
+        if (threadIdx.x == 0) padoc_record_error(prm.err, PADOC_DEVERR_SMEM_ALIGN, (int)(smem_u32(smem) & 1023u));
+        return;
+    }
+    const bool has_tc = (int)blockIdx.x < prm.tc_ctas;
+    if constexpr (!kFused) {
+        if (has_tc) decode_tc_role<kE4M3, false>(kmap, vmap, qmap, prm, wprm, smem);
+        return;
+    }
+    if (has_tc) {
+        decode_tc_role<kE4M3, true>(kmap, vmap, qmap, prm, wprm, smem);
+    } else {
+        // a CTA with warp lists only: the same wait for the previous kernel in the stream
+        pdl_wait_prerequisite();
+        pdl_launch_dependents();
+    }
+    const int wc = has_tc ? prm.early_ctas + (int)blockIdx.x : (int)blockIdx.x - prm.tc_ctas;
+    const bool lists = wc < prm.warp_ctas;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (warp >= padoc_warp::kWarps) {
+        if (lists) setmaxnreg_dec<kIdleRegs>();
+        return;
+    }
+    if (!lists) return;
+    setmaxnreg_inc<kWarpPathRegs>();
+    // the rings reuse shared memory that the tensor cores and TMA (the async proxy) last accessed
+    fence_proxy_async_smem();
+    const int wi = wc * padoc_warp::kWarps + warp;
+    if (wi < wprm.num_warps) padoc_warp::decode_warp_role<kE4M3>(wprm, smem, warp, lane, wi);
+}
+
 }  // namespace
 
 padoc_status padoc_launch_decode_tc(const CUtensorMap *kmap, const CUtensorMap *vmap, const CUtensorMap *qmap, const int32_t *plan,
                                     const padoc_decode_plan *info, const int32_t *page_table, int32_t page_stride,
                                     const int32_t *stream_table, int32_t stream_stride, int32_t num_blocks,
                                     const float *k_scales, const float *v_scales, float *part_o, float *part_lse,
-                                    float scale_log2, int *err, cudaStream_t stream)
+                                    float scale_log2, int *err, const padoc_warp::DecodeParams *wprm,
+                                    cudaStream_t stream)
 {
-    if (info->num_tc_items == 0 || info->tc_ctas == 0) return PADOC_OK;
+    const bool e4m3 = k_scales != nullptr;   // an E4M3 pool: the maps hold codes
+    const bool fused = !e4m3;
+    if (info->num_tc_items == 0 && (!fused || wprm->num_warps == 0)) return PADOC_OK;
     TcDecodeParams prm;
     prm.shared_len = plan + info->off_shared_len;
     prm.private_len = plan + info->off_private_len;
@@ -769,11 +858,13 @@ padoc_status padoc_launch_decode_tc(const CUtensorMap *kmap, const CUtensorMap *
     prm.part_lse = part_lse;
     prm.scale_log2 = scale_log2;
     prm.err = err;
-    const bool e4m3 = k_scales != nullptr;   // an E4M3 pool: the maps hold codes
-    auto kern = e4m3 ? decode_tc_kernel<true> : decode_tc_kernel<false>;
+    prm.tc_ctas = info->num_tc_items > 0 ? info->tc_ctas : 0;
+    prm.warp_ctas = fused ? (wprm->num_warps + padoc_warp::kWarps - 1) / padoc_warp::kWarps : 0;
+    prm.early_ctas = padoc_fused_early_ctas(prm.tc_ctas, prm.warp_ctas, padoc_default_ctas());
+    auto kern = e4m3 ? decode_tc_kernel<true, false> : decode_tc_kernel<false, true>;
     PADOC_CUDA_TRY(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes));
     cudaLaunchConfig_t lc = {};
-    lc.gridDim = dim3((unsigned)info->tc_ctas);
+    lc.gridDim = dim3((unsigned)(prm.tc_ctas + prm.early_ctas));
     lc.blockDim = dim3(kThreads);
     lc.dynamicSmemBytes = kSmemBytes;
     lc.stream = stream;
@@ -782,6 +873,6 @@ padoc_status padoc_launch_decode_tc(const CUtensorMap *kmap, const CUtensorMap *
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     lc.attrs = attr;
     lc.numAttrs = 1;
-    PADOC_CUDA_TRY(cudaLaunchKernelEx(&lc, kern, *kmap, *vmap, *qmap, prm));
+    PADOC_CUDA_TRY(cudaLaunchKernelEx(&lc, kern, *kmap, *vmap, *qmap, prm, *wprm));
     return padoc_launch_status();
 }

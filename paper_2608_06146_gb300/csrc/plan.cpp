@@ -228,9 +228,6 @@ extern "C" padoc_status padoc_prefill_bwd_tile_shapes(padoc_dtype dtype, int32_t
 // Decode plan
 // ------------------------------------------------------------------------------------------------
 
-namespace {
-
-
 // Multiprocessor count of the current CUDA device, or 152 (one GB300) when none is visible; the
 // device attribute is read once per device (a plan is built for every decode step).
 int32_t padoc_default_ctas()
@@ -253,6 +250,8 @@ int32_t padoc_default_ctas()
     if (dev >= 0 && dev < kMaxDevices) cached[dev].store(n, std::memory_order_relaxed);
     return n;
 }
+
+namespace {
 
 int32_t choose_tc_ctas(const PlanParts &pp, const padoc_decode_config *cfg, int64_t total_w, int64_t max_piece);
 
@@ -514,6 +513,27 @@ padoc_status build_work(int32_t num_pages, const padoc_decode_config *cfg, PlanP
         }
         ctas = (int32_t)walk(lo, true);
         pp.cta_ptr.push_back((int32_t)tc_items.size());
+        // The CTAs in order of planned load, lightest first, so that they are predicted to end in
+        // index order: warp CTA early + j then follows tensor-core CTA j's pieces in the decode grid,
+        // and takes the SM of the j-th CTA to end in a warp grid of its own (the E4M3 pool), both
+        // with the start the warp planning below gives it.
+        std::vector<int32_t> perm((size_t)ctas);
+        std::iota(perm.begin(), perm.end(), 0);
+        std::stable_sort(perm.begin(), perm.end(),
+                         [&](int32_t a, int32_t b) { return tc_load[(size_t)a] < tc_load[(size_t)b]; });
+        std::vector<padoc_item> items_sorted;
+        items_sorted.reserve(tc_items.size());
+        std::vector<int32_t> ptr_sorted(1, 0);
+        std::vector<int64_t> load_sorted;
+        for (int32_t c : perm) {
+            items_sorted.insert(items_sorted.end(), tc_items.begin() + pp.cta_ptr[(size_t)c],
+                                tc_items.begin() + pp.cta_ptr[(size_t)c + 1]);
+            ptr_sorted.push_back((int32_t)items_sorted.size());
+            load_sorted.push_back(tc_load[(size_t)c]);
+        }
+        tc_items.swap(items_sorted);
+        pp.cta_ptr.swap(ptr_sorted);
+        tc_load.swap(load_sorted);
     }
     pp.tc_ctas = ctas;
 
@@ -582,10 +602,10 @@ padoc_status build_work(int32_t num_pages, const padoc_decode_config *cfg, PlanP
     pp.items.resize(tc_items.size() + (size_t)nitems);
     std::copy(tc_items.begin(), tc_items.end(), pp.items.begin());
     if (nwarps > 0) {
-        // Warp CTAs start at different times: the first (SMs - tensor-core CTAs) of them on SMs the
-        // tensor-core grid leaves free, soon after launch; the others, in index order, on the SMs
-        // that tensor-core CTAs free as they finish (predicted from their planned loads). A warp's
-        // share of the work is sized to the time it has: its capacity is its rate times
+        // Warp CTAs start at different times (the fused grid's mapping is in plan_internal.h): the
+        // first `early` of them on SMs the tensor-core CTAs leave free, soon after launch; warp CTA
+        // early + j on tensor-core CTA j once its pieces end (predicted from its planned load). A
+        // warp's share of the work is sized to the time it has: its capacity is its rate times
         // (T - its CTA's start - the time to its first block), with T such that the capacities add
         // up to the work. Taking items longest first, each to the warp with the most capacity left,
         // puts the longest items on the warps that start first. Without tensor-core work every warp
@@ -596,17 +616,23 @@ padoc_status build_work(int32_t num_pages, const padoc_decode_config *cfg, PlanP
         for (int32_t c = 0; c < wctas; ++c)
             nw_of[(size_t)c] = std::min<int32_t>(PADOC_WARP_KERNEL_WARPS, nwarps - c * PADOC_WARP_KERNEL_WARPS);
         if (!tc_load.empty()) {
+            const int32_t nsm = padoc_default_ctas(), ntc = (int32_t)tc_load.size();
+            const int32_t early = padoc_fused_early_ctas(ntc, wctas, nsm);
+            // early warp CTAs past the SM count (a warp_ctas above it) wait for a CTA to end
+            const int32_t resident = std::min(early, std::max(0, nsm - ntc));
             std::vector<double> tend(tc_load.size());
-            for (size_t c = 0; c < tc_load.size(); ++c) tend[c] = PADOC_TC_END_US0 + PADOC_TC_US_PER_UNIT * (double)tc_load[c];
-            std::sort(tend.begin(), tend.end());
-            const int32_t nfree = std::max<int32_t>(0, padoc_default_ctas() - (int32_t)tc_load.size());
+            double tmax = 0.0;
+            for (size_t c = 0; c < tc_load.size(); ++c) {
+                tend[c] = PADOC_TC_END_US0 + PADOC_TC_US_PER_UNIT * (double)tc_load[c];
+                tmax = std::max(tmax, tend[c]);
+            }
             for (int32_t c = 0; c < wctas; ++c) {
-                if (c < nfree) {
+                if (c < resident) {
                     start[(size_t)c] = PADOC_WARP_EARLY_START_US;
                     rate[(size_t)c] = PADOC_WARP_EARLY_RATE;
                 } else {
-                    const size_t k = std::min<size_t>((size_t)(c - nfree), tend.size() - 1);
-                    start[(size_t)c] = tend[k] + PADOC_WARP_START_DELAY_US + PADOC_WARP_FIRST_US;
+                    const double t0 = c < early ? tmax : tend[(size_t)(c - early)];
+                    start[(size_t)c] = t0 + PADOC_WARP_SWITCH_US + PADOC_WARP_FIRST_US;
                 }
             }
         }
@@ -675,7 +701,7 @@ padoc_status build_work(int32_t num_pages, const padoc_decode_config *cfg, PlanP
 // it) gets a predicted end of step: the tensor-core CTAs end on average at
 // PADOC_TC_END_US0 + PADOC_TC_US_PER_UNIT * (total load / n + one piece) and the last of them
 // PADOC_TC_END_SPREAD_US later, and the warp work, sized to each warp's start as in the planner
-// (warp CTAs that wait for a tensor-core CTA start at the average end), ends at T; the count whose
+// (warp CTAs that follow a tensor-core CTA's pieces start at the average end), ends at T; the count whose
 // later of the two ends is earliest wins (the larger count on a tie).
 int32_t choose_tc_ctas(const PlanParts &pp, const padoc_decode_config *cfg, int64_t total_w, int64_t max_piece)
 {
@@ -707,7 +733,7 @@ int32_t choose_tc_ctas(const PlanParts &pp, const padoc_decode_config *cfg, int6
     for (int32_t n = nsm; n >= std::max(1, nsm / 2); n -= 8) {
         const double tc_end = PADOC_TC_END_US0 + PADOC_TC_US_PER_UNIT * ((double)total_w / n + (double)max_piece);
         const double ne = (double)std::min<int64_t>(std::max(0, nsm - n), wctas), nl = (double)wctas - ne;
-        const double se = PADOC_WARP_EARLY_START_US, sl = tc_end + PADOC_WARP_START_DELAY_US + PADOC_WARP_FIRST_US;
+        const double se = PADOC_WARP_EARLY_START_US, sl = tc_end + PADOC_WARP_SWITCH_US + PADOC_WARP_FIRST_US;
         const double ae = PADOC_WARP_KERNEL_WARPS * PADOC_WARP_EARLY_RATE * ne, al = PADOC_WARP_KERNEL_WARPS * PADOC_WARP_RATE * nl;
         // capacity at T: ae (T - se) + al max(0, T - sl) (se < sl); solve for T = the warp work
         double T = ae > 0 ? se + (double)wcost / ae : 1e300;

@@ -47,23 +47,53 @@
 #define PADOC_WARP_KERNEL_WARPS 8
 #define PADOC_WARP_ITEM_COST 2
 // Timing model of one decode step, fitted on GB300 to per-CTA and per-warp timelines of the serving
-// batch (times in microseconds from the start of the tensor-core grid), used to size each warp's
-// share: a tensor-core CTA with a planned load of L units (the weights above) ends at about
-// PADOC_TC_END_US0 + PADOC_TC_US_PER_UNIT * L; a warp CTA on an SM the tensor-core grid leaves free
+// batch (times in microseconds from the start of the decode grid), used to size each warp's share:
+// a tensor-core CTA with a planned load of L units (the weights above) ends at about
+// PADOC_TC_END_US0 + PADOC_TC_US_PER_UNIT * L; a warp CTA on an SM the tensor-core CTAs leave free
 // starts at PADOC_WARP_EARLY_START_US and works through PADOC_WARP_EARLY_RATE cost units (16-token
-// blocks plus PADOC_WARP_ITEM_COST per item) per microsecond; one that waits for a tensor-core CTA
-// starts PADOC_WARP_START_DELAY_US after it ends, needs PADOC_WARP_FIRST_US before its first block
-// lands (the memory system is busiest then) and then works through PADOC_WARP_RATE units per
+// blocks plus PADOC_WARP_ITEM_COST per item) per microsecond; one that a tensor-core CTA runs after
+// its pieces starts PADOC_WARP_SWITCH_US after they end, needs PADOC_WARP_FIRST_US before its first
+// block lands (the memory system is busiest then) and then works through PADOC_WARP_RATE units per
 // microsecond.
+#ifndef PADOC_TC_END_US0
 #define PADOC_TC_END_US0 5.6
+#endif
+#ifndef PADOC_TC_US_PER_UNIT
 #define PADOC_TC_US_PER_UNIT 0.238
+#endif
 // the last tensor-core CTA of a step ends about this long after the average one
+#ifndef PADOC_TC_END_SPREAD_US
 #define PADOC_TC_END_SPREAD_US 2.5
+#endif
+#ifndef PADOC_WARP_EARLY_START_US
 #define PADOC_WARP_EARLY_START_US 5.2
-#define PADOC_WARP_START_DELAY_US 0.4
+#endif
+#ifndef PADOC_WARP_SWITCH_US
+#define PADOC_WARP_SWITCH_US 0.2
+#endif
+#ifndef PADOC_WARP_FIRST_US
 #define PADOC_WARP_FIRST_US 5.3
+#endif
+#ifndef PADOC_WARP_RATE
 #define PADOC_WARP_RATE 1.53
+#endif
+#ifndef PADOC_WARP_EARLY_RATE
 #define PADOC_WARP_EARLY_RATE 1.28
+#endif
+
+// The fused decode grid: CTA c < tc_ctas runs tensor-core CTA c's pieces and then one warp CTA's
+// lists (8 warps); the CTAs from tc_ctas on run warp CTAs' lists from the start. Warp CTAs
+// [0, early) go to CTAs tc_ctas + c (the SMs the tensor-core CTAs leave free: they start first, so
+// the planner gives them the longest items), warp CTA early + j to tensor-core CTA j. early is the
+// number of free SMs, raised where needed so that every warp CTA has a CTA:
+// max(min(warp_ctas, sm_count - tc_ctas), warp_ctas - tc_ctas, 0). The grid has tc_ctas + early CTAs.
+static inline int32_t padoc_fused_early_ctas(int32_t tc_ctas, int32_t warp_ctas, int32_t sm_count)
+{
+    int32_t e = sm_count - tc_ctas;
+    if (e > warp_ctas) e = warp_ctas;
+    if (e < warp_ctas - tc_ctas) e = warp_ctas - tc_ctas;
+    return e > 0 ? e : 0;
+}
 
 #define PADOC_ITEM_INTS 8
 enum { PADOC_ITEM_SHARED = 0, PADOC_ITEM_PRIVATE = 1, PADOC_ITEM_SHARED_TC = 2, PADOC_ITEM_PRIVATE_TC = 3 };
@@ -80,9 +110,9 @@ enum { PADOC_ITEM_SHARED = 0, PADOC_ITEM_PRIVATE = 1, PADOC_ITEM_SHARED_TC = 2, 
 #define PADOC_ITEM_KIND(k) ((k) & 15)
 
 // One split-K work item of the decode kernels (8 int32 words in the plan blob). The blob holds
-// the tensor-core items first ([0, num_tc_items)), CTA c of the tensor-core grid owning items
-// [cta_ptr[c], cta_ptr[c+1]) in order, then the warp items, warp w of the warp grid owning
-// items num_tc_items + [warp_ptr[w], warp_ptr[w+1]) in order. A warp item's tok_end never passes
+// the tensor-core items first ([0, num_tc_items)), tensor-core CTA c owning items
+// [cta_ptr[c], cta_ptr[c+1]) in order, then the warp items, warp w (warp w % 8 of warp CTA w / 8)
+// owning items num_tc_items + [warp_ptr[w], warp_ptr[w+1]) in order. A warp item's tok_end never passes
 // its stream's cutoff (shared_len or private_len), so the warp kernel reads no cutoff.
 //   kind        PADOC_ITEM_SHARED_TC: tokens [tok_begin, tok_end) of page `index`'s shared stream for
 //               streams [first_stream, first_stream + num_streams) (<= 32) of that page, each with

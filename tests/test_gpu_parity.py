@@ -117,7 +117,7 @@ def test_decode_bf16_tensor_core_edge_pages():
     assert_close(*run_decode(wl, 10, split_tokens=128), torch.bfloat16)
 
 
-@pytest.mark.parametrize("tc_ctas,warp_ctas", [(1, 1), (3, 2), (7, 5), (40, 0), (1000, 1000)])
+@pytest.mark.parametrize("tc_ctas,warp_ctas", [(1, 1), (3, 2), (7, 5), (40, 0), (5, 400), (1000, 1000)])
 def test_decode_bf16_tensor_core_ctas_walk_many_pieces(tc_ctas, warp_ctas):
     # few CTAs: each walks many pieces of different pages, KV heads and M-tile counts back to back
     # (the K/V ring, barrier phases and query reloads carry across pieces), and each warp of the
@@ -132,6 +132,14 @@ def test_decode_bf16_tensor_core_ctas_walk_many_pieces(tc_ctas, warp_ctas):
     wl = Workload("tc walk", pages, 16, 2, 128, torch.bfloat16, "decode")
     assert_close(*run_decode(wl, 12, layout_streams=bool(tc_ctas & 1), tc_ctas=tc_ctas, warp_ctas=warp_ctas),
                  torch.bfloat16)
+
+
+def test_decode_bf16_serving_batch_warp_ctas_beyond_the_sm_count():
+    # few tensor-core CTAs and more warp CTAs than SMs: the grid holds more CTAs than fit at once,
+    # so warp CTAs past the SM count start only as others end (the pairing of warp CTAs with
+    # tensor-core CTAs in plan_internal.h)
+    wl = inputs.serving_batch()
+    assert_close(*run_decode(wl, 13, tc_ctas=5, warp_ctas=400), torch.bfloat16)
 
 
 def test_decode_repeated_calls_on_one_workspace():

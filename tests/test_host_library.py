@@ -225,6 +225,9 @@ def check_decode_plan(wl, layout, tc_ctas, warp_ctas):
                     for u in range(cta[c], cta[c + 1])) for c in range(info.tc_ctas)]
         if info.tc_ctas == want:
             assert max(work) <= sum(work) / want + 2 * (8 + 11)
+        # lightest first: the CTAs are predicted to end in index order, which the warp planning and
+        # the decode grid's pairing of warp CTAs with tensor-core CTAs rely on
+        assert all(a <= b for a, b in zip(work, work[1:]))
     else:
         assert info.tc_ctas == 0
     # the warp grid: warp lists cover the warp items in order, one wave, balanced by cost
