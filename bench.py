@@ -44,8 +44,10 @@ METRIC = "ancestor-attn decode queries/s, % of HBM roofline; packed prefill TFLO
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 # DRAM traffic per launch, dram__bytes_read.sum + dram__bytes_write.sum, copied from one ncu capture
 # of each kernel as it stands (cold caches); None where no capture of the current kernel exists.
-# Decode: one step = its three kernels' counters added up. Prefill backward: both passes.
-TRAFFIC_BYTES = {"decode": 224_800_000,
+# Decode: one step = its kernels' counters added up (bf16: the decode grid and the merge; E4M3: the
+# tensor-core grid, the warp grid and the merge). Prefill backward: both passes.
+TRAFFIC_BYTES = {"decode": 223_312_512,
+                 "decode_e4m3": 124_968_832,
                  "prefill": 260_600_000,
                  "prefill_bwd": 1_459_570_000}
 
@@ -1005,7 +1007,7 @@ def main():
             "workload": "the serving-batch decode step over the FP8 (E4M3) KV cache (codes + one fp32 scale per "
                         "(block, KV head)), quantized from the same bf16 cache",
             "roofline": {"bound": "hbm", "achieved": ach, "peak": peaks["hbm_gbs"], "unit": "GB/s",
-                         "frac": ach / peaks["hbm_gbs"], "traffic": None,
+                         "frac": ach / peaks["hbm_gbs"], "traffic": TRAFFIC_BYTES["decode_e4m3"],
                          "algorithmic_bytes": d8["bytes"],
                          "bytes_rule": "each page's visible shared stream once and every private row once at 1 byte "
                                        "per K/V element, plus a 4-byte K and V scale per (16-token block, KV head), Q "
