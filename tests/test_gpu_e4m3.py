@@ -57,10 +57,13 @@ def run_decode_e4m3(wl, seed, layout_streams=False, split_tokens=0, tc_ctas=0, w
     out = torch.full((S, wl.num_q_heads, wl.head_dim), float("nan"), dtype=torch.bfloat16, device=DEV)
     lse = torch.full((S, wl.num_q_heads), float("nan"), dtype=torch.float32, device=DEV)
     scale = 1.0 / math.sqrt(wl.head_dim)
-    pa.padoc_branch_decode_attn_e4m3(pool, plan.info, plan.plan_dev, torch.from_numpy(di.page_table).to(DEV),
-                                     torch.from_numpy(di.stream_table).to(DEV), di.q.to(DEV), scale, out, lse,
-                                     plan.workspace)
+    pt, st, q = torch.from_numpy(di.page_table).to(DEV), torch.from_numpy(di.stream_table).to(DEV), di.q.to(DEV)
+    pa.padoc_branch_decode_attn_e4m3(pool, plan.info, plan.plan_dev, pt, st, q, scale, out, lse, plan.workspace)
+    # a second call on the same plan and workspace: bit-identical
+    out2, lse2 = torch.full_like(out, float("nan")), torch.full_like(lse, float("nan"))
+    pa.padoc_branch_decode_attn_e4m3(pool, plan.info, plan.plan_dev, pt, st, q, scale, out2, lse2, plan.workspace)
     pa.padoc_check_device_errors()
+    assert torch.equal(out, out2) and torch.equal(lse, lse2)
     kc, ks, vc, vs = _codes(pool)
     ref_o, ref_l = oracle.decode_paged(wl.pages, oracle.dequantize_kv_blocks(kc, ks), oracle.dequantize_kv_blocks(vc, vs),
                                        di.page_table, di.stream_table, di.q, scale, layout_streams)

@@ -44,9 +44,15 @@ def run_decode(wl: Workload, seed: int, layout_streams=False, split_tokens=0, sc
     out = torch.full((S, wl.num_q_heads, wl.head_dim), float("nan"), dtype=wl.dtype, device=DEV)
     lse = torch.full((S, wl.num_q_heads), float("nan"), dtype=torch.float32, device=DEV)
     scale = 1.0 / math.sqrt(wl.head_dim)
-    plan.run(di.k_pool.to(DEV), di.v_pool.to(DEV), torch.from_numpy(di.page_table).to(DEV),
-             torch.from_numpy(di.stream_table).to(DEV), q, scale, out, lse)
+    args = (di.k_pool.to(DEV), di.v_pool.to(DEV), torch.from_numpy(di.page_table).to(DEV),
+            torch.from_numpy(di.stream_table).to(DEV), q, scale)
+    plan.run(*args, out, lse)
+    # a second call on the same plan and workspace gives a bit-identical result (every partial and
+    # the merge's order are fixed by the plan)
+    out2, lse2 = torch.full_like(out, float("nan")), torch.full_like(lse, float("nan"))
+    plan.run(*args, out2, lse2)
     pa.padoc_check_device_errors()
+    assert torch.equal(out, out2) and torch.equal(lse, lse2)
     ref_o, ref_lse = oracle.decode_pages(wl.pages, di, scale, layout_streams)
     return out.float().cpu().numpy(), lse.cpu().numpy(), ref_o, ref_lse
 
