@@ -45,11 +45,12 @@ FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustain
 # DRAM traffic per launch, dram__bytes_read.sum + dram__bytes_write.sum, copied from one ncu capture
 # of each kernel as it stands (cold caches); None where no capture of the current kernel exists.
 # Decode: one step = its kernels' counters added up (bf16: the decode grid and the merge; E4M3: the
-# tensor-core grid, the warp grid and the merge). Prefill backward: both passes.
+# tensor-core grid, the warp grid and the merge). Prefill backward: both passes and the merge of the
+# split key tiles.
 TRAFFIC_BYTES = {"decode": 223_312_512,
                  "decode_e4m3": 124_968_832,
                  "prefill": 260_600_000,
-                 "prefill_bwd": 1_459_570_000}
+                 "prefill_bwd": 1_670_324_480}
 
 
 def load_peaks():

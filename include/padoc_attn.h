@@ -626,7 +626,8 @@ typedef struct {
 } padoc_tile_map_dev;
 
 /* Workspace of padoc_ancestor_prefill_bwd: two fp32 arrays [Hq][ceil(T/128)*128] (per head the
- * negated base-2 log-sum-exp of the forward and D = rowsum(dO * O)), 256-byte aligned. */
+ * negated base-2 log-sum-exp of the forward and D = rowsum(dO * O)), then 2048 bytes per padded row
+ * for the fp32 partials of the heaviest key tiles, whose gradients two CTAs share; 256-byte aligned. */
 padoc_status padoc_prefill_bwd_workspace_size(int64_t total_tokens, int32_t num_q_heads, size_t *bytes);
 
 /* Gradients of the packed ancestor prefill for an upstream gradient dO (App. C.1; Sec. 3.2

@@ -379,8 +379,8 @@ padoc_status padoc_launch_prefill_bwd_tc(const void *q, const void *k, const voi
                                          const void *dout, const float *lse, int64_t total_tokens,
                                          int32_t num_q_heads, int32_t num_kv_heads, const int32_t *spans_dev,
                                          const padoc_tile_map_dev *q_map, const padoc_tile_map_dev *k_map, float *lt,
-                                         float *dt, int64_t t_pad, float scale, void *dq, void *dk, void *dv,
-                                         cudaStream_t stream);
+                                         float *dt, float *split, int64_t t_pad, float scale, void *dq, void *dk,
+                                         void *dv, cudaStream_t stream);
 int padoc_num_sms();
 // SM count the planner sizes grids for (the current device's, read once; 152 without a device)
 int32_t padoc_default_ctas();

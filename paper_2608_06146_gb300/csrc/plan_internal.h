@@ -16,6 +16,14 @@
 #define PADOC_BWD_DQ_K_TILE 64
 #define PADOC_BWD_DKV_Q_TILE 64
 #define PADOC_BWD_DKV_K_TILE 128
+// A dK/dV work unit (k-tile, KV head) of more steps ((q-tile, query head) pairs) than this is split
+// between two CTAs, each over half of its steps, whose fp32 partials a small kernel adds: the first
+// k-tiles of a page are seen by up to 64 q-tiles x 8 heads, and as single CTAs they set the pass's
+// tail (measured: 927 us against 681 us of work per SM). Only the heaviest units can split (those
+// whose position in the key-major order is below k-tiles / KV heads), so that the partials fit in
+// PADOC_BWD_SPLIT_BYTES_PER_TOKEN bytes of workspace per token.
+#define PADOC_BWD_SPLIT_STEPS 256
+#define PADOC_BWD_SPLIT_BYTES_PER_TOKEN 2048
 
 // Decode split-K: shared-stream tokens per partial result and private tokens per partial result.
 // 256 rather than 512: in decoding-loop steps with few streams the warp items on a page's shared

@@ -172,7 +172,10 @@ bool map_ok(const padoc_tile_map_dev *m, bool key_major, int32_t q_tile, int32_t
 extern "C" padoc_status padoc_prefill_bwd_workspace_size(int64_t total_tokens, int32_t num_q_heads, size_t *bytes)
 {
     if (!bytes || total_tokens < 0 || total_tokens >= INT32_MAX || num_q_heads < 1) return PADOC_ERR_INVALID_ARGUMENT;
-    *bytes = 2 * (size_t)num_q_heads * (size_t)pad_rows(total_tokens) * sizeof(float);
+    // -lse2 and D per head, then the split dK/dV units' fp32 partials: at most ceil(T / 128) units,
+    // each two halves x (dV, dK) x 128 keys x 128 dims
+    *bytes = 2 * (size_t)num_q_heads * (size_t)pad_rows(total_tokens) * sizeof(float) +
+             (size_t)pad_rows(total_tokens) * PADOC_BWD_SPLIT_BYTES_PER_TOKEN;
     return PADOC_OK;
 }
 
@@ -207,11 +210,12 @@ extern "C" padoc_status padoc_ancestor_prefill_bwd(const void *q, const void *k,
     const int64_t T = total_tokens, t_pad = pad_rows(T);
     float *lt = (float *)workspace;
     float *dt = lt + (size_t)num_q_heads * t_pad;
+    float *split = dt + (size_t)num_q_heads * t_pad;   // the split dK/dV units' partials
     const float c = scale * PADOC_LOG2E;
     const unsigned sgrid = (unsigned)((t_pad * num_q_heads + 7) / 8);
     if (dtype == PADOC_DTYPE_BF16)   // the tensor-core dQ pass computes the statistics itself
         return padoc_launch_prefill_bwd_tc(q, k, v, out, dout, lse, T, num_q_heads, num_kv_heads, spans_dev, q_map,
-                                           k_map, lt, dt, t_pad, scale, dq, dk, dv, cs);
+                                           k_map, lt, dt, split, t_pad, scale, dq, dk, dv, cs);
     const unsigned qgrid = (unsigned)((T * num_q_heads + 3) / 4), kgrid = (unsigned)((T * num_kv_heads + 3) / 4);
 #define PADOC_BWD_F32(D)                                                                                              \
     do {                                                                                                              \

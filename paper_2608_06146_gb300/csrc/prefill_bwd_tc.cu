@@ -7,7 +7,10 @@
 //   P = exp2(S c - lse2),  dS = P (dP - D),  S = Q K^T,  dP = dO V^T.
 //
 // dK/dV pass: one CTA per (128-key k-tile, KV head), k-tiles taken in the key-major map's order
-//   (most work first). K and V of the tile sit in tensor memory as A operands for the whole walk.
+//   (most work first); a unit with more than PADOC_BWD_SPLIT_STEPS steps runs as two CTAs over its
+//   two halves of steps, which write fp32 partials that prefill_bwd_dkv_merge_kernel adds (the
+//   heaviest units otherwise set the pass's tail). K and V of the tile sit in tensor memory as A
+//   operands for the whole walk.
 //   For every (32-row q-tile that sees the k-tile, query head reading the KV head) step the tensor
 //   cores form S^T = K Q^T and dP^T = V dO^T (M = 128 keys, N = 32 queries, B from shared memory),
 //   the softmax warps write P^T and dS^T back into tensor memory as bf16, and dV += P^T dO,
@@ -36,6 +39,7 @@
 // memory is released.
 #include <math.h>
 
+#include <algorithm>
 #include <type_traits>
 
 #include "common.cuh"
@@ -58,6 +62,8 @@ struct BwdParams {
     int32_t num_q_heads, num_kv_heads, num_tiles;
     float scale_log2, scale;
     __nv_bfloat16 *out0, *out1;         // dK/dV pass: dK, dV; dQ pass: dQ
+    float *split;                       // dK/dV pass: fp32 partials of the split units
+    int32_t split_units;                // dK/dV pass: units of the key-major order below this may split
     int *err;
 };
 
@@ -117,6 +123,24 @@ __device__ __forceinline__ void row_to_tmem(uint32_t taddr, const __nv_bfloat16 
     tmem_st32(taddr, w);
 }
 
+__device__ __forceinline__ int clamp_w(int x, int w) { return min(max(x, 0), w); }
+
+// 32 x 32 bit-matrix transpose across a warp: lane r holds row r (bit c = element (r, c)); on return
+// lane r holds column r (bit c = element (c, r)). Five exchange rounds, each swapping the off-diagonal
+// j x j blocks between lanes r and r ^ j.
+__device__ __forceinline__ uint32_t transpose32_warp(uint32_t x, int lane)
+{
+    uint32_t m = 0x0000FFFFu;
+#pragma unroll
+    for (int j = 16; j != 0; j >>= 1) {
+        const uint32_t o = __shfl_xor_sync(0xffffffffu, x, j);
+        if (lane & j) x ^= ((o >> j) ^ x) & m;
+        else x ^= (((x >> j) ^ o) & m) << j;
+        m ^= m << (j >> 1);
+    }
+    return x;
+}
+
 // ================================================================================================
 // dK/dV pass
 // ================================================================================================
@@ -162,9 +186,16 @@ prefill_bwd_dkv_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_co
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int hkv = prm.num_kv_heads, group = prm.num_q_heads / hkv;
-    const int kt = prm.order[blockIdx.x / hkv], g = (int)(blockIdx.x % hkv);
+    // CTA b: KV head b % hkv of the (b / hkv) % 2-th half of unit b / (2 hkv) of the key-major order;
+    // a unit of more than PADOC_BWD_SPLIT_STEPS steps (among the first split_units) runs as two
+    // halves that write fp32 partials, the others as one CTA (the second CTA leaves at once)
+    const int unit = (int)(blockIdx.x / (2 * hkv)), half = (int)((blockIdx.x / hkv) & 1), g = (int)(blockIdx.x % hkv);
+    const int kt = prm.order[unit];
     const int e0 = prm.ptr[kt], ne = prm.ptr[kt + 1] - e0;
-    const int nu = ne * group;
+    const bool split = ne * group > PADOC_BWD_SPLIT_STEPS && unit < prm.split_units;
+    if (half == 1 && !split) return;
+    const int ub = half ? ne * group / 2 : 0;                               // first step of this CTA
+    const int nu = split ? (half ? ne * group - ub : ne * group / 2) : ne * group;
     auto bar = [&](int i) { return smem_u32(&bars[i]); };
 
     if (tid == 0) {
@@ -198,7 +229,7 @@ prefill_bwd_dkv_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_co
                 const int s = u % kStages;
                 if (u >= kStages && !wait_or_abort(bar(B_QEMPTY + s), (u / kStages - 1) & 1, prm.err, 50, abort_flag))
                     break;
-                const int e = e0 + u / group, h = g * group + u % group;
+                const int e = e0 + (ub + u) / group, h = g * group + (ub + u) % group;
                 const int q0 = prm.idx[e] * kQT;
                 const int nsp = prm.kind[e] == PADOC_TILE_FULL ? 0 : min(kQT, (int)(prm.T - q0)) * 16;
                 const uint32_t fb = bar(B_QFULL + s);
@@ -299,7 +330,7 @@ prefill_bwd_dkv_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_co
         for (int u = 0; u < nu; ++u) {
             const int s = u % kStages;
             const uint32_t b = (uint32_t)(u & 1) * 64 + 32 * ch;
-            const int e = e0 + u / group;
+            const int e = e0 + (ub + u) / group;
             const bool partial = prm.kind[e] != PADOC_TILE_FULL;
             const int qbase = prm.idx[e] * kQT + 32 * ch;
             if (!wait_all(B_SFULL + (u & 1), (u >> 1) & 1, 70) || !wait_all(B_QFULL + s, (u / kStages) & 1, 71)) {
@@ -314,15 +345,21 @@ prefill_bwd_dkv_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_co
             const float4 *da = reinterpret_cast<const float4 *>(aux + s * kAuxBytes + kQT * 4) + 8 * ch;
             const int4 *sp = reinterpret_cast<const int4 *>(aux + s * kAuxBytes + 2 * kQT * 4) + 32 * ch;
             uint32_t vis = 0xffffffffu;
-            if (partial) {
-                vis = 0u;
+            if (partial) {   // (warp-uniform)
+                // lane i: which of the warp's 32 keys query qbase + i sees (its two spans as bit
+                // intervals); a 32 x 32 bit transpose across the warp then gives each key's bits over
+                // the 32 queries
                 const int64_t rem = prm.T - qbase;   // query columns past T hold no spans
                 const int nvalid = rem <= 0 ? 0 : (rem >= 32 ? 32 : (int)rem);
-                for (int i = 0; i < nvalid; ++i) {
-                    const int4 w = sp[i];
-                    const bool in = (key >= w.x && key < w.y) || (key >= w.z && key < w.w);
-                    vis |= (uint32_t)in << i;
+                const int kbase = kt * kKT + lq * 32;
+                uint32_t x = 0u;
+                if (lane < nvalid) {
+                    const int4 w = sp[lane];
+                    const int lo0 = clamp_w(w.x - kbase, 32), lo1 = clamp_w(w.z - kbase, 32);
+                    x = interval_bits(lo0, max(clamp_w(w.y - kbase, 32) - lo0, 0), 0) |
+                        interval_bits(lo1, max(clamp_w(w.w - kbase, 32) - lo1, 0), 0);
                 }
+                vis = transpose32_warp(x, lane);
             }
             tmem_ld_wait();
             uint32_t pk[16], dk[16];
@@ -359,11 +396,14 @@ prefill_bwd_dkv_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_co
             tc_fence_before();
             mbar_arrive(bar(B_PFULL + (u & 1)));
         }
-        // epilogue: column half 0 writes dV, half 1 writes dK (times scale), one key row per thread
+        // epilogue: column half 0 writes dV, half 1 writes dK (times scale), one key row per thread;
+        // a split unit's halves write their fp32 sums instead ([unit][g][half][dV, dK][key][dim])
         if (ok && (nu == 0 || wait_all(B_FINAL, 0, 72))) {
             tc_fence_after();
             const bool isk = ch == 1;
             __nv_bfloat16 *dst = (isk ? prm.out0 : prm.out1) + ((size_t)(key < prm.T ? key : 0) * hkv + g) * kD;
+            float *pdst = prm.split + ((((size_t)unit * hkv + g) * 2 + half) * 2 + (isk ? 1 : 0)) * (kKT * kD) +
+                          (size_t)(lq * 32 + lane) * kD;
             const float mul = isk ? prm.scale : 1.f;
 #pragma unroll
             for (int cc = 0; cc < 4; ++cc) {
@@ -375,7 +415,13 @@ prefill_bwd_dkv_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_co
 #pragma unroll
                     for (int i = 0; i < 32; ++i) o[i] = 0u;
                 }
-                if (key < prm.T) store_row_bf16(dst + 32 * cc, o, mul);
+                if (split) {
+#pragma unroll
+                    for (int i = 0; i < 32; i += 4)
+                        *reinterpret_cast<uint4 *>(pdst + 32 * cc + i) = make_uint4(o[i], o[i + 1], o[i + 2], o[i + 3]);
+                } else if (key < prm.T) {
+                    store_row_bf16(dst + 32 * cc, o, mul);
+                }
             }
         }
     }
@@ -384,6 +430,31 @@ prefill_bwd_dkv_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_co
     if (warp == 9) {
         tc_fence_after();
         tmem_dealloc(tmem, kTmemCols);
+    }
+}
+
+// The split units' halves added (fp32), dK times scale, rounded once to bf16: one CTA per unit that
+// may split (those that did not leave at once).
+__global__ void __launch_bounds__(256) prefill_bwd_dkv_merge_kernel(const BwdParams prm)
+{
+    using namespace dkv;
+    const int hkv = prm.num_kv_heads, group = prm.num_q_heads / hkv;
+    const int unit = (int)(blockIdx.x / hkv), g = (int)(blockIdx.x % hkv);
+    const int kt = prm.order[unit];
+    const int ne = prm.ptr[kt + 1] - prm.ptr[kt];
+    if (!(ne * group > PADOC_BWD_SPLIT_STEPS && unit < prm.split_units)) return;
+    const float4 *p = reinterpret_cast<const float4 *>(prm.split + ((size_t)unit * hkv + g) * 4 * (kKT * kD));
+    constexpr int kQuads = kKT * kD / 4;                  // float4 per tensor and half
+    for (int x = threadIdx.x; x < 2 * kQuads; x += blockDim.x) {
+        const int isk = x / kQuads, r = (x % kQuads) / (kD / 4), c4 = x % (kD / 4);
+        const int64_t key = (int64_t)kt * kKT + r;
+        if (key >= prm.T) continue;
+        const float4 a = p[isk * kQuads + x % kQuads], b = p[(2 + isk) * kQuads + x % kQuads];
+        const float mul = isk ? prm.scale : 1.f;
+        uint2 w;
+        w.x = pack_bf16x2((a.x + b.x) * mul, (a.y + b.y) * mul);
+        w.y = pack_bf16x2((a.z + b.z) * mul, (a.w + b.w) * mul);
+        *reinterpret_cast<uint2 *>((isk ? prm.out0 : prm.out1) + ((size_t)key * hkv + g) * kD + 4 * c4) = w;
     }
 }
 
@@ -412,8 +483,6 @@ struct DqCfg {
     static constexpr size_t kSmemBytes = 1024 + (size_t)kStages * 2 * kTile + B_COUNT * 8 + 64 + 2 * kQT * 4;
     static_assert(kDepth >= 1 && W % 32 == 0, "step width");
 };
-
-__device__ __forceinline__ int clamp_w(int x, int w) { return min(max(x, 0), w); }
 
 template <int W>
 __global__ void __launch_bounds__(kThreads, 1)
@@ -655,8 +724,8 @@ padoc_status padoc_launch_prefill_bwd_tc(const void *q, const void *k, const voi
                                          const void *dout, const float *lse, int64_t total_tokens,
                                          int32_t num_q_heads, int32_t num_kv_heads, const int32_t *spans_dev,
                                          const padoc_tile_map_dev *q_map, const padoc_tile_map_dev *k_map, float *lt,
-                                         float *dt, int64_t t_pad, float scale, void *dq, void *dk, void *dv,
-                                         cudaStream_t stream)
+                                         float *dt, float *split, int64_t t_pad, float scale, void *dq, void *dk,
+                                         void *dv, cudaStream_t stream)
 {
     constexpr int WQ = PADOC_BWD_DQ_K_TILE;
     using CQ = DqCfg<WQ>;
@@ -664,7 +733,7 @@ padoc_status padoc_launch_prefill_bwd_tc(const void *q, const void *k, const voi
     if (!err) return PADOC_ERR_CUDA;
     const int64_t T = total_tokens;
     const int64_t nkt = (T + dkv::kKT - 1) / dkv::kKT, nqt = (T + CQ::kQT - 1) / CQ::kQT;
-    if (nkt * num_kv_heads > INT32_MAX || nqt * num_q_heads > INT32_MAX) return PADOC_ERR_UNSUPPORTED;
+    if (2 * nkt * num_kv_heads > INT32_MAX || nqt * num_q_heads > INT32_MAX) return PADOC_ERR_UNSUPPORTED;
     const uint64_t qcols = (uint64_t)num_q_heads * kD, kcols = (uint64_t)num_kv_heads * kD;
     CUtensorMap q64, g64, k128, v128, kmap, vmap;
     if (!padoc_make_tmap_bf16(&q64, q, qcols, T, qcols * 2, 64, dkv::kQT) ||
@@ -687,6 +756,11 @@ padoc_status padoc_launch_prefill_bwd_tc(const void *q, const void *k, const voi
     prm.err = err;
     prm.o = nullptr;
     prm.lse = nullptr;
+    prm.split = split;
+    // the units that may split: their partials (2 halves x 2 tensors x 64 KB per KV head) fit in the
+    // workspace's PADOC_BWD_SPLIT_BYTES_PER_TOKEN bytes per token of t_pad
+    prm.split_units = (int32_t)std::min<int64_t>(nkt, t_pad * PADOC_BWD_SPLIT_BYTES_PER_TOKEN /
+                                                          ((int64_t)num_kv_heads * 4 * dkv::kKT * kD * 4));
 
     // the dQ pass first: it also writes -lse2 and D of every row for the dK/dV pass
     BwdParams pq = prm;   // dQ pass over the query-major map; Q and dO go to tensor memory
@@ -717,7 +791,10 @@ padoc_status padoc_launch_prefill_bwd_tc(const void *q, const void *k, const voi
     pk.out1 = (__nv_bfloat16 *)dv;
     PADOC_CUDA_TRY(cudaFuncSetAttribute(prefill_bwd_dkv_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                         (int)dkv::kSmemBytes));
-    prefill_bwd_dkv_kernel<<<(unsigned)(nkt * num_kv_heads), kThreads, dkv::kSmemBytes, stream>>>(q64, g64, k128, v128, pk);
-
+    prefill_bwd_dkv_kernel<<<(unsigned)(2 * nkt * num_kv_heads), kThreads, dkv::kSmemBytes, stream>>>(q64, g64, k128,
+                                                                                                       v128, pk);
+    st = padoc_launch_status();
+    if (st != PADOC_OK || pk.split_units == 0) return st;
+    prefill_bwd_dkv_merge_kernel<<<(unsigned)(pk.split_units * num_kv_heads), 256, 0, stream>>>(pk);
     return padoc_launch_status();
 }

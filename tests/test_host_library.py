@@ -115,8 +115,9 @@ def test_prefill_bwd_tile_shapes_and_workspace():
     with pytest.raises(pa.PadocError):
         pa.padoc_prefill_bwd_tile_shapes(pa.PADOC_DTYPE_BF16, 64)
     # lse2 and D per head, rows padded to 128
-    assert pa.padoc_prefill_bwd_workspace_size(1, 16) == 2 * 16 * 128 * 4
-    assert pa.padoc_prefill_bwd_workspace_size(32768, 16) == 2 * 16 * 32768 * 4
+    # -lse2 and D per head and padded row, then 2 KB per padded row for the split dK/dV partials
+    assert pa.padoc_prefill_bwd_workspace_size(1, 16) == 2 * 16 * 128 * 4 + 128 * 2048
+    assert pa.padoc_prefill_bwd_workspace_size(32768, 16) == 2 * 16 * 32768 * 4 + 32768 * 2048
     assert pa.padoc_prefill_bwd_workspace_size(0, 4) == 0
 
 
