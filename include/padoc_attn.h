@@ -49,8 +49,9 @@ extern "C" {
 /* 1: descriptors, decode, prefill, combine, prefill backward, no-alloc decode. 2 adds the
  * stream-list and chunked-prefill planners, Algorithm 1's loop (padoc_mpd_*) and the append call.
  * 3 adds the FP8 (E4M3) KV cache (padoc_kv_pool_e4m3 and its quantize, append and decode calls),
- * the bounded-wait self-test, the in-place plan advance and the one-call decode step. */
-#define PADOC_ATTN_VERSION 3
+ * the bounded-wait self-test, the in-place plan advance and the one-call decode step. 4 adds the
+ * merge key list to the decode plan (padoc_decode_plan.off_merge_keys, num_merge_keys). */
+#define PADOC_ATTN_VERSION 4
 
 /* A CUDA stream handle; identical to cudaStream_t. */
 typedef struct CUstream_st *padoc_stream_t;
@@ -210,6 +211,9 @@ typedef struct {
     int64_t off_cta_ptr;
     int64_t off_warp_ptr;
     int64_t kv_tokens;         /* algorithmic KV tokens read: each page's stream once + all private */
+    int64_t off_merge_keys;    /* the (stream, KV head) keys the split-K merge joins; the others have */
+    int32_t num_merge_keys;    /* one partial, written as the output directly */
+    int32_t reserved;
 } padoc_decode_plan;
 
 /* Size in int32 words of the plan blob for these pages and config. */

@@ -371,8 +371,8 @@ padoc_status padoc_launch_decode_tc(const CUtensorMap *kmap, const CUtensorMap *
                                     const padoc_decode_plan *info, const int32_t *page_table, int32_t page_stride,
                                     const int32_t *stream_table, int32_t stream_stride, int32_t num_blocks,
                                     const float *k_scales, const float *v_scales, float *part_o, float *part_lse,
-                                    float scale_log2, int *err, const padoc_warp::DecodeParams *wprm,
-                                    cudaStream_t stream);
+                                    __nv_bfloat16 *out, float *lse, float scale_log2, int *err,
+                                    const padoc_warp::DecodeParams *wprm, cudaStream_t stream);
 // tcgen05 prefill backward (prefill_bwd_tc.cu): the dQ pass, which also writes lt / dt (per head
 // [Hq][t_pad]: -lse2 and rowsum(dO * O)), then the dK/dV pass; arguments validated by the caller.
 padoc_status padoc_launch_prefill_bwd_tc(const void *q, const void *k, const void *v, const void *out,

@@ -61,7 +61,12 @@ struct UniformSlots {  // public combine: part_row = split * rows + row
 // the 128 dims of one head. One pass over the slots with an online reference (the running max of lse_s): four
 // partials' LSE and O loads are in flight per thread at a time. Registers are capped so that nine CTAs
 // fit on an SM: the serving batch's 1344 (stream, KV head) pairs then start in one wave.
+// kIndexed: CTA b joins key merge_keys[b] (a plan whose sole items write some keys directly);
+// otherwise every key is merged and CTA b joins key b (no index kept live: nine CTAs per SM need the
+// 56-register cap).
+template <bool kIndexed>
 __global__ void __launch_bounds__(128, 9) decode_combine_kernel(const int32_t *__restrict__ slot_ptr,
+                                                             const int32_t *__restrict__ merge_keys,
                                                              const float *__restrict__ part_o,
                                                              const float *__restrict__ part_lse,
                                                              __nv_bfloat16 *__restrict__ out, float *__restrict__ lse_out)
@@ -69,7 +74,7 @@ __global__ void __launch_bounds__(128, 9) decode_combine_kernel(const int32_t *_
     // The slot range comes from the plan, which no kernel of the step writes, so it is read before
     // the wait. Launched programmatically after the decode grid: wait for it (and its partials),
     // then let the next step's first kernel launch (it waits for this grid before touching memory).
-    const int key = blockIdx.x;                      // s * Hkv + g; output rows key * 8 + h
+    const int key = kIndexed ? merge_keys[blockIdx.x] : (int)blockIdx.x;   // s * Hkv + g; output rows key * 8 + h
     const int p0 = slot_ptr[key], n = slot_ptr[key + 1] - p0;
     pdl_wait_prerequisite();
     pdl_launch_dependents();
@@ -303,7 +308,7 @@ padoc_status decode_split_k(const DecodePool &pl, const padoc_decode_plan *info,
     padoc_status st = padoc_launch_decode_tc(&kmap, &vmap, &qmap, plan, info, page_block_table, page_table_stride,
                                              stream_block_table, stream_table_stride, pl.num_blocks,
                                              pl.e4m3 ? pl.k_scales : nullptr, pl.e4m3 ? pl.v_scales : nullptr,
-                                             part_o, part_lse, sl2, err, &prm, cs);
+                                             part_o, part_lse, (__nv_bfloat16 *)out, lse, sl2, err, &prm, cs);
     if (st != PADOC_OK) return st;
     if (pl.e4m3 && prm.num_warps > 0) {   // E4M3: the warp lists in a grid of their own
         const int after_tc = info->num_tc_items > 0 ? 1 : 0;
@@ -323,9 +328,9 @@ padoc_status decode_split_k(const DecodePool &pl, const padoc_decode_plan *info,
         st = padoc_launch_status();
         if (st != PADOC_OK) return st;
     }
-    {
+    if (info->num_merge_keys > 0) {   // the keys with more than one partial (or a warp item's one)
         cudaLaunchConfig_t lc = {};
-        lc.gridDim = dim3((unsigned)((int64_t)info->num_streams * cfg.num_kv_heads));
+        lc.gridDim = dim3((unsigned)info->num_merge_keys);
         lc.blockDim = dim3(128);
         lc.stream = cs;
         cudaLaunchAttribute attr[1];
@@ -333,8 +338,10 @@ padoc_status decode_split_k(const DecodePool &pl, const padoc_decode_plan *info,
         attr[0].val.programmaticStreamSerializationAllowed = 1;
         lc.attrs = attr;
         lc.numAttrs = 1;
-        PADOC_CUDA_TRY(cudaLaunchKernelEx(&lc, decode_combine_kernel, prm.slot_ptr, (const float *)part_o,
-                                          (const float *)part_lse, (__nv_bfloat16 *)out, lse));
+        const bool all_keys = (int64_t)info->num_merge_keys == (int64_t)info->num_streams * cfg.num_kv_heads;
+        PADOC_CUDA_TRY(cudaLaunchKernelEx(&lc, all_keys ? decode_combine_kernel<false> : decode_combine_kernel<true>,
+                                          prm.slot_ptr, (const int32_t *)(plan + info->off_merge_keys),
+                                          (const float *)part_o, (const float *)part_lse, (__nv_bfloat16 *)out, lse));
     }
     return padoc_launch_status();
 }

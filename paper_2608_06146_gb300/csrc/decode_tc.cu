@@ -102,6 +102,9 @@ struct TcDecodeParams {
     int32_t pool_rows;           // num_blocks * num_kv_heads * 16: first out-of-range row
     const float *k_scales, *v_scales;   // E4M3 pool: [num_blocks][num_kv_heads]
     float *part_o, *part_lse;
+    __nv_bfloat16 *out;          // [S][Hq][128]: written directly by PADOC_ITEM_SOLE items
+    float *lse;                  // [S][Hq]
+    int32_t num_q_heads;
     float scale_log2;
     int *err;
     // the fused grid (plan_internal.h): CTAs [0, tc_ctas) run pieces, then warp CTA early_ctas + c;
@@ -196,8 +199,9 @@ __device__ __forceinline__ void prefetch_warp_lists(const padoc_warp::DecodePara
 }
 
 // The pieces of tensor-core CTA blockIdx.x (every thread of the CTA; smem 1024-byte aligned).
-// kFused: the CTA runs warp lists next (their first blocks are pulled into L2 meanwhile).
-template <bool kE4M3, bool kFused>
+// kFused: the CTA runs warp lists next (their first blocks are pulled into L2 meanwhile). kSole:
+// the plan has PADOC_ITEM_SOLE items (otherwise their output path is compiled out).
+template <bool kE4M3, bool kFused, bool kSole>
 __device__ __forceinline__ void decode_tc_role(const CUtensorMap &kmap, const CUtensorMap &vmap, const CUtensorMap &qmap,
                                                const TcDecodeParams &prm, const padoc_warp::DecodeParams &wprm,
                                                uint8_t *smem)
@@ -538,7 +542,7 @@ __device__ __forceinline__ void decode_tc_role(const CUtensorMap &kmap, const CU
         // columns before their cutoff.
         const int b0 = row / kGroup, b1 = 16 + row / kGroup;
         int n_tb = 0, n_te = 0, n_nstr = 0, n_first = 0, n_kvh = 0, n_slot = 0, n_cut0 = 0, n_cut1 = 0;
-        bool n_priv = false, n_cont = false;
+        bool n_priv = false, n_cont = false, n_sole = false;
         auto fetch_item = [&](int uu) {
             const padoc_item *p = prm.items + uu;
             n_tb = p->tok_begin;
@@ -549,6 +553,7 @@ __device__ __forceinline__ void decode_tc_role(const CUtensorMap &kmap, const CU
             n_slot = p->slot;
             n_priv = PADOC_ITEM_KIND(p->kind) == PADOC_ITEM_PRIVATE_TC;
             n_cont = (p->kind & PADOC_ITEM_CONT) != 0;
+            n_sole = (p->kind & PADOC_ITEM_SOLE) != 0;
         };
         // a row's cutoff: its stream's shared length, or for a chunk's private rows its private length
         auto fetch_cut = [&]() {
@@ -565,7 +570,7 @@ __device__ __forceinline__ void decode_tc_role(const CUtensorMap &kmap, const CU
         for (int u = u0; u < u1; ++u) {
             const int tb = n_tb, te = n_te, nstr = n_nstr, first = n_first, kvh = n_kvh, slot = n_slot;
             const int cut0 = n_cut0, cut1 = n_cut1;
-            const bool cont_out = n_cont;
+            const bool cont_out = n_cont, sole = kSole && n_sole;
             const int ne = te > tb ? (te - tb + kKT - 1) / kKT : 0, mt = nstr > 16 ? 2 : 1;
             if (u + 1 < u1) fetch_item(u + 1);
             // first partial slot of each row's (stream, KV head), read during the piece's last tile
@@ -741,8 +746,10 @@ __device__ __forceinline__ void decode_tc_role(const CUtensorMap &kmap, const CU
                 const float inv = empty ? 0.f : 1.f / l;
                 const size_t prow = (size_t)(mi ? pb1 : pb0) * kGroup + hl;
                 // slot layout [16 chunks of 8 dims][8 heads][8]: the 8 rows (heads) of a stream write
-                // one contiguous 256-byte run per chunk
+                // one contiguous 256-byte run per chunk; a sole item writes the row's output itself
                 float *sb = prm.part_o + (size_t)(mi ? pb1 : pb0) * (kGroup * kD) + hl * 8;
+                const size_t orow = ((size_t)(first + (valid ? b : 0)) * prm.num_q_heads + kvh * kGroup + hl);
+                __nv_bfloat16 *ob = prm.out + orow * kD + 64 * hc;
                 const uint32_t tO = tmem + lanes + 256 + 128 * mi + 64 * hc;
 #pragma unroll
                 for (int q = 0; q < 2; ++q) {
@@ -755,12 +762,24 @@ __device__ __forceinline__ void decode_tc_role(const CUtensorMap &kmap, const CU
 #pragma unroll
                         for (int i = 0; i < 32; i += 8) {
                             auto v = [&](int k) { return empty ? 0.f : __uint_as_float(o[i + k]) * inv; };
-                            const int chunk = 8 * hc + 4 * q + i / 8;
-                            st_global_v8(sb + chunk * (kGroup * 8), v(0), v(1), v(2), v(3), v(4), v(5), v(6), v(7));
+                            if (sole) {
+                                uint4 w;
+                                w.x = pack_bf16x2(v(0), v(1));
+                                w.y = pack_bf16x2(v(2), v(3));
+                                w.z = pack_bf16x2(v(4), v(5));
+                                w.w = pack_bf16x2(v(6), v(7));
+                                *reinterpret_cast<uint4 *>(ob + 32 * q + i) = w;
+                            } else {
+                                const int chunk = 8 * hc + 4 * q + i / 8;
+                                st_global_v8(sb + chunk * (kGroup * 8), v(0), v(1), v(2), v(3), v(4), v(5), v(6), v(7));
+                            }
                         }
                     }
                 }
-                if (valid && hc == 0) prm.part_lse[prow] = empty ? -INFINITY : (m_ref * cm + log2f(l)) * PADOC_LN2;
+                if (valid && hc == 0) {
+                    const float lv = empty ? -INFINITY : (m_ref * cm + log2f(l)) * PADOC_LN2;
+                    if (sole) prm.lse[orow] = lv; else prm.part_lse[prow] = lv;
+                }
             }
         }
     }
@@ -786,7 +805,7 @@ static_assert(padoc_warp::kWarps * 32 == 256, "the warp path runs on warpgroups 
 // registers back and end. A plan without tensor-core work runs warp CTAs only. Without kFused the
 // grid runs the tensor-core pieces only (the E4M3 pool, whose warp lists run in a grid of their own:
 // there the warp path needs more registers than the split leaves it).
-template <bool kE4M3, bool kFused>
+template <bool kE4M3, bool kFused, bool kSole>
 __global__ void __launch_bounds__(kThreads, 1)
 decode_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap,
                  const __grid_constant__ CUtensorMap qmap, const TcDecodeParams prm,
@@ -799,11 +818,11 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
     }
     const bool has_tc = (int)blockIdx.x < prm.tc_ctas;
     if constexpr (!kFused) {
-        if (has_tc) decode_tc_role<kE4M3, false>(kmap, vmap, qmap, prm, wprm, smem);
+        if (has_tc) decode_tc_role<kE4M3, false, kSole>(kmap, vmap, qmap, prm, wprm, smem);
         return;
     }
     if (has_tc) {
-        decode_tc_role<kE4M3, true>(kmap, vmap, qmap, prm, wprm, smem);
+        decode_tc_role<kE4M3, true, kSole>(kmap, vmap, qmap, prm, wprm, smem);
     } else {
         // a CTA with warp lists only: the same wait for the previous kernel in the stream
         pdl_wait_prerequisite();
@@ -830,8 +849,8 @@ padoc_status padoc_launch_decode_tc(const CUtensorMap *kmap, const CUtensorMap *
                                     const padoc_decode_plan *info, const int32_t *page_table, int32_t page_stride,
                                     const int32_t *stream_table, int32_t stream_stride, int32_t num_blocks,
                                     const float *k_scales, const float *v_scales, float *part_o, float *part_lse,
-                                    float scale_log2, int *err, const padoc_warp::DecodeParams *wprm,
-                                    cudaStream_t stream)
+                                    __nv_bfloat16 *out, float *lse, float scale_log2, int *err,
+                                    const padoc_warp::DecodeParams *wprm, cudaStream_t stream)
 {
     const bool e4m3 = k_scales != nullptr;   // an E4M3 pool: the maps hold codes
     const bool fused = !e4m3;
@@ -856,12 +875,18 @@ padoc_status padoc_launch_decode_tc(const CUtensorMap *kmap, const CUtensorMap *
     prm.v_scales = v_scales;
     prm.part_o = part_o;
     prm.part_lse = part_lse;
+    prm.out = out;
+    prm.lse = lse;
+    prm.num_q_heads = info->cfg.num_q_heads;
     prm.scale_log2 = scale_log2;
     prm.err = err;
     prm.tc_ctas = info->num_tc_items > 0 ? info->tc_ctas : 0;
     prm.warp_ctas = fused ? (wprm->num_warps + padoc_warp::kWarps - 1) / padoc_warp::kWarps : 0;
     prm.early_ctas = padoc_fused_early_ctas(prm.tc_ctas, prm.warp_ctas, padoc_default_ctas());
-    auto kern = e4m3 ? decode_tc_kernel<true, false> : decode_tc_kernel<false, true>;
+    // plans with sole items (chunked prefill) take the variant that writes their outputs
+    const bool sole = (int64_t)info->num_merge_keys < (int64_t)info->num_streams * info->cfg.num_kv_heads;
+    auto kern = e4m3 ? (sole ? decode_tc_kernel<true, false, true> : decode_tc_kernel<true, false, false>)
+                     : (sole ? decode_tc_kernel<false, true, true> : decode_tc_kernel<false, true, false>);
     PADOC_CUDA_TRY(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes));
     cudaLaunchConfig_t lc = {};
     lc.gridDim = dim3((unsigned)(prm.tc_ctas + prm.early_ctas));

@@ -575,6 +575,24 @@ padoc_status build_work(int32_t num_pages, const padoc_decode_config *cfg, PlanP
             }
     pp.slot_ptr.assign((size_t)S * Hkv + 1, 0);
     for (size_t i = 0; i < (size_t)S * Hkv; ++i) pp.slot_ptr[i + 1] = pp.slot_ptr[i] + cnt[i];
+    // A tensor-core item whose every stream has this one partial for its KV head (a chunked
+    // prefill's group whose pieces stay on one CTA) writes their outputs itself; only the other
+    // (stream, KV head) keys go to the merge.
+    {
+        std::vector<uint8_t> direct((size_t)S * Hkv, 0);
+        for (padoc_item &it : tc_items) {
+            if (it.kind & PADOC_ITEM_CONT) continue;   // the next item of the chain writes
+            bool sole = true;
+            for (int32_t b = 0; sole && b < it.num_streams; ++b)
+                sole = cnt[(size_t)(it.first_stream + b) * Hkv + it.kv_head] == 1;
+            if (!sole) continue;
+            it.kind |= PADOC_ITEM_SOLE;
+            for (int32_t b = 0; b < it.num_streams; ++b) direct[(size_t)(it.first_stream + b) * Hkv + it.kv_head] = 1;
+        }
+        pp.merge_keys.clear();
+        for (size_t i = 0; i < (size_t)S * Hkv; ++i)
+            if (!direct[i]) pp.merge_keys.push_back((int32_t)i);
+    }
 
     // The warp grid runs as one wave. Items are taken longest first (LPT; a counting sort on the
     // block count keeps ties in plan order) and each goes to the warp with the most capacity left
@@ -750,12 +768,13 @@ int32_t choose_tc_ctas(const PlanParts &pp, const padoc_decode_config *cfg, int6
 }  // namespace
 
 // int32 words of the plan blob: stream_page, shared_len, private_len [S], slot_ptr [S Hkv + 1],
-// items [num_items][8], page_len [num_pages], cta_ptr [tc_ctas + 1], warp_ptr [num_warps + 1]
+// items [num_items][8], page_len [num_pages], cta_ptr [tc_ctas + 1], warp_ptr [num_warps + 1],
+// merge_keys [num_merge_keys]
 int64_t padoc_plan_blob_ints(const PlanParts &pp, int32_t num_pages, int32_t hkv)
 {
     const int64_t S = (int64_t)pp.streams.size();
     return 3 * S + (S * hkv + 1) + (int64_t)pp.items.size() * PADOC_ITEM_INTS + num_pages + (int64_t)pp.cta_ptr.size() +
-           (int64_t)pp.warp_ptr.size();
+           (int64_t)pp.warp_ptr.size() + (int64_t)pp.merge_keys.size();
 }
 
 namespace {
@@ -822,6 +841,8 @@ padoc_status padoc_plan_write_blob(const PlanParts &pp, int32_t num_pages, const
     info->off_page_len = o; o += num_pages;
     info->off_cta_ptr = o; o += (int64_t)pp.cta_ptr.size();
     info->off_warp_ptr = o; o += (int64_t)pp.warp_ptr.size();
+    info->off_merge_keys = o; o += (int64_t)pp.merge_keys.size();
+    info->num_merge_keys = (int32_t)pp.merge_keys.size();
     for (int64_t s = 0; s < S; ++s) {
         plan[info->off_stream_page + s] = pp.streams[s].page;
         plan[info->off_shared_len + s] = pp.streams[s].shared_len;
@@ -832,6 +853,8 @@ padoc_status padoc_plan_write_blob(const PlanParts &pp, int32_t num_pages, const
     for (int32_t p = 0; p < num_pages; ++p) plan[info->off_page_len + p] = pp.page_len[p];
     if (!pp.cta_ptr.empty()) std::memcpy(plan + info->off_cta_ptr, pp.cta_ptr.data(), pp.cta_ptr.size() * sizeof(int32_t));
     std::memcpy(plan + info->off_warp_ptr, pp.warp_ptr.data(), pp.warp_ptr.size() * sizeof(int32_t));
+    if (!pp.merge_keys.empty())
+        std::memcpy(plan + info->off_merge_keys, pp.merge_keys.data(), pp.merge_keys.size() * sizeof(int32_t));
     return PADOC_OK;
 }
 

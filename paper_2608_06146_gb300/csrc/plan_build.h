@@ -17,6 +17,7 @@ struct PlanParts {
     std::vector<int32_t> slot_ptr;      // [S * Hkv + 1]: partial slots of each (stream, KV head)
     std::vector<int32_t> cta_ptr;       // [tc_ctas + 1]: tensor-core items of each CTA
     std::vector<int32_t> warp_ptr;      // [num_warps + 1]: warp items of each warp (from the first)
+    std::vector<int32_t> merge_keys;    // the (stream, KV head) keys the merge joins (the others are written directly)
     std::vector<padoc_item> items;
     int32_t num_tc_items = 0, tc_ctas = 0, num_warps = 0;
     int32_t max_page_blocks = 0, max_stream_blocks = 0;

@@ -115,6 +115,10 @@ enum { PADOC_ITEM_SHARED = 0, PADOC_ITEM_PRIVATE = 1, PADOC_ITEM_SHARED_TC = 2, 
 // piece over a group's shared tiles and then its private ones): the same streams, KV head and
 // partial slot, one running softmax over both, one partial written after the second item.
 #define PADOC_ITEM_CONT 32
+// Flag of a tensor-core item that is the only partial of each of its streams for its KV head: it
+// writes their bf16 outputs and LSE itself (exactly the merge's result for one partial), and the
+// merge skips those keys (a chunked prefill's groups whose pieces stay on one CTA).
+#define PADOC_ITEM_SOLE 64
 #define PADOC_ITEM_KIND(k) ((k) & 15)
 
 // One split-K work item of the decode kernels (8 int32 words in the plan blob). The blob holds

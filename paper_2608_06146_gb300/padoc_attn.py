@@ -79,7 +79,8 @@ class padoc_decode_plan(ctypes.Structure):
                 ("plan_ints", ctypes.c_int64), ("off_stream_page", ctypes.c_int64), ("off_shared_len", ctypes.c_int64),
                 ("off_private_len", ctypes.c_int64), ("off_slot_ptr", ctypes.c_int64), ("off_items", ctypes.c_int64),
                 ("off_page_len", ctypes.c_int64), ("off_cta_ptr", ctypes.c_int64), ("off_warp_ptr", ctypes.c_int64),
-                ("kv_tokens", ctypes.c_int64)]
+                ("kv_tokens", ctypes.c_int64), ("off_merge_keys", ctypes.c_int64), ("num_merge_keys", ctypes.c_int32),
+                ("reserved", ctypes.c_int32)]
 
 
 class padoc_mpd_step(ctypes.Structure):

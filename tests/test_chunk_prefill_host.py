@@ -65,7 +65,7 @@ def check_chunk_plan(page_len, chunks, tc_ctas, warp_ctas=0):
     items = plan[info.off_items:info.off_items + 8 * info.num_items].reshape(-1, 8)
     ntc = info.num_tc_items
     assert np.isin(items[:ntc, 0] & 15, [2, 3]).all() and np.isin(items[ntc:, 0], [0, 1]).all()
-    assert not np.any(items[:, 0] & ~(15 | 16 | 32))
+    assert not np.any(items[:, 0] & ~(15 | 16 | 32 | 64))
     first_of = {c: int(np.nonzero(ch == c)[0][0]) for c in range(len(chunks))}
     cov_sh = {(s, g): np.zeros(sh[s], np.int32) for s in range(S) for g in range(Hkv)}
     cov_pv = {(s, g): np.zeros(pl[s], np.int32) for s in range(S) for g in range(Hkv)}
@@ -112,6 +112,28 @@ def check_chunk_plan(page_len, chunks, tc_ctas, warp_ctas=0):
         assert np.all(cov_sh[key] == 1), f"shared rows of token {s} head {g}"
         assert np.all(cov_pv[key] == 1), f"private rows of token {s} head {g}"
         assert sorted(slots[key]) == list(range(slot_ptr[s * Hkv + g + 1] - slot_ptr[s * Hkv + g]))
+    check_sole_and_merge_keys(plan, info, items, Hkv)
+
+
+def check_sole_and_merge_keys(plan, info, items, Hkv):
+    # SOLE (64): a tensor-core item that writes a partial (not the first of a chain) flagged exactly
+    # when each of its streams has that one partial for its KV head; the merge joins every other key
+    S, ntc = info.num_streams, info.num_tc_items
+    slot_ptr = plan[info.off_slot_ptr:info.off_slot_ptr + S * Hkv + 1]
+    nslots = np.diff(slot_ptr)
+    cont, sole = (items[:, 0] & 32) != 0, (items[:, 0] & 64) != 0
+    assert not sole[ntc:].any() and not (sole & cont).any()
+    direct = set()
+    for i in range(ntc):
+        if cont[i]:
+            continue
+        _, _, g, _, _, fs, ns, _ = items[i]
+        keys = [s * Hkv + g for s in range(fs, fs + ns)]
+        assert bool(sole[i]) == all(nslots[k] == 1 for k in keys)
+        if sole[i]:
+            direct.update(keys)
+    mk = plan[info.off_merge_keys:info.off_merge_keys + info.num_merge_keys]
+    assert mk.tolist() == sorted(set(range(S * Hkv)) - direct)
 
 
 def test_chunk_plan_validation_and_table():

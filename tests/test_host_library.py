@@ -39,7 +39,7 @@ def test_exports_every_declared_symbol(lib):
     for name in declared:
         assert hasattr(lib, name), f"{name} not exported"
     assert set(pa.exported_symbols()) == declared
-    assert pa.padoc_version() == 3
+    assert pa.padoc_version() == 4
     assert pa.padoc_status_string(0) == "ok"
 
 
@@ -260,6 +260,9 @@ def check_decode_plan(wl, layout, tc_ctas, warp_ctas):
         assert te <= (sh[fs] if kind == 0 else pl[fs])
     need = pa.padoc_decode_workspace_size(info)
     assert need >= info.num_slots * (wl.num_q_heads // Hkv) * (wl.head_dim + 1) * 4
+    # the merge joins every (stream, KV head) key but those a sole tensor-core item writes itself
+    from tests.test_chunk_prefill_host import check_sole_and_merge_keys
+    check_sole_and_merge_keys(plan, info, items, Hkv)
 
 
 def test_decode_plan_properties():
