@@ -445,8 +445,9 @@ padoc_status build_work(int32_t num_pages, const padoc_decode_config *cfg, PlanP
     // CTA loads count every piece's own cost too (its epilogue, and the query reload before it):
     // the smallest bound T for which a greedy walk along the sequences needs at most `want` CTAs
     // is found by bisection, then the walk is made once more to emit the pieces.
-    auto piece_cost = [](const Segment &sg) -> int64_t {
-        return sg.weight == PADOC_TC_WEIGHT_2M ? PADOC_TC_PIECE_COST_2M : PADOC_TC_PIECE_COST_1M;
+    auto piece_cost = [&](const Segment &sg) -> int64_t {
+        return (sg.weight == PADOC_TC_WEIGHT_2M ? PADOC_TC_PIECE_COST_2M : PADOC_TC_PIECE_COST_1M) +
+               (chunked ? PADOC_TC_PIECE_EXTRA_CHUNK : 0);
     };
     int64_t max_piece = 0;
     int64_t total_w = 0, max_w = 0;

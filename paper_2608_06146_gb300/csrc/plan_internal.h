@@ -49,6 +49,12 @@
 // for a one-M-tile piece, a tile and a half for a two-M-tile piece
 #define PADOC_TC_PIECE_COST_1M 7
 #define PADOC_TC_PIECE_COST_2M 11
+// ... plus this for a piece of a chunked prefill (a group's shared tiles and then its private ones:
+// two items, the switch between them, and tiles that other groups read too), fitted to per-CTA
+// timelines of the serving batch's branch prefill
+#ifndef PADOC_TC_PIECE_EXTRA_CHUNK
+#define PADOC_TC_PIECE_EXTRA_CHUNK 15
+#endif
 
 // Warps per CTA of the warp kernel, and the start-up cost of one warp item in 16-token blocks
 // (query fragments, the first blocks' latency, the partial's write), used to balance warps.
