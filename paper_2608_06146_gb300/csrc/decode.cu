@@ -61,6 +61,55 @@ struct UniformSlots {  // public combine: part_row = split * rows + row
 // the 128 dims of one head. One pass over the slots with an online reference (the running max of lse_s): four
 // partials' LSE and O loads are in flight per thread at a time. Registers are capped so that nine CTAs
 // fit on an SM: the serving batch's 1344 (stream, KV head) pairs then start in one wave.
+
+// The online pass of one thread over the key's slots in blocks of four, blocks b0, b0 + stride, ...:
+// (mref, ssum, acc) hold the running reference, the weights' sum and the weighted O sums.
+struct MergeState {
+    float mref = -INFINITY, ssum = 0.f;
+    float4 acc0 = make_float4(0.f, 0.f, 0.f, 0.f), acc1 = make_float4(0.f, 0.f, 0.f, 0.f);
+};
+__device__ __forceinline__ void merge_slots(const float *bo, const float *bl, int n, int b0, int stride, MergeState &ms)
+{
+    constexpr size_t kSlotO = (size_t)kGroup * kD;
+    for (int i = 4 * b0; i < n; i += 4 * stride) {
+        float li[4];
+        float4 v0[4], v1[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const bool in = i + u < n;
+            li[u] = in ? bl[(size_t)(i + u) * kGroup] : -INFINITY;
+            v0[u] = in ? *reinterpret_cast<const float4 *>(bo + (i + u) * kSlotO) : make_float4(0.f, 0.f, 0.f, 0.f);
+            v1[u] = in ? *reinterpret_cast<const float4 *>(bo + (i + u) * kSlotO + 4) : make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            if (li[u] == -INFINITY) continue;   // an empty partial weighs nothing
+            if (li[u] > ms.mref) {
+                const float a = ms.mref == -INFINITY ? 0.f : expf(ms.mref - li[u]);
+                ms.ssum *= a;
+                ms.acc0.x *= a; ms.acc0.y *= a; ms.acc0.z *= a; ms.acc0.w *= a;
+                ms.acc1.x *= a; ms.acc1.y *= a; ms.acc1.z *= a; ms.acc1.w *= a;
+                ms.mref = li[u];
+            }
+            const float w = expf(li[u] - ms.mref);
+            ms.ssum += w;
+            ms.acc0.x += w * v0[u].x; ms.acc0.y += w * v0[u].y; ms.acc0.z += w * v0[u].z; ms.acc0.w += w * v0[u].w;
+            ms.acc1.x += w * v1[u].x; ms.acc1.y += w * v1[u].y; ms.acc1.z += w * v1[u].z; ms.acc1.w += w * v1[u].w;
+        }
+    }
+}
+
+__device__ __forceinline__ void merge_store(const MergeState &ms, int key, int h, int part, __nv_bfloat16 *out,
+                                            float *lse_out)
+{
+    const float inv = ms.ssum > 0.f ? 1.f / ms.ssum : 0.f;
+    uint4 pk;
+    pk.x = pack_bf16x2(ms.acc0.x * inv, ms.acc0.y * inv); pk.y = pack_bf16x2(ms.acc0.z * inv, ms.acc0.w * inv);
+    pk.z = pack_bf16x2(ms.acc1.x * inv, ms.acc1.y * inv); pk.w = pack_bf16x2(ms.acc1.z * inv, ms.acc1.w * inv);
+    *reinterpret_cast<uint4 *>(out + ((size_t)key * kGroup + h) * kD + part * 8) = pk;
+    if (part == 0) lse_out[(size_t)key * kGroup + h] = ms.ssum > 0.f ? ms.mref + logf(ms.ssum) : -INFINITY;
+}
+
 // kIndexed: CTA b joins key merge_keys[b] (a plan whose sole items write some keys directly);
 // otherwise every key is merged and CTA b joins key b (no index kept live: nine CTAs per SM need the
 // 56-register cap).
@@ -82,41 +131,49 @@ __global__ void __launch_bounds__(128, 9) decode_combine_kernel(const int32_t *_
     const int h = tid & 7, part = tid >> 3;          // head, 8-dim chunk: a warp reads 4 chunks x 8 heads, contiguous
     const float *bo = part_o + (size_t)p0 * kGroup * kD + (part * kGroup + h) * 8;   // chunk `part` of head h
     const float *bl = part_lse + (size_t)p0 * kGroup + h;
-    constexpr size_t kSlotO = (size_t)kGroup * kD;
-    float mref = -INFINITY, ssum = 0.f;
-    float4 acc0 = make_float4(0.f, 0.f, 0.f, 0.f), acc1 = acc0;
-    for (int i = 0; i < n; i += 4) {
-        float li[4];
-        float4 v0[4], v1[4];
+    MergeState ms;
+    merge_slots(bo, bl, n, 0, 1, ms);
+    merge_store(ms, key, h, part, out, lse_out);
+}
+
+// The merge for steps with few keys and many partials each (a decoding loop's small steps): four
+// groups of 128 threads share a key, group q taking the blocks of four slots q, q + 4, ..., and
+// group 0 joins the four running states through shared memory. Launched instead of
+// decode_combine_kernel when the keys fit in one wave of these CTAs.
+constexpr int kWideGroups = 4;
+template <bool kIndexed>
+__global__ void __launch_bounds__(128 * kWideGroups, 2) decode_combine_wide_kernel(
+    const int32_t *__restrict__ slot_ptr, const int32_t *__restrict__ merge_keys, const float *__restrict__ part_o,
+    const float *__restrict__ part_lse, __nv_bfloat16 *__restrict__ out, float *__restrict__ lse_out)
+{
+    const int key = kIndexed ? merge_keys[blockIdx.x] : (int)blockIdx.x;
+    const int p0 = slot_ptr[key], n = slot_ptr[key + 1] - p0;
+    pdl_wait_prerequisite();
+    pdl_launch_dependents();
+    const int tid = threadIdx.x & 127, q = threadIdx.x >> 7;
+    const int h = tid & 7, part = tid >> 3;
+    const float *bo = part_o + (size_t)p0 * kGroup * kD + (part * kGroup + h) * 8;
+    const float *bl = part_lse + (size_t)p0 * kGroup + h;
+    MergeState ms;
+    merge_slots(bo, bl, n, q, kWideGroups, ms);
+    __shared__ MergeState st[kWideGroups - 1][128];
+    if (q > 0) st[q - 1][tid] = ms;
+    __syncthreads();
+    if (q > 0) return;
 #pragma unroll
-        for (int u = 0; u < 4; ++u) {
-            const bool in = i + u < n;
-            li[u] = in ? bl[(size_t)(i + u) * kGroup] : -INFINITY;
-            v0[u] = in ? *reinterpret_cast<const float4 *>(bo + (i + u) * kSlotO) : make_float4(0.f, 0.f, 0.f, 0.f);
-            v1[u] = in ? *reinterpret_cast<const float4 *>(bo + (i + u) * kSlotO + 4) : make_float4(0.f, 0.f, 0.f, 0.f);
-        }
-#pragma unroll
-        for (int u = 0; u < 4; ++u) {
-            if (li[u] == -INFINITY) continue;   // an empty partial weighs nothing
-            if (li[u] > mref) {
-                const float a = mref == -INFINITY ? 0.f : expf(mref - li[u]);
-                ssum *= a;
-                acc0.x *= a; acc0.y *= a; acc0.z *= a; acc0.w *= a;
-                acc1.x *= a; acc1.y *= a; acc1.z *= a; acc1.w *= a;
-                mref = li[u];
-            }
-            const float w = expf(li[u] - mref);
-            ssum += w;
-            acc0.x += w * v0[u].x; acc0.y += w * v0[u].y; acc0.z += w * v0[u].z; acc0.w += w * v0[u].w;
-            acc1.x += w * v1[u].x; acc1.y += w * v1[u].y; acc1.z += w * v1[u].z; acc1.w += w * v1[u].w;
-        }
+    for (int k = 0; k < kWideGroups - 1; ++k) {
+        const MergeState o = st[k][tid];
+        if (o.mref == -INFINITY) continue;   // that group saw no partial with weight
+        const float m = fmaxf(ms.mref, o.mref);
+        const float a = ms.mref == -INFINITY ? 0.f : expf(ms.mref - m), b = expf(o.mref - m);
+        ms.ssum = ms.ssum * a + o.ssum * b;
+        ms.acc0.x = ms.acc0.x * a + o.acc0.x * b; ms.acc0.y = ms.acc0.y * a + o.acc0.y * b;
+        ms.acc0.z = ms.acc0.z * a + o.acc0.z * b; ms.acc0.w = ms.acc0.w * a + o.acc0.w * b;
+        ms.acc1.x = ms.acc1.x * a + o.acc1.x * b; ms.acc1.y = ms.acc1.y * a + o.acc1.y * b;
+        ms.acc1.z = ms.acc1.z * a + o.acc1.z * b; ms.acc1.w = ms.acc1.w * a + o.acc1.w * b;
+        ms.mref = m;
     }
-    const float inv = ssum > 0.f ? 1.f / ssum : 0.f;
-    uint4 pk;
-    pk.x = pack_bf16x2(acc0.x * inv, acc0.y * inv); pk.y = pack_bf16x2(acc0.z * inv, acc0.w * inv);
-    pk.z = pack_bf16x2(acc1.x * inv, acc1.y * inv); pk.w = pack_bf16x2(acc1.z * inv, acc1.w * inv);
-    *reinterpret_cast<uint4 *>(out + ((size_t)key * kGroup + h) * kD + part * 8) = pk;
-    if (part == 0) lse_out[(size_t)key * kGroup + h] = ssum > 0.f ? mref + logf(ssum) : -INFINITY;
+    merge_store(ms, key, h, part, out, lse_out);
 }
 
 template <class Slots, class OutT>
@@ -339,8 +396,12 @@ padoc_status decode_split_k(const DecodePool &pl, const padoc_decode_plan *info,
         lc.attrs = attr;
         lc.numAttrs = 1;
         const bool all_keys = (int64_t)info->num_merge_keys == (int64_t)info->num_streams * cfg.num_kv_heads;
-        PADOC_CUDA_TRY(cudaLaunchKernelEx(&lc, all_keys ? decode_combine_kernel<false> : decode_combine_kernel<true>,
-                                          prm.slot_ptr, (const int32_t *)(plan + info->off_merge_keys),
+        // few keys with many partials each: four thread groups per key, in one wave (two CTAs per SM)
+        const bool wide = info->max_stream_slots > 8 && info->num_merge_keys <= 2 * padoc_default_ctas();
+        if (wide) lc.blockDim = dim3(128 * kWideGroups);
+        auto kern = wide ? (all_keys ? decode_combine_wide_kernel<false> : decode_combine_wide_kernel<true>)
+                         : (all_keys ? decode_combine_kernel<false> : decode_combine_kernel<true>);
+        PADOC_CUDA_TRY(cudaLaunchKernelEx(&lc, kern, prm.slot_ptr, (const int32_t *)(plan + info->off_merge_keys),
                                           (const float *)part_o, (const float *)part_lse, (__nv_bfloat16 *)out, lse));
     }
     return padoc_launch_status();
