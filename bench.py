@@ -560,9 +560,10 @@ def bench_chunk_prefill(args, torch, dev, rank, world):
 def bench_loop(args, torch, dev, rank, world):
     """Algorithm 1 over the serving batch's 32 pages: every page is admitted (its prefix K/V appended
     into the pool, untimed), then the loop runs every layout stream and branch from its first input
-    to its EOS. Timed twice: (a) end to end through the engine, as a caller runs it (host scheduler
-    and planner in one library call, one host->device copy and the append + decode launches per
-    step, the step's events handed to the scheduler); the synthetic token source stands in for the
+    to its EOS. Timed twice: (a) end to end through the engine, as a caller runs it (per step one
+    library call, padoc_mpd_runner_step: the host scheduler and planner, one host->device copy and
+    the append + decode launches; then the step's events handed to the scheduler, padoc_mpd_end_step;
+    the inputs' source rows in a table by stream id); the synthetic token source stands in for the
     decoder's sampled outputs, and its events depend only on the pages and the scheduler's stream
     order, so they are drawn once, before the timed region (a warm-up pass records each step's
     stream ids, source rows, forks and EOS flags; the timed pass replays them and checks that the
@@ -617,16 +618,18 @@ def bench_loop(args, torch, dev, rank, world):
     def run_replay(traj):
         _, loop = admit_all()
         cmax = max(len(t[0]) for t in traj)
+        n_ids = max(int(t[0].max()) for t in traj if len(t[0])) + 1
         outs_ = [torch.empty((cmax, Hq, d), dtype=wl.dtype, device=dev) for _ in range(2)]
         lses_ = [torch.empty((cmax, Hq), dtype=torch.float32, device=dev) for _ in range(2)]
+        row_of = np.zeros(n_ids, np.int32)   # each live stream's source row, by stream id
         torch.cuda.synchronize()
         toks = h2d = 0
         same = True
         t0 = time.perf_counter()
         for i, (ids_r, rows_r, nf_r, eos_r) in enumerate(traj):
-            C = len(ids_r)
-            ids, out, lse = loop.step(kd, vd, qd, lambda x: rows_r, scale, out=outs_[i & 1][:C], lse=lses_[i & 1][:C])
-            same = same and np.array_equal(ids, ids_r)
+            row_of[ids_r] = rows_r
+            C, ids = loop.run_step(kd, vd, qd, row_of, scale, outs_[i & 1], lses_[i & 1])
+            same = same and C == len(ids_r) and np.array_equal(ids, ids_r)
             toks += C
             h2d += loop.h2d_bytes
             loop.end_step(nf_r, eos_r)

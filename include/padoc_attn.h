@@ -22,8 +22,10 @@
  * Conventions for every call
  *   - Ownership: the caller owns every buffer. The library never allocates device memory, never
  *     keeps a pointer after a call returns and never synchronizes, except
- *     padoc_check_device_errors. The one object it allocates is the decoding loop's host-side
- *     scheduler state (padoc_mpd_create / padoc_mpd_destroy).
+ *     padoc_check_device_errors. The objects it allocates are the decoding loop's host-side
+ *     scheduler state (padoc_mpd_create / padoc_mpd_destroy) and the loop's step runner
+ *     (padoc_mpd_runner_*), which owns its staging and device buffers, keeps the scheduler and pool
+ *     it was made for, and waits for its own events.
  *   - Host pointers are marked (host); device pointers (device). Device calls are asynchronous on
  *     the given stream (a cudaStream_t; NULL is the legacy default stream).
  *   - Every argument is validated on the host before any launch; a failed check returns
@@ -50,8 +52,9 @@ extern "C" {
  * stream-list and chunked-prefill planners, Algorithm 1's loop (padoc_mpd_*) and the append call.
  * 3 adds the FP8 (E4M3) KV cache (padoc_kv_pool_e4m3 and its quantize, append and decode calls),
  * the bounded-wait self-test, the in-place plan advance and the one-call decode step. 4 adds the
- * merge key list to the decode plan (padoc_decode_plan.off_merge_keys, num_merge_keys). */
-#define PADOC_ATTN_VERSION 4
+ * merge key list to the decode plan (padoc_decode_plan.off_merge_keys, num_merge_keys). 5 adds the
+ * loop's step runner (padoc_mpd_runner_*). */
+#define PADOC_ATTN_VERSION 5
 
 /* A CUDA stream handle; identical to cudaStream_t. */
 typedef struct CUstream_st *padoc_stream_t;
@@ -463,8 +466,7 @@ padoc_status padoc_expand_chunk_table(const padoc_prefill_chunk *chunks, int32_t
  * ========================================================================================== */
 
 /* Host-side scheduler state of the loop for a batch of pages sharing one KV pool (opaque; created by
- * padoc_mpd_create, freed by padoc_mpd_destroy: the one object this library allocates, in host
- * memory). It keeps, per page, the shared stream's blocks (prefix X, then the layout stream's
+ * padoc_mpd_create, freed by padoc_mpd_destroy, in host memory). It keeps, per page, the shared stream's blocks (prefix X, then the layout stream's
  * tokens) and, per stream, its cutoff on the shared stream and its private blocks, and it hands out
  * and takes back pool blocks. It realises the logical mask M of App. E.1 without materialising it:
  *   - each step appends one input per live stream (M <- [M I_C]): the layout stream's input extends
@@ -576,6 +578,56 @@ padoc_status padoc_mpd_launch_step(const padoc_mpd_step *step, const int32_t *st
                                    const void *v_src, const void *q_src, int64_t src_total, void *q_dst, float scale,
                                    void *out, float *lse, void *workspace, size_t workspace_bytes,
                                    padoc_stream_t stream);
+
+/* The loop's per-step host work behind one call (Algorithm 1, App. E.1: "decode all live streams"
+ * once per iteration): a runner keeps, for one scheduler and one pool, two pinned staging buffers
+ * used in turn (a step's buffer is reused two steps later, after the event recorded behind that
+ * step's launches has completed), the device copy of the step's ints, the step's query buffer and
+ * the decode workspace. It allocates them (cudaHostAlloc / cudaMalloc) as the steps need and frees
+ * them in padoc_mpd_runner_destroy; to replace a device buffer it first waits for the step's
+ * stream. The scheduler and the pool must outlive the runner; cfg->layout_streams must be 0.
+ * Errors: INVALID_ARGUMENT (mismatched block size, KV heads or head_dim, a pool with fewer blocks
+ * than the scheduler), CUDA. */
+typedef struct padoc_mpd_runner padoc_mpd_runner;
+padoc_status padoc_mpd_runner_create(padoc_mpd *mpd, const padoc_decode_config *cfg, const padoc_kv_pool *pool,
+                                     padoc_mpd_runner **runner);
+void padoc_mpd_runner_destroy(padoc_mpd_runner *runner);
+
+/* Arguments of padoc_mpd_runner_step, kept by the caller from step to step. */
+typedef struct {
+    const void *k_src;                  /* (device) [src_total][Hkv][d]: the inputs' K rows, pool dtype */
+    const void *v_src;                  /* (device) [src_total][Hkv][d] */
+    const void *q_src;                  /* (device) [src_total][Hq][d] */
+    int64_t src_total;
+    const int32_t *src_row_of_stream;   /* (host) int32 [num_stream_ids]: the source row of each live
+                                           stream's next input, indexed by stream id */
+    int32_t num_stream_ids;             /* at least the number of stream ids created so far */
+    float scale;                        /* softmax scale */
+    void *out;                          /* (device) [out_rows][Hq][d], pool dtype: rows [0, C) receive the
+                                           step's outputs in step order */
+    float *lse;                         /* (device) fp32 [out_rows][Hq] */
+    int32_t out_rows;
+    int32_t ids_capacity;
+    int32_t *stream_ids;                /* (host) int32 [ids_capacity]: receives the step's stream ids */
+    padoc_stream_t stream;              /* every copy and launch of the step goes here */
+} padoc_mpd_run_args;
+
+/* One step: padoc_mpd_prepare_step into the runner's next staging buffer, the source row of each
+ * stream's input from a->src_row_of_stream, then padoc_mpd_launch_step with the runner's buffers,
+ * and an event behind it; no host synchronization except the wait for the staging buffer's copy of
+ * two steps ago (and, when a buffer grows, for the stream). num_streams: C (0: nothing launched);
+ * upload_bytes (NULL allowed): the bytes copied to the device for the step.
+ * The step stays begun until padoc_mpd_end_step. Errors: CAPACITY when out_rows or ids_capacity is
+ * below the live streams, or the pool lacks free blocks (nothing begins); INVALID_ARGUMENT (also a
+ * step already begun, num_stream_ids too small; nothing begins); past the planning (CUDA,
+ * UNSUPPORTED) the step has begun and the caller ends it. Source rows out of range set the device
+ * error word (padoc_append_inputs). */
+padoc_status padoc_mpd_runner_step(padoc_mpd_runner *runner, const padoc_mpd_run_args *args, int32_t *num_streams,
+                                   int64_t *upload_bytes);
+
+/* The last step the runner prepared and its staging buffer (valid until the runner's step after
+ * next): for callers that keep a record of the steps. Errors: INVALID_ARGUMENT (no step yet). */
+padoc_status padoc_mpd_runner_last_step(const padoc_mpd_runner *runner, padoc_mpd_step *step, const int32_t **stage);
 
 /* Live pages, live streams and free pool blocks. */
 padoc_status padoc_mpd_status(const padoc_mpd *mpd, int32_t *live_pages, int32_t *live_streams, int32_t *free_blocks);

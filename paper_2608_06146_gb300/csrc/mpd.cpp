@@ -390,3 +390,170 @@ extern "C" padoc_status padoc_mpd_launch_step(const padoc_mpd_step *step, const 
                                     step->page_stride, dev_ints + step->off_stream_table, step->stream_stride, q_dst,
                                     scale, out, lse, workspace, workspace_bytes, stream);
 }
+
+// ---- the step loop's host side in one call per step (padoc_mpd_runner_*) ----------------------
+
+struct padoc_mpd_runner {
+    padoc_mpd *m = nullptr;
+    padoc_decode_config cfg{};
+    padoc_kv_pool pool{};
+    int32_t *stage[2] = {nullptr, nullptr};   // pinned host staging, used in turn
+    int64_t stage_words[2] = {0, 0};
+    cudaEvent_t copied[2] = {nullptr, nullptr};   // recorded after the step whose stage it is
+    bool recorded[2] = {false, false};
+    int32_t *dev_ints = nullptr;
+    int64_t dev_words = 0;
+    void *q_step = nullptr;
+    size_t q_bytes = 0;
+    void *workspace = nullptr;
+    size_t workspace_bytes = 0;
+    int64_t turn = 0;
+    int last = -1;                 // stage of the last prepared step
+    padoc_mpd_step last_step{};
+};
+
+namespace {
+
+void runner_free(padoc_mpd_runner *r)
+{
+    for (int b = 0; b < 2; ++b) {
+        if (r->copied[b]) {
+            if (r->recorded[b]) cudaEventSynchronize(r->copied[b]);
+            cudaEventDestroy(r->copied[b]);
+        }
+        if (r->stage[b]) cudaFreeHost(r->stage[b]);
+    }
+    cudaFree(r->dev_ints);   // the events above cover every launch that read these
+    cudaFree(r->q_step);
+    cudaFree(r->workspace);
+}
+
+// Grows a device buffer to at least `need` bytes (twice the old size at least). The stream is
+// drained first: the step in flight may still read the old buffer.
+padoc_status grow_device(void **buf, size_t *bytes, size_t need, cudaStream_t stream)
+{
+    if (need <= *bytes) return PADOC_OK;
+    const size_t nb = std::max(need, 2 * *bytes);
+    if (*buf) {
+        if (cudaStreamSynchronize(stream) != cudaSuccess) return PADOC_ERR_CUDA;
+        cudaFree(*buf);
+        *buf = nullptr;
+        *bytes = 0;
+    }
+    if (cudaMalloc(buf, nb) != cudaSuccess) {
+        *buf = nullptr;
+        return PADOC_ERR_CUDA;
+    }
+    *bytes = nb;
+    return PADOC_OK;
+}
+
+}  // namespace
+
+extern "C" padoc_status padoc_mpd_runner_create(padoc_mpd *m, const padoc_decode_config *cfg,
+                                                const padoc_kv_pool *pool, padoc_mpd_runner **runner)
+{
+    if (!m || !cfg || !pool || !runner) return PADOC_ERR_INVALID_ARGUMENT;
+    if (cfg->block_size != m->bs || pool->block_size != m->bs || pool->num_blocks < m->num_blocks ||
+        pool->num_kv_heads != cfg->num_kv_heads || pool->head_dim != cfg->head_dim || cfg->layout_streams)
+        return PADOC_ERR_INVALID_ARGUMENT;
+    padoc_mpd_runner *r = new (std::nothrow) padoc_mpd_runner;
+    if (!r) return PADOC_ERR_INVALID_ARGUMENT;
+    r->m = m;
+    r->cfg = *cfg;
+    r->pool = *pool;
+    for (int b = 0; b < 2; ++b)
+        if (cudaEventCreateWithFlags(&r->copied[b], cudaEventDisableTiming) != cudaSuccess) {
+            r->copied[b] = nullptr;
+            runner_free(r);
+            delete r;
+            return PADOC_ERR_CUDA;
+        }
+    *runner = r;
+    return PADOC_OK;
+}
+
+extern "C" void padoc_mpd_runner_destroy(padoc_mpd_runner *r)
+{
+    if (!r) return;
+    runner_free(r);
+    delete r;
+}
+
+extern "C" padoc_status padoc_mpd_runner_step(padoc_mpd_runner *r, const padoc_mpd_run_args *a, int32_t *num_streams,
+                                              int64_t *upload_bytes)
+{
+    if (!r || !a || !num_streams) return PADOC_ERR_INVALID_ARGUMENT;
+    if (upload_bytes) *upload_bytes = 0;
+    padoc_mpd *m = r->m;
+    if (m->in_step || a->src_total < 0 || a->out_rows < 0 || a->ids_capacity < 0) return PADOC_ERR_INVALID_ARGUMENT;
+    // what the step needs of the caller's arrays, checked before anything begins
+    int64_t C = 0;
+    for (int32_t pid : m->live_pages) C += page_streams(m->pages[pid]);
+    if (C > a->out_rows || C > a->ids_capacity) return PADOC_ERR_CAPACITY;
+    if (C > 0 && (!a->stream_ids || !a->src_row_of_stream || !a->k_src || !a->v_src || !a->q_src || !a->out ||
+                  !a->lse))
+        return PADOC_ERR_INVALID_ARGUMENT;
+    if (C > 0 && (int64_t)a->num_stream_ids < (int64_t)m->streams.size()) return PADOC_ERR_INVALID_ARGUMENT;
+    const cudaStream_t stream = (cudaStream_t)a->stream;
+    const int b = (int)(r->turn & 1);
+    if (r->recorded[b]) {   // the copy that read this stage two steps ago
+        if (cudaEventSynchronize(r->copied[b]) != cudaSuccess) return PADOC_ERR_CUDA;
+        r->recorded[b] = false;
+    }
+    padoc_mpd_step step;
+    padoc_status st;
+    for (;;) {
+        st = padoc_mpd_prepare_step(m, &r->cfg, r->stage[b], r->stage_words[b], &step);
+        if (st != PADOC_ERR_CAPACITY || step.total_words <= r->stage_words[b]) break;
+        // a larger stage (nothing has begun): no copy reads this one any more
+        if (r->stage[b]) cudaFreeHost(r->stage[b]);
+        r->stage[b] = nullptr;
+        r->stage_words[b] = 0;
+        const int64_t words = std::max<int64_t>(step.total_words * 2, 1 << 16);
+        void *p = nullptr;
+        if (cudaHostAlloc(&p, (size_t)words * sizeof(int32_t), cudaHostAllocDefault) != cudaSuccess)
+            return PADOC_ERR_CUDA;
+        r->stage[b] = static_cast<int32_t *>(p);
+        r->stage_words[b] = words;
+    }
+    if (st != PADOC_OK) return st;
+    ++r->turn;
+    r->last = b;
+    r->last_step = step;
+    const int32_t n = step.num_streams;
+    *num_streams = n;
+    if (n == 0) return PADOC_OK;
+    int32_t *stage = r->stage[b];
+    const int32_t *ids = stage + step.off_stream_ids;
+    std::memcpy(a->stream_ids, ids, (size_t)n * sizeof(int32_t));
+    for (int32_t i = 0; i < n; ++i) stage[step.off_rows + i] = a->src_row_of_stream[ids[i]];
+    // device buffers for this step (the stream is drained before one is replaced)
+    const size_t elt = r->pool.dtype == PADOC_DTYPE_BF16 ? 2 : 4;
+    size_t ws = 0, dev_bytes = (size_t)r->dev_words * sizeof(int32_t);
+    padoc_decode_workspace_size(&step.plan, &ws);
+    st = grow_device(reinterpret_cast<void **>(&r->dev_ints), &dev_bytes, (size_t)step.upload_words * sizeof(int32_t),
+                     stream);
+    r->dev_words = (int64_t)(dev_bytes / sizeof(int32_t));
+    if (st == PADOC_OK)
+        st = grow_device(&r->q_step, &r->q_bytes, (size_t)n * r->cfg.num_q_heads * r->cfg.head_dim * elt, stream);
+    if (st == PADOC_OK) st = grow_device(&r->workspace, &r->workspace_bytes, std::max<size_t>(ws, 256), stream);
+    if (st != PADOC_OK) return st;
+    st = padoc_mpd_launch_step(&step, stage, r->dev_ints, r->dev_words, &r->pool, a->k_src, a->v_src, a->q_src,
+                               a->src_total, r->q_step, a->scale, a->out, a->lse, r->workspace, r->workspace_bytes,
+                               a->stream);
+    if (st != PADOC_OK) return st;
+    if (cudaEventRecord(r->copied[b], stream) != cudaSuccess) return PADOC_ERR_CUDA;
+    r->recorded[b] = true;
+    if (upload_bytes) *upload_bytes = step.upload_words * (int64_t)sizeof(int32_t);
+    return PADOC_OK;
+}
+
+extern "C" padoc_status padoc_mpd_runner_last_step(const padoc_mpd_runner *r, padoc_mpd_step *step,
+                                                   const int32_t **stage)
+{
+    if (!r || !step || !stage || r->last < 0) return PADOC_ERR_INVALID_ARGUMENT;
+    *step = r->last_step;
+    *stage = r->stage[r->last];
+    return PADOC_OK;
+}

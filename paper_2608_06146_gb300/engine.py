@@ -140,6 +140,7 @@ class MaskedParallelLoop:
         self.last_step = None
         self.last_stage = None
         self.h2d_bytes = 0
+        self._runner = None
 
     def _upload(self, parts, stream):
         """Copies int32 host arrays to the device in one transfer, each starting on a 128-byte
@@ -228,6 +229,21 @@ class MaskedParallelLoop:
                                  out, lse, self.workspace, stream)
         self._stage_free[b].record(stream)
         return ids, out, lse
+
+    def run_step(self, k_src, v_src, q_src, row_of_stream, scale: float, out, lse, stream=None):
+        """step() as one library call (padoc_mpd_runner_step): row_of_stream is an int32 numpy table
+        of each live stream's source row indexed by stream id; out [rows][Hq][d] and lse [rows][Hq]
+        (rows at least the live streams) receive the outputs in step order. Returns (C, stream ids
+        int32 [C], valid until the next step); end the step with end_step."""
+        if self._runner is None:
+            self._runner = pa.MpdRunner(self.mpd, self.cfg, self._pool)
+        n, ids = self._runner.step(k_src, v_src, q_src, row_of_stream, scale, out, lse, stream)
+        self.h2d_bytes = self._runner.upload_bytes
+        return n, ids
+
+    def last_run_step(self):
+        """(padoc_mpd_step, its staging words) of the last run_step."""
+        return self._runner.last_step()
 
     def end_step(self, num_forks=None, eos=None, num_streams=None):
         """Each stream's output event (forks, EOS) in step order; returns the new branches' ids."""

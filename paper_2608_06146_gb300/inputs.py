@@ -246,6 +246,14 @@ class LoopTokenSource:
         self._count[ids] = c + 1
         return out
 
+    def peek_rows(self, ids) -> np.ndarray:
+        """rows(ids) without advancing: each stream's next input row (meaningless for a stream that is
+        not live)."""
+        ids = np.asarray(ids, np.int64)
+        pg, fl, c = self._page[ids], self._flat[ids], self._count[ids]
+        lay = fl < 0
+        return np.where(lay, self.base[pg] + self._P[pg] + c, self._yabs[np.where(lay, 0, fl)] + c)
+
     def events(self, ids):
         """(num_forks int32 [C], eos uint8 [C]) of the outputs of this step's streams."""
         ids = np.asarray(ids, np.int64)

@@ -91,6 +91,14 @@ class padoc_mpd_step(ctypes.Structure):
                 ("plan", padoc_decode_plan)]
 
 
+class padoc_mpd_run_args(ctypes.Structure):
+    _fields_ = [("k_src", ctypes.c_void_p), ("v_src", ctypes.c_void_p), ("q_src", ctypes.c_void_p),
+                ("src_total", ctypes.c_int64), ("src_row_of_stream", ctypes.c_void_p),
+                ("num_stream_ids", ctypes.c_int32), ("scale", ctypes.c_float), ("out", ctypes.c_void_p),
+                ("lse", ctypes.c_void_p), ("out_rows", ctypes.c_int32), ("ids_capacity", ctypes.c_int32),
+                ("stream_ids", ctypes.c_void_p), ("stream", ctypes.c_void_p)]
+
+
 _lib = None
 _i32p = ctypes.POINTER(ctypes.c_int32)
 _i64p = ctypes.POINTER(ctypes.c_int64)
@@ -165,6 +173,11 @@ def load_library(path: Optional[str] = None):
         "padoc_mpd_launch_step": [ctypes.POINTER(padoc_mpd_step), _vp, _vp, ctypes.c_int64,
                                   ctypes.POINTER(padoc_kv_pool), _vp, _vp, _vp, ctypes.c_int64, _vp, ctypes.c_float, _vp,
                                   _vp, _vp, ctypes.c_size_t, _vp],
+        "padoc_mpd_runner_create": [_vp, ctypes.POINTER(padoc_decode_config), ctypes.POINTER(padoc_kv_pool),
+                                    ctypes.POINTER(_vp)],
+        "padoc_mpd_runner_destroy": [_vp],
+        "padoc_mpd_runner_step": [_vp, ctypes.POINTER(padoc_mpd_run_args), _i32p, _i64p],
+        "padoc_mpd_runner_last_step": [_vp, ctypes.POINTER(padoc_mpd_step), ctypes.POINTER(_i32p)],
         "padoc_selftest_tcgen05": [_vp, _vp, _vp, _vp, _vp, _vp, _vp],
         "padoc_selftest_wait_timeout": [ctypes.c_int32, ctypes.c_int32, _vp, _vp],
         "padoc_advance_decode_plan": [_i32p, ctypes.POINTER(padoc_decode_plan), _i32p, ctypes.c_int32],
@@ -190,6 +203,7 @@ def load_library(path: Optional[str] = None):
     lib.padoc_status_string.restype = ctypes.c_char_p
     lib.padoc_last_device_error.restype = None
     lib.padoc_mpd_destroy.restype = None
+    lib.padoc_mpd_runner_destroy.restype = None
     _lib = lib
     return lib
 
@@ -207,7 +221,8 @@ def exported_symbols() -> Sequence[str]:
                         "padoc_mpd_create", "padoc_mpd_destroy",
                         "padoc_mpd_add_page", "padoc_mpd_begin_step", "padoc_mpd_step_shape",
                         "padoc_mpd_step_tables", "padoc_mpd_end_step", "padoc_mpd_status", "padoc_mpd_prepare_step",
-                        "padoc_mpd_launch_step",
+                        "padoc_mpd_launch_step", "padoc_mpd_runner_create", "padoc_mpd_runner_destroy",
+                        "padoc_mpd_runner_step", "padoc_mpd_runner_last_step",
                         "padoc_append_inputs",
                         "padoc_selftest_tcgen05", "padoc_selftest_wait_timeout",
                         "padoc_quantize_kv_blocks", "padoc_append_inputs_e4m3", "padoc_branch_decode_attn_e4m3",
@@ -697,6 +712,97 @@ def padoc_mpd_launch_step(step: padoc_mpd_step, stage, dev_ints, pool: padoc_kv_
                                    _dev(lse, "lse"), _dev(workspace, "workspace"),
                                    workspace.numel() * workspace.element_size(), _stream_ptr(stream))
     _check("padoc_mpd_launch_step", st)
+
+
+class MpdRunner:
+    """padoc_mpd_runner_*: the loop's per-step host work in one library call. The runner owns its
+    staging and device buffers; the scheduler and the pool (their padoc_kv_pool and tensors) must
+    outlive it. ``step`` takes the source rows as an int32 table indexed by stream id."""
+
+    def __init__(self, mpd: Mpd, cfg: padoc_decode_config, pool: padoc_kv_pool):
+        self._lib = load_library()
+        self._mpd, self._cfg, self._pool = mpd, cfg, pool   # kept alive
+        h = _vp()
+        _check("padoc_mpd_runner_create", self._lib.padoc_mpd_runner_create(mpd._h, ctypes.byref(cfg),
+                                                                            ctypes.byref(pool), ctypes.byref(h)))
+        self._h = h
+        self._args = padoc_mpd_run_args()
+        self._args_ref = ctypes.byref(self._args)
+        self._n = ctypes.c_int32()
+        self._n_ref = ctypes.byref(self._n)
+        self._up = ctypes.c_int64()
+        self._up_ref = ctypes.byref(self._up)
+        self._ids = np.zeros(64, np.int32)
+        self._keep = ()
+
+    def close(self):
+        if self._h:
+            self._lib.padoc_mpd_runner_destroy(self._h)
+            self._h = _vp()
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def step(self, k_src, v_src, q_src, row_of_stream: np.ndarray, scale: float, out, lse, stream=None):
+        """One step: returns (C, stream ids int32 [C], a view of the runner's array valid until the
+        next step). out [rows >= C][Hq][d] and lse fp32 [rows][Hq] receive the outputs in step order;
+        row_of_stream: int32 [ids] (host), the source row of each live stream's input."""
+        a = self._args
+        keep = (k_src, v_src, q_src, row_of_stream, out, lse)
+        if len(self._keep) != 6 or any(x is not y for x, y in zip(keep, self._keep)):
+            self._set_arrays(keep)   # checked once per set of arrays
+        a.scale = scale
+        a.stream = _stream_ptr(stream)
+        _check("padoc_mpd_runner_step", self._lib.padoc_mpd_runner_step(self._h, self._args_ref, self._n_ref,
+                                                                        self._up_ref))
+        n = self._n.value
+        return n, self._ids[:n]
+
+    @property
+    def upload_bytes(self) -> int:
+        """Bytes the last step copied to the device."""
+        return self._up.value
+
+    def _set_arrays(self, keep):
+        k_src, v_src, q_src, row_of_stream, out, lse = keep
+        dt = PADOC_DTYPE_BF16 if self._pool.dtype == PADOC_DTYPE_BF16 else PADOC_DTYPE_F32
+        for t, nm in ((k_src, "k_src"), (v_src, "v_src"), (q_src, "q_src"), (out, "out")):
+            _dev(t, nm)
+            if _dtype_code(t) != dt:
+                raise TypeError(f"{nm} must have the pool's dtype")
+        _dev(lse, "lse")
+        if str(lse.dtype) != "torch.float32":
+            raise TypeError("lse must be float32")
+        c = self._cfg
+        if (tuple(k_src.shape[1:]) != (c.num_kv_heads, c.head_dim) or tuple(v_src.shape) != tuple(k_src.shape) or
+                tuple(q_src.shape[1:]) != (c.num_q_heads, c.head_dim) or q_src.shape[0] != k_src.shape[0] or
+                tuple(out.shape[1:]) != (c.num_q_heads, c.head_dim) or lse.dim() != 2 or lse.shape[1] != c.num_q_heads):
+            raise ValueError("k_src/v_src [rows][Hkv][d], q_src [rows][Hq][d], out [rows][Hq][d], lse [rows][Hq]")
+        if not isinstance(row_of_stream, np.ndarray) or row_of_stream.dtype != np.int32 or \
+                not row_of_stream.flags.c_contiguous:
+            raise ValueError("row_of_stream must be a contiguous int32 numpy array")
+        a = self._args
+        a.k_src, a.v_src, a.q_src = k_src.data_ptr(), v_src.data_ptr(), q_src.data_ptr()
+        a.src_total = k_src.shape[0]
+        a.src_row_of_stream = row_of_stream.ctypes.data
+        a.num_stream_ids = row_of_stream.size
+        cap = min(int(out.shape[0]), int(lse.shape[0]))
+        if self._ids.size < cap:
+            self._ids = np.zeros(cap, np.int32)
+        a.out, a.lse, a.out_rows = out.data_ptr(), lse.data_ptr(), cap
+        a.ids_capacity, a.stream_ids = self._ids.size, self._ids.ctypes.data
+        self._keep = keep
+
+    def last_step(self):
+        """(padoc_mpd_step, its staging buffer as an int32 numpy array [total_words])."""
+        st = padoc_mpd_step()
+        p = _i32p()
+        _check("padoc_mpd_runner_last_step", self._lib.padoc_mpd_runner_last_step(self._h, ctypes.byref(st),
+                                                                                  ctypes.byref(p)))
+        return st, np.ctypeslib.as_array(p, (max(int(st.total_words), 1),))
 
 
 def make_kv_pool(k_pool, v_pool) -> padoc_kv_pool:

@@ -36,9 +36,10 @@ def _blocks_needed(pages, bs=16):
     return sum(-(-(pg.prefix_len + pg.layout_len) // bs) + sum(-(-n // bs) for n in pg.branch_len) for pg in pages)
 
 
-def run_loop(wl: Workload, seed: int, admit_at=None, keep_rows=None, scale_in=1.0, slack=3):
+def run_loop(wl: Workload, seed: int, admit_at=None, keep_rows=None, scale_in=1.0, slack=3, runner=False):
     """Runs the loop over wl.pages; returns (packed rows decoded, O fp32, LSE) of the kept rows
-    (all rows when keep_rows is None) and the loop."""
+    (all rows when keep_rows is None) and the loop. runner: each step through the one-call runner
+    (padoc_mpd_runner_step, source rows from a table by stream id) instead of prepare + launch."""
     q, k, v = inputs.packed_qkv(wl, seed, scale_in)
     qd, kd, vd = q.to(DEV), k.to(DEV), v.to(DEV)
     src = LoopTokenSource(wl.pages)
@@ -50,6 +51,10 @@ def run_loop(wl: Workload, seed: int, admit_at=None, keep_rows=None, scale_in=1.
     pending = sorted(range(len(wl.pages)), key=lambda p: admit_at[p])
     keep = None if keep_rows is None else set(int(r) for r in keep_rows)
     rows_out, o_out, l_out = [], [], []
+    cap = sum(1 + pg.num_branches for pg in wl.pages)   # every stream id the loop can create
+    out_buf = torch.empty((cap, wl.num_q_heads, wl.head_dim), dtype=wl.dtype, device=DEV)
+    lse_buf = torch.empty((cap, wl.num_q_heads), dtype=torch.float32, device=DEV)
+    row_of = np.zeros(cap, np.int32)
     step = 0
     while True:
         while pending and admit_at[pending[0]] <= step:
@@ -62,7 +67,14 @@ def run_loop(wl: Workload, seed: int, admit_at=None, keep_rows=None, scale_in=1.
                 break
             step += 1
             continue
-        ids, out, lse = loop.step(kd, vd, qd, src.rows, scale)
+        if runner:
+            row_of[:] = src.peek_rows(np.arange(cap))
+            n, ids = loop.run_step(kd, vd, qd, row_of, scale, out_buf, lse_buf)
+            ids = ids.copy()
+            assert np.array_equal(src.rows(ids), row_of[ids])
+            out, lse = out_buf[:n], lse_buf[:n]
+        else:
+            ids, out, lse = loop.step(kd, vd, qd, src.rows, scale)
         rows = src.token_rows(ids)
         sel = np.arange(len(ids)) if keep is None else np.array([i for i, r in enumerate(rows) if int(r) in keep],
                                                                 np.int64)
@@ -116,6 +128,26 @@ def test_loop_bf16_edge_pages_staggered():
              PageSpec(130, 24, [24, 12], [2, 70])]
     wl = Workload("loop edge pages", pages, 16, 2, 128, torch.bfloat16, "decode")
     check_all_rows(wl, 5, admit_at=[0, 0, 4, 6, 30])
+
+
+def test_loop_runner_matches_two_call_loop():
+    """The one-call runner (padoc_mpd_runner_step) and the prepare + launch path make the same steps:
+    the same streams in the same order and bit-identical outputs and LSE, on the edge pages with
+    staggered admission; both match the oracle."""
+    pages = [PageSpec(37, 10, [0, 10, 3, 3, 7], [17, 5, 33, 1, 16]),
+             PageSpec(50, 0, [0, 0], [20, 3]),
+             PageSpec(0, 6, [6, 2], [4, 18]),
+             PageSpec(300, 40, [40, 4, 8, 12, 16, 20, 24, 28, 32, 36, 0, 1], [40, 35, 3, 60, 22, 17, 16, 33, 48, 9,
+                                                                               12, 25])]
+    wl = Workload("loop runner pages", pages, 16, 2, 128, torch.bfloat16, "decode")
+    a = run_loop(wl, 6, admit_at=[0, 2, 5, 9])
+    b = run_loop(wl, 6, admit_at=[0, 2, 5, 9], runner=True)
+    np.testing.assert_array_equal(a[0], b[0])
+    np.testing.assert_array_equal(a[1], b[1])
+    np.testing.assert_array_equal(a[2], b[2])
+    q, k, v = b[3], b[4], b[5]
+    ref_o, ref_lse = oracle.prefill_dense(wl.pages, q, k, v, 1.0 / math.sqrt(wl.head_dim))
+    assert_close(b[1], b[2], ref_o[b[0]], ref_lse[b[0]], wl.dtype)
 
 
 def test_loop_bf16_serving_batch_sampled():

@@ -306,3 +306,25 @@ def test_launch_step_validates_before_any_device_work(lib):
     assert call(None, 4096, st.upload_words, ctypes.byref(pool)) == 1     # no stage
     assert call(sp, 4096, st.upload_words, None) == 1                     # no pool
     m.end_step(np.zeros(3, np.int32), np.zeros(3, np.uint8))
+
+
+def test_runner_validates_before_any_device_work(lib):
+    """padoc_mpd_runner_create rejects a configuration or pool that does not fit the scheduler before
+    any CUDA call; without a GPU, a valid one fails with the CUDA status, loudly; a runner step
+    checks its arguments before it begins anything (these checks need no GPU)."""
+    import ctypes
+    m = pa.Mpd(64)
+    cfg = pa.make_decode_config(16, 2, 128)
+    h = ctypes.c_void_p()
+    mk = lambda nb, bs, hkv, d: pa.padoc_kv_pool(256, 512, nb, bs, hkv, d, pa.PADOC_DTYPE_BF16)
+    for pool in (mk(63, 16, 2, 128), mk(64, 8, 2, 128), mk(64, 16, 1, 128), mk(64, 16, 2, 64)):
+        assert lib.padoc_mpd_runner_create(m._h, ctypes.byref(cfg), ctypes.byref(pool), ctypes.byref(h)) == 1
+    lay = pa.make_decode_config(16, 2, 128, True)
+    assert lib.padoc_mpd_runner_create(m._h, ctypes.byref(lay), ctypes.byref(mk(64, 16, 2, 128)), ctypes.byref(h)) == 1
+    assert lib.padoc_mpd_runner_create(None, ctypes.byref(cfg), ctypes.byref(mk(64, 16, 2, 128)), ctypes.byref(h)) == 1
+    assert lib.padoc_mpd_runner_step(None, None, None, None) == 1
+    import torch
+    if not torch.cuda.is_available():
+        with pytest.raises(pa.PadocError) as e:
+            pa.MpdRunner(m, cfg, mk(64, 16, 2, 128))
+        assert e.value.status == 4
