@@ -1,6 +1,8 @@
 // api.cu -- status reporting, the per-device error word and tensor-map encoding for padoc_attn.
 #include <cudaTypedefs.h>
 #include <mutex>
+#include <tuple>
+#include <vector>
 
 #include "common.cuh"
 
@@ -42,9 +44,71 @@ int *padoc_device_error_word()
     return g_err_ptr[dev];
 }
 
+namespace {
+
+// The last few 2-D maps this thread encoded, by their arguments: a decoding loop encodes the same
+// pool's maps every step, and an encoding is a pure function of its arguments.
+struct TmapKey {
+    int dtype;
+    const void *base;
+    uint64_t cols, rows, stride;
+    uint32_t box_cols, box_rows;
+    bool operator==(const TmapKey &o) const
+    {
+        return dtype == o.dtype && base == o.base && cols == o.cols && rows == o.rows && stride == o.stride &&
+               box_cols == o.box_cols && box_rows == o.box_rows;
+    }
+};
+struct TmapCache {
+    TmapKey key[4];
+    CUtensorMap map[4];
+    bool used[4] = {false, false, false, false};
+    int next = 0;
+};
+thread_local TmapCache t_tmaps;
+
+bool tmap_cached(const TmapKey &k, CUtensorMap *map)
+{
+    for (int i = 0; i < 4; ++i)
+        if (t_tmaps.used[i] && t_tmaps.key[i] == k) {
+            *map = t_tmaps.map[i];
+            return true;
+        }
+    return false;
+}
+
+void tmap_remember(const TmapKey &k, const CUtensorMap &map)
+{
+    const int i = t_tmaps.next;
+    t_tmaps.next = (i + 1) & 3;
+    t_tmaps.key[i] = k;
+    t_tmaps.map[i] = map;
+    t_tmaps.used[i] = true;
+}
+
+}  // namespace
+
+padoc_status padoc_set_max_smem(const void *kernel, int bytes)
+{
+    // once per (kernel, size, device): the attribute stays set on the device's context
+    static std::mutex mu;
+    static std::vector<std::tuple<const void *, int, int>> done;
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return PADOC_ERR_CUDA;
+    std::lock_guard<std::mutex> lk(mu);
+    for (const auto &d : done)
+        if (std::get<0>(d) == kernel && std::get<1>(d) == bytes && std::get<2>(d) == dev) return PADOC_OK;
+    if (cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes) != cudaSuccess)
+        return PADOC_ERR_CUDA;
+    done.emplace_back(kernel, bytes, dev);
+    return PADOC_OK;
+}
+
 bool padoc_make_tmap_bf16(CUtensorMap *map, const void *base, uint64_t cols, uint64_t rows, uint64_t row_stride_bytes,
                           uint32_t box_cols, uint32_t box_rows)
 {
+    const TmapKey key{0, base, cols, rows, row_stride_bytes, box_cols, box_rows};
+    if (tmap_cached(key, map)) return true;
     PFN_cuTensorMapEncodeTiled_v12000 fn = encode_fn();
     if (!fn) return false;
     if ((((uintptr_t)base) & 15) || (row_stride_bytes & 15) || rows == 0 || cols == 0) return false;
@@ -55,12 +119,16 @@ bool padoc_make_tmap_bf16(CUtensorMap *map, const void *base, uint64_t cols, uin
     CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(base), dims, strides, box, estr,
                     CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-    return r == CUDA_SUCCESS;
+    if (r != CUDA_SUCCESS) return false;
+    tmap_remember(key, *map);
+    return true;
 }
 
 bool padoc_make_tmap_u8(CUtensorMap *map, const void *base, uint64_t cols, uint64_t rows, uint64_t row_stride_bytes,
                         uint32_t box_cols, uint32_t box_rows)
 {
+    const TmapKey key{1, base, cols, rows, row_stride_bytes, box_cols, box_rows};
+    if (tmap_cached(key, map)) return true;
     PFN_cuTensorMapEncodeTiled_v12000 fn = encode_fn();
     if (!fn) return false;
     if ((((uintptr_t)base) & 15) || (row_stride_bytes & 15) || rows == 0 || cols == 0 || box_cols > 128) return false;
@@ -71,7 +139,9 @@ bool padoc_make_tmap_u8(CUtensorMap *map, const void *base, uint64_t cols, uint6
     CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<void *>(base), dims, strides, box, estr,
                     CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-    return r == CUDA_SUCCESS;
+    if (r != CUDA_SUCCESS) return false;
+    tmap_remember(key, *map);
+    return true;
 }
 
 bool padoc_make_tmap_bf16_4d(CUtensorMap *map, const void *base, const uint64_t dims[4], const uint64_t strides_bytes[3],

@@ -344,6 +344,8 @@ __device__ __forceinline__ void pdl_wait_prerequisite() { asm volatile("griddepc
 int *padoc_device_error_word();
 // 2-D bf16 tensor map: rows x cols elements with a row pitch of `row_stride_bytes`, box of
 // box_rows x 64 columns, 128-byte swizzle. Returns false if the driver rejects it.
+// cudaFuncSetAttribute(kernel, MaxDynamicSharedMemorySize, bytes), once per kernel, size and device.
+padoc_status padoc_set_max_smem(const void *kernel, int bytes);
 bool padoc_make_tmap_bf16(CUtensorMap *map, const void *base, uint64_t cols, uint64_t rows,
                           uint64_t row_stride_bytes, uint32_t box_cols, uint32_t box_rows);
 // 2-D uint8 tensor map (E4M3 codes): rows x cols bytes with a row pitch of `row_stride_bytes`, box of

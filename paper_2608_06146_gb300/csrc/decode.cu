@@ -369,8 +369,8 @@ padoc_status decode_split_k(const DecodePool &pl, const padoc_decode_plan *info,
     if (st != PADOC_OK) return st;
     if (pl.e4m3 && prm.num_warps > 0) {   // E4M3: the warp lists in a grid of their own
         const int after_tc = info->num_tc_items > 0 ? 1 : 0;
-        PADOC_CUDA_TRY(cudaFuncSetAttribute(decode_warp_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                            (int)kDecodeSmemE4M3));
+        st = padoc_set_max_smem(reinterpret_cast<const void *>(decode_warp_kernel<true>), (int)kDecodeSmemE4M3);
+        if (st != PADOC_OK) return st;
         cudaLaunchConfig_t lc = {};
         lc.gridDim = dim3((unsigned)((prm.num_warps + kWarps - 1) / kWarps));
         lc.blockDim = dim3(kWarps * 32);

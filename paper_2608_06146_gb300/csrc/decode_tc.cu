@@ -887,7 +887,10 @@ padoc_status padoc_launch_decode_tc(const CUtensorMap *kmap, const CUtensorMap *
     const bool sole = (int64_t)info->num_merge_keys < (int64_t)info->num_streams * info->cfg.num_kv_heads;
     auto kern = e4m3 ? (sole ? decode_tc_kernel<true, false, true> : decode_tc_kernel<true, false, false>)
                      : (sole ? decode_tc_kernel<false, true, true> : decode_tc_kernel<false, true, false>);
-    PADOC_CUDA_TRY(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes));
+    {
+        const padoc_status ast = padoc_set_max_smem(reinterpret_cast<const void *>(kern), (int)kSmemBytes);
+        if (ast != PADOC_OK) return ast;
+    }
     cudaLaunchConfig_t lc = {};
     lc.gridDim = dim3((unsigned)(prm.tc_ctas + prm.early_ctas));
     lc.blockDim = dim3(kThreads);

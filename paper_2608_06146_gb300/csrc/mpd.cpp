@@ -497,8 +497,10 @@ extern "C" padoc_status padoc_mpd_runner_step(padoc_mpd_runner *r, const padoc_m
     if (C > 0 && (int64_t)a->num_stream_ids < (int64_t)m->streams.size()) return PADOC_ERR_INVALID_ARGUMENT;
     const cudaStream_t stream = (cudaStream_t)a->stream;
     const int b = (int)(r->turn & 1);
-    if (r->recorded[b]) {   // the copy that read this stage two steps ago
-        if (cudaEventSynchronize(r->copied[b]) != cudaSuccess) return PADOC_ERR_CUDA;
+    if (r->recorded[b]) {   // the copy that read this stage two steps ago (usually done: ask first)
+        const cudaError_t q = cudaEventQuery(r->copied[b]);
+        if (q != cudaSuccess && (q != cudaErrorNotReady || cudaEventSynchronize(r->copied[b]) != cudaSuccess))
+            return PADOC_ERR_CUDA;
         r->recorded[b] = false;
     }
     padoc_mpd_step step;

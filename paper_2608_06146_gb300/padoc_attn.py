@@ -163,8 +163,7 @@ def load_library(path: Optional[str] = None):
         "padoc_mpd_step_shape": [_vp, _i32p, _i32p, _i32p, _i32p],
         "padoc_mpd_step_tables": [_vp, _i32p, ctypes.POINTER(padoc_stream_desc), _i32p, ctypes.c_int32, _i32p,
                                   ctypes.c_int32],
-        "padoc_mpd_end_step": [_vp, _i32p, ctypes.POINTER(ctypes.c_uint8), ctypes.c_int32, _i32p, ctypes.c_int32,
-                               _i32p],
+        "padoc_mpd_end_step": [_vp, _vp, _vp, ctypes.c_int32, _vp, ctypes.c_int32, _i32p],
         "padoc_mpd_status": [_vp, _i32p, _i32p, _i32p],
         "padoc_mpd_prepare_step": [_vp, ctypes.POINTER(padoc_decode_config), _i32p, ctypes.c_int64,
                                    ctypes.POINTER(padoc_mpd_step)],
@@ -281,10 +280,18 @@ def _as_pages(pages) -> _Pages:
     return pages if isinstance(pages, _Pages) else _Pages(pages)
 
 
+_raw_stream = None
+
+
 def _stream_ptr(stream):
+    """The cudaStream_t of ``stream`` (a torch stream or a raw handle); None: torch's current stream."""
+    global _raw_stream
     if stream is None:
         import torch
-        return torch.cuda.current_stream().cuda_stream
+        if _raw_stream is None:
+            get, dev = getattr(torch._C, "_cuda_getCurrentRawStream", None), getattr(torch._C, "_cuda_getDevice", None)
+            _raw_stream = (lambda: get(dev())) if get and dev else (lambda: torch.cuda.current_stream().cuda_stream)
+        return _raw_stream()
     return getattr(stream, "cuda_stream", stream)
 
 
@@ -605,6 +612,14 @@ class Mpd:
         self.block_size = block_size
         self._cap = 0
         self._ids = self._slots = None
+        self._ev_cap = 64
+        self._nf = np.zeros(self._ev_cap, np.int32)
+        self._eos = np.zeros(self._ev_cap, np.uint8)
+        self._nf_p, self._eos_p = self._nf.ctypes.data, self._eos.ctypes.data
+        self._new = np.zeros(256, np.int32)
+        self._new_p = self._new.ctypes.data
+        self._k = ctypes.c_int32()
+        self._k_ref = ctypes.byref(self._k)
 
     def close(self):
         if self._h:
@@ -666,20 +681,31 @@ class Mpd:
         return page_len[:npg], streams[:ns], pt[:npg], stt[:ns]
 
     def end_step(self, num_forks=None, eos=None, num_streams=None):
-        """num_forks int32 [C], eos bool/uint8 [C] (None = all zero). Returns the new branches' ids."""
+        """num_forks int32 [C], eos bool/uint8 [C] (None = all zero). Returns the new branches' ids.
+        The events are copied into arrays kept here, whose addresses are marshalled once."""
         n = num_streams
         if n is None:
             n = len(num_forks) if num_forks is not None else len(eos) if eos is not None else 0
-        f = None if num_forks is None else np.ascontiguousarray(num_forks, np.int32)
-        e = None if eos is None else np.ascontiguousarray(eos, np.uint8)
-        total = int(f.sum()) if f is not None else 0
-        new = np.zeros(max(total, 1), np.int32)
-        k = ctypes.c_int32()
-        _check("padoc_mpd_end_step",
-               self._lib.padoc_mpd_end_step(self._h, None if f is None else f.ctypes.data_as(_i32p),
-                                            None if e is None else e.ctypes.data_as(ctypes.POINTER(ctypes.c_uint8)),
-                                            n, new.ctypes.data_as(_i32p), new.size, ctypes.byref(k)))
-        return new[:k.value]
+        if n > self._ev_cap:
+            self._ev_cap = max(n, 2 * self._ev_cap, 64)
+            self._nf = np.zeros(self._ev_cap, np.int32)
+            self._eos = np.zeros(self._ev_cap, np.uint8)
+            self._nf_p, self._eos_p = self._nf.ctypes.data, self._eos.ctypes.data
+        fp = ep = None
+        if num_forks is not None:
+            self._nf[:n] = num_forks
+            fp = self._nf_p
+        if eos is not None:
+            self._eos[:n] = eos
+            ep = self._eos_p
+        while True:
+            st = self._lib.padoc_mpd_end_step(self._h, fp, ep, n, self._new_p, self._new.size, self._k_ref)
+            if st != 6 or fp is None:
+                break
+            self._new = np.zeros(max(2 * self._new.size, int(self._nf[:n].sum())), np.int32)   # nothing changed
+            self._new_p = self._new.ctypes.data
+        _check("padoc_mpd_end_step", st)
+        return self._new[:self._k.value].copy()
 
     def prepare_step(self, cfg: padoc_decode_config, stage: np.ndarray) -> padoc_mpd_step:
         """padoc_mpd_prepare_step into ``stage`` (int32 numpy array, e.g. a view of pinned memory).
@@ -733,7 +759,9 @@ class MpdRunner:
         self._up = ctypes.c_int64()
         self._up_ref = ctypes.byref(self._up)
         self._ids = np.zeros(64, np.int32)
-        self._keep = ()
+        self._args.ids_capacity, self._args.stream_ids = self._ids.size, self._ids.ctypes.data
+        self._src = None
+        self._outs = {}
 
     def close(self):
         if self._h:
@@ -749,11 +777,17 @@ class MpdRunner:
     def step(self, k_src, v_src, q_src, row_of_stream: np.ndarray, scale: float, out, lse, stream=None):
         """One step: returns (C, stream ids int32 [C], a view of the runner's array valid until the
         next step). out [rows >= C][Hq][d] and lse fp32 [rows][Hq] receive the outputs in step order;
-        row_of_stream: int32 [ids] (host), the source row of each live stream's input."""
+        row_of_stream: int32 [ids] (host), the source row of each live stream's input. Arrays are
+        checked the first time they are seen (the runner keeps the last few)."""
         a = self._args
-        keep = (k_src, v_src, q_src, row_of_stream, out, lse)
-        if len(self._keep) != 6 or any(x is not y for x, y in zip(keep, self._keep)):
-            self._set_arrays(keep)   # checked once per set of arrays
+        src = self._src
+        if src is None or src[0] is not k_src or src[1] is not v_src or src[2] is not q_src or \
+                src[3] is not row_of_stream:
+            self._set_sources(k_src, v_src, q_src, row_of_stream)
+        o = self._outs.get((id(out), id(lse)))
+        if o is None or o[0] is not out or o[1] is not lse:
+            o = self._set_outputs(out, lse)
+        a.out, a.lse, a.out_rows = o[2], o[3], o[4]
         a.scale = scale
         a.stream = _stream_ptr(stream)
         _check("padoc_mpd_runner_step", self._lib.padoc_mpd_runner_step(self._h, self._args_ref, self._n_ref,
@@ -766,21 +800,16 @@ class MpdRunner:
         """Bytes the last step copied to the device."""
         return self._up.value
 
-    def _set_arrays(self, keep):
-        k_src, v_src, q_src, row_of_stream, out, lse = keep
+    def _set_sources(self, k_src, v_src, q_src, row_of_stream):
+        c = self._cfg
         dt = PADOC_DTYPE_BF16 if self._pool.dtype == PADOC_DTYPE_BF16 else PADOC_DTYPE_F32
-        for t, nm in ((k_src, "k_src"), (v_src, "v_src"), (q_src, "q_src"), (out, "out")):
+        for t, nm in ((k_src, "k_src"), (v_src, "v_src"), (q_src, "q_src")):
             _dev(t, nm)
             if _dtype_code(t) != dt:
                 raise TypeError(f"{nm} must have the pool's dtype")
-        _dev(lse, "lse")
-        if str(lse.dtype) != "torch.float32":
-            raise TypeError("lse must be float32")
-        c = self._cfg
         if (tuple(k_src.shape[1:]) != (c.num_kv_heads, c.head_dim) or tuple(v_src.shape) != tuple(k_src.shape) or
-                tuple(q_src.shape[1:]) != (c.num_q_heads, c.head_dim) or q_src.shape[0] != k_src.shape[0] or
-                tuple(out.shape[1:]) != (c.num_q_heads, c.head_dim) or lse.dim() != 2 or lse.shape[1] != c.num_q_heads):
-            raise ValueError("k_src/v_src [rows][Hkv][d], q_src [rows][Hq][d], out [rows][Hq][d], lse [rows][Hq]")
+                tuple(q_src.shape[1:]) != (c.num_q_heads, c.head_dim) or q_src.shape[0] != k_src.shape[0]):
+            raise ValueError("k_src/v_src [rows][Hkv][d], q_src [rows][Hq][d]")
         if not isinstance(row_of_stream, np.ndarray) or row_of_stream.dtype != np.int32 or \
                 not row_of_stream.flags.c_contiguous:
             raise ValueError("row_of_stream must be a contiguous int32 numpy array")
@@ -789,12 +818,28 @@ class MpdRunner:
         a.src_total = k_src.shape[0]
         a.src_row_of_stream = row_of_stream.ctypes.data
         a.num_stream_ids = row_of_stream.size
+        self._src = (k_src, v_src, q_src, row_of_stream)
+
+    def _set_outputs(self, out, lse):
+        c = self._cfg
+        dt = PADOC_DTYPE_BF16 if self._pool.dtype == PADOC_DTYPE_BF16 else PADOC_DTYPE_F32
+        _dev(out, "out")
+        _dev(lse, "lse")
+        if _dtype_code(out) != dt:
+            raise TypeError("out must have the pool's dtype")
+        if str(lse.dtype) != "torch.float32":
+            raise TypeError("lse must be float32")
+        if tuple(out.shape[1:]) != (c.num_q_heads, c.head_dim) or lse.dim() != 2 or lse.shape[1] != c.num_q_heads:
+            raise ValueError("out [rows][Hq][d], lse [rows][Hq]")
         cap = min(int(out.shape[0]), int(lse.shape[0]))
         if self._ids.size < cap:
             self._ids = np.zeros(cap, np.int32)
-        a.out, a.lse, a.out_rows = out.data_ptr(), lse.data_ptr(), cap
-        a.ids_capacity, a.stream_ids = self._ids.size, self._ids.ctypes.data
-        self._keep = keep
+            self._args.ids_capacity, self._args.stream_ids = self._ids.size, self._ids.ctypes.data
+        if len(self._outs) >= 8:
+            self._outs.clear()
+        o = (out, lse, out.data_ptr(), lse.data_ptr(), cap)
+        self._outs[(id(out), id(lse))] = o
+        return o
 
     def last_step(self):
         """(padoc_mpd_step, its staging buffer as an int32 numpy array [total_words])."""

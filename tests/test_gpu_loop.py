@@ -208,3 +208,12 @@ def test_append_inputs_bit_exact():
         b, o = divmod(int(slots[i]), 16)
         assert torch.equal(kp[b, :, o], ks[src[i]]) and torch.equal(vp[b, :, o], vs[src[i]])
     assert torch.equal(q_dst.cpu(), qs[torch.from_numpy(src).long()])
+
+
+def test_current_stream_handle():
+    """The binding's default stream is torch's current stream, also inside a stream context."""
+    assert pa._stream_ptr(None) == torch.cuda.current_stream().cuda_stream
+    s = torch.cuda.Stream()
+    with torch.cuda.stream(s):
+        assert pa._stream_ptr(None) == s.cuda_stream
+    assert pa._stream_ptr(None) == torch.cuda.current_stream().cuda_stream
