@@ -179,9 +179,11 @@ typedef struct {
     int32_t layout_streams;  /* 1: also decode each page's layout stream (Alg. 1 decodes every live
                                 stream): cutoff P + L over the shared stream, no private rows */
     int32_t split_tokens;    /* shared-stream tokens per split-K partial of the warp kernel (pages with
-                                too few streams for the tensor cores); 0 = library default (256);
-                                a positive value must be a multiple of block_size; values above
-                                512 act as 512 */
+                                too few streams for the tensor cores); a positive value must be a
+                                multiple of block_size, values above 512 act as 512, and private
+                                histories are then cut every 256 tokens; 0 = the planner's choice:
+                                256 tokens for both, or 128 / 64 when the warp work is small
+                                against the warp grid (a decoding loop's steps with few streams) */
     int32_t tc_ctas;         /* CTAs the tensor-core shared-stream work is balanced over (one range of
                                 equal work each); 0 = the current device's multiprocessor count */
     int32_t warp_ctas;       /* CTAs (of 8 warps) the warp-kernel work is balanced over, one wave;

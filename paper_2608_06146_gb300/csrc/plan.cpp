@@ -253,7 +253,9 @@ int32_t padoc_default_ctas()
 
 namespace {
 
-int32_t choose_tc_ctas(const PlanParts &pp, const padoc_decode_config *cfg, int64_t total_w, int64_t max_piece);
+int32_t choose_tc_ctas(const PlanParts &pp, const padoc_decode_config *cfg, int64_t total_w, int64_t max_piece,
+                       int32_t split, int32_t psplit);
+int32_t warp_split_tokens(const PlanParts &pp, const padoc_decode_config *cfg);
 
 padoc_status check_config(const padoc_decode_config *cfg)
 {
@@ -368,9 +370,9 @@ padoc_status streams_of_chunks(const int32_t *page_len, int32_t num_pages, const
 padoc_status build_work(int32_t num_pages, const padoc_decode_config *cfg, PlanParts &pp)
 {
     const int32_t bs = cfg->block_size;
-    const int32_t split = std::min(cfg->split_tokens > 0 ? cfg->split_tokens : PADOC_DEFAULT_SPLIT_TOKENS,
-                                   PADOC_WARP_MAX_ITEM_TOKENS);
-    const int32_t psplit = PADOC_PRIVATE_SPLIT_TOKENS;
+    const int32_t auto_split = cfg->split_tokens > 0 ? 0 : warp_split_tokens(pp, cfg);
+    const int32_t split = cfg->split_tokens > 0 ? std::min(cfg->split_tokens, PADOC_WARP_MAX_ITEM_TOKENS) : auto_split;
+    const int32_t psplit = cfg->split_tokens > 0 ? PADOC_PRIVATE_SPLIT_TOKENS : auto_split;
     const int32_t group = cfg->num_q_heads / cfg->num_kv_heads;
 
     for (int32_t p = 0; p < num_pages; ++p) {
@@ -500,7 +502,7 @@ padoc_status build_work(int32_t num_pages, const padoc_decode_config *cfg, PlanP
     };
     int32_t ctas = 0;
     if (!segs.empty()) {
-        const int64_t want = cfg->tc_ctas > 0 ? cfg->tc_ctas : choose_tc_ctas(pp, cfg, total_w, max_piece);
+        const int64_t want = cfg->tc_ctas > 0 ? cfg->tc_ctas : choose_tc_ctas(pp, cfg, total_w, max_piece, split, psplit);
         // Every CTA's load stays within T (T >= max_w + max_piece), so T below total_w / want needs
         // more than `want` CTAs: that is a lower bound. A CTA is closed only once less than a piece
         // and a tile fit, and cutting adds at most one piece per CTA, so T = total_w / (want - 1) +
@@ -722,12 +724,36 @@ padoc_status build_work(int32_t num_pages, const padoc_decode_config *cfg, PlanP
 // PADOC_TC_END_SPREAD_US later, and the warp work, sized to each warp's start as in the planner
 // (warp CTAs that follow a tensor-core CTA's pieces start at the average end), ends at T; the count whose
 // later of the two ends is earliest wins (the larger count on a tie).
-int32_t choose_tc_ctas(const PlanParts &pp, const padoc_decode_config *cfg, int64_t total_w, int64_t max_piece)
+// Tokens per warp item when the caller leaves the split to the planner (shared-stream and private
+// items alike): PADOC_DEFAULT_SPLIT_TOKENS, or shorter items when the warp work is small against the
+// warp grid. A step of a decoding loop with few live streams is latency-bound: its time is the
+// longest item's chain of 16-token blocks (each warp keeps three in flight) plus the merge, so
+// shorter items (more partials to merge) finish sooner once there are fewer than
+// PADOC_SPLIT_128_BLOCKS (PADOC_SPLIT_64_BLOCKS) 16-token blocks of warp work per warp (measured on
+// GB300 over the serving batch's decoding loop: 20.2 -> 15.2 us per step at 1-2 live streams, 21.4
+// -> 19.3 us at 17, while steps of 70 or more streams are fastest with 256).
+int32_t warp_split_tokens(const PlanParts &pp, const padoc_decode_config *cfg)
+{
+    const int32_t group = cfg->num_q_heads / cfg->num_kv_heads, bs = cfg->block_size;
+    int64_t blocks = 0;   // per KV head: sparse pages' shared rows of every stream, every private row
+    for (size_t p = 0; p < pp.page_len.size(); ++p) {
+        const int32_t f0 = pp.page_first_stream[p], ns = pp.page_num_streams[p];
+        if ((int64_t)ns * group >= PADOC_TC_MIN_ROWS) continue;
+        for (int32_t st = f0; st < f0 + ns; ++st) blocks += (pp.streams[(size_t)st].shared_len + bs - 1) / bs;
+    }
+    for (const PlanStream &st : pp.streams) blocks += (st.private_len + bs - 1) / bs;
+    blocks *= cfg->num_kv_heads;
+    const int64_t warps = (int64_t)(cfg->warp_ctas > 0 ? cfg->warp_ctas : padoc_default_ctas()) * PADOC_WARP_KERNEL_WARPS;
+    if (blocks < PADOC_SPLIT_64_BLOCKS * warps) return 64;
+    if (blocks < PADOC_SPLIT_128_BLOCKS * warps) return 128;
+    return PADOC_DEFAULT_SPLIT_TOKENS;
+}
+
+int32_t choose_tc_ctas(const PlanParts &pp, const padoc_decode_config *cfg, int64_t total_w, int64_t max_piece,
+                       int32_t split, int32_t psplit)
 {
     const int32_t nsm = padoc_default_ctas();
     const int32_t group = cfg->num_q_heads / cfg->num_kv_heads;
-    const int32_t split = std::min(cfg->split_tokens > 0 ? cfg->split_tokens : PADOC_DEFAULT_SPLIT_TOKENS,
-                                   PADOC_WARP_MAX_ITEM_TOKENS);
     // the warp work: its items and their cost, as the planner will cut them
     int64_t wcost = 0, witems = 0;
     auto add = [&](int32_t len, int32_t step) {
@@ -742,7 +768,7 @@ int32_t choose_tc_ctas(const PlanParts &pp, const padoc_decode_config *cfg, int6
             if ((int64_t)ns * group >= PADOC_TC_MIN_ROWS) continue;
             for (int32_t st = f0; st < f0 + ns; ++st) add(pp.streams[(size_t)st].shared_len, split);
         }
-        for (const PlanStream &st : pp.streams) add(st.private_len, PADOC_PRIVATE_SPLIT_TOKENS);
+        for (const PlanStream &st : pp.streams) add(st.private_len, psplit);
     }
     const int64_t wctas = std::min<int64_t>(cfg->warp_ctas > 0 ? cfg->warp_ctas : nsm,
                                             (witems + PADOC_WARP_KERNEL_WARPS - 1) / PADOC_WARP_KERNEL_WARPS);

@@ -33,6 +33,14 @@
 // Longest warp item: a warp keeps one block id per lane, so an item spans at most 32 blocks.
 #define PADOC_WARP_MAX_ITEM_TOKENS 512
 #define PADOC_PRIVATE_SPLIT_TOKENS 256
+// The planner's own split (split_tokens 0) is 64 tokens below this many 16-token blocks of warp work
+// per warp of the grid and 128 below the next; 256 above.
+#ifndef PADOC_SPLIT_64_BLOCKS
+#define PADOC_SPLIT_64_BLOCKS 3
+#endif
+#ifndef PADOC_SPLIT_128_BLOCKS
+#define PADOC_SPLIT_128_BLOCKS 8
+#endif
 // Shared-stream rows (streams x query heads of one KV head) from which the tensor-core kernel
 // takes a page: below this the rows are too few for a dense M = 128 contraction and each stream
 // reads the shared stream with warp-level MMAs instead.

@@ -439,3 +439,39 @@ def test_advance_decode_plan_refuses_and_changes_nothing():
         assert bytes(info) == info0
     with pytest.raises(pa.PadocError):
         pa.padoc_advance_decode_plan(plan, info, pl[:-1])           # a wrong stream count
+
+
+def _warp_item_cuts(plan, info):
+    items = _plan_items(plan, info)[info.num_tc_items:]
+    sh = {(k & 15, tb, te) for k, _, _, tb, te, *_ in items}
+    return items, sh
+
+
+@pytest.mark.parametrize("warp_ctas", [0, 2])
+def test_planner_split_follows_warp_work(warp_ctas):
+    """split_tokens 0: the warp items (shared and private) are cut every 64 tokens when the warp work
+    is under 3 16-token blocks per warp of the grid, every 128 under 8, else every 256; an explicit
+    split_tokens cuts the shared rows at it and private rows at 256."""
+    def cuts(pages, split):
+        wl = inputs.Workload("split", pages, 16, 2, 128, None, "decode")
+        cfg = pa.make_decode_config(16, 2, 128, 16, False, split, 0, warp_ctas)
+        plan, info = pa.padoc_build_decode_plan(wl.pages, cfg)
+        items = _plan_items(plan, info)[info.num_tc_items:]
+        sp, sh, pl = oracle.decode_streams(wl.pages, False)
+        blocks = 2 * sum(-(-int(sh[s]) // 16) + -(-int(pl[s]) // 16) for s in range(len(sp)))   # no tensor-core page
+        return items, blocks
+    warps = (warp_ctas or 152) * 8
+    seen = set()
+    for pages in ([PageSpec(200, 0, [0], [100])], [PageSpec(600, 0, [0], [300])],
+                  [PageSpec(700, 0, [0, 0], [300, 1000])], [PageSpec(3000, 0, [0] * 5, [900] * 5)] * 3,
+                  [PageSpec(3000, 0, [0] * 5, [900] * 5)] * 6, [PageSpec(4000, 0, [0] * 7, [2000] * 7)] * 40):
+        items, blocks = cuts(pages, 0)
+        want = 64 if blocks < 3 * warps else 128 if blocks < 8 * warps else 256
+        seen.add(want)
+        for kind, idx, g, tb, te, *_ in items:
+            assert tb % want == 0 and te - tb <= want
+        assert max(te - tb for _, _, _, tb, te, *_ in items) == want
+        items, _ = cuts(pages, 512)
+        for kind, idx, g, tb, te, *_ in items:
+            assert (tb % 512 == 0 and te - tb <= 512) if kind == 0 else (tb % 256 == 0 and te - tb <= 256)
+    assert seen == {64, 128, 256}
