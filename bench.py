@@ -658,11 +658,13 @@ def bench_loop(args, torch, dev, rank, world):
         nbytes += (shared + int(pl.sum())) * Hkv * d * 4 + S * Hq * d * 4 + S * Hq * 4
         nbytes += S * Hkv * d * 4 + S * Hq * d * 4
 
-    # (b) the recorded steps' ints in one device buffer, their launches captured in a CUDA graph
+    # (b) the recorded steps' ints in one device buffer (each step's words from a 256-byte boundary),
+    # their launches (padoc_mpd_launch_step with the words already on the device: the append, then the
+    # decode behind it) captured in a CUDA graph
     offs, n = [], 0
     for host, stp in rec:
         offs.append(n)
-        n += (host.size + 31) // 32 * 32
+        n += (host.size + 63) // 64 * 64
     allh = np.zeros(max(n, 1), np.int32)
     for (host, stp), o in zip(rec, offs):
         allh[o:o + host.size] = host
@@ -675,21 +677,12 @@ def bench_loop(args, torch, dev, rank, world):
     lse = torch.empty((cmax, Hq), dtype=torch.float32, device=dev)
     _, loop0 = admit_all()   # a fresh pool holding the prefixes, as at the loop's start
     torch.cuda.synchronize()
-    views = []
-    for (host, stp), o in zip(rec, offs):
-        C = int(stp.num_streams)
-        v_ = lambda a, m: ints[o + a:o + a + m]
-        views.append((stp.plan, C, v_(stp.off_plan, int(stp.plan.plan_ints)),
-                      v_(stp.off_page_table, stp.num_pages * stp.page_stride).view(stp.num_pages, stp.page_stride),
-                      v_(stp.off_stream_table, C * stp.stream_stride).view(C, stp.stream_stride),
-                      v_(stp.off_slots, C), v_(stp.off_rows, C)))
+    views = [(stp, ints[o:o + int(stp.upload_words)]) for (host, stp), o in zip(rec, offs)]
+    pool0 = pa.make_kv_pool(loop0.k_pool, loop0.v_pool)
 
     def replay(s):
-        for info, C, plan_d, pt_d, st_d, slots_d, rows_d in views:
-            pa.padoc_append_inputs(loop0.k_pool, loop0.v_pool, kd, vd, slots_d, q_src=qd, q_dst=q_step[:C],
-                                   src_rows=rows_d, count=C, stream=s)
-            pa.padoc_branch_decode_attn(loop0.k_pool, loop0.v_pool, info, plan_d, pt_d, st_d, q_step[:C], scale,
-                                        out[:C], lse[:C], ws, s)
+        for stp, ints_d in views:
+            pa.padoc_mpd_launch_step(stp, None, ints_d, pool0, kd, vd, qd, q_step, scale, out, lse, ws, s)
 
     replay(stream)
     pa.padoc_check_device_errors(stream)

@@ -567,12 +567,15 @@ padoc_status padoc_mpd_prepare_step(padoc_mpd *mpd, const padoc_decode_config *c
 
 /* Runs a step prepared by padoc_mpd_prepare_step, all on `stream`, with no host synchronization:
  * copies stage[0, step->upload_words) (host; pinned memory makes the copy asynchronous, and the
- * stage must stay unchanged until the copy has run) to dev_ints ((device) int32
- * [dev_capacity_words], 256-byte aligned), appends every input (padoc_append_inputs with the step's
+ * stage must stay unchanged until the copy has run; NULL: dev_ints already holds those words) to
+ * dev_ints ((device) int32 [dev_capacity_words], 256-byte aligned), appends every input (padoc_append_inputs with the step's
  * slots and the source rows the caller wrote at stage[step->off_rows]; k_src / v_src
  * [src_total][Hkv][d], q_src [src_total][Hq][d], q_dst (device) [C][Hq][d] receives the step's
  * queries) and decodes every stream (padoc_branch_decode_attn: out [C][Hq][d], lse fp32 [C][Hq],
- * workspace >= padoc_decode_workspace_size(&step->plan) bytes). Nothing is launched for C = 0.
+ * workspace >= padoc_decode_workspace_size(&step->plan) bytes). The decode is launched behind the
+ * append with programmatic dependent launch, and its warps without tensor-core work read the plan,
+ * the block tables and the paged blocks that hold no stream's newest row before they wait for the
+ * append. Nothing is launched for C = 0.
  * Errors: INVALID_ARGUMENT (also dev_capacity_words < upload_words), UNSUPPORTED,
  * WORKSPACE_TOO_SMALL, CUDA. */
 padoc_status padoc_mpd_launch_step(const padoc_mpd_step *step, const int32_t *stage, int32_t *dev_ints,

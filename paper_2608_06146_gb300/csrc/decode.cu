@@ -11,11 +11,13 @@
 // the rest start on the warp lists at once; for the E4M3 pool the warp lists run in a grid of their
 // own. A split-K merge then joins each (stream, head)'s partials.
 #include <math.h>
+#include <stddef.h>
 
 #include <mutex>
 
 #include "common.cuh"
 #include "decode_warp.cuh"
+#include "plan_build.h"
 
 namespace {
 
@@ -99,6 +101,20 @@ __device__ __forceinline__ void merge_slots(const float *bo, const float *bl, in
     }
 }
 
+// Joins state o into ms (both over disjoint sets of partials, each with its own reference).
+__device__ __forceinline__ void merge_join(MergeState &ms, const MergeState &o)
+{
+    if (o.mref == -INFINITY) return;   // that state saw no partial with weight
+    const float m = fmaxf(ms.mref, o.mref);
+    const float a = ms.mref == -INFINITY ? 0.f : expf(ms.mref - m), b = expf(o.mref - m);
+    ms.ssum = ms.ssum * a + o.ssum * b;
+    ms.acc0.x = ms.acc0.x * a + o.acc0.x * b; ms.acc0.y = ms.acc0.y * a + o.acc0.y * b;
+    ms.acc0.z = ms.acc0.z * a + o.acc0.z * b; ms.acc0.w = ms.acc0.w * a + o.acc0.w * b;
+    ms.acc1.x = ms.acc1.x * a + o.acc1.x * b; ms.acc1.y = ms.acc1.y * a + o.acc1.y * b;
+    ms.acc1.z = ms.acc1.z * a + o.acc1.z * b; ms.acc1.w = ms.acc1.w * a + o.acc1.w * b;
+    ms.mref = m;
+}
+
 __device__ __forceinline__ void merge_store(const MergeState &ms, int key, int h, int part, __nv_bfloat16 *out,
                                             float *lse_out)
 {
@@ -136,16 +152,17 @@ __global__ void __launch_bounds__(128, 9) decode_combine_kernel(const int32_t *_
     merge_store(ms, key, h, part, out, lse_out);
 }
 
-// The merge for steps with few keys and many partials each (a decoding loop's small steps): four
-// groups of 128 threads share a key, group q taking the blocks of four slots q, q + 4, ..., and
-// group 0 joins the four running states through shared memory. Launched instead of
-// decode_combine_kernel when the keys fit in one wave of these CTAs.
-constexpr int kWideGroups = 4;
-template <bool kIndexed>
-__global__ void __launch_bounds__(128 * kWideGroups, 2) decode_combine_wide_kernel(
+// The merge for steps with few keys and many partials each (a decoding loop's small steps): kGroups
+// groups of 128 threads share a key, group q taking the blocks of four slots q, q + kGroups, ...,
+// and group 0 joins the running states through shared memory. Launched instead of
+// decode_combine_kernel for keys of more than 8 partials when the keys fit in one wave of these CTAs
+// (two per SM) and the cluster merge below is not taken.
+template <bool kIndexed, int kGroups>
+__global__ void __launch_bounds__(128 * kGroups, 8 / kGroups) decode_combine_wide_kernel(
     const int32_t *__restrict__ slot_ptr, const int32_t *__restrict__ merge_keys, const float *__restrict__ part_o,
     const float *__restrict__ part_lse, __nv_bfloat16 *__restrict__ out, float *__restrict__ lse_out)
 {
+    constexpr int kWideGroups = kGroups;
     const int key = kIndexed ? merge_keys[blockIdx.x] : (int)blockIdx.x;
     const int p0 = slot_ptr[key], n = slot_ptr[key + 1] - p0;
     pdl_wait_prerequisite();
@@ -161,19 +178,84 @@ __global__ void __launch_bounds__(128 * kWideGroups, 2) decode_combine_wide_kern
     __syncthreads();
     if (q > 0) return;
 #pragma unroll
-    for (int k = 0; k < kWideGroups - 1; ++k) {
-        const MergeState o = st[k][tid];
-        if (o.mref == -INFINITY) continue;   // that group saw no partial with weight
-        const float m = fmaxf(ms.mref, o.mref);
-        const float a = ms.mref == -INFINITY ? 0.f : expf(ms.mref - m), b = expf(o.mref - m);
-        ms.ssum = ms.ssum * a + o.ssum * b;
-        ms.acc0.x = ms.acc0.x * a + o.acc0.x * b; ms.acc0.y = ms.acc0.y * a + o.acc0.y * b;
-        ms.acc0.z = ms.acc0.z * a + o.acc0.z * b; ms.acc0.w = ms.acc0.w * a + o.acc0.w * b;
-        ms.acc1.x = ms.acc1.x * a + o.acc1.x * b; ms.acc1.y = ms.acc1.y * a + o.acc1.y * b;
-        ms.acc1.z = ms.acc1.z * a + o.acc1.z * b; ms.acc1.w = ms.acc1.w * a + o.acc1.w * b;
-        ms.mref = m;
-    }
+    for (int k = 0; k < kWideGroups - 1; ++k) merge_join(ms, st[k][tid]);
     merge_store(ms, key, h, part, out, lse_out);
+}
+
+// The merge for keys with very many partials (a decoding loop's small steps cut into short items):
+// one thread-block cluster of kMergeCluster CTAs per key, so that the key's partials are read by as
+// many SMs. Group q of CTA r takes the blocks of four slots r + kMergeCluster q, then every
+// 4 kMergeCluster-th block; each CTA joins its four groups in shared memory, and CTA 0 joins the
+// CTAs' states through distributed shared memory and writes the key's outputs. Two cluster
+// barriers: the CTAs' states are complete before CTA 0 reads them, and stay until it has.
+constexpr int kMergeCluster = 8;
+#ifndef PADOC_MERGE_CLUSTER_MAX_KEYS
+#define PADOC_MERGE_CLUSTER_MAX_KEYS 8
+#endif
+
+__device__ __forceinline__ uint32_t cluster_ctarank()
+{
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+    return r;
+}
+
+__device__ __forceinline__ void cluster_barrier()
+{
+    asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
+// The state at shared address `addr` of cluster CTA `rank`.
+__device__ __forceinline__ MergeState load_remote_state(uint32_t addr, uint32_t rank)
+{
+    uint32_t ra;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(ra) : "r"(addr), "r"(rank));
+    MergeState o;
+    asm volatile("ld.shared::cluster.v2.f32 {%0, %1}, [%2];" : "=f"(o.mref), "=f"(o.ssum) : "r"(ra) : "memory");
+    asm volatile("ld.shared::cluster.v4.f32 {%0, %1, %2, %3}, [%4];"
+                 : "=f"(o.acc0.x), "=f"(o.acc0.y), "=f"(o.acc0.z), "=f"(o.acc0.w)
+                 : "r"(ra + (uint32_t)offsetof(MergeState, acc0))
+                 : "memory");
+    asm volatile("ld.shared::cluster.v4.f32 {%0, %1, %2, %3}, [%4];"
+                 : "=f"(o.acc1.x), "=f"(o.acc1.y), "=f"(o.acc1.z), "=f"(o.acc1.w)
+                 : "r"(ra + (uint32_t)offsetof(MergeState, acc1))
+                 : "memory");
+    return o;
+}
+
+template <bool kIndexed>
+__global__ void __launch_bounds__(512, 2) decode_combine_cluster_kernel(
+    const int32_t *__restrict__ slot_ptr, const int32_t *__restrict__ merge_keys, const float *__restrict__ part_o,
+    const float *__restrict__ part_lse, __nv_bfloat16 *__restrict__ out, float *__restrict__ lse_out)
+{
+    const uint32_t rank = cluster_ctarank();
+    const int kidx = (int)(blockIdx.x / kMergeCluster);
+    const int key = kIndexed ? merge_keys[kidx] : kidx;
+    const int p0 = slot_ptr[key], n = slot_ptr[key + 1] - p0;
+    pdl_wait_prerequisite();
+    pdl_launch_dependents();
+    const int tid = threadIdx.x & 127, q = threadIdx.x >> 7;
+    const int h = tid & 7, part = tid >> 3;
+    const float *bo = part_o + (size_t)p0 * kGroup * kD + (part * kGroup + h) * 8;
+    const float *bl = part_lse + (size_t)p0 * kGroup + h;
+    MergeState ms;
+    merge_slots(bo, bl, n, (int)rank + kMergeCluster * q, 4 * kMergeCluster, ms);
+    __shared__ MergeState st[4][128];
+    st[q][tid] = ms;
+    __syncthreads();
+    if (q == 0) {
+#pragma unroll
+        for (int k = 1; k < 4; ++k) merge_join(ms, st[k][tid]);
+        st[0][tid] = ms;
+    }
+    cluster_barrier();
+    if (rank == 0 && q == 0) {
+        const uint32_t addr = smem_u32(&st[0][tid]);
+#pragma unroll 1
+        for (uint32_t r = 1; r < (uint32_t)kMergeCluster; ++r) merge_join(ms, load_remote_state(addr, r));
+        merge_store(ms, key, h, part, out, lse_out);
+    }
+    cluster_barrier();
 }
 
 template <class Slots, class OutT>
@@ -297,7 +379,8 @@ struct DecodePool {
 padoc_status decode_split_k(const DecodePool &pl, const padoc_decode_plan *info, const int32_t *plan,
                             const int32_t *page_block_table, int32_t page_table_stride,
                             const int32_t *stream_block_table, int32_t stream_table_stride, const void *q, float scale,
-                            void *out, float *lse, void *workspace, size_t workspace_bytes, cudaStream_t cs)
+                            void *out, float *lse, void *workspace, size_t workspace_bytes, cudaStream_t cs,
+                            bool after_append = false)
 {
     const padoc_decode_config &cfg = info->cfg;
     if (cfg.head_dim != kD || cfg.num_q_heads != kGroup * cfg.num_kv_heads || cfg.block_size != kBlk)
@@ -337,6 +420,8 @@ padoc_status decode_split_k(const DecodePool &pl, const padoc_decode_plan *info,
     prm.shared_len = plan + info->off_shared_len;
     prm.private_len = plan + info->off_private_len;
     prm.slot_ptr = plan + info->off_slot_ptr;
+    prm.page_len = plan + info->off_page_len;
+    prm.pre_wait = after_append && !pl.e4m3 ? 1 : 0;
     prm.items = reinterpret_cast<const padoc_item *>(plan + info->off_items);
     prm.first_item = info->num_tc_items;
     prm.warp_ptr = plan + info->off_warp_ptr;
@@ -396,11 +481,28 @@ padoc_status decode_split_k(const DecodePool &pl, const padoc_decode_plan *info,
         lc.attrs = attr;
         lc.numAttrs = 1;
         const bool all_keys = (int64_t)info->num_merge_keys == (int64_t)info->num_streams * cfg.num_kv_heads;
-        // few keys with many partials each: four thread groups per key, in one wave (two CTAs per SM)
-        const bool wide = info->max_stream_slots > 8 && info->num_merge_keys <= 2 * padoc_default_ctas();
-        if (wide) lc.blockDim = dim3(128 * kWideGroups);
-        auto kern = wide ? (all_keys ? decode_combine_wide_kernel<false> : decode_combine_wide_kernel<true>)
-                         : (all_keys ? decode_combine_kernel<false> : decode_combine_kernel<true>);
+        // few keys with many partials each: four or eight thread groups per key, in one wave
+        const int sms = padoc_default_ctas();
+        // very many partials per key and few keys: a cluster of CTAs per key
+        const bool clustered = info->max_stream_slots > 32 && info->num_merge_keys <= PADOC_MERGE_CLUSTER_MAX_KEYS;
+        const bool wide = !clustered && info->max_stream_slots > 8 && info->num_merge_keys <= 2 * sms;
+        cudaLaunchAttribute cattr[2];
+        if (clustered) {
+            lc.gridDim = dim3((unsigned)(info->num_merge_keys * kMergeCluster));
+            lc.blockDim = dim3(512);
+            cattr[0] = attr[0];
+            cattr[1].id = cudaLaunchAttributeClusterDimension;
+            cattr[1].val.clusterDim.x = kMergeCluster;
+            cattr[1].val.clusterDim.y = 1;
+            cattr[1].val.clusterDim.z = 1;
+            lc.attrs = cattr;
+            lc.numAttrs = 2;
+        } else if (wide) {
+            lc.blockDim = dim3(512);
+        }
+        auto kern = clustered ? (all_keys ? decode_combine_cluster_kernel<false> : decode_combine_cluster_kernel<true>)
+                    : wide    ? (all_keys ? decode_combine_wide_kernel<false, 4> : decode_combine_wide_kernel<true, 4>)
+                              : (all_keys ? decode_combine_kernel<false> : decode_combine_kernel<true>);
         PADOC_CUDA_TRY(cudaLaunchKernelEx(&lc, kern, prm.slot_ptr, (const int32_t *)(plan + info->off_merge_keys),
                                           (const float *)part_o, (const float *)part_lse, (__nv_bfloat16 *)out, lse));
     }
@@ -413,12 +515,13 @@ padoc_status decode_split_k(const DecodePool &pl, const padoc_decode_plan *info,
 // Host entry points
 // ------------------------------------------------------------------------------------------------
 
-extern "C" padoc_status padoc_branch_decode_attn(const padoc_kv_pool *pool, const padoc_decode_plan *info,
-                                                 const int32_t *plan_dev, const int32_t *page_block_table,
-                                                 int32_t page_table_stride, const int32_t *stream_block_table,
-                                                 int32_t stream_table_stride, const void *q, float scale, void *out,
-                                                 float *lse, void *workspace, size_t workspace_bytes,
-                                                 padoc_stream_t stream)
+namespace {
+
+padoc_status branch_decode(const padoc_kv_pool *pool, const padoc_decode_plan *info, const int32_t *plan_dev,
+                           const int32_t *page_block_table, int32_t page_table_stride,
+                           const int32_t *stream_block_table, int32_t stream_table_stride, const void *q, float scale,
+                           void *out, float *lse, void *workspace, size_t workspace_bytes, padoc_stream_t stream,
+                           bool after_append)
 {
     if (!pool || !info || !plan_dev || !q || !out || !lse) return PADOC_ERR_INVALID_ARGUMENT;
     const padoc_decode_config &cfg = info->cfg;
@@ -456,7 +559,31 @@ extern "C" padoc_status padoc_branch_decode_attn(const padoc_kv_pool *pool, cons
     if (pool->dtype != PADOC_DTYPE_BF16) return PADOC_ERR_UNSUPPORTED;
     const DecodePool dp{false, pool->k_pool, pool->v_pool, nullptr, nullptr, pool->num_blocks};
     return decode_split_k(dp, info, plan, page_block_table, page_table_stride, stream_block_table, stream_table_stride,
-                          q, scale, out, lse, workspace, workspace_bytes, cs);
+                          q, scale, out, lse, workspace, workspace_bytes, cs, after_append);
+}
+
+}  // namespace
+
+extern "C" padoc_status padoc_branch_decode_attn(const padoc_kv_pool *pool, const padoc_decode_plan *info,
+                                                 const int32_t *plan_dev, const int32_t *page_block_table,
+                                                 int32_t page_table_stride, const int32_t *stream_block_table,
+                                                 int32_t stream_table_stride, const void *q, float scale, void *out,
+                                                 float *lse, void *workspace, size_t workspace_bytes,
+                                                 padoc_stream_t stream)
+{
+    return branch_decode(pool, info, plan_dev, page_block_table, page_table_stride, stream_block_table,
+                         stream_table_stride, q, scale, out, lse, workspace, workspace_bytes, stream, false);
+}
+
+padoc_status padoc_branch_decode_attn_after_append(const padoc_kv_pool *pool, const padoc_decode_plan *info,
+                                                   const int32_t *plan_dev, const int32_t *page_block_table,
+                                                   int32_t page_table_stride, const int32_t *stream_block_table,
+                                                   int32_t stream_table_stride, const void *q, float scale, void *out,
+                                                   float *lse, void *workspace, size_t workspace_bytes,
+                                                   padoc_stream_t stream)
+{
+    return branch_decode(pool, info, plan_dev, page_block_table, page_table_stride, stream_block_table,
+                         stream_table_stride, q, scale, out, lse, workspace, workspace_bytes, stream, true);
 }
 
 extern "C" padoc_status padoc_branch_decode_attn_e4m3(const padoc_kv_pool_e4m3 *pool, const padoc_decode_plan *info,

@@ -823,8 +823,9 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
     }
     if (has_tc) {
         decode_tc_role<kE4M3, true, kSole>(kmap, vmap, qmap, prm, wprm, smem);
-    } else {
-        // a CTA with warp lists only: the same wait for the previous kernel in the stream
+    } else if (!wprm.pre_wait) {
+        // a CTA with warp lists only: the same wait for the previous kernel in the stream (with
+        // pre_wait each warp of the warp path waits itself, after its first loads)
         pdl_wait_prerequisite();
         pdl_launch_dependents();
     }
@@ -840,7 +841,7 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
     // the rings reuse shared memory that the tensor cores and TMA (the async proxy) last accessed
     fence_proxy_async_smem();
     const int wi = wc * padoc_warp::kWarps + warp;
-    if (wi < wprm.num_warps) padoc_warp::decode_warp_role<kE4M3>(wprm, smem, warp, lane, wi);
+    if (wi < wprm.num_warps) padoc_warp::decode_warp_role<kE4M3>(wprm, smem, warp, lane, wi, has_tc || !wprm.pre_wait);
 }
 
 }  // namespace

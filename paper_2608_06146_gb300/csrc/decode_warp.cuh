@@ -42,6 +42,12 @@ static_assert(PADOC_E4M3_BF16_SHIFT_LOG2 == 112, "expansion factor");
 
 struct DecodeParams {
     const int32_t *stream_page, *shared_len, *private_len, *slot_ptr;
+    const int32_t *page_len;     // each page's shared-stream length (the plan's)
+    // 1: the previous kernel in the stream is this step's append (padoc_mpd_launch_step), which
+    // writes only each stream's newest row and the step's queries: warps of CTAs without
+    // tensor-core work read their headers and block ids and start their first blocks (those
+    // without a newest row) before they wait for it
+    int32_t pre_wait;
     const padoc_item *items;
     int32_t first_item;          // warp items start here
     const int32_t *warp_ptr;     // warp w owns warp items [warp_ptr[w], warp_ptr[w+1])
@@ -61,8 +67,11 @@ struct DecodeParams {
 
 // One warp of the warp path: warp `warp` of its CTA (its ring starts at smem + warp x the ring
 // size; smem is 1024-byte aligned) runs warp list wi < prm.num_warps, whole warp, no CTA barrier.
+// waited: the CTA has already waited for the previous kernel in the stream; otherwise (prm.pre_wait)
+// the warp waits itself once its first safe blocks are on the way.
 template <bool kE4M3>
-__device__ __forceinline__ void decode_warp_role(const DecodeParams &prm, uint8_t *smem, int warp, int lane, int wi)
+__device__ __forceinline__ void decode_warp_role(const DecodeParams &prm, uint8_t *smem, int warp, int lane, int wi,
+                                                 bool waited = true)
 {
     uint8_t *wbuf = smem + (size_t)warp * (kE4M3 ? kE8WarpBytes : kWarpRing);
     uint8_t *cbuf = wbuf + kWStages * kE8StageBytes;   // E4M3: the expanded bf16 block
@@ -151,7 +160,22 @@ __device__ __forceinline__ void decode_warp_role(const DecodeParams &prm, uint8_
         }
         cp_async_commit();
     };
-    for (int k = 0; k < kWStages; ++k) issue_next();
+    int pre = 0;
+    if (!waited) {
+        // Before the wait: the first item's blocks ahead of the block holding its stream's newest
+        // row (page_len - 1 of a shared item's page, private_len - 1 of a private item's stream),
+        // which the append may be writing; everything read so far (plan, block tables) was copied
+        // before the append started.
+        if (i0 < i1) {
+            const padoc_item it0 = load_item(i0);
+            const int32_t len = it0.kind == PADOC_ITEM_SHARED ? prm.page_len[it0.index] : prm.private_len[it0.first_stream];
+            pre = min(min(kWStages, pc.nblk), max(0, (len - 1) / kBlk - pc.blk0));
+        }
+        for (int k = 0; k < pre; ++k) issue_next();
+        pdl_wait_prerequisite();
+        pdl_launch_dependents();
+    }
+    for (int k = pre; k < kWStages; ++k) issue_next();
 
     // Consumer: header of the next item (ch_n) and of the one after (ch_n2), and the next item's
     // query fragments (B operand Q^T[128 dims x 8 heads]) and first partial row.

@@ -371,7 +371,7 @@ extern "C" padoc_status padoc_mpd_launch_step(const padoc_mpd_step *step, const 
                                               int64_t src_total, void *q_dst, float scale, void *out, float *lse,
                                               void *workspace, size_t workspace_bytes, padoc_stream_t stream)
 {
-    if (!step || !stage || !dev_ints || !pool) return PADOC_ERR_INVALID_ARGUMENT;
+    if (!step || !dev_ints || !pool) return PADOC_ERR_INVALID_ARGUMENT;
     const int32_t C = step->num_streams;
     if (C == 0) return PADOC_OK;
     if (C < 0 || step->upload_words < 0 || dev_capacity_words < step->upload_words || (((uintptr_t)dev_ints) & 255))
@@ -380,13 +380,13 @@ extern "C" padoc_status padoc_mpd_launch_step(const padoc_mpd_step *step, const 
     if (info.num_streams != C || step->off_plan + info.plan_ints > step->upload_words ||
         step->off_rows + C > step->upload_words)
         return PADOC_ERR_INVALID_ARGUMENT;
-    if (cudaMemcpyAsync(dev_ints, stage, (size_t)step->upload_words * sizeof(int32_t), cudaMemcpyHostToDevice,
-                        (cudaStream_t)stream) != cudaSuccess)
+    if (stage && cudaMemcpyAsync(dev_ints, stage, (size_t)step->upload_words * sizeof(int32_t), cudaMemcpyHostToDevice,
+                                 (cudaStream_t)stream) != cudaSuccess)
         return PADOC_ERR_CUDA;
     padoc_status st = padoc_append_inputs(pool, k_src, v_src, q_src, src_total, info.cfg.num_q_heads, q_dst,
                                           dev_ints + step->off_rows, dev_ints + step->off_slots, C, stream);
     if (st != PADOC_OK) return st;
-    return padoc_branch_decode_attn(pool, &info, dev_ints + step->off_plan, dev_ints + step->off_page_table,
+    return padoc_branch_decode_attn_after_append(pool, &info, dev_ints + step->off_plan, dev_ints + step->off_page_table,
                                     step->page_stride, dev_ints + step->off_stream_table, step->stream_stride, q_dst,
                                     scale, out, lse, workspace, workspace_bytes, stream);
 }

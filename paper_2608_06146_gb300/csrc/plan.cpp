@@ -255,7 +255,8 @@ namespace {
 
 int32_t choose_tc_ctas(const PlanParts &pp, const padoc_decode_config *cfg, int64_t total_w, int64_t max_piece,
                        int32_t split, int32_t psplit);
-int32_t warp_split_tokens(const PlanParts &pp, const padoc_decode_config *cfg);
+double warp_blocks_per_warp(const PlanParts &pp, const padoc_decode_config *cfg);
+int32_t warp_split_tokens(double blocks_per_warp);
 
 padoc_status check_config(const padoc_decode_config *cfg)
 {
@@ -370,7 +371,16 @@ padoc_status streams_of_chunks(const int32_t *page_len, int32_t num_pages, const
 padoc_status build_work(int32_t num_pages, const padoc_decode_config *cfg, PlanParts &pp)
 {
     const int32_t bs = cfg->block_size;
-    const int32_t auto_split = cfg->split_tokens > 0 ? 0 : warp_split_tokens(pp, cfg);
+    const bool chunked = !pp.chunk_of.empty();
+    // Pages whose shared stream the tensor cores read (once for all the page's streams): those of at
+    // least PADOC_TC_MIN_ROWS rows (streams x query heads), and in a decode step with much warp work
+    // those of at least PADOC_TC_MIN_ROWS_BUSY: there the warp path, which reads a page's shared
+    // stream once per stream, would read it two to seven times (measured on GB300 over the decoding
+    // loop's steps of 70 to 300 streams: 41.6 -> 31.1 and 33.3 -> 29.3 us per step)
+    const double bpw = warp_blocks_per_warp(pp, cfg);
+    const int32_t min_rows = !chunked && bpw >= PADOC_SPLIT_128_BLOCKS ? PADOC_TC_MIN_ROWS_BUSY : PADOC_TC_MIN_ROWS;
+    pp.tc_min_rows = min_rows;
+    const int32_t auto_split = cfg->split_tokens > 0 ? 0 : warp_split_tokens(bpw);
     const int32_t split = cfg->split_tokens > 0 ? std::min(cfg->split_tokens, PADOC_WARP_MAX_ITEM_TOKENS) : auto_split;
     const int32_t psplit = cfg->split_tokens > 0 ? PADOC_PRIVATE_SPLIT_TOKENS : auto_split;
     const int32_t group = cfg->num_q_heads / cfg->num_kv_heads;
@@ -403,13 +413,12 @@ padoc_status build_work(int32_t num_pages, const padoc_decode_config *cfg, PlanP
         int32_t kind2, p2, vis2, ntiles2;   // the private continuation (ntiles2 = 0: none)
     };
     std::vector<Segment> segs;
-    const bool chunked = !pp.chunk_of.empty();
     std::vector<uint8_t> priv_tc(chunked ? (size_t)S : 0, 0);
     auto weight_of = [](int32_t nb) { return nb > PADOC_TC_ITEM_STREAMS / 2 ? PADOC_TC_WEIGHT_2M : PADOC_TC_WEIGHT_1M; };
     for (int32_t g = 0; g < cfg->num_kv_heads; ++g) {
         for (int32_t p = 0; p < num_pages; ++p) {
             const int32_t f0 = pp.page_first_stream[p], ns = pp.page_num_streams[p];
-            if ((int64_t)ns * group < PADOC_TC_MIN_ROWS) continue;
+            if ((int64_t)ns * group < min_rows) continue;
             for (int32_t r = 0; r < ns;) {
                 int32_t nb = std::min(PADOC_TC_ITEM_STREAMS, ns - r);
                 if (chunked)
@@ -426,7 +435,7 @@ padoc_status build_work(int32_t num_pages, const padoc_decode_config *cfg, PlanP
                 if (chunked) {
                     // a group of a chunk with private rows on the tensor cores continues over them
                     const int32_t c = pp.chunk_of[f0 + r], first = pp.chunk_first[c], len = pp.chunk_len[c];
-                    if (pp.chunk_private[c] && (int64_t)len * group >= PADOC_TC_MIN_ROWS) {
+                    if (pp.chunk_private[c] && (int64_t)len * group >= min_rows) {
                         const int32_t vis2 = pp.streams[f0 + r + nb - 1].private_len;   // increasing within a chunk
                         for (int32_t st = f0 + r; st < f0 + r + nb; ++st) priv_tc[st] = 1;
                         sg.kind2 = PADOC_ITEM_PRIVATE_TC | (nb < len ? PADOC_ITEM_REREAD : 0);
@@ -546,7 +555,7 @@ padoc_status build_work(int32_t num_pages, const padoc_decode_config *cfg, PlanP
         int64_t n = 0;   // exact count, so the list is allocated once
         for (int32_t p = 0; p < num_pages; ++p) {
             const int32_t f0 = pp.page_first_stream[p], ns = pp.page_num_streams[p];
-            if ((int64_t)ns * group >= PADOC_TC_MIN_ROWS) continue;
+            if ((int64_t)ns * group >= min_rows) continue;
             for (int32_t st = f0; st < f0 + ns; ++st) n += (pp.streams[st].shared_len + split - 1) / split;
         }
         for (int32_t st = 0; st < S; ++st) n += (pp.streams[st].private_len + psplit - 1) / psplit + 1;
@@ -555,7 +564,7 @@ padoc_status build_work(int32_t num_pages, const padoc_decode_config *cfg, PlanP
     for (int32_t g = 0; g < Hkv; ++g) {
         for (int32_t p = 0; p < num_pages; ++p) {
             const int32_t f0 = pp.page_first_stream[p], ns = pp.page_num_streams[p];
-            if ((int64_t)ns * group >= PADOC_TC_MIN_ROWS) continue;
+            if ((int64_t)ns * group >= min_rows) continue;
             for (int32_t st = f0; st < f0 + ns; ++st)
                 for (int32_t tb = 0; tb < pp.streams[st].shared_len; tb += split)
                     warp_items.push_back({PADOC_ITEM_SHARED, p, g, tb, std::min(pp.streams[st].shared_len, tb + split),
@@ -732,7 +741,9 @@ padoc_status build_work(int32_t num_pages, const padoc_decode_config *cfg, PlanP
 // PADOC_SPLIT_128_BLOCKS (PADOC_SPLIT_64_BLOCKS) 16-token blocks of warp work per warp (measured on
 // GB300 over the serving batch's decoding loop: 20.2 -> 15.2 us per step at 1-2 live streams, 21.4
 // -> 19.3 us at 17, while steps of 70 or more streams are fastest with 256).
-int32_t warp_split_tokens(const PlanParts &pp, const padoc_decode_config *cfg)
+// 16-token blocks of warp work per warp of the grid when the pages below PADOC_TC_MIN_ROWS rows
+// (streams x query heads) read their shared streams on the warp path.
+double warp_blocks_per_warp(const PlanParts &pp, const padoc_decode_config *cfg)
 {
     const int32_t group = cfg->num_q_heads / cfg->num_kv_heads, bs = cfg->block_size;
     int64_t blocks = 0;   // per KV head: sparse pages' shared rows of every stream, every private row
@@ -744,8 +755,13 @@ int32_t warp_split_tokens(const PlanParts &pp, const padoc_decode_config *cfg)
     for (const PlanStream &st : pp.streams) blocks += (st.private_len + bs - 1) / bs;
     blocks *= cfg->num_kv_heads;
     const int64_t warps = (int64_t)(cfg->warp_ctas > 0 ? cfg->warp_ctas : padoc_default_ctas()) * PADOC_WARP_KERNEL_WARPS;
-    if (blocks < PADOC_SPLIT_64_BLOCKS * warps) return 64;
-    if (blocks < PADOC_SPLIT_128_BLOCKS * warps) return 128;
+    return (double)blocks / (double)warps;
+}
+
+int32_t warp_split_tokens(double blocks_per_warp)
+{
+    if (blocks_per_warp < PADOC_SPLIT_64_BLOCKS) return 64;
+    if (blocks_per_warp < PADOC_SPLIT_128_BLOCKS) return 128;
     return PADOC_DEFAULT_SPLIT_TOKENS;
 }
 
@@ -765,7 +781,7 @@ int32_t choose_tc_ctas(const PlanParts &pp, const padoc_decode_config *cfg, int6
     for (int32_t g = 0; g < cfg->num_kv_heads; ++g) {
         for (size_t p = 0; p < pp.page_len.size(); ++p) {
             const int32_t f0 = pp.page_first_stream[p], ns = pp.page_num_streams[p];
-            if ((int64_t)ns * group >= PADOC_TC_MIN_ROWS) continue;
+            if ((int64_t)ns * group >= pp.tc_min_rows) continue;
             for (int32_t st = f0; st < f0 + ns; ++st) add(pp.streams[(size_t)st].shared_len, split);
         }
         for (const PlanStream &st : pp.streams) add(st.private_len, psplit);

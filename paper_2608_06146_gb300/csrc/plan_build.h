@@ -20,6 +20,7 @@ struct PlanParts {
     std::vector<int32_t> merge_keys;    // the (stream, KV head) keys the merge joins (the others are written directly)
     std::vector<padoc_item> items;
     int32_t num_tc_items = 0, tc_ctas = 0, num_warps = 0;
+    int32_t tc_min_rows = PADOC_TC_MIN_ROWS;   // rows from which a page's shared stream goes to the tensor cores
     int32_t max_page_blocks = 0, max_stream_blocks = 0;
     int64_t kv_tokens = 0;
     // chunked prefill plans only (empty otherwise): the chunk of each stream, and per chunk its
@@ -39,3 +40,14 @@ int64_t padoc_plan_blob_ints(const PlanParts &pp, int32_t num_pages, int32_t hkv
 // Writes the blob and its host summary (CAPACITY when capacity_ints is too small).
 padoc_status padoc_plan_write_blob(const PlanParts &pp, int32_t num_pages, const padoc_decode_config *cfg, int32_t *plan,
                                    int64_t capacity_ints, padoc_decode_plan *info);
+
+// padoc_branch_decode_attn for a decoding-loop step launched right after that step's append on the
+// same stream (padoc_mpd_launch_step): the append writes only each stream's newest K/V row and the
+// step's queries, and the plan and block tables were copied before it started, so warps without
+// tensor-core work read those and start their first paged blocks before they wait for the append.
+padoc_status padoc_branch_decode_attn_after_append(const padoc_kv_pool *pool, const padoc_decode_plan *info,
+                                                   const int32_t *plan_dev, const int32_t *page_block_table,
+                                                   int32_t page_table_stride, const int32_t *stream_block_table,
+                                                   int32_t stream_table_stride, const void *q, float scale, void *out,
+                                                   float *lse, void *workspace, size_t workspace_bytes,
+                                                   padoc_stream_t stream);

@@ -44,7 +44,14 @@
 // Shared-stream rows (streams x query heads of one KV head) from which the tensor-core kernel
 // takes a page: below this the rows are too few for a dense M = 128 contraction and each stream
 // reads the shared stream with warp-level MMAs instead.
+#ifndef PADOC_TC_MIN_ROWS
 #define PADOC_TC_MIN_ROWS 64
+#endif
+// ... and from this many in a decode plan with much warp work (at least PADOC_SPLIT_128_BLOCKS
+// blocks per warp): two streams of eight query heads
+#ifndef PADOC_TC_MIN_ROWS_BUSY
+#define PADOC_TC_MIN_ROWS_BUSY 16
+#endif
 // Streams per tensor-core work item: two M = 128 tiles of 16 streams x 8 query heads.
 #define PADOC_TC_ITEM_STREAMS 32
 // Tokens per K/V tile of the tensor-core kernel, and the relative cost of one tile for a group of

@@ -729,10 +729,12 @@ class Mpd:
 
 def padoc_mpd_launch_step(step: padoc_mpd_step, stage, dev_ints, pool: padoc_kv_pool, k_src, v_src, q_src, q_dst,
                           scale, out, lse, workspace, stream=None):
-    """stage: pinned int32 CPU tensor holding the prepared step; dev_ints: int32 CUDA tensor; pool: a
-    padoc_kv_pool (make_kv_pool); other tensors as in padoc_append_inputs / padoc_branch_decode_attn."""
+    """stage: pinned int32 CPU tensor holding the prepared step (None: dev_ints already holds it);
+    dev_ints: int32 CUDA tensor; pool: a padoc_kv_pool (make_kv_pool); other tensors as in
+    padoc_append_inputs / padoc_branch_decode_attn."""
     lib = load_library()
-    st = lib.padoc_mpd_launch_step(ctypes.byref(step), stage.data_ptr(), _dev(dev_ints, "dev_ints"), dev_ints.numel(),
+    st = lib.padoc_mpd_launch_step(ctypes.byref(step), None if stage is None else stage.data_ptr(),
+                                   _dev(dev_ints, "dev_ints"), dev_ints.numel(),
                                    ctypes.byref(pool), _dev(k_src, "k_src"), _dev(v_src, "v_src"), _dev(q_src, "q_src"),
                                    k_src.shape[0], _dev(q_dst, "q_dst"), float(scale), _dev(out, "out"),
                                    _dev(lse, "lse"), _dev(workspace, "workspace"),

@@ -148,6 +148,38 @@ def test_decode_bf16_serving_batch_warp_ctas_beyond_the_sm_count():
     assert_close(*run_decode(wl, 13, tc_ctas=5, warp_ctas=400), torch.bfloat16)
 
 
+@pytest.mark.parametrize("prefix,split,merge", [(1000, 64, "wide"), (3000, 64, "cluster"), (4000, 0, "cluster")])
+def test_decode_bf16_many_partials_per_key(prefix, split, merge):
+    """Few streams with long shared streams cut into short items: every (stream, KV head) key has
+    many partials, which the merge joins with four thread groups per key (9 to 32 partials) or a
+    cluster of eight CTAs per key joined through distributed shared memory (more); split 0 is the
+    planner's own choice for so little work (64-token items)."""
+    pages = [PageSpec(prefix, 40, [0, 17, 40], [1500, 33, 260]), PageSpec(prefix // 2, 0, [0, 0], [700, 1])]
+    wl = Workload("many partials", pages, 16, 2, 128, torch.bfloat16, "decode")
+    plan = DecodePlan(wl.pages, 16, 2, 128, DEV, 16, False, split)
+    info = plan.info
+    assert info.num_merge_keys * 8 <= 2 * 152 and (32 < info.max_stream_slots if merge == "cluster" else
+                                                   8 < info.max_stream_slots <= 32)
+    assert_close(*run_decode(wl, 21, split_tokens=split), torch.bfloat16)
+
+
+def test_decode_bf16_sparse_pages_on_tensor_cores():
+    """Pages of two to seven streams whose plan has much warp work (few warp CTAs): their shared
+    streams go to the tensor cores, one M-tile of 16 stream slots per group, mostly empty rows."""
+    rng = np.random.default_rng(5)
+    pages = []
+    for n in (2, 3, 5, 7, 2):
+        L = int(rng.integers(0, 60))
+        pages.append(PageSpec(int(rng.integers(300, 1500)), L, [int(x) for x in rng.integers(0, L + 1, n)],
+                              [int(x) for x in rng.integers(1, 400, n)]))
+    wl = Workload("sparse pages", pages, 16, 2, 128, torch.bfloat16, "decode")
+    plan = DecodePlan(wl.pages, 16, 2, 128, DEV, 16, False, 0, 0, 2)
+    items = plan.plan_host[plan.info.off_items:plan.info.off_items + 8 * plan.info.num_tc_items].reshape(-1, 8)
+    assert plan.info.num_tc_items > 0 and {0, 1, 4} <= set(int(i) for i in items[:, 1])
+    assert_close(*run_decode(wl, 23, warp_ctas=2), torch.bfloat16)
+    assert_close(*run_decode(wl, 24, layout_streams=True, warp_ctas=2), torch.bfloat16)
+
+
 def test_decode_repeated_calls_on_one_workspace():
     # one plan and workspace serve several calls with new inputs; each call is exact
     wl = inputs.serving_batch(num_pages=6)

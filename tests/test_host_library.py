@@ -190,13 +190,20 @@ def check_decode_plan(wl, layout, tc_ctas, warp_ctas):
     assert all(kinds[:ntc] == 2) and not any(kinds[ntc:] == 2)
     assert not np.any(items[:, 0] & 16), "decode plans load every tile evict-first"
     page_streams = np.bincount(sp, minlength=len(wl.pages))
+    # a page's shared stream goes to the tensor cores from 64 rows (streams x 8 query heads), or
+    # from 16 in a plan with much warp work: one threshold for every page of the plan
+    tc_pages = set(int(i) for i in items[:ntc, 1])
+    min_rows = 16 if any(page_streams[p] * 8 < 64 for p in tc_pages) else 64
+    for p in range(len(wl.pages)):
+        if page_streams[p] and any(sh[s] > 0 for s in np.nonzero(sp == p)[0]):
+            assert (p in tc_pages) == (page_streams[p] * 8 >= min_rows), f"page {p}"
     for kind, idx, g, tb, te, fs, ns, slot in items:
         kind &= 15
         assert tb % 16 == 0
         if kind == 2:      # tensor-core piece: whole 128-token tiles of up to 32 streams of a page
-            assert 1 <= ns <= 32 and te > tb and page_streams[idx] * 8 >= 64 and tb % 128 == 0
+            assert 1 <= ns <= 32 and te > tb and page_streams[idx] * 8 >= min_rows and tb % 128 == 0
         elif kind == 0:    # warp item over one stream's view of the shared stream
-            assert ns == 1 and te >= tb and page_streams[idx] * 8 < 64
+            assert ns == 1 and te >= tb and page_streams[idx] * 8 < min_rows
         else:
             assert kind == 1 and ns == 1 and te > tb
         for s in range(fs, fs + ns):

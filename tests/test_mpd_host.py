@@ -288,8 +288,8 @@ def test_prepare_step_equals_granular_calls(seed):
 
 
 def test_launch_step_validates_before_any_device_work(lib):
-    """padoc_mpd_launch_step rejects a device buffer too small for the stage or not 256-byte aligned,
-    and a null stage or pool, before it touches the device (these checks need no GPU)."""
+    """padoc_mpd_launch_step rejects a device buffer too small for the stage, not 256-byte aligned or
+    null, and a null pool, before it touches the device (these checks need no GPU)."""
     import ctypes
     m = pa.Mpd(64)
     m.add_page(40, 2)
@@ -303,7 +303,7 @@ def test_launch_step_validates_before_any_device_work(lib):
         ctypes.byref(st), stage_p, dev, cap, pool_p, 1024, 1024, 1024, 10, 1024, 0.1, 1024, 1024, 1024, 1 << 20, None)
     assert call(sp, 4096, st.upload_words - 1, ctypes.byref(pool)) == 1   # too small
     assert call(sp, 4096 + 4, st.upload_words, ctypes.byref(pool)) == 1   # not 256-byte aligned
-    assert call(None, 4096, st.upload_words, ctypes.byref(pool)) == 1     # no stage
+    assert call(sp, None, st.upload_words, ctypes.byref(pool)) == 1       # no device buffer
     assert call(sp, 4096, st.upload_words, None) == 1                     # no pool
     m.end_step(np.zeros(3, np.int32), np.zeros(3, np.uint8))
 
