@@ -804,8 +804,10 @@ static_assert(padoc_warp::kWarps * 32 == 256, "the warp path runs on warpgroups 
 // CTA's lists on warps 0-7 with the larger register budget (decode_warp.cuh); warps 8-11 give their
 // registers back and end. A plan without tensor-core work runs warp CTAs only. Without kFused the
 // grid runs the tensor-core pieces only (the E4M3 pool, whose warp lists run in a grid of their own:
-// there the warp path needs more registers than the split leaves it).
-template <bool kE4M3, bool kFused, bool kSole>
+// there the warp path needs more registers than the split leaves it). kPreWait: the previous kernel
+// in the stream is the step's append (a decoding loop's step), and the warps of CTAs without
+// tensor-core pieces start their first paged blocks before they wait for it.
+template <bool kE4M3, bool kFused, bool kSole, bool kPreWait>
 __global__ void __launch_bounds__(kThreads, 1)
 decode_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap,
                  const __grid_constant__ CUtensorMap qmap, const TcDecodeParams prm,
@@ -823,9 +825,9 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
     }
     if (has_tc) {
         decode_tc_role<kE4M3, true, kSole>(kmap, vmap, qmap, prm, wprm, smem);
-    } else if (!wprm.pre_wait) {
-        // a CTA with warp lists only: the same wait for the previous kernel in the stream (with
-        // pre_wait each warp of the warp path waits itself, after its first loads)
+    } else if constexpr (!kPreWait) {
+        // a CTA with warp lists only: the same wait for the previous kernel in the stream (kPreWait:
+        // each warp of the warp path waits itself, after its first loads)
         pdl_wait_prerequisite();
         pdl_launch_dependents();
     }
@@ -841,7 +843,11 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
     // the rings reuse shared memory that the tensor cores and TMA (the async proxy) last accessed
     fence_proxy_async_smem();
     const int wi = wc * padoc_warp::kWarps + warp;
-    if (wi < wprm.num_warps) padoc_warp::decode_warp_role<kE4M3>(wprm, smem, warp, lane, wi, has_tc || !wprm.pre_wait);
+    if (wi >= wprm.num_warps) return;
+    if (kPreWait && !has_tc)
+        padoc_warp::decode_warp_role<kE4M3, true>(wprm, smem, warp, lane, wi);
+    else
+        padoc_warp::decode_warp_role<kE4M3, false>(wprm, smem, warp, lane, wi);
 }
 
 }  // namespace
@@ -886,8 +892,12 @@ padoc_status padoc_launch_decode_tc(const CUtensorMap *kmap, const CUtensorMap *
     prm.early_ctas = padoc_fused_early_ctas(prm.tc_ctas, prm.warp_ctas, padoc_default_ctas());
     // plans with sole items (chunked prefill) take the variant that writes their outputs
     const bool sole = (int64_t)info->num_merge_keys < (int64_t)info->num_streams * info->cfg.num_kv_heads;
-    auto kern = e4m3 ? (sole ? decode_tc_kernel<true, false, true> : decode_tc_kernel<true, false, false>)
-                     : (sole ? decode_tc_kernel<false, true, true> : decode_tc_kernel<false, true, false>);
+    // a decoding-loop step right after its append (no sole items): warps of warp-only CTAs load
+    // before they wait
+    const bool pre_wait = fused && wprm->pre_wait && !sole;
+    auto kern = e4m3       ? (sole ? decode_tc_kernel<true, false, true, false> : decode_tc_kernel<true, false, false, false>)
+                : pre_wait ? decode_tc_kernel<false, true, false, true>
+                           : (sole ? decode_tc_kernel<false, true, true, false> : decode_tc_kernel<false, true, false, false>);
     {
         const padoc_status ast = padoc_set_max_smem(reinterpret_cast<const void *>(kern), (int)kSmemBytes);
         if (ast != PADOC_OK) return ast;

@@ -67,11 +67,10 @@ struct DecodeParams {
 
 // One warp of the warp path: warp `warp` of its CTA (its ring starts at smem + warp x the ring
 // size; smem is 1024-byte aligned) runs warp list wi < prm.num_warps, whole warp, no CTA barrier.
-// waited: the CTA has already waited for the previous kernel in the stream; otherwise (prm.pre_wait)
-// the warp waits itself once its first safe blocks are on the way.
-template <bool kE4M3>
-__device__ __forceinline__ void decode_warp_role(const DecodeParams &prm, uint8_t *smem, int warp, int lane, int wi,
-                                                 bool waited = true)
+// kPreWait: the CTA has not waited for the previous kernel in the stream (prm.pre_wait): the warp
+// waits itself once its first safe blocks are on the way.
+template <bool kE4M3, bool kPreWait = false>
+__device__ __forceinline__ void decode_warp_role(const DecodeParams &prm, uint8_t *smem, int warp, int lane, int wi)
 {
     uint8_t *wbuf = smem + (size_t)warp * (kE4M3 ? kE8WarpBytes : kWarpRing);
     uint8_t *cbuf = wbuf + kWStages * kE8StageBytes;   // E4M3: the expanded bf16 block
@@ -161,7 +160,7 @@ __device__ __forceinline__ void decode_warp_role(const DecodeParams &prm, uint8_
         cp_async_commit();
     };
     int pre = 0;
-    if (!waited) {
+    if constexpr (kPreWait) {
         // Before the wait: the first item's blocks ahead of the block holding its stream's newest
         // row (page_len - 1 of a shared item's page, private_len - 1 of a private item's stream),
         // which the append may be writing; everything read so far (plan, block tables) was copied

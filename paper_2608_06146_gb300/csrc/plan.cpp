@@ -255,7 +255,7 @@ namespace {
 
 int32_t choose_tc_ctas(const PlanParts &pp, const padoc_decode_config *cfg, int64_t total_w, int64_t max_piece,
                        int32_t split, int32_t psplit);
-double warp_blocks_per_warp(const PlanParts &pp, const padoc_decode_config *cfg);
+double warp_blocks_per_warp(const PlanParts &pp, const padoc_decode_config *cfg, int32_t min_rows);
 int32_t warp_split_tokens(double blocks_per_warp);
 
 padoc_status check_config(const padoc_decode_config *cfg)
@@ -376,9 +376,9 @@ padoc_status build_work(int32_t num_pages, const padoc_decode_config *cfg, PlanP
     // least PADOC_TC_MIN_ROWS rows (streams x query heads), and in a decode step with much warp work
     // those of at least PADOC_TC_MIN_ROWS_BUSY: there the warp path, which reads a page's shared
     // stream once per stream, would read it two to seven times (measured on GB300 over the decoding
-    // loop's steps of 70 to 300 streams: 41.6 -> 31.1 and 33.3 -> 29.3 us per step)
-    const double bpw = warp_blocks_per_warp(pp, cfg);
-    const int32_t min_rows = !chunked && bpw >= PADOC_SPLIT_128_BLOCKS ? PADOC_TC_MIN_ROWS_BUSY : PADOC_TC_MIN_ROWS;
+    // loop's steps of 200-300 and of about 76 streams: 41.6 -> 31.5 and 33.3 -> 27.1 us per step)
+    const double bpw = warp_blocks_per_warp(pp, cfg, PADOC_TC_MIN_ROWS);
+    const int32_t min_rows = !chunked && bpw >= PADOC_TC_BUSY_BLOCKS ? PADOC_TC_MIN_ROWS_BUSY : PADOC_TC_MIN_ROWS;
     pp.tc_min_rows = min_rows;
     const int32_t auto_split = cfg->split_tokens > 0 ? 0 : warp_split_tokens(bpw);
     const int32_t split = cfg->split_tokens > 0 ? std::min(cfg->split_tokens, PADOC_WARP_MAX_ITEM_TOKENS) : auto_split;
@@ -741,15 +741,15 @@ padoc_status build_work(int32_t num_pages, const padoc_decode_config *cfg, PlanP
 // PADOC_SPLIT_128_BLOCKS (PADOC_SPLIT_64_BLOCKS) 16-token blocks of warp work per warp (measured on
 // GB300 over the serving batch's decoding loop: 20.2 -> 15.2 us per step at 1-2 live streams, 21.4
 // -> 19.3 us at 17, while steps of 70 or more streams are fastest with 256).
-// 16-token blocks of warp work per warp of the grid when the pages below PADOC_TC_MIN_ROWS rows
-// (streams x query heads) read their shared streams on the warp path.
-double warp_blocks_per_warp(const PlanParts &pp, const padoc_decode_config *cfg)
+// 16-token blocks of warp work per warp of the grid when the pages below min_rows rows (streams x
+// query heads) read their shared streams on the warp path.
+double warp_blocks_per_warp(const PlanParts &pp, const padoc_decode_config *cfg, int32_t min_rows)
 {
     const int32_t group = cfg->num_q_heads / cfg->num_kv_heads, bs = cfg->block_size;
     int64_t blocks = 0;   // per KV head: sparse pages' shared rows of every stream, every private row
     for (size_t p = 0; p < pp.page_len.size(); ++p) {
         const int32_t f0 = pp.page_first_stream[p], ns = pp.page_num_streams[p];
-        if ((int64_t)ns * group >= PADOC_TC_MIN_ROWS) continue;
+        if ((int64_t)ns * group >= min_rows) continue;
         for (int32_t st = f0; st < f0 + ns; ++st) blocks += (pp.streams[(size_t)st].shared_len + bs - 1) / bs;
     }
     for (const PlanStream &st : pp.streams) blocks += (st.private_len + bs - 1) / bs;

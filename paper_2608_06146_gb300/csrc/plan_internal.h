@@ -47,10 +47,13 @@
 #ifndef PADOC_TC_MIN_ROWS
 #define PADOC_TC_MIN_ROWS 64
 #endif
-// ... and from this many in a decode plan with much warp work (at least PADOC_SPLIT_128_BLOCKS
-// blocks per warp): two streams of eight query heads
+// ... and from this many in a decode plan with much warp work (at least PADOC_TC_BUSY_BLOCKS
+// 16-token blocks per warp of the grid): two streams of eight query heads
 #ifndef PADOC_TC_MIN_ROWS_BUSY
 #define PADOC_TC_MIN_ROWS_BUSY 16
+#endif
+#ifndef PADOC_TC_BUSY_BLOCKS
+#define PADOC_TC_BUSY_BLOCKS 6
 #endif
 // Streams per tensor-core work item: two M = 128 tiles of 16 streams x 8 query heads.
 #define PADOC_TC_ITEM_STREAMS 32
