@@ -372,7 +372,7 @@ struct DecodeParams;
 padoc_status padoc_launch_decode_tc(const CUtensorMap *kmap, const CUtensorMap *vmap, const CUtensorMap *qmap, const int32_t *plan,
                                     const padoc_decode_plan *info, const int32_t *page_table, int32_t page_stride,
                                     const int32_t *stream_table, int32_t stream_stride, int32_t num_blocks,
-                                    const float *k_scales, const float *v_scales, float *part_o, float *part_lse,
+                                    const float *k_scales, const float *v_scales, __nv_bfloat16 *part_o, float *part_lse,
                                     __nv_bfloat16 *out, float *lse, float scale_log2, int *err,
                                     const padoc_warp::DecodeParams *wprm, cudaStream_t stream);
 // tcgen05 prefill backward (prefill_bwd_tc.cu): the dQ pass, which also writes lt / dt (per head

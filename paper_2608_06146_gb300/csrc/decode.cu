@@ -70,21 +70,24 @@ struct MergeState {
     float mref = -INFINITY, ssum = 0.f;
     float4 acc0 = make_float4(0.f, 0.f, 0.f, 0.f), acc1 = make_float4(0.f, 0.f, 0.f, 0.f);
 };
-__device__ __forceinline__ void merge_slots(const float *bo, const float *bl, int n, int b0, int stride, MergeState &ms)
+// bo: this thread's 8 dims of its head in the key's first slot (bf16 partials, a slot every
+// kGroup * kD values); bl: its head's LSE in the first slot. kPer partials' loads in flight.
+template <int kPer>
+__device__ __forceinline__ void merge_slots(const __nv_bfloat16 *bo, const float *bl, int n, int b0, int stride,
+                                            MergeState &ms)
 {
     constexpr size_t kSlotO = (size_t)kGroup * kD;
-    for (int i = 4 * b0; i < n; i += 4 * stride) {
-        float li[4];
-        float4 v0[4], v1[4];
+    for (int i = kPer * b0; i < n; i += kPer * stride) {
+        float li[kPer];
+        uint4 v[kPer];
 #pragma unroll
-        for (int u = 0; u < 4; ++u) {
+        for (int u = 0; u < kPer; ++u) {
             const bool in = i + u < n;
             li[u] = in ? bl[(size_t)(i + u) * kGroup] : -INFINITY;
-            v0[u] = in ? *reinterpret_cast<const float4 *>(bo + (i + u) * kSlotO) : make_float4(0.f, 0.f, 0.f, 0.f);
-            v1[u] = in ? *reinterpret_cast<const float4 *>(bo + (i + u) * kSlotO + 4) : make_float4(0.f, 0.f, 0.f, 0.f);
+            v[u] = in ? *reinterpret_cast<const uint4 *>(bo + (i + u) * kSlotO) : make_uint4(0u, 0u, 0u, 0u);
         }
 #pragma unroll
-        for (int u = 0; u < 4; ++u) {
+        for (int u = 0; u < kPer; ++u) {
             if (li[u] == -INFINITY) continue;   // an empty partial weighs nothing
             if (li[u] > ms.mref) {
                 const float a = ms.mref == -INFINITY ? 0.f : expf(ms.mref - li[u]);
@@ -95,8 +98,11 @@ __device__ __forceinline__ void merge_slots(const float *bo, const float *bl, in
             }
             const float w = expf(li[u] - ms.mref);
             ms.ssum += w;
-            ms.acc0.x += w * v0[u].x; ms.acc0.y += w * v0[u].y; ms.acc0.z += w * v0[u].z; ms.acc0.w += w * v0[u].w;
-            ms.acc1.x += w * v1[u].x; ms.acc1.y += w * v1[u].y; ms.acc1.z += w * v1[u].z; ms.acc1.w += w * v1[u].w;
+            // bf16 to fp32: the upper 16 bits of each float
+            ms.acc0.x += w * __uint_as_float(v[u].x << 16); ms.acc0.y += w * __uint_as_float(v[u].x & 0xffff0000u);
+            ms.acc0.z += w * __uint_as_float(v[u].y << 16); ms.acc0.w += w * __uint_as_float(v[u].y & 0xffff0000u);
+            ms.acc1.x += w * __uint_as_float(v[u].z << 16); ms.acc1.y += w * __uint_as_float(v[u].z & 0xffff0000u);
+            ms.acc1.z += w * __uint_as_float(v[u].w << 16); ms.acc1.w += w * __uint_as_float(v[u].w & 0xffff0000u);
         }
     }
 }
@@ -132,7 +138,7 @@ __device__ __forceinline__ void merge_store(const MergeState &ms, int key, int h
 template <bool kIndexed>
 __global__ void __launch_bounds__(128, 9) decode_combine_kernel(const int32_t *__restrict__ slot_ptr,
                                                              const int32_t *__restrict__ merge_keys,
-                                                             const float *__restrict__ part_o,
+                                                             const __nv_bfloat16 *__restrict__ part_o,
                                                              const float *__restrict__ part_lse,
                                                              __nv_bfloat16 *__restrict__ out, float *__restrict__ lse_out)
 {
@@ -145,10 +151,10 @@ __global__ void __launch_bounds__(128, 9) decode_combine_kernel(const int32_t *_
     pdl_launch_dependents();
     const int tid = threadIdx.x;
     const int h = tid & 7, part = tid >> 3;          // head, 8-dim chunk: a warp reads 4 chunks x 8 heads, contiguous
-    const float *bo = part_o + (size_t)p0 * kGroup * kD + (part * kGroup + h) * 8;   // chunk `part` of head h
+    const __nv_bfloat16 *bo = part_o + (size_t)p0 * kGroup * kD + (part * kGroup + h) * 8;   // chunk `part` of head h
     const float *bl = part_lse + (size_t)p0 * kGroup + h;
     MergeState ms;
-    merge_slots(bo, bl, n, 0, 1, ms);
+    merge_slots<6>(bo, bl, n, 0, 1, ms);
     merge_store(ms, key, h, part, out, lse_out);
 }
 
@@ -159,7 +165,7 @@ __global__ void __launch_bounds__(128, 9) decode_combine_kernel(const int32_t *_
 // (two per SM) and the cluster merge below is not taken.
 template <bool kIndexed, int kGroups>
 __global__ void __launch_bounds__(128 * kGroups, 8 / kGroups) decode_combine_wide_kernel(
-    const int32_t *__restrict__ slot_ptr, const int32_t *__restrict__ merge_keys, const float *__restrict__ part_o,
+    const int32_t *__restrict__ slot_ptr, const int32_t *__restrict__ merge_keys, const __nv_bfloat16 *__restrict__ part_o,
     const float *__restrict__ part_lse, __nv_bfloat16 *__restrict__ out, float *__restrict__ lse_out)
 {
     constexpr int kWideGroups = kGroups;
@@ -169,10 +175,10 @@ __global__ void __launch_bounds__(128 * kGroups, 8 / kGroups) decode_combine_wid
     pdl_launch_dependents();
     const int tid = threadIdx.x & 127, q = threadIdx.x >> 7;
     const int h = tid & 7, part = tid >> 3;
-    const float *bo = part_o + (size_t)p0 * kGroup * kD + (part * kGroup + h) * 8;
+    const __nv_bfloat16 *bo = part_o + (size_t)p0 * kGroup * kD + (part * kGroup + h) * 8;
     const float *bl = part_lse + (size_t)p0 * kGroup + h;
     MergeState ms;
-    merge_slots(bo, bl, n, q, kWideGroups, ms);
+    merge_slots<4>(bo, bl, n, q, kWideGroups, ms);
     __shared__ MergeState st[kWideGroups - 1][128];
     if (q > 0) st[q - 1][tid] = ms;
     __syncthreads();
@@ -225,7 +231,7 @@ __device__ __forceinline__ MergeState load_remote_state(uint32_t addr, uint32_t 
 
 template <bool kIndexed>
 __global__ void __launch_bounds__(512, 2) decode_combine_cluster_kernel(
-    const int32_t *__restrict__ slot_ptr, const int32_t *__restrict__ merge_keys, const float *__restrict__ part_o,
+    const int32_t *__restrict__ slot_ptr, const int32_t *__restrict__ merge_keys, const __nv_bfloat16 *__restrict__ part_o,
     const float *__restrict__ part_lse, __nv_bfloat16 *__restrict__ out, float *__restrict__ lse_out)
 {
     const uint32_t rank = cluster_ctarank();
@@ -236,10 +242,10 @@ __global__ void __launch_bounds__(512, 2) decode_combine_cluster_kernel(
     pdl_launch_dependents();
     const int tid = threadIdx.x & 127, q = threadIdx.x >> 7;
     const int h = tid & 7, part = tid >> 3;
-    const float *bo = part_o + (size_t)p0 * kGroup * kD + (part * kGroup + h) * 8;
+    const __nv_bfloat16 *bo = part_o + (size_t)p0 * kGroup * kD + (part * kGroup + h) * 8;
     const float *bl = part_lse + (size_t)p0 * kGroup + h;
     MergeState ms;
-    merge_slots(bo, bl, n, (int)rank + kMergeCluster * q, 4 * kMergeCluster, ms);
+    merge_slots<4>(bo, bl, n, (int)rank + kMergeCluster * q, 4 * kMergeCluster, ms);
     __shared__ MergeState st[4][128];
     st[q][tid] = ms;
     __syncthreads();
@@ -402,8 +408,8 @@ padoc_status decode_split_k(const DecodePool &pl, const padoc_decode_plan *info,
         return PADOC_ERR_CUDA;
 
     if ((int64_t)pl.num_blocks * cfg.num_kv_heads * kBlk >= INT32_MAX) return PADOC_ERR_UNSUPPORTED;
-    float *part_o = (float *)workspace;
-    float *part_lse = (float *)((uint8_t *)workspace + padoc_align256((size_t)info->num_slots * kGroup * kD * 4));
+    __nv_bfloat16 *part_o = (__nv_bfloat16 *)workspace;
+    float *part_lse = (float *)((uint8_t *)workspace + padoc_align256((size_t)info->num_slots * kGroup * kD * 2));
     const float sl2 = scale * PADOC_LOG2E;
 
     // shared streams of dense pages on the tensor cores
@@ -504,7 +510,7 @@ padoc_status decode_split_k(const DecodePool &pl, const padoc_decode_plan *info,
                     : wide    ? (all_keys ? decode_combine_wide_kernel<false, 4> : decode_combine_wide_kernel<true, 4>)
                               : (all_keys ? decode_combine_kernel<false> : decode_combine_kernel<true>);
         PADOC_CUDA_TRY(cudaLaunchKernelEx(&lc, kern, prm.slot_ptr, (const int32_t *)(plan + info->off_merge_keys),
-                                          (const float *)part_o, (const float *)part_lse, (__nv_bfloat16 *)out, lse));
+                                          (const __nv_bfloat16 *)part_o, (const float *)part_lse, (__nv_bfloat16 *)out, lse));
     }
     return padoc_launch_status();
 }

@@ -101,7 +101,8 @@ struct TcDecodeParams {
     int32_t num_blocks, num_kv_heads;
     int32_t pool_rows;           // num_blocks * num_kv_heads * 16: first out-of-range row
     const float *k_scales, *v_scales;   // E4M3 pool: [num_blocks][num_kv_heads]
-    float *part_o, *part_lse;
+    __nv_bfloat16 *part_o;       // partial O, bf16 (workspace layout in plan_internal.h)
+    float *part_lse;
     __nv_bfloat16 *out;          // [S][Hq][128]: written directly by PADOC_ITEM_SOLE items
     float *lse;                  // [S][Hq]
     int32_t num_q_heads;
@@ -747,7 +748,7 @@ __device__ __forceinline__ void decode_tc_role(const CUtensorMap &kmap, const CU
                 const size_t prow = (size_t)(mi ? pb1 : pb0) * kGroup + hl;
                 // slot layout [16 chunks of 8 dims][8 heads][8]: the 8 rows (heads) of a stream write
                 // one contiguous 256-byte run per chunk; a sole item writes the row's output itself
-                float *sb = prm.part_o + (size_t)(mi ? pb1 : pb0) * (kGroup * kD) + hl * 8;
+                __nv_bfloat16 *sb = prm.part_o + (size_t)(mi ? pb1 : pb0) * (kGroup * kD) + hl * 8;
                 const size_t orow = ((size_t)(first + (valid ? b : 0)) * prm.num_q_heads + kvh * kGroup + hl);
                 __nv_bfloat16 *ob = prm.out + orow * kD + 64 * hc;
                 const uint32_t tO = tmem + lanes + 256 + 128 * mi + 64 * hc;
@@ -762,16 +763,16 @@ __device__ __forceinline__ void decode_tc_role(const CUtensorMap &kmap, const CU
 #pragma unroll
                         for (int i = 0; i < 32; i += 8) {
                             auto v = [&](int k) { return empty ? 0.f : __uint_as_float(o[i + k]) * inv; };
+                            uint4 w;
+                            w.x = pack_bf16x2(v(0), v(1));
+                            w.y = pack_bf16x2(v(2), v(3));
+                            w.z = pack_bf16x2(v(4), v(5));
+                            w.w = pack_bf16x2(v(6), v(7));
                             if (sole) {
-                                uint4 w;
-                                w.x = pack_bf16x2(v(0), v(1));
-                                w.y = pack_bf16x2(v(2), v(3));
-                                w.z = pack_bf16x2(v(4), v(5));
-                                w.w = pack_bf16x2(v(6), v(7));
                                 *reinterpret_cast<uint4 *>(ob + 32 * q + i) = w;
                             } else {
                                 const int chunk = 8 * hc + 4 * q + i / 8;
-                                st_global_v8(sb + chunk * (kGroup * 8), v(0), v(1), v(2), v(3), v(4), v(5), v(6), v(7));
+                                *reinterpret_cast<uint4 *>(sb + chunk * (kGroup * 8)) = w;
                             }
                         }
                     }
@@ -855,7 +856,7 @@ decode_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant
 padoc_status padoc_launch_decode_tc(const CUtensorMap *kmap, const CUtensorMap *vmap, const CUtensorMap *qmap, const int32_t *plan,
                                     const padoc_decode_plan *info, const int32_t *page_table, int32_t page_stride,
                                     const int32_t *stream_table, int32_t stream_stride, int32_t num_blocks,
-                                    const float *k_scales, const float *v_scales, float *part_o, float *part_lse,
+                                    const float *k_scales, const float *v_scales, __nv_bfloat16 *part_o, float *part_lse,
                                     __nv_bfloat16 *out, float *lse, float scale_log2, int *err,
                                     const padoc_warp::DecodeParams *wprm, cudaStream_t stream)
 {

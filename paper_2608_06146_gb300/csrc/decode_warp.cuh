@@ -60,7 +60,8 @@ struct DecodeParams {
     const uint8_t *k_codes, *v_codes;     // E4M3 pool (k_pool / v_pool unused)
     const float *k_scales, *v_scales;
     const __nv_bfloat16 *q;
-    float *part_o, *part_lse;
+    __nv_bfloat16 *part_o;       // partial O, bf16 (workspace layout in plan_internal.h)
+    float *part_lse;
     float scale_log2;
     int *err;
 };
@@ -317,19 +318,25 @@ __device__ __forceinline__ void decode_warp_role(const DecodeParams &prm, uint8_
             l[0] += __shfl_xor_sync(0xffffffffu, l[0], sh);
             l[1] += __shfl_xor_sync(0xffffffffu, l[1], sh);
         }
-        // the partial, straight from the accumulators, in the slot layout [16 chunks of 8 dims]
-        // [8 heads][8]: for each (mt, register) the 8 lanes of a head write one chunk's 8 dims, so
-        // every store fills whole 32-byte sectors
+        // the partial in bf16, in the slot layout [16 chunks of 8 dims][8 heads][8]: lane l holds dim
+        // l / 4 of heads h0, h0 + 1 (h0 = 2 (l % 4)); with its partner l ^ 4 (the next or previous dim)
+        // a lane of an even dim writes the dim pair of head h0, one of an odd dim that of head
+        // h0 + 1, so that the warp writes each chunk's [8 heads][8 dims] as one 128-byte run
         {
-            const int h0 = (lane & 3) * 2;
+            const int h0 = (lane & 3) * 2, dm = lane >> 2;
+            const bool ev = (dm & 1) == 0;
             const float i0f = l[0] > 0.f ? 1.f / l[0] : 0.f, i1f = l[1] > 0.f ? 1.f / l[1] : 0.f;
-            float *p = prm.part_o + row0 * kD + h0 * 8 + (lane >> 2);   // row0 = slot * 8
+            // element offset of this lane's pair inside a chunk
+            const int off = ev ? h0 * 8 + dm : (h0 + 1) * 8 + dm - 1;
+            uint32_t *p = reinterpret_cast<uint32_t *>(prm.part_o + row0 * kD);   // row0 = slot * 8
 #pragma unroll
             for (int mt = 0; mt < 8; ++mt) {
-                p[mt * 128] = o[mt][0] * i0f;           // chunk 2 mt, head h0
-                p[mt * 128 + 8] = o[mt][1] * i1f;       // chunk 2 mt, head h0 + 1
-                p[mt * 128 + 64] = o[mt][2] * i0f;      // chunk 2 mt + 1, head h0
-                p[mt * 128 + 72] = o[mt][3] * i1f;      // chunk 2 mt + 1, head h0 + 1
+#pragma unroll
+                for (int c = 0; c < 2; ++c) {   // chunk 2 mt + c: registers 2c (head h0), 2c + 1 (h0 + 1)
+                    const float a = o[mt][2 * c] * i0f, b = o[mt][2 * c + 1] * i1f;
+                    const float pa = __shfl_xor_sync(0xffffffffu, a, 4), pb = __shfl_xor_sync(0xffffffffu, b, 4);
+                    p[((2 * mt + c) * 64 + off) >> 1] = ev ? pack_bf16x2(a, pa) : pack_bf16x2(pb, b);
+                }
             }
         }
         if (lane < 4) {

@@ -167,11 +167,12 @@ typedef struct {
 
 static inline size_t padoc_align256(size_t x) { return (x + 255) & ~(size_t)255; }
 
-// Workspace: part_o fp32 [slots][d / 8][group][8] (a slot's dims in chunks of 8, the group's heads
-// inside a chunk, so that the heads of one stream are written as one contiguous run per chunk), then
+// Workspace: part_o bf16 [slots][d / 8][group][8] (a slot's dims in chunks of 8, the group's heads
+// inside a chunk, so that the heads of one stream are written as one contiguous run per chunk; each
+// partial is O / l, so bf16 adds at most 2^-9 of its magnitude before the merge's fp32 sums), then
 // part_lse fp32 [slots][group] at a 256-byte boundary; a slot holds one partial of the
 // group = Hq / Hkv query heads of one (stream, KV head).
 static inline size_t padoc_decode_workspace_bytes(int64_t slots, int32_t group, int32_t d)
 {
-    return padoc_align256((size_t)slots * group * d * 4) + padoc_align256((size_t)slots * group * 4);
+    return padoc_align256((size_t)slots * group * d * 2) + padoc_align256((size_t)slots * group * 4);
 }

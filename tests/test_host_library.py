@@ -266,7 +266,8 @@ def check_decode_plan(wl, layout, tc_ctas, warp_ctas):
     for kind, idx, g, tb, te, fs, ns, slot in items[ntc:]:
         assert te <= (sh[fs] if kind == 0 else pl[fs])
     need = pa.padoc_decode_workspace_size(info)
-    assert need >= info.num_slots * (wl.num_q_heads // Hkv) * (wl.head_dim + 1) * 4
+    # bf16 partial O and fp32 LSE per slot and query head of the group
+    assert need >= info.num_slots * (wl.num_q_heads // Hkv) * (wl.head_dim * 2 + 4)
     # the merge joins every (stream, KV head) key but those a sole tensor-core item writes itself
     from tests.test_chunk_prefill_host import check_sole_and_merge_keys
     check_sole_and_merge_keys(plan, info, items, Hkv)

@@ -60,7 +60,7 @@ def test_noalloc_decode_matches_oracle_and_workspace_decode_on_two_calls():
 
 def test_noalloc_rejects_a_plan_beyond_the_array():
     pa.load_library()
-    wl = inputs.serving_batch(num_pages=128)      # its split-K partials need more than 32 MiB
+    wl = inputs.serving_batch(num_pages=256)      # its split-K partials need more than 32 MiB
     plan = DecodePlan(wl.pages, wl.num_q_heads, wl.num_kv_heads, wl.head_dim, DEV)
     assert pa.padoc_decode_workspace_size(plan.info) > pa.PADOC_STATIC_WORKSPACE_BYTES
     S = plan.num_streams
