@@ -47,8 +47,8 @@ FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustain
 # Decode: one step = its kernels' counters added up (bf16: the decode grid and the merge; E4M3: the
 # tensor-core grid, the warp grid and the merge). Prefill backward: both passes and the merge of the
 # split key tiles.
-TRAFFIC_BYTES = {"decode": 223_312_512,
-                 "decode_e4m3": 124_968_832,
+TRAFFIC_BYTES = {"decode": 212_294_656,
+                 "decode_e4m3": 114_668_800,
                  "prefill": 260_600_000,
                  "prefill_bwd": 1_670_324_480}
 
