@@ -53,8 +53,9 @@ extern "C" {
  * 3 adds the FP8 (E4M3) KV cache (padoc_kv_pool_e4m3 and its quantize, append and decode calls),
  * the bounded-wait self-test, the in-place plan advance and the one-call decode step. 4 adds the
  * merge key list to the decode plan (padoc_decode_plan.off_merge_keys, num_merge_keys). 5 adds the
- * loop's step runner (padoc_mpd_runner_*). */
-#define PADOC_ATTN_VERSION 5
+ * loop's step runner (padoc_mpd_runner_*). 6 adds padoc_mpd_step.off_first_blocks and stores the
+ * split-K partials in bf16 (the decode workspace's size changes with it). */
+#define PADOC_ATTN_VERSION 6
 
 /* A CUDA stream handle; identical to cudaStream_t. */
 typedef struct CUstream_st *padoc_stream_t;
@@ -550,6 +551,11 @@ typedef struct {
     int64_t off_slots;         /* int32 [num_streams]: each stream's append slot */
     int64_t off_rows;          /* int32 [num_streams]: left for the caller (e.g. the source rows of the
                                   inputs for padoc_append_inputs), not written */
+    int64_t off_first_blocks;  /* int32 [plan.num_warps][4]: the pool rows ((block id x Hkv + KV head) x
+                                  block_size) of the first four 16-token blocks of each warp list's
+                                  first item, -2 - row for the block holding its stream's newest row,
+                                  -1 past its end; padoc_mpd_launch_step's decode warps start these
+                                  blocks before they read their item headers */
     int64_t off_stream_ids;    /* int32 [num_streams]: the step's stream ids (host use) */
     int64_t upload_words;      /* [0, upload_words) is what the device needs: everything but the ids */
     int64_t total_words;       /* words the step needs in the staging buffer */

@@ -386,7 +386,7 @@ padoc_status decode_split_k(const DecodePool &pl, const padoc_decode_plan *info,
                             const int32_t *page_block_table, int32_t page_table_stride,
                             const int32_t *stream_block_table, int32_t stream_table_stride, const void *q, float scale,
                             void *out, float *lse, void *workspace, size_t workspace_bytes, cudaStream_t cs,
-                            bool after_append = false)
+                            bool after_append = false, const int32_t *first_blocks = nullptr)
 {
     const padoc_decode_config &cfg = info->cfg;
     if (cfg.head_dim != kD || cfg.num_q_heads != kGroup * cfg.num_kv_heads || cfg.block_size != kBlk)
@@ -428,6 +428,7 @@ padoc_status decode_split_k(const DecodePool &pl, const padoc_decode_plan *info,
     prm.slot_ptr = plan + info->off_slot_ptr;
     prm.page_len = plan + info->off_page_len;
     prm.pre_wait = after_append && !pl.e4m3 ? 1 : 0;
+    prm.first_blocks = prm.pre_wait ? first_blocks : nullptr;
     prm.items = reinterpret_cast<const padoc_item *>(plan + info->off_items);
     prm.first_item = info->num_tc_items;
     prm.warp_ptr = plan + info->off_warp_ptr;
@@ -527,7 +528,7 @@ padoc_status branch_decode(const padoc_kv_pool *pool, const padoc_decode_plan *i
                            const int32_t *page_block_table, int32_t page_table_stride,
                            const int32_t *stream_block_table, int32_t stream_table_stride, const void *q, float scale,
                            void *out, float *lse, void *workspace, size_t workspace_bytes, padoc_stream_t stream,
-                           bool after_append)
+                           bool after_append, const int32_t *first_blocks = nullptr)
 {
     if (!pool || !info || !plan_dev || !q || !out || !lse) return PADOC_ERR_INVALID_ARGUMENT;
     const padoc_decode_config &cfg = info->cfg;
@@ -565,7 +566,7 @@ padoc_status branch_decode(const padoc_kv_pool *pool, const padoc_decode_plan *i
     if (pool->dtype != PADOC_DTYPE_BF16) return PADOC_ERR_UNSUPPORTED;
     const DecodePool dp{false, pool->k_pool, pool->v_pool, nullptr, nullptr, pool->num_blocks};
     return decode_split_k(dp, info, plan, page_block_table, page_table_stride, stream_block_table, stream_table_stride,
-                          q, scale, out, lse, workspace, workspace_bytes, cs, after_append);
+                          q, scale, out, lse, workspace, workspace_bytes, cs, after_append, first_blocks);
 }
 
 }  // namespace
@@ -586,10 +587,10 @@ padoc_status padoc_branch_decode_attn_after_append(const padoc_kv_pool *pool, co
                                                    int32_t page_table_stride, const int32_t *stream_block_table,
                                                    int32_t stream_table_stride, const void *q, float scale, void *out,
                                                    float *lse, void *workspace, size_t workspace_bytes,
-                                                   padoc_stream_t stream)
+                                                   padoc_stream_t stream, const int32_t *first_blocks)
 {
     return branch_decode(pool, info, plan_dev, page_block_table, page_table_stride, stream_block_table,
-                         stream_table_stride, q, scale, out, lse, workspace, workspace_bytes, stream, true);
+                         stream_table_stride, q, scale, out, lse, workspace, workspace_bytes, stream, true, first_blocks);
 }
 
 extern "C" padoc_status padoc_branch_decode_attn_e4m3(const padoc_kv_pool_e4m3 *pool, const padoc_decode_plan *info,

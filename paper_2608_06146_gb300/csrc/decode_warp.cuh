@@ -48,6 +48,10 @@ struct DecodeParams {
     // tensor-core work read their headers and block ids and start their first blocks (those
     // without a newest row) before they wait for it
     int32_t pre_wait;
+    // with pre_wait (may be null): [num_warps][4] pool rows of the first four blocks of each warp's
+    // first item (-2 - row: the block of its stream's newest row; -1 past its end), read beside the
+    // item header instead of after it
+    const int32_t *first_blocks;
     const padoc_item *items;
     int32_t first_item;          // warp items start here
     const int32_t *warp_ptr;     // warp w owns warp items [warp_ptr[w], warp_ptr[w+1])
@@ -99,6 +103,10 @@ __device__ __forceinline__ void decode_warp_role(const DecodeParams &prm, uint8_
     // The warp walks its items with one ring of kWStages paged blocks that runs on from one item
     // into the next. Producer: the next block to fetch is block pb of item pu (walk pc, ids ids_c);
     // item pu + 1 (walk pn, ids ids_n) and the header of item pu + 2 (hn2) are already on the way.
+    // kPreWait with first_blocks: lane k < 4 holds the pool row of block k of the first item (>= 0),
+    // -2 - that row for the block holding its stream's newest row, -1 past the item's end
+    const bool have_fb = kPreWait && prm.first_blocks != nullptr;
+    const int32_t fb = have_fb && lane < 4 ? prm.first_blocks[(size_t)wi * 4 + lane] : -1;
     int pu = i0, pb = 0;
     Walk pc{prm.page_table, 0, 0, 0}, pn{prm.page_table, 0, 0, 0};
     int32_t ids_c = 0, ids_n = 0;
@@ -166,12 +174,33 @@ __device__ __forceinline__ void decode_warp_role(const DecodeParams &prm, uint8_
         // row (page_len - 1 of a shared item's page, private_len - 1 of a private item's stream),
         // which the append may be writing; everything read so far (plan, block tables) was copied
         // before the append started.
-        if (i0 < i1) {
+        if (have_fb) {
+            // straight from the rows the host wrote, without waiting for the item header: the
+            // leading blocks that exist, are in the pool and hold no newest row
+            const bool ok = lane < 4 && fb >= 0 && fb <= prm.pool_rows - kBlk;
+            const uint32_t okm = __ballot_sync(0xffffffffu, ok) & 0xfu;
+            pre = min(__ffs(~okm) - 1, kWStages);
+            for (int k = 0; k < pre; ++k) {
+                const size_t rowbase = (size_t)__shfl_sync(0xffffffffu, fb, k);
+                const uint32_t base = smem_u32(wbuf + k * kWStageBytes);
+#pragma unroll
+                for (int c = 0; c < 16; ++c) {
+                    const int q = lane + 32 * c;
+                    const int panel = q >> 7, r = (q >> 3) & 15, cc = q & 7;
+                    const __nv_bfloat16 *src = (panel < 2 ? prm.k_pool : prm.v_pool) +
+                                               (rowbase + r) * kD + (panel & 1) * 64 + cc * 8;
+                    cp_async_16_hint(base + panel * kBoxBytes + r * 128 + ((cc ^ (r & 7)) << 4), src, 16u, kv_policy);
+                }
+                cp_async_commit();
+            }
+            pb = pre;
+            ring = pre;
+        } else if (i0 < i1) {
             const padoc_item it0 = load_item(i0);
             const int32_t len = it0.kind == PADOC_ITEM_SHARED ? prm.page_len[it0.index] : prm.private_len[it0.first_stream];
             pre = min(min(kWStages, pc.nblk), max(0, (len - 1) / kBlk - pc.blk0));
+            for (int k = 0; k < pre; ++k) issue_next();
         }
-        for (int k = 0; k < pre; ++k) issue_next();
         pdl_wait_prerequisite();
         pdl_launch_dependents();
     }

@@ -10,6 +10,7 @@
 // appended, which is the shared stream's current length. Retiring removes the row and returns the
 // stream's private blocks; a page's shared blocks return once its last stream has retired.
 #include <algorithm>
+#include <climits>
 #include <cstdint>
 #include <cstring>
 #include <deque>
@@ -347,7 +348,8 @@ extern "C" padoc_status padoc_mpd_prepare_step(padoc_mpd *m, const padoc_decode_
     step->off_stream_table = step->off_page_table + align32((int64_t)P * pstride);
     step->off_slots = step->off_stream_table + align32((int64_t)C * sstride);
     step->off_rows = step->off_slots + align32(C);
-    step->off_stream_ids = step->off_rows + align32(C);
+    step->off_first_blocks = step->off_rows + align32(C);
+    step->off_stream_ids = step->off_first_blocks + align32((int64_t)pp.num_warps * 4);
     step->upload_words = step->off_stream_ids;
     step->total_words = step->off_stream_ids + align32(C);
     if (capacity_words < step->total_words || !stage) return PADOC_ERR_CAPACITY;
@@ -358,6 +360,30 @@ extern "C" padoc_status padoc_mpd_prepare_step(padoc_mpd *m, const padoc_decode_
                                stage + step->off_stream_table, sstride);
     if (st == PADOC_OK) st = padoc_plan_write_blob(pp, P, cfg, stage + step->off_plan, plan_ints, &step->plan);
     if (st != PADOC_OK) return st;   // not reached: both were checked above
+    // the pool rows of the first four blocks of each warp's first item, from the tables just
+    // written, so that the decode's warps start them before they read their item headers; the block
+    // that holds the item's stream's newest row (which the step's append writes) as -2 - row
+    int32_t *fb = stage + step->off_first_blocks;
+    for (int32_t w = 0; w < pp.num_warps; ++w) {
+        int32_t *f = fb + (size_t)w * 4;
+        f[0] = f[1] = f[2] = f[3] = -1;
+        const int32_t u = pp.num_tc_items + pp.warp_ptr[(size_t)w];
+        if (pp.warp_ptr[(size_t)w] >= pp.warp_ptr[(size_t)w + 1]) continue;
+        const padoc_item &it = pp.items[(size_t)u];
+        const bool shared = it.kind == PADOC_ITEM_SHARED;
+        const int32_t *row = shared ? stage + step->off_page_table + (size_t)it.index * pstride
+                                    : stage + step->off_stream_table + (size_t)it.first_stream * sstride;
+        const int32_t width = shared ? pstride : sstride;
+        const int32_t len = shared ? pp.page_len[(size_t)it.index] : pp.streams[(size_t)it.first_stream].private_len;
+        const int32_t hot = (len - 1) / m->bs;
+        const int32_t b0 = it.tok_begin / m->bs, nb = it.tok_end > it.tok_begin ? (it.tok_end - it.tok_begin + m->bs - 1) / m->bs : 0;
+        for (int32_t k = 0; k < 4 && k < nb && b0 + k < width; ++k) {
+            const int32_t id = row[b0 + k];
+            const int64_t r = ((int64_t)id * cfg->num_kv_heads + it.kv_head) * m->bs;
+            if (id < 0 || id >= m->num_blocks || r > INT32_MAX - 2) break;   // left to the decode's own checks
+            f[k] = b0 + k == hot ? (int32_t)(-2 - r) : (int32_t)r;
+        }
+    }
     step->num_streams = n;
     step->num_pages = P;
     step->page_stride = pstride;
@@ -388,7 +414,8 @@ extern "C" padoc_status padoc_mpd_launch_step(const padoc_mpd_step *step, const 
     if (st != PADOC_OK) return st;
     return padoc_branch_decode_attn_after_append(pool, &info, dev_ints + step->off_plan, dev_ints + step->off_page_table,
                                     step->page_stride, dev_ints + step->off_stream_table, step->stream_stride, q_dst,
-                                    scale, out, lse, workspace, workspace_bytes, stream);
+                                    scale, out, lse, workspace, workspace_bytes, stream,
+                                                 step->plan.num_warps > 0 ? dev_ints + step->off_first_blocks : nullptr);
 }
 
 // ---- the step loop's host side in one call per step (padoc_mpd_runner_*) ----------------------

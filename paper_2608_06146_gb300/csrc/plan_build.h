@@ -45,9 +45,12 @@ padoc_status padoc_plan_write_blob(const PlanParts &pp, int32_t num_pages, const
 // same stream (padoc_mpd_launch_step): the append writes only each stream's newest K/V row and the
 // step's queries, and the plan and block tables were copied before it started, so warps without
 // tensor-core work read those and start their first paged blocks before they wait for the append.
+// first_blocks (device, may be NULL): int32 [num_warps][4], the pool rows of the first four blocks
+// of each warp's first item (-2 - row for the block of its stream's newest row, -1 past its end),
+// read in parallel with the item headers (padoc_mpd_step.off_first_blocks).
 padoc_status padoc_branch_decode_attn_after_append(const padoc_kv_pool *pool, const padoc_decode_plan *info,
                                                    const int32_t *plan_dev, const int32_t *page_block_table,
                                                    int32_t page_table_stride, const int32_t *stream_block_table,
                                                    int32_t stream_table_stride, const void *q, float scale, void *out,
                                                    float *lse, void *workspace, size_t workspace_bytes,
-                                                   padoc_stream_t stream);
+                                                   padoc_stream_t stream, const int32_t *first_blocks);

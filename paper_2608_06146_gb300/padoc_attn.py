@@ -86,7 +86,7 @@ class padoc_decode_plan(ctypes.Structure):
 class padoc_mpd_step(ctypes.Structure):
     _fields_ = [("num_streams", ctypes.c_int32), ("num_pages", ctypes.c_int32), ("page_stride", ctypes.c_int32),
                 ("stream_stride", ctypes.c_int32), ("off_plan", ctypes.c_int64), ("off_page_table", ctypes.c_int64),
-                ("off_stream_table", ctypes.c_int64), ("off_slots", ctypes.c_int64), ("off_rows", ctypes.c_int64),
+                ("off_stream_table", ctypes.c_int64), ("off_slots", ctypes.c_int64), ("off_rows", ctypes.c_int64), ("off_first_blocks", ctypes.c_int64),
                 ("off_stream_ids", ctypes.c_int64), ("upload_words", ctypes.c_int64), ("total_words", ctypes.c_int64),
                 ("plan", padoc_decode_plan)]
 

@@ -39,7 +39,7 @@ def test_exports_every_declared_symbol(lib):
     for name in declared:
         assert hasattr(lib, name), f"{name} not exported"
     assert set(pa.exported_symbols()) == declared
-    assert pa.padoc_version() == 5
+    assert pa.padoc_version() == 6
     assert pa.padoc_status_string(0) == "ok"
 
 

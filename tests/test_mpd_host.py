@@ -239,6 +239,29 @@ def test_stream_list_validation():
                                            pa.make_decode_config(16, 2, 128, layout_streams=True))
 
 
+
+
+def check_first_blocks(stage, st, plan, info, page_len, streams, pt, stt, Hkv=2):
+    """The step's first-block rows: for each warp list, the pool rows of its first item's first four
+    blocks, read from that item's block-table row, -2 - row for the block holding the stream's
+    newest row (the last shared row of the page for a shared item, the last private row for a
+    private one), -1 past the item's end."""
+    W = info.num_warps
+    fb = stage[st.off_first_blocks:st.off_first_blocks + 4 * W].reshape(W, 4)
+    wp = plan[info.off_warp_ptr:info.off_warp_ptr + W + 1]
+    items = plan[info.off_items:info.off_items + 8 * info.num_items].reshape(-1, 8)[info.num_tc_items:]
+    for w in range(W):
+        want = [-1] * 4
+        if wp[w] < wp[w + 1]:
+            kind, idx, g, tb, te, fs, ns, slot = items[wp[w]]
+            row, hot = (pt[idx], (page_len[idx] - 1) // BS) if kind == 0 else (stt[fs], (streams[fs]["private_len"] - 1) // BS)
+            nb = -(-(te - tb) // BS) if te > tb else 0
+            for k in range(min(4, nb)):
+                r = (int(row[tb // BS + k]) * Hkv + int(g)) * BS
+                want[k] = -2 - r if tb // BS + k == hot else r
+        assert fb[w].tolist() == want, f"warp {w}"
+
+
 @pytest.mark.parametrize("seed", range(4))
 def test_prepare_step_equals_granular_calls(seed):
     """padoc_mpd_prepare_step writes exactly what begin_step, step_tables and the stream-list planner
@@ -276,9 +299,11 @@ def test_prepare_step_equals_granular_calls(seed):
             stage[st.off_page_table:st.off_page_table + st.num_pages * st.page_stride].reshape(-1, st.page_stride), pt)
         np.testing.assert_array_equal(
             stage[st.off_stream_table:st.off_stream_table + C * st.stream_stride].reshape(-1, st.stream_stride), stt)
-        for off in (st.off_page_table, st.off_stream_table, st.off_slots, st.off_rows, st.off_stream_ids):
+        for off in (st.off_page_table, st.off_stream_table, st.off_slots, st.off_rows, st.off_first_blocks,
+                    st.off_stream_ids):
             assert off % 32 == 0
         assert st.plan.num_items == info.num_items and st.plan.num_slots == info.num_slots
+        check_first_blocks(stage, st, plan, info, page_len, streams, pt, stt)
         src.rows(ids)
         nf, eos = src.events(ids)
         new = b.end_step(nf, eos)
