@@ -43,11 +43,13 @@ sys.path.insert(0, ROOT)
 METRIC = "ancestor-attn decode queries/s, % of HBM roofline; packed prefill TFLOP/s"
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 # DRAM traffic per launch, dram__bytes_read.sum + dram__bytes_write.sum, copied from one ncu capture
-# of each kernel as it stands (cold caches); None where no capture of the current kernel exists.
-# Decode: one step = its kernels' counters added up (bf16: the decode grid and the merge; E4M3: the
-# tensor-core grid, the warp grid and the merge). Prefill backward: both passes and the merge of the
-# split key tiles.
-TRAFFIC_BYTES = {"decode": 212_294_656,
+# of each kernel as it stands; None where no capture of the current kernel exists. Decode: one step =
+# its kernels' counters added up (bf16: the decode grid and the merge, captured with the caches left
+# as the pipeline leaves them, so that the merge reads its partials from L2 as it does in the timed
+# step, the mean of two consecutive steps; E4M3: the tensor-core grid, the warp grid and the merge,
+# cold caches). Prefill: cold caches. Prefill backward: both passes and the merge of the split key
+# tiles, cold caches.
+TRAFFIC_BYTES = {"decode": 201_274_880,
                  "decode_e4m3": 114_668_800,
                  "prefill": 260_600_000,
                  "prefill_bwd": 1_670_324_480}
