@@ -8,12 +8,15 @@
 #define PADOC_PREFILL_Q_TILE 128
 #define PADOC_PREFILL_K_TILE 128
 
-// Prefill backward tiles. The dQ pass keeps 128 query rows (the M of its MMAs) and walks 32-key
-// k-tiles; the dK/dV pass keeps 128 keys (the M of its MMAs) and walks 32-row q-tiles. Narrow
-// steps let several steps' scores sit in tensor memory beside the accumulators and the resident
-// A operands, so the exponentials of one step overlap the MMAs of the next ones.
+// Prefill backward tiles. The dQ pass keeps 128 query rows (the M of its MMAs) and walks 64-key
+// k-tiles; the dK/dV pass keeps 128 keys (the M of its MMAs) and walks 64-row q-tiles. Narrow
+// steps let two steps' scores sit in tensor memory beside the accumulators and the resident A
+// operands, so the exponentials of one step overlap the MMAs of the next one (128-key dQ steps, one
+// step buffer, halve the S and dP MMA instructions but serialize the two: 1.305 -> 1.388 ms).
 #define PADOC_BWD_DQ_Q_TILE 128
+#ifndef PADOC_BWD_DQ_K_TILE
 #define PADOC_BWD_DQ_K_TILE 64
+#endif
 #define PADOC_BWD_DKV_Q_TILE 64
 #define PADOC_BWD_DKV_K_TILE 128
 // A dK/dV work unit (k-tile, KV head) of more steps ((q-tile, query head) pairs) than this is split

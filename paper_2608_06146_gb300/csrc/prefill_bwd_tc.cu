@@ -467,7 +467,7 @@ template <int W>
 struct DqCfg {
     static constexpr int kQT = PADOC_BWD_DQ_Q_TILE;    // 128 query rows: the M of every MMA
     static constexpr int kDepth = 256 / (2 * W);
-    static constexpr int kStages = W == 32 ? 8 : 5;
+    static constexpr int kStages = W == 32 ? 8 : W == 64 ? 5 : 3;
     static constexpr int kPanel = W * 128;
     static constexpr int kTile = 2 * kPanel;            // K or V of one step
     static constexpr uint32_t kColQ = 0, kColG = 64, kColBuf = 128, kColDQ = 384;
@@ -658,36 +658,43 @@ prefill_bwd_dq_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_con
             const int cb = prm.idx[e0 + u] * W + HW * ch;
             if (!wait_all(C::B_SFULL + u % DEPTH, (u / DEPTH) & 1, 95)) { ok = false; break; }
             tc_fence_after();
-            uint32_t sr[HW], dr[HW];
-            tmem_ld_cols<HW>(tmem + lanes + b, sr);
-            tmem_ld_cols<HW>(tmem + lanes + b + W, dr);
-            uint32_t vis = 0xffffffffu;
-            if (partial) {
-                const int lo0 = clamp_w(a0 - cb, HW), lo1 = clamp_w(b0 - cb, HW);
-                vis = interval_bits(lo0, max(clamp_w(a1 - cb, HW) - lo0, 0), 0) |
-                      interval_bits(lo1, max(clamp_w(b1 - cb, HW) - lo1, 0), 0);
-            }
-            tmem_ld_wait();
-            uint32_t dk[HW / 2];
-            // two key columns per packed instruction: P = exp2(S c - lse2), dS = P (dP - D)
-            auto column_pairs = [&](auto masked) {
+            // the thread's HW key columns in blocks of at most 32: block j's dS (bf16 pairs) goes to
+            // columns 16 j .. of its half of the dP buffer, which block j has already read
+            constexpr int HB = HW < 32 ? HW : 32;
 #pragma unroll
-                for (int i = 0; i < HW; i += 2) {
-                    float x0, x1;
-                    f2_unpack(f2_fma(f2_pack(__uint_as_float(sr[i]), __uint_as_float(sr[i + 1])), c2, nl2), x0, x1);
-                    float p0 = fast_exp2(x0), p1 = fast_exp2(x1);
-                    if (decltype(masked)::value) {
-                        p0 = (vis >> i) & 1u ? p0 : 0.f;
-                        p1 = (vis >> (i + 1)) & 1u ? p1 : 0.f;
-                    }
-                    const uint64_t t = f2_sub(f2_pack(__uint_as_float(dr[i]), __uint_as_float(dr[i + 1])), d2);
-                    float d0, d1;
-                    f2_unpack(f2_mul(f2_pack(p0, p1), t), d0, d1);
-                    dk[i >> 1] = pack_bf16x2(d0, d1);
+            for (int j = 0; j < HW / HB; ++j) {
+                uint32_t sr[HB], dr[HB];
+                tmem_ld_cols<HB>(tmem + lanes + b + HB * j, sr);
+                tmem_ld_cols<HB>(tmem + lanes + b + W + HB * j, dr);
+                uint32_t vis = 0xffffffffu;
+                if (partial) {
+                    const int cj = cb + HB * j;
+                    const int lo0 = clamp_w(a0 - cj, HB), lo1 = clamp_w(b0 - cj, HB);
+                    vis = interval_bits(lo0, max(clamp_w(a1 - cj, HB) - lo0, 0), 0) |
+                          interval_bits(lo1, max(clamp_w(b1 - cj, HB) - lo1, 0), 0);
                 }
-            };
-            if (partial) column_pairs(std::true_type{}); else column_pairs(std::false_type{});
-            tmem_st_cols<HW / 2>(tmem + lanes + b + W, dk);
+                tmem_ld_wait();
+                uint32_t dk[HB / 2];
+                // two key columns per packed instruction: P = exp2(S c - lse2), dS = P (dP - D)
+                auto column_pairs = [&](auto masked) {
+#pragma unroll
+                    for (int i = 0; i < HB; i += 2) {
+                        float x0, x1;
+                        f2_unpack(f2_fma(f2_pack(__uint_as_float(sr[i]), __uint_as_float(sr[i + 1])), c2, nl2), x0, x1);
+                        float p0 = fast_exp2(x0), p1 = fast_exp2(x1);
+                        if (decltype(masked)::value) {
+                            p0 = (vis >> i) & 1u ? p0 : 0.f;
+                            p1 = (vis >> (i + 1)) & 1u ? p1 : 0.f;
+                        }
+                        const uint64_t t = f2_sub(f2_pack(__uint_as_float(dr[i]), __uint_as_float(dr[i + 1])), d2);
+                        float d0, d1;
+                        f2_unpack(f2_mul(f2_pack(p0, p1), t), d0, d1);
+                        dk[i >> 1] = pack_bf16x2(d0, d1);
+                    }
+                };
+                if (partial) column_pairs(std::true_type{}); else column_pairs(std::false_type{});
+                tmem_st_cols<HB / 2>(tmem + lanes + b + W + (HB / 2) * j, dk);
+            }
             tmem_st_wait();
             tc_fence_before();
             mbar_arrive(bar(C::B_PFULL + u % DEPTH));
