@@ -820,6 +820,8 @@ def main():
     ap.add_argument("--only", default="all", choices=["all", "decode", "prefill", "prefill_bwd", "loop",
                                                       "chunk_prefill", "variants", "decode_e4m3", "replicas"])
     ap.add_argument("--replicas", type=int, default=0, help="decode input replicas (0: enough to exceed 4x L2)")
+    ap.add_argument("--shape", choices=["decode_page", "dense_page"], default=None,
+                    help="with --only replicas: that page shape alone")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-steady", action="store_true", help="skip the long back-to-back decode run")
     ap.add_argument("--tc-ctas", type=int, default=0, help="tensor-core decode CTAs (0: one per SM)")
@@ -856,7 +858,7 @@ def main():
                               "prefill_shuffled_ms": b["ms"], "prefill_shuffled_tflops": b["flops"] / (b["ms"] * 1e-3) / 1e12}))
         return 0
     if args.only == "replicas":
-        for shape in ("decode_page", "dense_page"):
+        for shape in (args.shape,) if args.shape else ("decode_page", "dense_page"):
             r = bench_decode_replicas(args, torch, dev, rank, world, shape)
             if rank == 0:
                 print(json.dumps({"shape": shape, "pages": r["pages"], "streams": r["streams"], "us": r["ms"] * 1e3,
