@@ -315,19 +315,18 @@ def bench_decode(args, torch, dev, rank, world, layout_streams=False):
                          l_host=torch.empty((S, wl.num_q_heads), dtype=torch.float32).pin_memory(), ev=evs))
     ws2 = [plan.workspace, torch.empty_like(plan.workspace)]
     lens = np.ascontiguousarray(plan.plan_host[plan.info.off_private_len:plan.info.off_private_len + S])
+    # one pa.DecodeStep per (buffer set, input replica): the arguments are marshalled once, as a caller
+    # with a fixed pool does
+    calls = [[pa.DecodeStep(k_pools[r], v_pools[r], st_["info"], st_["stage"], words, plan_ints, off_pt, PT, off_st,
+                            STW, st_["dev_ints"], st_["q_host"], st_["q_dev"], scale, st_["out"], st_["lse"],
+                            st_["o_host"], st_["l_host"], ws2[b], lens, stream, copy_in, copy_out, st_["ev"][0],
+                            st_["ev"][1], st_["ev"][2]) for r in range(R)] for b, st_ in enumerate(sets)]
 
     def e2e_step(i):
-        r = i % R
         b = i & 1
-        st_ = sets[b]
-        st_["ev"][1].synchronize()     # this set's previous copies in have run: its stage may change
-        h = st_["stage"].numpy()
-        if not pa.padoc_advance_decode_plan(h[:plan_ints], st_["info"], lens):
+        sets[b]["ev"][1].synchronize()     # this set's previous copies in have run: its stage may change
+        if not calls[b][i % R]():
             raise RuntimeError("plan advance refused")
-        pa.padoc_launch_decode_step(k_pools[r], v_pools[r], st_["info"], st_["stage"], words, off_pt, PT, off_st, STW,
-                                    st_["dev_ints"], st_["q_host"], st_["q_dev"], scale, st_["out"], st_["lse"],
-                                    st_["o_host"], st_["l_host"], ws2[b], stream, copy_in, copy_out,
-                                    st_["ev"][0], st_["ev"][1], st_["ev"][2])
 
     for i in range(max(args.warmup, 2)):
         e2e_step(i)

@@ -568,6 +568,46 @@ def padoc_launch_decode_step(k_pool, v_pool, info: padoc_decode_plan, stage, sta
     _check("padoc_launch_decode_step", st)
 
 
+class DecodeStep:
+    """One buffer set of a decode loop's host side with its arguments marshalled once: each call
+    patches the set's host plan for the streams' new private lengths (padoc_advance_decode_plan;
+    False, with nothing launched, when a new plan is needed) and runs padoc_launch_decode_step. The
+    arguments are those of the two functions; the tensors, arrays and streams must stay alive and
+    unmoved while the object is used."""
+
+    def __init__(self, k_pool, v_pool, info: padoc_decode_plan, stage, stage_words: int, plan_ints: int,
+                 off_page_table: int, page_stride: int, off_stream_table: int, stream_stride: int, dev_ints, q_host,
+                 q_dev, scale, out_dev, lse_dev, out_host, lse_host, workspace, private_len, stream=None,
+                 copy_in=None, copy_out=None, ev_free=None, ev_in=None, ev_dec=None):
+        lib = load_library()
+        self._f_adv, self._f_launch = lib.padoc_advance_decode_plan, lib.padoc_launch_decode_step
+        self._pool = padoc_kv_pool(_dev(k_pool, "k_pool"), _dev(v_pool, "v_pool"), k_pool.shape[0], k_pool.shape[2],
+                                   k_pool.shape[1], k_pool.shape[3], _dtype_code(k_pool))
+        self._info = info
+        plan = stage.numpy()[:plan_ints]
+        self._pl = np.ascontiguousarray(np.asarray(private_len, np.int32))
+        self._keep = (k_pool, v_pool, stage, dev_ints, q_host, q_dev, out_dev, lse_dev, out_host, lse_host, workspace,
+                      plan, stream, copy_in, copy_out, ev_free, ev_in, ev_dec)
+        ev = lambda e: None if e is None else e.cuda_event
+        self._adv_args = (plan.ctypes.data_as(_i32p), ctypes.byref(info), self._pl.ctypes.data_as(_i32p), self._pl.size)
+        self._launch_args = (ctypes.byref(self._pool), ctypes.byref(info), stage.data_ptr(), int(stage_words),
+                             int(off_page_table), int(page_stride), int(off_stream_table), int(stream_stride),
+                             _dev(dev_ints, "dev_ints"), dev_ints.numel(), q_host.data_ptr(), _dev(q_dev, "q_dev"),
+                             float(scale), _dev(out_dev, "out_dev"), _dev(lse_dev, "lse_dev"), out_host.data_ptr(),
+                             lse_host.data_ptr(), _dev(workspace, "workspace"),
+                             workspace.numel() * workspace.element_size(), _stream_ptr(stream),
+                             None if copy_in is None else _stream_ptr(copy_in),
+                             None if copy_out is None else _stream_ptr(copy_out), ev(ev_free), ev(ev_in), ev(ev_dec))
+
+    def __call__(self) -> bool:
+        st = self._f_adv(*self._adv_args)
+        if st == 6:
+            return False
+        _check("padoc_advance_decode_plan", st)
+        _check("padoc_launch_decode_step", self._f_launch(*self._launch_args))
+        return True
+
+
 PADOC_STATIC_WORKSPACE_BYTES = 32 << 20
 
 

@@ -57,8 +57,11 @@ def test_advanced_plan_decodes_the_grown_batch():
     _check(out.float().cpu().numpy(), lse.cpu().numpy(), ref_o, ref_l)
 
 
-@pytest.mark.parametrize("piped", [False, True])
-def test_one_call_step_from_host_memory(piped):
+@pytest.mark.parametrize("piped,prepared", [(False, False), (True, False), (True, True)])
+def test_one_call_step_from_host_memory(piped, prepared):
+    """padoc_launch_decode_step from pinned host memory, with the copies on the compute stream or on
+    copy streams ordered by the buffer set's events; prepared: through pa.DecodeStep (arguments
+    marshalled once; its plan advance to the same lengths changes nothing), three calls in a row."""
     wl = inputs.dense_page()
     di = inputs.decode_inputs(wl, 71)
     cfg = pa.make_decode_config(16, 2, 128, 16, False, 0, 0, 0)
@@ -89,8 +92,18 @@ def test_one_call_step_from_host_memory(piped):
         for e in evs:
             e.record()
         kw = dict(copy_in=torch.cuda.Stream(), copy_out=torch.cuda.Stream(), ev_free=evs[0], ev_in=evs[1], ev_dec=evs[2])
-    pa.padoc_launch_decode_step(di.k_pool.to(DEV), di.v_pool.to(DEV), info, stage, words, off_pt, PT, off_st, STW,
-                                dev_ints, q_host, q_dev, scale, out, lse, o_host, l_host, ws, **kw)
+    k_pool, v_pool = di.k_pool.to(DEV), di.v_pool.to(DEV)
+    if prepared:
+        lens = plan[info.off_private_len:info.off_private_len + S].copy()
+        step = pa.DecodeStep(k_pool, v_pool, info, stage, words, int(info.plan_ints), off_pt, PT, off_st, STW, dev_ints,
+                             q_host, q_dev, scale, out, lse, o_host, l_host, ws, lens, **kw)
+        for _ in range(3):
+            kw["ev_in"].synchronize()       # the set's previous copies in have run
+            assert step()
+        np.testing.assert_array_equal(h[:info.plan_ints], plan)
+    else:
+        pa.padoc_launch_decode_step(k_pool, v_pool, info, stage, words, off_pt, PT, off_st, STW, dev_ints, q_host, q_dev,
+                                    scale, out, lse, o_host, l_host, ws, **kw)
     if piped:
         kw["ev_free"].synchronize()         # the results' copies out have run
     pa.padoc_check_device_errors()          # synchronizes the stream: the results are in host memory
