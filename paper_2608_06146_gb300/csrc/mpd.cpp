@@ -53,6 +53,7 @@ struct padoc_mpd {
     std::vector<int32_t> step_streams; // stream ids in step order
     std::vector<int32_t> scratch_len;  // padoc_mpd_prepare_step: the step's page lengths and streams
     std::vector<padoc_stream_desc> scratch_streams;
+    PlanParts plan_parts;              // the step's plan (kept: its arrays are reused step after step)
 };
 
 namespace {
@@ -338,7 +339,7 @@ extern "C" padoc_status padoc_mpd_prepare_step(padoc_mpd *m, const padoc_decode_
     }
     if (need > (int64_t)m->free_blocks.size()) return PADOC_ERR_CAPACITY;
     const int32_t P = (int32_t)plen.size(), C = (int32_t)descs.size();
-    PlanParts pp;
+    PlanParts &pp = m->plan_parts;
     padoc_status st = padoc_plan_parts_of_list(plen.data(), P, descs.data(), C, cfg, pp);
     if (st != PADOC_OK) return st;
     const int64_t plan_ints = padoc_plan_blob_ints(pp, P, cfg->num_kv_heads);

@@ -408,12 +408,12 @@ padoc_status build_work(int32_t num_pages, const padoc_decode_config *cfg, PlanP
     // one sequence with one running softmax, so that a piece covering both writes one partial. A
     // piece that crosses from the shared to the private tiles becomes two items, the first flagged
     // PADOC_ITEM_CONT; every stream of a group receives the same items and partial-slot numbers.
-    struct Segment {
-        int32_t kind, g, p, first, ns, vis, ntiles, weight;
-        int32_t kind2, p2, vis2, ntiles2;   // the private continuation (ntiles2 = 0: none)
-    };
-    std::vector<Segment> segs;
-    std::vector<uint8_t> priv_tc(chunked ? (size_t)S : 0, 0);
+    using Segment = PlanSegment;
+    PlanScratch &sc = pp.scratch;
+    std::vector<Segment> &segs = sc.segs;
+    segs.clear();
+    std::vector<uint8_t> &priv_tc = sc.priv_tc;
+    priv_tc.assign(chunked ? (size_t)S : 0, 0);
     auto weight_of = [](int32_t nb) { return nb > PADOC_TC_ITEM_STREAMS / 2 ? PADOC_TC_WEIGHT_2M : PADOC_TC_WEIGHT_1M; };
     for (int32_t g = 0; g < cfg->num_kv_heads; ++g) {
         for (int32_t p = 0; p < num_pages; ++p) {
@@ -450,8 +450,10 @@ padoc_status build_work(int32_t num_pages, const padoc_decode_config *cfg, PlanP
         }
     }
     const int32_t Hkv = cfg->num_kv_heads;
-    std::vector<int32_t> cnt((size_t)S * Hkv, 0);   // partial slots handed out per (stream, KV head)
-    std::vector<padoc_item> tc_items;
+    std::vector<int32_t> &cnt = sc.cnt;   // partial slots handed out per (stream, KV head)
+    cnt.assign((size_t)S * Hkv, 0);
+    std::vector<padoc_item> &tc_items = sc.tc_items;
+    tc_items.clear();
     tc_items.reserve(segs.size() * 2 + 64);
     // CTA loads count every piece's own cost too (its epilogue, and the query reload before it):
     // the smallest bound T for which a greedy walk along the sequences needs at most `want` CTAs
@@ -467,7 +469,8 @@ padoc_status build_work(int32_t num_pages, const padoc_decode_config *cfg, PlanP
         max_piece = std::max(max_piece, piece_cost(sg));
         max_w = std::max<int64_t>(max_w, sg.weight);
     }
-    std::vector<int64_t> tc_load;   // planned load of each tensor-core CTA (emitting walk)
+    std::vector<int64_t> &tc_load = sc.tc_load;   // planned load of each tensor-core CTA (emitting walk)
+    tc_load.clear();
     auto walk = [&](int64_t T, bool emit) {
         int64_t used = 0, load = 0;
         for (const Segment &sg : segs) {
@@ -529,14 +532,18 @@ padoc_status build_work(int32_t num_pages, const padoc_decode_config *cfg, PlanP
         // index order: warp CTA early + j then follows tensor-core CTA j's pieces in the decode grid,
         // and takes the SM of the j-th CTA to end in a warp grid of its own (the E4M3 pool), both
         // with the start the warp planning below gives it.
-        std::vector<int32_t> perm((size_t)ctas);
+        std::vector<int32_t> &perm = sc.perm;
+        perm.resize((size_t)ctas);
         std::iota(perm.begin(), perm.end(), 0);
         std::stable_sort(perm.begin(), perm.end(),
                          [&](int32_t a, int32_t b) { return tc_load[(size_t)a] < tc_load[(size_t)b]; });
-        std::vector<padoc_item> items_sorted;
+        std::vector<padoc_item> &items_sorted = sc.items_sorted;
+        items_sorted.clear();
         items_sorted.reserve(tc_items.size());
-        std::vector<int32_t> ptr_sorted(1, 0);
-        std::vector<int64_t> load_sorted;
+        std::vector<int32_t> &ptr_sorted = sc.ptr_sorted;
+        ptr_sorted.assign(1, 0);
+        std::vector<int64_t> &load_sorted = sc.load_sorted;
+        load_sorted.clear();
         for (int32_t c : perm) {
             items_sorted.insert(items_sorted.end(), tc_items.begin() + pp.cta_ptr[(size_t)c],
                                 tc_items.begin() + pp.cta_ptr[(size_t)c + 1]);
@@ -550,7 +557,8 @@ padoc_status build_work(int32_t num_pages, const padoc_decode_config *cfg, PlanP
     pp.tc_ctas = ctas;
 
     // ---- warp work: shared streams of sparse pages (per stream) and every private history ------
-    std::vector<padoc_item> warp_items;
+    std::vector<padoc_item> &warp_items = sc.warp_items;
+    warp_items.clear();
     {
         int64_t n = 0;   // exact count, so the list is allocated once
         for (int32_t p = 0; p < num_pages; ++p) {
@@ -591,7 +599,8 @@ padoc_status build_work(int32_t num_pages, const padoc_decode_config *cfg, PlanP
     // prefill's group whose pieces stay on one CTA) writes their outputs itself; only the other
     // (stream, KV head) keys go to the merge.
     {
-        std::vector<uint8_t> direct((size_t)S * Hkv, 0);
+        std::vector<uint8_t> &direct = sc.direct;
+        direct.assign((size_t)S * Hkv, 0);
         for (padoc_item &it : tc_items) {
             if (it.kind & PADOC_ITEM_CONT) continue;   // the next item of the chain writes
             bool sole = true;
@@ -610,7 +619,9 @@ padoc_status build_work(int32_t num_pages, const padoc_decode_config *cfg, PlanP
     // block count keeps ties in plan order) and each goes to the warp with the most capacity left
     // (below). Cost: 16-token blocks plus a fixed start-up cost per item.
     const int32_t nitems = (int32_t)warp_items.size();
-    std::vector<int32_t> cost((size_t)nitems), order((size_t)nitems);
+    std::vector<int32_t> &cost = sc.cost, &order = sc.order;
+    cost.resize((size_t)nitems);
+    order.resize((size_t)nitems);
     int32_t maxb = 0;
     for (int32_t i = 0; i < nitems; ++i) {
         const int32_t nb = (warp_items[(size_t)i].tok_end - warp_items[(size_t)i].tok_begin + 15) / 16;
@@ -618,10 +629,11 @@ padoc_status build_work(int32_t num_pages, const padoc_decode_config *cfg, PlanP
         maxb = std::max(maxb, nb);
     }
     {
-        std::vector<int32_t> start((size_t)maxb + 2, 0);
-        for (int32_t i = 0; i < nitems; ++i) ++start[(size_t)(maxb - cost[(size_t)i]) + 1];
-        for (int32_t b = 0; b <= maxb; ++b) start[(size_t)b + 1] += start[(size_t)b];
-        for (int32_t i = 0; i < nitems; ++i) order[(size_t)start[(size_t)(maxb - cost[(size_t)i])]++] = i;
+        std::vector<int32_t> &first = sc.counts;   // first position of each block count, longest first
+        first.assign((size_t)maxb + 2, 0);
+        for (int32_t i = 0; i < nitems; ++i) ++first[(size_t)(maxb - cost[(size_t)i]) + 1];
+        for (int32_t b = 0; b <= maxb; ++b) first[(size_t)b + 1] += first[(size_t)b];
+        for (int32_t i = 0; i < nitems; ++i) order[(size_t)first[(size_t)(maxb - cost[(size_t)i])]++] = i;
     }
     for (int32_t i = 0; i < nitems; ++i) cost[(size_t)i] += PADOC_WARP_ITEM_COST;
     const int32_t wctas = (int32_t)std::min<int64_t>(cfg->warp_ctas > 0 ? cfg->warp_ctas : padoc_default_ctas(),
@@ -641,8 +653,11 @@ padoc_status build_work(int32_t num_pages, const padoc_decode_config *cfg, PlanP
         // puts the longest items on the warps that start first. Without tensor-core work every warp
         // starts at once and the capacities are equal.
         // the warps of a CTA start together: start, rate and warp count per CTA
-        std::vector<double> start((size_t)wctas, 0.0), rate((size_t)wctas, PADOC_WARP_RATE);
-        std::vector<int32_t> nw_of((size_t)wctas);
+        std::vector<double> &start = sc.start, &rate = sc.rate;
+        start.assign((size_t)wctas, 0.0);
+        rate.assign((size_t)wctas, PADOC_WARP_RATE);
+        std::vector<int32_t> &nw_of = sc.nw_of;
+        nw_of.resize((size_t)wctas);
         for (int32_t c = 0; c < wctas; ++c)
             nw_of[(size_t)c] = std::min<int32_t>(PADOC_WARP_KERNEL_WARPS, nwarps - c * PADOC_WARP_KERNEL_WARPS);
         if (!tc_load.empty()) {
@@ -650,7 +665,8 @@ padoc_status build_work(int32_t num_pages, const padoc_decode_config *cfg, PlanP
             const int32_t early = padoc_fused_early_ctas(ntc, wctas, nsm);
             // early warp CTAs past the SM count (a warp_ctas above it) wait for a CTA to end
             const int32_t resident = std::min(early, std::max(0, nsm - ntc));
-            std::vector<double> tend(tc_load.size());
+            std::vector<double> &tend = sc.tend;
+            tend.resize(tc_load.size());
             double tmax = 0.0;
             for (size_t c = 0; c < tc_load.size(); ++c) {
                 tend[c] = PADOC_TC_END_US0 + PADOC_TC_US_PER_UNIT * (double)tc_load[c];
@@ -670,7 +686,8 @@ padoc_status build_work(int32_t num_pages, const padoc_decode_config *cfg, PlanP
         for (int32_t i = 0; i < nitems; ++i) total += cost[(size_t)i];
         // T solves sum_c nw_c rate_c max(0, T - start_c) = total, which is piecewise linear in T:
         // walk the CTAs in order of start, adding each one's slope, until the line reaches total
-        std::vector<int32_t> by_start((size_t)wctas);
+        std::vector<int32_t> &by_start = sc.by_start;
+        by_start.resize((size_t)wctas);
         std::iota(by_start.begin(), by_start.end(), 0);
         std::sort(by_start.begin(), by_start.end(), [&](int32_t x, int32_t y) { return start[(size_t)x] < start[(size_t)y]; });
         double T = 0.0, slope = 0.0, icpt = 0.0;   // capacity at T = slope * T - icpt
@@ -688,14 +705,18 @@ padoc_status build_work(int32_t num_pages, const padoc_decode_config *cfg, PlanP
         // item + 2).
         int64_t max_cost = 0, max_room = 0;
         for (int32_t i = 0; i < nitems; ++i) max_cost = std::max<int64_t>(max_cost, cost[(size_t)i]);
-        std::vector<int64_t> room((size_t)nwarps);
+        std::vector<int64_t> &room = sc.room;
+        room.resize((size_t)nwarps);
         for (int32_t w = 0; w < nwarps; ++w) {
             const int32_t c = w / PADOC_WARP_KERNEL_WARPS;
             room[(size_t)w] = (int64_t)(rate[(size_t)c] * std::max(0.0, T - start[(size_t)c]));
             max_room = std::max(max_room, room[(size_t)w]);
         }
         const int64_t off = max_cost + 2, nbuckets = max_room + off + 1;
-        std::vector<int32_t> head((size_t)nbuckets, -1), tail((size_t)nbuckets, -1), next((size_t)nwarps, -1);
+        std::vector<int32_t> &head = sc.head, &tail = sc.tail, &next = sc.next;
+        head.assign((size_t)nbuckets, -1);
+        tail.assign((size_t)nbuckets, -1);
+        next.assign((size_t)nwarps, -1);
         auto push = [&](int32_t w) {
             const int64_t b = std::max<int64_t>(0, room[(size_t)w] + off);
             next[(size_t)w] = -1;
@@ -703,7 +724,8 @@ padoc_status build_work(int32_t num_pages, const padoc_decode_config *cfg, PlanP
             tail[(size_t)b] = w;
         };
         for (int32_t w = 0; w < nwarps; ++w) push(w);
-        std::vector<int32_t> warp_of((size_t)nitems);
+        std::vector<int32_t> &warp_of = sc.warp_of;
+        warp_of.resize((size_t)nitems);
         int64_t cur = nbuckets - 1;
         for (int32_t k : order) {
             while (head[(size_t)cur] < 0) --cur;
@@ -716,7 +738,8 @@ padoc_status build_work(int32_t num_pages, const padoc_decode_config *cfg, PlanP
             push(w);
         }
         for (int32_t w = 0; w < nwarps; ++w) pp.warp_ptr[(size_t)w + 1] += pp.warp_ptr[(size_t)w];
-        std::vector<int32_t> wpos(pp.warp_ptr.begin(), pp.warp_ptr.end() - 1);
+        std::vector<int32_t> &wpos = sc.wpos;
+        wpos.assign(pp.warp_ptr.begin(), pp.warp_ptr.end() - 1);
         padoc_item *dst = pp.items.data() + tc_items.size();
         for (int32_t k : order) dst[wpos[(size_t)warp_of[(size_t)k]]++] = warp_items[(size_t)k];   // longest first per warp
     }
@@ -825,6 +848,7 @@ namespace {
 padoc_status parts_of_pages(const padoc_page *pages, int32_t num_pages, const padoc_decode_config *cfg,
                            PlanParts &pp)
 {
+    pp.reset();
     padoc_status st = check_config(cfg);
     if (st == PADOC_OK) st = streams_of_pages(pages, num_pages, cfg, pp);
     if (st == PADOC_OK) st = build_work(num_pages, cfg, pp);
@@ -836,6 +860,7 @@ padoc_status parts_of_pages(const padoc_page *pages, int32_t num_pages, const pa
 padoc_status padoc_plan_parts_of_list(const int32_t *page_len, int32_t num_pages, const padoc_stream_desc *streams,
                                       int32_t num_streams, const padoc_decode_config *cfg, PlanParts &pp)
 {
+    pp.reset();
     padoc_status st = check_config(cfg);
     if (st == PADOC_OK && cfg->layout_streams) st = PADOC_ERR_INVALID_ARGUMENT;  // the list names every stream
     if (st == PADOC_OK) st = streams_of_list(page_len, num_pages, streams, num_streams, pp);
@@ -846,6 +871,7 @@ padoc_status padoc_plan_parts_of_list(const int32_t *page_len, int32_t num_pages
 padoc_status padoc_plan_parts_of_chunks(const int32_t *page_len, int32_t num_pages, const padoc_prefill_chunk *chunks,
                                         int32_t num_chunks, const padoc_decode_config *cfg, PlanParts &pp)
 {
+    pp.reset();
     padoc_status st = check_config(cfg);
     if (st == PADOC_OK && cfg->layout_streams) st = PADOC_ERR_INVALID_ARGUMENT;
     if (st == PADOC_OK) st = streams_of_chunks(page_len, num_pages, chunks, num_chunks, pp);

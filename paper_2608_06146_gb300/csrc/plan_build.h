@@ -11,6 +11,25 @@
 
 struct PlanStream { int32_t page, shared_len, private_len; };
 
+// One (KV head, page, group of streams) of tensor-core work and the shared-stream tiles it sees, with
+// the private continuation of a chunked prefill's group (ntiles2 = 0: none); build_work's comment has
+// the rest.
+struct PlanSegment {
+    int32_t kind, g, p, first, ns, vis, ntiles, weight;
+    int32_t kind2, p2, vis2, ntiles2;
+};
+
+// Working arrays of build_work, kept with the parts so that a caller planning step after step (the
+// decoding loop's scheduler) reuses their memory.
+struct PlanScratch {
+    std::vector<uint8_t> priv_tc, direct;
+    std::vector<int32_t> cnt, perm, ptr_sorted, cost, order, counts, nw_of, by_start, head, tail, next, warp_of, wpos;
+    std::vector<int64_t> tc_load, load_sorted, room;
+    std::vector<double> start, rate, tend;
+    std::vector<padoc_item> tc_items, items_sorted, warp_items;
+    std::vector<PlanSegment> segs;
+};
+
 struct PlanParts {
     std::vector<PlanStream> streams;
     std::vector<int32_t> page_len, page_first_stream, page_num_streams;
@@ -27,6 +46,29 @@ struct PlanParts {
     // first stream, its token count and whether its tokens have private rows
     std::vector<int32_t> chunk_of, chunk_first, chunk_len;
     std::vector<uint8_t> chunk_private;
+    PlanScratch scratch;
+
+    // Empties every part (their memory and the scratch arrays stay allocated).
+    void reset()
+    {
+        streams.clear();
+        page_len.clear();
+        page_first_stream.clear();
+        page_num_streams.clear();
+        slot_ptr.clear();
+        cta_ptr.clear();
+        warp_ptr.clear();
+        merge_keys.clear();
+        items.clear();
+        num_tc_items = tc_ctas = num_warps = 0;
+        tc_min_rows = PADOC_TC_MIN_ROWS;
+        max_page_blocks = max_stream_blocks = 0;
+        kv_tokens = 0;
+        chunk_of.clear();
+        chunk_first.clear();
+        chunk_len.clear();
+        chunk_private.clear();
+    }
 };
 
 // The split-K work of an explicit stream list (padoc_build_decode_plan_streams' rules).

@@ -263,14 +263,16 @@ def check_first_blocks(stage, st, plan, info, page_len, streams, pt, stt, Hkv=2)
 
 
 @pytest.mark.parametrize("seed", range(4))
-def test_prepare_step_equals_granular_calls(seed):
+@pytest.mark.parametrize("ctas", [(96, 152), (0, 0)])
+def test_prepare_step_equals_granular_calls(seed, ctas):
     """padoc_mpd_prepare_step writes exactly what begin_step, step_tables and the stream-list planner
-    give, step after step, for two schedulers driven by the same events."""
+    give, step after step, for two schedulers driven by the same events (the scheduler keeps its
+    planner's arrays from step to step; each comparison plan is built from nothing)."""
     rng = np.random.default_rng(500 + seed)
     pages = _rand_pages(rng, int(rng.integers(2, 6)), P_max=300, L_max=40, N_max=12, n_max=70)
     nb = _blocks_needed(pages) + 5
     order = rng.permutation(nb).astype(np.int32)
-    cfg = pa.make_decode_config(16, 2, 128, tc_ctas=96, warp_ctas=152)
+    cfg = pa.make_decode_config(16, 2, 128, tc_ctas=ctas[0], warp_ctas=ctas[1])
     a, b = pa.Mpd(nb, BS, order), pa.Mpd(nb, BS, order)
     src = LoopTokenSource(pages)
     for p in range(len(pages)):
