@@ -519,12 +519,27 @@ padoc_status build_work(int32_t num_pages, const padoc_decode_config *cfg, PlanP
         // more than `want` CTAs: that is a lower bound. A CTA is closed only once less than a piece
         // and a tile fit, and cutting adds at most one piece per CTA, so T = total_w / (want - 1) +
         // 2 max_piece + max_w fits in `want`; it is checked, with the one-CTA bound behind it.
-        int64_t lo = std::max<int64_t>(max_w + max_piece, (total_w + want - 1) / want);
-        int64_t hi = (want > 1 ? (total_w + want - 2) / (want - 1) : total_w) + 2 * max_piece + max_w + 1;
-        if (hi < lo || walk(hi, false) > want) hi = std::max(lo, total_w + max_w);   // walk(total_w + max_w) needs one CTA
-        while (lo < hi) {
-            const int64_t mid = lo + (hi - lo) / 2;
-            if (walk(mid, false) <= want) hi = mid; else lo = mid + 1;
+        // The search depends only on `want` and each segment's tile count and weight (the rest follows
+        // from them); a caller that plans step after step with the same parts (the decoding loop's
+        // scheduler) often repeats them, and then the last bound is taken as it is.
+        std::vector<int64_t> &key = sc.bound_key;
+        key.clear();
+        key.push_back(want);
+        key.push_back(chunked ? 1 : 0);
+        for (const Segment &sg : segs) key.push_back(((int64_t)(sg.ntiles + sg.ntiles2) << 8) | sg.weight);
+        int64_t lo;
+        if (sc.bound >= 0 && key == sc.last_bound_key) {
+            lo = sc.bound;
+        } else {
+            lo = std::max<int64_t>(max_w + max_piece, (total_w + want - 1) / want);
+            int64_t hi = (want > 1 ? (total_w + want - 2) / (want - 1) : total_w) + 2 * max_piece + max_w + 1;
+            if (hi < lo || walk(hi, false) > want) hi = std::max(lo, total_w + max_w);   // walk(total_w + max_w) needs one CTA
+            while (lo < hi) {
+                const int64_t mid = lo + (hi - lo) / 2;
+                if (walk(mid, false) <= want) hi = mid; else lo = mid + 1;
+            }
+            sc.last_bound_key.swap(key);
+            sc.bound = lo;
         }
         ctas = (int32_t)walk(lo, true);
         pp.cta_ptr.push_back((int32_t)tc_items.size());

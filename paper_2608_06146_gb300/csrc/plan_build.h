@@ -28,6 +28,10 @@ struct PlanScratch {
     std::vector<double> start, rate, tend;
     std::vector<padoc_item> tc_items, items_sorted, warp_items;
     std::vector<PlanSegment> segs;
+    // the tensor-core bound search's inputs (want, chunked, each segment's tiles and weight) and its
+    // result, from the last search (bound < 0: none yet)
+    std::vector<int64_t> bound_key, last_bound_key;
+    int64_t bound = -1;
 };
 
 struct PlanParts {
