@@ -263,16 +263,19 @@ def check_first_blocks(stage, st, plan, info, page_len, streams, pt, stt, Hkv=2)
 
 
 @pytest.mark.parametrize("seed", range(4))
-@pytest.mark.parametrize("ctas", [(96, 152), (0, 0)])
+@pytest.mark.parametrize("ctas", [(96, 152), (0, 0), "alternating"])
 def test_prepare_step_equals_granular_calls(seed, ctas):
     """padoc_mpd_prepare_step writes exactly what begin_step, step_tables and the stream-list planner
     give, step after step, for two schedulers driven by the same events (the scheduler keeps its
-    planner's arrays from step to step; each comparison plan is built from nothing)."""
+    planner's arrays and its last tensor-core bound search from step to step; each comparison plan
+    is built from nothing; "alternating" changes the CTA counts asked for at every step)."""
     rng = np.random.default_rng(500 + seed)
     pages = _rand_pages(rng, int(rng.integers(2, 6)), P_max=300, L_max=40, N_max=12, n_max=70)
     nb = _blocks_needed(pages) + 5
     order = rng.permutation(nb).astype(np.int32)
-    cfg = pa.make_decode_config(16, 2, 128, tc_ctas=ctas[0], warp_ctas=ctas[1])
+    cfgs = [pa.make_decode_config(16, 2, 128, tc_ctas=t, warp_ctas=w)
+            for t, w in ([(96, 152), (40, 0), (0, 0)] if ctas == "alternating" else [ctas])]
+    step_no = 0
     a, b = pa.Mpd(nb, BS, order), pa.Mpd(nb, BS, order)
     src = LoopTokenSource(pages)
     for p in range(len(pages)):
@@ -282,6 +285,8 @@ def test_prepare_step_equals_granular_calls(seed, ctas):
         src.admitted(p, new)
     stage = np.zeros(16, np.int32)
     while b.status()[1] > 0:
+        cfg = cfgs[step_no % len(cfgs)]
+        step_no += 1
         try:
             st = a.prepare_step(cfg, stage)
         except pa.PadocError as e:
